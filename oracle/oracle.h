@@ -1,0 +1,68 @@
+/*
+ * Reference oracle for the FastRL kept-token GRPO path — TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, fp64 CPU restatement of what the path computes, written from the paper's
+ * definitions ("Learn from the Gap", Sec. 3 and Algorithm 1).  Only the test suite, the smoke
+ * check and the benchmark's CPU-baseline leg may load it.  It shares no code, header, table or
+ * helper with the CUDA library: nothing here includes or links anything from the package, and
+ * the package never loads this.
+ *
+ * Every function follows one passage of the paper; the pins that check each one against what
+ * the paper and the mathematics fix live in tests/test_oracle_*.py.  Floating point is fp64
+ * throughout, on inputs given in f32 or as bf16 bit patterns (both exact in fp64).  Build with
+ * -ffp-contract=off so that no multiply-add is fused: advantages and pruning keys are then
+ * reproducible bit for bit from their written order of operations.
+ */
+#ifndef FASTRL_ORACLE_H_
+#define FASTRL_ORACLE_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Eq. 5: per-group advantages; see advantage.cpp. */
+int oracle_advantage(const float* rewards, int P, int G, int std_mode, float* adv, double* key);
+
+/* Eqs. 6-9 and Algorithm 1 (Phase 2 and DP alignment): MDAP keep mask; see mdap.cpp. */
+int oracle_prune(const float* rewards, const int32_t* ids, const int64_t* off, int P, int G,
+                 int ngram_n, float tau, int keep_cap, int dp_divisor, uint8_t* keep,
+                 int32_t* kept_per_prompt);
+
+/* Eq. 7 alone, for tests: theta_ij for rollouts i and j (indices into off). */
+double oracle_jaccard_distance(const int32_t* ids, const int64_t* off, int i, int j, int ngram_n);
+
+/* Compaction of kept rollouts' tokens (Sec. 3.2 after Eq. 9); see compact.cpp. */
+int oracle_compact(const uint8_t* keep, const int64_t* off, int n_rollouts, int32_t* kept_idx,
+                   int64_t* kept_off, int64_t* src_token, int32_t* token_rollout, int64_t* counts);
+
+/* Eqs. 1-3: GRPO token loss and dlogits; see loss.cpp.
+ * logits_dtype 0 = f32, 1 = bf16 bit patterns (uint16).  dlogits_dtype 0 = f32, 1 = bf16 bits.
+ * dlogits_f64 (nullable) receives the unrounded fp64 gradient.  rho_out (nullable) the ratios. */
+int oracle_loss(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
+                int64_t n_rows, int V, const int32_t* y, const float* old_logp,
+                const float* ref_logp, const float* adv, const int32_t* row_rollout, float eps_low,
+                float eps_high, float beta, int agg_mode, int64_t denom_tokens,
+                const int64_t* seq_off, int64_t n_seq, void* dlogits, int dlogits_dtype,
+                double* dlogits_f64, double* logp_out, double* rho_out, double* row_loss_out,
+                double* loss_out);
+
+/* Round an fp64 value to bf16 (nearest, ties to even, bf16 subnormals kept); returns the bits. */
+uint16_t oracle_round_bf16(double x);
+
+/* Eqs. 10-14 and Algorithm 1 (Phases 1a/1b): adaptive rollout sampling; see ars.cpp. */
+void* oracle_ars_new(int G1);
+void oracle_ars_free(void* st);
+int oracle_ars_step(void* st, const int32_t* kept_per_prompt, int P, int64_t step,
+                    int64_t total_steps, int epoch_end);
+double oracle_ars_get(void* st, int what); /* 0: G'_ref or NaN, 1: G'_t or NaN */
+
+/* Worker threads the loss uses (OpenMP); 0 keeps the runtime default.  Returns the count. */
+int oracle_set_threads(int n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FASTRL_ORACLE_H_ */
