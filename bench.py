@@ -1,0 +1,415 @@
+"""Benchmark: one FastRL kept-token GRPO step per iteration on GB300.
+
+A step is the whole data-parallel path on one batch: grpo_advantage -> grpo_prune ->
+grpo_compact -> (host: kept counts, adaptive rollout count) -> grpo_loss_fwd_bwd over the kept
+tokens.  The default workload is the Qwen2.5-vocabulary batch: 16 prompts x G=8 rollouts,
+lognormal completion lengths (median 384, capped at 1024), V = 152064, bf16 logits with a
+Zipf(1.1) rank bias plus N(0, 2^2) noise, keep ratio 0.5, bf16 dlogits.  The logits of every
+token (~16 GB) are resident before timing; the loss reads only the kept rows.
+
+Output: one JSON line (rank 0).  `value` is kept tokens per second over all ranks (device
+time, CUDA events); `e2e` repeats the step with the inputs copied from pinned host memory and
+the loss read back inside the timed region; `roofline` relates the loss kernel's event-timed
+duration to the measured HBM copy bandwidth; `cpu_baseline` times the fp64 oracle on a bounded
+sample on this machine's host cores.  `--impl reference` times that oracle as the reference
+arm.  Under torchrun each rank runs its own batch (weak scaling); the only collectives are the
+barrier and the max-over-ranks timing.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "kept-token GRPO loss fwd+bwd tokens/s and logits HBM GB/s (% of GB300 peak)"
+UNIT = "kept tokens/s"
+SIDE_BYTES_PER_ROW = 36  # y, old, ref, logp (4 each), src_token 8, row rollout 4, row loss 8
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="qwen", help="tiny|small|qwen|large|long or 0-4")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def workload_desc(w, T, T_kept, K):
+    return {
+        "workload": "%s: %d prompts x G=%d rollouts, lengths %s, V=%d, %s logits (%s), rewards %s,"
+                    " %.0f%% zero-advantage groups, keep ratio %.2f (cap %d/prompt), %s dlogits"
+                    % (w.name, w.P, w.G, w.length, w.V, w.logits_dtype, w.logits_kind,
+                       w.reward_kind, 100 * w.zero_adv_frac, w.keep_ratio, w.keep_cap,
+                       w.dlogits_dtype),
+        "V": w.V, "prompts": w.P, "G": w.G, "T_tokens": T, "T_kept": T_kept, "kept_rollouts": K,
+        "eps": w.eps, "beta": w.beta, "tau": w.tau, "ngram_n": w.ngram_n,
+        "io": "%s logits -> %s dlogits" % (w.logits_dtype, w.dlogits_dtype),
+        "l2": "inputs larger than L2 (logits %.1f GB vs 129 MB L2); no flush" % (T * w.V * w.in_bytes / 1e9),
+    }
+
+
+def measured_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs, copy read+write)"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback 6.8 TB/s (no MEASURED_PEAKS.json)"
+
+
+def loss_source_hash():
+    h = hashlib.sha256()
+    for f in ("loss.cu", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload_name):
+    """DRAM bytes per kept row of the loss kernel from the committed ncu summary, if it was
+    taken on the current kernel source; else None."""
+    p = os.path.join(ROOT, "profiles", "loss_kernel_traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+    except Exception:
+        return None
+    e = d.get(workload_name)
+    if not e or e.get("source_hash") != loss_source_hash():
+        return None
+    return float(e["dram_bytes_per_row"])
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + ",".join(self.FIELDS), "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, pw, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) != len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+                pw.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "power_w_max": max(pw) if pw else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def build_inputs(w, seed, device):
+    """Seeded synthetic batch, resident on `device` (logits of every token)."""
+    import torch
+    from paper_2609_36932_gb300 import workloads
+    b = workloads.make_batch(w, seed)
+    T = b["T"]
+    rewards = torch.from_numpy(b["rewards"]).to(device)
+    ids = torch.from_numpy(b["ids"]).to(device)
+    off = torch.from_numpy(b["off"]).to(device)
+    logits = workloads.logits_rows(w, seed, range(T), device)
+    old, ref = workloads.old_ref_logp(logits, b["ids"], b["noise_old"], b["noise_ref"])
+    return b, dict(rewards=rewards, ids=ids, off=off, logits=logits, old=old, ref=ref)
+
+
+def make_step(w, dev_inputs):
+    from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
+    p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
+                   eps_low=w.eps, eps_high=w.eps, beta=w.beta, dlogits_dtype=w.dlogits_dtype)
+    d = dev_inputs
+    return GrpoStep(p, d["rewards"], d["ids"], d["off"], d["logits"], d["old"], d["ref"])
+
+
+def oracle_sample(w, b, rows_src, rows_rollout, T_kept, logits_rows_host, old, ref, threads=0):
+    """Time the oracle: selection on the whole batch, then the loss on the given kept rows."""
+    import oracle
+    oracle.set_threads(threads)
+    t0 = time.perf_counter()
+    adv, _ = oracle.advantage(b["rewards"], w.G)
+    keep, kpp = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+    comp = oracle.compact(keep, b["off"])
+    t_sel = time.perf_counter() - t0
+    n = len(rows_src)
+    t1 = time.perf_counter()
+    oracle.loss(logits_rows_host, w.V, b["ids"][rows_src], old[rows_src], ref[rows_src], adv,
+                rows_rollout, eps_low=w.eps, eps_high=w.eps, beta=w.beta, denom_tokens=T_kept,
+                dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0, n_rows=n)
+    t_loss = time.perf_counter() - t1
+    return t_sel, t_loss, comp, int(oracle.set_threads(0))
+
+
+def host_logits_bits(t):
+    import torch
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.float().cpu().numpy()
+
+
+def cpu_baseline_ours(w, b, step, dev_inputs, target_s):
+    """Oracle timed on a bounded sample of this workload (the first kept rows)."""
+    src, rr = step.kept_rows()
+    old = dev_inputs["old"].cpu().numpy()
+    ref = dev_inputs["ref"].cpu().numpy()
+    # calibrate on 8 rows, then size the sample for ~target_s seconds of loss work
+    n0 = min(8, len(src))
+    _, tl0, _, cores = oracle_sample(w, b, src[:n0], rr[:n0], step.T_kept,
+                                     host_logits_bits(dev_inputs["logits"][src[:n0]]), old, ref)
+    per_row = max(tl0 / max(n0, 1), 1e-6)
+    n = int(min(len(src), max(n0, target_s / per_row)))
+    rows = src[:n]
+    t_sel, t_loss, _, cores = oracle_sample(w, b, rows, rr[:n], step.T_kept,
+                                            host_logits_bits(dev_inputs["logits"][rows]), old, ref)
+    t_per_token = t_loss / n + t_sel / max(step.T_kept, 1)
+    return {"value": 1.0 / t_per_token, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "fp64 oracle: advantage+prune+compact on the whole batch (%.2f s, amortised"
+                      " over its %d kept tokens) + loss fwd/bwd on the first %d kept rows (%.2f s)"
+                      % (t_sel, step.T_kept, n, t_loss)}
+
+
+def run_reference(args, w):
+    """The reference arm: the fp64 oracle as it stands, on this machine's host cores."""
+    import torch
+    from paper_2609_36932_gb300 import workloads
+    import oracle
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    b = workloads.make_batch(w, args.seed)
+    keep, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+    comp = oracle.compact(keep, b["off"])
+    T_kept = comp["T_kept"]
+    src_all, rr_all = comp["src_token"], comp["token_rollout"]
+    # a bounded sample of kept rows, generated on the host
+    n = min(len(src_all), 4)
+    lg = workloads.logits_rows(w, args.seed, src_all[:n], "cpu")
+    old, ref = workloads.old_ref_logp(lg, b["ids"][src_all[:n]], b["noise_old"][src_all[:n]],
+                                      b["noise_ref"][src_all[:n]])
+    old_full = np.zeros(b["T"], np.float32)
+    ref_full = np.zeros(b["T"], np.float32)
+    old_full[src_all[:n]] = old.numpy()
+    ref_full[src_all[:n]] = ref.numpy()
+    bits = host_logits_bits(lg)
+    t_sel, t_loss, _, cores = oracle_sample(w, b, src_all[:n], rr_all[:n], T_kept, bits, old_full, ref_full)
+    # size each step's sample so the whole run stays within ~2 minutes
+    budget = 120.0 / max(args.steps + args.warmup, 1)
+    per_row = t_loss / n
+    rows = int(max(1, min(len(src_all), (budget - t_sel) / per_row))) if budget > t_sel else 1
+    rows = min(rows, 512)
+    sel = src_all[:rows]
+    lg = workloads.logits_rows(w, args.seed, sel, "cpu")
+    o, r = workloads.old_ref_logp(lg, b["ids"][sel], b["noise_old"][sel], b["noise_ref"][sel])
+    old_full[sel] = o.numpy()
+    ref_full[sel] = r.numpy()
+    bits = host_logits_bits(lg)
+    times = []
+    for i in range(args.warmup + args.steps):
+        t_sel, t_loss, _, cores = oracle_sample(w, b, sel, rr_all[:rows], T_kept, bits, old_full, ref_full)
+        if i >= args.warmup:
+            times.append(t_loss / rows + t_sel / T_kept)
+    value = 1.0 / statistics.mean(times)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_desc(w, b["T"], T_kept, comp["K"]),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": "per step: fp64 oracle advantage+prune+compact on the whole batch"
+                                   " (amortised over %d kept tokens) + loss fwd/bwd on the first %d"
+                                   " kept rows" % (T_kept, rows)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    from paper_2609_36932_gb300 import workloads
+    w = workloads.get(args.config)
+    if args.impl == "reference":
+        run_reference(args, w)
+        return
+    import torch
+    import torch.distributed as dist
+    import paper_2609_36932_gb300 as g
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    g.lib()
+
+    b, d = build_inputs(w, args.seed + rank, dev)
+    step = make_step(w, d)
+    for _ in range(max(args.warmup, 3)):
+        step.run()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    l0 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    l1 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    if local == 0:
+        sampler.start()
+        time.sleep(0.3)
+    launches0 = g.grpo_kernel_launches()
+    kept = 0
+    ev0.record(stream)
+    for i in range(K):
+        step.select()
+        l0[i].record(stream)
+        step.loss_step()
+        l1[i].record(stream)
+        kept += step.T_kept
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    launches = g.grpo_kernel_launches() - launches0
+    clocks = sampler.stop() if local == 0 else None
+    g.check_status(step.status)
+    elapsed_ms = ev0.elapsed_time(ev1)
+    loss_ms = statistics.mean(a.elapsed_time(z) for a, z in zip(l0, l1))
+    tot = torch.tensor([elapsed_ms, float(kept)], dtype=torch.float64, device=dev)
+    if world > 1:
+        mx = tot[:1].clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        sm = tot[1:].clone()
+        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+        elapsed_ms, kept_all = float(mx.item()), float(sm.item())
+    else:
+        kept_all = float(kept)
+    value = kept_all / (elapsed_ms / 1e3)
+
+    # roofline of the dominant kernel (the fused loss), from its event-timed launches
+    bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
+    achieved = step.T_kept * bytes_per_row / (loss_ms / 1e3) / 1e9
+    peak, peak_src = measured_peak()
+    per_row_traffic = profiled_traffic(w.name)
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak,
+                "traffic": None if per_row_traffic is None else per_row_traffic * step.T_kept,
+                "kernel": "grpo_loss_kernel (+ 1-CTA fixed-order loss sum)",
+                "algorithmic_bytes_per_launch": step.T_kept * bytes_per_row,
+                "launch_ms": loss_ms, "peak_source": peak_src}
+
+    # end to end: inputs copied from pinned host memory, loss read back, inside the timed region
+    e2e = None
+    if args.e2e_steps > 0:
+        names = ["rewards", "ids", "off", "logits", "old", "ref"]
+        host = {k: d[k].cpu().pin_memory() for k in names}
+        h2d = sum(host[k].numel() * host[k].element_size() for k in names)
+        loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
+        d2h = 8 + 16 + 4 * w.P
+        step.run()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        kept_e = 0
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            for k in names:
+                d[k].copy_(host[k], non_blocking=True)
+            step.run()
+            loss_host.copy_(step.loss, non_blocking=True)
+            kept_e += step.T_kept
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = e0.elapsed_time(e1)
+        et = torch.tensor([e_ms, float(kept_e)], dtype=torch.float64, device=dev)
+        if world > 1:
+            mx = et[:1].clone()
+            dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+            sm = et[1:].clone()
+            dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+            e_ms, kept_e = float(mx.item()), float(sm.item())
+        e2e = {"value": kept_e / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "steps": args.e2e_steps}
+        del host
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline_ours(w, b, step, d, args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded; shapes and distributions of the paper's GRPO batches)",
+            "config": workload_desc(w, b["T"], step.T_kept, step.K),
+            "gpu_launches": int(launches), "roofline": roofline, "e2e": e2e,
+            "cpu_baseline": cpu, "clocks": clocks,
+            "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

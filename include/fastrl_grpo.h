@@ -1,0 +1,226 @@
+/*
+ * fastrl_grpo.h — C ABI of the GB300 kept-token GRPO library (libfastrl_grpo.so).
+ *
+ * The library computes, on one GPU, the data-parallel core of one FastRL training step
+ * ("Learn from the Gap", Sec. 3 and Algorithm 1):
+ *
+ *   grpo_advantage          group-relative advantages                          (Eq. 5)
+ *   grpo_prune              maximising-differential advantage pruning (MDAP)   (Eqs. 6-9, Algorithm 1)
+ *   grpo_compact            compaction of the kept rollouts' tokens            (Sec. 3.2, after Eq. 9)
+ *   grpo_loss_fwd_bwd       fused GRPO token loss, forward and dlogits         (Eqs. 1-3)
+ *   adaptive_rollout_count  host-side adaptive rollout sampling (ARS)          (Eqs. 10-14, Algorithm 1)
+ *
+ * Conventions shared by every call:
+ *   - Every call returns a grpo_status; GRPO_OK is 0.  On failure, grpo_last_error() returns a
+ *     message for the calling thread.  No C++ exception and no abort crosses this boundary.
+ *   - Buffers marked "device" are device pointers owned by the caller (for instance memory held
+ *     by PyTorch tensors).  The library never allocates or frees device memory.  Scratch memory
+ *     comes from a caller workspace: a call with ws == NULL and ws_bytes != NULL only writes the
+ *     size it needs into *ws_bytes and enqueues nothing.  The real call passes ws (256-byte
+ *     aligned) with *ws_bytes >= that size, or ws == NULL and ws_bytes == NULL when the size
+ *     is 0.
+ *   - GPU work is enqueued asynchronously on `stream` (a cudaStream_t; NULL is the legacy
+ *     default stream).  Host-side argument errors are returned before anything is enqueued.
+ *   - Data errors that only the GPU can see (a token id outside [0, V), non-finite logits, a
+ *     wait that ran out of time) never trap: kernels OR a GRPO_DEVFLAG_* bit into the caller's
+ *     int32 device status word, which the caller reads after synchronising the stream.
+ *   - All arrays are dense and row-major unless a stride argument says otherwise.
+ */
+#ifndef FASTRL_GRPO_H_
+#define FASTRL_GRPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef void* grpo_stream_t; /* a cudaStream_t */
+
+typedef enum {
+  GRPO_OK = 0,
+  GRPO_ERR_INVALID_ARG = 1,  /* a null pointer, a negative size or an out-of-range parameter */
+  GRPO_ERR_UNSUPPORTED = 2,  /* a valid request outside this build's limits (stated per call) */
+  GRPO_ERR_WORKSPACE = 3,    /* workspace missing or smaller than the size query returned */
+  GRPO_ERR_CUDA = 4,         /* a CUDA runtime call failed; grpo_last_error() names it */
+  GRPO_ERR_TIMEOUT = 5,      /* reserved for host-side waits */
+  GRPO_ERR_DEVICE_CHECK = 6  /* reserved for callers that turn device status bits into a status */
+} grpo_status;
+
+typedef enum { GRPO_DTYPE_F32 = 0, GRPO_DTYPE_BF16 = 1 } grpo_dtype;
+
+/* Bits a kernel ORs into the caller's device status word. */
+#define GRPO_DEVFLAG_BAD_TOKEN 1 /* a token id outside [0, V) */
+#define GRPO_DEVFLAG_NONFINITE 2 /* a row's log-sum-exp or log-prob was NaN or infinite */
+#define GRPO_DEVFLAG_TIMEOUT 4   /* a bounded wait on an asynchronous copy gave up */
+
+/* Message describing the last failure on the calling thread ("" if none). */
+const char* grpo_last_error(void);
+
+/* Library version string. */
+const char* grpo_version(void);
+
+/* Number of kernels this process has launched through the library so far (host counter). */
+uint64_t grpo_kernel_launches(void);
+
+/*
+ * grpo_advantage — group-relative advantage, Eq. 5 (Sec. 3.2):
+ *   A_i = (r_i - mean{r_1..r_G}) / std{r_1..r_G}, one group of G rollouts per prompt.
+ * rewards   device f32 [P*G], prompt-major (rollout i of prompt p at p*G + i).
+ * std_mode  0: sample std (divide by G-1); 1: population std (divide by G).
+ * adv       device f32 [P*G] out.  A group whose std is 0 (all rewards equal), or G == 1 in
+ *           mode 0, gets A = 0.  mean and std are taken in fp64, summed in index order, and
+ *           A is rounded once to f32.
+ * key       device f64 [P*G] out, nullable: |r_i - mean| in fp64, the ordering key MDAP uses.
+ * Limits: 1 <= G <= 1024.  P = 0 is a no-op.
+ */
+grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G, int32_t std_mode,
+                           float* adv, double* key, grpo_stream_t stream);
+
+/*
+ * grpo_prune — maximising-differential advantage pruning, Eqs. 6-9 and Algorithm 1 (Phase 2).
+ * Per prompt q, rollouts are partitioned into classes of equal advantage (Eq. 6); inside a
+ * group A is a strictly increasing function of r, so classes are taken by exact f32 reward
+ * equality.  Rollouts are visited by |r_i - mean| descending (fp64), ties by lower index, and
+ * a rollout is kept unless an already kept rollout of its class has Jaccard distance
+ * theta_ij = 1 - |N_n(o_i) & N_n(o_j)| / |N_n(o_i) | N_n(o_j)| < tau (Eqs. 7-8), where N_n is
+ * the set of distinct n-grams of a completion.  Two rollouts that both have no n-gram
+ * (length < n) have theta = 0.  The kept set is S(q), the union over classes (Eq. 9).
+ * Then, if |S(q)| > keep_cap, keep_cap rollouts are kept by round-robin over the classes
+ * (classes ordered by |r - mean| descending, then by lowest member index; each round takes each
+ * class's next kept rollout, lowest index first).  keep_cap >= G disables the cap (the paper's
+ * rule).  Finally, while the total kept count is not a multiple of dp_divisor, prompts are
+ * visited cyclically from prompt 0 and each visit adds that prompt's unkept rollout with the
+ * largest |r - mean| (lowest index on ties); prompts with none left are skipped (Algorithm 1,
+ * DP alignment).  dp_divisor = 1 does nothing.
+ * rewards          device f32 [P*G].
+ * ids              device i32 [T]: completion token ids of all rollouts, packed.
+ * off              device i64 [P*G+1]: rollout r owns ids[off[r] .. off[r+1]); off[0] = 0,
+ *                  off[P*G] = T, non-decreasing.
+ * ngram_n          1..3.  Token ids must lie in [0, V); an id outside it sets
+ *                  GRPO_DEVFLAG_BAD_TOKEN and leaves that prompt's keep mask unspecified.
+ * tau              Jaccard-distance threshold (the paper uses 0.8).
+ * keep_cap         >= 1, per-prompt cap after MDAP.
+ * dp_divisor       >= 1.
+ * keep             device u8 [P*G] out: 1 = kept.
+ * kept_per_prompt  device i32 [P] out: |S(q)| after cap and fill.
+ * status           device i32 [1], nullable: GRPO_DEVFLAG_* bits are ORed in.
+ * ws, ws_bytes     workspace (see conventions); its size depends on T, P and G.
+ * Limits: 1 <= G <= 32; 1 <= V <= 2^18 (three 18-bit ids fit one 64-bit n-gram key).
+ */
+grpo_status grpo_prune(const float* rewards, const int32_t* ids, const int64_t* off,
+                       int32_t P, int32_t G, int64_t T, int32_t V, int32_t ngram_n, float tau,
+                       int32_t keep_cap, int32_t dp_divisor, uint8_t* keep,
+                       int32_t* kept_per_prompt, int32_t* status, void* ws, size_t* ws_bytes,
+                       grpo_stream_t stream);
+
+/*
+ * grpo_compact — token compaction of the kept rollouts (Sec. 3.2: only retained trajectories
+ * are fed to the old, current and reference models).
+ * keep           device u8 [n_rollouts].
+ * off            device i64 [n_rollouts+1] token offsets of all rollouts.
+ * kept_idx       device i32 [n_rollouts] out: indices of the K kept rollouts, ascending.
+ * kept_off       device i64 [n_rollouts+1] out: kept_off[k] = tokens of kept rollouts before k;
+ *                kept_off[K] = T_kept.
+ * src_token      device i64 [T] out: for kept row t < T_kept, its token index in `off` layout.
+ * token_rollout  device i32 [T] out: for kept row t < T_kept, its rollout index (0..n_rollouts).
+ * counts         device i64 [2] out: {K, T_kept}.
+ * counts_host    host i64 [2], nullable: if given, {K, T_kept} are copied there (a stream-ordered
+ *                copy; use pinned memory and synchronise the stream before reading).
+ * Entries past K (kept_idx, kept_off) and past T_kept (src_token, token_rollout) are untouched.
+ */
+grpo_status grpo_compact(const uint8_t* keep, const int64_t* off, int32_t n_rollouts,
+                         int32_t* kept_idx, int64_t* kept_off, int64_t* src_token,
+                         int32_t* token_rollout, int64_t* counts, int64_t* counts_host,
+                         grpo_stream_t stream);
+
+/*
+ * grpo_loss_fwd_bwd — fused GRPO token loss and its gradient w.r.t. the logits, Eqs. 1-3.
+ * For every row t < n_rows, with z the logits row, y the sampled token and A the advantage:
+ *   lse = log sum_v exp(z_v);  logp = z_y - lse;  rho = exp(logp - old_logp)
+ *   surr = min(rho*A, clip(rho, 1-eps_low, 1+eps_high)*A)
+ *   x = ref_logp - logp;  kl = exp(x) - x - 1                      (per-token KL estimate)
+ *   l_t = -(surr - beta*kl);  loss = sum_t w_t * l_t
+ *   c = [A>=0][rho<=1+eps_high] + [A<0][rho>=1-eps_low]             (clip indicator, Sec. 3.1)
+ *   g_t = -(c*rho*A + beta*(exp(x) - 1))                            (bracket of Eq. 3, negated)
+ *   dlogits[t, v] = w_t * g_t * ([v == y] - exp(z_v - lse))
+ * Weights: agg_mode 0 (token mean): w_t = 1/denom_tokens.  agg_mode 1 (Eq. 1's sequence mean):
+ *   w_t = 1/(n_seq * L_r), L_r = seq_off[r+1] - seq_off[r] for the row's rollout r.
+ * Inputs:
+ *   logits        device, dtype logits_dtype (GRPO_DTYPE_BF16 or GRPO_DTYPE_F32); row s starts
+ *                 at element s*row_stride (row_stride >= V).
+ *   row_index     device i64 [n_rows], nullable: row t reads logits row src = row_index[t]
+ *                 (for instance grpo_compact's src_token); if NULL, src = t.
+ *   y, old_logp, ref_logp   device i32 / f32 / f32, indexed by src.
+ *   adv           device f32 advantage per rollout; row_rollout device i32 [n_rows] gives the
+ *                 rollout of row t (indexed by t, for instance grpo_compact's token_rollout).
+ *   eps_low, eps_high  clip range; beta >= 0 the KL weight.
+ *   denom_tokens  > 0 in agg_mode 0 (for data parallelism: the global kept-token count).
+ *   seq_off, n_seq  used in agg_mode 1 only (device i64 rollout offsets, host count > 0).
+ * Outputs (indexed by t):
+ *   dlogits       device [n_rows, V] contiguous, dtype dlogits_dtype, rounded to nearest even.
+ *   logp_out      device f32 [n_rows], nullable.
+ *   row_loss_out  device f64 [n_rows], nullable: w_t * l_t.
+ *   loss_out      device f64 [1]: the sum, reduced in a fixed order (bitwise reproducible).
+ *   status        device i32 [1], nullable: GRPO_DEVFLAG_* bits.  A row whose y lies outside
+ *                 [0, V) gets logp = NaN, a zero dlogits row and a zero loss term.
+ * Workspace: n_rows f64 when row_loss_out is NULL, else none.
+ * Limits: V >= 1, V*element size <= 16 * 200 KiB; n_rows < 2^31.
+ */
+grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
+                              const int64_t* row_index, int64_t n_rows, int32_t V,
+                              const int32_t* y, const float* old_logp, const float* ref_logp,
+                              const float* adv, const int32_t* row_rollout, float eps_low,
+                              float eps_high, float beta, int32_t agg_mode, int64_t denom_tokens,
+                              const int64_t* seq_off, int64_t n_seq, void* dlogits,
+                              int32_t dlogits_dtype, float* logp_out, double* row_loss_out,
+                              double* loss_out, int32_t* status, void* ws, size_t* ws_bytes,
+                              grpo_stream_t stream);
+
+/*
+ * grpo_loss_tune — launch shape of grpo_loss_fwd_bwd's main kernel for this process.
+ * cluster_ctas: CTAs sharing one logits row (1..16, 0 = automatic); threads: 128/256/512
+ * (0 = automatic); chunks: copies each CTA splits its slice into (1..16, 0 = automatic).
+ * Results do not depend on the shape.  Returns GRPO_ERR_INVALID_ARG for other values.
+ */
+grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int32_t chunks);
+
+/*
+ * Adaptive rollout sampling state, Algorithm 1 (the "adaptive sampling state" and the two
+ * epoch-level buffers).  Plain data: it may be copied or saved and restored byte for byte.
+ */
+typedef struct grpo_ars_state {
+  int32_t G1;          /* initial rollout count G_1 */
+  int32_t n;           /* rollout count chosen for the next step */
+  int32_t have_ref;    /* G'_ref is set */
+  int32_t have_gt;     /* G'_t is set */
+  double g_ref;        /* G'_ref, Eq. 12 */
+  double g_t;          /* G'_t, Eq. 11 */
+  double buf_mean_sum; /* sum of the per-step G'^mean values buffered this epoch */
+  double buf_max_sum;  /* sum of the per-step G'^max values buffered this epoch */
+  int64_t buf_count;   /* number of buffered steps */
+} grpo_ars_state;
+
+/* Reset `st` for initial rollout count G1 >= 2 (n = G1, nothing buffered, no reference). */
+grpo_status grpo_ars_init(grpo_ars_state* st, int32_t G1);
+
+/*
+ * adaptive_rollout_count — ARS update after one step, Eqs. 10-14 and Algorithm 1 (Phases 1a/1b).
+ * kept_per_prompt  host i32 [P], P >= 1: |S(q)| of this step.  Their mean and max are buffered
+ *                  (Eq. 10).  At an epoch end (epoch_end != 0), with alpha = step/total_steps,
+ *                  G'_t = alpha*mean(B_mean) + (1-alpha)*mean(B_max) (Eq. 11); the first epoch end
+ *                  also sets G'_ref = (mean(B_mean) + mean(B_max))/2 (Eq. 12); buffers reset.
+ * Returns the rollout count for step+1:
+ *   max(round(min(G1 - (G'_ref - G'_t), G1)), 2) when both are set and G'_t < G'_ref, else G1
+ *   (Eqs. 13-14; round() is round-half-to-even), or -(grpo_status) on an argument error.
+ * step is 1-based, 1 <= step <= total_steps.  Host only; touches no GPU.
+ */
+int32_t adaptive_rollout_count(grpo_ars_state* st, const int32_t* kept_per_prompt, int32_t P,
+                               int64_t step, int64_t total_steps, int32_t epoch_end);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FASTRL_GRPO_H_ */

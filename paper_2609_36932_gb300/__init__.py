@@ -1,0 +1,13 @@
+"""GB300 kept-token GRPO path of FastRL ("Learn from the Gap", Sec. 3 and Algorithm 1).
+
+The computation lives in libfastrl_grpo.so (hand-written CUDA for sm_103a behind the C ABI of
+include/fastrl_grpo.h); `binding` marshals torch tensors into it.  `workloads` draws the seeded
+synthetic inputs.  Importing the package does not load the library; the first call does.
+"""
+from .binding import (ArsState, GrpoError, adaptive_rollout_count, check_status, grpo_advantage,
+                      grpo_ars_init, grpo_compact, grpo_kernel_launches, grpo_last_error,
+                      grpo_loss_fwd_bwd, grpo_loss_tune, grpo_prune, lib, library_path, version)
+
+__all__ = ["ArsState", "GrpoError", "adaptive_rollout_count", "check_status", "grpo_advantage",
+           "grpo_ars_init", "grpo_compact", "grpo_kernel_launches", "grpo_last_error",
+           "grpo_loss_fwd_bwd", "grpo_loss_tune", "grpo_prune", "lib", "library_path", "version"]

@@ -1,0 +1,328 @@
+"""Python binding of libfastrl_grpo: the C ABI of include/fastrl_grpo.h, one function per entry.
+
+Argument marshalling only: tensors become device pointers, outputs that the caller does not
+pass are allocated with torch on the input's device, and the work is enqueued on the current
+torch CUDA stream.  Every computation runs in the library's CUDA kernels; there is no CPU or
+PyTorch fallback, and loading fails loudly if the library cannot be built or loaded.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+_c_p = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_i64 = ctypes.c_int64
+_f32 = ctypes.c_float
+
+GRPO_DTYPE_F32 = 0
+GRPO_DTYPE_BF16 = 1
+DEVFLAG_BAD_TOKEN = 1
+DEVFLAG_NONFINITE = 2
+DEVFLAG_TIMEOUT = 4
+
+STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTED",
+                3: "GRPO_ERR_WORKSPACE", 4: "GRPO_ERR_CUDA", 5: "GRPO_ERR_TIMEOUT",
+                6: "GRPO_ERR_DEVICE_CHECK"}
+
+# Every function include/fastrl_grpo.h declares.
+EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
+           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_tune", "grpo_ars_init",
+           "adaptive_rollout_count"]
+
+
+class GrpoError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__("%s: %s" % (STATUS_NAMES.get(status, str(status)), message))
+        self.status = status
+
+
+class ArsState(ctypes.Structure):
+    """grpo_ars_state (Algorithm 1's adaptive sampling state)."""
+    _fields_ = [("G1", _i32), ("n", _i32), ("have_ref", _i32), ("have_gt", _i32),
+                ("g_ref", ctypes.c_double), ("g_t", ctypes.c_double),
+                ("buf_mean_sum", ctypes.c_double), ("buf_max_sum", ctypes.c_double),
+                ("buf_count", _i64)]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load libfastrl_grpo.so (building it first if it is missing or stale)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.build()
+    if not os.path.exists(path):
+        raise RuntimeError("libfastrl_grpo.so is missing at %s" % path)
+    L = ctypes.CDLL(path)
+    L.grpo_last_error.restype = ctypes.c_char_p
+    L.grpo_last_error.argtypes = []
+    L.grpo_version.restype = ctypes.c_char_p
+    L.grpo_version.argtypes = []
+    L.grpo_kernel_launches.restype = ctypes.c_uint64
+    L.grpo_kernel_launches.argtypes = []
+    L.grpo_advantage.argtypes = [_c_p, _i32, _i32, _i32, _c_p, _c_p, _c_p]
+    L.grpo_advantage.restype = _i32
+    L.grpo_prune.argtypes = [_c_p, _c_p, _c_p, _i32, _i32, _i64, _i32, _i32, _f32, _i32, _i32, _c_p,
+                             _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_prune.restype = _i32
+    L.grpo_compact.argtypes = [_c_p, _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
+    L.grpo_compact.restype = _i32
+    L.grpo_loss_fwd_bwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                    _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p, _c_p,
+                                    _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_loss_fwd_bwd.restype = _i32
+    L.grpo_loss_tune.argtypes = [_i32, _i32, _i32]
+    L.grpo_loss_tune.restype = _i32
+    L.grpo_ars_init.argtypes = [ctypes.POINTER(ArsState), _i32]
+    L.grpo_ars_init.restype = _i32
+    L.adaptive_rollout_count.argtypes = [ctypes.POINTER(ArsState), _c_p, _i32, _i64, _i64, _i32]
+    L.adaptive_rollout_count.restype = _i32
+    _lib = L
+    return L
+
+
+def _check(rc: int):
+    if rc != 0:
+        raise GrpoError(rc, lib().grpo_last_error().decode(errors="replace"))
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    torch = _torch()
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, dtype, n, what):
+    torch = _torch()
+    if t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (what, dtype, t.dtype))
+    if not t.is_cuda:
+        raise TypeError("%s must be a CUDA tensor" % what)
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % what)
+    if n is not None and t.numel() < n:
+        raise ValueError("%s has %d elements, needs %d" % (what, t.numel(), n))
+    return t
+
+
+def _workspace(nbytes: int, device, ws=None):
+    torch = _torch()
+    if nbytes == 0:
+        return None
+    if ws is not None and ws.numel() >= nbytes + 256:
+        return ws
+    return torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+
+
+def _aligned(ws):
+    """A 256-byte aligned view of a workspace tensor."""
+    if ws is None:
+        return None, 0
+    p = ws.data_ptr()
+    pad = (-p) % 256
+    return ctypes.c_void_p(p + pad), ws.numel() - pad
+
+
+def _ws_args(wst):
+    """(ws pointer, pointer to its size) for a real call; (NULL, NULL) when no workspace."""
+    if wst is None:
+        return None, None
+    wp, wn = _aligned(wst)
+    return wp, ctypes.byref(ctypes.c_size_t(wn))
+
+
+def version() -> str:
+    return lib().grpo_version().decode()
+
+
+def grpo_kernel_launches() -> int:
+    return int(lib().grpo_kernel_launches())
+
+
+def grpo_last_error() -> str:
+    return lib().grpo_last_error().decode(errors="replace")
+
+
+def grpo_loss_tune(cluster_ctas: int = 0, threads: int = 0, chunks: int = 0):
+    _check(lib().grpo_loss_tune(cluster_ctas, threads, chunks))
+
+
+def grpo_advantage(rewards, G: int, std_mode: int = 0, adv=None, key=None, stream=None):
+    """Eq. 5 on the GPU.  Returns (adv f32, key f64 or None)."""
+    torch = _torch()
+    _need(rewards, torch.float32, None, "rewards")
+    n = rewards.numel()
+    if G < 1 or n % G:
+        raise ValueError("rewards has %d elements, not a multiple of G=%d" % (n, G))
+    P = n // G
+    if adv is None:
+        adv = torch.empty(n, dtype=torch.float32, device=rewards.device)
+    _need(adv, torch.float32, n, "adv")
+    if key is not None:
+        _need(key, torch.float64, n, "key")
+    _check(lib().grpo_advantage(_ptr(rewards), P, G, std_mode, _ptr(adv), _ptr(key), _stream(stream)))
+    return adv, key
+
+
+def grpo_prune(rewards, ids, off, G: int, V: int, ngram_n: int = 1, tau: float = 0.8,
+               keep_cap: int | None = None, dp_divisor: int = 1, keep=None, kept_per_prompt=None,
+               status=None, ws=None, stream=None):
+    """Eqs. 6-9 + Algorithm 1 on the GPU.  Returns (keep u8 [P*G], kept_per_prompt i32 [P])."""
+    torch = _torch()
+    _need(rewards, torch.float32, None, "rewards")
+    n = rewards.numel()
+    P = n // G
+    _need(off, torch.int64, n + 1, "off")
+    _need(ids, torch.int32, None, "ids")
+    T = ids.numel()
+    cap = G if keep_cap is None else int(keep_cap)
+    if keep is None:
+        keep = torch.empty(n, dtype=torch.uint8, device=rewards.device)
+    if kept_per_prompt is None:
+        kept_per_prompt = torch.empty(max(P, 1), dtype=torch.int32, device=rewards.device)
+    L = lib()
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_prune(_ptr(rewards), _ptr(ids), _ptr(off), P, G, T, V, ngram_n, float(tau), cap,
+                        dp_divisor, _ptr(keep), _ptr(kept_per_prompt), _ptr(status), None,
+                        ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, rewards.device, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_prune(_ptr(rewards), _ptr(ids), _ptr(off), P, G, T, V, ngram_n, float(tau), cap,
+                        dp_divisor, _ptr(keep), _ptr(kept_per_prompt), _ptr(status), wp, size,
+                        _stream(stream)))
+    return keep, kept_per_prompt[:P]
+
+
+def grpo_compact(keep, off, kept_idx=None, kept_off=None, src_token=None, token_rollout=None,
+                 counts=None, counts_host=None, stream=None):
+    """Token compaction on the GPU.  Returns a dict of the output tensors (full capacity)."""
+    torch = _torch()
+    _need(keep, torch.uint8, None, "keep")
+    n = keep.numel()
+    _need(off, torch.int64, n + 1, "off")
+    dev = keep.device
+    T = None
+    if src_token is None or token_rollout is None:
+        T = int(off[n].item())
+    if kept_idx is None:
+        kept_idx = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    if kept_off is None:
+        kept_off = torch.empty(n + 1, dtype=torch.int64, device=dev)
+    if src_token is None:
+        src_token = torch.empty(max(T, 1), dtype=torch.int64, device=dev)
+    if token_rollout is None:
+        token_rollout = torch.empty(max(T, 1), dtype=torch.int32, device=dev)
+    if counts is None:
+        counts = torch.empty(2, dtype=torch.int64, device=dev)
+    hp = None if counts_host is None else ctypes.c_void_p(counts_host.data_ptr())
+    _check(lib().grpo_compact(_ptr(keep), _ptr(off), n, _ptr(kept_idx), _ptr(kept_off),
+                              _ptr(src_token), _ptr(token_rollout), _ptr(counts), hp, _stream(stream)))
+    return dict(kept_idx=kept_idx, kept_off=kept_off, src_token=src_token,
+                token_rollout=token_rollout, counts=counts)
+
+
+def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int | None = None,
+                      row_stride: int | None = None, row_index=None, n_rows: int | None = None,
+                      eps_low: float = 0.2, eps_high: float = 0.2, beta: float = 0.04,
+                      agg_mode: int = 0, denom_tokens: int | None = None, seq_off=None,
+                      n_seq: int = 0, dlogits=None, dlogits_dtype=None, logp_out=None,
+                      row_loss_out=None, loss_out=None, status=None, ws=None, stream=None):
+    """Eqs. 1-3 on the GPU.  Returns dict(loss (f64 [1] tensor), dlogits, logp, row_loss)."""
+    torch = _torch()
+    if logits.dtype == torch.bfloat16:
+        ldt = GRPO_DTYPE_BF16
+    elif logits.dtype == torch.float32:
+        ldt = GRPO_DTYPE_F32
+    else:
+        raise TypeError("logits must be bf16 or f32")
+    if not logits.is_cuda:
+        raise TypeError("logits must be a CUDA tensor")
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be 2-D with unit stride along the vocabulary")
+    if V is None:
+        V = logits.shape[1]
+    stride = logits.stride(0) if row_stride is None else int(row_stride)
+    if n_rows is None:
+        n_rows = row_index.numel() if row_index is not None else logits.shape[0]
+    dev = logits.device
+    if dlogits_dtype is None:
+        dlogits_dtype = ldt
+    elif dlogits_dtype in (torch.bfloat16, "bf16"):
+        dlogits_dtype = GRPO_DTYPE_BF16
+    elif dlogits_dtype in (torch.float32, "f32"):
+        dlogits_dtype = GRPO_DTYPE_F32
+    out_t = torch.bfloat16 if dlogits_dtype == GRPO_DTYPE_BF16 else torch.float32
+    if dlogits is None:
+        dlogits = torch.empty((n_rows, V), dtype=out_t, device=dev)
+    _need(dlogits, out_t, n_rows * V, "dlogits")
+    if loss_out is None:
+        loss_out = torch.empty(1, dtype=torch.float64, device=dev)
+    if denom_tokens is None:
+        denom_tokens = max(int(n_rows), 1)
+    _need(y, torch.int32, None, "y")
+    _need(old_logp, torch.float32, None, "old_logp")
+    _need(ref_logp, torch.float32, None, "ref_logp")
+    _need(adv, torch.float32, None, "adv")
+    _need(row_rollout, torch.int32, n_rows, "row_rollout")
+    if row_index is not None:
+        _need(row_index, torch.int64, n_rows, "row_index")
+    L = lib()
+    args_head = (_ptr(logits), ldt, stride, _ptr(row_index), int(n_rows), int(V), _ptr(y),
+                 _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(row_rollout), float(eps_low),
+                 float(eps_high), float(beta), int(agg_mode), int(denom_tokens), _ptr(seq_off),
+                 int(n_seq), _ptr(dlogits), dlogits_dtype, _ptr(logp_out), _ptr(row_loss_out),
+                 _ptr(loss_out), _ptr(status))
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_loss_fwd_bwd(*args_head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, dev, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_loss_fwd_bwd(*args_head, wp, size, _stream(stream)))
+    return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
+
+
+def grpo_ars_init(G1: int) -> ArsState:
+    st = ArsState()
+    _check(lib().grpo_ars_init(ctypes.byref(st), G1))
+    return st
+
+
+def adaptive_rollout_count(state: ArsState, kept_per_prompt, step: int, total_steps: int,
+                           epoch_end: bool) -> int:
+    """Eqs. 10-14 (host).  kept_per_prompt: host integers."""
+    k = np.ascontiguousarray(np.asarray(kept_per_prompt), dtype=np.int32)
+    n = lib().adaptive_rollout_count(ctypes.byref(state), k.ctypes.data_as(_c_p), k.size, step,
+                                     total_steps, int(bool(epoch_end)))
+    if n < 0:
+        _check(-n)
+    return int(n)
+
+
+def check_status(status) -> int:
+    """Raise GrpoError(GRPO_ERR_DEVICE_CHECK) if a device status word has bits set."""
+    v = int(status.item()) if hasattr(status, "item") else int(status)
+    if v:
+        names = [nm for bit, nm in ((DEVFLAG_BAD_TOKEN, "bad token id"),
+                                    (DEVFLAG_NONFINITE, "non-finite logits"),
+                                    (DEVFLAG_TIMEOUT, "copy wait timed out")) if v & bit]
+        raise GrpoError(6, "device status 0x%x: %s" % (v, ", ".join(names)))
+    return v

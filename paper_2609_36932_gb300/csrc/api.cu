@@ -1,0 +1,135 @@
+// Host-side parts of libfastrl_grpo: error reporting, the launch counter, the workspace protocol
+// and adaptive rollout sampling (Sec. 3.3, Eqs. 10-14; Algorithm 1 Phases 1a and 1b).
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "common.cuh"
+
+namespace fastrl {
+
+namespace {
+thread_local char g_msg[512] = {0};
+std::atomic<uint64_t> g_launches{0};
+}  // namespace
+
+grpo_status fail(grpo_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+void clear_error() { g_msg[0] = 0; }
+
+void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+grpo_status check_launch(const char* what) {
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+  return GRPO_OK;
+}
+
+grpo_status workspace_check(void* ws, size_t* ws_bytes, size_t need, const char* who,
+                            bool* query_only) {
+  *query_only = false;
+  if (ws == nullptr) {
+    if (ws_bytes == nullptr) {
+      if (need == 0) return GRPO_OK;
+      return fail(GRPO_ERR_WORKSPACE, "%s: needs %zu workspace bytes but ws and ws_bytes are NULL",
+                  who, need);
+    }
+    *ws_bytes = need;
+    *query_only = true;
+    return GRPO_OK;
+  }
+  if (ws_bytes == nullptr || *ws_bytes < need)
+    return fail(GRPO_ERR_WORKSPACE, "%s: workspace of %zu bytes given, %zu needed", who,
+                ws_bytes ? *ws_bytes : (size_t)0, need);
+  if (reinterpret_cast<uintptr_t>(ws) % 256 != 0)
+    return fail(GRPO_ERR_WORKSPACE, "%s: workspace must be 256-byte aligned", who);
+  return GRPO_OK;
+}
+
+}  // namespace fastrl
+
+using namespace fastrl;
+
+extern "C" const char* grpo_last_error(void) { return g_msg; }
+
+extern "C" const char* grpo_version(void) { return "fastrl_grpo 0.1.0 (sm_103a)"; }
+
+extern "C" uint64_t grpo_kernel_launches(void) {
+  return g_launches.load(std::memory_order_relaxed);
+}
+
+extern "C" grpo_status grpo_ars_init(grpo_ars_state* st, int32_t G1) {
+  clear_error();
+  if (st == nullptr) return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_init: state is NULL");
+  if (G1 < 2) return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_init: G1 = %d, must be >= 2", G1);
+  std::memset(st, 0, sizeof *st);
+  st->G1 = G1;
+  st->n = G1;
+  return GRPO_OK;
+}
+
+// One ARS update.  The epoch buffers are kept as running sums in append order, which gives the
+// same fp64 means as summing the buffered values at the epoch end.
+extern "C" int32_t adaptive_rollout_count(grpo_ars_state* st, const int32_t* kept_per_prompt,
+                                          int32_t P, int64_t step, int64_t total_steps,
+                                          int32_t epoch_end) {
+  clear_error();
+  if (st == nullptr || kept_per_prompt == nullptr) {
+    fail(GRPO_ERR_INVALID_ARG, "adaptive_rollout_count: NULL argument");
+    return -GRPO_ERR_INVALID_ARG;
+  }
+  if (P < 1 || step < 1 || total_steps < step || st->G1 < 2) {
+    fail(GRPO_ERR_INVALID_ARG,
+         "adaptive_rollout_count: need P >= 1, 1 <= step <= total_steps, G1 >= 2 "
+         "(P=%d step=%lld total=%lld G1=%d)",
+         P, (long long)step, (long long)total_steps, st->G1);
+    return -GRPO_ERR_INVALID_ARG;
+  }
+  // Eq. 10: mean and max of the retained counts over this step's prompts.
+  int64_t total = 0;
+  int32_t most = kept_per_prompt[0];
+  for (int32_t q = 0; q < P; ++q) {
+    if (kept_per_prompt[q] < 0) {
+      fail(GRPO_ERR_INVALID_ARG, "adaptive_rollout_count: kept_per_prompt[%d] < 0", q);
+      return -GRPO_ERR_INVALID_ARG;
+    }
+    total += kept_per_prompt[q];
+    if (kept_per_prompt[q] > most) most = kept_per_prompt[q];
+  }
+  st->buf_mean_sum += (double)total / (double)P;
+  st->buf_max_sum += (double)most;
+  st->buf_count += 1;
+  if (epoch_end) {
+    const double alpha = (double)step / (double)total_steps;
+    const double mean_bar = st->buf_mean_sum / (double)st->buf_count;
+    const double max_bar = st->buf_max_sum / (double)st->buf_count;
+    st->g_t = alpha * mean_bar + (1.0 - alpha) * max_bar;  // Eq. 11
+    st->have_gt = 1;
+    if (!st->have_ref) {  // Eq. 12, once, after the first epoch
+      st->g_ref = (mean_bar + max_bar) / 2.0;
+      st->have_ref = 1;
+    }
+    st->buf_mean_sum = 0.0;
+    st->buf_max_sum = 0.0;
+    st->buf_count = 0;
+  }
+  // Eqs. 13-14 for the next step.
+  int32_t n = st->G1;
+  if (st->have_gt && st->have_ref && st->g_t < st->g_ref) {
+    const double delta = st->g_ref - st->g_t;
+    double target = (double)st->G1 - delta;
+    if (target > (double)st->G1) target = (double)st->G1;
+    const int32_t r = (int32_t)std::nearbyint(target);  // current rounding mode: half to even
+    n = r > 2 ? r : 2;
+  }
+  st->n = n;
+  return n;
+}

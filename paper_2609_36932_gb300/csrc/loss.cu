@@ -1,0 +1,674 @@
+// grpo_loss_fwd_bwd: fused GRPO token loss and dlogits, Sec. 3.1 Eqs. 1-3, one read of the
+// logits and one write of the gradient.
+//
+// Design (HBM-bound: ~2 bytes read + 2-4 bytes written per vocabulary entry, ~10 flops):
+//   * A row of V logits is split over a cluster of C CTAs; CTA c holds the slice
+//     [c*slice, (c+1)*slice) of the row in shared memory for the whole row, so the logits are
+//     read from HBM exactly once.  (V = 152064 bf16 is 297 KiB, more than one SM holds; C = 8
+//     gives 37 KiB slices and several resident CTAs per SM.)
+//   * Each slice arrives by non-tensor bulk copies (cp.async.bulk, 16-byte granules) in a few
+//     chunks, each completing on its own mbarrier, so the CTA starts reducing chunk 0 while
+//     the rest is in flight.
+//   * Pass A: per-thread online max and sum of exp (base 2, MUFU ex2) over the slice, leaving
+//     out the sampled token y; warp shuffles and shared memory combine the CTA's threads.
+//   * Exchange: each CTA publishes (max, sum, z_y) in shared memory; after a cluster barrier
+//     warp 0 reads every CTA's entry through distributed shared memory (mapa +
+//     ld.shared::cluster) and forms the row's log-sum-exp, log-prob, ratio, clipped surrogate,
+//     KL term and gradient coefficient.  Every CTA of the cluster computes the same numbers.
+//   * Pass B: dlogits[v] = -coef * exp(z_v - lse) (+coef at v = y) from the shared-memory slice,
+//     written with 16-byte streaming stores.  As soon as chunk k has been consumed, thread 0
+//     starts the copy of chunk k of the cluster's next row into the same buffer.
+//   * The grid is persistent: as many clusters as fit at once; cluster i takes rows i, i+n, ...
+//   * Per-row loss terms go to a buffer; a one-CTA kernel sums them in a fixed order.
+// Every wait on a copy is bounded (about one second); on expiry the kernel records
+// GRPO_DEVFLAG_TIMEOUT, stops waiting and issuing copies, and runs to the end.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cmath>
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "common.cuh"
+
+namespace fastrl {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+constexpr int kMaxChunks = 16;
+constexpr int kMaxCluster = 16;
+
+struct LossArgs {
+  const char* logits;
+  int64_t row_stride_bytes;
+  const int64_t* row_index;
+  int64_t n_rows;
+  int32_t V;
+  const int32_t* y;
+  const float* old_logp;
+  const float* ref_logp;
+  const float* adv;
+  const int32_t* row_rollout;
+  double clip_lo;  // 1 - eps_low
+  double clip_hi;  // 1 + eps_high
+  float beta;
+  int32_t agg_mode;
+  double inv_denom;  // agg 0: 1 / denom_tokens
+  const int64_t* seq_off;
+  double inv_nseq;  // agg 1: 1 / n_seq
+  char* dlogits;
+  float* logp_out;
+  double* row_loss;
+  int32_t* status;
+  int32_t slice;       // elements per CTA, a multiple of the 16-byte vector width
+  int32_t chunk_vecs;  // 16-byte vectors per copy
+  int32_t n_chunks;
+  int32_t bulk;     // rows 16-byte aligned: slices arrive by bulk copies
+  int32_t out_vec;  // dlogits rows 16-byte aligned: vector stores
+};
+
+// ---- PTX helpers ------------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_count_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t local_addr, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local_addr), "r"(rank));
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(remote)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                              uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ float ex2(float x) {  // 2^x on the MUFU, subnormal results kept
+  float y;
+  asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// ---- element formats --------------------------------------------------------------------------
+
+template <typename T>
+struct Fmt;
+template <>
+struct Fmt<float> {
+  static constexpr int kVec = 4;  // elements per 16 bytes
+  __device__ static void unpack(const uint4& q, float (&f)[4]) {
+    f[0] = __uint_as_float(q.x);
+    f[1] = __uint_as_float(q.y);
+    f[2] = __uint_as_float(q.z);
+    f[3] = __uint_as_float(q.w);
+  }
+  __device__ static float load(const float* p) { return *p; }
+  __device__ static void store(float* p, float v) { *p = v; }
+};
+template <>
+struct Fmt<__nv_bfloat16> {
+  static constexpr int kVec = 8;
+  __device__ static void unpack(const uint4& q, float (&f)[8]) {
+    f[0] = __uint_as_float(q.x << 16);
+    f[1] = __uint_as_float(q.x & 0xffff0000u);
+    f[2] = __uint_as_float(q.y << 16);
+    f[3] = __uint_as_float(q.y & 0xffff0000u);
+    f[4] = __uint_as_float(q.z << 16);
+    f[5] = __uint_as_float(q.z & 0xffff0000u);
+    f[6] = __uint_as_float(q.w << 16);
+    f[7] = __uint_as_float(q.w & 0xffff0000u);
+  }
+  __device__ static float load(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+  __device__ static void store(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Store kVec results at p (aligned to kVec * sizeof(OutT) bytes), streaming (evict-first).
+template <typename OutT, int kVec>
+__device__ __forceinline__ void store_vec(OutT* p, const float (&d)[kVec]);
+template <>
+__device__ __forceinline__ void store_vec<__nv_bfloat16, 8>(__nv_bfloat16* p, const float (&d)[8]) {
+  __stcs(reinterpret_cast<uint4*>(p), make_uint4(pack_bf16x2(d[0], d[1]), pack_bf16x2(d[2], d[3]),
+                                                 pack_bf16x2(d[4], d[5]), pack_bf16x2(d[6], d[7])));
+}
+template <>
+__device__ __forceinline__ void store_vec<float, 8>(float* p, const float (&d)[8]) {
+  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0], d[1], d[2], d[3]));
+  __stcs(reinterpret_cast<float4*>(p) + 1, make_float4(d[4], d[5], d[6], d[7]));
+}
+template <>
+__device__ __forceinline__ void store_vec<float, 4>(float* p, const float (&d)[4]) {
+  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0], d[1], d[2], d[3]));
+}
+template <>
+__device__ __forceinline__ void store_vec<__nv_bfloat16, 4>(__nv_bfloat16* p, const float (&d)[4]) {
+  __stcs(reinterpret_cast<uint2*>(p), make_uint2(pack_bf16x2(d[0], d[1]), pack_bf16x2(d[2], d[3])));
+}
+
+// Combine two (max, sum of exp relative to max) pairs.
+__device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float so) {
+  const float M = fmaxf(m, mo);
+  const float a = (m == -INFINITY) ? 0.f : s * ex2((m - M) * kLog2e);
+  const float b = (mo == -INFINITY) ? 0.f : so * ex2((mo - M) * kLog2e);
+  m = M;
+  s = a + b;
+}
+
+// ---- the kernel -------------------------------------------------------------------------------
+
+template <typename InT, typename OutT, int kThreads>
+__global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
+  constexpr int kVec = Fmt<InT>::kVec;
+  constexpr int kWarps = kThreads / 32;
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int buf_bytes = (int)align_up((size_t)a.slice * sizeof(InT), 128);
+  InT* buf = reinterpret_cast<InT*>(smem);
+  const uint4* buf4 = reinterpret_cast<const uint4*>(smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + buf_bytes);
+  float4* stats = reinterpret_cast<float4*>(smem + buf_bytes + kMaxChunks * 8);  // 2 slots
+  float* red = reinterpret_cast<float*>(stats + 2);                               // 2*kWarps
+  float* rowsc = red + 2 * kWarps;                                                // 4 floats
+  int* abort_flag = reinterpret_cast<int*>(rowsc + 4);
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t C = cluster_nctarank();
+  const int64_t ncl = cluster_count_x();
+  const int s0 = (int)rank * a.slice;
+  const int len = max(0, min(a.V - s0, a.slice));  // my slice's elements
+  const int nvec = a.bulk ? len / kVec : 0;        // vectors that arrive by bulk copy
+  const int tail0 = nvec * kVec;                   // first element loaded one by one
+  const uint32_t buf_s = smem_addr(buf);
+  const uint32_t bar_s = smem_addr(bars);
+
+  if (tid == 0) {
+    for (int k = 0; k < a.n_chunks; ++k) mbar_init(bar_s + 8 * k, 1);
+    *abort_flag = 0;
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  auto row_base = [&](int64_t row) -> const char* {
+    const int64_t src = a.row_index ? a.row_index[row] : row;
+    return a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
+  };
+  auto issue_chunk = [&](const char* g, int k) {  // thread 0 only
+    const int v0 = k * a.chunk_vecs;
+    const int v1 = min(nvec, v0 + a.chunk_vecs);
+    const uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
+    mbar_expect_tx(bar_s + 8 * k, bytes);
+    if (bytes) bulk_copy_g2s(buf_s + v0 * 16, g + (int64_t)v0 * 16, bytes, bar_s + 8 * k);
+  };
+  auto wait_chunk = [&](int k, uint32_t parity) {
+    if (*(volatile int*)abort_flag) return;
+    if (mbar_try_wait(bar_s + 8 * k, parity)) return;
+    const uint64_t t0 = global_timer_ns();
+    while (!mbar_try_wait(bar_s + 8 * k, parity)) {
+      if (*(volatile int*)abort_flag) return;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *(volatile int*)abort_flag = 1;
+        if (a.status) atomicOr(a.status, GRPO_DEVFLAG_TIMEOUT);
+        return;
+      }
+    }
+  };
+
+  int64_t row = cluster_id_x();
+  uint32_t phase = 0;
+  if (tid == 0 && row < a.n_rows) {
+    const char* g = row_base(row);
+    for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
+  }
+
+  for (; row < a.n_rows; row += ncl, phase ^= 1u) {
+    const int64_t src = a.row_index ? a.row_index[row] : row;
+    const int32_t yv = a.y[src];
+    const bool yvalid = yv >= 0 && yv < a.V;
+    const int yl = yvalid ? yv - s0 : -1;  // y's position in my slice, if there
+    const char* grow = a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
+
+    // ---- pass A: max and sum of exp over my elements, y left out ----
+    float m = -INFINITY, s = 0.f;
+    for (int k = 0; k < a.n_chunks; ++k) {
+      wait_chunk(k, phase);
+      const int v0 = k * a.chunk_vecs;
+      const int v1 = min(nvec, v0 + a.chunk_vecs);
+      const bool last = (k == a.n_chunks - 1);
+      float cm = -INFINITY;
+      for (int j = v0 + tid; j < v1; j += kThreads) {
+        float f[kVec];
+        Fmt<InT>::unpack(buf4[j], f);
+#pragma unroll
+        for (int i = 0; i < kVec; ++i) cm = fmaxf(cm, f[i]);
+      }
+      if (last) {
+        for (int e = tail0 + tid; e < len; e += kThreads) {
+          const InT v = *reinterpret_cast<const InT*>(grow + (int64_t)e * sizeof(InT));
+          buf[e] = v;  // this thread reads it back below and in pass B
+          cm = fmaxf(cm, Fmt<InT>::load(&buf[e]));
+        }
+      }
+      if (cm > m) {
+        s = (m == -INFINITY) ? 0.f : s * ex2((m - cm) * kLog2e);
+        m = cm;
+      }
+      if (m != -INFINITY) {
+        const float sh = -m * kLog2e;
+        for (int j = v0 + tid; j < v1; j += kThreads) {
+          float f[kVec];
+          Fmt<InT>::unpack(buf4[j], f);
+          const int yi = yl - j * kVec;
+          float acc = 0.f;
+          if ((unsigned)yi < (unsigned)kVec) {
+#pragma unroll
+            for (int i = 0; i < kVec; ++i)
+              if (i != yi) acc += ex2(fmaf(f[i], kLog2e, sh));
+          } else {
+#pragma unroll
+            for (int i = 0; i < kVec; ++i) acc += ex2(fmaf(f[i], kLog2e, sh));
+          }
+          s += acc;
+        }
+        if (last)
+          for (int e = tail0 + tid; e < len; e += kThreads)
+            if (e != yl) s += ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, sh));
+      }
+    }
+    // CTA reduction of (m, s)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float mo = __shfl_xor_sync(0xffffffffu, m, o);
+      const float so = __shfl_xor_sync(0xffffffffu, s, o);
+      lse_combine(m, s, mo, so);
+    }
+    if (lane == 0) {
+      red[2 * warp] = m;
+      red[2 * warp + 1] = s;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      m = lane < kWarps ? red[2 * lane] : -INFINITY;
+      s = lane < kWarps ? red[2 * lane + 1] : 0.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float mo = __shfl_xor_sync(0xffffffffu, m, o);
+        const float so = __shfl_xor_sync(0xffffffffu, s, o);
+        lse_combine(m, s, mo, so);
+      }
+      if (lane == 0) {
+        const float zy = ((unsigned)yl < (unsigned)len) ? Fmt<InT>::load(&buf[yl]) : 0.f;
+        stats[phase] = make_float4(m, s, zy, 0.f);
+      }
+    }
+    cluster_sync();  // every CTA's (max, sum, z_y) for this row is published
+
+    // ---- exchange and row scalars (warp 0) ----
+    if (warp == 0) {
+      const uint32_t st_addr = smem_addr(&stats[phase]);
+      float mc = -INFINITY, sc = 0.f;
+      if (lane < (int)C) {
+        const float4 v = ld_cluster_f4(st_addr, lane);
+        mc = v.x;
+        sc = v.y;
+      }
+      float M = mc;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      float term = (mc == -INFINITY) ? 0.f : sc * expf(mc - M);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) term += __shfl_xor_sync(0xffffffffu, term, o);
+      if (lane == 0) {
+        float neg_scale = 0.f, dy = 0.f, shB = 0.f;
+        if (!yvalid) {
+          if (rank == 0) {
+            if (a.logp_out) a.logp_out[row] = __int_as_float(0x7fc00000);
+            a.row_loss[row] = 0.0;
+            if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
+          }
+        } else {
+          const float zy = ld_cluster_f4(st_addr, (uint32_t)(yv / a.slice)).z;
+          const float S_excl = term;
+          const float ey = expf(zy - M);
+          const float S = S_excl + ey;
+          const float logp = (zy - M) - logf(S);
+          // Eq. 1: ratio, clipped surrogate, KL term; Eqs. 2-3: gradient coefficient.
+          const float A = a.adv[a.row_rollout[row]];
+          const float rho = expf(logp - a.old_logp[src]);
+          const double rho_d = (double)rho;
+          const float clipped = (float)fmin(fmax(rho_d, a.clip_lo), a.clip_hi);
+          const float surr = fminf(rho * A, clipped * A);
+          const float x = a.ref_logp[src] - logp;
+          const float em1 = expm1f(x);
+          const float kl = em1 - x;
+          const float ell = -(surr - a.beta * kl);
+          double w;
+          if (a.agg_mode == 0) {
+            w = a.inv_denom;
+          } else {
+            const int32_t r = a.row_rollout[row];
+            w = a.inv_nseq / (double)(a.seq_off[r + 1] - a.seq_off[r]);
+          }
+          const bool c = (A >= 0.f) ? (rho_d <= a.clip_hi) : (rho_d >= a.clip_lo);
+          const float g = -((c ? rho * A : 0.f) + a.beta * em1);
+          const float coef = (float)(w * (double)g);
+          neg_scale = -coef / S;
+          dy = coef * (S_excl / S);
+          shB = -M * kLog2e;
+          if (rank == 0) {
+            if (a.logp_out) a.logp_out[row] = logp;
+            a.row_loss[row] = w * (double)ell;
+            if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
+          }
+        }
+        rowsc[0] = neg_scale;
+        rowsc[1] = dy;
+        rowsc[2] = shB;
+        rowsc[3] = yvalid ? 0.f : 1.f;
+      }
+    }
+    __syncthreads();
+
+    // ---- pass B: dlogits from the shared-memory slice; refill chunk by chunk ----
+    const float neg_scale = rowsc[0], dy = rowsc[1], shB = rowsc[2];
+    const bool zero_row = rowsc[3] != 0.f;
+    OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V + s0;
+    const int64_t next = row + ncl;
+    const char* gnext = (tid == 0 && next < a.n_rows) ? row_base(next) : nullptr;
+    for (int k = 0; k < a.n_chunks; ++k) {
+      const int v0 = k * a.chunk_vecs;
+      const int v1 = min(nvec, v0 + a.chunk_vecs);
+      for (int j = v0 + tid; j < v1; j += kThreads) {
+        float f[kVec], d[kVec];
+        Fmt<InT>::unpack(buf4[j], f);
+#pragma unroll
+        for (int i = 0; i < kVec; ++i) d[i] = zero_row ? 0.f : neg_scale * ex2(fmaf(f[i], kLog2e, shB));
+        const int yi = yl - j * kVec;
+        if ((unsigned)yi < (unsigned)kVec && !zero_row) {
+#pragma unroll
+          for (int i = 0; i < kVec; ++i)
+            if (i == yi) d[i] = dy;
+        }
+        if (a.out_vec) {
+          store_vec<OutT, kVec>(orow + j * kVec, d);
+        } else {
+#pragma unroll
+          for (int i = 0; i < kVec; ++i) Fmt<OutT>::store(orow + j * kVec + i, d[i]);
+        }
+      }
+      if (k == a.n_chunks - 1) {
+        for (int e = tail0 + tid; e < len; e += kThreads) {
+          float d = zero_row ? 0.f : neg_scale * ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, shB));
+          if (e == yl && !zero_row) d = dy;
+          Fmt<OutT>::store(orow + e, d);
+        }
+      }
+      __syncthreads();  // chunk k consumed by every thread
+      if (gnext && !*(volatile int*)abort_flag) issue_chunk(gnext, k);
+    }
+  }
+  cluster_sync();  // partners are done reading this CTA's shared memory
+}
+
+__global__ void sum_rows_kernel(const double* __restrict__ v, int64_t n, double* __restrict__ out) {
+  __shared__ double sh[1024];
+  double acc = 0.0;
+  for (int64_t i = threadIdx.x; i < n; i += 1024) acc += v[i];
+  sh[threadIdx.x] = acc;
+  __syncthreads();
+  for (int s = 512; s > 0; s >>= 1) {
+    if ((int)threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out = sh[0];
+}
+
+// ---- host side --------------------------------------------------------------------------------
+
+struct Tune {
+  int cluster = 0, threads = 0, chunks = 0;
+};
+Tune g_tune;
+std::mutex g_mu;
+std::map<std::tuple<const void*, int, int, int>, int> g_max_clusters;  // (kernel, dev, C, smem)
+
+using KernelFn = void (*)(LossArgs);
+
+template <typename InT, typename OutT>
+KernelFn pick_kernel(int threads) {
+  switch (threads) {
+    case 128: return grpo_loss_kernel<InT, OutT, 128>;
+    case 512: return grpo_loss_kernel<InT, OutT, 512>;
+    default: return grpo_loss_kernel<InT, OutT, 256>;
+  }
+}
+
+KernelFn kernel_for(int in_dtype, int out_dtype, int threads) {
+  if (in_dtype == GRPO_DTYPE_BF16)
+    return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16>(threads)
+                                        : pick_kernel<__nv_bfloat16, float>(threads);
+  return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<float, __nv_bfloat16>(threads)
+                                      : pick_kernel<float, float>(threads);
+}
+
+}  // namespace
+}  // namespace fastrl
+
+using namespace fastrl;
+
+extern "C" grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int32_t chunks) {
+  clear_error();
+  if (cluster_ctas < 0 || cluster_ctas > kMaxCluster)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_loss_tune: cluster_ctas = %d", cluster_ctas);
+  if (threads != 0 && threads != 128 && threads != 256 && threads != 512)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_loss_tune: threads = %d", threads);
+  if (chunks < 0 || chunks > kMaxChunks)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_loss_tune: chunks = %d", chunks);
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_tune.cluster = cluster_ctas;
+  g_tune.threads = threads;
+  g_tune.chunks = chunks;
+  return GRPO_OK;
+}
+
+extern "C" grpo_status grpo_loss_fwd_bwd(
+    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
+    int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,
+    const float* adv, const int32_t* row_rollout, float eps_low, float eps_high, float beta,
+    int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq, void* dlogits,
+    int32_t dlogits_dtype, float* logp_out, double* row_loss_out, double* loss_out, int32_t* status,
+    void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  const char* who = "grpo_loss_fwd_bwd";
+  if (logits_dtype != GRPO_DTYPE_BF16 && logits_dtype != GRPO_DTYPE_F32)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: logits_dtype = %d", who, logits_dtype);
+  if (dlogits_dtype != GRPO_DTYPE_BF16 && dlogits_dtype != GRPO_DTYPE_F32)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: dlogits_dtype = %d", who, dlogits_dtype);
+  if (n_rows < 0 || n_rows >= (int64_t(1) << 31))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: n_rows = %lld", who, (long long)n_rows);
+  if (V < 1 || row_stride < V)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: V = %d, row_stride = %lld", who, V, (long long)row_stride);
+  if (agg_mode != 0 && agg_mode != 1)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: agg_mode = %d", who, agg_mode);
+  if (agg_mode == 0 && denom_tokens <= 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: denom_tokens = %lld", who, (long long)denom_tokens);
+  if (agg_mode == 1 && (seq_off == nullptr || n_seq <= 0))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: agg_mode 1 needs seq_off and n_seq > 0", who);
+  if (!(beta >= 0.f) || !(eps_low >= 0.f) || !(eps_high >= 0.f))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: beta, eps_low, eps_high must be >= 0", who);
+  const size_t need = row_loss_out ? 0 : align_up((size_t)n_rows * 8, 256);
+  bool query = false;
+  grpo_status st = workspace_check(ws, ws_bytes, need, who, &query);
+  if (st != GRPO_OK || query) return st;
+  if (loss_out == nullptr) return fail(GRPO_ERR_INVALID_ARG, "%s: loss_out is NULL", who);
+  double* row_loss = row_loss_out ? row_loss_out : static_cast<double*>(ws);
+  cudaStream_t s = as_stream(stream);
+  if (n_rows == 0) {
+    sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, 0, loss_out);
+    count_launches(1);
+    return check_launch(who);
+  }
+  if (!logits || !y || !old_logp || !ref_logp || !adv || !row_rollout || !dlogits)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: NULL array", who);
+
+  Tune tune;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    tune = g_tune;
+  }
+  const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+  const int out_bytes = dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+  const int vec = 16 / in_bytes;
+  const int threads = tune.threads ? tune.threads : 256;
+  // Cluster size: the smallest C whose slices are at most ~40 KiB (several CTAs per SM).
+  int C = tune.cluster;
+  if (C == 0) {
+    C = 1;
+    while (C < 8 && (int64_t)V * in_bytes > (int64_t)C * 40 * 1024) C *= 2;
+  }
+  int slice = (int)align_up((size_t)((V + C - 1) / C), vec);
+  while (C > 1 && (int64_t)(C - 1) * slice >= V) {  // no empty slices
+    --C;
+    slice = (int)align_up((size_t)((V + C - 1) / C), vec);
+  }
+  const size_t slice_bytes = (size_t)slice * in_bytes;
+  int chunks = tune.chunks ? tune.chunks : (int)std::min<size_t>(8, std::max<size_t>(1, slice_bytes / 8192));
+  const int slice_vecs = slice / vec;
+  int chunk_vecs = (slice_vecs + chunks - 1) / chunks;
+  if (chunk_vecs < 1) chunk_vecs = 1;
+  chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
+  if (chunks < 1) chunks = 1;
+  const size_t smem = align_up(slice_bytes, 128) + kMaxChunks * 8 + 2 * 16 +
+                      2 * (threads / 32) * 4 + 4 * 4 + 16;
+  if (smem > 227 * 1024)
+    return fail(GRPO_ERR_UNSUPPORTED, "%s: V = %d needs %zu bytes of shared memory per CTA at %d CTAs", who,
+                V, smem, C);
+
+  LossArgs a;
+  a.logits = static_cast<const char*>(logits);
+  a.row_stride_bytes = row_stride * in_bytes;
+  a.row_index = row_index;
+  a.n_rows = n_rows;
+  a.V = V;
+  a.y = y;
+  a.old_logp = old_logp;
+  a.ref_logp = ref_logp;
+  a.adv = adv;
+  a.row_rollout = row_rollout;
+  a.clip_lo = 1.0 - (double)eps_low;
+  a.clip_hi = 1.0 + (double)eps_high;
+  a.beta = beta;
+  a.agg_mode = agg_mode;
+  a.inv_denom = agg_mode == 0 ? 1.0 / (double)denom_tokens : 0.0;
+  a.seq_off = seq_off;
+  a.inv_nseq = agg_mode == 1 ? 1.0 / (double)n_seq : 0.0;
+  a.dlogits = static_cast<char*>(dlogits);
+  a.logp_out = logp_out;
+  a.row_loss = row_loss;
+  a.status = status;
+  a.slice = slice;
+  a.chunk_vecs = chunk_vecs;
+  a.n_chunks = chunks;
+  a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
+  a.out_vec = (reinterpret_cast<uintptr_t>(dlogits) % 16 == 0) && (((int64_t)V * out_bytes) % 16 == 0);
+
+  KernelFn fn = kernel_for(logits_dtype, dlogits_dtype, threads);
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess && C > 8)
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
+
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(threads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int max_cl = 0;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    const auto key = std::make_tuple((const void*)fn, dev, C, (int)smem);
+    auto it = g_max_clusters.find(key);
+    if (it != g_max_clusters.end()) {
+      max_cl = it->second;
+    } else {
+      cfg.gridDim = dim3(C, 1, 1);
+      e = cudaOccupancyMaxActiveClusters(&max_cl, fn, &cfg);
+      if (e != cudaSuccess)
+        return fail(GRPO_ERR_CUDA, "%s: cudaOccupancyMaxActiveClusters: %s", who, cudaGetErrorString(e));
+      if (max_cl < 1)
+        return fail(GRPO_ERR_UNSUPPORTED, "%s: a cluster of %d CTAs with %zu bytes each cannot be resident",
+                    who, C, smem);
+      g_max_clusters[key] = max_cl;
+    }
+  }
+  const int64_t n_clusters = std::min<int64_t>(n_rows, max_cl);
+  cfg.gridDim = dim3((unsigned)(n_clusters * C), 1, 1);
+  e = cudaLaunchKernelEx(&cfg, fn, a);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: launch: %s", who, cudaGetErrorString(e));
+  sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, n_rows, loss_out);
+  count_launches(2);
+  return check_launch(who);
+}

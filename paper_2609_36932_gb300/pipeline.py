@@ -1,0 +1,147 @@
+"""One FastRL step's data-parallel core on one GPU, through the C ABI (orchestration only).
+
+    grpo_advantage  ->  grpo_prune  ->  grpo_compact  ->  [host: kept counts, ARS]  ->
+    grpo_loss_fwd_bwd over the kept tokens only
+
+This mirrors Algorithm 1's order within a step: advantages (Eq. 5), MDAP pruning (Phase 2),
+the ARS update from the kept counts (Phase 1b), then the policy loss over the selected
+trajectories.  Every computation is a library kernel; this class only owns the device buffers,
+passes pointers and performs the step's single device-to-host read (the kept counts, which the
+host needs for ARS and to size the loss launch).
+"""
+from __future__ import annotations
+
+import dataclasses
+
+from . import binding as B
+
+
+@dataclasses.dataclass
+class StepParams:
+    G: int
+    V: int
+    ngram_n: int = 1
+    tau: float = 0.8
+    keep_cap: int | None = None
+    dp_divisor: int = 1
+    eps_low: float = 0.2
+    eps_high: float = 0.2
+    beta: float = 0.04
+    agg_mode: int = 0
+    dlogits_dtype: str = "bf16"
+    std_mode: int = 0
+
+
+class GrpoStep:
+    """Device buffers and the launch sequence of one step.
+
+    Inputs (device tensors, resident): rewards f32 [P*G], ids i32 [T] (also the sampled tokens y),
+    off i64 [P*G+1], logits [T, V] (bf16 or f32, all tokens of all rollouts), old_logp and
+    ref_logp f32 [T].  dlogits are produced for the kept tokens only, in compacted order."""
+
+    def __init__(self, params: StepParams, rewards, ids, off, logits, old_logp, ref_logp,
+                 ars_total_steps: int = 1, steps_per_epoch: int = 1, G1: int | None = None):
+        import torch
+        self.torch = torch
+        self.p = params
+        self.rewards, self.ids, self.off = rewards, ids, off
+        self.logits, self.old, self.ref = logits, old_logp, ref_logp
+        dev = rewards.device
+        self.dev = dev
+        n = rewards.numel()
+        self.P = n // params.G
+        self.T = ids.numel()
+        self.adv = torch.empty(n, dtype=torch.float32, device=dev)
+        self.keep = torch.empty(n, dtype=torch.uint8, device=dev)
+        self.kpp = torch.empty(max(self.P, 1), dtype=torch.int32, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.kept_idx = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+        self.kept_off = torch.empty(n + 1, dtype=torch.int64, device=dev)
+        self.src_token = torch.empty(max(self.T, 1), dtype=torch.int64, device=dev)
+        self.token_rollout = torch.empty(max(self.T, 1), dtype=torch.int32, device=dev)
+        self.counts = torch.empty(2, dtype=torch.int64, device=dev)
+        self.counts_host = torch.empty(2, dtype=torch.int64, pin_memory=True)
+        self.kpp_host = torch.empty(max(self.P, 1), dtype=torch.int32, pin_memory=True)
+        self.loss = torch.empty(1, dtype=torch.float64, device=dev)
+        self.logp = torch.empty(max(self.T, 1), dtype=torch.float32, device=dev)
+        self.out_dtype = torch.bfloat16 if params.dlogits_dtype == "bf16" else torch.float32
+        self.dlogits = None
+        self.prune_ws = None
+        self.loss_ws = None
+        self.ars = B.grpo_ars_init(G1 if G1 is not None else params.G)
+        self.ars_total = ars_total_steps
+        self.steps_per_epoch = steps_per_epoch
+        self.step_index = 0
+        self.n_next = params.G
+        self.T_kept = 0
+        self.K = 0
+        self.set_workspaces()
+
+    def _ensure_dlogits(self, rows: int):
+        if self.dlogits is None or self.dlogits.shape[0] < rows:
+            self.dlogits = None
+            self.dlogits = self.torch.empty((max(rows, 1), self.p.V), dtype=self.out_dtype,
+                                            device=self.dev)
+
+    def select(self):
+        """Advantages, pruning and compaction; then the step's one host read (kept counts)."""
+        p = self.p
+        B.grpo_advantage(self.rewards, p.G, p.std_mode, adv=self.adv)
+        B.grpo_prune(self.rewards, self.ids, self.off, p.G, p.V, p.ngram_n, p.tau, p.keep_cap,
+                     p.dp_divisor, keep=self.keep, kept_per_prompt=self.kpp, status=self.status,
+                     ws=self.prune_ws)
+        B.grpo_compact(self.keep, self.off, kept_idx=self.kept_idx, kept_off=self.kept_off,
+                       src_token=self.src_token, token_rollout=self.token_rollout,
+                       counts=self.counts, counts_host=self.counts_host)
+        self.kpp_host[:self.P].copy_(self.kpp[:self.P], non_blocking=True)
+        self.torch.cuda.current_stream().synchronize()
+        self.K = int(self.counts_host[0])
+        self.T_kept = int(self.counts_host[1])
+        # Algorithm 1, Phase 1(b) then 1(a): the rollout count for the next step.
+        self.step_index += 1
+        s = (self.step_index - 1) % self.ars_total + 1
+        self.n_next = B.adaptive_rollout_count(self.ars, self.kpp_host[:self.P].numpy(), s,
+                                               self.ars_total, s % self.steps_per_epoch == 0)
+        return self.T_kept
+
+    def set_workspaces(self):
+        """Allocate persistent workspaces (sizes from the library's queries)."""
+        import ctypes
+        L = B.lib()
+        need = ctypes.c_size_t(0)
+        p = self.p
+        rc = L.grpo_prune(None, None, None, self.P, p.G, self.T, p.V, p.ngram_n, float(p.tau),
+                          p.keep_cap or p.G, p.dp_divisor, None, None, None, None,
+                          ctypes.byref(need), None)
+        B._check(rc)
+        self.prune_ws = self.torch.empty(need.value + 256, dtype=self.torch.uint8, device=self.dev)
+        self.loss_ws = self.torch.empty(self.T * 8 + 512, dtype=self.torch.uint8, device=self.dev)
+
+    def loss_step(self):
+        p = self.p
+        self._ensure_dlogits(self.T_kept)
+        return B.grpo_loss_fwd_bwd(
+            self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout,
+            V=p.V, row_index=self.src_token, n_rows=self.T_kept, eps_low=p.eps_low,
+            eps_high=p.eps_high, beta=p.beta, agg_mode=p.agg_mode,
+            denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
+            dlogits=self.dlogits, logp_out=self.logp, loss_out=self.loss, status=self.status,
+            ws=self.loss_ws)
+
+    def run(self):
+        self.select()
+        self.loss_step()
+        return self.loss
+
+    def kept_rows(self):
+        """(src_token, token_rollout) of the kept rows as host arrays."""
+        return (self.src_token[:self.T_kept].cpu().numpy(),
+                self.token_rollout[:self.T_kept].cpu().numpy())
+
+
+def as_device(batch: dict, device):
+    """Host arrays of a workloads batch -> device tensors (rewards, ids, off)."""
+    import torch
+    return (torch.from_numpy(batch["rewards"]).to(device),
+            torch.from_numpy(batch["ids"]).to(device),
+            torch.from_numpy(batch["off"]).to(device))

@@ -1,0 +1,129 @@
+"""Host-side parts of the C-ABI library, checked without a GPU: the library loads and exports
+every function include/fastrl_grpo.h declares, argument errors come back as statuses before any
+GPU work, workspace queries answer without a device, and the host adaptive rollout sampling
+equals the oracle's."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from helpers import golden
+from test_oracle_ars import run_trace
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "fastrl_grpo.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b([a-z_][a-z0-9_]*)\s*\(", text)) - {"sizeof"})
+
+
+def test_exports_every_declared_function(grpo):
+    names = declared_functions()
+    assert len(names) >= 10
+    lib = ctypes.CDLL(grpo.library_path())
+    for nm in names:
+        assert hasattr(lib, nm), nm
+    assert sorted(grpo.binding.EXPORTS) == names
+
+
+def test_version_and_counter(grpo):
+    assert "sm_103a" in grpo.version()
+    assert grpo.grpo_kernel_launches() >= 0
+
+
+def test_library_host_ars_matches_oracle(oracle_mod, grpo):
+    """adaptive_rollout_count (host C++ in the library) equals the oracle step for step."""
+    rng = np.random.default_rng(4)
+    g = golden("ars_trace.json")
+    st = grpo.grpo_ars_init(g["G1"])
+    assert run_trace(lambda k, s, M, e: grpo.adaptive_rollout_count(st, k, s, M, e), g) == g["n_after_step"]
+    for trial in range(100):
+        G1 = int(rng.integers(2, 33))
+        M = int(rng.integers(2, 80))
+        spe = int(rng.integers(1, 10))
+        P = int(rng.integers(1, 40))
+        o = oracle_mod.Ars(G1)
+        lib_st = grpo.grpo_ars_init(G1)
+        n = G1
+        for s in range(1, M + 1):
+            kept = np.minimum(rng.integers(0, G1 + 1, size=P), n).astype(np.int32)
+            end = (s % spe == 0)
+            n_o = o.step(kept, s, M, end)
+            n_l = grpo.adaptive_rollout_count(lib_st, kept, s, M, end)
+            assert n_o == n_l, (trial, s)
+            n = n_l
+
+
+def test_library_host_ars_rejects_bad_args(grpo):
+    st = grpo.grpo_ars_init(8)
+    with pytest.raises(grpo.GrpoError):
+        grpo.adaptive_rollout_count(st, [1, 2], 0, 10, False)
+    with pytest.raises(grpo.GrpoError):
+        grpo.adaptive_rollout_count(st, [1, 2], 11, 10, False)
+    with pytest.raises(grpo.GrpoError):
+        grpo.grpo_ars_init(1)
+
+
+def raw():
+    import paper_2609_36932_gb300 as g
+    return g.lib()
+
+
+def test_argument_errors_return_status_without_gpu_work(grpo):
+    L = raw()
+    assert L.grpo_advantage(None, 4, 0, 0, None, None, None) == 1
+    assert L.grpo_advantage(None, 4, 4, 2, None, None, None) == 1
+    assert L.grpo_advantage(None, 0, 4, 0, None, None, None) == 0  # P = 0 is a no-op
+    size = ctypes.c_size_t(0)
+    # G above 32, V above 2^18, n-gram order 4 are outside the supported limits
+    assert L.grpo_prune(None, None, None, 4, 33, 10, 100, 1, 0.8, 4, 1, None, None, None, None,
+                        ctypes.byref(size), None) == 2
+    assert L.grpo_prune(None, None, None, 4, 8, 10, (1 << 18) + 1, 1, 0.8, 4, 1, None, None, None,
+                        None, ctypes.byref(size), None) == 2
+    assert L.grpo_prune(None, None, None, 4, 8, 10, 100, 4, 0.8, 4, 1, None, None, None, None,
+                        ctypes.byref(size), None) == 2
+    assert L.grpo_prune(None, None, None, 4, 8, 10, 100, 1, 0.8, 0, 1, None, None, None, None,
+                        ctypes.byref(size), None) == 1
+    assert L.grpo_compact(None, None, -1, None, None, None, None, None, None, None) == 1
+    assert L.grpo_loss_tune(17, 0, 0) == 1 and L.grpo_loss_tune(0, 96, 0) == 1
+    assert L.grpo_loss_tune(0, 0, 0) == 0
+    assert b"cluster" in L.grpo_last_error() or L.grpo_last_error() == b""
+
+
+def loss_call(L, n_rows, V, ws, size_p, ldt=1, agg=0, denom=1, row_loss=None, beta=0.04):
+    return L.grpo_loss_fwd_bwd(None, ldt, V, None, n_rows, V, None, None, None, None, None, 0.2,
+                               0.2, beta, agg, denom, None, 0, None, 1, None, row_loss, None, None,
+                               ws, size_p, None)
+
+
+def test_workspace_queries_answer_without_a_device(grpo):
+    L = raw()
+    size = ctypes.c_size_t(0)
+    assert L.grpo_prune(None, None, None, 16, 8, 5000, 152064, 2, 0.8, 4, 1, None, None, None,
+                        None, ctypes.byref(size), None) == 0
+    def up(x):
+        return (x + 255) // 256 * 256
+    assert size.value == up(2 * 5000 * 8) + up(16 * 8 * 4) + up(16 * 8 * 8 * 4)
+    assert loss_call(L, 1000, 152064, None, ctypes.byref(size)) == 0
+    assert size.value == up(1000 * 8)
+    # with a row-loss output the loss needs no workspace
+    assert loss_call(L, 1000, 152064, None, ctypes.byref(size), row_loss=ctypes.c_void_p(256)) == 0
+    assert size.value == 0
+    # too small a workspace is refused before any launch
+    small = ctypes.c_size_t(8)
+    assert loss_call(L, 1000, 152064, ctypes.c_void_p(4096), ctypes.byref(small)) == 3
+
+
+def test_loss_argument_errors(grpo):
+    L = raw()
+    size = ctypes.c_size_t(0)
+    assert loss_call(L, 10, 100, None, ctypes.byref(size), ldt=7) == 1
+    assert loss_call(L, -1, 100, None, ctypes.byref(size)) == 1
+    assert loss_call(L, 10, 0, None, ctypes.byref(size)) == 1
+    assert loss_call(L, 10, 100, None, ctypes.byref(size), denom=0) == 1
+    assert loss_call(L, 10, 100, None, ctypes.byref(size), agg=1) == 1  # needs seq_off
+    assert loss_call(L, 10, 100, None, ctypes.byref(size), beta=-1.0) == 1

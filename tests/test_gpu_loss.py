@@ -1,0 +1,258 @@
+"""GPU parity of grpo_loss_fwd_bwd (Eqs. 1-3) with the oracle, through the C ABI: vocabulary
+sizes with ragged tails, both input and output dtypes, launch shapes, gathered and strided
+rows, Eq. 1's sequence mean, and the documented edge cases."""
+import numpy as np
+import pytest
+
+from helpers import bf16_bits_to_f32
+from loss_compare import compare
+
+pytestmark = pytest.mark.gpu
+
+
+def bf16_bits(x):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+class Case:
+    def __init__(self, rng, n, V, in_dtype="bf16", out_dtype="bf16", scale=2.0, n_roll=4,
+                 stride=None, beta=0.04, A=None):
+        import torch
+        self.n, self.V, self.in_dtype, self.out_dtype = n, V, in_dtype, out_dtype
+        self.stride = V if stride is None else stride
+        z = (rng.standard_normal((n, self.stride)) * scale).astype(np.float32)
+        if in_dtype == "bf16":
+            self.host = bf16_bits(z)
+            zf = bf16_bits_to_f32(self.host)
+            self.dev = torch.from_numpy(self.host.view(np.int16)).cuda().view(torch.bfloat16)
+        else:
+            self.host = z
+            zf = z
+            self.dev = torch.from_numpy(z).cuda()
+        self.y = rng.integers(0, V, size=n).astype(np.int32)
+        zz = zf[:, :V].astype(np.float64)
+        m = zz.max(1, keepdims=True)
+        logp = zz[np.arange(n), self.y] - (m[:, 0] + np.log(np.exp(zz - m).sum(1)))
+        self.old = (logp + 0.05 * rng.standard_normal(n)).astype(np.float32)
+        self.ref = (logp + 0.1 * rng.standard_normal(n)).astype(np.float32)
+        self.adv = (rng.standard_normal(n_roll) if A is None else np.asarray(A)).astype(np.float32)
+        self.rr = rng.integers(0, self.adv.size, size=n).astype(np.int32)
+        self.beta = beta
+
+    def t(self, a):
+        import torch
+        return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+    def run_gpu(self, grpo, **kw):
+        import torch
+        n = kw.pop("n_rows", self.n)
+        rr = kw.pop("rr", self.rr)
+        logp = torch.empty(max(n, 1), dtype=torch.float32, device="cuda")
+        rl = torch.empty(max(n, 1), dtype=torch.float64, device="cuda")
+        status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        logits = self.dev.view(self.n, self.stride)[:, :self.V] if self.stride != self.V else self.dev
+        args = dict(V=self.V, row_stride=self.stride, beta=self.beta,
+                    dlogits_dtype=self.out_dtype, logp_out=logp, row_loss_out=rl, status=status)
+        args.update(kw)
+        out = grpo.grpo_loss_fwd_bwd(logits, self.t(self.y), self.t(self.old), self.t(self.ref),
+                                     self.t(self.adv), self.t(rr), n_rows=n, **args)
+        torch.cuda.synchronize()
+        d = out["dlogits"]
+        if self.out_dtype == "bf16":
+            d = d.view(torch.int16).cpu().numpy().view(np.uint16)
+        else:
+            d = d.cpu().numpy()
+        return dict(loss=float(out["loss"].item()), dlogits=d.reshape(n, self.V) if n else d,
+                    logp=logp[:n].cpu().numpy(), row_loss=rl[:n].cpu().numpy(),
+                    status=int(status.item()))
+
+    def run_oracle(self, oracle_mod, **kw):
+        kw.setdefault("beta", self.beta)
+        return oracle_mod.loss(self.host, self.V, self.y, self.old, self.ref, self.adv, self.rr,
+                               row_stride=self.stride, n_rows=kw.pop("n_rows", self.n),
+                               dlogits_dtype=1 if self.out_dtype == "bf16" else 0, **kw)
+
+
+SHAPES = [(1, "f32", "f32"), (7, "bf16", "bf16"), (8, "bf16", "bf16"), (9, "f32", "bf16"),
+          (1000, "bf16", "f32"), (1001, "bf16", "bf16"), (1024, "f32", "f32"),
+          (4097, "bf16", "bf16"), (32000, "bf16", "bf16"), (32001, "f32", "f32"),
+          (152064, "bf16", "bf16"), (152067, "bf16", "f32")]
+
+
+@pytest.mark.parametrize("V,ind,outd", SHAPES)
+def test_vocab_sizes_and_dtypes(grpo, oracle_mod, V, ind, outd):
+    rng = np.random.default_rng(V)
+    n = 37 if V < 100000 else 19
+    c = Case(rng, n, V, ind, outd)
+    g = c.run_gpu(grpo)
+    r = c.run_oracle(oracle_mod)
+    assert g["status"] == 0
+    compare(g["logp"], g["dlogits"], g["loss"], r, outd, gpu_row_loss=g["row_loss"])
+
+
+@pytest.mark.parametrize("cluster,threads,chunks", [(2, 256, 0), (3, 128, 3), (4, 512, 5),
+                                                    (5, 256, 7), (8, 256, 1), (8, 128, 16),
+                                                    (16, 128, 4), (16, 512, 2)])
+def test_launch_shapes(grpo, oracle_mod, cluster, threads, chunks):
+    rng = np.random.default_rng(cluster * 100 + threads + chunks)
+    c = Case(rng, 23, 152064, "bf16", "bf16")
+    r = c.run_oracle(oracle_mod)
+    try:
+        grpo.grpo_loss_tune(cluster, threads, chunks)
+        g = c.run_gpu(grpo)
+        g2 = c.run_gpu(grpo)
+    finally:
+        grpo.grpo_loss_tune(0, 0, 0)
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    assert g["loss"] == g2["loss"] and np.array_equal(g["dlogits"], g2["dlogits"])
+
+
+def test_single_cta_row_too_large_is_rejected(grpo):
+    rng = np.random.default_rng(1)
+    c = Case(rng, 2, 152064, "bf16", "bf16")
+    try:
+        grpo.grpo_loss_tune(1, 0, 0)
+        with pytest.raises(grpo.GrpoError) as ei:
+            c.run_gpu(grpo)
+        assert ei.value.status == 2
+    finally:
+        grpo.grpo_loss_tune(0, 0, 0)
+
+
+@pytest.mark.parametrize("V,ind", [(32000, "bf16"), (1001, "bf16"), (4096, "f32")])
+def test_gathered_strided_rows(grpo, oracle_mod, V, ind):
+    """row_index gathers rows from a larger buffer with a padded row stride."""
+    import torch
+    rng = np.random.default_rng(2)
+    c = Case(rng, 64, V, ind, "bf16", stride=V + 24)
+    idx = rng.choice(64, size=29, replace=False).astype(np.int64)
+    rr = rng.integers(0, c.adv.size, size=29).astype(np.int32)
+    g = c.run_gpu(grpo, n_rows=29, row_index=c.t(idx), rr=rr)
+    r = oracle_mod.loss(c.host, V, c.y, c.old, c.ref, c.adv, rr, row_stride=c.stride,
+                        row_index=idx, dlogits_dtype=1, beta=c.beta)
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+
+
+def test_unaligned_rows_take_the_element_path(grpo, oracle_mod):
+    """A base pointer one element past a 16-byte boundary disables the bulk copies."""
+    import torch
+    rng = np.random.default_rng(3)
+    V = 5000
+    c = Case(rng, 11, V, "bf16", "f32", stride=V + 8)
+    full = c.dev.view(11, V + 8)
+    logits = full[:, 1:V + 1]
+    host = bf16_bits_to_f32(c.host).reshape(11, V + 8)[:, 1:V + 1]
+    zz = host.astype(np.float64)
+    m = zz.max(1, keepdims=True)
+    logp = zz[np.arange(11), c.y] - (m[:, 0] + np.log(np.exp(zz - m).sum(1)))
+    old = (logp + 0.05 * rng.standard_normal(11)).astype(np.float32)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    lp = torch.empty(11, dtype=torch.float32, device="cuda")
+    out = grpo.grpo_loss_fwd_bwd(logits, c.t(c.y), c.t(old), c.t(c.ref), c.t(c.adv), c.t(c.rr),
+                                 dlogits_dtype="f32", logp_out=lp, status=status, beta=c.beta)
+    torch.cuda.synchronize()
+    r = oracle_mod.loss(np.ascontiguousarray(host), V, c.y, old, c.ref, c.adv, c.rr, beta=c.beta)
+    compare(lp.cpu().numpy(), out["dlogits"].cpu().numpy(), float(out["loss"].item()), r, "f32")
+
+
+def test_sequence_mean(grpo, oracle_mod):
+    import torch
+    rng = np.random.default_rng(4)
+    c = Case(rng, 40, 32000, "bf16", "bf16", n_roll=5)
+    rr = np.sort(rng.integers(0, 5, size=40)).astype(np.int32)
+    lens = np.bincount(rr, minlength=5)
+    seq_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    n_seq = int((lens > 0).sum())
+    g = c.run_gpu(grpo, rr=rr, agg_mode=1, seq_off=c.t(seq_off), n_seq=n_seq)
+    r = oracle_mod.loss(c.host, c.V, c.y, c.old, c.ref, c.adv, rr, agg_mode=1, seq_off=seq_off,
+                        n_seq=n_seq, dlogits_dtype=1, beta=c.beta)
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+
+
+def test_deterministic(grpo):
+    rng = np.random.default_rng(5)
+    c = Case(rng, 50, 152064, "bf16", "bf16")
+    a, b = c.run_gpu(grpo), c.run_gpu(grpo)
+    assert a["loss"] == b["loss"]
+    assert np.array_equal(a["dlogits"], b["dlogits"]) and np.array_equal(a["logp"], b["logp"])
+
+
+def test_no_rows(grpo):
+    rng = np.random.default_rng(6)
+    c = Case(rng, 3, 1000, "bf16", "bf16")
+    g = c.run_gpu(grpo, n_rows=0)
+    assert g["loss"] == 0.0 and g["status"] == 0
+
+
+def test_zero_advantage_without_kl_is_exactly_zero(grpo):
+    rng = np.random.default_rng(7)
+    c = Case(rng, 9, 32000, "bf16", "bf16", beta=0.0, A=[0.0, 0.0])
+    g = c.run_gpu(grpo)
+    assert np.all((g["dlogits"] & 0x7FFF) == 0) and g["loss"] == 0.0
+
+
+def test_bad_token_sets_status_and_zero_row(grpo, oracle_mod):
+    rng = np.random.default_rng(8)
+    c = Case(rng, 6, 1000, "bf16", "bf16")
+    c.y[2] = 1000
+    c.y[4] = -5
+    g = c.run_gpu(grpo)
+    assert g["status"] & grpo.binding.DEVFLAG_BAD_TOKEN
+    r = c.run_oracle(oracle_mod)
+    assert np.isnan(g["logp"][2]) and np.isnan(g["logp"][4])
+    assert np.all((g["dlogits"][[2, 4]] & 0x7FFF) == 0)
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16")
+
+
+def test_nonfinite_logits_set_status(grpo):
+    import torch
+    rng = np.random.default_rng(9)
+    c = Case(rng, 4, 2000, "f32", "f32")
+    host = c.host.copy()
+    host[1, 17] = np.nan
+    c.host = host
+    c.dev = torch.from_numpy(host).cuda()
+    g = c.run_gpu(grpo)
+    assert g["status"] & grpo.binding.DEVFLAG_NONFINITE
+    assert np.isnan(g["logp"][1]) and np.all(np.isfinite(g["logp"][[0, 2, 3]]))
+
+
+def test_masked_vocabulary(grpo, oracle_mod):
+    """-inf logits (a masked vocabulary range, whole slices included) contribute nothing."""
+    import torch
+    rng = np.random.default_rng(10)
+    c = Case(rng, 8, 152064, "bf16", "bf16")
+    host = c.host.copy()
+    host[:, 40000:120000] = 0xFF80  # bf16 -inf
+    c.y = rng.integers(0, 40000, size=8).astype(np.int32)
+    c.host = host
+    c.dev = torch.from_numpy(host.view(np.int16)).cuda().view(torch.bfloat16)
+    zz = bf16_bits_to_f32(host).astype(np.float64)
+    m = zz.max(1, keepdims=True)
+    logp = zz[np.arange(8), c.y] - (m[:, 0] + np.log(np.exp(zz - m).sum(1)))
+    c.old = (logp + 0.05 * rng.standard_normal(8)).astype(np.float32)
+    g = c.run_gpu(grpo)
+    r = c.run_oracle(oracle_mod)
+    assert g["status"] == 0
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+
+
+def test_peaked_rows_keep_one_minus_p_accurate(grpo, oracle_mod):
+    """When p_y is close to 1 the y entry is coef*(1 - p_y); it is formed from the sum that
+    leaves y out, so it keeps full relative accuracy."""
+    rng = np.random.default_rng(11)
+    c = Case(rng, 12, 32000, "bf16", "bf16", scale=1.0)
+    host = bf16_bits_to_f32(c.host).reshape(12, 32000).copy()
+    host[np.arange(12), c.y] = 24.0
+    c.host = bf16_bits(host)
+    import torch
+    c.dev = torch.from_numpy(c.host.view(np.int16)).cuda().view(torch.bfloat16)
+    zz = host.astype(np.float64)
+    m = zz.max(1, keepdims=True)
+    logp = zz[np.arange(12), c.y] - (m[:, 0] + np.log(np.exp(zz - m).sum(1)))
+    c.old = (logp + 0.05 * rng.standard_normal(12)).astype(np.float32)
+    c.ref = (logp + 0.1 * rng.standard_normal(12)).astype(np.float32)
+    g = c.run_gpu(grpo)
+    r = c.run_oracle(oracle_mod)
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16")
