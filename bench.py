@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="qwen", help="tiny|small|qwen|large|long or 0-4")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--prompts", type=int, default=0,
+                    help="override the workload's prompt count (a smaller case for profiling)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
@@ -282,8 +284,11 @@ def run_reference(args, w):
 
 def main():
     args = parse()
+    import dataclasses
     from paper_2609_36932_gb300 import workloads
     w = workloads.get(args.config)
+    if args.prompts > 0:
+        w = dataclasses.replace(w, P=args.prompts)
     if args.impl == "reference":
         run_reference(args, w)
         return
