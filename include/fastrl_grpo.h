@@ -179,6 +179,36 @@ grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t 
                               grpo_stream_t stream);
 
 /*
+ * grpo_loss_fwd_bwd_noalloc — grpo_loss_fwd_bwd for callers that cannot allocate device memory.
+ * The paper has no counterpart: this is an interface convenience of this library.
+ * Some callers run the loss where no allocation is possible: a plugin or custom-op host that
+ * passes only input and output buffers and has no workspace hook, or a runtime that forbids
+ * allocation after start-up to keep its memory footprint fixed.  This entry takes the same
+ * arguments as grpo_loss_fwd_bwd without ws/ws_bytes and computes the same results.  Its
+ * per-row loss scratch is a fixed array inside the library (2 MiB of fp64, 262144 rows), which
+ * every GPU that loads the library holds until the process exits.
+ *   - n_rows above 262144 with row_loss_out == NULL returns GRPO_ERR_UNSUPPORTED (pass
+ *     row_loss_out, which needs no scratch, or split the rows into several calls).
+ *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
+ *     with that device current; make that first call before any stream capture.
+ *   - Every call uses the same array, which keeps the previous call's contents; each call
+ *     writes every entry it later reads, so nothing needs clearing.  Calls whose GPU work
+ *     overlaps (for instance on two streams at once) race on the array: order them on one
+ *     stream.
+ *   - It calls no cudaMalloc, cudaFree or other allocating routine.
+ */
+grpo_status grpo_loss_fwd_bwd_noalloc(const void* logits, int32_t logits_dtype,
+                                      int64_t row_stride, const int64_t* row_index,
+                                      int64_t n_rows, int32_t V, const int32_t* y,
+                                      const float* old_logp, const float* ref_logp,
+                                      const float* adv, const int32_t* row_rollout, float eps_low,
+                                      float eps_high, float beta, int32_t agg_mode,
+                                      int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq,
+                                      void* dlogits, int32_t dlogits_dtype, float* logp_out,
+                                      double* row_loss_out, double* loss_out, int32_t* status,
+                                      grpo_stream_t stream);
+
+/*
  * grpo_loss_tune — launch shape of grpo_loss_fwd_bwd's main kernel for this process.
  * cluster_ctas: CTAs sharing one logits row (1..16, 0 = automatic); threads: 128/256/512
  * (0 = automatic); chunks: copies each CTA splits its slice into (1..16, 0 = automatic).

@@ -31,8 +31,8 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_tune", "grpo_ars_init",
-           "adaptive_rollout_count"]
+           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_noalloc",
+           "grpo_loss_tune", "grpo_ars_init", "adaptive_rollout_count"]
 
 
 class GrpoError(RuntimeError):
@@ -82,6 +82,10 @@ def lib():
                                     _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p, _c_p,
                                     _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
     L.grpo_loss_fwd_bwd.restype = _i32
+    L.grpo_loss_fwd_bwd_noalloc.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p,
+                                            _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64,
+                                            _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p]
+    L.grpo_loss_fwd_bwd_noalloc.restype = _i32
     L.grpo_loss_tune.argtypes = [_i32, _i32, _i32]
     L.grpo_loss_tune.restype = _i32
     L.grpo_ars_init.argtypes = [ctypes.POINTER(ArsState), _i32]
@@ -298,6 +302,50 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
     wp, size = _ws_args(wst)
     _check(L.grpo_loss_fwd_bwd(*args_head, wp, size, _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
+
+
+def grpo_loss_fwd_bwd_noalloc(logits, y, old_logp, ref_logp, adv, row_rollout, *, dlogits,
+                              logp_out=None, row_loss_out=None, loss_out, status=None,
+                              row_index=None, n_rows: int | None = None, V: int | None = None,
+                              row_stride: int | None = None, eps_low: float = 0.2,
+                              eps_high: float = 0.2, beta: float = 0.04, agg_mode: int = 0,
+                              denom_tokens: int | None = None, seq_off=None, n_seq: int = 0,
+                              stream=None):
+    """The allocation-free loss entry: for callers that cannot allocate device memory when the
+    loss runs (a host that passes only inputs and outputs and has no workspace hook, or a
+    runtime that forbids allocation after start-up).  Every output buffer must be passed in;
+    the library's fixed scratch holds the per-row loss terms (at most 262144 rows per call
+    unless row_loss_out is given).  Nothing here allocates."""
+    torch = _torch()
+    if logits.dtype == torch.bfloat16:
+        ldt = GRPO_DTYPE_BF16
+    elif logits.dtype == torch.float32:
+        ldt = GRPO_DTYPE_F32
+    else:
+        raise TypeError("logits must be bf16 or f32")
+    if logits.dim() != 2 or logits.stride(1) != 1 or not logits.is_cuda:
+        raise ValueError("logits must be a 2-D CUDA tensor with unit stride along the vocabulary")
+    if V is None:
+        V = logits.shape[1]
+    stride = logits.stride(0) if row_stride is None else int(row_stride)
+    if n_rows is None:
+        n_rows = row_index.numel() if row_index is not None else logits.shape[0]
+    if dlogits.dtype == torch.bfloat16:
+        odt = GRPO_DTYPE_BF16
+    elif dlogits.dtype == torch.float32:
+        odt = GRPO_DTYPE_F32
+    else:
+        raise TypeError("dlogits must be bf16 or f32")
+    _need(dlogits, dlogits.dtype, n_rows * V, "dlogits")
+    _need(loss_out, torch.float64, 1, "loss_out")
+    if denom_tokens is None:
+        denom_tokens = max(int(n_rows), 1)
+    _check(lib().grpo_loss_fwd_bwd_noalloc(
+        _ptr(logits), ldt, stride, _ptr(row_index), int(n_rows), int(V), _ptr(y), _ptr(old_logp),
+        _ptr(ref_logp), _ptr(adv), _ptr(row_rollout), float(eps_low), float(eps_high),
+        float(beta), int(agg_mode), int(denom_tokens), _ptr(seq_off), int(n_seq), _ptr(dlogits),
+        odt, _ptr(logp_out), _ptr(row_loss_out), _ptr(loss_out), _ptr(status), _stream(stream)))
+    return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out)
 
 
 def grpo_ars_init(G1: int) -> ArsState:

@@ -672,3 +672,75 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   count_launches(2);
   return check_launch(who);
 }
+
+// ---- allocation-free variant ------------------------------------------------------------------
+//
+// Some callers cannot allocate device memory at the point where they run the loss: for
+// example a plugin or custom-op host that hands over only input and output buffers and offers
+// no workspace hook, or a runtime that forbids allocation after its start-up phase (to keep
+// memory use fixed and latency predictable).  For them, grpo_loss_fwd_bwd_noalloc keeps the
+// per-row loss scratch in a fixed array of this library instead of a caller workspace.
+//
+// The array below lives in every GPU that loads the library, until the process exits.  Host
+// code cannot use its name as an address (on the host it names a stand-in object), so the
+// device address is looked up with cudaGetSymbolAddress, once per device, with that device
+// current, on the first call made on it.
+
+namespace fastrl {
+namespace {
+
+constexpr int64_t kNoAllocMaxRows = 262144;  // 2 MiB of fp64 row-loss scratch
+static __device__ __align__(256) double g_noalloc_row_loss[kNoAllocMaxRows];
+
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {nullptr};
+
+}  // namespace
+}  // namespace fastrl
+
+extern "C" grpo_status grpo_loss_fwd_bwd_noalloc(
+    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
+    int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,
+    const float* adv, const int32_t* row_rollout, float eps_low, float eps_high, float beta,
+    int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq, void* dlogits,
+    int32_t dlogits_dtype, float* logp_out, double* row_loss_out, double* loss_out, int32_t* status,
+    grpo_stream_t stream) {
+  clear_error();
+  const char* who = "grpo_loss_fwd_bwd_noalloc";
+  if (row_loss_out != nullptr)  // the caller's row-loss buffer is the only scratch: none needed
+    return grpo_loss_fwd_bwd(logits, logits_dtype, row_stride, row_index, n_rows, V, y, old_logp,
+                             ref_logp, adv, row_rollout, eps_low, eps_high, beta, agg_mode,
+                             denom_tokens, seq_off, n_seq, dlogits, dlogits_dtype, logp_out,
+                             row_loss_out, loss_out, status, nullptr, nullptr, stream);
+  if (n_rows > kNoAllocMaxRows)
+    return fail(GRPO_ERR_UNSUPPORTED,
+                "%s: n_rows = %lld exceeds the fixed scratch of %lld rows; pass row_loss_out, "
+                "split the rows into calls of at most %lld, or use grpo_loss_fwd_bwd",
+                who, (long long)n_rows, (long long)kNoAllocMaxRows, (long long)kNoAllocMaxRows);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaGetDevice: %s", who, cudaGetErrorString(e));
+  if (dev < 0 || dev >= kNoAllocMaxDevices)
+    return fail(GRPO_ERR_UNSUPPORTED, "%s: device %d beyond %d", who, dev, kNoAllocMaxDevices);
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (g_noalloc_ptr[dev] == nullptr) {
+      e = cudaGetSymbolAddress(&g_noalloc_ptr[dev], g_noalloc_row_loss);
+      if (e != cudaSuccess) {
+        g_noalloc_ptr[dev] = nullptr;
+        return fail(GRPO_ERR_CUDA, "%s: cudaGetSymbolAddress of the scratch array: %s", who,
+                    cudaGetErrorString(e));
+      }
+    }
+    scratch = g_noalloc_ptr[dev];
+  }
+  // Every row loss the sum reads is written by the same call, so the scratch needs no clearing.
+  size_t bytes = sizeof(g_noalloc_row_loss);
+  return grpo_loss_fwd_bwd(logits, logits_dtype, row_stride, row_index, n_rows, V, y, old_logp,
+                           ref_logp, adv, row_rollout, eps_low, eps_high, beta, agg_mode,
+                           denom_tokens, seq_off, n_seq, dlogits, dlogits_dtype, logp_out,
+                           nullptr, loss_out, status, n_rows > 0 ? scratch : nullptr,
+                           n_rows > 0 ? &bytes : nullptr, stream);
+}
