@@ -270,7 +270,10 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
         n_rows = row_index.numel() if row_index is not None else logits.shape[0]
     dev = logits.device
     if dlogits_dtype is None:
-        dlogits_dtype = ldt
+        if dlogits is not None:
+            dlogits_dtype = GRPO_DTYPE_BF16 if dlogits.dtype == torch.bfloat16 else GRPO_DTYPE_F32
+        else:
+            dlogits_dtype = ldt
     elif dlogits_dtype in (torch.bfloat16, "bf16"):
         dlogits_dtype = GRPO_DTYPE_BF16
     elif dlogits_dtype in (torch.float32, "f32"):

@@ -11,10 +11,11 @@
 //     the rest is in flight.
 //   * Pass A: per-thread online max and sum of exp (base 2, MUFU ex2) over the slice, leaving
 //     out the sampled token y; warp shuffles and shared memory combine the CTA's threads.
-//   * Exchange: each CTA publishes (max, sum, z_y) in shared memory; after a cluster barrier
-//     warp 0 reads every CTA's entry through distributed shared memory (mapa +
-//     ld.shared::cluster) and forms the row's log-sum-exp, log-prob, ratio, clipped surrogate,
-//     KL term and gradient coefficient.  Every CTA of the cluster computes the same numbers.
+//   * Exchange: each CTA pushes its (max, sum, z_y) into every cluster peer's shared memory with
+//     st.async, which completes bytes on the peer's mbarrier (no cluster-wide barrier, so no
+//     CTA waits for another's outstanding stores); warp 0 waits on its own mbarrier, reads the
+//     C entries locally and forms the row's log-sum-exp, log-prob, ratio, clipped surrogate, KL
+//     term and gradient coefficient.  Every CTA of the cluster computes the same numbers.
 //   * Pass B: dlogits[v] = -coef * exp(z_v - lse) (+coef at v = y) from the shared-memory slice,
 //     written with 16-byte streaming stores.  As soon as chunk k has been consumed, thread 0
 //     starts the copy of chunk k of the cluster's next row into the same buffer.
@@ -95,16 +96,6 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
                    : "memory");
 }
-__device__ __forceinline__ float4 ld_cluster_f4(uint32_t local_addr, uint32_t rank) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local_addr), "r"(rank));
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(remote)
-               : "memory");
-  return v;
-}
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
@@ -115,16 +106,32 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
+// Test the phase; while it is incomplete the thread may be suspended for up to ~0.1 ms
+// (the hint, in ns) instead of spinning and taking issue slots.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(100000u)
       : "memory");
   return ok != 0;
+}
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t local_addr, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local_addr), "r"(rank));
+  return remote;
+}
+// 16-byte store into a cluster peer's shared memory that completes 16 bytes of that peer's
+// mbarrier transaction count (both addresses already mapped to the peer).
+__device__ __forceinline__ void st_async_f4(uint32_t remote_addr, float4 v, uint32_t remote_bar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+          remote_addr),
+      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(remote_bar)
+      : "memory");
 }
 __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
                                               uint32_t bar) {
@@ -134,70 +141,106 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
       "l"(src), "r"(bytes), "r"(bar)
       : "memory");
 }
-__device__ __forceinline__ float ex2(float x) {  // 2^x on the MUFU, subnormal results kept
+// 2^x on the MUFU (one instruction); results below 2^-126 flush to zero.  Pass A only loses
+// terms 2^126 times smaller than the running maximum; pass B shifts its argument (see
+// kShiftB) so that no representable gradient entry is lost.
+__device__ __forceinline__ float ex2(float x) {
   float y;
-  asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+__device__ __forceinline__ float2 ex2x2(float2 t) { return make_float2(ex2(t.x), ex2(t.y)); }
+// Lane-wise maximum of two bf16 pairs; a NaN operand yields the other operand.
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
 
-// ---- element formats --------------------------------------------------------------------------
+// Pass B evaluates 2^(t + kShiftB) * (scale * 2^-kShiftB) when |scale| >= 2^-100, which moves the
+// flush-to-zero point of ex2 below every gradient entry that bf16 or f32 can represent.
+constexpr float kShiftB = 16.f;
+
+// ---- element formats: 16-byte vectors of the logits, unpacked into f32 pairs -----------------
 
 template <typename T>
 struct Fmt;
 template <>
 struct Fmt<float> {
   static constexpr int kVec = 4;  // elements per 16 bytes
-  __device__ static void unpack(const uint4& q, float (&f)[4]) {
-    f[0] = __uint_as_float(q.x);
-    f[1] = __uint_as_float(q.y);
-    f[2] = __uint_as_float(q.z);
-    f[3] = __uint_as_float(q.w);
+  static constexpr int kPairs = 2;
+  __device__ static void pairs(const uint4& q, float2 (&p)[2]) {
+    p[0] = make_float2(__uint_as_float(q.x), __uint_as_float(q.y));
+    p[1] = make_float2(__uint_as_float(q.z), __uint_as_float(q.w));
   }
+  struct Max {  // running maximum over vectors
+    float m = -INFINITY;
+    __device__ void add(const uint4& q) {
+      m = fmaxf(m, fmaxf(fmaxf(__uint_as_float(q.x), __uint_as_float(q.y)),
+                         fmaxf(__uint_as_float(q.z), __uint_as_float(q.w))));
+    }
+    __device__ float get() const { return m; }
+  };
   __device__ static float load(const float* p) { return *p; }
   __device__ static void store(float* p, float v) { *p = v; }
 };
 template <>
 struct Fmt<__nv_bfloat16> {
   static constexpr int kVec = 8;
-  __device__ static void unpack(const uint4& q, float (&f)[8]) {
-    f[0] = __uint_as_float(q.x << 16);
-    f[1] = __uint_as_float(q.x & 0xffff0000u);
-    f[2] = __uint_as_float(q.y << 16);
-    f[3] = __uint_as_float(q.y & 0xffff0000u);
-    f[4] = __uint_as_float(q.z << 16);
-    f[5] = __uint_as_float(q.z & 0xffff0000u);
-    f[6] = __uint_as_float(q.w << 16);
-    f[7] = __uint_as_float(q.w & 0xffff0000u);
+  static constexpr int kPairs = 4;
+  __device__ static float2 pair(uint32_t w) {
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
   }
+  __device__ static void pairs(const uint4& q, float2 (&p)[4]) {
+    p[0] = pair(q.x);
+    p[1] = pair(q.y);
+    p[2] = pair(q.z);
+    p[3] = pair(q.w);
+  }
+  struct Max {  // running maximum kept as a bf16 pair: one instruction per two elements
+    uint32_t m = 0xFF80FF80u;  // (-inf, -inf)
+    __device__ void add(const uint4& q) { m = bmax2(m, bmax2(bmax2(q.x, q.y), bmax2(q.z, q.w))); }
+    __device__ float get() const {
+      return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
+    }
+  };
   __device__ static float load(const __nv_bfloat16* p) { return __bfloat162float(*p); }
   __device__ static void store(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
 };
 
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+__device__ __forceinline__ uint32_t pack_bf16x2(float2 v) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(v.x, v.y);
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// Store kVec results at p (aligned to kVec * sizeof(OutT) bytes), streaming (evict-first).
-template <typename OutT, int kVec>
-__device__ __forceinline__ void store_vec(OutT* p, const float (&d)[kVec]);
+// Store one vector of results at p (aligned to its width), streaming (evict-first).
+template <typename OutT, int kPairs>
+__device__ __forceinline__ void store_pairs(OutT* p, const float2 (&d)[kPairs]);
 template <>
-__device__ __forceinline__ void store_vec<__nv_bfloat16, 8>(__nv_bfloat16* p, const float (&d)[8]) {
-  __stcs(reinterpret_cast<uint4*>(p), make_uint4(pack_bf16x2(d[0], d[1]), pack_bf16x2(d[2], d[3]),
-                                                 pack_bf16x2(d[4], d[5]), pack_bf16x2(d[6], d[7])));
+__device__ __forceinline__ void store_pairs<__nv_bfloat16, 4>(__nv_bfloat16* p, const float2 (&d)[4]) {
+  __stcs(reinterpret_cast<uint4*>(p),
+         make_uint4(pack_bf16x2(d[0]), pack_bf16x2(d[1]), pack_bf16x2(d[2]), pack_bf16x2(d[3])));
 }
 template <>
-__device__ __forceinline__ void store_vec<float, 8>(float* p, const float (&d)[8]) {
-  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0], d[1], d[2], d[3]));
-  __stcs(reinterpret_cast<float4*>(p) + 1, make_float4(d[4], d[5], d[6], d[7]));
+__device__ __forceinline__ void store_pairs<float, 4>(float* p, const float2 (&d)[4]) {
+  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0].x, d[0].y, d[1].x, d[1].y));
+  __stcs(reinterpret_cast<float4*>(p) + 1, make_float4(d[2].x, d[2].y, d[3].x, d[3].y));
 }
 template <>
-__device__ __forceinline__ void store_vec<float, 4>(float* p, const float (&d)[4]) {
-  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0], d[1], d[2], d[3]));
+__device__ __forceinline__ void store_pairs<float, 2>(float* p, const float2 (&d)[2]) {
+  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0].x, d[0].y, d[1].x, d[1].y));
 }
 template <>
-__device__ __forceinline__ void store_vec<__nv_bfloat16, 4>(__nv_bfloat16* p, const float (&d)[4]) {
-  __stcs(reinterpret_cast<uint2*>(p), make_uint2(pack_bf16x2(d[0], d[1]), pack_bf16x2(d[2], d[3])));
+__device__ __forceinline__ void store_pairs<__nv_bfloat16, 2>(__nv_bfloat16* p, const float2 (&d)[2]) {
+  __stcs(reinterpret_cast<uint2*>(p), make_uint2(pack_bf16x2(d[0]), pack_bf16x2(d[1])));
+}
+template <typename OutT, int kPairs>
+__device__ __forceinline__ void store_pairs_scalar(OutT* p, const float2 (&d)[kPairs]) {
+#pragma unroll
+  for (int i = 0; i < kPairs; ++i) {
+    Fmt<OutT>::store(p + 2 * i, d[i].x);
+    Fmt<OutT>::store(p + 2 * i + 1, d[i].y);
+  }
 }
 
 // Combine two (max, sum of exp relative to max) pairs.
@@ -214,15 +257,17 @@ __device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float 
 template <typename InT, typename OutT, int kThreads>
 __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
+  constexpr int kPairs = Fmt<InT>::kPairs;
   constexpr int kWarps = kThreads / 32;
   extern __shared__ __align__(128) unsigned char smem[];
   const int buf_bytes = (int)align_up((size_t)a.slice * sizeof(InT), 128);
   InT* buf = reinterpret_cast<InT*>(smem);
   const uint4* buf4 = reinterpret_cast<const uint4*>(smem);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + buf_bytes);
-  float4* stats = reinterpret_cast<float4*>(smem + buf_bytes + kMaxChunks * 8);  // 2 slots
-  float* red = reinterpret_cast<float*>(stats + 2);                               // 2*kWarps
-  float* rowsc = red + 2 * kWarps;                                                // 4 floats
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + buf_bytes);  // kMaxChunks copy barriers
+  uint64_t* xbars = bars + kMaxChunks;                               // 2 exchange barriers
+  float4* exch = reinterpret_cast<float4*>(xbars + 2);               // [2][kMaxCluster] entries
+  float* red = reinterpret_cast<float*>(exch + 2 * kMaxCluster);     // 2*kWarps
+  float* rowsc = red + 2 * kWarps;                                   // 4 floats
   int* abort_flag = reinterpret_cast<int*>(rowsc + 4);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -235,13 +280,19 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
   const int tail0 = nvec * kVec;                   // first element loaded one by one
   const uint32_t buf_s = smem_addr(buf);
   const uint32_t bar_s = smem_addr(bars);
+  const uint32_t xbar_s = smem_addr(xbars);
+  const uint32_t exch_s = smem_addr(exch);
+  const float2 l2e2 = make_float2(kLog2e, kLog2e);
 
   if (tid == 0) {
     for (int k = 0; k < a.n_chunks; ++k) mbar_init(bar_s + 8 * k, 1);
+    mbar_init(xbar_s, 1);
+    mbar_init(xbar_s + 8, 1);
     *abort_flag = 0;
     mbar_fence_init();
   }
   __syncthreads();
+  cluster_sync();  // peers' exchange barriers exist before anyone sends to them
 
   auto row_base = [&](int64_t row) -> const char* {
     const int64_t src = a.row_index ? a.row_index[row] : row;
@@ -254,11 +305,12 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
     mbar_expect_tx(bar_s + 8 * k, bytes);
     if (bytes) bulk_copy_g2s(buf_s + v0 * 16, g + (int64_t)v0 * 16, bytes, bar_s + 8 * k);
   };
-  auto wait_chunk = [&](int k, uint32_t parity) {
+  auto wait_bar = [&](uint32_t bar, uint32_t parity) {  // bounded: about kWaitLimitNs
     if (*(volatile int*)abort_flag) return;
-    if (mbar_try_wait(bar_s + 8 * k, parity)) return;
+    if (mbar_try_wait(bar, parity)) return;
     const uint64_t t0 = global_timer_ns();
-    while (!mbar_try_wait(bar_s + 8 * k, parity)) {
+    for (uint32_t it = 1; !mbar_try_wait(bar, parity); ++it) {
+      if ((it & 63u) != 0) continue;
       if (*(volatile int*)abort_flag) return;
       if (global_timer_ns() - t0 > kWaitLimitNs) {
         *(volatile int*)abort_flag = 1;
@@ -267,15 +319,19 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
       }
     }
   };
+  auto wait_chunk = [&](int k, uint32_t parity) { wait_bar(bar_s + 8 * k, parity); };
 
   int64_t row = cluster_id_x();
-  uint32_t phase = 0;
+  uint32_t phase = 0;  // parity of the copy barriers (one completion per row)
+  uint32_t iter = 0;   // rows done; exchange slot = iter & 1, its parity = (iter >> 1) & 1
   if (tid == 0 && row < a.n_rows) {
     const char* g = row_base(row);
     for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
   }
 
-  for (; row < a.n_rows; row += ncl, phase ^= 1u) {
+  for (; row < a.n_rows; row += ncl, phase ^= 1u, ++iter) {
+    const uint32_t slot = iter & 1u;
+    if (tid == 0) mbar_expect_tx(xbar_s + 8 * slot, 16u * C);  // one entry from every CTA
     const int64_t src = a.row_index ? a.row_index[row] : row;
     const int32_t yv = a.y[src];
     const bool yvalid = yv >= 0 && yv < a.V;
@@ -289,13 +345,9 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
       const int v0 = k * a.chunk_vecs;
       const int v1 = min(nvec, v0 + a.chunk_vecs);
       const bool last = (k == a.n_chunks - 1);
-      float cm = -INFINITY;
-      for (int j = v0 + tid; j < v1; j += kThreads) {
-        float f[kVec];
-        Fmt<InT>::unpack(buf4[j], f);
-#pragma unroll
-        for (int i = 0; i < kVec; ++i) cm = fmaxf(cm, f[i]);
-      }
+      typename Fmt<InT>::Max mx;
+      for (int j = v0 + tid; j < v1; j += kThreads) mx.add(buf4[j]);
+      float cm = mx.get();
       if (last) {
         for (int e = tail0 + tid; e < len; e += kThreads) {
           const InT v = *reinterpret_cast<const InT*>(grow + (int64_t)e * sizeof(InT));
@@ -309,21 +361,28 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
       }
       if (m != -INFINITY) {
         const float sh = -m * kLog2e;
+        const float2 sh2 = make_float2(sh, sh);
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
         for (int j = v0 + tid; j < v1; j += kThreads) {
-          float f[kVec];
-          Fmt<InT>::unpack(buf4[j], f);
+          float2 p[kPairs];
+          Fmt<InT>::pairs(buf4[j], p);
           const int yi = yl - j * kVec;
-          float acc = 0.f;
-          if ((unsigned)yi < (unsigned)kVec) {
+          if ((unsigned)yi < (unsigned)kVec) {  // the vector holding y: leave y out
 #pragma unroll
-            for (int i = 0; i < kVec; ++i)
-              if (i != yi) acc += ex2(fmaf(f[i], kLog2e, sh));
+            for (int i = 0; i < kPairs; ++i) {
+              const float2 e = ex2x2(__ffma2_rn(p[i], l2e2, sh2));
+              if (2 * i != yi) acc0.x += e.x;
+              if (2 * i + 1 != yi) acc0.y += e.y;
+            }
           } else {
 #pragma unroll
-            for (int i = 0; i < kVec; ++i) acc += ex2(fmaf(f[i], kLog2e, sh));
+            for (int i = 0; i < kPairs; i += 2) {
+              acc0 = __fadd2_rn(acc0, ex2x2(__ffma2_rn(p[i], l2e2, sh2)));
+              acc1 = __fadd2_rn(acc1, ex2x2(__ffma2_rn(p[i + 1], l2e2, sh2)));
+            }
           }
-          s += acc;
         }
+        s += (acc0.x + acc0.y) + (acc1.x + acc1.y);
         if (last)
           for (int e = tail0 + tid; e < len; e += kThreads)
             if (e != yl) s += ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, sh));
@@ -350,19 +409,22 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
         const float so = __shfl_xor_sync(0xffffffffu, s, o);
         lse_combine(m, s, mo, so);
       }
-      if (lane == 0) {
+      // push (max, sum, z_y) into entry [slot][rank] of every CTA of the cluster (self too)
+      if (lane < (int)C) {
         const float zy = ((unsigned)yl < (unsigned)len) ? Fmt<InT>::load(&buf[yl]) : 0.f;
-        stats[phase] = make_float4(m, s, zy, 0.f);
+        const uint32_t dst = exch_s + (uint32_t)(slot * kMaxCluster + rank) * 16u;
+        st_async_f4(mapa_shared(dst, lane), make_float4(m, s, zy, 0.f),
+                    mapa_shared(xbar_s + 8 * slot, lane));
       }
     }
-    cluster_sync();  // every CTA's (max, sum, z_y) for this row is published
 
     // ---- exchange and row scalars (warp 0) ----
     if (warp == 0) {
-      const uint32_t st_addr = smem_addr(&stats[phase]);
+      wait_bar(xbar_s + 8 * slot, (iter >> 1) & 1u);  // every CTA's entry has landed here
+      const float4* ex = exch + slot * kMaxCluster;
       float mc = -INFINITY, sc = 0.f;
       if (lane < (int)C) {
-        const float4 v = ld_cluster_f4(st_addr, lane);
+        const float4 v = ex[lane];
         mc = v.x;
         sc = v.y;
       }
@@ -381,7 +443,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
             if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
           }
         } else {
-          const float zy = ld_cluster_f4(st_addr, (uint32_t)(yv / a.slice)).z;
+          const float zy = ex[yv / a.slice].z;
           const float S_excl = term;
           const float ey = expf(zy - M);
           const float S = S_excl + ey;
@@ -409,6 +471,10 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           neg_scale = -coef / S;
           dy = coef * (S_excl / S);
           shB = -M * kLog2e;
+          if (fabsf(neg_scale) >= 0x1p-100f) {
+            shB += kShiftB;
+            neg_scale *= 0x1p-16f;  // 2^-kShiftB
+          }
           if (rank == 0) {
             if (a.logp_out) a.logp_out[row] = logp;
             a.row_loss[row] = w * (double)ell;
@@ -426,36 +492,47 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
     // ---- pass B: dlogits from the shared-memory slice; refill chunk by chunk ----
     const float neg_scale = rowsc[0], dy = rowsc[1], shB = rowsc[2];
     const bool zero_row = rowsc[3] != 0.f;
+    const float2 shb2 = make_float2(shB, shB), ns2 = make_float2(neg_scale, neg_scale);
     OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V + s0;
     const int64_t next = row + ncl;
     const char* gnext = (tid == 0 && next < a.n_rows) ? row_base(next) : nullptr;
     for (int k = 0; k < a.n_chunks; ++k) {
       const int v0 = k * a.chunk_vecs;
       const int v1 = min(nvec, v0 + a.chunk_vecs);
-      for (int j = v0 + tid; j < v1; j += kThreads) {
-        float f[kVec], d[kVec];
-        Fmt<InT>::unpack(buf4[j], f);
+      const bool last = (k == a.n_chunks - 1);
+      if (!zero_row) {
+        for (int j = v0 + tid; j < v1; j += kThreads) {
+          float2 p[kPairs], d[kPairs];
+          Fmt<InT>::pairs(buf4[j], p);
 #pragma unroll
-        for (int i = 0; i < kVec; ++i) d[i] = zero_row ? 0.f : neg_scale * ex2(fmaf(f[i], kLog2e, shB));
-        const int yi = yl - j * kVec;
-        if ((unsigned)yi < (unsigned)kVec && !zero_row) {
+          for (int i = 0; i < kPairs; ++i) d[i] = __fmul2_rn(ex2x2(__ffma2_rn(p[i], l2e2, shb2)), ns2);
+          const int yi = yl - j * kVec;
+          if ((unsigned)yi < (unsigned)kVec) {
 #pragma unroll
-          for (int i = 0; i < kVec; ++i)
-            if (i == yi) d[i] = dy;
+            for (int i = 0; i < kPairs; ++i) {
+              if (2 * i == yi) d[i].x = dy;
+              if (2 * i + 1 == yi) d[i].y = dy;
+            }
+          }
+          if (a.out_vec)
+            store_pairs<OutT, kPairs>(orow + j * kVec, d);
+          else
+            store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
         }
-        if (a.out_vec) {
-          store_vec<OutT, kVec>(orow + j * kVec, d);
-        } else {
+        if (last) {
+          for (int e = tail0 + tid; e < len; e += kThreads) {
+            float d = neg_scale * ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, shB));
+            if (e == yl) d = dy;
+            Fmt<OutT>::store(orow + e, d);
+          }
+        }
+      } else {
+        float2 d[kPairs];
 #pragma unroll
-          for (int i = 0; i < kVec; ++i) Fmt<OutT>::store(orow + j * kVec + i, d[i]);
-        }
-      }
-      if (k == a.n_chunks - 1) {
-        for (int e = tail0 + tid; e < len; e += kThreads) {
-          float d = zero_row ? 0.f : neg_scale * ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, shB));
-          if (e == yl && !zero_row) d = dy;
-          Fmt<OutT>::store(orow + e, d);
-        }
+        for (int i = 0; i < kPairs; ++i) d[i] = make_float2(0.f, 0.f);
+        for (int j = v0 + tid; j < v1; j += kThreads) store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
+        if (last)
+          for (int e = tail0 + tid; e < len; e += kThreads) Fmt<OutT>::store(orow + e, 0.f);
       }
       __syncthreads();  // chunk k consumed by every thread
       if (gnext && !*(volatile int*)abort_flag) issue_chunk(gnext, k);
@@ -574,11 +651,14 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   const int out_bytes = dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   const int vec = 16 / in_bytes;
   const int threads = tune.threads ? tune.threads : 256;
-  // Cluster size: the smallest C whose slices are at most ~40 KiB (several CTAs per SM).
+  // Cluster size: slices of at most 80 KiB (two CTAs per SM), and at least two CTAs per row once
+  // a row exceeds 32 KiB.  Measured on GB300 over cluster sizes 1-16, 128-512 threads and 1-5
+  // copies per slice, this shape moved the most bytes per second for V = 32000 and 152064.
   int C = tune.cluster;
   if (C == 0) {
-    C = 1;
-    while (C < 8 && (int64_t)V * in_bytes > (int64_t)C * 40 * 1024) C *= 2;
+    const int64_t row_bytes = (int64_t)V * in_bytes;
+    C = (int)std::min<int64_t>(kMaxCluster, (row_bytes + 80 * 1024 - 1) / (80 * 1024));
+    if (C == 1 && row_bytes > 32 * 1024) C = 2;
   }
   int slice = (int)align_up((size_t)((V + C - 1) / C), vec);
   while (C > 1 && (int64_t)(C - 1) * slice >= V) {  // no empty slices
@@ -586,13 +666,22 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
     slice = (int)align_up((size_t)((V + C - 1) / C), vec);
   }
   const size_t slice_bytes = (size_t)slice * in_bytes;
-  int chunks = tune.chunks ? tune.chunks : (int)std::min<size_t>(8, std::max<size_t>(1, slice_bytes / 8192));
+  // about 36 KiB per bulk copy
+  int chunks = tune.chunks ? tune.chunks
+                           : (int)std::min<size_t>(kMaxChunks, std::max<size_t>(1, (slice_bytes + 18 * 1024) / (36 * 1024)));
   const int slice_vecs = slice / vec;
   int chunk_vecs = (slice_vecs + chunks - 1) / chunks;
   if (chunk_vecs < 1) chunk_vecs = 1;
+  // whole vectors per thread in every chunk but the last one
+  const int even = (chunk_vecs + threads - 1) / threads * threads;
+  if (even <= slice_vecs) chunk_vecs = even;
   chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
   if (chunks < 1) chunks = 1;
-  const size_t smem = align_up(slice_bytes, 128) + kMaxChunks * 8 + 2 * 16 +
+  if (chunks > kMaxChunks) {
+    chunk_vecs = (slice_vecs + kMaxChunks - 1) / kMaxChunks;
+    chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
+  }
+  const size_t smem = align_up(slice_bytes, 128) + kMaxChunks * 8 + 2 * 8 + 2 * kMaxCluster * 16 +
                       2 * (threads / 32) * 4 + 4 * 4 + 16;
   if (smem > 227 * 1024)
     return fail(GRPO_ERR_UNSUPPORTED, "%s: V = %d needs %zu bytes of shared memory per CTA at %d CTAs", who,

@@ -125,7 +125,7 @@ class GrpoStep:
             V=p.V, row_index=self.src_token, n_rows=self.T_kept, eps_low=p.eps_low,
             eps_high=p.eps_high, beta=p.beta, agg_mode=p.agg_mode,
             denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
-            dlogits=self.dlogits, logp_out=self.logp, loss_out=self.loss, status=self.status,
+            dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp, loss_out=self.loss, status=self.status,
             ws=self.loss_ws)
 
     def run(self):
