@@ -159,6 +159,35 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def host_mem_available():
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return float("inf")
+
+
+def combine_ranks(elapsed_ms, kept, world, device):
+    """(max over ranks of the timed region, sum over ranks of the kept tokens processed)."""
+    if world <= 1:
+        return float(elapsed_ms), float(kept)
+    import torch
+    import torch.distributed as dist
+    mx = torch.tensor([float(elapsed_ms)], dtype=torch.float64, device=device)
+    sm = torch.tensor([float(kept)], dtype=torch.float64, device=device)
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return float(mx.item()), float(sm.item())
+
+
+def rank_seed(base_seed, rank):
+    """Each rank draws its own batch (weak scaling: per-rank work is fixed as ranks grow)."""
+    return base_seed + rank
+
+
 def build_inputs(w, seed, device):
     """Seeded synthetic batch, resident on `device` (logits of every token)."""
     import torch
@@ -176,7 +205,8 @@ def build_inputs(w, seed, device):
 def make_step(w, dev_inputs):
     from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
     p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
-                   eps_low=w.eps, eps_high=w.eps, beta=w.beta, dlogits_dtype=w.dlogits_dtype)
+                   eps_low=w.eps, eps_high=w.eps, beta=w.beta, dlogits_dtype=w.dlogits_dtype,
+                   chunk_rows=w.chunk_rows)
     d = dev_inputs
     return GrpoStep(p, d["rewards"], d["ids"], d["off"], d["logits"], d["old"], d["ref"])
 
@@ -303,7 +333,7 @@ def main():
     dev = torch.device("cuda", local)
     g.lib()
 
-    b, d = build_inputs(w, args.seed + rank, dev)
+    b, d = build_inputs(w, rank_seed(args.seed, rank), dev)
     step = make_step(w, d)
     for _ in range(max(args.warmup, 3)):
         step.run()
@@ -337,15 +367,7 @@ def main():
     g.check_status(step.status)
     elapsed_ms = ev0.elapsed_time(ev1)
     loss_ms = statistics.mean(a.elapsed_time(z) for a, z in zip(l0, l1))
-    tot = torch.tensor([elapsed_ms, float(kept)], dtype=torch.float64, device=dev)
-    if world > 1:
-        mx = tot[:1].clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = tot[1:].clone()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        elapsed_ms, kept_all = float(mx.item()), float(sm.item())
-    else:
-        kept_all = float(kept)
+    elapsed_ms, kept_all = combine_ranks(elapsed_ms, kept, world, dev)
     value = kept_all / (elapsed_ms / 1e3)
 
     # roofline of the dominant kernel (the fused loss), from its event-timed launches
@@ -362,10 +384,17 @@ def main():
 
     # end to end: inputs copied from pinned host memory, loss read back, inside the timed region
     e2e = None
-    if args.e2e_steps > 0:
-        names = ["rewards", "ids", "off", "logits", "old", "ref"]
-        host = {k: d[k].cpu().pin_memory() for k in names}
-        h2d = sum(host[k].numel() * host[k].element_size() for k in names)
+    names = ["rewards", "ids", "off", "logits", "old", "ref"]
+    h2d = sum(d[k].numel() * d[k].element_size() for k in names)
+    if args.e2e_steps > 0 and h2d > 0.6 * host_mem_available():
+        e2e = {"value": None, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 0,
+               "skipped": "pinned host copies of the inputs (%.0f GB) exceed 60%% of available host"
+                          " memory" % (h2d / 1e9)}
+    elif args.e2e_steps > 0:
+        host = {}
+        for k in names:
+            host[k] = torch.empty(d[k].shape, dtype=d[k].dtype, pin_memory=True)
+            host[k].copy_(d[k])
         loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
         d2h = 8 + 16 + 4 * w.P
         step.run()
@@ -383,14 +412,7 @@ def main():
             kept_e += step.T_kept
         e1.record(stream)
         torch.cuda.synchronize()
-        e_ms = e0.elapsed_time(e1)
-        et = torch.tensor([e_ms, float(kept_e)], dtype=torch.float64, device=dev)
-        if world > 1:
-            mx = et[:1].clone()
-            dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-            sm = et[1:].clone()
-            dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-            e_ms, kept_e = float(mx.item()), float(sm.item())
+        e_ms, kept_e = combine_ranks(e0.elapsed_time(e1), kept_e, world, dev)
         e2e = {"value": kept_e / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "steps": args.e2e_steps}
         del host

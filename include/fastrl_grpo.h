@@ -179,6 +179,15 @@ grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t 
                               grpo_stream_t stream);
 
 /*
+ * grpo_sum_f64 — *out = v[0] + ... + v[n-1] in fp64, in the same fixed order grpo_loss_fwd_bwd
+ * uses for loss_out (bitwise reproducible).  With row_loss_out, a loss computed over rows in
+ * several calls (for example chunks of kept rows sharing one dlogits buffer) then sums to
+ * exactly the value a single call over all rows gives.
+ * v device f64 [n]; out device f64 [1].
+ */
+grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grpo_stream_t stream);
+
+/*
  * grpo_loss_fwd_bwd_noalloc — grpo_loss_fwd_bwd for callers that cannot allocate device memory.
  * The paper has no counterpart: this is an interface convenience of this library.
  * Some callers run the loss where no allocation is possible: a plugin or custom-op host that

@@ -31,7 +31,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_noalloc",
+           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64",
            "grpo_loss_tune", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -86,6 +86,8 @@ def lib():
                                             _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64,
                                             _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p]
     L.grpo_loss_fwd_bwd_noalloc.restype = _i32
+    L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
+    L.grpo_sum_f64.restype = _i32
     L.grpo_loss_tune.argtypes = [_i32, _i32, _i32]
     L.grpo_loss_tune.restype = _i32
     L.grpo_ars_init.argtypes = [ctypes.POINTER(ArsState), _i32]
@@ -349,6 +351,18 @@ def grpo_loss_fwd_bwd_noalloc(logits, y, old_logp, ref_logp, adv, row_rollout, *
         float(beta), int(agg_mode), int(denom_tokens), _ptr(seq_off), int(n_seq), _ptr(dlogits),
         odt, _ptr(logp_out), _ptr(row_loss_out), _ptr(loss_out), _ptr(status), _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out)
+
+
+def grpo_sum_f64(v, n: int | None = None, out=None, stream=None):
+    """Fixed-order fp64 sum of v[:n] on the GPU (the loss's own reduction)."""
+    torch = _torch()
+    _need(v, torch.float64, n, "v")
+    if n is None:
+        n = v.numel()
+    if out is None:
+        out = torch.empty(1, dtype=torch.float64, device=v.device)
+    _check(lib().grpo_sum_f64(_ptr(v), int(n), _ptr(out), _stream(stream)))
+    return out
 
 
 def grpo_ars_init(G1: int) -> ArsState:

@@ -602,6 +602,15 @@ extern "C" grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int
   return GRPO_OK;
 }
 
+extern "C" grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grpo_stream_t stream) {
+  clear_error();
+  if (n < 0 || out == nullptr || (n > 0 && v == nullptr))
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_sum_f64: n = %lld, v or out NULL", (long long)n);
+  sum_rows_kernel<<<1, 1024, 0, as_stream(stream)>>>(v, n, out);
+  count_launches(1);
+  return check_launch("grpo_sum_f64");
+}
+
 extern "C" grpo_status grpo_loss_fwd_bwd(
     const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
     int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,

@@ -30,6 +30,7 @@ class StepParams:
     agg_mode: int = 0
     dlogits_dtype: str = "bf16"
     std_mode: int = 0
+    chunk_rows: int = 0  # >0: the loss runs over the kept rows in chunks sharing one dlogits buffer
 
 
 class GrpoStep:
@@ -119,6 +120,8 @@ class GrpoStep:
 
     def loss_step(self):
         p = self.p
+        if p.chunk_rows > 0:
+            return self._loss_chunked()
         self._ensure_dlogits(self.T_kept)
         return B.grpo_loss_fwd_bwd(
             self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout,
@@ -127,6 +130,28 @@ class GrpoStep:
             denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
             dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp, loss_out=self.loss, status=self.status,
             ws=self.loss_ws)
+
+    def _loss_chunked(self):
+        """Kept rows in chunks of p.chunk_rows; each chunk overwrites the same dlogits buffer
+        (a consumer would use it before the next chunk).  Per-row loss terms are kept and summed
+        once at the end in the loss's own fixed order, so the total equals a single call's."""
+        p = self.p
+        torch = self.torch
+        self._ensure_dlogits(min(p.chunk_rows, max(self.T_kept, 1)))
+        if getattr(self, "row_loss", None) is None:
+            self.row_loss = torch.empty(max(self.T, 1), dtype=torch.float64, device=self.dev)
+            self.chunk_loss = torch.empty(1, dtype=torch.float64, device=self.dev)
+        for c0 in range(0, self.T_kept, p.chunk_rows):
+            c1 = min(self.T_kept, c0 + p.chunk_rows)
+            B.grpo_loss_fwd_bwd(
+                self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout[c0:c1],
+                V=p.V, row_index=self.src_token[c0:c1], n_rows=c1 - c0, eps_low=p.eps_low,
+                eps_high=p.eps_high, beta=p.beta, agg_mode=p.agg_mode,
+                denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
+                dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp[c0:c1],
+                row_loss_out=self.row_loss[c0:c1], loss_out=self.chunk_loss, status=self.status)
+        B.grpo_sum_f64(self.row_loss, self.T_kept, out=self.loss)
+        return dict(loss=self.loss, dlogits=self.dlogits, logp=self.logp)
 
     def run(self):
         self.select()

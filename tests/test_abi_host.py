@@ -127,3 +127,27 @@ def test_loss_argument_errors(grpo):
     assert loss_call(L, 10, 100, None, ctypes.byref(size), denom=0) == 1
     assert loss_call(L, 10, 100, None, ctypes.byref(size), agg=1) == 1  # needs seq_off
     assert loss_call(L, 10, 100, None, ctypes.byref(size), beta=-1.0) == 1
+
+
+def test_ars_closed_loop_of_the_large_group_workload(oracle_mod, grpo):
+    """20 steps, G1 = 16, 5 steps per epoch, pruning ratios U(0.1, 0.6) per prompt: the library's
+    host ARS and the oracle choose the same rollout count at every step."""
+    from paper_2609_36932_gb300 import workloads
+    w = workloads.get("large")
+    steps, spe = 20, 5
+    ratios = workloads.ars_pruning_ratios(0, steps, w.P)
+
+    def loop(step_fn):
+        n, seq = w.G, []
+        for s in range(1, steps + 1):
+            kept = workloads.synthetic_kept_counts(ratios[s - 1], n)
+            n = step_fn(kept, s, s % spe == 0)
+            seq.append(n)
+        return seq
+
+    o = oracle_mod.Ars(w.G)
+    st = grpo.grpo_ars_init(w.G)
+    seq_o = loop(lambda k, s, e: o.step(k, s, steps, e))
+    seq_l = loop(lambda k, s, e: grpo.adaptive_rollout_count(st, k, s, steps, e))
+    assert seq_o == seq_l
+    assert all(2 <= n <= w.G for n in seq_o)
