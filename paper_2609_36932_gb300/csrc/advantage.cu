@@ -1,29 +1,40 @@
 // grpo_advantage: group-relative advantages, Eq. 5 (Sec. 3.2).
 //
-// One thread per prompt.  A group has at most a few dozen rewards, so the fp64 sums run
-// sequentially in index order with explicitly rounded operations (no fused multiply-add); the
-// result is then reproducible bit for bit from the order of operations written here.
+// One warp per prompt.  The fp64 sums run in index order (every lane executes the same
+// sequence of explicitly rounded additions on values exchanged by shuffles), so the mean, the
+// std and each A are reproducible bit for bit from the order of operations written here; the
+// per-rollout divisions then run in parallel across lanes.
 #include "common.cuh"
 
 namespace fastrl {
 namespace {
 
+constexpr unsigned kFull = 0xffffffffu;
+
 __global__ void advantage_kernel(const float* __restrict__ rewards, int P, int G, int std_mode,
                                  float* __restrict__ adv, double* __restrict__ key) {
-  const int p = blockIdx.x * blockDim.x + threadIdx.x;
-  if (p >= P) return;
+  const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (p >= P) return;  // uniform per warp
   const float* r = rewards + (int64_t)p * G;
   double sum = 0.0;
-  for (int i = 0; i < G; ++i) sum = __dadd_rn(sum, (double)r[i]);
+  for (int base = 0; base < G; base += 32) {
+    const float v = base + lane < G ? r[base + lane] : 0.f;
+    const int nb = min(32, G - base);
+    for (int k = 0; k < nb; ++k) sum = __dadd_rn(sum, (double)__shfl_sync(kFull, v, k));
+  }
   const double mean = __ddiv_rn(sum, (double)G);
   double ss = 0.0;
-  for (int i = 0; i < G; ++i) {
-    const double dev = __dsub_rn((double)r[i], mean);
-    ss = __dadd_rn(ss, __dmul_rn(dev, dev));
+  for (int base = 0; base < G; base += 32) {
+    const float v = base + lane < G ? r[base + lane] : 0.f;
+    const double dev = __dsub_rn((double)v, mean);
+    const double sq = __dmul_rn(dev, dev);
+    const int nb = min(32, G - base);
+    for (int k = 0; k < nb; ++k) ss = __dadd_rn(ss, __shfl_sync(kFull, sq, k));
   }
   const int divisor = std_mode == 0 ? G - 1 : G;
   const double sd = divisor > 0 ? __dsqrt_rn(__ddiv_rn(ss, (double)divisor)) : 0.0;
-  for (int i = 0; i < G; ++i) {
+  for (int i = lane; i < G; i += 32) {
     const double dev = __dsub_rn((double)r[i], mean);
     const double a = sd > 0.0 ? __ddiv_rn(dev, sd) : 0.0;
     adv[(int64_t)p * G + i] = __double2float_rn(a);
@@ -46,8 +57,8 @@ extern "C" grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G
   if (P == 0) return GRPO_OK;
   if (rewards == nullptr || adv == nullptr)
     return fail(GRPO_ERR_INVALID_ARG, "grpo_advantage: rewards and adv must not be NULL");
-  const int threads = 128;
-  advantage_kernel<<<(P + threads - 1) / threads, threads, 0, as_stream(stream)>>>(
+  const int threads = 128;  // four prompts per CTA
+  advantage_kernel<<<(unsigned)(((int64_t)P * 32 + threads - 1) / threads), threads, 0, as_stream(stream)>>>(
       rewards, P, G, std_mode, adv, key);
   count_launches(1);
   return check_launch("grpo_advantage");

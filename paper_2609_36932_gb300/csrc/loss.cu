@@ -52,13 +52,17 @@ struct LossArgs {
   const float* ref_logp;
   const float* adv;
   const int32_t* row_rollout;
-  double clip_lo;  // 1 - eps_low
-  double clip_hi;  // 1 + eps_high
+  // Clip bounds 1 - eps_low and 1 + eps_high are defined in fp64.  For an f32 ratio rho,
+  // rho <= hi_dn and rho >= lo_up decide exactly as the fp64 comparisons (hi_dn: largest f32
+  // <= 1 + eps_high; lo_up: smallest f32 >= 1 - eps_low); clamped values round to nearest.
+  // The row scalars then need no fp64 arithmetic, which is scarce on this GPU.
+  float lo_up, hi_dn, lo_rn, hi_rn;
   float beta;
   int32_t agg_mode;
   double inv_denom;  // agg 0: 1 / denom_tokens
+  float inv_denom_f;
   const int64_t* seq_off;
-  double inv_nseq;  // agg 1: 1 / n_seq
+  float inv_nseq_f;  // agg 1: 1 / n_seq
   char* dlogits;
   float* logp_out;
   double* row_loss;
@@ -451,23 +455,22 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           // Eq. 1: ratio, clipped surrogate, KL term; Eqs. 2-3: gradient coefficient.
           const float A = a.adv[a.row_rollout[row]];
           const float rho = expf(logp - a.old_logp[src]);
-          const double rho_d = (double)rho;
-          const float clipped = (float)fmin(fmax(rho_d, a.clip_lo), a.clip_hi);
+          const float clipped = rho < a.lo_up ? a.lo_rn : (rho > a.hi_dn ? a.hi_rn : rho);
           const float surr = fminf(rho * A, clipped * A);
           const float x = a.ref_logp[src] - logp;
           const float em1 = expm1f(x);
           const float kl = em1 - x;
           const float ell = -(surr - a.beta * kl);
-          double w;
+          float w;
           if (a.agg_mode == 0) {
-            w = a.inv_denom;
+            w = a.inv_denom_f;
           } else {
             const int32_t r = a.row_rollout[row];
-            w = a.inv_nseq / (double)(a.seq_off[r + 1] - a.seq_off[r]);
+            w = a.inv_nseq_f / (float)(a.seq_off[r + 1] - a.seq_off[r]);
           }
-          const bool c = (A >= 0.f) ? (rho_d <= a.clip_hi) : (rho_d >= a.clip_lo);
+          const bool c = (A >= 0.f) ? (rho <= a.hi_dn) : (rho >= a.lo_up);
           const float g = -((c ? rho * A : 0.f) + a.beta * em1);
-          const float coef = (float)(w * (double)g);
+          const float coef = w * g;
           neg_scale = -coef / S;
           dy = coef * (S_excl / S);
           shB = -M * kLog2e;
@@ -477,7 +480,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           }
           if (rank == 0) {
             if (a.logp_out) a.logp_out[row] = logp;
-            a.row_loss[row] = w * (double)ell;
+            a.row_loss[row] = (a.agg_mode == 0 ? a.inv_denom : (double)w) * (double)ell;
             if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
           }
         }
@@ -707,13 +710,20 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   a.ref_logp = ref_logp;
   a.adv = adv;
   a.row_rollout = row_rollout;
-  a.clip_lo = 1.0 - (double)eps_low;
-  a.clip_hi = 1.0 + (double)eps_high;
+  {
+    const double lo = 1.0 - (double)eps_low, hi = 1.0 + (double)eps_high;
+    const float lo_f = (float)lo, hi_f = (float)hi;  // nearest
+    a.lo_rn = lo_f;
+    a.hi_rn = hi_f;
+    a.lo_up = (double)lo_f < lo ? std::nextafter(lo_f, INFINITY) : lo_f;
+    a.hi_dn = (double)hi_f > hi ? std::nextafter(hi_f, -INFINITY) : hi_f;
+  }
   a.beta = beta;
   a.agg_mode = agg_mode;
   a.inv_denom = agg_mode == 0 ? 1.0 / (double)denom_tokens : 0.0;
+  a.inv_denom_f = (float)a.inv_denom;
   a.seq_off = seq_off;
-  a.inv_nseq = agg_mode == 1 ? 1.0 / (double)n_seq : 0.0;
+  a.inv_nseq_f = agg_mode == 1 ? (float)(1.0 / (double)n_seq) : 0.f;
   a.dlogits = static_cast<char*>(dlogits);
   a.logp_out = logp_out;
   a.row_loss = row_loss;

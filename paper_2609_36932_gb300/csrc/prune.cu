@@ -1,17 +1,19 @@
 // grpo_prune: maximising-differential advantage pruning (MDAP), Sec. 3.2 Eqs. 6-9, with the
 // traversal order, per-class guarantee and DP-alignment fill of Algorithm 1 (Phase 2).
 //
-// Three kernels (a fourth when dp_divisor > 1):
-//   1. ngram_set_kernel   one CTA per rollout: pack each length-n window of token ids into a
-//                         64-bit key (18 bits per id), bitonic-sort the keys (in shared memory
-//                         when they fit, else in the workspace), drop repeats -> N_n(o_i) (Eq. 7)
-//                         as a sorted array plus its size.
-//   2. intersect_kernel   one warp per pair (i < j) of a prompt with equal rewards: |N_i & N_j|
-//                         by binary search of the smaller set's keys in the larger one.
-//   3. select_kernel      one thread per prompt: fp64 |r - mean| order, greedy Eq. 8 per reward
-//                         class, per-prompt cap by round-robin over classes.
-//   4. dp_fill_kernel     one thread: cyclic fill until the kept total is a multiple of d.
-// All decisions are integer or exactly rounded fp64 operations, so the keep mask is bit-exact.
+// Kernels, in stream order:
+//   1. the n-gram sets N_n(o_i) of Eq. 7, one CTA per rollout:
+//        n = 1   unigram_set_kernel: a bitmap over the vocabulary built in shared memory;
+//        n = 2,3 ngram_set_kernel: each length-n window packed into a 64-bit key (18 bits per id),
+//                bitonic-sorted (shared memory when it fits, else the workspace), repeats dropped;
+//   2. the pair test theta_ij < tau for every pair i < j of a prompt with equal rewards:
+//        n = 1   bitmap_pair_kernel: |N_i & N_j| = popcount of the AND, one CTA per pair;
+//        n = 2,3 sorted_pair_kernel: binary search of the smaller set in the larger, a warp per pair;
+//      each writes one byte per ordered pair: 1 when the two are in one class and too close;
+//   3. select_kernel, one warp per prompt: fp64 |r - mean| visiting order, the greedy of Eq. 8 as
+//      bitmask operations, and the per-prompt cap by round-robin over classes;
+//   4. dp_fill_kernel (dp_divisor > 1), one thread: cyclic fill to a multiple of the divisor.
+// Every decision is an integer or exactly rounded fp64 operation, so the keep mask is bit-exact.
 #include <algorithm>
 
 #include "common.cuh"
@@ -25,26 +27,33 @@ constexpr uint64_t kSentinel = ~0ull;  // sorts after every real key (< 2^54)
 constexpr int kMaxG = 32;
 
 struct PruneWs {
-  uint64_t* keys;  // [2T]: rollout r owns keys[2*off[r] .. 2*off[r+1])
-  int32_t* nuniq;  // [P*G]
-  int32_t* inter;  // [P*G*G]
+  uint64_t* keys;     // n >= 2: [2T]; rollout r owns keys[2*off[r] .. 2*off[r+1])
+  uint64_t* bitmaps;  // n == 1: [P*G][words]
+  int32_t* nuniq;     // [P*G] set sizes
+  uint8_t* close;     // [P*G*G]: close[(p*G + i)*G + j] = 1 if same class and theta_ij < tau
+  int words;          // ceil(V / 64)
 };
 
-__host__ __device__ inline size_t ws_keys_bytes(int64_t T) { return (size_t)(2 * T) * 8; }
+__host__ __device__ inline int bitmap_words(int V) { return (V + 63) / 64; }
 
-size_t prune_ws_bytes(int64_t T, int P, int G) {
-  return align_up(ws_keys_bytes(T), 256) + align_up((size_t)P * G * 4, 256) +
-         align_up((size_t)P * G * G * 4, 256);
+size_t prune_ws_bytes(int64_t T, int P, int G, int V, int n) {
+  const size_t keys = n >= 2 ? (size_t)(2 * T) * 8 : 0;
+  const size_t bitmaps = n == 1 ? (size_t)P * G * bitmap_words(V) * 8 : 0;
+  return align_up(keys, 256) + align_up(bitmaps, 256) + align_up((size_t)P * G * 4, 256) +
+         align_up((size_t)P * G * G, 256);
 }
 
-PruneWs prune_ws(void* ws, int64_t T, int P, int G) {
+PruneWs prune_ws(void* ws, int64_t T, int P, int G, int V, int n) {
   char* p = static_cast<char*>(ws);
   PruneWs w;
+  w.words = bitmap_words(V);
   w.keys = reinterpret_cast<uint64_t*>(p);
-  p += align_up(ws_keys_bytes(T), 256);
+  p += align_up(n >= 2 ? (size_t)(2 * T) * 8 : 0, 256);
+  w.bitmaps = reinterpret_cast<uint64_t*>(p);
+  p += align_up(n == 1 ? (size_t)P * G * w.words * 8 : 0, 256);
   w.nuniq = reinterpret_cast<int32_t*>(p);
   p += align_up((size_t)P * G * 4, 256);
-  w.inter = reinterpret_cast<int32_t*>(p);
+  w.close = reinterpret_cast<uint8_t*>(p);
   return w;
 }
 
@@ -149,24 +158,100 @@ __global__ void __launch_bounds__(kSortThreads)
   if (threadIdx.x == 0) w.nuniq[r] = out_base;
 }
 
-__global__ void intersect_kernel(const float* __restrict__ rewards, const int64_t* __restrict__ off,
-                                 int P, int G, PruneWs w) {
-  const int pairs_per_prompt = G * (G - 1) / 2;
-  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (gw >= (int64_t)P * pairs_per_prompt) return;
-  const int p = (int)(gw / pairs_per_prompt);
-  int k = (int)(gw % pairs_per_prompt);
-  int i = 0;
-  while (k >= G - 1 - i) {  // pair index -> (i, j), i < j
+// theta_ij < tau (Eqs. 7-8), from integer set sizes; two empty sets have theta = 0.
+__device__ bool too_close(int I, int ni, int nj, float tau) {
+  const int U = ni + nj - I;
+  if (U == 0) return 0.0 < (double)tau;
+  const double theta = __dsub_rn(1.0, __ddiv_rn((double)I, (double)U));
+  return theta < (double)tau;
+}
+
+// pair index k of a prompt -> (i, j), i < j, in row-major order of the upper triangle
+__device__ void pair_of(int k, int G, int& i, int& j) {
+  i = 0;
+  while (k >= G - 1 - i) {
     k -= G - 1 - i;
     ++i;
   }
-  const int j = i + 1 + k;
+  j = i + 1 + k;
+}
+
+__global__ void unigram_set_kernel(const int32_t* __restrict__ ids, const int64_t* __restrict__ off,
+                                   int V, PruneWs w, int32_t* status) {
+  extern __shared__ __align__(16) unsigned long long bm[];
+  __shared__ int warp_cnt[32];
+  const int r = blockIdx.x;
+  const int64_t o = off[r];
+  const int64_t L = off[r + 1] - o;
+  for (int k = threadIdx.x; k < w.words; k += blockDim.x) bm[k] = 0ull;
+  __syncthreads();
+  bool bad = false;
+  for (int64_t t = threadIdx.x; t < L; t += blockDim.x) {
+    const int32_t id = ids[o + t];
+    if (id < 0 || id >= V) {
+      bad = true;
+      continue;
+    }
+    atomicOr(&bm[id >> 6], 1ull << (id & 63));
+  }
+  if (bad && status) atomicOr(status, GRPO_DEVFLAG_BAD_TOKEN);
+  __syncthreads();
+  uint64_t* out = w.bitmaps + (int64_t)r * w.words;
+  int cnt = 0;
+  for (int k = threadIdx.x; k < w.words; k += blockDim.x) {
+    const unsigned long long v = bm[k];
+    out[k] = v;
+    cnt += __popcll(v);
+  }
+  for (int s = 16; s > 0; s >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, s);
+  if ((threadIdx.x & 31) == 0) warp_cnt[threadIdx.x >> 5] = cnt;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int total = 0;
+    for (int q = 0; q < (int)(blockDim.x >> 5); ++q) total += warp_cnt[q];
+    w.nuniq[r] = total;
+  }
+}
+
+__global__ void bitmap_pair_kernel(const float* __restrict__ rewards, int G, float tau, PruneWs w) {
+  __shared__ int warp_cnt[32];
+  const int pairs = G * (G - 1) / 2;
+  const int p = blockIdx.x / pairs;
+  int i, j;
+  pair_of(blockIdx.x % pairs, G, i, j);
   const int ri = p * G + i, rj = p * G + j;
-  int32_t* inter = w.inter + (int64_t)p * G * G;
+  uint8_t* close = w.close + (int64_t)p * G * G;
   if (rewards[ri] != rewards[rj]) {  // different classes never compare (Eq. 8 is per class)
-    if (lane == 0) inter[i * G + j] = inter[j * G + i] = -1;
+    if (threadIdx.x == 0) close[i * G + j] = close[j * G + i] = 0;
+    return;
+  }
+  const uint64_t* a = w.bitmaps + (int64_t)ri * w.words;
+  const uint64_t* b = w.bitmaps + (int64_t)rj * w.words;
+  int cnt = 0;
+  for (int k = threadIdx.x; k < w.words; k += blockDim.x) cnt += __popcll(a[k] & b[k]);
+  for (int s = 16; s > 0; s >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, s);
+  if ((threadIdx.x & 31) == 0) warp_cnt[threadIdx.x >> 5] = cnt;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int I = 0;
+    for (int q = 0; q < (int)(blockDim.x >> 5); ++q) I += warp_cnt[q];
+    close[i * G + j] = close[j * G + i] = too_close(I, w.nuniq[ri], w.nuniq[rj], tau) ? 1 : 0;
+  }
+}
+
+__global__ void sorted_pair_kernel(const float* __restrict__ rewards, const int64_t* __restrict__ off,
+                                   int P, int G, float tau, PruneWs w) {
+  const int pairs = G * (G - 1) / 2;
+  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (gw >= (int64_t)P * pairs) return;
+  const int p = (int)(gw / pairs);
+  int i, j;
+  pair_of((int)(gw % pairs), G, i, j);
+  const int ri = p * G + i, rj = p * G + j;
+  uint8_t* close = w.close + (int64_t)p * G * G;
+  if (rewards[ri] != rewards[rj]) {
+    if (lane == 0) close[i * G + j] = close[j * G + i] = 0;
     return;
   }
   int na = w.nuniq[ri], nb = w.nuniq[rj];
@@ -194,7 +279,8 @@ __global__ void intersect_kernel(const float* __restrict__ rewards, const int64_
     cnt += (lo < nb && b[lo] == key) ? 1 : 0;
   }
   for (int s = 16; s > 0; s >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, s);
-  if (lane == 0) inter[i * G + j] = inter[j * G + i] = cnt;
+  if (lane == 0)
+    close[i * G + j] = close[j * G + i] = too_close(cnt, w.nuniq[ri], w.nuniq[rj], tau) ? 1 : 0;
 }
 
 // |r_i - mean| in fp64 with Eq. 5's index-order mean; the visiting key of Algorithm 1.
@@ -205,84 +291,66 @@ __device__ void group_dist(const float* r, int G, double* dist) {
   for (int i = 0; i < G; ++i) dist[i] = fabs(__dsub_rn((double)r[i], mean));
 }
 
-// theta_ij < tau (Eqs. 7-8), from integer set sizes; two empty sets have theta = 0.
-__device__ bool too_close(int I, int ni, int nj, float tau) {
-  const int U = ni + nj - I;
-  if (U == 0) return 0.0 < (double)tau;
-  const double theta = __dsub_rn(1.0, __ddiv_rn((double)I, (double)U));
-  return theta < (double)tau;
-}
-
-__global__ void select_kernel(const float* __restrict__ rewards, int P, int G, float tau,
-                              int keep_cap, PruneWs w, uint8_t* __restrict__ keep,
+// One warp per prompt; lane i holds rollout i (G <= 32).
+__global__ void select_kernel(const float* __restrict__ rewards, int P, int G, int keep_cap,
+                              PruneWs w, uint8_t* __restrict__ keep,
                               int32_t* __restrict__ kept_per_prompt) {
-  const int p = blockIdx.x * blockDim.x + threadIdx.x;
-  if (p >= P) return;
-  const float* r = rewards + (int64_t)p * G;
-  const int32_t* nu = w.nuniq + (int64_t)p * G;
-  const int32_t* inter = w.inter + (int64_t)p * G * G;
-  double dist[kMaxG];
-  int order[kMaxG];
-  bool kept[kMaxG];
-  group_dist(r, G, dist);
-  for (int i = 0; i < G; ++i) {  // stable insertion sort: dist descending, index ascending
-    int k = i;
-    while (k > 0 && dist[order[k - 1]] < dist[i]) {
-      order[k] = order[k - 1];
-      --k;
-    }
-    order[k] = i;
-    kept[i] = false;
+  constexpr unsigned FULL = 0xffffffffu;
+  const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (p >= P) return;  // uniform per warp
+  const bool act = lane < G;
+  const float r = act ? rewards[(int64_t)p * G + lane] : 0.f;
+  // Eq. 5's mean, summed in index order (every lane runs the same sequence)
+  double sum = 0.0;
+  for (int i = 0; i < G; ++i) sum = __dadd_rn(sum, (double)__shfl_sync(FULL, r, i));
+  const double mean = __ddiv_rn(sum, (double)G);
+  const double dist = act ? fabs(__dsub_rn((double)r, mean)) : -1.0;
+  // visiting position: |A| descending (|r - mean| descending), lower index first on ties
+  int rank = 0;
+  for (int j = 0; j < G; ++j) {
+    const double dj = __shfl_sync(FULL, dist, j);
+    rank += (dj > dist || (dj == dist && j < lane)) ? 1 : 0;
   }
-  // Eq. 8, greedily along the visiting order, inside each reward class.
-  int count = 0;
+  // same-class rollouts within tau of this one
+  uint32_t near = 0;
+  if (act) {
+    const uint8_t* row = w.close + ((int64_t)p * G + lane) * G;
+    for (int j = 0; j < G; ++j)
+      if (j != lane && row[j]) near |= 1u << j;
+  }
+  // Eq. 8, greedily along the visiting order
+  uint32_t kept = 0;
   for (int a = 0; a < G; ++a) {
-    const int i = order[a];
-    bool drop = false;
-    for (int b = 0; b < a && !drop; ++b) {
-      const int j = order[b];
-      if (!kept[j] || r[j] != r[i]) continue;
-      drop = too_close(inter[i * G + j], nu[i], nu[j], tau);
-    }
-    kept[i] = !drop;
-    count += kept[i] ? 1 : 0;
+    const int i = __ffs(__ballot_sync(FULL, act && rank == a)) - 1;
+    if ((__shfl_sync(FULL, near, i) & kept) == 0) kept |= 1u << i;
   }
-  // Per-prompt cap: classes (dist descending, then lowest member) take turns, each turn adding
-  // its next kept member in index order.
+  int count = __popc(kept);
+  // Per-prompt cap: classes take turns in visiting order of their lowest member; each turn adds
+  // the class's next kept member by index.  Equivalently keep the keep_cap kept rollouts with the
+  // smallest (turn, class position).
   if (count > keep_cap) {
-    int cls_first[kMaxG];  // class representative (its lowest index), in turn order
-    int ncls = 0;
-    for (int a = 0; a < G; ++a) {  // visiting order lists classes by (dist desc, first index)
-      const int i = order[a];
-      if (!kept[i]) continue;
-      bool seen = false;
-      for (int c = 0; c < ncls; ++c) seen |= (r[cls_first[c]] == r[i]);
-      if (!seen) cls_first[ncls++] = i;
+    const bool mine = act && ((kept >> lane) & 1u);
+    uint32_t cls = 0;  // kept rollouts of my class
+    for (int i = 0; i < G; ++i) {
+      const float ri = __shfl_sync(FULL, r, i);
+      const uint32_t m = __ballot_sync(FULL, act && ((kept >> lane) & 1u) && r == ri);
+      if (lane == i) cls = m;
     }
-    bool capped[kMaxG];
-    int next[kMaxG];  // per class: next index to look at
-    for (int i = 0; i < G; ++i) capped[i] = false;
-    for (int c = 0; c < ncls; ++c) next[c] = 0;
-    int taken = 0;
-    while (taken < keep_cap) {
-      for (int c = 0; c < ncls && taken < keep_cap; ++c) {
-        const float rc = r[cls_first[c]];
-        int i = next[c];
-        while (i < G && !(kept[i] && r[i] == rc)) ++i;
-        if (i < G) {
-          capped[i] = true;
-          ++taken;
-          next[c] = i + 1;
-        } else {
-          next[c] = G;
-        }
-      }
+    const int first = mine ? __ffs(cls) - 1 : 0;
+    const int turn = mine ? __popc(cls & ((1u << lane) - 1u)) : 0;
+    const int crank = __shfl_sync(FULL, rank, first);
+    const int key = turn * 64 + crank;
+    int before = 0;
+    for (int j = 0; j < G; ++j) {
+      const int kj = __shfl_sync(FULL, key, j);
+      before += (((kept >> j) & 1u) && kj < key) ? 1 : 0;
     }
-    for (int i = 0; i < G; ++i) kept[i] = capped[i];
+    kept = __ballot_sync(FULL, mine && before < keep_cap);
     count = keep_cap;
   }
-  for (int i = 0; i < G; ++i) keep[(int64_t)p * G + i] = kept[i] ? 1 : 0;
-  kept_per_prompt[p] = count;
+  if (act) keep[(int64_t)p * G + lane] = (kept >> lane) & 1u;
+  if (lane == 0) kept_per_prompt[p] = count;
 }
 
 __global__ void dp_fill_kernel(const float* __restrict__ rewards, int P, int G, int d,
@@ -335,28 +403,40 @@ extern "C" grpo_status grpo_prune(const float* rewards, const int32_t* ids, cons
   if (dp_divisor < 1) return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: dp_divisor = %d < 1", dp_divisor);
   if (tau != tau) return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: tau is NaN");
   bool query = false;
-  const grpo_status ws_ok = workspace_check(ws, ws_bytes, prune_ws_bytes(T, P, G), "grpo_prune", &query);
+  const grpo_status ws_ok =
+      workspace_check(ws, ws_bytes, prune_ws_bytes(T, P, G, V, ngram_n), "grpo_prune", &query);
   if (ws_ok != GRPO_OK || query) return ws_ok;
   if (P == 0) return GRPO_OK;
   if (!rewards || !off || !keep || !kept_per_prompt || (T > 0 && !ids))
     return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: NULL array");
   cudaStream_t s = as_stream(stream);
-  const PruneWs w = prune_ws(ws, T, P, G);
+  const PruneWs w = prune_ws(ws, T, P, G, V, ngram_n);
   const int nroll = P * G;
-  const int smem = kSmemKeys * 8;
-  if (cudaFuncSetAttribute(ngram_set_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
-      cudaSuccess)
-    return check_launch("grpo_prune: cudaFuncSetAttribute");
-  ngram_set_kernel<<<nroll, kSortThreads, smem, s>>>(ids, off, V, ngram_n, w, status);
-  int launches = 1;
-  const int64_t warps = (int64_t)P * (G * (G - 1) / 2);
-  if (warps > 0) {
-    const int tpb = 256;
-    const int64_t blocks = (warps * 32 + tpb - 1) / tpb;
-    intersect_kernel<<<(unsigned)blocks, tpb, 0, s>>>(rewards, off, P, G, w);
+  const int pairs = G * (G - 1) / 2;
+  int launches = 0;
+  if (ngram_n == 1) {
+    unigram_set_kernel<<<nroll, 256, (size_t)w.words * 8, s>>>(ids, off, V, w, status);
     ++launches;
+    if (pairs > 0) {
+      bitmap_pair_kernel<<<(unsigned)((int64_t)P * pairs), 128, 0, s>>>(rewards, G, tau, w);
+      ++launches;
+    }
+  } else {
+    const int smem = kSmemKeys * 8;
+    if (cudaFuncSetAttribute(ngram_set_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+        cudaSuccess)
+      return check_launch("grpo_prune: cudaFuncSetAttribute");
+    ngram_set_kernel<<<nroll, kSortThreads, smem, s>>>(ids, off, V, ngram_n, w, status);
+    ++launches;
+    if (pairs > 0) {
+      const int tpb = 256;
+      const int64_t blocks = ((int64_t)P * pairs * 32 + tpb - 1) / tpb;
+      sorted_pair_kernel<<<(unsigned)blocks, tpb, 0, s>>>(rewards, off, P, G, tau, w);
+      ++launches;
+    }
   }
-  select_kernel<<<(P + 127) / 128, 128, 0, s>>>(rewards, P, G, tau, keep_cap, w, keep, kept_per_prompt);
+  select_kernel<<<(unsigned)(((int64_t)P * 32 + 127) / 128), 128, 0, s>>>(rewards, P, G, keep_cap, w,
+                                                                          keep, kept_per_prompt);
   ++launches;
   if (dp_divisor > 1) {
     dp_fill_kernel<<<1, 32, 0, s>>>(rewards, P, G, dp_divisor, keep, kept_per_prompt);

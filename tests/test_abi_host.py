@@ -107,7 +107,12 @@ def test_workspace_queries_answer_without_a_device(grpo):
                         None, ctypes.byref(size), None) == 0
     def up(x):
         return (x + 255) // 256 * 256
-    assert size.value == up(2 * 5000 * 8) + up(16 * 8 * 4) + up(16 * 8 * 8 * 4)
+    # bigrams: sorted keys (2T u64), set sizes, one byte per ordered pair
+    assert size.value == up(2 * 5000 * 8) + up(16 * 8 * 4) + up(16 * 8 * 8)
+    assert L.grpo_prune(None, None, None, 16, 8, 5000, 152064, 1, 0.8, 4, 1, None, None, None,
+                        None, ctypes.byref(size), None) == 0
+    # unigrams: a vocabulary bitmap per rollout instead of keys
+    assert size.value == up(16 * 8 * ((152064 + 63) // 64) * 8) + up(16 * 8 * 4) + up(16 * 8 * 8)
     assert loss_call(L, 1000, 152064, None, ctypes.byref(size)) == 0
     assert size.value == up(1000 * 8)
     # with a row-loss output the loss needs no workspace
