@@ -382,6 +382,30 @@ def main():
                 "algorithmic_bytes_per_launch": step.T_kept * bytes_per_row,
                 "launch_ms": loss_ms, "peak_source": peak_src}
 
+    # the logp-only forward over the same kept rows (old/reference policy evaluation); one read
+    logp_fwd = None
+    if w.chunk_rows == 0:
+        lp_out = torch.empty(max(step.T_kept, 1), dtype=torch.float32, device=dev)
+        rows_src = step.src_token[:step.T_kept]
+        for _ in range(3):
+            g.grpo_logp_fwd(d["logits"], d["ids"], row_index=rows_src, n_rows=step.T_kept,
+                            logp_out=lp_out)
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        nrep = 20
+        f0.record(stream)
+        for _ in range(nrep):
+            g.grpo_logp_fwd(d["logits"], d["ids"], row_index=rows_src, n_rows=step.T_kept,
+                            logp_out=lp_out)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        f_ms = f0.elapsed_time(f1) / nrep
+        f_bytes = step.T_kept * (w.V * w.in_bytes + 16)
+        logp_fwd = {"kernel": "grpo_loss_kernel<..., forward only>", "launch_ms": f_ms,
+                    "achieved": f_bytes / (f_ms / 1e3) / 1e9, "unit": "GB/s",
+                    "frac": f_bytes / (f_ms / 1e3) / 1e9 / peak,
+                    "kept_tokens_per_s": step.T_kept / (f_ms / 1e3),
+                    "algorithmic_bytes_per_launch": f_bytes}
+
     # end to end: inputs copied from pinned host memory, loss read back, inside the timed region
     e2e = None
     names = ["rewards", "ids", "off", "logits", "old", "ref"]
@@ -429,7 +453,7 @@ def main():
             "data": "synthetic (seeded; shapes and distributions of the paper's GRPO batches)",
             "config": workload_desc(w, b["T"], step.T_kept, step.K),
             "gpu_launches": int(launches), "roofline": roofline, "e2e": e2e,
-            "cpu_baseline": cpu, "clocks": clocks,
+            "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd,
             "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,
         }
         print(json.dumps(line), flush=True)

@@ -179,6 +179,20 @@ grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t 
                               grpo_stream_t stream);
 
 /*
+ * grpo_logp_fwd — log-probability of the sampled token alone, for the old- and reference-policy
+ * evaluations over the kept trajectories (Sec. 3.2: the retained trajectories go through the old,
+ * current and reference models; logits -> softmax over the vocabulary -> token probability):
+ *   logp_out[t] = z_y - log sum_v exp(z_v),  z = logits row src, y = y[src], src = row_index[t]
+ *   (or t when row_index is NULL).  One read of the logits, no gradient, no loss.
+ * logits, row_stride, row_index, y: as grpo_loss_fwd_bwd.  logp_out device f32 [n_rows].
+ * status: device i32, nullable (GRPO_DEVFLAG_BAD_TOKEN leaves logp = NaN, GRPO_DEVFLAG_NONFINITE).
+ * Limits: as grpo_loss_fwd_bwd.  No workspace.
+ */
+grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
+                          const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
+                          float* logp_out, int32_t* status, grpo_stream_t stream);
+
+/*
  * grpo_sum_f64 — *out = v[0] + ... + v[n-1] in fp64, in the same fixed order grpo_loss_fwd_bwd
  * uses for loss_out (bitwise reproducible).  With row_loss_out, a loss computed over rows in
  * several calls (for example chunks of kept rows sharing one dlogits buffer) then sums to

@@ -40,6 +40,8 @@ def lib():
                                   _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p,
                                   _c_p, _c_p, _c_p, _c_p]
         L.oracle_loss.restype = _i32
+        L.oracle_logp.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p]
+        L.oracle_logp.restype = _i32
         L.oracle_round_bf16.argtypes = [_f64]
         L.oracle_round_bf16.restype = ctypes.c_uint16
         L.oracle_ars_new.argtypes = [_i32]
@@ -162,6 +164,24 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
         raise ValueError("oracle_loss: bad arguments")
     return dict(loss=float(total[0]), logp=logp[:n_rows], rho=rho[:n_rows], row_loss=rl[:n_rows],
                 dlogits=dl, dlogits_f64=d64)
+
+
+def logp(logits, V: int, y, *, row_index=None, n_rows=None, row_stride=None, logits_dtype=None):
+    """log pi(y) per row: the old/reference policy evaluation.  Returns f64 [n_rows]."""
+    lg = np.ascontiguousarray(logits)
+    if logits_dtype is None:
+        logits_dtype = 1 if lg.dtype == np.uint16 else 0
+    if logits_dtype == 0:
+        lg = lg.astype(np.float32, copy=False)
+    stride = V if row_stride is None else int(row_stride)
+    ri = None if row_index is None else _arr(row_index, np.int64)
+    if n_rows is None:
+        n_rows = ri.size if ri is not None else lg.size // stride
+    y_ = _arr(y, np.int32)
+    out = np.empty(max(n_rows, 1), np.float64)
+    if lib().oracle_logp(_p(lg), logits_dtype, stride, _p(ri), n_rows, V, _p(y_), _p(out)) != 0:
+        raise ValueError("oracle_logp: bad arguments")
+    return out[:n_rows]
 
 
 def round_bf16(x) -> np.ndarray:

@@ -157,3 +157,28 @@ extern "C" int oracle_loss(const void* logits, int logits_dtype, int64_t row_str
   if (loss_out) *loss_out = total;
   return 0;
 }
+
+// Per-token log-probability alone (the old- and reference-policy evaluations of Sec. 3.2: logits
+// -> softmax over the vocabulary -> probability of the sampled token): logp = z_y - log sum exp z.
+extern "C" int oracle_logp(const void* logits, int logits_dtype, int64_t row_stride,
+                           const int64_t* row_index, int64_t n_rows, int V, const int32_t* y,
+                           double* logp_out) {
+  if (n_rows < 0 || V < 1 || row_stride < V) return 1;
+  const double nan = std::numeric_limits<double>::quiet_NaN();
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t t = 0; t < n_rows; ++t) {
+    const int64_t src = row_index ? row_index[t] : t;
+    const int64_t base = src * row_stride;
+    const int32_t yt = y[src];
+    if (yt < 0 || yt >= V) {
+      logp_out[t] = nan;
+      continue;
+    }
+    double m = -std::numeric_limits<double>::infinity();
+    for (int v = 0; v < V; ++v) m = std::fmax(m, load_logit(logits, logits_dtype, base + v));
+    double s = 0.0;
+    for (int v = 0; v < V; ++v) s += std::exp(load_logit(logits, logits_dtype, base + v) - m);
+    logp_out[t] = load_logit(logits, logits_dtype, base + yt) - (m + std::log(s));
+  }
+  return 0;
+}

@@ -48,6 +48,10 @@ int oracle_loss(const void* logits, int logits_dtype, int64_t row_stride, const 
                 double* dlogits_f64, double* logp_out, double* rho_out, double* row_loss_out,
                 double* loss_out);
 
+/* logp of the sampled token alone (old/reference policy evaluation); NaN for ids outside [0,V). */
+int oracle_logp(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
+                int64_t n_rows, int V, const int32_t* y, double* logp_out);
+
 /* Round an fp64 value to bf16 (nearest, ties to even, bf16 subnormals kept); returns the bits. */
 uint16_t oracle_round_bf16(double x);
 

@@ -31,7 +31,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64",
+           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
            "grpo_loss_tune", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -86,6 +86,8 @@ def lib():
                                             _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64,
                                             _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p]
     L.grpo_loss_fwd_bwd_noalloc.restype = _i32
+    L.grpo_logp_fwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p]
+    L.grpo_logp_fwd.restype = _i32
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
     L.grpo_sum_f64.restype = _i32
     L.grpo_loss_tune.argtypes = [_i32, _i32, _i32]
@@ -351,6 +353,35 @@ def grpo_loss_fwd_bwd_noalloc(logits, y, old_logp, ref_logp, adv, row_rollout, *
         float(beta), int(agg_mode), int(denom_tokens), _ptr(seq_off), int(n_seq), _ptr(dlogits),
         odt, _ptr(logp_out), _ptr(row_loss_out), _ptr(loss_out), _ptr(status), _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out)
+
+
+def grpo_logp_fwd(logits, y, *, V: int | None = None, row_stride: int | None = None,
+                  row_index=None, n_rows: int | None = None, logp_out=None, status=None,
+                  stream=None):
+    """log pi(y) of each row on the GPU (old/reference policy evaluation).  Returns logp f32."""
+    torch = _torch()
+    if logits.dtype == torch.bfloat16:
+        ldt = GRPO_DTYPE_BF16
+    elif logits.dtype == torch.float32:
+        ldt = GRPO_DTYPE_F32
+    else:
+        raise TypeError("logits must be bf16 or f32")
+    if logits.dim() != 2 or logits.stride(1) != 1 or not logits.is_cuda:
+        raise ValueError("logits must be a 2-D CUDA tensor with unit stride along the vocabulary")
+    if V is None:
+        V = logits.shape[1]
+    stride = logits.stride(0) if row_stride is None else int(row_stride)
+    if n_rows is None:
+        n_rows = row_index.numel() if row_index is not None else logits.shape[0]
+    _need(y, torch.int32, None, "y")
+    if row_index is not None:
+        _need(row_index, torch.int64, n_rows, "row_index")
+    if logp_out is None:
+        logp_out = torch.empty(max(int(n_rows), 1), dtype=torch.float32, device=logits.device)
+    _need(logp_out, torch.float32, n_rows, "logp_out")
+    _check(lib().grpo_logp_fwd(_ptr(logits), ldt, stride, _ptr(row_index), int(n_rows), int(V),
+                               _ptr(y), _ptr(logp_out), _ptr(status), _stream(stream)))
+    return logp_out
 
 
 def grpo_sum_f64(v, n: int | None = None, out=None, stream=None):

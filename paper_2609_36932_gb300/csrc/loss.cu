@@ -258,7 +258,9 @@ __device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float 
 
 // ---- the kernel -------------------------------------------------------------------------------
 
-template <typename InT, typename OutT, int kThreads>
+// kBwd = false: forward only (log-probabilities of the sampled tokens, no gradient, no loss);
+// each chunk is refilled with the next row as soon as the CTA has reduced its slice.
+template <typename InT, typename OutT, int kThreads, bool kBwd>
 __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
   constexpr int kPairs = Fmt<InT>::kPairs;
@@ -420,6 +422,13 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
         st_async_f4(mapa_shared(dst, lane), make_float4(m, s, zy, 0.f),
                     mapa_shared(xbar_s + 8 * slot, lane));
       }
+      if constexpr (!kBwd) {  // forward only: the slice is consumed; fetch the next row now
+        __syncwarp();
+        if (lane == 0 && row + ncl < a.n_rows && !*(volatile int*)abort_flag) {
+          const char* g = row_base(row + ncl);
+          for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
+        }
+      }
     }
 
     // ---- exchange and row scalars (warp 0) ----
@@ -443,7 +452,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
         if (!yvalid) {
           if (rank == 0) {
             if (a.logp_out) a.logp_out[row] = __int_as_float(0x7fc00000);
-            a.row_loss[row] = 0.0;
+            if (kBwd) a.row_loss[row] = 0.0;
             if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
           }
         } else {
@@ -452,6 +461,12 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           const float ey = expf(zy - M);
           const float S = S_excl + ey;
           const float logp = (zy - M) - logf(S);
+          if constexpr (!kBwd) {
+            if (rank == 0) {
+              a.logp_out[row] = logp;
+              if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
+            }
+          } else {
           // Eq. 1: ratio, clipped surrogate, KL term; Eqs. 2-3: gradient coefficient.
           const float A = a.adv[a.row_rollout[row]];
           const float rho = expf(logp - a.old_logp[src]);
@@ -483,6 +498,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
             a.row_loss[row] = (a.agg_mode == 0 ? a.inv_denom : (double)w) * (double)ell;
             if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
           }
+          }  // kBwd
         }
         rowsc[0] = neg_scale;
         rowsc[1] = dy;
@@ -490,6 +506,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
         rowsc[3] = yvalid ? 0.f : 1.f;
       }
     }
+    if constexpr (kBwd) {
     __syncthreads();
 
     // ---- pass B: dlogits from the shared-memory slice; refill chunk by chunk ----
@@ -540,6 +557,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
       __syncthreads();  // chunk k consumed by every thread
       if (gnext && !*(volatile int*)abort_flag) issue_chunk(gnext, k);
     }
+    }  // kBwd
   }
   cluster_sync();  // partners are done reading this CTA's shared memory
 }
@@ -568,13 +586,18 @@ std::map<std::tuple<const void*, int, int, int>, int> g_max_clusters;  // (kerne
 
 using KernelFn = void (*)(LossArgs);
 
-template <typename InT, typename OutT>
+template <typename InT, typename OutT, bool kBwd = true>
 KernelFn pick_kernel(int threads) {
   switch (threads) {
-    case 128: return grpo_loss_kernel<InT, OutT, 128>;
-    case 512: return grpo_loss_kernel<InT, OutT, 512>;
-    default: return grpo_loss_kernel<InT, OutT, 256>;
+    case 128: return grpo_loss_kernel<InT, OutT, 128, kBwd>;
+    case 512: return grpo_loss_kernel<InT, OutT, 512, kBwd>;
+    default: return grpo_loss_kernel<InT, OutT, 256, kBwd>;
   }
+}
+
+KernelFn fwd_kernel_for(int in_dtype, int threads) {
+  return in_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16, false>(threads)
+                                     : pick_kernel<float, float, false>(threads);
 }
 
 KernelFn kernel_for(int in_dtype, int out_dtype, int threads) {
@@ -583,6 +606,111 @@ KernelFn kernel_for(int in_dtype, int out_dtype, int threads) {
                                         : pick_kernel<__nv_bfloat16, float>(threads);
   return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<float, __nv_bfloat16>(threads)
                                       : pick_kernel<float, float>(threads);
+}
+
+// Launch shape of the row kernel for a vocabulary of V entries of in_bytes each.
+struct Shape {
+  int C = 1, threads = 256, slice = 0, chunk_vecs = 0, chunks = 1;
+  size_t smem = 0;
+};
+
+grpo_status pick_shape(int V, int in_bytes, const char* who, Shape* out) {
+  Tune tune;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    tune = g_tune;
+  }
+  const int vec = 16 / in_bytes;
+  const int threads = tune.threads ? tune.threads : 256;
+  // Cluster size: slices of at most 80 KiB (two CTAs per SM), and at least two CTAs per row once
+  // a row exceeds 32 KiB.  Measured on GB300 over cluster sizes 1-16, 128-512 threads and 1-5
+  // copies per slice, this shape moved the most bytes per second for V = 32000 and 152064.
+  int C = tune.cluster;
+  if (C == 0) {
+    const int64_t row_bytes = (int64_t)V * in_bytes;
+    C = (int)std::min<int64_t>(kMaxCluster, (row_bytes + 80 * 1024 - 1) / (80 * 1024));
+    if (C == 1 && row_bytes > 32 * 1024) C = 2;
+  }
+  int slice = (int)align_up((size_t)((V + C - 1) / C), vec);
+  while (C > 1 && (int64_t)(C - 1) * slice >= V) {  // no empty slices
+    --C;
+    slice = (int)align_up((size_t)((V + C - 1) / C), vec);
+  }
+  const size_t slice_bytes = (size_t)slice * in_bytes;
+  // about 36 KiB per bulk copy
+  int chunks = tune.chunks ? tune.chunks
+                           : (int)std::min<size_t>(kMaxChunks, std::max<size_t>(1, (slice_bytes + 18 * 1024) / (36 * 1024)));
+  const int slice_vecs = slice / vec;
+  int chunk_vecs = (slice_vecs + chunks - 1) / chunks;
+  if (chunk_vecs < 1) chunk_vecs = 1;
+  // whole vectors per thread in every chunk but the last one
+  const int even = (chunk_vecs + threads - 1) / threads * threads;
+  if (even <= slice_vecs) chunk_vecs = even;
+  chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
+  if (chunks < 1) chunks = 1;
+  if (chunks > kMaxChunks) {
+    chunk_vecs = (slice_vecs + kMaxChunks - 1) / kMaxChunks;
+    chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
+  }
+  const size_t smem = align_up(slice_bytes, 128) + kMaxChunks * 8 + 2 * 8 + 2 * kMaxCluster * 16 +
+                      2 * (threads / 32) * 4 + 4 * 4 + 16;
+  if (smem > 227 * 1024)
+    return fail(GRPO_ERR_UNSUPPORTED, "%s: V = %d needs %zu bytes of shared memory per CTA at %d CTAs", who,
+                V, smem, C);
+  out->C = C;
+  out->threads = threads;
+  out->slice = slice;
+  out->chunk_vecs = chunk_vecs;
+  out->chunks = chunks;
+  out->smem = smem;
+  return GRPO_OK;
+}
+
+// Persistent cluster launch: as many clusters as can be resident, at most one per row.
+grpo_status launch_rows(KernelFn fn, const Shape& sh, LossArgs a, cudaStream_t s, const char* who) {
+  a.slice = sh.slice;
+  a.chunk_vecs = sh.chunk_vecs;
+  a.n_chunks = sh.chunks;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh.smem);
+  if (e == cudaSuccess && sh.C > 8)
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = sh.C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(sh.threads, 1, 1);
+  cfg.dynamicSmemBytes = sh.smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int max_cl = 0;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    const auto key = std::make_tuple((const void*)fn, dev, sh.C, (int)sh.smem);
+    auto it = g_max_clusters.find(key);
+    if (it != g_max_clusters.end()) {
+      max_cl = it->second;
+    } else {
+      cfg.gridDim = dim3(sh.C, 1, 1);
+      e = cudaOccupancyMaxActiveClusters(&max_cl, fn, &cfg);
+      if (e != cudaSuccess)
+        return fail(GRPO_ERR_CUDA, "%s: cudaOccupancyMaxActiveClusters: %s", who, cudaGetErrorString(e));
+      if (max_cl < 1)
+        return fail(GRPO_ERR_UNSUPPORTED, "%s: a cluster of %d CTAs with %zu bytes each cannot be resident",
+                    who, sh.C, sh.smem);
+      g_max_clusters[key] = max_cl;
+    }
+  }
+  const int64_t n_clusters = std::min<int64_t>(a.n_rows, max_cl);
+  cfg.gridDim = dim3((unsigned)(n_clusters * sh.C), 1, 1);
+  e = cudaLaunchKernelEx(&cfg, fn, a);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: launch: %s", who, cudaGetErrorString(e));
+  return GRPO_OK;
 }
 
 }  // namespace
@@ -654,52 +782,13 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   if (!logits || !y || !old_logp || !ref_logp || !adv || !row_rollout || !dlogits)
     return fail(GRPO_ERR_INVALID_ARG, "%s: NULL array", who);
 
-  Tune tune;
-  {
-    std::lock_guard<std::mutex> lk(g_mu);
-    tune = g_tune;
-  }
   const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   const int out_bytes = dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
-  const int vec = 16 / in_bytes;
-  const int threads = tune.threads ? tune.threads : 256;
-  // Cluster size: slices of at most 80 KiB (two CTAs per SM), and at least two CTAs per row once
-  // a row exceeds 32 KiB.  Measured on GB300 over cluster sizes 1-16, 128-512 threads and 1-5
-  // copies per slice, this shape moved the most bytes per second for V = 32000 and 152064.
-  int C = tune.cluster;
-  if (C == 0) {
-    const int64_t row_bytes = (int64_t)V * in_bytes;
-    C = (int)std::min<int64_t>(kMaxCluster, (row_bytes + 80 * 1024 - 1) / (80 * 1024));
-    if (C == 1 && row_bytes > 32 * 1024) C = 2;
-  }
-  int slice = (int)align_up((size_t)((V + C - 1) / C), vec);
-  while (C > 1 && (int64_t)(C - 1) * slice >= V) {  // no empty slices
-    --C;
-    slice = (int)align_up((size_t)((V + C - 1) / C), vec);
-  }
-  const size_t slice_bytes = (size_t)slice * in_bytes;
-  // about 36 KiB per bulk copy
-  int chunks = tune.chunks ? tune.chunks
-                           : (int)std::min<size_t>(kMaxChunks, std::max<size_t>(1, (slice_bytes + 18 * 1024) / (36 * 1024)));
-  const int slice_vecs = slice / vec;
-  int chunk_vecs = (slice_vecs + chunks - 1) / chunks;
-  if (chunk_vecs < 1) chunk_vecs = 1;
-  // whole vectors per thread in every chunk but the last one
-  const int even = (chunk_vecs + threads - 1) / threads * threads;
-  if (even <= slice_vecs) chunk_vecs = even;
-  chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
-  if (chunks < 1) chunks = 1;
-  if (chunks > kMaxChunks) {
-    chunk_vecs = (slice_vecs + kMaxChunks - 1) / kMaxChunks;
-    chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
-  }
-  const size_t smem = align_up(slice_bytes, 128) + kMaxChunks * 8 + 2 * 8 + 2 * kMaxCluster * 16 +
-                      2 * (threads / 32) * 4 + 4 * 4 + 16;
-  if (smem > 227 * 1024)
-    return fail(GRPO_ERR_UNSUPPORTED, "%s: V = %d needs %zu bytes of shared memory per CTA at %d CTAs", who,
-                V, smem, C);
+  Shape sh;
+  st = pick_shape(V, in_bytes, who, &sh);
+  if (st != GRPO_OK) return st;
 
-  LossArgs a;
+  LossArgs a = {};
   a.logits = static_cast<const char*>(logits);
   a.row_stride_bytes = row_stride * in_bytes;
   a.row_index = row_index;
@@ -728,57 +817,48 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   a.logp_out = logp_out;
   a.row_loss = row_loss;
   a.status = status;
-  a.slice = slice;
-  a.chunk_vecs = chunk_vecs;
-  a.n_chunks = chunks;
   a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
   a.out_vec = (reinterpret_cast<uintptr_t>(dlogits) % 16 == 0) && (((int64_t)V * out_bytes) % 16 == 0);
 
-  KernelFn fn = kernel_for(logits_dtype, dlogits_dtype, threads);
-  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess && C > 8)
-    e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
-
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = C;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cudaLaunchConfig_t cfg = {};
-  cfg.blockDim = dim3(threads, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-
-  int dev = 0;
-  cudaGetDevice(&dev);
-  int max_cl = 0;
-  {
-    std::lock_guard<std::mutex> lk(g_mu);
-    const auto key = std::make_tuple((const void*)fn, dev, C, (int)smem);
-    auto it = g_max_clusters.find(key);
-    if (it != g_max_clusters.end()) {
-      max_cl = it->second;
-    } else {
-      cfg.gridDim = dim3(C, 1, 1);
-      e = cudaOccupancyMaxActiveClusters(&max_cl, fn, &cfg);
-      if (e != cudaSuccess)
-        return fail(GRPO_ERR_CUDA, "%s: cudaOccupancyMaxActiveClusters: %s", who, cudaGetErrorString(e));
-      if (max_cl < 1)
-        return fail(GRPO_ERR_UNSUPPORTED, "%s: a cluster of %d CTAs with %zu bytes each cannot be resident",
-                    who, C, smem);
-      g_max_clusters[key] = max_cl;
-    }
-  }
-  const int64_t n_clusters = std::min<int64_t>(n_rows, max_cl);
-  cfg.gridDim = dim3((unsigned)(n_clusters * C), 1, 1);
-  e = cudaLaunchKernelEx(&cfg, fn, a);
-  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: launch: %s", who, cudaGetErrorString(e));
+  st = launch_rows(kernel_for(logits_dtype, dlogits_dtype, sh.threads), sh, a, s, who);
+  if (st != GRPO_OK) return st;
   sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, n_rows, loss_out);
   count_launches(2);
   return check_launch(who);
+}
+
+extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
+                                     const int64_t* row_index, int64_t n_rows, int32_t V,
+                                     const int32_t* y, float* logp_out, int32_t* status,
+                                     grpo_stream_t stream) {
+  clear_error();
+  const char* who = "grpo_logp_fwd";
+  if (logits_dtype != GRPO_DTYPE_BF16 && logits_dtype != GRPO_DTYPE_F32)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: logits_dtype = %d", who, logits_dtype);
+  if (n_rows < 0 || n_rows >= (int64_t(1) << 31))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: n_rows = %lld", who, (long long)n_rows);
+  if (V < 1 || row_stride < V)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: V = %d, row_stride = %lld", who, V, (long long)row_stride);
+  if (n_rows == 0) return GRPO_OK;
+  if (!logits || !y || !logp_out) return fail(GRPO_ERR_INVALID_ARG, "%s: NULL array", who);
+  const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+  Shape sh;
+  grpo_status st = pick_shape(V, in_bytes, who, &sh);
+  if (st != GRPO_OK) return st;
+  LossArgs a = {};
+  a.logits = static_cast<const char*>(logits);
+  a.row_stride_bytes = row_stride * in_bytes;
+  a.row_index = row_index;
+  a.n_rows = n_rows;
+  a.V = V;
+  a.y = y;
+  a.logp_out = logp_out;
+  a.status = status;
+  a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
+  st = launch_rows(fwd_kernel_for(logits_dtype, sh.threads), sh, a, as_stream(stream), who);
+  if (st != GRPO_OK) return st;
+  count_launches(1);
+  return GRPO_OK;
 }
 
 // ---- allocation-free variant ------------------------------------------------------------------

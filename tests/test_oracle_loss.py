@@ -168,3 +168,25 @@ def test_round_bf16(oracle_mod):
     assert oracle_mod.round_bf16(np.array([1.0 + 2.0 ** -8 + 2.0 ** -40]))[0] == 0x3F81
     assert oracle_mod.round_bf16(np.array([1.0 + 2.0 ** -8]))[0] == 0x3F80
     assert oracle_mod.round_bf16(np.array([float("inf"), float("nan")])).tolist()[0] == 0x7F80
+
+
+def test_logp_only_matches_library_logsumexp_and_the_loss(oracle_mod):
+    """oracle_logp is the plain z_y - logsumexp(z); it agrees with scipy and with the logp the
+    loss reports, including gathered rows and invalid ids."""
+    rng = np.random.default_rng(17)
+    for V, scale in ((5, 1.0), (3000, 4.0)):
+        z = rows(rng, 9, V, scale)
+        y = rng.integers(0, V, size=9).astype(np.int32)
+        y[4] = V  # invalid
+        idx = np.array([8, 0, 4, 3], np.int64)
+        got = oracle_mod.logp(z, V, y, row_index=idx)
+        zz = z.astype(np.float64)
+        for k, r in enumerate(idx):
+            if y[r] >= V:
+                assert math.isnan(got[k])
+            else:
+                assert got[k] == pytest.approx(zz[r, y[r]] - scipy.special.logsumexp(zz[r]), abs=1e-12)
+        yl = np.where(y >= V, 0, y).astype(np.int32)
+        lo = oracle_mod.loss(z, V, yl, np.zeros(9, np.float32), np.zeros(9, np.float32),
+                             np.zeros(1, np.float32), np.zeros(9, np.int32), want_dlogits=False)
+        np.testing.assert_array_equal(oracle_mod.logp(z, V, yl), lo["logp"])
