@@ -88,13 +88,19 @@ grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G, int32_t s
  * the set of distinct n-grams of a completion.  Two rollouts that both have no n-gram
  * (length < n) have theta = 0.  The kept set is S(q), the union over classes (Eq. 9).
  * Then, if |S(q)| > keep_cap, keep_cap rollouts are kept by round-robin over the classes
- * (classes ordered by |r - mean| descending, then by lowest member index; each round takes each
- * class's next kept rollout, lowest index first).  keep_cap >= G disables the cap (the paper's
- * rule).  Finally, while the total kept count is not a multiple of dp_divisor, prompts are
+ * (classes ordered by the visiting position of their first member; each round takes each
+ * class's next kept rollout in visiting order, which for equal rewards is the lowest index).
+ * keep_cap >= G disables the cap (the paper's rule).  Finally, while the total kept count is not a multiple of dp_divisor, prompts are
  * visited cyclically from prompt 0 and each visit adds that prompt's unkept rollout with the
  * largest |r - mean| (lowest index on ties); prompts with none left are skipped (Algorithm 1,
  * DP alignment).  dp_divisor = 1 does nothing.
  * rewards          device f32 [P*G].
+ * adv, class_eps   class_eps = 0: classes by exact reward equality (adv may be NULL).
+ *                  class_eps > 0: the continuous-reward grouping of the paper's grounding
+ *                  extension, |A_i - A_j| < class_eps (the paper uses 1e-4), closed under
+ *                  transitivity: with the advantages adv (device f32 [P*G], e.g. grpo_advantage's)
+ *                  sorted ascending (ties by index), a new class starts wherever the gap to the
+ *                  previous value is >= class_eps (differences in fp64).
  * ids              device i32 [T]: completion token ids of all rollouts, packed.
  * off              device i64 [P*G+1]: rollout r owns ids[off[r] .. off[r+1]); off[0] = 0,
  *                  off[P*G] = T, non-decreasing.
@@ -109,11 +115,11 @@ grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G, int32_t s
  * ws, ws_bytes     workspace (see conventions); its size depends on T, P and G.
  * Limits: 1 <= G <= 32; 1 <= V <= 2^18 (three 18-bit ids fit one 64-bit n-gram key).
  */
-grpo_status grpo_prune(const float* rewards, const int32_t* ids, const int64_t* off,
-                       int32_t P, int32_t G, int64_t T, int32_t V, int32_t ngram_n, float tau,
-                       int32_t keep_cap, int32_t dp_divisor, uint8_t* keep,
-                       int32_t* kept_per_prompt, int32_t* status, void* ws, size_t* ws_bytes,
-                       grpo_stream_t stream);
+grpo_status grpo_prune(const float* rewards, const float* adv, float class_eps, const int32_t* ids,
+                       const int64_t* off, int32_t P, int32_t G, int64_t T, int32_t V,
+                       int32_t ngram_n, float tau, int32_t keep_cap, int32_t dp_divisor,
+                       uint8_t* keep, int32_t* kept_per_prompt, int32_t* status, void* ws,
+                       size_t* ws_bytes, grpo_stream_t stream);
 
 /*
  * grpo_compact — token compaction of the kept rollouts (Sec. 3.2: only retained trajectories

@@ -32,6 +32,9 @@ def lib():
         L.oracle_advantage.restype = _i32
         L.oracle_prune.argtypes = [_c_p, _c_p, _c_p, _i32, _i32, _i32, _f32, _i32, _i32, _c_p, _c_p]
         L.oracle_prune.restype = _i32
+        L.oracle_prune_classes.argtypes = [_c_p, _c_p, _f32, _c_p, _c_p, _i32, _i32, _i32, _f32,
+                                           _i32, _i32, _c_p, _c_p]
+        L.oracle_prune_classes.restype = _i32
         L.oracle_jaccard_distance.argtypes = [_c_p, _c_p, _i32, _i32, _i32]
         L.oracle_jaccard_distance.restype = _f64
         L.oracle_compact.argtypes = [_c_p, _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p]
@@ -83,8 +86,9 @@ def advantage(rewards, G: int, std_mode: int = 0):
 
 
 def prune(rewards, ids, off, G: int, ngram_n: int = 1, tau: float = 0.8, keep_cap=None,
-          dp_divisor: int = 1):
-    """Eqs. 6-9 + Algorithm 1.  Returns (keep u8 [P*G], kept_per_prompt i32 [P])."""
+          dp_divisor: int = 1, adv=None, class_eps: float = 0.0):
+    """Eqs. 6-9 + Algorithm 1.  Returns (keep u8 [P*G], kept_per_prompt i32 [P]).
+    class_eps > 0 (with adv) groups by chained advantages (the continuous-reward extension)."""
     r = _arr(rewards, np.float32)
     P = r.size // G
     ids_ = _arr(ids, np.int32)
@@ -92,8 +96,14 @@ def prune(rewards, ids, off, G: int, ngram_n: int = 1, tau: float = 0.8, keep_ca
     keep = np.zeros(P * G, np.uint8)
     kpp = np.zeros(max(P, 1), np.int32)
     cap = G if keep_cap is None else int(keep_cap)
-    if lib().oracle_prune(_p(r), _p(ids_), _p(off_), P, G, ngram_n, float(tau), cap, dp_divisor,
-                          _p(keep), _p(kpp)) != 0:
+    a = None if adv is None else _arr(adv, np.float32)
+    if class_eps > 0 or a is not None:
+        rc = lib().oracle_prune_classes(_p(r), _p(a), float(class_eps), _p(ids_), _p(off_), P, G,
+                                        ngram_n, float(tau), cap, dp_divisor, _p(keep), _p(kpp))
+    else:
+        rc = lib().oracle_prune(_p(r), _p(ids_), _p(off_), P, G, ngram_n, float(tau), cap,
+                                dp_divisor, _p(keep), _p(kpp))
+    if rc != 0:
         raise ValueError("oracle_prune: bad arguments")
     return keep, kpp[:P]
 

@@ -14,9 +14,14 @@
 //  - Eq. 7's n is not given; it is a parameter.  N_n(o) holds the distinct length-n windows of
 //    the completion's token ids.  Two completions that both have no window are identical, so
 //    their distance is 0.
+//  - Continuous rewards (the grounding extension): two trajectories share an advantage group
+//    when |A_i - A_j| < eps.  That relation is not transitive; its transitive closure is taken:
+//    sorted by A, a new class starts wherever the gap to the previous value is >= eps.  With
+//    class_eps = 0 the classes are the exact-equality classes above.
 //  - The per-prompt cap (keep_cap) is not in the paper; keep_cap >= G leaves Eq. 9's set as is.
-//    Above the cap, classes take turns (ordered by |r - mean| descending, then by lowest
-//    member) and each turn adds the class's next kept member, lowest index first.
+//    Above the cap, classes take turns (ordered by the visiting position of their first visited
+//    member) and each turn adds the class's next kept member in visiting order (for classes of
+//    equal rewards: lowest index first).
 //  - DP alignment "adds the unselected trajectory with the highest |A_i| via round-robin":
 //    prompts are visited cyclically from prompt 0; each visit adds that prompt's unselected
 //    rollout with the largest |r - mean| (lower index on ties); prompts with none are skipped.
@@ -77,13 +82,58 @@ extern "C" double oracle_jaccard_distance(const int32_t* ids, const int64_t* off
   return jaccard_distance(a, b);
 }
 
+// Class of each rollout of a group: exact reward equality, or chains of sorted advantages whose
+// consecutive gaps are below class_eps.  Returns the class label (its smallest member index).
+static std::vector<int> classes_of(const float* r, const float* a, int G, float class_eps) {
+  std::vector<int> cls(G);
+  if (class_eps <= 0.0f) {
+    for (int i = 0; i < G; ++i) {
+      cls[i] = i;
+      for (int j = 0; j < i; ++j)
+        if (r[j] == r[i]) {
+          cls[i] = j;
+          break;
+        }
+    }
+    return cls;
+  }
+  std::vector<int> by_a(G);
+  for (int i = 0; i < G; ++i) by_a[i] = i;
+  std::stable_sort(by_a.begin(), by_a.end(), [&](int x, int y) { return a[x] < a[y]; });
+  std::vector<int> chain(G);
+  int c = 0;
+  for (int k = 0; k < G; ++k) {
+    if (k > 0 && (double)a[by_a[k]] - (double)a[by_a[k - 1]] >= (double)class_eps) ++c;
+    chain[by_a[k]] = c;
+  }
+  for (int i = 0; i < G; ++i) {
+    cls[i] = i;
+    for (int j = 0; j < i; ++j)
+      if (chain[j] == chain[i]) {
+        cls[i] = j;
+        break;
+      }
+  }
+  return cls;
+}
+
 extern "C" int oracle_prune(const float* rewards, const int32_t* ids, const int64_t* off, int P,
                             int G, int ngram_n, float tau, int keep_cap, int dp_divisor,
                             uint8_t* keep, int32_t* kept_per_prompt) {
+  return oracle_prune_classes(rewards, nullptr, 0.0f, ids, off, P, G, ngram_n, tau, keep_cap,
+                              dp_divisor, keep, kept_per_prompt);
+}
+
+extern "C" int oracle_prune_classes(const float* rewards, const float* adv, float class_eps,
+                                    const int32_t* ids, const int64_t* off, int P, int G,
+                                    int ngram_n, float tau, int keep_cap, int dp_divisor,
+                                    uint8_t* keep, int32_t* kept_per_prompt) {
   if (P < 0 || G < 1 || ngram_n < 1 || keep_cap < 1 || dp_divisor < 1) return 1;
+  if (class_eps > 0.0f && adv == nullptr) return 1;
   std::vector<Group> groups(P);
   for (int p = 0; p < P; ++p) {
     const float* r = rewards + (long)p * G;
+    const std::vector<int> cls = classes_of(r, adv ? adv + (long)p * G : nullptr, G, class_eps);
     Group& grp = groups[p];
     grp = order_group(r, G);
     std::vector<GramSet> sets(G);
@@ -96,7 +146,7 @@ extern "C" int oracle_prune(const float* rewards, const int32_t* ids, const int6
     for (int i : grp.order) {
       bool drop = false;
       for (int j : grp.order) {
-        if (!kept[j] || r[j] != r[i]) continue;
+        if (!kept[j] || cls[j] != cls[i]) continue;
         if (jaccard_distance(sets[i], sets[j]) < (double)tau) drop = true;
       }
       kept[i] = !drop;
@@ -106,27 +156,22 @@ extern "C" int oracle_prune(const float* rewards, const int32_t* ids, const int6
     for (int i = 0; i < G; ++i) count += kept[i] ? 1 : 0;
     if (count > keep_cap) {
       struct Cls {
-        double dist;
-        int first;
-        std::vector<int> members;  // kept members, ascending index
+        int label;
+        std::vector<int> members;  // kept members, in visiting order
       };
-      std::vector<Cls> classes;
-      for (int i = 0; i < G; ++i) {
+      std::vector<Cls> classes;  // in visiting order of their first visited member
+      for (int i : grp.order) {
         if (!kept[i]) continue;
         bool placed = false;
         for (Cls& c : classes) {
-          if (r[c.first] == r[i]) {
+          if (c.label == cls[i]) {
             c.members.push_back(i);
             placed = true;
             break;
           }
         }
-        if (!placed) classes.push_back(Cls{grp.dist[i], i, {i}});
+        if (!placed) classes.push_back(Cls{cls[i], {i}});
       }
-      std::stable_sort(classes.begin(), classes.end(), [](const Cls& a, const Cls& b) {
-        if (a.dist != b.dist) return a.dist > b.dist;
-        return a.first < b.first;
-      });
       std::vector<bool> capped(G, false);
       int taken = 0;
       for (size_t round = 0; taken < keep_cap; ++round) {

@@ -30,6 +30,13 @@ int oracle_prune(const float* rewards, const int32_t* ids, const int64_t* off, i
                  int ngram_n, float tau, int keep_cap, int dp_divisor, uint8_t* keep,
                  int32_t* kept_per_prompt);
 
+/* The same with the continuous-reward grouping: class_eps > 0 groups rollouts whose advantages
+ * (adv, f32 [P*G]) chain with consecutive sorted gaps below class_eps. */
+int oracle_prune_classes(const float* rewards, const float* adv, float class_eps,
+                         const int32_t* ids, const int64_t* off, int P, int G, int ngram_n,
+                         float tau, int keep_cap, int dp_divisor, uint8_t* keep,
+                         int32_t* kept_per_prompt);
+
 /* Eq. 7 alone, for tests: theta_ij for rollouts i and j (indices into off). */
 double oracle_jaccard_distance(const int32_t* ids, const int64_t* off, int i, int j, int ngram_n);
 

@@ -73,8 +73,8 @@ def lib():
     L.grpo_kernel_launches.argtypes = []
     L.grpo_advantage.argtypes = [_c_p, _i32, _i32, _i32, _c_p, _c_p, _c_p]
     L.grpo_advantage.restype = _i32
-    L.grpo_prune.argtypes = [_c_p, _c_p, _c_p, _i32, _i32, _i64, _i32, _i32, _f32, _i32, _i32, _c_p,
-                             _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_prune.argtypes = [_c_p, _c_p, _f32, _c_p, _c_p, _i32, _i32, _i64, _i32, _i32, _f32, _i32,
+                             _i32, _c_p, _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
     L.grpo_prune.restype = _i32
     L.grpo_compact.argtypes = [_c_p, _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
     L.grpo_compact.restype = _i32
@@ -194,8 +194,9 @@ def grpo_advantage(rewards, G: int, std_mode: int = 0, adv=None, key=None, strea
 
 def grpo_prune(rewards, ids, off, G: int, V: int, ngram_n: int = 1, tau: float = 0.8,
                keep_cap: int | None = None, dp_divisor: int = 1, keep=None, kept_per_prompt=None,
-               status=None, ws=None, stream=None):
-    """Eqs. 6-9 + Algorithm 1 on the GPU.  Returns (keep u8 [P*G], kept_per_prompt i32 [P])."""
+               status=None, ws=None, stream=None, adv=None, class_eps: float = 0.0):
+    """Eqs. 6-9 + Algorithm 1 on the GPU.  Returns (keep u8 [P*G], kept_per_prompt i32 [P]).
+    class_eps > 0 with adv: classes by chained advantages (continuous rewards)."""
     torch = _torch()
     _need(rewards, torch.float32, None, "rewards")
     n = rewards.numel()
@@ -208,16 +209,16 @@ def grpo_prune(rewards, ids, off, G: int, V: int, ngram_n: int = 1, tau: float =
         keep = torch.empty(n, dtype=torch.uint8, device=rewards.device)
     if kept_per_prompt is None:
         kept_per_prompt = torch.empty(max(P, 1), dtype=torch.int32, device=rewards.device)
+    if adv is not None:
+        _need(adv, torch.float32, n, "adv")
     L = lib()
+    head = (_ptr(rewards), _ptr(adv), float(class_eps), _ptr(ids), _ptr(off), P, G, T, V, ngram_n,
+            float(tau), cap, dp_divisor, _ptr(keep), _ptr(kept_per_prompt), _ptr(status))
     need = ctypes.c_size_t(0)
-    _check(L.grpo_prune(_ptr(rewards), _ptr(ids), _ptr(off), P, G, T, V, ngram_n, float(tau), cap,
-                        dp_divisor, _ptr(keep), _ptr(kept_per_prompt), _ptr(status), None,
-                        ctypes.byref(need), _stream(stream)))
+    _check(L.grpo_prune(*head, None, ctypes.byref(need), _stream(stream)))
     wst = _workspace(need.value, rewards.device, ws)
     wp, size = _ws_args(wst)
-    _check(L.grpo_prune(_ptr(rewards), _ptr(ids), _ptr(off), P, G, T, V, ngram_n, float(tau), cap,
-                        dp_divisor, _ptr(keep), _ptr(kept_per_prompt), _ptr(status), wp, size,
-                        _stream(stream)))
+    _check(L.grpo_prune(*head, wp, size, _stream(stream)))
     return keep, kept_per_prompt[:P]
 
 

@@ -1,7 +1,7 @@
 // grpo_prune: maximising-differential advantage pruning (MDAP), Sec. 3.2 Eqs. 6-9, with the
 // traversal order, per-class guarantee and DP-alignment fill of Algorithm 1 (Phase 2).
 //
-// Kernels, in stream order:
+// Kernels, in stream order (0 first):
 //   1. the n-gram sets N_n(o_i) of Eq. 7, one CTA per rollout:
 //        n = 1   unigram_set_kernel: a bitmap over the vocabulary built in shared memory;
 //        n = 2,3 ngram_set_kernel: each length-n window packed into a 64-bit key (18 bits per id),
@@ -10,8 +10,10 @@
 //        n = 1   bitmap_pair_kernel: |N_i & N_j| = popcount of the AND, one CTA per pair;
 //        n = 2,3 sorted_pair_kernel: binary search of the smaller set in the larger, a warp per pair;
 //      each writes one byte per ordered pair: 1 when the two are in one class and too close;
-//   3. select_kernel, one warp per prompt: fp64 |r - mean| visiting order, the greedy of Eq. 8 as
-//      bitmask operations, and the per-prompt cap by round-robin over classes;
+//   0. class_kernel, one warp per prompt: advantage classes (exact reward equality, or chained
+//      advantages for continuous rewards) and the fp64 |r - mean| visiting order;
+//   3. select_kernel, one warp per prompt: the greedy of Eq. 8 as bitmask operations and the
+//      per-prompt cap by round-robin over classes;
 //   4. dp_fill_kernel (dp_divisor > 1), one thread: cyclic fill to a multiple of the divisor.
 // Every decision is an integer or exactly rounded fp64 operation, so the keep mask is bit-exact.
 #include <algorithm>
@@ -30,6 +32,8 @@ struct PruneWs {
   uint64_t* keys;     // n >= 2: [2T]; rollout r owns keys[2*off[r] .. 2*off[r+1])
   uint64_t* bitmaps;  // n == 1: [P*G][words]
   int32_t* nuniq;     // [P*G] set sizes
+  int32_t* cls;       // [P*G] class label: the smallest index in the rollout's class
+  int32_t* rank;      // [P*G] visiting position inside the prompt
   uint8_t* close;     // [P*G*G]: close[(p*G + i)*G + j] = 1 if same class and theta_ij < tau
   int words;          // ceil(V / 64)
 };
@@ -39,7 +43,7 @@ __host__ __device__ inline int bitmap_words(int V) { return (V + 63) / 64; }
 size_t prune_ws_bytes(int64_t T, int P, int G, int V, int n) {
   const size_t keys = n >= 2 ? (size_t)(2 * T) * 8 : 0;
   const size_t bitmaps = n == 1 ? (size_t)P * G * bitmap_words(V) * 8 : 0;
-  return align_up(keys, 256) + align_up(bitmaps, 256) + align_up((size_t)P * G * 4, 256) +
+  return align_up(keys, 256) + align_up(bitmaps, 256) + 3 * align_up((size_t)P * G * 4, 256) +
          align_up((size_t)P * G * G, 256);
 }
 
@@ -52,6 +56,10 @@ PruneWs prune_ws(void* ws, int64_t T, int P, int G, int V, int n) {
   w.bitmaps = reinterpret_cast<uint64_t*>(p);
   p += align_up(n == 1 ? (size_t)P * G * w.words * 8 : 0, 256);
   w.nuniq = reinterpret_cast<int32_t*>(p);
+  p += align_up((size_t)P * G * 4, 256);
+  w.cls = reinterpret_cast<int32_t*>(p);
+  p += align_up((size_t)P * G * 4, 256);
+  w.rank = reinterpret_cast<int32_t*>(p);
   p += align_up((size_t)P * G * 4, 256);
   w.close = reinterpret_cast<uint8_t*>(p);
   return w;
@@ -213,7 +221,7 @@ __global__ void unigram_set_kernel(const int32_t* __restrict__ ids, const int64_
   }
 }
 
-__global__ void bitmap_pair_kernel(const float* __restrict__ rewards, int G, float tau, PruneWs w) {
+__global__ void bitmap_pair_kernel(int G, float tau, PruneWs w) {
   __shared__ int warp_cnt[32];
   const int pairs = G * (G - 1) / 2;
   const int p = blockIdx.x / pairs;
@@ -221,7 +229,7 @@ __global__ void bitmap_pair_kernel(const float* __restrict__ rewards, int G, flo
   pair_of(blockIdx.x % pairs, G, i, j);
   const int ri = p * G + i, rj = p * G + j;
   uint8_t* close = w.close + (int64_t)p * G * G;
-  if (rewards[ri] != rewards[rj]) {  // different classes never compare (Eq. 8 is per class)
+  if (w.cls[ri] != w.cls[rj]) {  // different classes never compare (Eq. 8 is per class)
     if (threadIdx.x == 0) close[i * G + j] = close[j * G + i] = 0;
     return;
   }
@@ -239,8 +247,8 @@ __global__ void bitmap_pair_kernel(const float* __restrict__ rewards, int G, flo
   }
 }
 
-__global__ void sorted_pair_kernel(const float* __restrict__ rewards, const int64_t* __restrict__ off,
-                                   int P, int G, float tau, PruneWs w) {
+__global__ void sorted_pair_kernel(const int64_t* __restrict__ off, int P, int G, float tau,
+                                   PruneWs w) {
   const int pairs = G * (G - 1) / 2;
   const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
@@ -250,7 +258,7 @@ __global__ void sorted_pair_kernel(const float* __restrict__ rewards, const int6
   pair_of((int)(gw % pairs), G, i, j);
   const int ri = p * G + i, rj = p * G + j;
   uint8_t* close = w.close + (int64_t)p * G * G;
-  if (rewards[ri] != rewards[rj]) {
+  if (w.cls[ri] != w.cls[rj]) {
     if (lane == 0) close[i * G + j] = close[j * G + i] = 0;
     return;
   }
@@ -291,27 +299,72 @@ __device__ void group_dist(const float* r, int G, double* dist) {
   for (int i = 0; i < G; ++i) dist[i] = fabs(__dsub_rn((double)r[i], mean));
 }
 
-// One warp per prompt; lane i holds rollout i (G <= 32).
-__global__ void select_kernel(const float* __restrict__ rewards, int P, int G, int keep_cap,
-                              PruneWs w, uint8_t* __restrict__ keep,
-                              int32_t* __restrict__ kept_per_prompt) {
+// Classes and visiting order, one warp per prompt (lane i holds rollout i, G <= 32).
+//   classes: exact reward equality (Eq. 6 for discrete rewards), or, with class_eps > 0, chains
+//     of the advantages sorted ascending (ties by index) whose consecutive gaps are < class_eps
+//     (the continuous-reward grouping |A_i - A_j| < eps, closed under transitivity);
+//   visiting order: |A| descending as |r - mean| descending (fp64, Eq. 5's index-order mean),
+//     lower index first on ties.
+__global__ void class_kernel(const float* __restrict__ rewards, const float* __restrict__ adv,
+                             float class_eps, int P, int G, PruneWs w) {
   constexpr unsigned FULL = 0xffffffffu;
   const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
   const int lane = threadIdx.x & 31;
   if (p >= P) return;  // uniform per warp
   const bool act = lane < G;
   const float r = act ? rewards[(int64_t)p * G + lane] : 0.f;
-  // Eq. 5's mean, summed in index order (every lane runs the same sequence)
   double sum = 0.0;
   for (int i = 0; i < G; ++i) sum = __dadd_rn(sum, (double)__shfl_sync(FULL, r, i));
   const double mean = __ddiv_rn(sum, (double)G);
   const double dist = act ? fabs(__dsub_rn((double)r, mean)) : -1.0;
-  // visiting position: |A| descending (|r - mean| descending), lower index first on ties
   int rank = 0;
   for (int j = 0; j < G; ++j) {
     const double dj = __shfl_sync(FULL, dist, j);
     rank += (dj > dist || (dj == dist && j < lane)) ? 1 : 0;
   }
+  int label = lane;
+  if (class_eps <= 0.f) {
+    for (int j = G - 1; j >= 0; --j)  // smallest j with an equal reward
+      if (__shfl_sync(FULL, r, j) == r) label = j;
+  } else {
+    const float a = act ? adv[(int64_t)p * G + lane] : 0.f;
+    int spos = 0;  // position when sorted by a ascending, ties by index
+    for (int j = 0; j < G; ++j) {
+      const float aj = __shfl_sync(FULL, a, j);
+      spos += (aj < a || (aj == a && j < lane)) ? 1 : 0;
+    }
+    float prev = a;
+    for (int j = 0; j < G; ++j) {
+      const float aj = __shfl_sync(FULL, a, j);
+      const int sj = __shfl_sync(FULL, spos, j);
+      if (sj == spos - 1) prev = aj;
+    }
+    const bool brk = act && (spos == 0 || __dsub_rn((double)a, (double)prev) >= (double)class_eps);
+    int chain = 0;  // breaks at or before my sorted position
+    for (int j = 0; j < G; ++j) {
+      const int sj = __shfl_sync(FULL, spos, j);
+      const bool bj = __shfl_sync(FULL, brk, j);
+      chain += (bj && sj <= spos) ? 1 : 0;
+    }
+    for (int j = G - 1; j >= 0; --j)
+      if (__shfl_sync(FULL, chain, j) == chain) label = j;
+  }
+  if (act) {
+    w.cls[(int64_t)p * G + lane] = label;
+    w.rank[(int64_t)p * G + lane] = rank;
+  }
+}
+
+// One warp per prompt: the greedy of Eq. 8 and the per-prompt cap as bitmask operations.
+__global__ void select_kernel(int P, int G, int keep_cap, PruneWs w, uint8_t* __restrict__ keep,
+                              int32_t* __restrict__ kept_per_prompt) {
+  constexpr unsigned FULL = 0xffffffffu;
+  const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (p >= P) return;  // uniform per warp
+  const bool act = lane < G;
+  const int rank = act ? w.rank[(int64_t)p * G + lane] : 64 + lane;
+  const int label = act ? w.cls[(int64_t)p * G + lane] : -1 - lane;
   // same-class rollouts within tau of this one
   uint32_t near = 0;
   if (act) {
@@ -326,20 +379,25 @@ __global__ void select_kernel(const float* __restrict__ rewards, int P, int G, i
     if ((__shfl_sync(FULL, near, i) & kept) == 0) kept |= 1u << i;
   }
   int count = __popc(kept);
-  // Per-prompt cap: classes take turns in visiting order of their lowest member; each turn adds
-  // the class's next kept member by index.  Equivalently keep the keep_cap kept rollouts with the
-  // smallest (turn, class position).
+  // Per-prompt cap: classes take turns in visiting order of their first member; each turn adds
+  // the class's next kept member in visiting order.  Equivalently keep the keep_cap kept
+  // rollouts with the smallest (turn, class position).
   if (count > keep_cap) {
     const bool mine = act && ((kept >> lane) & 1u);
     uint32_t cls = 0;  // kept rollouts of my class
     for (int i = 0; i < G; ++i) {
-      const float ri = __shfl_sync(FULL, r, i);
-      const uint32_t m = __ballot_sync(FULL, act && ((kept >> lane) & 1u) && r == ri);
+      const int li = __shfl_sync(FULL, label, i);
+      const uint32_t m = __ballot_sync(FULL, act && ((kept >> lane) & 1u) && label == li);
       if (lane == i) cls = m;
     }
-    const int first = mine ? __ffs(cls) - 1 : 0;
-    const int turn = mine ? __popc(cls & ((1u << lane) - 1u)) : 0;
-    const int crank = __shfl_sync(FULL, rank, first);
+    int turn = 0, crank = 64;
+    for (int j = 0; j < G; ++j) {
+      const int rj = __shfl_sync(FULL, rank, j);
+      if ((cls >> j) & 1u) {
+        turn += rj < rank ? 1 : 0;
+        crank = min(crank, rj);
+      }
+    }
     const int key = turn * 64 + crank;
     int before = 0;
     for (int j = 0; j < G; ++j) {
@@ -387,12 +445,13 @@ __global__ void dp_fill_kernel(const float* __restrict__ rewards, int P, int G, 
 
 using namespace fastrl;
 
-extern "C" grpo_status grpo_prune(const float* rewards, const int32_t* ids, const int64_t* off,
-                                  int32_t P, int32_t G, int64_t T, int32_t V, int32_t ngram_n,
-                                  float tau, int32_t keep_cap, int32_t dp_divisor, uint8_t* keep,
-                                  int32_t* kept_per_prompt, int32_t* status, void* ws,
-                                  size_t* ws_bytes, grpo_stream_t stream) {
+extern "C" grpo_status grpo_prune(const float* rewards, const float* adv, float class_eps,
+                                  const int32_t* ids, const int64_t* off, int32_t P, int32_t G,
+                                  int64_t T, int32_t V, int32_t ngram_n, float tau, int32_t keep_cap,
+                                  int32_t dp_divisor, uint8_t* keep, int32_t* kept_per_prompt,
+                                  int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
   clear_error();
+  if (!(class_eps >= 0.f)) return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: class_eps must be >= 0");
   if (P < 0 || T < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: P = %d, T = %lld", P, (long long)T);
   if (G < 1 || G > kMaxG) return fail(GRPO_ERR_UNSUPPORTED, "grpo_prune: G = %d not in [1, %d]", G, kMaxG);
   if (V < 1 || V > (1 << 18))
@@ -407,18 +466,20 @@ extern "C" grpo_status grpo_prune(const float* rewards, const int32_t* ids, cons
       workspace_check(ws, ws_bytes, prune_ws_bytes(T, P, G, V, ngram_n), "grpo_prune", &query);
   if (ws_ok != GRPO_OK || query) return ws_ok;
   if (P == 0) return GRPO_OK;
-  if (!rewards || !off || !keep || !kept_per_prompt || (T > 0 && !ids))
+  if (!rewards || !off || !keep || !kept_per_prompt || (T > 0 && !ids) || (class_eps > 0.f && !adv))
     return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: NULL array");
   cudaStream_t s = as_stream(stream);
   const PruneWs w = prune_ws(ws, T, P, G, V, ngram_n);
   const int nroll = P * G;
   const int pairs = G * (G - 1) / 2;
-  int launches = 0;
+  const unsigned warp_blocks = (unsigned)(((int64_t)P * 32 + 127) / 128);
+  class_kernel<<<warp_blocks, 128, 0, s>>>(rewards, adv, class_eps, P, G, w);
+  int launches = 1;
   if (ngram_n == 1) {
     unigram_set_kernel<<<nroll, 256, (size_t)w.words * 8, s>>>(ids, off, V, w, status);
     ++launches;
     if (pairs > 0) {
-      bitmap_pair_kernel<<<(unsigned)((int64_t)P * pairs), 128, 0, s>>>(rewards, G, tau, w);
+      bitmap_pair_kernel<<<(unsigned)((int64_t)P * pairs), 128, 0, s>>>(G, tau, w);
       ++launches;
     }
   } else {
@@ -431,12 +492,11 @@ extern "C" grpo_status grpo_prune(const float* rewards, const int32_t* ids, cons
     if (pairs > 0) {
       const int tpb = 256;
       const int64_t blocks = ((int64_t)P * pairs * 32 + tpb - 1) / tpb;
-      sorted_pair_kernel<<<(unsigned)blocks, tpb, 0, s>>>(rewards, off, P, G, tau, w);
+      sorted_pair_kernel<<<(unsigned)blocks, tpb, 0, s>>>(off, P, G, tau, w);
       ++launches;
     }
   }
-  select_kernel<<<(unsigned)(((int64_t)P * 32 + 127) / 128), 128, 0, s>>>(rewards, P, G, keep_cap, w,
-                                                                          keep, kept_per_prompt);
+  select_kernel<<<warp_blocks, 128, 0, s>>>(P, G, keep_cap, w, keep, kept_per_prompt);
   ++launches;
   if (dp_divisor > 1) {
     dp_fill_kernel<<<1, 32, 0, s>>>(rewards, P, G, dp_divisor, keep, kept_per_prompt);

@@ -31,6 +31,7 @@ class StepParams:
     dlogits_dtype: str = "bf16"
     std_mode: int = 0
     chunk_rows: int = 0  # >0: the loss runs over the kept rows in chunks sharing one dlogits buffer
+    class_eps: float = 0.0  # >0: continuous-reward grouping of advantages (the paper uses 1e-4)
 
 
 class GrpoStep:
@@ -90,7 +91,7 @@ class GrpoStep:
         B.grpo_advantage(self.rewards, p.G, p.std_mode, adv=self.adv)
         B.grpo_prune(self.rewards, self.ids, self.off, p.G, p.V, p.ngram_n, p.tau, p.keep_cap,
                      p.dp_divisor, keep=self.keep, kept_per_prompt=self.kpp, status=self.status,
-                     ws=self.prune_ws)
+                     ws=self.prune_ws, adv=self.adv, class_eps=p.class_eps)
         B.grpo_compact(self.keep, self.off, kept_idx=self.kept_idx, kept_off=self.kept_off,
                        src_token=self.src_token, token_rollout=self.token_rollout,
                        counts=self.counts, counts_host=self.counts_host)
@@ -111,9 +112,9 @@ class GrpoStep:
         L = B.lib()
         need = ctypes.c_size_t(0)
         p = self.p
-        rc = L.grpo_prune(None, None, None, self.P, p.G, self.T, p.V, p.ngram_n, float(p.tau),
-                          p.keep_cap or p.G, p.dp_divisor, None, None, None, None,
-                          ctypes.byref(need), None)
+        rc = L.grpo_prune(None, None, float(p.class_eps), None, None, self.P, p.G, self.T, p.V,
+                          p.ngram_n, float(p.tau), p.keep_cap or p.G, p.dp_divisor, None, None,
+                          None, None, ctypes.byref(need), None)
         B._check(rc)
         self.prune_ws = self.torch.empty(need.value + 256, dtype=self.torch.uint8, device=self.dev)
         self.loss_ws = self.torch.empty(self.T * 8 + 512, dtype=self.torch.uint8, device=self.dev)

@@ -80,13 +80,13 @@ def test_argument_errors_return_status_without_gpu_work(grpo):
     assert L.grpo_advantage(None, 0, 4, 0, None, None, None) == 0  # P = 0 is a no-op
     size = ctypes.c_size_t(0)
     # G above 32, V above 2^18, n-gram order 4 are outside the supported limits
-    assert L.grpo_prune(None, None, None, 4, 33, 10, 100, 1, 0.8, 4, 1, None, None, None, None,
+    assert L.grpo_prune(None, None, 0.0, None, None, 4, 33, 10, 100, 1, 0.8, 4, 1, None, None, None, None,
                         ctypes.byref(size), None) == 2
-    assert L.grpo_prune(None, None, None, 4, 8, 10, (1 << 18) + 1, 1, 0.8, 4, 1, None, None, None,
+    assert L.grpo_prune(None, None, 0.0, None, None, 4, 8, 10, (1 << 18) + 1, 1, 0.8, 4, 1, None, None, None,
                         None, ctypes.byref(size), None) == 2
-    assert L.grpo_prune(None, None, None, 4, 8, 10, 100, 4, 0.8, 4, 1, None, None, None, None,
+    assert L.grpo_prune(None, None, 0.0, None, None, 4, 8, 10, 100, 4, 0.8, 4, 1, None, None, None, None,
                         ctypes.byref(size), None) == 2
-    assert L.grpo_prune(None, None, None, 4, 8, 10, 100, 1, 0.8, 0, 1, None, None, None, None,
+    assert L.grpo_prune(None, None, 0.0, None, None, 4, 8, 10, 100, 1, 0.8, 0, 1, None, None, None, None,
                         ctypes.byref(size), None) == 1
     assert L.grpo_compact(None, None, -1, None, None, None, None, None, None, None) == 1
     assert L.grpo_loss_tune(17, 0, 0) == 1 and L.grpo_loss_tune(0, 96, 0) == 1
@@ -103,16 +103,16 @@ def loss_call(L, n_rows, V, ws, size_p, ldt=1, agg=0, denom=1, row_loss=None, be
 def test_workspace_queries_answer_without_a_device(grpo):
     L = raw()
     size = ctypes.c_size_t(0)
-    assert L.grpo_prune(None, None, None, 16, 8, 5000, 152064, 2, 0.8, 4, 1, None, None, None,
+    assert L.grpo_prune(None, None, 0.0, None, None, 16, 8, 5000, 152064, 2, 0.8, 4, 1, None, None, None,
                         None, ctypes.byref(size), None) == 0
     def up(x):
         return (x + 255) // 256 * 256
     # bigrams: sorted keys (2T u64), set sizes, one byte per ordered pair
-    assert size.value == up(2 * 5000 * 8) + up(16 * 8 * 4) + up(16 * 8 * 8)
-    assert L.grpo_prune(None, None, None, 16, 8, 5000, 152064, 1, 0.8, 4, 1, None, None, None,
+    assert size.value == up(2 * 5000 * 8) + 3 * up(16 * 8 * 4) + up(16 * 8 * 8)
+    assert L.grpo_prune(None, None, 0.0, None, None, 16, 8, 5000, 152064, 1, 0.8, 4, 1, None, None, None,
                         None, ctypes.byref(size), None) == 0
     # unigrams: a vocabulary bitmap per rollout instead of keys
-    assert size.value == up(16 * 8 * ((152064 + 63) // 64) * 8) + up(16 * 8 * 4) + up(16 * 8 * 8)
+    assert size.value == up(16 * 8 * ((152064 + 63) // 64) * 8) + 3 * up(16 * 8 * 4) + up(16 * 8 * 8)
     assert loss_call(L, 1000, 152064, None, ctypes.byref(size)) == 0
     assert size.value == up(1000 * 8)
     # with a row-loss output the loss needs no workspace

@@ -149,3 +149,35 @@ def test_compact_bit_exact(grpo, oracle_mod, n):
         assert np.array_equal(out["kept_off"][:K + 1].cpu().numpy(), o["kept_off"])
         assert np.array_equal(out["src_token"][:TK].cpu().numpy(), o["src_token"])
         assert np.array_equal(out["token_rollout"][:TK].cpu().numpy(), o["token_rollout"])
+
+
+@pytest.mark.parametrize("eps", [1e-4, 1e-2, 0.5])
+@pytest.mark.parametrize("n", [1, 2])
+def test_prune_continuous_grouping(grpo, oracle_mod, eps, n):
+    """Classes by chained advantages (continuous rewards): the GPU takes grpo_advantage's
+    advantages, the oracle its own; both keep masks agree bit for bit."""
+    import torch
+    from mdap_ref import clustered_rewards
+    rng = np.random.default_rng(int(eps * 1e4) + n)
+    for trial in range(6):
+        P = int(rng.integers(1, 10))
+        G = int(rng.integers(2, 33))
+        rewards, seqs = [], []
+        for _ in range(P):
+            _, s = random_structured_prompt(rng, G, vocab=int(rng.integers(3, 30)), max_len=25,
+                                            q=float(rng.choice([0.1, 0.4])))
+            rewards += clustered_rewards(rng, G, spread=float(rng.choice([1e-5, 1e-3])))
+            seqs += s
+        ids, off = pack_rollouts(seqs)
+        r = np.asarray(rewards, np.float32)
+        cap = int(rng.integers(1, G + 2))
+        dp = int(rng.choice([1, 3]))
+        adv_g, _ = grpo.grpo_advantage(t(r), G)
+        status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        keep, kpp = grpo.grpo_prune(t(r), t(ids), t(off), G, 64, n, 0.8, cap, dp, status=status,
+                                    adv=adv_g, class_eps=eps)
+        torch.cuda.synchronize()
+        adv_o, _ = oracle_mod.advantage(r, G)
+        o_keep, o_kpp = oracle_mod.prune(r, ids, off, G, n, 0.8, cap, dp, adv=adv_o, class_eps=eps)
+        assert np.array_equal(keep.cpu().numpy(), o_keep), (trial, P, G, cap, dp)
+        assert np.array_equal(kpp.cpu().numpy(), o_kpp)

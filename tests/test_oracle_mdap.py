@@ -110,3 +110,61 @@ def test_dp_fill_properties(oracle_mod):
                 best = sorted(left, key=lambda j: (-dist[p][j], j))[:int(per_prompt[p])]
                 assert i in best
         assert kpp.tolist() == filled.reshape(P, G).sum(1).tolist()
+
+
+from mdap_ref import (brute_force_mdap_labels, cap_by_sort_labels, chain_classes,
+                      clustered_rewards)
+
+
+def run_oracle_cont(oracle_mod, rewards, seqs, G, n, tau, eps, cap=None, dp=1):
+    ids, off = pack_rollouts(seqs)
+    adv, _ = oracle_mod.advantage(np.asarray(rewards, np.float32), G)
+    keep, kpp = oracle_mod.prune(np.asarray(rewards, np.float32), ids, off, G, n, tau, cap, dp,
+                                 adv=adv, class_eps=eps)
+    return keep, kpp, adv
+
+
+@pytest.mark.parametrize("G", [3, 5, 8])
+@pytest.mark.parametrize("eps", [1e-4, 1e-2, 0.5])
+def test_continuous_grouping_brute_force(oracle_mod, G, eps):
+    """Chained-advantage classes (the continuous-reward extension), then per class the
+    lexicographically largest independent set, found by enumeration."""
+    rng = np.random.default_rng(int(G * 1000 + eps * 1e4))
+    for trial in range(20):
+        _, seqs = random_structured_prompt(rng, G, vocab=5, max_len=6, q=0.3)
+        rewards = clustered_rewards(rng, G)
+        keep, _, adv = run_oracle_cont(oracle_mod, rewards, seqs, G, 1, 0.8, eps)
+        labels = chain_classes(adv, eps)
+        assert keep.astype(bool).tolist() == brute_force_mdap_labels(rewards, seqs, 1, 0.8, labels)
+
+
+def test_continuous_grouping_limits(oracle_mod):
+    rng = np.random.default_rng(31)
+    for _ in range(100):
+        G = int(rng.integers(2, 9))
+        rewards, seqs = random_structured_prompt(rng, G, vocab=4, max_len=6, q=0.3)
+        ids, off = pack_rollouts(seqs)
+        r = np.asarray(rewards, np.float32)
+        exact, _ = oracle_mod.prune(r, ids, off, G, 1, 0.8)
+        adv, _ = oracle_mod.advantage(r, G)
+        # eps below every gap between distinct advantages: the exact-equality classes
+        tiny, _ = oracle_mod.prune(r, ids, off, G, 1, 0.8, adv=adv, class_eps=1e-30)
+        assert np.array_equal(tiny, exact)
+        # eps above every gap: one class, so the greedy runs over the whole group
+        one, _ = oracle_mod.prune(r, ids, off, G, 1, 0.8, adv=adv, class_eps=1e30)
+        assert one.astype(bool).tolist() == brute_force_mdap_labels(rewards, seqs, 1, 0.8, [0] * G)
+
+
+def test_continuous_cap_in_visiting_order(oracle_mod):
+    rng = np.random.default_rng(32)
+    for _ in range(200):
+        G = int(rng.integers(2, 17))
+        _, seqs = random_structured_prompt(rng, G, vocab=40, max_len=5, q=0.9)
+        rewards = clustered_rewards(rng, G, spread=3e-3)
+        eps = float(rng.choice([1e-4, 1e-2, 0.2]))
+        uncapped, _, adv = run_oracle_cont(oracle_mod, rewards, seqs, G, 1, 0.8, eps)
+        cap = int(rng.integers(1, G + 1))
+        capped, kpp, _ = run_oracle_cont(oracle_mod, rewards, seqs, G, 1, 0.8, eps, cap)
+        labels = chain_classes(adv, eps)
+        assert capped.astype(bool).tolist() == cap_by_sort_labels(rewards, uncapped.astype(bool),
+                                                                  cap, labels)
