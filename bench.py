@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="run each step's calls directly instead of replaying captured CUDA graphs")
     return ap.parse_args()
 
 
@@ -338,6 +340,15 @@ def main():
     for _ in range(max(args.warmup, 3)):
         step.run()
     torch.cuda.synchronize()
+    l_before = g.grpo_kernel_launches()
+    step.run()
+    torch.cuda.synchronize()
+    launches_per_step = g.grpo_kernel_launches() - l_before
+    use_graph = not args.no_graph and w.chunk_rows == 0
+    if use_graph:
+        step.capture()
+        for _ in range(max(args.warmup, 3)):
+            step.run_graph()
 
     K = args.steps
     stream = torch.cuda.current_stream()
@@ -355,14 +366,21 @@ def main():
     kept = 0
     ev0.record(stream)
     for i in range(K):
-        step.select()
-        l0[i].record(stream)
-        step.loss_step()
-        l1[i].record(stream)
+        if use_graph:  # the step as two graph replays; the host reads the counts at its end
+            step.replay_select()
+            l0[i].record(stream)
+            step.replay_loss()
+            l1[i].record(stream)
+            step.finish()
+        else:
+            step.select()
+            l0[i].record(stream)
+            step.loss_step()
+            l1[i].record(stream)
         kept += step.T_kept
     ev1.record(stream)
     torch.cuda.synchronize()
-    launches = g.grpo_kernel_launches() - launches0
+    launches = launches_per_step * K if use_graph else g.grpo_kernel_launches() - launches0
     clocks = sampler.stop() if local == 0 else None
     g.check_status(step.status)
     elapsed_ms = ev0.elapsed_time(ev1)
@@ -431,8 +449,14 @@ def main():
         for _ in range(args.e2e_steps):
             for k in names:
                 d[k].copy_(host[k], non_blocking=True)
-            step.run()
-            loss_host.copy_(step.loss, non_blocking=True)
+            if use_graph:
+                step.replay_select()
+                step.replay_loss()
+                loss_host.copy_(step.loss, non_blocking=True)
+                step.finish()
+            else:
+                step.run()
+                loss_host.copy_(step.loss, non_blocking=True)
             kept_e += step.T_kept
         e1.record(stream)
         torch.cuda.synchronize()
@@ -452,7 +476,8 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded; shapes and distributions of the paper's GRPO batches)",
             "config": workload_desc(w, b["T"], step.T_kept, step.K),
-            "gpu_launches": int(launches), "roofline": roofline, "e2e": e2e,
+            "gpu_launches": int(launches), "cuda_graph": use_graph,
+            "roofline": roofline, "e2e": e2e,
             "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd,
             "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,
         }

@@ -208,6 +208,28 @@ grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_
 grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grpo_stream_t stream);
 
 /*
+ * grpo_loss_fwd_bwd_dev — grpo_loss_fwd_bwd with the row count read on the device, so that a
+ * whole step (advantage, prune, compact, loss) is enqueued without a host round trip and can be
+ * captured once in a CUDA graph (same Eqs. 1-3).
+ * counts    device i64 [2] = {K, T_kept}, e.g. grpo_compact's counts.  Rows processed:
+ *           min(max_rows, T_kept).  denom_tokens <= 0 (token mean) takes T_kept as the
+ *           denominator and n_seq <= 0 (sequence mean) takes K.
+ * max_rows  host capacity: row_index, row_rollout, dlogits [max_rows, V], logp_out and the
+ *           workspace (or row_loss_out) are sized for it.
+ * All other arguments as grpo_loss_fwd_bwd.
+ */
+grpo_status grpo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype, int64_t row_stride,
+                                  const int64_t* row_index, int64_t max_rows, const int64_t* counts,
+                                  int32_t V, const int32_t* y, const float* old_logp,
+                                  const float* ref_logp, const float* adv,
+                                  const int32_t* row_rollout, float eps_low, float eps_high,
+                                  float beta, int32_t agg_mode, int64_t denom_tokens,
+                                  const int64_t* seq_off, int64_t n_seq, void* dlogits,
+                                  int32_t dlogits_dtype, float* logp_out, double* row_loss_out,
+                                  double* loss_out, int32_t* status, void* ws, size_t* ws_bytes,
+                                  grpo_stream_t stream);
+
+/*
  * grpo_loss_fwd_bwd_noalloc — grpo_loss_fwd_bwd for callers that cannot allocate device memory.
  * The paper has no counterpart: this is an interface convenience of this library.
  * Some callers run the loss where no allocation is possible: a plugin or custom-op host that

@@ -31,7 +31,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
+           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
            "grpo_loss_tune", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -82,6 +82,11 @@ def lib():
                                     _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p, _c_p,
                                     _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
     L.grpo_loss_fwd_bwd.restype = _i32
+    L.grpo_loss_fwd_bwd_dev.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p, _c_p, _c_p,
+                                        _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p,
+                                        _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                        ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_loss_fwd_bwd_dev.restype = _i32
     L.grpo_loss_fwd_bwd_noalloc.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p,
                                             _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64,
                                             _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p]
@@ -354,6 +359,31 @@ def grpo_loss_fwd_bwd_noalloc(logits, y, old_logp, ref_logp, adv, row_rollout, *
         float(beta), int(agg_mode), int(denom_tokens), _ptr(seq_off), int(n_seq), _ptr(dlogits),
         odt, _ptr(logp_out), _ptr(row_loss_out), _ptr(loss_out), _ptr(status), _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out)
+
+
+def grpo_loss_fwd_bwd_dev(logits, y, old_logp, ref_logp, adv, row_rollout, counts, *,
+                          max_rows: int, dlogits, loss_out, ws, V: int | None = None,
+                          row_stride: int | None = None, row_index=None, eps_low: float = 0.2,
+                          eps_high: float = 0.2, beta: float = 0.04, agg_mode: int = 0,
+                          denom_tokens: int = 0, seq_off=None, n_seq: int = 0, logp_out=None,
+                          row_loss_out=None, status=None, stream=None):
+    """Eqs. 1-3 with the row count {K, T_kept} read on the device (capturable in a CUDA graph).
+    All buffers are passed in, sized for max_rows; nothing is allocated here."""
+    torch = _torch()
+    ldt = GRPO_DTYPE_BF16 if logits.dtype == torch.bfloat16 else GRPO_DTYPE_F32
+    odt = GRPO_DTYPE_BF16 if dlogits.dtype == torch.bfloat16 else GRPO_DTYPE_F32
+    if V is None:
+        V = logits.shape[1]
+    stride = logits.stride(0) if row_stride is None else int(row_stride)
+    _need(counts, torch.int64, 2, "counts")
+    wp, size = _ws_args(ws)
+    _check(lib().grpo_loss_fwd_bwd_dev(
+        _ptr(logits), ldt, stride, _ptr(row_index), int(max_rows), _ptr(counts), int(V), _ptr(y),
+        _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(row_rollout), float(eps_low),
+        float(eps_high), float(beta), int(agg_mode), int(denom_tokens), _ptr(seq_off), int(n_seq),
+        _ptr(dlogits), odt, _ptr(logp_out), _ptr(row_loss_out), _ptr(loss_out), _ptr(status), wp,
+        size, _stream(stream)))
+    return loss_out
 
 
 def grpo_logp_fwd(logits, y, *, V: int | None = None, row_stride: int | None = None,

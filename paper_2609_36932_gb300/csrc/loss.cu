@@ -72,6 +72,10 @@ struct LossArgs {
   int32_t n_chunks;
   int32_t bulk;     // rows 16-byte aligned: slices arrive by bulk copies
   int32_t out_vec;  // dlogits rows 16-byte aligned: vector stores
+  // Device counts {K, T_kept} (nullable): rows processed = min(n_rows, T_kept); with
+  // denom_from_counts the token-mean denominator is T_kept and Eq. 1's n_seq is K.
+  const int64_t* counts;
+  int32_t denom_from_counts;
 };
 
 // ---- PTX helpers ------------------------------------------------------------------------------
@@ -327,15 +331,28 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
   };
   auto wait_chunk = [&](int k, uint32_t parity) { wait_bar(bar_s + 8 * k, parity); };
 
+  int64_t n_rows = a.n_rows;
+  double inv_denom = a.inv_denom;
+  float inv_denom_f = a.inv_denom_f, inv_nseq_f = a.inv_nseq_f;
+  if (a.counts) {
+    const int64_t k_kept = a.counts[0], t_kept = a.counts[1];
+    n_rows = t_kept < n_rows ? t_kept : n_rows;
+    if (a.denom_from_counts) {
+      inv_denom = t_kept > 0 ? 1.0 / (double)t_kept : 0.0;
+      inv_denom_f = (float)inv_denom;
+      inv_nseq_f = k_kept > 0 ? (float)(1.0 / (double)k_kept) : 0.f;
+    }
+  }
+
   int64_t row = cluster_id_x();
   uint32_t phase = 0;  // parity of the copy barriers (one completion per row)
   uint32_t iter = 0;   // rows done; exchange slot = iter & 1, its parity = (iter >> 1) & 1
-  if (tid == 0 && row < a.n_rows) {
+  if (tid == 0 && row < n_rows) {
     const char* g = row_base(row);
     for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
   }
 
-  for (; row < a.n_rows; row += ncl, phase ^= 1u, ++iter) {
+  for (; row < n_rows; row += ncl, phase ^= 1u, ++iter) {
     const uint32_t slot = iter & 1u;
     if (tid == 0) mbar_expect_tx(xbar_s + 8 * slot, 16u * C);  // one entry from every CTA
     const int64_t src = a.row_index ? a.row_index[row] : row;
@@ -424,7 +441,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
       }
       if constexpr (!kBwd) {  // forward only: the slice is consumed; fetch the next row now
         __syncwarp();
-        if (lane == 0 && row + ncl < a.n_rows && !*(volatile int*)abort_flag) {
+        if (lane == 0 && row + ncl < n_rows && !*(volatile int*)abort_flag) {
           const char* g = row_base(row + ncl);
           for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
         }
@@ -478,10 +495,10 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           const float ell = -(surr - a.beta * kl);
           float w;
           if (a.agg_mode == 0) {
-            w = a.inv_denom_f;
+            w = inv_denom_f;
           } else {
             const int32_t r = a.row_rollout[row];
-            w = a.inv_nseq_f / (float)(a.seq_off[r + 1] - a.seq_off[r]);
+            w = inv_nseq_f / (float)(a.seq_off[r + 1] - a.seq_off[r]);
           }
           const bool c = (A >= 0.f) ? (rho <= a.hi_dn) : (rho >= a.lo_up);
           const float g = -((c ? rho * A : 0.f) + a.beta * em1);
@@ -495,7 +512,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           }
           if (rank == 0) {
             if (a.logp_out) a.logp_out[row] = logp;
-            a.row_loss[row] = (a.agg_mode == 0 ? a.inv_denom : (double)w) * (double)ell;
+            a.row_loss[row] = (a.agg_mode == 0 ? inv_denom : (double)w) * (double)ell;
             if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
           }
           }  // kBwd
@@ -515,7 +532,7 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
     const float2 shb2 = make_float2(shB, shB), ns2 = make_float2(neg_scale, neg_scale);
     OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V + s0;
     const int64_t next = row + ncl;
-    const char* gnext = (tid == 0 && next < a.n_rows) ? row_base(next) : nullptr;
+    const char* gnext = (tid == 0 && next < n_rows) ? row_base(next) : nullptr;
     for (int k = 0; k < a.n_chunks; ++k) {
       const int v0 = k * a.chunk_vecs;
       const int v1 = min(nvec, v0 + a.chunk_vecs);
@@ -562,8 +579,10 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
   cluster_sync();  // partners are done reading this CTA's shared memory
 }
 
-__global__ void sum_rows_kernel(const double* __restrict__ v, int64_t n, double* __restrict__ out) {
+__global__ void sum_rows_kernel(const double* __restrict__ v, int64_t n, const int64_t* __restrict__ counts,
+                                double* __restrict__ out) {
   __shared__ double sh[1024];
+  if (counts && counts[1] < n) n = counts[1];
   double acc = 0.0;
   for (int64_t i = threadIdx.x; i < n; i += 1024) acc += v[i];
   sh[threadIdx.x] = acc;
@@ -583,6 +602,7 @@ struct Tune {
 Tune g_tune;
 std::mutex g_mu;
 std::map<std::tuple<const void*, int, int, int>, int> g_max_clusters;  // (kernel, dev, C, smem)
+std::map<std::pair<const void*, int>, size_t> g_smem_attr;            // (kernel, dev) -> bytes set
 
 using KernelFn = void (*)(LossArgs);
 
@@ -671,10 +691,7 @@ grpo_status launch_rows(KernelFn fn, const Shape& sh, LossArgs a, cudaStream_t s
   a.slice = sh.slice;
   a.chunk_vecs = sh.chunk_vecs;
   a.n_chunks = sh.chunks;
-  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh.smem);
-  if (e == cudaSuccess && sh.C > 8)
-    e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
+  cudaError_t e = cudaSuccess;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = sh.C;
@@ -695,7 +712,16 @@ grpo_status launch_rows(KernelFn fn, const Shape& sh, LossArgs a, cudaStream_t s
     auto it = g_max_clusters.find(key);
     if (it != g_max_clusters.end()) {
       max_cl = it->second;
-    } else {
+    } else {  // first launch of this kernel and shape on this device: set it up once
+      size_t& have = g_smem_attr[std::make_pair((const void*)fn, dev)];
+      if (sh.smem > have) {  // the attribute is a maximum: only ever raise it
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh.smem);
+        if (e == cudaSuccess) have = sh.smem;
+      }
+      if (e == cudaSuccess && sh.C > 8)
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e != cudaSuccess)
+        return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
       cfg.gridDim = dim3(sh.C, 1, 1);
       e = cudaOccupancyMaxActiveClusters(&max_cl, fn, &cfg);
       if (e != cudaSuccess)
@@ -737,20 +763,30 @@ extern "C" grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grp
   clear_error();
   if (n < 0 || out == nullptr || (n > 0 && v == nullptr))
     return fail(GRPO_ERR_INVALID_ARG, "grpo_sum_f64: n = %lld, v or out NULL", (long long)n);
-  sum_rows_kernel<<<1, 1024, 0, as_stream(stream)>>>(v, n, out);
+  sum_rows_kernel<<<1, 1024, 0, as_stream(stream)>>>(v, n, nullptr, out);
   count_launches(1);
   return check_launch("grpo_sum_f64");
 }
 
-extern "C" grpo_status grpo_loss_fwd_bwd(
-    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
-    int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,
-    const float* adv, const int32_t* row_rollout, float eps_low, float eps_high, float beta,
-    int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq, void* dlogits,
-    int32_t dlogits_dtype, float* logp_out, double* row_loss_out, double* loss_out, int32_t* status,
-    void* ws, size_t* ws_bytes, grpo_stream_t stream) {
-  clear_error();
-  const char* who = "grpo_loss_fwd_bwd";
+namespace fastrl {
+namespace {
+
+// The fused loss; counts (device {K, T_kept}, nullable) bounds the rows on the device and, with
+// a non-positive denom_tokens / n_seq, supplies the token-mean denominator / sequence count.
+grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype, int64_t row_stride,
+                      const int64_t* row_index, int64_t n_rows, const int64_t* counts, int32_t V,
+                      const int32_t* y, const float* old_logp, const float* ref_logp,
+                      const float* adv, const int32_t* row_rollout, float eps_low, float eps_high,
+                      float beta, int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off,
+                      int64_t n_seq, void* dlogits, int32_t dlogits_dtype, float* logp_out,
+                      double* row_loss_out, double* loss_out, int32_t* status, void* ws,
+                      size_t* ws_bytes, grpo_stream_t stream) {
+  const bool from_counts = counts != nullptr && ((agg_mode == 0 && denom_tokens <= 0) ||
+                                                 (agg_mode == 1 && n_seq <= 0));
+  if (from_counts) {  // both denominators come from the device counts
+    denom_tokens = 1;
+    n_seq = 1;
+  }
   if (logits_dtype != GRPO_DTYPE_BF16 && logits_dtype != GRPO_DTYPE_F32)
     return fail(GRPO_ERR_INVALID_ARG, "%s: logits_dtype = %d", who, logits_dtype);
   if (dlogits_dtype != GRPO_DTYPE_BF16 && dlogits_dtype != GRPO_DTYPE_F32)
@@ -775,7 +811,7 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   double* row_loss = row_loss_out ? row_loss_out : static_cast<double*>(ws);
   cudaStream_t s = as_stream(stream);
   if (n_rows == 0) {
-    sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, 0, loss_out);
+    sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, 0, nullptr, loss_out);
     count_launches(1);
     return check_launch(who);
   }
@@ -819,13 +855,49 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
   a.status = status;
   a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
   a.out_vec = (reinterpret_cast<uintptr_t>(dlogits) % 16 == 0) && (((int64_t)V * out_bytes) % 16 == 0);
+  a.counts = counts;
+  a.denom_from_counts = from_counts ? 1 : 0;
 
   st = launch_rows(kernel_for(logits_dtype, dlogits_dtype, sh.threads), sh, a, s, who);
   if (st != GRPO_OK) return st;
-  sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, n_rows, loss_out);
+  sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, n_rows, counts, loss_out);
   count_launches(2);
   return check_launch(who);
 }
+
+}  // namespace
+}  // namespace fastrl
+
+extern "C" grpo_status grpo_loss_fwd_bwd(
+    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
+    int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,
+    const float* adv, const int32_t* row_rollout, float eps_low, float eps_high, float beta,
+    int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq, void* dlogits,
+    int32_t dlogits_dtype, float* logp_out, double* row_loss_out, double* loss_out, int32_t* status,
+    void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  return loss_impl("grpo_loss_fwd_bwd", logits, logits_dtype, row_stride, row_index, n_rows, nullptr,
+                   V, y, old_logp, ref_logp, adv, row_rollout, eps_low, eps_high, beta, agg_mode,
+                   denom_tokens, seq_off, n_seq, dlogits, dlogits_dtype, logp_out, row_loss_out,
+                   loss_out, status, ws, ws_bytes, stream);
+}
+
+extern "C" grpo_status grpo_loss_fwd_bwd_dev(
+    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
+    int64_t max_rows, const int64_t* counts, int32_t V, const int32_t* y, const float* old_logp,
+    const float* ref_logp, const float* adv, const int32_t* row_rollout, float eps_low,
+    float eps_high, float beta, int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off,
+    int64_t n_seq, void* dlogits, int32_t dlogits_dtype, float* logp_out, double* row_loss_out,
+    double* loss_out, int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  if (counts == nullptr)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_loss_fwd_bwd_dev: counts is NULL");
+  return loss_impl("grpo_loss_fwd_bwd_dev", logits, logits_dtype, row_stride, row_index, max_rows,
+                   counts, V, y, old_logp, ref_logp, adv, row_rollout, eps_low, eps_high, beta,
+                   agg_mode, denom_tokens, seq_off, n_seq, dlogits, dlogits_dtype, logp_out,
+                   row_loss_out, loss_out, status, ws, ws_bytes, stream);
+}
+
 
 extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
                                      const int64_t* row_index, int64_t n_rows, int32_t V,

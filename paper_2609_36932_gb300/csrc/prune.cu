@@ -17,6 +17,7 @@
 //   4. dp_fill_kernel (dp_divisor > 1), one thread: cyclic fill to a multiple of the divisor.
 // Every decision is an integer or exactly rounded fp64 operation, so the keep mask is bit-exact.
 #include <algorithm>
+#include <atomic>
 
 #include "common.cuh"
 
@@ -484,9 +485,16 @@ extern "C" grpo_status grpo_prune(const float* rewards, const float* adv, float 
     }
   } else {
     const int smem = kSmemKeys * 8;
-    if (cudaFuncSetAttribute(ngram_set_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
-        cudaSuccess)
-      return check_launch("grpo_prune: cudaFuncSetAttribute");
+    static std::atomic<uint64_t> attr_set{0};  // bit d: the attribute is set on device d
+    int dev = 0;
+    cudaGetDevice(&dev);
+    const uint64_t bit = dev < 64 ? (1ull << dev) : 0ull;
+    if (!bit || !(attr_set.load() & bit)) {  // once per device, before any stream capture
+      if (cudaFuncSetAttribute(ngram_set_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+          cudaSuccess)
+        return check_launch("grpo_prune: cudaFuncSetAttribute");
+      attr_set.fetch_or(bit);
+    }
     ngram_set_kernel<<<nroll, kSortThreads, smem, s>>>(ids, off, V, ngram_n, w, status);
     ++launches;
     if (pairs > 0) {

@@ -154,6 +154,69 @@ class GrpoStep:
         B.grpo_sum_f64(self.row_loss, self.T_kept, out=self.loss)
         return dict(loss=self.loss, dlogits=self.dlogits, logp=self.logp)
 
+    # ---- CUDA-graph mode: no host round trip inside the step ----------------------------------
+
+    def _enqueue_select(self):
+        p = self.p
+        B.grpo_advantage(self.rewards, p.G, p.std_mode, adv=self.adv)
+        B.grpo_prune(self.rewards, self.ids, self.off, p.G, p.V, p.ngram_n, p.tau, p.keep_cap,
+                     p.dp_divisor, keep=self.keep, kept_per_prompt=self.kpp, status=self.status,
+                     ws=self.prune_ws, adv=self.adv, class_eps=p.class_eps)
+        B.grpo_compact(self.keep, self.off, kept_idx=self.kept_idx, kept_off=self.kept_off,
+                       src_token=self.src_token, token_rollout=self.token_rollout,
+                       counts=self.counts)
+        self.counts_host.copy_(self.counts, non_blocking=True)
+        self.kpp_host[:self.P].copy_(self.kpp[:self.P], non_blocking=True)
+
+    def _enqueue_loss(self):
+        p = self.p
+        B.grpo_loss_fwd_bwd_dev(
+            self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout, self.counts,
+            max_rows=self.T, dlogits=self.dlogits, loss_out=self.loss, ws=self.loss_ws, V=p.V,
+            row_index=self.src_token, eps_low=p.eps_low, eps_high=p.eps_high, beta=p.beta,
+            agg_mode=p.agg_mode, seq_off=self.off, logp_out=self.logp, status=self.status)
+
+    def capture(self):
+        """Capture the selection (advantage, prune, compact, count copies) and the loss as two
+        CUDA graphs.  The loss reads the kept-row count on the device, so nothing waits for the
+        host between them; dlogits are sized for all T rows."""
+        torch = self.torch
+        if self.p.chunk_rows > 0:
+            raise ValueError("graph mode runs the loss in one call (chunk_rows = 0)")
+        self._ensure_dlogits(self.T)
+        for _ in range(2):  # warm-up outside capture (kernel attributes, occupancy queries)
+            self._enqueue_select()
+            self._enqueue_loss()
+        torch.cuda.synchronize()
+        self.g_select, self.g_loss = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.g_select):
+            self._enqueue_select()
+        with torch.cuda.graph(self.g_loss):
+            self._enqueue_loss()
+        torch.cuda.synchronize()
+
+    def replay_select(self):
+        self.g_select.replay()
+
+    def replay_loss(self):
+        self.g_loss.replay()
+
+    def finish(self):
+        """After a replayed step: wait for it, read the kept counts and update ARS (Phase 1b)."""
+        self.torch.cuda.current_stream().synchronize()
+        self.K = int(self.counts_host[0])
+        self.T_kept = int(self.counts_host[1])
+        self.step_index += 1
+        s = (self.step_index - 1) % self.ars_total + 1
+        self.n_next = B.adaptive_rollout_count(self.ars, self.kpp_host[:self.P].numpy(), s,
+                                               self.ars_total, s % self.steps_per_epoch == 0)
+        return self.T_kept
+
+    def run_graph(self):
+        self.replay_select()
+        self.replay_loss()
+        return self.finish()
+
     def run(self):
         self.select()
         self.loss_step()

@@ -256,3 +256,36 @@ def test_peaked_rows_keep_one_minus_p_accurate(grpo, oracle_mod):
     g = c.run_gpu(grpo)
     r = c.run_oracle(oracle_mod)
     compare(g["logp"], g["dlogits"], g["loss"], r, "bf16")
+
+
+@pytest.mark.parametrize("agg_mode", [0, 1])
+def test_device_row_count_matches_host_count(grpo, agg_mode):
+    """grpo_loss_fwd_bwd_dev over min(max_rows, T_kept) rows, with its denominators from the
+    device counts, equals grpo_loss_fwd_bwd given the same numbers on the host, bit for bit."""
+    import torch
+    rng = np.random.default_rng(40 + agg_mode)
+    c = Case(rng, 64, 32000, "bf16", "bf16", n_roll=6)
+    rr = np.sort(rng.integers(0, 6, size=64)).astype(np.int32)
+    lens = np.bincount(rr, minlength=6)
+    seq_off = c.t(np.concatenate([[0], np.cumsum(lens)]).astype(np.int64))
+    for t_kept in (0, 1, 37, 64):
+        K = int((lens[:6] > 0).sum())
+        counts = c.t(np.array([K, t_kept], np.int64))
+        dl_a = torch.zeros((64, 32000), dtype=torch.bfloat16, device="cuda")
+        dl_b = torch.zeros_like(dl_a)
+        la = torch.empty(1, dtype=torch.float64, device="cuda")
+        lb = torch.empty(1, dtype=torch.float64, device="cuda")
+        ws = torch.empty(64 * 8 + 512, dtype=torch.uint8, device="cuda")
+        grpo.grpo_loss_fwd_bwd_dev(c.dev, c.t(c.y), c.t(c.old), c.t(c.ref), c.t(c.adv), c.t(rr),
+                                   counts, max_rows=64, dlogits=dl_a, loss_out=la, ws=ws,
+                                   beta=c.beta, agg_mode=agg_mode, seq_off=seq_off)
+        if t_kept:
+            grpo.grpo_loss_fwd_bwd(c.dev, c.t(c.y), c.t(c.old), c.t(c.ref), c.t(c.adv), c.t(rr),
+                                   n_rows=t_kept, beta=c.beta, agg_mode=agg_mode,
+                                   denom_tokens=t_kept, seq_off=seq_off, n_seq=K, dlogits=dl_b,
+                                   loss_out=lb)
+        else:
+            lb.zero_()
+        torch.cuda.synchronize()
+        assert la.item() == lb.item()
+        assert torch.equal(dl_a, dl_b)  # rows past T_kept untouched (still zero) in both

@@ -122,3 +122,27 @@ def test_full_size_sampled(oracle_mod, name):
         assert np.array_equal(step.logp[:TK].cpu().numpy(), logp)
         n_last = TK - (TK - 1) // w.chunk_rows * w.chunk_rows
         assert torch.equal(step.dlogits[:n_last][-100:], d_last)
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen"])
+def test_graph_mode_equals_host_synced_step(name):
+    """The step captured as two CUDA graphs (the loss reads the kept count on the device) gives
+    the same selection, loss, logp and dlogits as the host-synced step, on two replays."""
+    import torch
+    w, b, step, h = build(name, chunk_rows=0)
+    step.run()
+    torch.cuda.synchronize()
+    TK = step.T_kept
+    ref_loss = float(step.loss.item())
+    ref_logp = step.logp[:TK].clone()
+    ref_dl = step.dlogits[:TK].clone()
+    ref_keep = step.keep.clone()
+    step.capture()
+    for _ in range(2):
+        step.loss.zero_()
+        assert step.run_graph() == TK
+        assert float(step.loss.item()) == ref_loss
+        assert torch.equal(step.keep, ref_keep)
+        assert torch.equal(step.logp[:TK], ref_logp)
+        assert torch.equal(step.dlogits[:TK], ref_dl)
+        assert int(step.status.item()) == 0
