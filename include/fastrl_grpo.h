@@ -268,6 +268,15 @@ grpo_status grpo_loss_fwd_bwd_noalloc(const void* logits, int32_t logits_dtype,
 grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int32_t chunks);
 
 /*
+ * grpo_test_skip_copy — test hook for the bounded-wait path (no counterpart in the paper).
+ * With enable != 0, the next grpo_loss_fwd_bwd / grpo_loss_fwd_bwd_dev launch arms the first
+ * copy of its first row in one CTA but never issues it.  That CTA's wait runs out after about
+ * one second: the kernel ORs GRPO_DEVFLAG_TIMEOUT into the status word and returns normally
+ * (that launch's results are invalid); the context stays usable.  Not for production use.
+ */
+grpo_status grpo_test_skip_copy(int32_t enable);
+
+/*
  * Adaptive rollout sampling state, Algorithm 1 (the "adaptive sampling state" and the two
  * epoch-level buffers).  Plain data: it may be copied or saved and restored byte for byte.
  */

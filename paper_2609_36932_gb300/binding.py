@@ -32,7 +32,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
            "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
-           "grpo_loss_tune", "grpo_ars_init", "adaptive_rollout_count"]
+           "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
 class GrpoError(RuntimeError):
@@ -95,6 +95,8 @@ def lib():
     L.grpo_logp_fwd.restype = _i32
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
     L.grpo_sum_f64.restype = _i32
+    L.grpo_test_skip_copy.argtypes = [_i32]
+    L.grpo_test_skip_copy.restype = _i32
     L.grpo_loss_tune.argtypes = [_i32, _i32, _i32]
     L.grpo_loss_tune.restype = _i32
     L.grpo_ars_init.argtypes = [ctypes.POINTER(ArsState), _i32]

@@ -26,6 +26,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <map>
 #include <mutex>
@@ -76,6 +77,7 @@ struct LossArgs {
   // denom_from_counts the token-mean denominator is T_kept and Eq. 1's n_seq is K.
   const int64_t* counts;
   int32_t denom_from_counts;
+  int32_t skip_copy;  // test hook (grpo_test_skip_copy): one copy is armed but never issued
 };
 
 // ---- PTX helpers ------------------------------------------------------------------------------
@@ -264,8 +266,15 @@ __device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float 
 
 // kBwd = false: forward only (log-probabilities of the sampled tokens, no gradient, no loss);
 // each chunk is refilled with the next row as soon as the CTA has reduced its slice.
-template <typename InT, typename OutT, int kThreads, bool kBwd>
-__global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
+// kCap: compile for 1536 resident threads per SM (40 registers; 1024 threads when the output is
+// wider than the input).  Used when the slice is small enough that shared memory would allow
+// that many threads; otherwise the register count is free and the compiler schedules better.
+template <typename InT, typename OutT>
+constexpr int kResidentThreads = sizeof(OutT) > sizeof(InT) ? 1024 : 1536;
+
+template <typename InT, typename OutT, int kThreads, bool kBwd, bool kCap>
+__global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> / kThreads : 0)
+    grpo_loss_kernel(const LossArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
   constexpr int kPairs = Fmt<InT>::kPairs;
   constexpr int kWarps = kThreads / 32;
@@ -308,28 +317,39 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
     const int64_t src = a.row_index ? a.row_index[row] : row;
     return a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
   };
-  auto issue_chunk = [&](const char* g, int k) {  // thread 0 only
+  // Copies thread 0 armed whose completion no wait of thread 0 has seen yet (bit k: chunk k, with
+  // the phase parity in pend_par); drained before the CTA exits.
+  uint32_t pend = 0, pend_par = 0;
+  auto issue_chunk = [&](const char* g, int k, uint32_t parity) {  // thread 0 only
     const int v0 = k * a.chunk_vecs;
     const int v1 = min(nvec, v0 + a.chunk_vecs);
     const uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
     mbar_expect_tx(bar_s + 8 * k, bytes);
     if (bytes) bulk_copy_g2s(buf_s + v0 * 16, g + (int64_t)v0 * 16, bytes, bar_s + 8 * k);
+    pend |= 1u << k;
+    pend_par = (pend_par & ~(1u << k)) | (parity << k);
   };
-  auto wait_bar = [&](uint32_t bar, uint32_t parity) {  // bounded: about kWaitLimitNs
-    if (*(volatile int*)abort_flag) return;
-    if (mbar_try_wait(bar, parity)) return;
+  // Bounded wait (about kWaitLimitNs).  A copy that never lands sets GRPO_DEVFLAG_TIMEOUT and
+  // the abort flag, after which this CTA stops waiting for and issuing copies (its results are
+  // then invalid) but still completes every exchange, so no peer writes into a CTA that left.
+  auto wait_bar = [&](uint32_t bar, uint32_t parity, bool copy) -> bool {  // true: phase done
+    if (copy && *(volatile int*)abort_flag) return false;
+    if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 1; !mbar_try_wait(bar, parity); ++it) {
       if ((it & 63u) != 0) continue;
-      if (*(volatile int*)abort_flag) return;
+      if (copy && *(volatile int*)abort_flag) return false;
       if (global_timer_ns() - t0 > kWaitLimitNs) {
-        *(volatile int*)abort_flag = 1;
+        if (copy) *(volatile int*)abort_flag = 1;
         if (a.status) atomicOr(a.status, GRPO_DEVFLAG_TIMEOUT);
-        return;
+        return false;
       }
     }
+    return true;
   };
-  auto wait_chunk = [&](int k, uint32_t parity) { wait_bar(bar_s + 8 * k, parity); };
+  auto wait_chunk = [&](int k, uint32_t parity) {
+    if (wait_bar(bar_s + 8 * k, parity, true) && tid == 0) pend &= ~(1u << k);
+  };
 
   int64_t n_rows = a.n_rows;
   double inv_denom = a.inv_denom;
@@ -349,7 +369,14 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
   uint32_t iter = 0;   // rows done; exchange slot = iter & 1, its parity = (iter >> 1) & 1
   if (tid == 0 && row < n_rows) {
     const char* g = row_base(row);
-    for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
+    for (int k = 0; k < a.n_chunks; ++k) {
+      if (a.skip_copy && k == 0 && row == 0 && rank == 0) {  // test hook: arm, never copy
+        mbar_expect_tx(bar_s, 16u);
+        pend |= 1u;
+        continue;
+      }
+      issue_chunk(g, k, 0u);
+    }
   }
 
   for (; row < n_rows; row += ncl, phase ^= 1u, ++iter) {
@@ -443,14 +470,14 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
         __syncwarp();
         if (lane == 0 && row + ncl < n_rows && !*(volatile int*)abort_flag) {
           const char* g = row_base(row + ncl);
-          for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k);
+          for (int k = 0; k < a.n_chunks; ++k) issue_chunk(g, k, phase ^ 1u);
         }
       }
     }
 
     // ---- exchange and row scalars (warp 0) ----
     if (warp == 0) {
-      wait_bar(xbar_s + 8 * slot, (iter >> 1) & 1u);  // every CTA's entry has landed here
+      wait_bar(xbar_s + 8 * slot, (iter >> 1) & 1u, false);  // every CTA's entry is here
       const float4* ex = exch + slot * kMaxCluster;
       float mc = -INFINITY, sc = 0.f;
       if (lane < (int)C) {
@@ -572,9 +599,13 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_kernel(const LossArgs a) {
           for (int e = tail0 + tid; e < len; e += kThreads) Fmt<OutT>::store(orow + e, 0.f);
       }
       __syncthreads();  // chunk k consumed by every thread
-      if (gnext && !*(volatile int*)abort_flag) issue_chunk(gnext, k);
+      if (gnext && !*(volatile int*)abort_flag) issue_chunk(gnext, k, phase ^ 1u);
     }
     }  // kBwd
+  }
+  if (tid == 0) {  // copies still in flight into this CTA's shared memory land before it exits
+    for (int k = 0; k < a.n_chunks; ++k)
+      if ((pend >> k) & 1u) wait_bar(bar_s + 8 * k, (pend_par >> k) & 1u, false);
   }
   cluster_sync();  // partners are done reading this CTA's shared memory
 }
@@ -601,31 +632,44 @@ struct Tune {
 };
 Tune g_tune;
 std::mutex g_mu;
+std::atomic<int> g_skip_copy{0};
 std::map<std::tuple<const void*, int, int, int>, int> g_max_clusters;  // (kernel, dev, C, smem)
 std::map<std::pair<const void*, int>, size_t> g_smem_attr;            // (kernel, dev) -> bytes set
 
 using KernelFn = void (*)(LossArgs);
 
-template <typename InT, typename OutT, bool kBwd = true>
-KernelFn pick_kernel(int threads) {
+template <typename InT, typename OutT, bool kBwd, bool kCap>
+KernelFn pick_threads(int threads) {
   switch (threads) {
-    case 128: return grpo_loss_kernel<InT, OutT, 128, kBwd>;
-    case 512: return grpo_loss_kernel<InT, OutT, 512, kBwd>;
-    default: return grpo_loss_kernel<InT, OutT, 256, kBwd>;
+    case 128: return grpo_loss_kernel<InT, OutT, 128, kBwd, kCap>;
+    case 512: return grpo_loss_kernel<InT, OutT, 512, kBwd, kCap>;
+    default: return grpo_loss_kernel<InT, OutT, 256, kBwd, kCap>;
   }
 }
 
-KernelFn fwd_kernel_for(int in_dtype, int threads) {
-  return in_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16, false>(threads)
-                                     : pick_kernel<float, float, false>(threads);
+template <typename InT, typename OutT, bool kBwd = true>
+KernelFn pick_kernel(int threads, bool cap) {
+  return cap ? pick_threads<InT, OutT, kBwd, true>(threads) : pick_threads<InT, OutT, kBwd, false>(threads);
 }
 
-KernelFn kernel_for(int in_dtype, int out_dtype, int threads) {
+KernelFn fwd_kernel_for(int in_dtype, int threads, bool cap) {
+  return in_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16, false>(threads, cap)
+                                     : pick_kernel<float, float, false>(threads, cap);
+}
+
+KernelFn kernel_for(int in_dtype, int out_dtype, int threads, bool cap) {
   if (in_dtype == GRPO_DTYPE_BF16)
-    return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16>(threads)
-                                        : pick_kernel<__nv_bfloat16, float>(threads);
-  return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<float, __nv_bfloat16>(threads)
-                                      : pick_kernel<float, float>(threads);
+    return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16>(threads, cap)
+                                        : pick_kernel<__nv_bfloat16, float>(threads, cap);
+  return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<float, __nv_bfloat16>(threads, cap)
+                                      : pick_kernel<float, float>(threads, cap);
+}
+
+// Whether shared memory would let more than 1024 threads of this shape reside on an SM (then the
+// register-capped instance keeps that occupancy).
+bool want_cap(size_t smem, int threads) {
+  const size_t per_sm = 228 * 1024, reserved = 1024;
+  return (per_sm / (smem + reserved)) * (size_t)threads > 1024;
 }
 
 // Launch shape of the row kernel for a vocabulary of V entries of in_bytes each.
@@ -744,6 +788,12 @@ grpo_status launch_rows(KernelFn fn, const Shape& sh, LossArgs a, cudaStream_t s
 
 using namespace fastrl;
 
+extern "C" grpo_status grpo_test_skip_copy(int32_t enable) {
+  clear_error();
+  g_skip_copy.store(enable ? 1 : 0);
+  return GRPO_OK;
+}
+
 extern "C" grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int32_t chunks) {
   clear_error();
   if (cluster_ctas < 0 || cluster_ctas > kMaxCluster)
@@ -857,8 +907,10 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   a.out_vec = (reinterpret_cast<uintptr_t>(dlogits) % 16 == 0) && (((int64_t)V * out_bytes) % 16 == 0);
   a.counts = counts;
   a.denom_from_counts = from_counts ? 1 : 0;
+  a.skip_copy = g_skip_copy.exchange(0);
 
-  st = launch_rows(kernel_for(logits_dtype, dlogits_dtype, sh.threads), sh, a, s, who);
+  st = launch_rows(kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads)),
+                   sh, a, s, who);
   if (st != GRPO_OK) return st;
   sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, n_rows, counts, loss_out);
   count_launches(2);
@@ -927,7 +979,8 @@ extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, i
   a.logp_out = logp_out;
   a.status = status;
   a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
-  st = launch_rows(fwd_kernel_for(logits_dtype, sh.threads), sh, a, as_stream(stream), who);
+  st = launch_rows(fwd_kernel_for(logits_dtype, sh.threads, want_cap(sh.smem, sh.threads)), sh, a,
+                   as_stream(stream), who);
   if (st != GRPO_OK) return st;
   count_launches(1);
   return GRPO_OK;

@@ -289,3 +289,22 @@ def test_device_row_count_matches_host_count(grpo, agg_mode):
         torch.cuda.synchronize()
         assert la.item() == lb.item()
         assert torch.equal(dl_a, dl_b)  # rows past T_kept untouched (still zero) in both
+
+
+def test_lost_copy_times_out_and_the_context_stays_usable(grpo, oracle_mod):
+    """Failure detection without a fault: the test hook arms one copy that is never issued.  The
+    waiting CTA gives up after about a second, the kernel reports GRPO_DEVFLAG_TIMEOUT and
+    returns; the next launch on the same context is correct."""
+    import time
+    rng = np.random.default_rng(99)
+    c = Case(rng, 24, 152064, "bf16", "bf16")
+    grpo.binding.lib().grpo_test_skip_copy(1)
+    t0 = time.time()
+    bad = c.run_gpu(grpo)
+    elapsed = time.time() - t0
+    assert bad["status"] & grpo.binding.DEVFLAG_TIMEOUT
+    assert elapsed < 30.0
+    good = c.run_gpu(grpo)
+    assert good["status"] == 0
+    compare(good["logp"], good["dlogits"], good["loss"], c.run_oracle(oracle_mod), "bf16",
+            gpu_row_loss=good["row_loss"])
