@@ -8,8 +8,9 @@ Zipf(1.1) rank bias plus N(0, 2^2) noise, keep ratio 0.5, bf16 dlogits.  The log
 token (~16 GB) are resident before timing; the loss reads only the kept rows.
 
 Output: one JSON line (rank 0).  `value` is kept tokens per second over all ranks (device
-time, CUDA events); `e2e` repeats the step with the inputs copied from pinned host memory and
-the loss read back inside the timed region; `roofline` relates the loss kernel's event-timed
+time, CUDA events); `e2e` repeats the step from inputs in pinned host memory (the selection
+inputs copied whole, then only the kept rollouts' logit rows) with the loss read back, all inside
+the timed region; `roofline` relates the loss kernel's event-timed
 duration to the measured HBM copy bandwidth; `cpu_baseline` times the fp64 oracle on a bounded
 sample on this machine's host cores.  `--impl reference` times that oracle as the reference
 arm.  Under torchrun each rank runs its own batch (weak scaling); the only collectives are the
@@ -438,31 +439,27 @@ def main():
             host[k] = torch.empty(d[k].shape, dtype=d[k].dtype, pin_memory=True)
             host[k].copy_(d[k])
         loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
-        d2h = 8 + 16 + 4 * w.P
-        step.run()
+        step.run_from_host(host, loss_host)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        kept_e = 0
+        kept_e, h2d_e, d2h_e = 0, 0, 0
         e0.record(stream)
         for _ in range(args.e2e_steps):
-            for k in names:
-                d[k].copy_(host[k], non_blocking=True)
-            if use_graph:
-                step.replay_select()
-                step.replay_loss()
-                loss_host.copy_(step.loss, non_blocking=True)
-                step.finish()
-            else:
-                step.run()
-                loss_host.copy_(step.loss, non_blocking=True)
+            hb, db = step.run_from_host(host, loss_host)
+            h2d_e += hb
+            d2h_e += db
             kept_e += step.T_kept
         e1.record(stream)
         torch.cuda.synchronize()
         e_ms, kept_e = combine_ranks(e0.elapsed_time(e1), kept_e, world, dev)
-        e2e = {"value": kept_e / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "steps": args.e2e_steps}
+        e2e = {"value": kept_e / (e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d_e // args.e2e_steps),
+               "d2h_bytes_per_step": int(d2h_e // args.e2e_steps), "steps": args.e2e_steps,
+               "host_inputs_bytes": int(h2d),
+               "transfer": "selection inputs and per-token log-probs whole; logits of the kept "
+                           "rollouts only (grpo_upload_kept), after the selection"}
         del host
 
     cpu = None

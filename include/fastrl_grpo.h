@@ -7,6 +7,7 @@
  *   grpo_advantage          group-relative advantages                          (Eq. 5)
  *   grpo_prune              maximising-differential advantage pruning (MDAP)   (Eqs. 6-9, Algorithm 1)
  *   grpo_compact            compaction of the kept rollouts' tokens            (Sec. 3.2, after Eq. 9)
+ *   grpo_upload_kept        host-to-device copy of the kept rollouts' rows      (Sec. 3.2)
  *   grpo_loss_fwd_bwd       fused GRPO token loss, forward and dlogits         (Eqs. 1-3)
  *   adaptive_rollout_count  host-side adaptive rollout sampling (ARS)          (Eqs. 10-14, Algorithm 1)
  *
@@ -140,6 +141,29 @@ grpo_status grpo_compact(const uint8_t* keep, const int64_t* off, int32_t n_roll
                          int32_t* kept_idx, int64_t* kept_off, int64_t* src_token,
                          int32_t* token_rollout, int64_t* counts, int64_t* counts_host,
                          grpo_stream_t stream);
+
+/*
+ * grpo_upload_kept — host-to-device transfer of the kept rollouts' token rows only.  Sec. 3.2
+ * feeds only the retained trajectories to the models, so a step whose per-token inputs (for
+ * instance logits) live in host memory need not move the pruned rollouts' rows at all.
+ * For every maximal run of consecutive kept rollouts i..j (keep_host[r] != 0) one
+ * cudaMemcpyAsync on `stream` copies bytes [off_host[i]*row_bytes, off_host[j+1]*row_bytes) of
+ * src_host to the same offset of dst_dev.  Rows of pruned rollouts in dst_dev are not written.
+ * src_host   host, token rows of row_bytes bytes in `off_host` layout.  Pinned memory makes the
+ *            copies asynchronous; the runtime copies pageable memory synchronously.
+ * dst_dev    device, the same layout and size.
+ * keep_host  host u8 [n_rollouts] (grpo_prune's keep, copied back); off_host host i64
+ *            [n_rollouts+1], off_host[0] >= 0 and non-decreasing.
+ * bytes_out, copies_out  host, nullable: bytes and copies enqueued.
+ * Errors (before any copy is enqueued): GRPO_ERR_INVALID_ARG for a NULL array with
+ * n_rollouts > 0, n_rollouts < 0, row_bytes <= 0, decreasing or negative offsets, or a byte
+ * offset that overflows int64.  GRPO_ERR_CUDA if a copy cannot be enqueued (copies enqueued
+ * before it stay enqueued).  No kernel is launched.
+ */
+grpo_status grpo_upload_kept(const void* src_host, void* dst_dev, int64_t row_bytes,
+                             const uint8_t* keep_host, const int64_t* off_host,
+                             int32_t n_rollouts, int64_t* bytes_out, int32_t* copies_out,
+                             grpo_stream_t stream);
 
 /*
  * grpo_loss_fwd_bwd — fused GRPO token loss and its gradient w.r.t. the logits, Eqs. 1-3.

@@ -31,7 +31,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
+           "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -78,6 +78,8 @@ def lib():
     L.grpo_prune.restype = _i32
     L.grpo_compact.argtypes = [_c_p, _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
     L.grpo_compact.restype = _i32
+    L.grpo_upload_kept.argtypes = [_c_p, _c_p, _i64, _c_p, _c_p, _i32, _c_p, _c_p, _c_p]
+    L.grpo_upload_kept.restype = _i32
     L.grpo_loss_fwd_bwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
                                     _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p, _c_p,
                                     _c_p, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
@@ -255,6 +257,39 @@ def grpo_compact(keep, off, kept_idx=None, kept_off=None, src_token=None, token_
                               _ptr(src_token), _ptr(token_rollout), _ptr(counts), hp, _stream(stream)))
     return dict(kept_idx=kept_idx, kept_off=kept_off, src_token=src_token,
                 token_rollout=token_rollout, counts=counts)
+
+
+def grpo_upload_kept(src_host, dst, keep_host, off_host, stream=None):
+    """Copy the kept rollouts' token rows of `src_host` (a host tensor, pinned for the copies to be
+    asynchronous) into the same rows of the device tensor `dst`.  keep_host: host u8
+    [n_rollouts]; off_host: host i64 [n_rollouts+1].  Rows are dim 0 of src_host and dst.
+    Returns (bytes, copies) enqueued on the stream."""
+    torch = _torch()
+    if src_host.is_cuda or not dst.is_cuda:
+        raise ValueError("grpo_upload_kept: src_host must be a host tensor and dst a device tensor")
+    if src_host.shape != dst.shape or src_host.dtype != dst.dtype:
+        raise ValueError("grpo_upload_kept: src_host and dst differ in shape or dtype")
+    if not (src_host.is_contiguous() and dst.is_contiguous()):
+        raise ValueError("grpo_upload_kept: src_host and dst must be contiguous")
+    if keep_host.is_cuda or off_host.is_cuda:
+        raise ValueError("grpo_upload_kept: keep_host and off_host must be host tensors")
+    if keep_host.dtype != torch.uint8 or off_host.dtype != torch.int64:
+        raise TypeError("grpo_upload_kept: keep_host must be uint8 and off_host int64")
+    if not (keep_host.is_contiguous() and off_host.is_contiguous()):
+        raise ValueError("grpo_upload_kept: keep_host and off_host must be contiguous")
+    n = keep_host.numel()
+    if off_host.numel() < n + 1:
+        raise ValueError("grpo_upload_kept: off_host needs n_rollouts + 1 entries")
+    rows = src_host.shape[0] if src_host.dim() else 1
+    if n and int(off_host[n]) > rows:
+        raise ValueError("grpo_upload_kept: off_host[-1] = %d exceeds the %d rows"
+                         % (int(off_host[n]), rows))
+    row_bytes = src_host.numel() * src_host.element_size() // max(rows, 1)
+    nbytes, ncopies = ctypes.c_int64(0), ctypes.c_int32(0)
+    _check(lib().grpo_upload_kept(_ptr(src_host), _ptr(dst), row_bytes, _ptr(keep_host),
+                                  _ptr(off_host), n, ctypes.byref(nbytes), ctypes.byref(ncopies),
+                                  _stream(stream)))
+    return nbytes.value, ncopies.value
 
 
 def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int | None = None,

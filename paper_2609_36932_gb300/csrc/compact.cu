@@ -115,12 +115,12 @@ extern "C" grpo_status grpo_compact(const uint8_t* keep, const int64_t* off, int
   if (n_rollouts < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_compact: n_rollouts < 0");
   if (!off || !kept_off || !counts || (n_rollouts > 0 && (!keep || !kept_idx)))
     return fail(GRPO_ERR_INVALID_ARG, "grpo_compact: NULL array");
+  if (n_rollouts > 0 && (!src_token || !token_rollout))
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_compact: NULL token arrays");
   cudaStream_t s = as_stream(stream);
   compact_scan_kernel<<<1, kScanThreads, 0, s>>>(keep, off, n_rollouts, kept_idx, kept_off, counts);
   int launches = 1;
   if (n_rollouts > 0) {
-    if (!src_token || !token_rollout)
-      return fail(GRPO_ERR_INVALID_ARG, "grpo_compact: NULL token arrays");
     compact_fill_kernel<<<n_rollouts, 256, 0, s>>>(keep, off, kept_idx, kept_off, counts, src_token,
                                                     token_rollout);
     ++launches;
@@ -133,6 +133,53 @@ extern "C" grpo_status grpo_compact(const uint8_t* keep, const int64_t* off, int
         cudaMemcpyAsync(counts_host, counts, 2 * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
     if (e != cudaSuccess)
       return fail(GRPO_ERR_CUDA, "grpo_compact: copy of counts: %s", cudaGetErrorString(e));
+  }
+  return GRPO_OK;
+}
+
+extern "C" grpo_status grpo_upload_kept(const void* src_host, void* dst_dev, int64_t row_bytes,
+                                        const uint8_t* keep_host, const int64_t* off_host,
+                                        int32_t n_rollouts, int64_t* bytes_out,
+                                        int32_t* copies_out, grpo_stream_t stream) {
+  clear_error();
+  if (bytes_out) *bytes_out = 0;
+  if (copies_out) *copies_out = 0;
+  if (n_rollouts < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_upload_kept: n_rollouts < 0");
+  if (row_bytes <= 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_upload_kept: row_bytes <= 0");
+  if (n_rollouts == 0) return GRPO_OK;
+  if (!src_host || !dst_dev || !keep_host || !off_host)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_upload_kept: NULL array");
+  if (off_host[0] < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_upload_kept: off_host[0] < 0");
+  for (int32_t r = 0; r < n_rollouts; ++r)
+    if (off_host[r + 1] < off_host[r])
+      return fail(GRPO_ERR_INVALID_ARG, "grpo_upload_kept: off_host decreases at %d", r);
+  if (off_host[n_rollouts] > INT64_MAX / row_bytes)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_upload_kept: byte offsets overflow int64");
+  cudaStream_t s = as_stream(stream);
+  const char* src = static_cast<const char*>(src_host);
+  char* dst = static_cast<char*>(dst_dev);
+  int64_t bytes = 0;
+  int32_t copies = 0;
+  for (int32_t r = 0; r < n_rollouts;) {
+    if (!keep_host[r]) {
+      ++r;
+      continue;
+    }
+    int32_t e = r;
+    while (e < n_rollouts && keep_host[e]) ++e;  // kept run r..e-1
+    const int64_t b0 = off_host[r] * row_bytes, n = (off_host[e] - off_host[r]) * row_bytes;
+    if (n > 0) {
+      const cudaError_t err =
+          cudaMemcpyAsync(dst + b0, src + b0, (size_t)n, cudaMemcpyHostToDevice, s);
+      if (err != cudaSuccess)
+        return fail(GRPO_ERR_CUDA, "grpo_upload_kept: copy of rollouts %d..%d: %s", r, e - 1,
+                    cudaGetErrorString(err));
+      bytes += n;
+      ++copies;
+      if (bytes_out) *bytes_out = bytes;
+      if (copies_out) *copies_out = copies;
+    }
+    r = e;
   }
   return GRPO_OK;
 }

@@ -64,6 +64,7 @@ class GrpoStep:
         self.counts = torch.empty(2, dtype=torch.int64, device=dev)
         self.counts_host = torch.empty(2, dtype=torch.int64, pin_memory=True)
         self.kpp_host = torch.empty(max(self.P, 1), dtype=torch.int32, pin_memory=True)
+        self.keep_host = torch.empty(max(n, 1), dtype=torch.uint8, pin_memory=True)
         self.loss = torch.empty(1, dtype=torch.float64, device=dev)
         self.logp = torch.empty(max(self.T, 1), dtype=torch.float32, device=dev)
         self.out_dtype = torch.bfloat16 if params.dlogits_dtype == "bf16" else torch.float32
@@ -97,14 +98,7 @@ class GrpoStep:
                        counts=self.counts, counts_host=self.counts_host)
         self.kpp_host[:self.P].copy_(self.kpp[:self.P], non_blocking=True)
         self.torch.cuda.current_stream().synchronize()
-        self.K = int(self.counts_host[0])
-        self.T_kept = int(self.counts_host[1])
-        # Algorithm 1, Phase 1(b) then 1(a): the rollout count for the next step.
-        self.step_index += 1
-        s = (self.step_index - 1) % self.ars_total + 1
-        self.n_next = B.adaptive_rollout_count(self.ars, self.kpp_host[:self.P].numpy(), s,
-                                               self.ars_total, s % self.steps_per_epoch == 0)
-        return self.T_kept
+        return self._read_counts()
 
     def set_workspaces(self):
         """Allocate persistent workspaces (sizes from the library's queries)."""
@@ -167,6 +161,7 @@ class GrpoStep:
                        counts=self.counts)
         self.counts_host.copy_(self.counts, non_blocking=True)
         self.kpp_host[:self.P].copy_(self.kpp[:self.P], non_blocking=True)
+        self.keep_host[:self.keep.numel()].copy_(self.keep, non_blocking=True)
 
     def _enqueue_loss(self):
         p = self.p
@@ -204,6 +199,11 @@ class GrpoStep:
     def finish(self):
         """After a replayed step: wait for it, read the kept counts and update ARS (Phase 1b)."""
         self.torch.cuda.current_stream().synchronize()
+        return self._read_counts()
+
+    def _read_counts(self):
+        """Kept counts from the host copies; then Algorithm 1, Phase 1(b) then 1(a): the rollout
+        count for the next step."""
         self.K = int(self.counts_host[0])
         self.T_kept = int(self.counts_host[1])
         self.step_index += 1
@@ -221,6 +221,45 @@ class GrpoStep:
         self.select()
         self.loss_step()
         return self.loss
+
+    # ---- inputs in pinned host memory ---------------------------------------------------------
+
+    SMALL_INPUTS = ("rewards", "ids", "off", "old", "ref")
+
+    def run_from_host(self, host: dict, loss_host=None):
+        """One step whose inputs start in host memory (pinned, for asynchronous copies): `host`
+        holds tensors 'rewards', 'ids', 'off', 'old', 'ref' and 'logits' shaped like the device
+        inputs.  The selection inputs and the per-token log-probs are copied whole; after the
+        selection, only the kept rollouts' logit rows are copied (grpo_upload_kept), since the
+        pruned rollouts take no further part in the step (Sec. 3.2).  Uses the captured graphs
+        when `capture()` has run.  The loss is copied into `loss_host` (f64 [1]) if given.
+        Returns (h2d_bytes, d2h_bytes) moved by this step."""
+        torch = self.torch
+        dev_of = dict(rewards=self.rewards, ids=self.ids, off=self.off, old=self.old, ref=self.ref)
+        h2d = 0
+        for k in self.SMALL_INPUTS:
+            dev_of[k].copy_(host[k], non_blocking=True)
+            h2d += host[k].numel() * host[k].element_size()
+        graphed = getattr(self, "g_select", None) is not None
+        if graphed:
+            self.replay_select()
+        else:
+            self._enqueue_select()
+        torch.cuda.current_stream().synchronize()
+        self._read_counts()
+        n = self.keep.numel()
+        up, _ = B.grpo_upload_kept(host["logits"], self.logits, self.keep_host[:n], host["off"])
+        h2d += up
+        if graphed:
+            self.replay_loss()
+        else:
+            self.loss_step()
+        d2h = 2 * 8 + 4 * self.P + n
+        if loss_host is not None:
+            loss_host.copy_(self.loss, non_blocking=True)
+            d2h += 8
+        torch.cuda.current_stream().synchronize()
+        return h2d, d2h
 
     def kept_rows(self):
         """(src_token, token_rollout) of the kept rows as host arrays."""

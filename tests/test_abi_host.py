@@ -94,6 +94,32 @@ def test_argument_errors_return_status_without_gpu_work(grpo):
     assert b"cluster" in L.grpo_last_error() or L.grpo_last_error() == b""
 
 
+def test_upload_kept_argument_errors(grpo):
+    """grpo_upload_kept validates everything before its first copy; with nothing kept it
+    enqueues nothing, so these calls need no device."""
+    L = raw()
+    keep = np.array([1, 0, 1, 1], np.uint8)
+    off = np.array([0, 3, 5, 9, 12], np.int64)
+    src, dst = ctypes.c_void_p(4096), ctypes.c_void_p(8192)  # never dereferenced here
+    nb, nc = ctypes.c_int64(-1), ctypes.c_int32(-1)
+
+    def call(k, o, n, row_bytes=64, s=src, d=dst):
+        return L.grpo_upload_kept(s, d, row_bytes, k.ctypes.data if k is not None else None,
+                                  o.ctypes.data if o is not None else None, n,
+                                  ctypes.byref(nb), ctypes.byref(nc), None)
+
+    assert call(keep, off, -1) == 1
+    assert call(keep, off, 4, row_bytes=0) == 1
+    assert call(None, off, 4) == 1 and call(keep, None, 4) == 1
+    assert call(keep, off, 4, s=None) == 1 and call(keep, off, 4, d=None) == 1
+    assert call(keep, np.array([0, 3, 2, 9, 12], np.int64), 4) == 1  # decreasing
+    assert call(keep, np.array([-1, 3, 5, 9, 12], np.int64), 4) == 1
+    assert call(keep, np.array([0, 3, 5, 9, 1 << 40], np.int64), 4, row_bytes=1 << 30) == 1
+    assert b"overflow" in L.grpo_last_error()
+    assert call(keep, off, 0) == 0 and (nb.value, nc.value) == (0, 0)
+    assert call(np.zeros(4, np.uint8), off, 4) == 0 and (nb.value, nc.value) == (0, 0)
+
+
 def loss_call(L, n_rows, V, ws, size_p, ldt=1, agg=0, denom=1, row_loss=None, beta=0.04):
     return L.grpo_loss_fwd_bwd(None, ldt, V, None, n_rows, V, None, None, None, None, None, 0.2,
                                0.2, beta, agg, denom, None, 0, None, 1, None, row_loss, None, None,

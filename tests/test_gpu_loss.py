@@ -17,7 +17,7 @@ def bf16_bits(x):
 
 class Case:
     def __init__(self, rng, n, V, in_dtype="bf16", out_dtype="bf16", scale=2.0, n_roll=4,
-                 stride=None, beta=0.04, A=None):
+                 stride=None, beta=0.04, A=None, old_noise=0.05):
         import torch
         self.n, self.V, self.in_dtype, self.out_dtype = n, V, in_dtype, out_dtype
         self.stride = V if stride is None else stride
@@ -34,7 +34,7 @@ class Case:
         zz = zf[:, :V].astype(np.float64)
         m = zz.max(1, keepdims=True)
         logp = zz[np.arange(n), self.y] - (m[:, 0] + np.log(np.exp(zz - m).sum(1)))
-        self.old = (logp + 0.05 * rng.standard_normal(n)).astype(np.float32)
+        self.old = (logp + old_noise * rng.standard_normal(n)).astype(np.float32)
         self.ref = (logp + 0.1 * rng.standard_normal(n)).astype(np.float32)
         self.adv = (rng.standard_normal(n_roll) if A is None else np.asarray(A)).astype(np.float32)
         self.rr = rng.integers(0, self.adv.size, size=n).astype(np.int32)
@@ -168,6 +168,29 @@ def test_sequence_mean(grpo, oracle_mod):
     r = oracle_mod.loss(c.host, c.V, c.y, c.old, c.ref, c.adv, rr, agg_mode=1, seq_off=seq_off,
                         n_seq=n_seq, dlogits_dtype=1, beta=c.beta)
     compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+
+
+@pytest.mark.parametrize("beta", [0.0, 0.04])
+def test_asymmetric_clip(grpo, oracle_mod, beta):
+    """Eq. 2 with different lower and upper clip widths (eps_low 0.2, eps_high 0.28).  Old
+    log-probs far from the current ones put many rows outside the clip range on both sides.
+    Where the clip is active (A > 0 above 1 + eps_high, A < 0 below 1 - eps_low) the surrogate
+    is constant, so with beta = 0 those rows' gradient is exactly zero."""
+    rng = np.random.default_rng(12)
+    c = Case(rng, 96, 32000, "bf16", "bf16", beta=beta, old_noise=0.35, n_roll=8)
+    g = c.run_gpu(grpo, eps_low=0.2, eps_high=0.28)
+    r = c.run_oracle(oracle_mod, eps_low=0.2, eps_high=0.28)
+    assert g["status"] == 0
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", eps_low=0.2, eps_high=0.28,
+            gpu_row_loss=g["row_loss"])
+    A = c.adv[c.rr].astype(np.float64)
+    rho = r["rho"][:c.n]
+    active = ((A > 0) & (rho > 1.28 * (1 + 1e-5))) | ((A < 0) & (rho < 0.8 * (1 - 1e-5)))
+    inside = (rho > 0.8 * (1 + 1e-5)) & (rho < 1.28 * (1 - 1e-5)) & (A != 0)
+    assert active.sum() >= 10 and inside.sum() >= 10
+    if beta == 0.0:
+        assert np.all((g["dlogits"][active] & 0x7FFF) == 0)
+        assert np.all(np.any(g["dlogits"][inside] & 0x7FFF, axis=1))
 
 
 def test_deterministic(grpo):

@@ -3,6 +3,8 @@ advantage -> prune -> compact -> loss over the kept rows.  'tiny' and 'small' ar
 with the oracle row by row in full; the three Qwen-vocabulary workloads at full size are
 compared on sampled rows, and their total loss through a property that holds at any size
 (the loss is the weighted sum of Eq. 1's per-token terms evaluated at the kernel's logp)."""
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -13,7 +15,7 @@ from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
 pytestmark = pytest.mark.gpu
 
 
-def build(name, seed=0, chunk_rows=None):
+def build(name, seed=0, chunk_rows=None, **overrides):
     import torch
     w = workloads.get(name)
     b = workloads.make_batch(w, seed)
@@ -26,6 +28,7 @@ def build(name, seed=0, chunk_rows=None):
     p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
                    eps_low=w.eps, eps_high=w.eps, beta=w.beta, dlogits_dtype=w.dlogits_dtype,
                    chunk_rows=w.chunk_rows if chunk_rows is None else chunk_rows)
+    p = dataclasses.replace(p, **overrides)
     step = GrpoStep(p, rewards, ids, off, logits, old, ref)
     return w, b, step, dict(logits=logits, old=old.cpu().numpy(), ref=ref.cpu().numpy())
 
@@ -146,3 +149,124 @@ def test_graph_mode_equals_host_synced_step(name):
         assert torch.equal(step.logp[:TK], ref_logp)
         assert torch.equal(step.dlogits[:TK], ref_dl)
         assert int(step.status.item()) == 0
+
+
+VARIANTS = {
+    # DP fill to a multiple of 7, a keep cap of 3, Eq. 1's per-sequence mean, clip-higher
+    # widths and no KL term, bigram sets
+    "small-dp7-cap3-seqmean-cliphigher": ("small", dict(ngram_n=2, keep_cap=3, dp_divisor=7,
+                                                         agg_mode=1, eps_low=0.2, eps_high=0.28,
+                                                         beta=0.0)),
+    # population std, trigram sets, a tight tau, continuous-reward grouping
+    "tiny-popstd-tri-classeps": ("tiny", dict(std_mode=1, ngram_n=3, tau=0.3, class_eps=1e-4,
+                                              dp_divisor=3)),
+}
+
+
+@pytest.mark.parametrize("variant", list(VARIANTS))
+def test_step_variants(oracle_mod, variant):
+    """The whole step under non-default step parameters, compared with the oracle in full, then
+    replayed as CUDA graphs and compared with itself bit for bit."""
+    import torch
+    name, kw = VARIANTS[variant]
+    w, b, step, h = build(name, chunk_rows=0, **kw)
+    p = step.p
+    step.run()
+    torch.cuda.synchronize()
+    assert int(step.status.item()) == 0
+    adv, _ = oracle_mod.advantage(b["rewards"], w.G, p.std_mode)
+    keep, kpp = oracle_mod.prune(b["rewards"], b["ids"], b["off"], w.G, p.ngram_n, p.tau,
+                                 p.keep_cap, p.dp_divisor, adv=adv, class_eps=p.class_eps)
+    comp = oracle_mod.compact(keep, b["off"])
+    assert np.array_equal(step.adv.cpu().numpy().view(np.uint32), adv.view(np.uint32))
+    assert np.array_equal(step.keep.cpu().numpy(), keep)
+    assert np.array_equal(step.kpp[:w.P].cpu().numpy(), kpp)
+    assert (step.K, step.T_kept) == (comp["K"], comp["T_kept"])
+    assert comp["K"] % p.dp_divisor == 0
+    TK = step.T_kept
+    ref = oracle_mod.loss(host_bits(h["logits"]), w.V, b["ids"], h["old"], h["ref"], adv,
+                          comp["token_rollout"], row_index=comp["src_token"],
+                          eps_low=p.eps_low, eps_high=p.eps_high, beta=p.beta,
+                          agg_mode=p.agg_mode, denom_tokens=TK, seq_off=b["off"],
+                          n_seq=comp["K"], dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
+    compare(step.logp[:TK].cpu().numpy(), host_bits(step.dlogits[:TK]), float(step.loss.item()),
+            ref, w.dlogits_dtype, eps_low=p.eps_low, eps_high=p.eps_high)
+    loss0, dl0 = float(step.loss.item()), step.dlogits[:TK].clone()
+    step.capture()
+    assert step.run_graph() == TK
+    assert float(step.loss.item()) == loss0 and torch.equal(step.dlogits[:TK], dl0)
+
+
+def test_upload_kept_copies_only_kept_rows():
+    """grpo_upload_kept: kept rollouts' rows arrive intact, pruned rows keep their old contents,
+    one copy per run of consecutive kept rollouts, on two row widths."""
+    import torch
+    from paper_2609_36932_gb300 import binding as B
+    rng = np.random.default_rng(21)
+    for n, width, dtype in ((37, 1000, torch.bfloat16), (200, 33, torch.float32)):
+        lens = rng.integers(0, 9, size=n)
+        off = torch.from_numpy(np.concatenate([[0], np.cumsum(lens)]).astype(np.int64))
+        T = int(off[-1])
+        keep = torch.from_numpy((rng.random(n) < 0.5).astype(np.uint8))
+        src = torch.randn(T, width).to(dtype).pin_memory()
+        dst = torch.full((T, width), -7.0, dtype=dtype, device="cuda")
+        nbytes, copies = B.grpo_upload_kept(src, dst, keep, off)
+        torch.cuda.synchronize()
+        kept_row = np.repeat(keep.numpy().astype(bool), lens)
+        got = dst.cpu()
+        assert torch.equal(got[torch.from_numpy(kept_row)], src[torch.from_numpy(kept_row)])
+        assert bool((got[torch.from_numpy(~kept_row)] == -7.0).all())
+        assert nbytes == int(kept_row.sum()) * width * src.element_size()
+        # runs of kept rollouts, counting only runs that hold at least one token
+        runs, r = 0, 0
+        kk = keep.numpy().astype(bool)
+        while r < n:
+            if not kk[r]:
+                r += 1
+                continue
+            e = r
+            while e < n and kk[e]:
+                e += 1
+            runs += int(lens[r:e].sum() > 0)
+            r = e
+        assert copies == runs and runs >= 1
+
+
+@pytest.mark.parametrize("name,graph", [("tiny", False), ("tiny", True), ("small", True),
+                                        ("qwen", True)])
+def test_host_inputs_step_equals_resident_step(name, graph):
+    """A step from pinned host inputs copies only the kept rollouts' logit rows.  It gives the
+    resident step's selection, loss, logp and dlogits bit for bit, although every device input
+    was poisoned beforehand (NaN logits everywhere): no pruned row is read."""
+    import torch
+    w, b, step, h = build(name, chunk_rows=0)
+    step.run()
+    torch.cuda.synchronize()
+    TK, K = step.T_kept, step.K
+    ref_loss = float(step.loss.item())
+    ref_logp, ref_dl = step.logp[:TK].clone(), step.dlogits[:TK].clone()
+    ref_keep = step.keep.clone()
+    host = {}
+    for k in ("rewards", "ids", "off", "old", "ref", "logits"):
+        d = getattr(step, k)
+        host[k] = torch.empty(d.shape, dtype=d.dtype, pin_memory=True)
+        host[k].copy_(d)
+    if graph:
+        step.capture()
+    step.logits.fill_(float("nan"))
+    for t in (step.old, step.ref, step.rewards):
+        t.fill_(float("nan"))
+    step.ids.fill_(-1)
+    step.off.fill_(0)
+    step.status.zero_()
+    loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
+    small = sum(host[k].numel() * host[k].element_size() for k in step.SMALL_INPUTS)
+    for _ in range(2):
+        h2d, d2h = step.run_from_host(host, loss_host)
+        assert (step.T_kept, step.K) == (TK, K)
+        assert float(loss_host.item()) == ref_loss
+        assert torch.equal(step.keep, ref_keep)
+        assert torch.equal(step.logp[:TK], ref_logp) and torch.equal(step.dlogits[:TK], ref_dl)
+        assert int(step.status.item()) == 0
+        assert h2d == small + TK * w.V * host["logits"].element_size()
+        assert d2h == 16 + 4 * step.P + step.keep.numel() + 8

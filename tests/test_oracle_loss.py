@@ -124,6 +124,30 @@ def test_gradient_invariants(oracle_mod):
     np.testing.assert_allclose(ratio, ratio[:, :1].repeat(200, 1), rtol=1e-9)
 
 
+def test_asymmetric_clip_regions(oracle_mod):
+    """Eq. 2 with eps_low = 0.2, eps_high = 0.28 against the clipped surrogate's closed form,
+    one token at a time (beta = 0, denominator 1): loss = -min(rho*A, clip(rho)*A), and dlogits
+    = -A*rho*(e_y - p) where the unclipped term is the minimum, else 0.  The ratios sit between
+    the two widths (1.25, 0.75) and outside both (1.3, 0.7), so a swapped or shared width fails."""
+    z = np.array([0.5, -1.0, 2.0, 0.25, -0.5], np.float32)
+    zz = z.astype(np.float64)
+    logp = zz[0] - scipy.special.logsumexp(zz)
+    p = np.exp(zz - scipy.special.logsumexp(zz))
+    e = np.zeros(5)
+    e[0] = 1.0
+    for rho_t, A, clipped in ((1.25, 1.0, False), (1.3, 1.0, True), (0.85, 1.0, False),
+                              (0.75, -1.0, True), (0.7, -1.0, True), (0.85, -1.0, False),
+                              (1.25, -1.0, False), (0.75, 1.0, False)):
+        old = np.float32(logp - math.log(rho_t))
+        out = oracle_mod.loss(z[None, :], 5, [0], [old], [old], [A], [0], eps_low=0.2,
+                              eps_high=0.28, beta=0.0, denom_tokens=1, want_f64=True)
+        rho = math.exp(logp - float(old))
+        cl = min(max(rho, 1.0 - float(np.float32(0.2))), 1.0 + float(np.float32(0.28)))
+        assert out["loss"] == pytest.approx(-min(rho * A, cl * A), rel=1e-12)
+        expect = np.zeros(5) if clipped else -A * rho * (e - p)
+        np.testing.assert_allclose(out["dlogits_f64"][0], expect, rtol=1e-12, atol=1e-15)
+
+
 def test_zero_advantage_without_kl_gives_zero_gradient(oracle_mod):
     rng = np.random.default_rng(14)
     z = rows(rng, 5, 64)
