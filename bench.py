@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--prompts", type=int, default=0,
                     help="override the workload's prompt count (a smaller case for profiling)")
+    ap.add_argument("--group", type=int, default=0,
+                    help="override the rollouts per prompt G (a smaller case for profiling)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
@@ -322,6 +324,8 @@ def main():
     w = workloads.get(args.config)
     if args.prompts > 0:
         w = dataclasses.replace(w, P=args.prompts)
+    if args.group > 0:
+        w = dataclasses.replace(w, G=args.group)
     if args.impl == "reference":
         run_reference(args, w)
         return

@@ -678,21 +678,27 @@ struct Shape {
   size_t smem = 0;
 };
 
-grpo_status pick_shape(int V, int in_bytes, const char* who, Shape* out) {
+// out_bytes: bytes per dlogits element (2 or 4), or 0 for the forward-only instance.
+grpo_status pick_shape(int V, int in_bytes, int out_bytes, const char* who, Shape* out) {
   Tune tune;
   {
     std::lock_guard<std::mutex> lk(g_mu);
     tune = g_tune;
   }
   const int vec = 16 / in_bytes;
-  const int threads = tune.threads ? tune.threads : 256;
-  // Cluster size: slices of at most 80 KiB (two CTAs per SM), and at least two CTAs per row once
-  // a row exceeds 32 KiB.  Measured on GB300 over cluster sizes 1-16, 128-512 threads and 1-5
-  // copies per slice, this shape moved the most bytes per second for V = 32000 and 152064.
+  // Default shape, from sweeps on GB300 over cluster sizes 1-16, 128-512 threads and 1-8 copies
+  // per slice for V = 32000 and 152064, bf16 logits:
+  //  - slices of at most 80 KiB, or 40 KiB when dlogits are wider than the logits (the wider
+  //    write phase then gains from more CTAs per SM); at least two CTAs per row once a row
+  //    exceeds 32 KiB;
+  //  - 256 threads when a slice has at least 128 elements per thread, else 128;
+  //  - two bulk copies per slice (about 45% of the slice limit each) for the fused loss, one
+  //    for the forward-only instance.
+  const int64_t limit = (out_bytes > in_bytes ? 40 : 80) * 1024;
   int C = tune.cluster;
   if (C == 0) {
     const int64_t row_bytes = (int64_t)V * in_bytes;
-    C = (int)std::min<int64_t>(kMaxCluster, (row_bytes + 80 * 1024 - 1) / (80 * 1024));
+    C = (int)std::min<int64_t>(kMaxCluster, (row_bytes + limit - 1) / limit);
     if (C == 1 && row_bytes > 32 * 1024) C = 2;
   }
   int slice = (int)align_up((size_t)((V + C - 1) / C), vec);
@@ -700,10 +706,12 @@ grpo_status pick_shape(int V, int in_bytes, const char* who, Shape* out) {
     --C;
     slice = (int)align_up((size_t)((V + C - 1) / C), vec);
   }
+  const int threads = tune.threads ? tune.threads : (slice >= 128 * 256 ? 256 : 128);
   const size_t slice_bytes = (size_t)slice * in_bytes;
-  // about 36 KiB per bulk copy
+  const size_t copy = (size_t)limit * 9 / 20;
   int chunks = tune.chunks ? tune.chunks
-                           : (int)std::min<size_t>(kMaxChunks, std::max<size_t>(1, (slice_bytes + 18 * 1024) / (36 * 1024)));
+               : out_bytes == 0 ? 1
+                                : (int)std::min<size_t>(kMaxChunks, std::max<size_t>(1, (slice_bytes + copy / 2) / copy));
   const int slice_vecs = slice / vec;
   int chunk_vecs = (slice_vecs + chunks - 1) / chunks;
   if (chunk_vecs < 1) chunk_vecs = 1;
@@ -871,7 +879,7 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   const int out_bytes = dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   Shape sh;
-  st = pick_shape(V, in_bytes, who, &sh);
+  st = pick_shape(V, in_bytes, out_bytes, who, &sh);
   if (st != GRPO_OK) return st;
 
   LossArgs a = {};
@@ -967,7 +975,7 @@ extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, i
   if (!logits || !y || !logp_out) return fail(GRPO_ERR_INVALID_ARG, "%s: NULL array", who);
   const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   Shape sh;
-  grpo_status st = pick_shape(V, in_bytes, who, &sh);
+  grpo_status st = pick_shape(V, in_bytes, 0, who, &sh);
   if (st != GRPO_OK) return st;
   LossArgs a = {};
   a.logits = static_cast<const char*>(logits);

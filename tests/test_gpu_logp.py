@@ -76,19 +76,33 @@ def test_logp_gathered_rows_and_bad_ids(grpo, oracle_mod):
     assert np.abs(got[ok] - ref[ok]).max() <= LOGP_ATOL
 
 
-def test_logp_agrees_with_the_loss_kernel(grpo):
-    """The forward-only kernel and the fused loss report the same log-probabilities."""
+@pytest.mark.parametrize("V", [32000, 152064])
+def test_logp_agrees_with_the_loss_kernel(grpo, V):
+    """The forward-only kernel and the fused loss report the same log-probabilities: bit for
+    bit at one launch shape (the ratio of a policy to itself is then exactly 1), and within a
+    few ulps at their automatic shapes, which split a slice into different copies."""
     import torch
     rng = np.random.default_rng(6)
-    host, dev, y = case(rng, 64, 152064, "bf16")
-    lp, _ = run(grpo, dev, y, 152064, 152064)
+    host, dev, y = case(rng, 64, V, "bf16")
     yt = torch.from_numpy(y).cuda()
     z = torch.zeros(64, dtype=torch.float32, device="cuda")
-    lp2 = torch.empty(64, dtype=torch.float32, device="cuda")
-    grpo.grpo_loss_fwd_bwd(dev.view(64, 152064), yt, z, z, torch.zeros(1, device="cuda"),
-                           torch.zeros(64, dtype=torch.int32, device="cuda"), logp_out=lp2)
-    torch.cuda.synchronize()
-    assert np.array_equal(lp, lp2.cpu().numpy())
+
+    def fused():
+        lp2 = torch.empty(64, dtype=torch.float32, device="cuda")
+        grpo.grpo_loss_fwd_bwd(dev.view(64, V), yt, z, z, torch.zeros(1, device="cuda"),
+                               torch.zeros(64, dtype=torch.int32, device="cuda"), logp_out=lp2)
+        torch.cuda.synchronize()
+        return lp2.cpu().numpy()
+
+    lp, lp2 = run(grpo, dev, y, V, V)[0], fused()
+    ulp = np.spacing(np.abs(lp2).astype(np.float32)).astype(np.float64)
+    assert np.all(np.abs(lp.astype(np.float64) - lp2) <= 4 * ulp)
+    for shape in ((4, 256, 2), (2, 128, 1)):
+        try:
+            grpo.grpo_loss_tune(*shape)
+            assert np.array_equal(run(grpo, dev, y, V, V)[0], fused())
+        finally:
+            grpo.grpo_loss_tune(0, 0, 0)
 
 
 def test_logp_full_size_sampled(grpo, oracle_mod):
