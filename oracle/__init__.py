@@ -43,6 +43,10 @@ def lib():
                                   _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p,
                                   _c_p, _c_p, _c_p, _c_p]
         L.oracle_loss.restype = _i32
+        L.oracle_gspo_loss.argtypes = [_c_p, _i32, _i64, _c_p, _i32, _c_p, _c_p, _c_p, _c_p,
+                                       _c_p, _c_p, _i64, _i64, _f32, _f32, _f32, _c_p, _i32,
+                                       _c_p, _c_p, _c_p, _c_p, _c_p]
+        L.oracle_gspo_loss.restype = _i32
         L.oracle_logp.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p]
         L.oracle_logp.restype = _i32
         L.oracle_round_bf16.argtypes = [_f64]
@@ -173,6 +177,44 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
     if rc != 0:
         raise ValueError("oracle_loss: bad arguments")
     return dict(loss=float(total[0]), logp=logp[:n_rows], rho=rho[:n_rows], row_loss=rl[:n_rows],
+                dlogits=dl, dlogits_f64=d64)
+
+
+def gspo_loss(logits, V: int, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,
+              n_seq=None, eps_low=0.2, eps_high=0.2, beta=0.0, row_index=None, row_stride=None,
+              logits_dtype=None, dlogits_dtype=0, want_f64=False, want_dlogits=True):
+    """GSPO's sequence-level loss over kept rollouts (see loss.cpp).  Sequence k owns rows
+    [seq_row_off[k], seq_row_off[k+1]) and rollout seq_rollout[k].  n_seq defaults to the number
+    of sequences.  Returns dict(loss, logp [rows], seq_ratio [seqs], seq_loss [seqs], dlogits,
+    dlogits_f64)."""
+    lg = np.ascontiguousarray(logits)
+    if logits_dtype is None:
+        logits_dtype = 1 if lg.dtype == np.uint16 else 0
+    if logits_dtype == 0:
+        lg = lg.astype(np.float32, copy=False)
+    stride = V if row_stride is None else int(row_stride)
+    ri = None if row_index is None else _arr(row_index, np.int64)
+    so = _arr(seq_row_off, np.int64)
+    K = so.size - 1
+    n_rows = int(so[-1])
+    if n_seq is None:
+        n_seq = K
+    out_np = np.float32 if dlogits_dtype == 0 else np.uint16
+    dl = np.empty((n_rows, V), out_np) if want_dlogits else None
+    d64 = np.empty((n_rows, V), np.float64) if want_f64 else None
+    lp = np.empty(max(n_rows, 1), np.float64)
+    sr = np.empty(max(K, 1), np.float64)
+    sl = np.empty(max(K, 1), np.float64)
+    total = np.zeros(1, np.float64)
+    rc = lib().oracle_gspo_loss(_p(lg), logits_dtype, stride, _p(ri), V, _p(_arr(y, np.int32)),
+                                _p(_arr(old_logp, np.float32)), _p(_arr(ref_logp, np.float32)),
+                                _p(_arr(adv, np.float32)), _p(_arr(seq_rollout, np.int32)),
+                                _p(so), K, int(n_seq), float(eps_low), float(eps_high),
+                                float(beta), _p(dl), dlogits_dtype, _p(d64), _p(lp), _p(sr),
+                                _p(sl), _p(total))
+    if rc != 0:
+        raise ValueError("oracle_gspo_loss: bad arguments")
+    return dict(loss=float(total[0]), logp=lp[:n_rows], seq_ratio=sr[:K], seq_loss=sl[:K],
                 dlogits=dl, dlogits_f64=d64)
 
 

@@ -182,3 +182,110 @@ extern "C" int oracle_logp(const void* logits, int logits_dtype, int64_t row_str
   }
   return 0;
 }
+
+// GSPO's sequence-level loss over the kept rollouts: the base-algorithm variant FastRL is
+// combined with in its experiments (Sec. 1 and Sec. 4, "GSPO"), with the objective of Group
+// Sequence Policy Optimization (Zheng et al., 2025) restated here.  Rows come grouped by sequence:
+// sequence k owns rows [seq_row_off[k], seq_row_off[k+1]) and rollout seq_rollout[k].
+//   log s_k = (1/L_k) * sum_{t in k} (logp_t - old_logp_t)          (length-normalised ratio)
+//   l_k = -( min(s_k*A, clip(s_k, 1-eps_low, 1+eps_high)*A) - beta*(1/L_k)*sum_t kl_t )
+//   loss = (1/n_seq) * sum_k l_k,  kl_t = exp(x_t) - x_t - 1,  x_t = ref_logp_t - logp_t
+// Gradient: d loss / d logp_t = w_t*g_t with w_t = 1/(n_seq*L_k) and
+//   g_t = -(c_k*s_k*A + beta*(exp(x_t) - 1)),  c_k = [A>=0][s_k<=1+eps_high] + [A<0][s_k>=1-eps_low],
+// so dlogits[t, v] = w_t*g_t*([v == y] - softmax(z)_v), as for the token-level ratio.
+// A sequence holding an invalid token (y outside [0, V)) has no ratio: s_k = NaN, l_k = 0 and its
+// rows' dlogits are 0.  Empty sequences (L_k = 0) contribute nothing.
+extern "C" int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t row_stride,
+                                const int64_t* row_index, int V, const int32_t* y,
+                                const float* old_logp, const float* ref_logp, const float* adv,
+                                const int32_t* seq_rollout, const int64_t* seq_row_off,
+                                int64_t n_seq_rows, int64_t n_seq, float eps_low, float eps_high,
+                                float beta, void* dlogits, int dlogits_dtype, double* dlogits_f64,
+                                double* logp_out, double* seq_ratio_out, double* seq_loss_out,
+                                double* loss_out) {
+  if (V < 1 || row_stride < V || n_seq_rows < 0 || n_seq <= 0 || seq_row_off == nullptr)
+    return 1;
+  if (seq_row_off[0] != 0) return 1;
+  for (int64_t k = 0; k < n_seq_rows; ++k)
+    if (seq_row_off[k + 1] < seq_row_off[k]) return 1;
+  const int64_t n_rows = seq_row_off[n_seq_rows];
+  const double nan = std::numeric_limits<double>::quiet_NaN();
+  std::vector<double> logp(n_rows), lse(n_rows);
+
+  // Per-row log-sum-exp and log-probability (as in oracle_loss).
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t t = 0; t < n_rows; ++t) {
+    const int64_t src = row_index ? row_index[t] : t;
+    const int64_t base = src * row_stride;
+    const int32_t yt = y[src];
+    if (yt < 0 || yt >= V) {
+      logp[t] = nan;
+      lse[t] = nan;
+      continue;
+    }
+    double m = -std::numeric_limits<double>::infinity();
+    for (int v = 0; v < V; ++v) m = std::fmax(m, load_logit(logits, logits_dtype, base + v));
+    double s = 0.0;
+    for (int v = 0; v < V; ++v) s += std::exp(load_logit(logits, logits_dtype, base + v) - m);
+    lse[t] = m + std::log(s);
+    logp[t] = load_logit(logits, logits_dtype, base + yt) - lse[t];
+  }
+
+  const double lo = 1.0 - (double)eps_low;
+  const double hi = 1.0 + (double)eps_high;
+  std::vector<double> seq_loss(n_seq_rows, 0.0);
+  std::vector<double> coef(n_rows, 0.0);  // w_t * g_t
+  for (int64_t k = 0; k < n_seq_rows; ++k) {
+    const int64_t r0 = seq_row_off[k], r1 = seq_row_off[k + 1];
+    const int64_t L = r1 - r0;
+    if (seq_ratio_out) seq_ratio_out[k] = nan;
+    if (L == 0) continue;
+    double sum_lr = 0.0, sum_kl = 0.0;
+    bool valid = true;
+    for (int64_t t = r0; t < r1; ++t) {
+      const int64_t src = row_index ? row_index[t] : t;
+      if (std::isnan(logp[t])) valid = false;
+      sum_lr += logp[t] - (double)old_logp[src];
+      const double x = (double)ref_logp[src] - logp[t];
+      sum_kl += std::exp(x) - x - 1.0;
+    }
+    if (!valid) continue;
+    const double A = (double)adv[seq_rollout[k]];
+    const double s = std::exp(sum_lr / (double)L);
+    const double clipped = std::fmin(std::fmax(s, lo), hi);
+    const double surrogate = std::fmin(s * A, clipped * A);
+    seq_loss[k] = -(surrogate - (double)beta * sum_kl / (double)L) / (double)n_seq;
+    if (seq_ratio_out) seq_ratio_out[k] = s;
+    const bool c = (A >= 0.0 && s <= hi) || (A < 0.0 && s >= lo);
+    const double w = 1.0 / ((double)n_seq * (double)L);
+    for (int64_t t = r0; t < r1; ++t) {
+      const int64_t src = row_index ? row_index[t] : t;
+      const double x = (double)ref_logp[src] - logp[t];
+      coef[t] = w * -((c ? s * A : 0.0) + (double)beta * (std::exp(x) - 1.0));
+    }
+  }
+
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t t = 0; t < n_rows; ++t) {
+    const int64_t src = row_index ? row_index[t] : t;
+    const int64_t base = src * row_stride;
+    const int32_t yt = y[src];
+    const bool ok = yt >= 0 && yt < V;
+    for (int v = 0; v < V; ++v) {
+      double d = 0.0;
+      if (ok && coef[t] != 0.0) {
+        const double p = std::exp(load_logit(logits, logits_dtype, base + v) - lse[t]);
+        d = coef[t] * ((v == yt ? 1.0 : 0.0) - p);
+      }
+      if (dlogits) store_grad(dlogits, dlogits_dtype, t * (int64_t)V + v, d);
+      if (dlogits_f64) dlogits_f64[t * (int64_t)V + v] = d;
+    }
+    if (logp_out) logp_out[t] = logp[t];
+  }
+  double total = 0.0;
+  for (int64_t k = 0; k < n_seq_rows; ++k) total += seq_loss[k];
+  if (seq_loss_out)
+    for (int64_t k = 0; k < n_seq_rows; ++k) seq_loss_out[k] = seq_loss[k];
+  if (loss_out) *loss_out = total;
+  return 0;
+}

@@ -55,6 +55,18 @@ int oracle_loss(const void* logits, int logits_dtype, int64_t row_stride, const 
                 double* dlogits_f64, double* logp_out, double* rho_out, double* row_loss_out,
                 double* loss_out);
 
+/* GSPO's sequence-level loss (length-normalised sequence ratio, clipped per sequence) over kept
+ * rollouts; see loss.cpp.  Sequence k owns rows [seq_row_off[k], seq_row_off[k+1]) of the
+ * n_seq_rows sequences and rollout seq_rollout[k]; loss = (1/n_seq) sum_k l_k.
+ * seq_ratio_out [n_seq_rows] (nullable): s_k (NaN when undefined); seq_loss_out: l_k / n_seq. */
+int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t row_stride,
+                     const int64_t* row_index, int V, const int32_t* y, const float* old_logp,
+                     const float* ref_logp, const float* adv, const int32_t* seq_rollout,
+                     const int64_t* seq_row_off, int64_t n_seq_rows, int64_t n_seq, float eps_low,
+                     float eps_high, float beta, void* dlogits, int dlogits_dtype,
+                     double* dlogits_f64, double* logp_out, double* seq_ratio_out,
+                     double* seq_loss_out, double* loss_out);
+
 /* logp of the sampled token alone (old/reference policy evaluation); NaN for ids outside [0,V). */
 int oracle_logp(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
                 int64_t n_rows, int V, const int32_t* y, double* logp_out);
