@@ -36,6 +36,9 @@ sys.path.insert(0, ROOT)
 METRIC = "kept-token GRPO loss fwd+bwd tokens/s and logits HBM GB/s (% of GB300 peak)"
 UNIT = "kept tokens/s"
 SIDE_BYTES_PER_ROW = 36  # y, old, ref, logp (4 each), src_token 8, row rollout 4, row loss 8
+# GSPO: forward (src 8, y 4, logp 4, stats 16), sequence pass (src 8, logp, old, ref, coef 4
+# each), dlogits pass (src 8, coef 4, stats 16, y 4)
+GSPO_SIDE_BYTES_PER_ROW = 88
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -51,6 +54,9 @@ def parse():
                     help="override the workload's prompt count (a smaller case for profiling)")
     ap.add_argument("--group", type=int, default=0,
                     help="override the rollouts per prompt G (a smaller case for profiling)")
+    ap.add_argument("--loss", choices=["grpo", "gspo"], default="grpo",
+                    help="grpo: Eq. 1's token-level ratio (fused, one pass); gspo: the sequence-level "
+                         "ratio of FastRL's GSPO variant (three passes, host-synced)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
@@ -207,11 +213,12 @@ def build_inputs(w, seed, device):
     return b, dict(rewards=rewards, ids=ids, off=off, logits=logits, old=old, ref=ref)
 
 
-def make_step(w, dev_inputs):
+def make_step(w, dev_inputs, loss="grpo"):
     from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
     p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
                    eps_low=w.eps, eps_high=w.eps, beta=w.beta, dlogits_dtype=w.dlogits_dtype,
-                   chunk_rows=w.chunk_rows)
+                   chunk_rows=0 if loss == "gspo" else w.chunk_rows,
+                   ratio_level="sequence" if loss == "gspo" else "token")
     d = dev_inputs
     return GrpoStep(p, d["rewards"], d["ids"], d["off"], d["logits"], d["old"], d["ref"])
 
@@ -341,7 +348,7 @@ def main():
     g.lib()
 
     b, d = build_inputs(w, rank_seed(args.seed, rank), dev)
-    step = make_step(w, d)
+    step = make_step(w, d, args.loss)
     for _ in range(max(args.warmup, 3)):
         step.run()
     torch.cuda.synchronize()
@@ -349,7 +356,7 @@ def main():
     step.run()
     torch.cuda.synchronize()
     launches_per_step = g.grpo_kernel_launches() - l_before
-    use_graph = not args.no_graph and w.chunk_rows == 0
+    use_graph = not args.no_graph and w.chunk_rows == 0 and args.loss == "grpo"
     if use_graph:
         step.capture()
         for _ in range(max(args.warmup, 3)):
@@ -394,14 +401,22 @@ def main():
     value = kept_all / (elapsed_ms / 1e3)
 
     # roofline of the dominant kernel (the fused loss), from its event-timed launches
-    bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
+    if args.loss == "gspo":  # two reads and one write of every kept row (no row has zero gradient
+        # in these workloads: beta > 0)
+        bytes_per_row = w.V * (2 * w.in_bytes + w.out_bytes) + GSPO_SIDE_BYTES_PER_ROW
+        per_row_traffic = profiled_traffic(w.name + "/gspo")
+        kernel = ("GSPO loss: grpo_loss_kernel<..., forward only> with row statistics, "
+                  "gspo_seq_kernel, gspo_dlogits_kernel, fixed-order sum")
+    else:
+        bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
+        per_row_traffic = profiled_traffic(w.name)
+        kernel = "grpo_loss_kernel (+ 1-CTA fixed-order loss sum)"
     achieved = step.T_kept * bytes_per_row / (loss_ms / 1e3) / 1e9
     peak, peak_src = measured_peak()
-    per_row_traffic = profiled_traffic(w.name)
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak,
                 "traffic": None if per_row_traffic is None else per_row_traffic * step.T_kept,
-                "kernel": "grpo_loss_kernel (+ 1-CTA fixed-order loss sum)",
+                "kernel": kernel,
                 "algorithmic_bytes_per_launch": step.T_kept * bytes_per_row,
                 "launch_ms": loss_ms, "peak_source": peak_src}
 
@@ -467,7 +482,7 @@ def main():
         del host
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.loss == "grpo":
         cpu = cpu_baseline_ours(w, b, step, d, args.cpu_seconds)
 
     if rank == 0:
@@ -476,7 +491,7 @@ def main():
             "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded; shapes and distributions of the paper's GRPO batches)",
-            "config": workload_desc(w, b["T"], step.T_kept, step.K),
+            "config": dict(workload_desc(w, b["T"], step.T_kept, step.K), loss=args.loss),
             "gpu_launches": int(launches), "cuda_graph": use_graph,
             "roofline": roofline, "e2e": e2e,
             "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd,

@@ -8,6 +8,7 @@
  *   grpo_prune              maximising-differential advantage pruning (MDAP)   (Eqs. 6-9, Algorithm 1)
  *   grpo_compact            compaction of the kept rollouts' tokens            (Sec. 3.2, after Eq. 9)
  *   grpo_upload_kept        host-to-device copy of the kept rollouts' rows      (Sec. 3.2)
+ *   grpo_gspo_loss_fwd_bwd  GSPO's sequence-level loss, for FastRL on GSPO     (Sec. 1, Sec. 4)
  *   grpo_loss_fwd_bwd       fused GRPO token loss, forward and dlogits         (Eqs. 1-3)
  *   adaptive_rollout_count  host-side adaptive rollout sampling (ARS)          (Eqs. 10-14, Algorithm 1)
  *
@@ -224,6 +225,40 @@ grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t 
 grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
                           const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
                           float* logp_out, int32_t* status, grpo_stream_t stream);
+
+/*
+ * grpo_gspo_loss_fwd_bwd — GSPO's sequence-level loss and its dlogits over the kept rollouts.
+ * GSPO (Group Sequence Policy Optimization) is one of the base algorithms FastRL is combined with
+ * (Sec. 1, Sec. 4); its objective over the kept sequences, with sequence k owning rows
+ * [seq_row_off[k], seq_row_off[k+1]) (L_k rows) and advantage A = adv[seq_rollout[k]]:
+ *   log s_k = (1/L_k) sum_{t in k} (logp_t - old_logp_t)        (length-normalised ratio)
+ *   l_k = -( min(s_k*A, clip(s_k, 1-eps_low, 1+eps_high)*A) - beta*(1/L_k)*sum_t kl_t )
+ *   loss = (1/n_seq) sum_k l_k,  kl_t = exp(x_t) - x_t - 1,  x_t = ref_logp_t - logp_t
+ *   dlogits[t, v] = w_t*g_t*([v == y] - softmax(z)_v),  w_t = 1/(n_seq*L_k),
+ *   g_t = -(c_k*s_k*A + beta*(exp(x_t) - 1)),  c_k = [A>=0][s_k<=1+eps_high] + [A<0][s_k>=1-eps_low]
+ * Rows: row t < n_rows reads logits row src = row_index[t] (or t) and y, old_logp, ref_logp at
+ *   src, as grpo_loss_fwd_bwd.  Sequences: seq_row_off device i64 [n_seq_rows+1] and
+ *   seq_rollout device i32 [n_seq_rows], for instance grpo_compact's kept_off and kept_idx
+ *   (n_seq_rows = K, n_rows = T_kept).  Offsets are clamped to [0, n_rows]; rows outside every
+ *   sequence get zero gradient.  n_seq > 0: the mean's denominator (the global kept-sequence
+ *   count under data parallelism).
+ * A sequence with a non-finite log-probability (a token id outside [0, V), non-finite logits)
+ *   has no ratio: seq_ratio NaN, no loss term, zero dlogits; the status word says why.
+ * Outputs: dlogits [n_rows, V] (dtype dlogits_dtype), logp_out f32 [n_rows] (required),
+ *   seq_ratio_out f32 [n_seq_rows] (nullable), loss_out f64 [1], reduced in a fixed order.
+ * Workspace: 20 bytes per row + 8 per sequence (size query as everywhere).  Three passes over
+ *   the logits' bytes (two reads, one write): log-probabilities with softmax statistics, the
+ *   sequence ratios, then dlogits.  Deterministic for a given input.
+ */
+grpo_status grpo_gspo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
+                                   const int64_t* row_index, int64_t n_rows, int32_t V,
+                                   const int32_t* y, const float* old_logp, const float* ref_logp,
+                                   const float* adv, const int32_t* seq_rollout,
+                                   const int64_t* seq_row_off, int32_t n_seq_rows, int64_t n_seq,
+                                   float eps_low, float eps_high, float beta, void* dlogits,
+                                   int32_t dlogits_dtype, float* logp_out, float* seq_ratio_out,
+                                   double* loss_out, int32_t* status, void* ws, size_t* ws_bytes,
+                                   grpo_stream_t stream);
 
 /*
  * grpo_sum_f64 — *out = v[0] + ... + v[n-1] in fp64, in the same fixed order grpo_loss_fwd_bwd

@@ -31,7 +31,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_sum_f64", "grpo_logp_fwd",
+           "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_sum_f64", "grpo_logp_fwd",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -93,6 +93,11 @@ def lib():
                                             _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64,
                                             _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p]
     L.grpo_loss_fwd_bwd_noalloc.restype = _i32
+    L.grpo_gspo_loss_fwd_bwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p,
+                                         _c_p, _c_p, _c_p, _i32, _i64, _f32, _f32, _f32, _c_p,
+                                         _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                         ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_gspo_loss_fwd_bwd.restype = _i32
     L.grpo_logp_fwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p]
     L.grpo_logp_fwd.restype = _i32
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
@@ -352,6 +357,77 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
     wp, size = _ws_args(wst)
     _check(L.grpo_loss_fwd_bwd(*args_head, wp, size, _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
+
+
+def grpo_gspo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,
+                           n_rows: int, n_seq_rows: int | None = None, n_seq: int | None = None,
+                           V: int | None = None, row_stride: int | None = None, row_index=None,
+                           eps_low: float = 0.2, eps_high: float = 0.2, beta: float = 0.0,
+                           dlogits=None, dlogits_dtype=None, logp_out=None, seq_ratio_out=None,
+                           loss_out=None, status=None, ws=None, stream=None):
+    """GSPO's sequence-level loss on the GPU (see the header).  seq_row_off / seq_rollout: device
+    i64 [K+1] / i32 [K] (grpo_compact's kept_off and kept_idx); n_rows: the rows they cover
+    (T_kept).  n_seq_rows defaults to seq_rollout.numel(), n_seq to n_seq_rows.  Returns
+    dict(loss, dlogits, logp, seq_ratio)."""
+    torch = _torch()
+    if logits.dtype == torch.bfloat16:
+        ldt = GRPO_DTYPE_BF16
+    elif logits.dtype == torch.float32:
+        ldt = GRPO_DTYPE_F32
+    else:
+        raise TypeError("logits must be bf16 or f32")
+    if not logits.is_cuda:
+        raise TypeError("logits must be a CUDA tensor")
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be 2-D with unit stride along the vocabulary")
+    if V is None:
+        V = logits.shape[1]
+    stride = logits.stride(0) if row_stride is None else int(row_stride)
+    if n_seq_rows is None:
+        n_seq_rows = seq_rollout.numel()
+    if n_seq is None:
+        n_seq = max(int(n_seq_rows), 1)
+    dev = logits.device
+    if dlogits_dtype is None:
+        if dlogits is not None:
+            dlogits_dtype = GRPO_DTYPE_BF16 if dlogits.dtype == torch.bfloat16 else GRPO_DTYPE_F32
+        else:
+            dlogits_dtype = ldt
+    elif dlogits_dtype in (torch.bfloat16, "bf16"):
+        dlogits_dtype = GRPO_DTYPE_BF16
+    elif dlogits_dtype in (torch.float32, "f32"):
+        dlogits_dtype = GRPO_DTYPE_F32
+    out_t = torch.bfloat16 if dlogits_dtype == GRPO_DTYPE_BF16 else torch.float32
+    if dlogits is None:
+        dlogits = torch.empty((max(n_rows, 1), V), dtype=out_t, device=dev)
+    _need(dlogits, out_t, n_rows * V, "dlogits")
+    if logp_out is None:
+        logp_out = torch.empty(max(n_rows, 1), dtype=torch.float32, device=dev)
+    _need(logp_out, torch.float32, n_rows, "logp_out")
+    if seq_ratio_out is not None:
+        _need(seq_ratio_out, torch.float32, n_seq_rows, "seq_ratio_out")
+    if loss_out is None:
+        loss_out = torch.empty(1, dtype=torch.float64, device=dev)
+    _need(y, torch.int32, None, "y")
+    _need(old_logp, torch.float32, None, "old_logp")
+    _need(ref_logp, torch.float32, None, "ref_logp")
+    _need(adv, torch.float32, None, "adv")
+    _need(seq_rollout, torch.int32, n_seq_rows, "seq_rollout")
+    _need(seq_row_off, torch.int64, n_seq_rows + 1, "seq_row_off")
+    if row_index is not None:
+        _need(row_index, torch.int64, n_rows, "row_index")
+    L = lib()
+    head = (_ptr(logits), ldt, stride, _ptr(row_index), int(n_rows), int(V), _ptr(y),
+            _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(seq_rollout), _ptr(seq_row_off),
+            int(n_seq_rows), int(n_seq), float(eps_low), float(eps_high), float(beta),
+            _ptr(dlogits), dlogits_dtype, _ptr(logp_out), _ptr(seq_ratio_out), _ptr(loss_out),
+            _ptr(status))
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_gspo_loss_fwd_bwd(*head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, dev, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_gspo_loss_fwd_bwd(*head, wp, size, _stream(stream)))
+    return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, seq_ratio=seq_ratio_out, ws=wst)
 
 
 def grpo_loss_fwd_bwd_noalloc(logits, y, old_logp, ref_logp, adv, row_rollout, *, dlogits,

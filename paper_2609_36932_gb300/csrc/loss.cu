@@ -33,11 +33,11 @@
 #include <tuple>
 
 #include "common.cuh"
+#include "rowops.cuh"
 
 namespace fastrl {
 namespace {
 
-constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int kMaxChunks = 16;
 constexpr int kMaxCluster = 16;
@@ -66,6 +66,7 @@ struct LossArgs {
   float inv_nseq_f;  // agg 1: 1 / n_seq
   char* dlogits;
   float* logp_out;
+  float4* stats_out;  // forward only, nullable: per row {max, sum of exp, that sum without y, 0}
   double* row_loss;
   int32_t* status;
   int32_t slice;       // elements per CTA, a multiple of the 16-byte vector width
@@ -151,108 +152,6 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
       "l"(src), "r"(bytes), "r"(bar)
       : "memory");
 }
-// 2^x on the MUFU (one instruction); results below 2^-126 flush to zero.  Pass A only loses
-// terms 2^126 times smaller than the running maximum; pass B shifts its argument (see
-// kShiftB) so that no representable gradient entry is lost.
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-__device__ __forceinline__ float2 ex2x2(float2 t) { return make_float2(ex2(t.x), ex2(t.y)); }
-// Lane-wise maximum of two bf16 pairs; a NaN operand yields the other operand.
-__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-
-// Pass B evaluates 2^(t + kShiftB) * (scale * 2^-kShiftB) when |scale| >= 2^-100, which moves the
-// flush-to-zero point of ex2 below every gradient entry that bf16 or f32 can represent.
-constexpr float kShiftB = 16.f;
-
-// ---- element formats: 16-byte vectors of the logits, unpacked into f32 pairs -----------------
-
-template <typename T>
-struct Fmt;
-template <>
-struct Fmt<float> {
-  static constexpr int kVec = 4;  // elements per 16 bytes
-  static constexpr int kPairs = 2;
-  __device__ static void pairs(const uint4& q, float2 (&p)[2]) {
-    p[0] = make_float2(__uint_as_float(q.x), __uint_as_float(q.y));
-    p[1] = make_float2(__uint_as_float(q.z), __uint_as_float(q.w));
-  }
-  struct Max {  // running maximum over vectors
-    float m = -INFINITY;
-    __device__ void add(const uint4& q) {
-      m = fmaxf(m, fmaxf(fmaxf(__uint_as_float(q.x), __uint_as_float(q.y)),
-                         fmaxf(__uint_as_float(q.z), __uint_as_float(q.w))));
-    }
-    __device__ float get() const { return m; }
-  };
-  __device__ static float load(const float* p) { return *p; }
-  __device__ static void store(float* p, float v) { *p = v; }
-};
-template <>
-struct Fmt<__nv_bfloat16> {
-  static constexpr int kVec = 8;
-  static constexpr int kPairs = 4;
-  __device__ static float2 pair(uint32_t w) {
-    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
-  }
-  __device__ static void pairs(const uint4& q, float2 (&p)[4]) {
-    p[0] = pair(q.x);
-    p[1] = pair(q.y);
-    p[2] = pair(q.z);
-    p[3] = pair(q.w);
-  }
-  struct Max {  // running maximum kept as a bf16 pair: one instruction per two elements
-    uint32_t m = 0xFF80FF80u;  // (-inf, -inf)
-    __device__ void add(const uint4& q) { m = bmax2(m, bmax2(bmax2(q.x, q.y), bmax2(q.z, q.w))); }
-    __device__ float get() const {
-      return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
-    }
-  };
-  __device__ static float load(const __nv_bfloat16* p) { return __bfloat162float(*p); }
-  __device__ static void store(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
-};
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float2 v) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(v.x, v.y);
-  return *reinterpret_cast<const uint32_t*>(&h);
-}
-
-// Store one vector of results at p (aligned to its width), streaming (evict-first).
-template <typename OutT, int kPairs>
-__device__ __forceinline__ void store_pairs(OutT* p, const float2 (&d)[kPairs]);
-template <>
-__device__ __forceinline__ void store_pairs<__nv_bfloat16, 4>(__nv_bfloat16* p, const float2 (&d)[4]) {
-  __stcs(reinterpret_cast<uint4*>(p),
-         make_uint4(pack_bf16x2(d[0]), pack_bf16x2(d[1]), pack_bf16x2(d[2]), pack_bf16x2(d[3])));
-}
-template <>
-__device__ __forceinline__ void store_pairs<float, 4>(float* p, const float2 (&d)[4]) {
-  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0].x, d[0].y, d[1].x, d[1].y));
-  __stcs(reinterpret_cast<float4*>(p) + 1, make_float4(d[2].x, d[2].y, d[3].x, d[3].y));
-}
-template <>
-__device__ __forceinline__ void store_pairs<float, 2>(float* p, const float2 (&d)[2]) {
-  __stcs(reinterpret_cast<float4*>(p), make_float4(d[0].x, d[0].y, d[1].x, d[1].y));
-}
-template <>
-__device__ __forceinline__ void store_pairs<__nv_bfloat16, 2>(__nv_bfloat16* p, const float2 (&d)[2]) {
-  __stcs(reinterpret_cast<uint2*>(p), make_uint2(pack_bf16x2(d[0]), pack_bf16x2(d[1])));
-}
-template <typename OutT, int kPairs>
-__device__ __forceinline__ void store_pairs_scalar(OutT* p, const float2 (&d)[kPairs]) {
-#pragma unroll
-  for (int i = 0; i < kPairs; ++i) {
-    Fmt<OutT>::store(p + 2 * i, d[i].x);
-    Fmt<OutT>::store(p + 2 * i + 1, d[i].y);
-  }
-}
-
 // Combine two (max, sum of exp relative to max) pairs.
 __device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float so) {
   const float M = fmaxf(m, mo);
@@ -496,6 +395,7 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
         if (!yvalid) {
           if (rank == 0) {
             if (a.logp_out) a.logp_out[row] = __int_as_float(0x7fc00000);
+            if (!kBwd && a.stats_out) a.stats_out[row] = make_float4(NAN, NAN, NAN, 0.f);
             if (kBwd) a.row_loss[row] = 0.0;
             if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
           }
@@ -508,6 +408,7 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
           if constexpr (!kBwd) {
             if (rank == 0) {
               a.logp_out[row] = logp;
+              if (a.stats_out) a.stats_out[row] = make_float4(M, S, S_excl, 0.f);
               if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
             }
           } else {
@@ -959,12 +860,11 @@ extern "C" grpo_status grpo_loss_fwd_bwd_dev(
 }
 
 
-extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
-                                     const int64_t* row_index, int64_t n_rows, int32_t V,
-                                     const int32_t* y, float* logp_out, int32_t* status,
-                                     grpo_stream_t stream) {
-  clear_error();
-  const char* who = "grpo_logp_fwd";
+namespace fastrl {
+
+grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype, int64_t row_stride,
+                      const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
+                      float* logp_out, float4* stats_out, int32_t* status, cudaStream_t s) {
   if (logits_dtype != GRPO_DTYPE_BF16 && logits_dtype != GRPO_DTYPE_F32)
     return fail(GRPO_ERR_INVALID_ARG, "%s: logits_dtype = %d", who, logits_dtype);
   if (n_rows < 0 || n_rows >= (int64_t(1) << 31))
@@ -985,13 +885,25 @@ extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, i
   a.V = V;
   a.y = y;
   a.logp_out = logp_out;
+  a.stats_out = stats_out;
   a.status = status;
   a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
   st = launch_rows(fwd_kernel_for(logits_dtype, sh.threads, want_cap(sh.smem, sh.threads)), sh, a,
-                   as_stream(stream), who);
+                   s, who);
   if (st != GRPO_OK) return st;
   count_launches(1);
   return GRPO_OK;
+}
+
+}  // namespace fastrl
+
+extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
+                                     const int64_t* row_index, int64_t n_rows, int32_t V,
+                                     const int32_t* y, float* logp_out, int32_t* status,
+                                     grpo_stream_t stream) {
+  clear_error();
+  return logp_rows("grpo_logp_fwd", logits, logits_dtype, row_stride, row_index, n_rows, V, y,
+                   logp_out, nullptr, status, as_stream(stream));
 }
 
 // ---- allocation-free variant ------------------------------------------------------------------

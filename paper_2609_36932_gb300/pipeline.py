@@ -32,6 +32,9 @@ class StepParams:
     std_mode: int = 0
     chunk_rows: int = 0  # >0: the loss runs over the kept rows in chunks sharing one dlogits buffer
     class_eps: float = 0.0  # >0: continuous-reward grouping of advantages (the paper uses 1e-4)
+    # "token": Eq. 1's token-level ratio (GRPO, DAPO); "sequence": GSPO's length-normalised
+    # sequence ratio, clipped per sequence, with the sequence mean (agg_mode is then unused)
+    ratio_level: str = "token"
 
 
 class GrpoStep:
@@ -115,6 +118,8 @@ class GrpoStep:
 
     def loss_step(self):
         p = self.p
+        if p.ratio_level == "sequence":
+            return self._loss_gspo()
         if p.chunk_rows > 0:
             return self._loss_chunked()
         self._ensure_dlogits(self.T_kept)
@@ -125,6 +130,26 @@ class GrpoStep:
             denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
             dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp, loss_out=self.loss, status=self.status,
             ws=self.loss_ws)
+
+    def _loss_gspo(self):
+        """GSPO's sequence-level loss over the kept rollouts: the compaction's kept offsets and
+        kept rollout indices are the sequences."""
+        p = self.p
+        if p.chunk_rows > 0:
+            raise ValueError("the sequence-level ratio runs the loss in one call (chunk_rows = 0)")
+        self._ensure_dlogits(self.T_kept)
+        if getattr(self, "seq_ratio", None) is None:
+            self.seq_ratio = self.torch.empty(max(self.keep.numel(), 1), dtype=self.torch.float32,
+                                              device=self.dev)
+        out = B.grpo_gspo_loss_fwd_bwd(
+            self.logits, self.ids, self.old, self.ref, self.adv, self.kept_idx, self.kept_off,
+            n_rows=self.T_kept, n_seq_rows=self.K, n_seq=max(self.K, 1), V=p.V,
+            row_index=self.src_token, eps_low=p.eps_low, eps_high=p.eps_high, beta=p.beta,
+            dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp,
+            seq_ratio_out=self.seq_ratio, loss_out=self.loss, status=self.status,
+            ws=getattr(self, "gspo_ws", None))
+        self.gspo_ws = out["ws"]
+        return out
 
     def _loss_chunked(self):
         """Kept rows in chunks of p.chunk_rows; each chunk overwrites the same dlogits buffer
@@ -178,6 +203,9 @@ class GrpoStep:
         torch = self.torch
         if self.p.chunk_rows > 0:
             raise ValueError("graph mode runs the loss in one call (chunk_rows = 0)")
+        if self.p.ratio_level != "token":
+            raise ValueError("graph mode runs the token-level loss; the sequence-level ratio "
+                             "runs host-synced")
         self._ensure_dlogits(self.T)
         for _ in range(2):  # warm-up outside capture (kernel attributes, occupancy queries)
             self._enqueue_select()

@@ -120,6 +120,33 @@ def test_upload_kept_argument_errors(grpo):
     assert call(np.zeros(4, np.uint8), off, 4) == 0 and (nb.value, nc.value) == (0, 0)
 
 
+def gspo_call(L, n_rows, V, K, ws, size_p, n_seq=1, ldt=1, beta=0.0, eps=0.2, logp=4096):
+    return L.grpo_gspo_loss_fwd_bwd(None, ldt, V, None, n_rows, V, None, None, None, None, None,
+                                    None, K, n_seq, eps, eps, beta, None, 1,
+                                    ctypes.c_void_p(logp) if logp else None, None, None, None,
+                                    ws, size_p, None)
+
+
+def test_gspo_workspace_query_and_argument_errors(grpo):
+    L = raw()
+    size = ctypes.c_size_t(0)
+    def up(x):
+        return (x + 255) // 256 * 256
+    assert gspo_call(L, 1000, 152064, 16, None, ctypes.byref(size)) == 0
+    assert size.value == up(1000 * 16) + up(1000 * 4) + up(16 * 8)  # stats, coef, seq terms
+    assert gspo_call(L, 1000, 152064, 16, None, ctypes.byref(size), n_seq=0) == 1
+    assert gspo_call(L, 1000, 152064, -1, None, ctypes.byref(size)) == 1
+    assert gspo_call(L, -1, 152064, 16, None, ctypes.byref(size)) == 1
+    assert gspo_call(L, 10, 0, 1, None, ctypes.byref(size)) == 1
+    assert gspo_call(L, 10, 100, 1, None, ctypes.byref(size), ldt=5) == 1
+    assert gspo_call(L, 10, 100, 1, None, ctypes.byref(size), beta=-1.0) == 1
+    small = ctypes.c_size_t(8)
+    assert gspo_call(L, 1000, 152064, 16, ctypes.c_void_p(4096), ctypes.byref(small)) == 3
+    # a real call with NULL sequence arrays is refused before any launch
+    big = ctypes.c_size_t(1 << 20)
+    assert gspo_call(L, 1000, 152064, 16, ctypes.c_void_p(4096), ctypes.byref(big)) == 1
+
+
 def loss_call(L, n_rows, V, ws, size_p, ldt=1, agg=0, denom=1, row_loss=None, beta=0.04):
     return L.grpo_loss_fwd_bwd(None, ldt, V, None, n_rows, V, None, None, None, None, None, 0.2,
                                0.2, beta, agg, denom, None, 0, None, 1, None, row_loss, None, None,

@@ -1,0 +1,174 @@
+"""GPU parity of grpo_gspo_loss_fwd_bwd (GSPO's sequence-level loss, FastRL's GSPO variant) with
+the oracle, through the C ABI: vocabulary sizes with ragged tails, both dtypes, gathered rows,
+GSPO's narrow clip range, sequences of one token, invalid tokens, empty sequences."""
+import numpy as np
+import pytest
+
+from helpers import bf16_bits_to_f32, bf16_ulp_distance
+from loss_compare import F32_ATOL, LOGP_ATOL, LOSS_ATOL, LOSS_RTOL
+
+pytestmark = pytest.mark.gpu
+
+RATIO_RTOL = 3e-5  # s_k from f32 log-probs (each within 2e-5 of the oracle's)
+
+
+def bf16_bits(x):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(torch.bfloat16).view(
+        torch.int16).numpy().view(np.uint16)
+
+
+class SeqCase:
+    def __init__(self, rng, lens, V, in_dtype="bf16", out_dtype="bf16", old_sd=0.05, beta=0.04,
+                 eps=(0.2, 0.28), gather=False):
+        import torch
+        self.lens = np.asarray(lens, np.int64)
+        self.K = len(lens)
+        self.n = int(self.lens.sum())
+        self.V, self.out_dtype, self.beta, self.eps = V, out_dtype, beta, eps
+        n_src = self.n + (7 if gather else 0)
+        z = (rng.standard_normal((n_src, V)) * 2.5).astype(np.float32)
+        if in_dtype == "bf16":
+            self.host = bf16_bits(z)
+            zf = bf16_bits_to_f32(self.host)
+            self.dev = torch.from_numpy(self.host.view(np.int16)).cuda().view(torch.bfloat16)
+        else:
+            self.host, zf = z, z
+            self.dev = torch.from_numpy(z).cuda()
+        self.y = rng.integers(0, V, size=n_src).astype(np.int32)
+        zz = zf.astype(np.float64)
+        m = zz.max(1, keepdims=True)
+        logp = zz[np.arange(n_src), self.y] - (m[:, 0] + np.log(np.exp(zz - m).sum(1)))
+        # a per-sequence drift of the old policy, so whole sequences leave the clip range
+        drift = np.repeat(rng.standard_normal(self.K) * old_sd * 2, lens)
+        drift = np.concatenate([drift, np.zeros(n_src - self.n)])
+        self.old = (logp - drift + old_sd * rng.standard_normal(n_src)).astype(np.float32)
+        self.ref = (logp + 0.1 * rng.standard_normal(n_src)).astype(np.float32)
+        self.adv = rng.standard_normal(self.K + 3).astype(np.float32)
+        self.seq_rollout = rng.permutation(self.K + 3)[:self.K].astype(np.int32)
+        self.seq_row_off = np.concatenate([[0], np.cumsum(self.lens)]).astype(np.int64)
+        self.row_index = rng.permutation(n_src)[:self.n].astype(np.int64) if gather else None
+
+    def t(self, a):
+        import torch
+        return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+    def run_gpu(self, grpo, n_seq=None):
+        import torch
+        status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        ratio = torch.empty(max(self.K, 1), dtype=torch.float32, device="cuda")
+        out = grpo.grpo_gspo_loss_fwd_bwd(
+            self.dev, self.t(self.y), self.t(self.old), self.t(self.ref), self.t(self.adv),
+            self.t(self.seq_rollout), self.t(self.seq_row_off), n_rows=self.n, n_seq=n_seq,
+            row_index=None if self.row_index is None else self.t(self.row_index),
+            eps_low=self.eps[0], eps_high=self.eps[1], beta=self.beta,
+            dlogits_dtype=self.out_dtype, seq_ratio_out=ratio, status=status)
+        torch.cuda.synchronize()
+        d = out["dlogits"][:self.n]
+        d = d.view(torch.int16).cpu().numpy().view(np.uint16) if self.out_dtype == "bf16" else d.cpu().numpy()
+        return dict(loss=float(out["loss"].item()), dlogits=d, logp=out["logp"][:self.n].cpu().numpy(),
+                    ratio=ratio[:self.K].cpu().numpy(), status=int(status.item()))
+
+    def run_oracle(self, oracle_mod, n_seq=None):
+        return oracle_mod.gspo_loss(self.host, self.V, self.y, self.old, self.ref, self.adv,
+                                    self.seq_rollout, self.seq_row_off, n_seq=n_seq,
+                                    eps_low=self.eps[0], eps_high=self.eps[1], beta=self.beta,
+                                    row_index=self.row_index,
+                                    dlogits_dtype=1 if self.out_dtype == "bf16" else 0)
+
+
+def compare_gspo(g, r, case):
+    """Tolerances as the token-level loss; rows of sequences whose ratio lies within RATIO_RTOL
+    of a clip boundary may take either branch and are not compared."""
+    valid = ~np.isnan(r["logp"])
+    assert np.all(np.isnan(g["logp"][~valid]) | ~np.isfinite(g["logp"][~valid]))
+    assert np.abs(g["logp"][valid].astype(np.float64) - r["logp"][valid]).max(initial=0) <= LOGP_ATOL
+    s = r["seq_ratio"]
+    ok = ~np.isnan(s)
+    assert np.array_equal(np.isnan(g["ratio"]), ~ok)
+    np.testing.assert_allclose(g["ratio"][ok], s[ok], rtol=RATIO_RTOL)
+    lo, hi = 1.0 - np.float64(np.float32(case.eps[0])), 1.0 + np.float64(np.float32(case.eps[1]))
+    near = ok & ((np.abs(s - lo) <= RATIO_RTOL * lo) | (np.abs(s - hi) <= RATIO_RTOL * hi))
+    rows = ~np.repeat(near, case.lens)
+    if case.out_dtype == "bf16":
+        assert int(bf16_ulp_distance(g["dlogits"][rows], r["dlogits"][rows]).max(initial=0)) <= 1
+    else:
+        diff = np.abs(g["dlogits"][rows].astype(np.float64) - r["dlogits"][rows].astype(np.float64))
+        assert diff.max(initial=0.0) <= F32_ATOL
+    if not near.any():
+        assert abs(g["loss"] - r["loss"]) <= LOSS_RTOL * abs(r["loss"]) + LOSS_ATOL
+    return int(near.sum())
+
+
+SHAPES = [(1000, "bf16", "bf16"), (1001, "f32", "f32"), (4097, "f32", "bf16"),
+          (32000, "bf16", "bf16"), (152064, "bf16", "bf16"), (152067, "bf16", "f32")]
+
+
+@pytest.mark.parametrize("V,ind,outd", SHAPES)
+def test_gspo_matches_oracle(grpo, oracle_mod, V, ind, outd):
+    rng = np.random.default_rng(V)
+    lens = list(rng.integers(4, 24 if V > 100000 else 48, size=7)) + [0, 9]
+    c = SeqCase(rng, lens, V, ind, outd, old_sd=0.15)
+    g, r = c.run_gpu(grpo), c.run_oracle(oracle_mod)
+    assert g["status"] == 0
+    compare_gspo(g, r, c)
+    s = r["seq_ratio"][~np.isnan(r["seq_ratio"])]
+    assert ((s > 1.28) | (s < 0.8)).any() and ((s < 1.28) & (s > 0.8)).any()
+
+
+def test_gspo_gathered_rows_and_global_sequence_count(grpo, oracle_mod):
+    """Rows gathered through row_index from a larger buffer; n_seq larger than the local
+    sequence count (data parallelism: the global count)."""
+    rng = np.random.default_rng(41)
+    c = SeqCase(rng, [5, 17, 1, 30, 8], 32000, gather=True)
+    g, r = c.run_gpu(grpo, n_seq=13), c.run_oracle(oracle_mod, n_seq=13)
+    compare_gspo(g, r, c)
+
+
+def test_gspo_narrow_clip_range(grpo, oracle_mod):
+    """GSPO's own clip widths are far narrower than the token-level ones (3e-4 / 4e-4 here):
+    most sequences are clipped and get zero gradient when beta = 0."""
+    rng = np.random.default_rng(42)
+    c = SeqCase(rng, list(rng.integers(8, 40, size=16)), 32000, old_sd=0.01, beta=0.0,
+                eps=(3e-4, 4e-4))
+    g, r = c.run_gpu(grpo), c.run_oracle(oracle_mod)
+    compare_gspo(g, r, c)
+    A = c.adv[c.seq_rollout].astype(np.float64)
+    s = r["seq_ratio"]
+    active = ((A > 0) & (s > (1 + 4e-4) * (1 + RATIO_RTOL))) | ((A < 0) & (s < (1 - 3e-4) * (1 - RATIO_RTOL)))
+    assert active.sum() >= 4
+    zero_rows = np.repeat(active, c.lens)
+    assert np.all((g["dlogits"][zero_rows] & 0x7FFF) == 0)
+
+
+def test_gspo_one_token_sequences(grpo, oracle_mod):
+    """Every sequence one token long: the case where GSPO's ratio is the token ratio."""
+    rng = np.random.default_rng(43)
+    c = SeqCase(rng, [1] * 64, 32000, old_sd=0.2)
+    compare_gspo(c.run_gpu(grpo), c.run_oracle(oracle_mod), c)
+
+
+def test_gspo_invalid_token_drops_its_sequence(grpo, oracle_mod):
+    rng = np.random.default_rng(44)
+    c = SeqCase(rng, [6, 6, 6], 5000)
+    c.y[8] = 5000  # row 8 belongs to sequence 1
+    g, r = c.run_gpu(grpo), c.run_oracle(oracle_mod)
+    assert g["status"] & grpo.binding.DEVFLAG_BAD_TOKEN
+    assert np.isnan(g["ratio"][1]) and np.all((g["dlogits"][6:12] & 0x7FFF) == 0)
+    compare_gspo(g, r, c)
+
+
+def test_gspo_deterministic(grpo):
+    rng = np.random.default_rng(45)
+    c = SeqCase(rng, list(rng.integers(10, 200, size=12)), 152064)
+    a, b = c.run_gpu(grpo), c.run_gpu(grpo)
+    assert a["loss"] == b["loss"] and np.array_equal(a["dlogits"], b["dlogits"])
+    assert np.array_equal(a["ratio"], b["ratio"])
+
+
+def test_gspo_no_rows(grpo):
+    """Two empty sequences (no rows gathered from a 7-row buffer): the loss is 0."""
+    rng = np.random.default_rng(46)
+    c = SeqCase(rng, [0, 0], 1000, gather=True)
+    g = c.run_gpu(grpo)
+    assert g["loss"] == 0.0 and g["status"] == 0 and np.all(np.isnan(g["ratio"]))

@@ -270,3 +270,31 @@ def test_host_inputs_step_equals_resident_step(name, graph):
         assert int(step.status.item()) == 0
         assert h2d == small + TK * w.V * host["logits"].element_size()
         assert d2h == 16 + 4 * step.P + step.keep.numel() + 8
+
+
+@pytest.mark.parametrize("name", ["tiny", "small"])
+def test_gspo_step_matches_oracle(oracle_mod, name):
+    """The whole step with GSPO's sequence-level ratio: the compaction's kept offsets and kept
+    rollout indices are the sequences; loss, logp, ratios and dlogits against the oracle."""
+    import torch
+    from test_gpu_gspo import RATIO_RTOL
+    w, b, step, h = build(name, chunk_rows=0, ratio_level="sequence", eps_low=0.2,
+                          eps_high=0.28)
+    step.run()
+    torch.cuda.synchronize()
+    assert int(step.status.item()) == 0
+    adv, comp = check_selection(oracle_mod, w, b, step)
+    TK, K = step.T_kept, step.K
+    ref = oracle_mod.gspo_loss(host_bits(h["logits"]), w.V, b["ids"], h["old"], h["ref"], adv,
+                               comp["kept_idx"][:K], comp["kept_off"][:K + 1], eps_low=0.2, eps_high=0.28,
+                               beta=w.beta, row_index=comp["src_token"],
+                               dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
+    np.testing.assert_allclose(step.seq_ratio[:K].cpu().numpy(), ref["seq_ratio"], rtol=RATIO_RTOL)
+    assert np.abs(step.logp[:TK].cpu().numpy().astype(np.float64) - ref["logp"]).max() <= 2e-5
+    d = host_bits(step.dlogits[:TK])
+    if w.dlogits_dtype == "bf16":
+        from helpers import bf16_ulp_distance
+        assert int(bf16_ulp_distance(d, ref["dlogits"]).max()) <= 1
+    else:
+        assert np.abs(d.astype(np.float64) - ref["dlogits"].astype(np.float64)).max() <= 1e-6
+    assert abs(float(step.loss.item()) - ref["loss"]) <= LOSS_RTOL * abs(ref["loss"]) + 1e-12
