@@ -99,7 +99,7 @@ def measured_peak():
 
 def loss_source_hash():
     h = hashlib.sha256()
-    for f in ("loss.cu", "common.cuh"):
+    for f in ("loss.cu", "gspo.cu", "rowops.cuh", "common.cuh"):
         with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
