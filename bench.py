@@ -365,6 +365,7 @@ def main():
     K = args.steps
     stream = torch.cuda.current_stream()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
     l0 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
     l1 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
     if world > 1:
@@ -378,6 +379,7 @@ def main():
     kept = 0
     ev0.record(stream)
     for i in range(K):
+        s0[i].record(stream)
         if use_graph:  # the step as two graph replays; the host reads the counts at its end
             step.replay_select()
             l0[i].record(stream)
@@ -397,6 +399,7 @@ def main():
     g.check_status(step.status)
     elapsed_ms = ev0.elapsed_time(ev1)
     loss_ms = statistics.mean(a.elapsed_time(z) for a, z in zip(l0, l1))
+    select_ms = statistics.mean(a.elapsed_time(z) for a, z in zip(s0, l0))
     elapsed_ms, kept_all = combine_ranks(elapsed_ms, kept, world, dev)
     value = kept_all / (elapsed_ms / 1e3)
 
@@ -495,6 +498,11 @@ def main():
             "gpu_launches": int(launches), "cuda_graph": use_graph,
             "roofline": roofline, "e2e": e2e,
             "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd,
+            "path_overhead": {"select_ms": select_ms,
+                              "other_ms": elapsed_ms / K - select_ms - loss_ms,
+                              "note": "select_ms: advantage, prune, compaction (and the kept-count"
+                                      " read when host-synced), CUDA events; other_ms: the rest"
+                                      " of the step (host ARS update, launch gaps)"},
             "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,
         }
         print(json.dumps(line), flush=True)

@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libfastrl_grpo.so")
-SOURCES = ["api.cu", "advantage.cu", "prune.cu", "compact.cu", "loss.cu", "gspo.cu"]
+SOURCES = ["api.cu", "advantage.cu", "prune.cu", "compact.cu", "loss.cu", "gspo.cu", "reduce.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I", INCLUDE, "-I", CSRC]

@@ -34,6 +34,11 @@ grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype,
                       const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
                       float* logp_out, float4* stats_out, int32_t* status, cudaStream_t s);
 
+// reduce.cu: *out = v[0] + ... + v[m-1] in fp64 in a fixed order, m = n or, with counts
+// (device {K, T_kept}, nullable), min(n, T_kept); one single-CTA launch on `s`.
+grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* counts, double* out,
+                            cudaStream_t s, const char* who);
+
 // ---- device side -----------------------------------------------------------------------------
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {

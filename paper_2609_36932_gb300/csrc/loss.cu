@@ -511,21 +511,6 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
   cluster_sync();  // partners are done reading this CTA's shared memory
 }
 
-__global__ void sum_rows_kernel(const double* __restrict__ v, int64_t n, const int64_t* __restrict__ counts,
-                                double* __restrict__ out) {
-  __shared__ double sh[1024];
-  if (counts && counts[1] < n) n = counts[1];
-  double acc = 0.0;
-  for (int64_t i = threadIdx.x; i < n; i += 1024) acc += v[i];
-  sh[threadIdx.x] = acc;
-  __syncthreads();
-  for (int s = 512; s > 0; s >>= 1) {
-    if ((int)threadIdx.x < s) sh[threadIdx.x] += sh[threadIdx.x + s];
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) *out = sh[0];
-}
-
 // ---- host side --------------------------------------------------------------------------------
 
 struct Tune {
@@ -718,14 +703,6 @@ extern "C" grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int
   return GRPO_OK;
 }
 
-extern "C" grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grpo_stream_t stream) {
-  clear_error();
-  if (n < 0 || out == nullptr || (n > 0 && v == nullptr))
-    return fail(GRPO_ERR_INVALID_ARG, "grpo_sum_f64: n = %lld, v or out NULL", (long long)n);
-  sum_rows_kernel<<<1, 1024, 0, as_stream(stream)>>>(v, n, nullptr, out);
-  count_launches(1);
-  return check_launch("grpo_sum_f64");
-}
 
 namespace fastrl {
 namespace {
@@ -770,9 +747,7 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   double* row_loss = row_loss_out ? row_loss_out : static_cast<double*>(ws);
   cudaStream_t s = as_stream(stream);
   if (n_rows == 0) {
-    sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, 0, nullptr, loss_out);
-    count_launches(1);
-    return check_launch(who);
+    return launch_sum_rows(row_loss, 0, nullptr, loss_out, s, who);
   }
   if (!logits || !y || !old_logp || !ref_logp || !adv || !row_rollout || !dlogits)
     return fail(GRPO_ERR_INVALID_ARG, "%s: NULL array", who);
@@ -821,9 +796,8 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   st = launch_rows(kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads)),
                    sh, a, s, who);
   if (st != GRPO_OK) return st;
-  sum_rows_kernel<<<1, 1024, 0, s>>>(row_loss, n_rows, counts, loss_out);
-  count_launches(2);
-  return check_launch(who);
+  count_launches(1);
+  return launch_sum_rows(row_loss, n_rows, counts, loss_out, s, who);
 }
 
 }  // namespace

@@ -222,7 +222,10 @@ __global__ void unigram_set_kernel(const int32_t* __restrict__ ids, const int64_
   }
 }
 
-__global__ void bitmap_pair_kernel(int G, float tau, PruneWs w) {
+constexpr int kPairThreads = 256;
+constexpr int kPairUnroll = 4;
+
+__global__ void __launch_bounds__(kPairThreads) bitmap_pair_kernel(int G, float tau, PruneWs w) {
   __shared__ int warp_cnt[32];
   const int pairs = G * (G - 1) / 2;
   const int p = blockIdx.x / pairs;
@@ -237,7 +240,18 @@ __global__ void bitmap_pair_kernel(int G, float tau, PruneWs w) {
   const uint64_t* a = w.bitmaps + (int64_t)ri * w.words;
   const uint64_t* b = w.bitmaps + (int64_t)rj * w.words;
   int cnt = 0;
-  for (int k = threadIdx.x; k < w.words; k += blockDim.x) cnt += __popcll(a[k] & b[k]);
+  // kPairUnroll independent loads of each bitmap per thread before any is used
+  for (int k0 = threadIdx.x; k0 < w.words; k0 += blockDim.x * kPairUnroll) {
+    uint64_t x[kPairUnroll], y[kPairUnroll];
+#pragma unroll
+    for (int u = 0; u < kPairUnroll; ++u) {
+      const int k = k0 + u * (int)blockDim.x;
+      x[u] = k < w.words ? a[k] : 0ull;
+      y[u] = k < w.words ? b[k] : 0ull;
+    }
+#pragma unroll
+    for (int u = 0; u < kPairUnroll; ++u) cnt += __popcll(x[u] & y[u]);
+  }
   for (int s = 16; s > 0; s >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, s);
   if ((threadIdx.x & 31) == 0) warp_cnt[threadIdx.x >> 5] = cnt;
   __syncthreads();
@@ -480,7 +494,7 @@ extern "C" grpo_status grpo_prune(const float* rewards, const float* adv, float 
     unigram_set_kernel<<<nroll, 256, (size_t)w.words * 8, s>>>(ids, off, V, w, status);
     ++launches;
     if (pairs > 0) {
-      bitmap_pair_kernel<<<(unsigned)((int64_t)P * pairs), 128, 0, s>>>(G, tau, w);
+      bitmap_pair_kernel<<<(unsigned)((int64_t)P * pairs), kPairThreads, 0, s>>>(G, tau, w);
       ++launches;
     }
   } else {

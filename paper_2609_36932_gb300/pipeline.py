@@ -68,6 +68,10 @@ class GrpoStep:
         self.counts_host = torch.empty(2, dtype=torch.int64, pin_memory=True)
         self.kpp_host = torch.empty(max(self.P, 1), dtype=torch.int32, pin_memory=True)
         self.keep_host = torch.empty(max(n, 1), dtype=torch.uint8, pin_memory=True)
+        # numpy views of the pinned buffers: the per-step host reads avoid tensor indexing
+        self._stream = torch.cuda.current_stream(dev)
+        self._counts_np = self.counts_host.numpy()
+        self._kpp_np = self.kpp_host[:max(self.P, 1)].numpy()[:self.P]
         self.loss = torch.empty(1, dtype=torch.float64, device=dev)
         self.logp = torch.empty(max(self.T, 1), dtype=torch.float32, device=dev)
         self.out_dtype = torch.bfloat16 if params.dlogits_dtype == "bf16" else torch.float32
@@ -217,6 +221,7 @@ class GrpoStep:
         with torch.cuda.graph(self.g_loss):
             self._enqueue_loss()
         torch.cuda.synchronize()
+        self._stream = torch.cuda.current_stream()
 
     def replay_select(self):
         self.g_select.replay()
@@ -226,18 +231,18 @@ class GrpoStep:
 
     def finish(self):
         """After a replayed step: wait for it, read the kept counts and update ARS (Phase 1b)."""
-        self.torch.cuda.current_stream().synchronize()
+        self._stream.synchronize()
         return self._read_counts()
 
     def _read_counts(self):
         """Kept counts from the host copies; then Algorithm 1, Phase 1(b) then 1(a): the rollout
         count for the next step."""
-        self.K = int(self.counts_host[0])
-        self.T_kept = int(self.counts_host[1])
+        self.K = int(self._counts_np[0])
+        self.T_kept = int(self._counts_np[1])
         self.step_index += 1
         s = (self.step_index - 1) % self.ars_total + 1
-        self.n_next = B.adaptive_rollout_count(self.ars, self.kpp_host[:self.P].numpy(), s,
-                                               self.ars_total, s % self.steps_per_epoch == 0)
+        self.n_next = B.adaptive_rollout_count(self.ars, self._kpp_np, s, self.ars_total,
+                                               s % self.steps_per_epoch == 0)
         return self.T_kept
 
     def run_graph(self):
