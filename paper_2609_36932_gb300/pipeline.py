@@ -13,6 +13,8 @@ from __future__ import annotations
 
 import dataclasses
 
+import numpy as np
+
 from . import binding as B
 
 
@@ -259,15 +261,22 @@ class GrpoStep:
 
     SMALL_INPUTS = ("rewards", "ids", "off", "old", "ref")
 
-    def run_from_host(self, host: dict, loss_host=None):
+    def run_from_host(self, host: dict, loss_host=None, overlap_groups: int = 4):
         """One step whose inputs start in host memory (pinned, for asynchronous copies): `host`
         holds tensors 'rewards', 'ids', 'off', 'old', 'ref' and 'logits' shaped like the device
         inputs.  The selection inputs and the per-token log-probs are copied whole; after the
         selection, only the kept rollouts' logit rows are copied (grpo_upload_kept), since the
-        pruned rollouts take no further part in the step (Sec. 3.2).  Uses the captured graphs
-        when `capture()` has run.  The loss is copied into `loss_host` (f64 [1]) if given.
-        Returns (h2d_bytes, d2h_bytes) moved by this step."""
+        pruned rollouts take no further part in the step (Sec. 3.2).
+
+        With overlap_groups > 1 (token-level loss in one call), the kept rollouts are uploaded in
+        that many groups on a copy stream, and the loss runs over each group's rows as soon as
+        they have landed; the per-row terms are summed once at the end in the loss's fixed order,
+        so the result equals a single call's bit for bit.  Otherwise the upload completes first
+        and the loss runs as in `loss_step` (the captured graph when `capture()` has run).
+        The loss is copied into `loss_host` (f64 [1]) if given.  Returns (h2d_bytes, d2h_bytes)
+        moved by this step."""
         torch = self.torch
+        p = self.p
         dev_of = dict(rewards=self.rewards, ids=self.ids, off=self.off, old=self.old, ref=self.ref)
         h2d = 0
         for k in self.SMALL_INPUTS:
@@ -278,21 +287,75 @@ class GrpoStep:
             self.replay_select()
         else:
             self._enqueue_select()
-        torch.cuda.current_stream().synchronize()
+        self._stream.synchronize()
         self._read_counts()
         n = self.keep.numel()
-        up, _ = B.grpo_upload_kept(host["logits"], self.logits, self.keep_host[:n], host["off"])
-        h2d += up
-        if graphed:
-            self.replay_loss()
+        overlap = overlap_groups > 1 and p.chunk_rows == 0 and p.ratio_level == "token"
+        if overlap and self.T_kept > 0:
+            h2d += self._upload_and_loss_overlapped(host, overlap_groups)
         else:
-            self.loss_step()
+            up, _ = B.grpo_upload_kept(host["logits"], self.logits, self.keep_host[:n], host["off"])
+            h2d += up
+            if graphed and p.chunk_rows == 0 and p.ratio_level == "token":
+                self.replay_loss()
+            else:
+                self.loss_step()
         d2h = 2 * 8 + 4 * self.P + n
         if loss_host is not None:
             loss_host.copy_(self.loss, non_blocking=True)
             d2h += 8
-        torch.cuda.current_stream().synchronize()
+        self._stream.synchronize()
         return h2d, d2h
+
+    def _upload_and_loss_overlapped(self, host, groups: int) -> int:
+        """Upload the kept rollouts' logit rows in `groups` groups of about equal rows on a copy
+        stream; the loss over each group's compacted rows waits only for that group."""
+        torch = self.torch
+        p = self.p
+        n = self.keep.numel()
+        keep = self.keep_host.numpy()[:n].astype(bool)
+        off = host["off"].numpy()
+        lens = np.diff(off)
+        kept = np.flatnonzero(keep)
+        # compacted row offset of each kept rollout, and group boundaries by rows
+        rows_before = np.concatenate([[0], np.cumsum(lens[kept])])
+        T = int(rows_before[-1])
+        bounds = [0]
+        for g in range(1, groups):
+            k = int(np.searchsorted(rows_before, T * g / groups, side="left"))
+            if k > bounds[-1] and k < kept.size:
+                bounds.append(k)
+        bounds.append(kept.size)
+        if getattr(self, "_copy_stream", None) is None:
+            self._copy_stream = torch.cuda.Stream(self.dev)
+            self.row_loss = torch.empty(max(self.T, 1), dtype=torch.float64, device=self.dev)
+        self._ensure_dlogits(self.T_kept)
+        cs = self._copy_stream
+        cs.wait_stream(self._stream)  # the previous step's loss is done with the logits buffer
+        up = 0
+        for g in range(len(bounds) - 1):
+            ka, kb = bounds[g], bounds[g + 1]
+            ra, rb = int(kept[ka]), int(kept[kb - 1]) + 1  # rollouts covering the group
+            with torch.cuda.stream(cs):
+                sub_keep = self.keep_host[ra:rb]
+                nb, _ = B.grpo_upload_kept(host["logits"], self.logits, sub_keep,
+                                           host["off"][ra:rb + 1])
+                up += nb
+                ev = torch.cuda.Event()
+                ev.record(cs)
+            self._stream.wait_event(ev)
+            c0, c1 = int(rows_before[ka]), int(rows_before[kb])
+            if c1 > c0:
+                B.grpo_loss_fwd_bwd(
+                    self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout[c0:c1],
+                    V=p.V, row_index=self.src_token[c0:c1], n_rows=c1 - c0, eps_low=p.eps_low,
+                    eps_high=p.eps_high, beta=p.beta, agg_mode=p.agg_mode,
+                    denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
+                    dlogits=self.dlogits[c0:c1], dlogits_dtype=self.out_dtype,
+                    logp_out=self.logp[c0:c1], row_loss_out=self.row_loss[c0:c1],
+                    loss_out=self.loss, status=self.status)
+        B.grpo_sum_f64(self.row_loss, self.T_kept, out=self.loss)
+        return up
 
     def kept_rows(self):
         """(src_token, token_rollout) of the kept rows as host arrays."""

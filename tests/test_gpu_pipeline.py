@@ -232,12 +232,14 @@ def test_upload_kept_copies_only_kept_rows():
         assert copies == runs and runs >= 1
 
 
-@pytest.mark.parametrize("name,graph", [("tiny", False), ("tiny", True), ("small", True),
-                                        ("qwen", True)])
-def test_host_inputs_step_equals_resident_step(name, graph):
-    """A step from pinned host inputs copies only the kept rollouts' logit rows.  It gives the
-    resident step's selection, loss, logp and dlogits bit for bit, although every device input
-    was poisoned beforehand (NaN logits everywhere): no pruned row is read."""
+@pytest.mark.parametrize("name,graph,groups", [("tiny", False, 1), ("tiny", True, 4),
+                                               ("small", True, 1), ("small", False, 4),
+                                               ("qwen", True, 4)])
+def test_host_inputs_step_equals_resident_step(name, graph, groups):
+    """A step from pinned host inputs copies only the kept rollouts' logit rows, whole (groups = 1)
+    or in groups whose loss starts as each lands (groups = 4).  It gives the resident step's
+    selection, loss, logp and dlogits bit for bit, although every device input was poisoned
+    beforehand (NaN logits everywhere): no pruned row is read."""
     import torch
     w, b, step, h = build(name, chunk_rows=0)
     step.run()
@@ -262,7 +264,7 @@ def test_host_inputs_step_equals_resident_step(name, graph):
     loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
     small = sum(host[k].numel() * host[k].element_size() for k in step.SMALL_INPUTS)
     for _ in range(2):
-        h2d, d2h = step.run_from_host(host, loss_host)
+        h2d, d2h = step.run_from_host(host, loss_host, overlap_groups=groups)
         assert (step.T_kept, step.K) == (TK, K)
         assert float(loss_host.item()) == ref_loss
         assert torch.equal(step.keep, ref_keep)
