@@ -451,10 +451,18 @@ def main():
     e2e = None
     names = ["rewards", "ids", "off", "logits", "old", "ref"]
     h2d = sum(d[k].numel() * d[k].element_size() for k in names)
-    if args.e2e_steps > 0 and h2d > 0.6 * host_mem_available():
+    # every rank of this host pins its own copy: the budget is shared, and all ranks must agree
+    # (the end-to-end leg has a barrier and cross-rank reductions)
+    local_ranks = max(1, int(os.environ.get("LOCAL_WORLD_SIZE", "1")))
+    fits = h2d <= 0.6 * host_mem_available() / local_ranks
+    if world > 1:
+        flag = torch.tensor([1 if fits else 0], dtype=torch.int32, device=dev)
+        dist.all_reduce(flag, op=dist.ReduceOp.MIN)
+        fits = bool(flag.item())
+    if args.e2e_steps > 0 and not fits:
         e2e = {"value": None, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 0,
-               "skipped": "pinned host copies of the inputs (%.0f GB) exceed 60%% of available host"
-                          " memory" % (h2d / 1e9)}
+               "skipped": "pinned host copies of the inputs (%.0f GB per rank) exceed 60%% of the"
+                          " available host memory shared by this host's ranks" % (h2d / 1e9)}
     elif args.e2e_steps > 0:
         host = {}
         for k in names:
