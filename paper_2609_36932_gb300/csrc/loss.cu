@@ -177,6 +177,9 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
   constexpr int kVec = Fmt<InT>::kVec;
   constexpr int kPairs = Fmt<InT>::kPairs;
   constexpr int kWarps = kThreads / 32;
+  // Two vectors per thread in flight in the element loops (measured on GB300: +0.7-1.5% with
+  // bf16 dlogits, within +-0.4% with f32 dlogits, where a forced 1 was 1% slower).
+  constexpr int kUnroll = 2;
   extern __shared__ __align__(128) unsigned char smem[];
   const int buf_bytes = (int)align_up((size_t)a.slice * sizeof(InT), 128);
   InT* buf = reinterpret_cast<InT*>(smem);
@@ -295,6 +298,7 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
       const int v1 = min(nvec, v0 + a.chunk_vecs);
       const bool last = (k == a.n_chunks - 1);
       typename Fmt<InT>::Max mx;
+#pragma unroll 4
       for (int j = v0 + tid; j < v1; j += kThreads) mx.add(buf4[j]);
       float cm = mx.get();
       if (last) {
@@ -312,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
         const float sh = -m * kLog2e;
         const float2 sh2 = make_float2(sh, sh);
         float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll kUnroll
         for (int j = v0 + tid; j < v1; j += kThreads) {
           float2 p[kPairs];
           Fmt<InT>::pairs(buf4[j], p);
@@ -466,6 +471,7 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
       const int v1 = min(nvec, v0 + a.chunk_vecs);
       const bool last = (k == a.n_chunks - 1);
       if (!zero_row) {
+#pragma unroll kUnroll
         for (int j = v0 + tid; j < v1; j += kThreads) {
           float2 p[kPairs], d[kPairs];
           Fmt<InT>::pairs(buf4[j], p);
