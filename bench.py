@@ -408,7 +408,7 @@ def main():
         # in these workloads: beta > 0)
         bytes_per_row = w.V * (2 * w.in_bytes + w.out_bytes) + GSPO_SIDE_BYTES_PER_ROW
         per_row_traffic = profiled_traffic(w.name + "/gspo")
-        kernel = ("GSPO loss: grpo_loss_kernel<..., forward only> with row statistics, "
+        kernel = ("GSPO loss: logp_stream_kernel with row statistics, "
                   "gspo_seq_kernel, gspo_dlogits_kernel, fixed-order sum")
     else:
         bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
@@ -441,7 +441,7 @@ def main():
         torch.cuda.synchronize()
         f_ms = f0.elapsed_time(f1) / nrep
         f_bytes = step.T_kept * (w.V * w.in_bytes + 16)
-        logp_fwd = {"kernel": "grpo_loss_kernel<..., forward only>", "launch_ms": f_ms,
+        logp_fwd = {"kernel": "logp_stream_kernel", "launch_ms": f_ms,
                     "achieved": f_bytes / (f_ms / 1e3) / 1e9, "unit": "GB/s",
                     "frac": f_bytes / (f_ms / 1e3) / 1e9 / peak,
                     "kept_tokens_per_s": step.T_kept / (f_ms / 1e3),

@@ -218,9 +218,9 @@ grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t 
  * logits, row_stride, row_index, y: as grpo_loss_fwd_bwd.  logp_out device f32 [n_rows].
  * status: device i32, nullable (GRPO_DEVFLAG_BAD_TOKEN leaves logp = NaN, GRPO_DEVFLAG_NONFINITE).
  * Limits: as grpo_loss_fwd_bwd.  No workspace.
- * At the same launch shape (grpo_loss_tune) logp_out equals grpo_loss_fwd_bwd's bit for bit, so
- * the ratio of a policy to itself is exactly 1.  The automatic shapes differ (one copy per slice
- * here, two in the fused loss), and then the two agree to within rounding of the sum.
+ * Kernel: one CTA streams each row (no cluster, no shared-memory slice; grpo_loss_tune does not
+ * apply).  Its sums run in a different order from the fused loss's, so the two log-probabilities
+ * agree to within a few ulps, not bit for bit; each is deterministic.
  */
 grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
                           const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
@@ -327,7 +327,7 @@ grpo_status grpo_loss_fwd_bwd_noalloc(const void* logits, int32_t logits_dtype,
  * (0 = automatic); chunks: copies each CTA splits its slice into (1..16, 0 = automatic).
  * Every shape meets the same accuracy; the shape sets the order of the floating-point sums, so
  * results may differ between shapes in the last bits, and one shape always gives the same bits.
- * grpo_logp_fwd uses the same settings.  Returns GRPO_ERR_INVALID_ARG for other values.
+ * grpo_logp_fwd does not use these settings.  Returns GRPO_ERR_INVALID_ARG for other values.
  */
 grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int32_t chunks);
 
