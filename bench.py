@@ -269,6 +269,50 @@ def cpu_baseline_ours(w, b, step, dev_inputs, target_s):
                       % (t_sel, step.T_kept, n, t_loss)}
 
 
+def cpu_baseline_gspo(w, b, step, dev_inputs, target_s):
+    """GSPO's oracle timed on a bounded sample: selection on the whole batch, then the sequence-
+    level loss over the first kept sequences (whole sequences: a ratio needs all of its rows)."""
+    import torch
+    import oracle
+    cores = int(oracle.set_threads(0))
+    t0 = time.perf_counter()
+    adv, _ = oracle.advantage(b["rewards"], w.G)
+    keep, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+    comp = oracle.compact(keep, b["off"])
+    t_sel = time.perf_counter() - t0
+    K, T_kept = comp["K"], comp["T_kept"]
+    if K == 0 or T_kept == 0:
+        return None
+    kept_idx, kept_off = comp["kept_idx"][:K], comp["kept_off"][:K + 1]
+    old = dev_inputs["old"].cpu().numpy()
+    ref = dev_inputs["ref"].cpu().numpy()
+    dev = dev_inputs["logits"].device
+
+    def run(nseq):
+        rows = comp["src_token"][:kept_off[nseq]]
+        bits = host_logits_bits(dev_inputs["logits"][torch.from_numpy(rows).to(dev)])
+        t = time.perf_counter()
+        oracle.gspo_loss(bits, w.V, b["ids"][rows], old[rows], ref[rows], adv, kept_idx[:nseq],
+                         kept_off[:nseq + 1], n_seq=K, eps_low=w.eps, eps_high=w.eps, beta=w.beta,
+                         dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
+        return time.perf_counter() - t, int(kept_off[nseq])
+
+    k = 1
+    while k < K and kept_off[k] == 0:
+        k += 1
+    t1, r1 = run(k)
+    per_row = max(t1 / max(r1, 1), 1e-6)
+    target_rows = target_s / per_row
+    while k < K and kept_off[k + 1] <= target_rows:
+        k += 1
+    t, rows = run(k)
+    t_per_token = t / max(rows, 1) + t_sel / max(T_kept, 1)
+    return {"value": 1.0 / t_per_token, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "fp64 oracle: advantage+prune+compact on the whole batch (%.2f s, amortised"
+                      " over its %d kept tokens) + GSPO's sequence-level loss on the first %d kept"
+                      " sequences (%d rows, %.2f s)" % (t_sel, T_kept, k, rows, t)}
+
+
 def run_reference(args, w):
     """The reference arm: the fp64 oracle as it stands, on this machine's host cores."""
     import torch
@@ -493,8 +537,11 @@ def main():
         del host
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.loss == "grpo":
-        cpu = cpu_baseline_ours(w, b, step, d, args.cpu_seconds)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        if args.loss == "gspo":
+            cpu = cpu_baseline_gspo(w, b, step, d, args.cpu_seconds)
+        else:
+            cpu = cpu_baseline_ours(w, b, step, d, args.cpu_seconds)
 
     if rank == 0:
         line = {
