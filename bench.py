@@ -400,7 +400,7 @@ def main():
     step.run()
     torch.cuda.synchronize()
     launches_per_step = g.grpo_kernel_launches() - l_before
-    use_graph = not args.no_graph and w.chunk_rows == 0 and args.loss == "grpo"
+    use_graph = not args.no_graph and step.p.chunk_rows == 0
     if use_graph:
         step.capture()
         for _ in range(max(args.warmup, 3)):

@@ -261,6 +261,29 @@ grpo_status grpo_gspo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int
                                    grpo_stream_t stream);
 
 /*
+ * grpo_gspo_loss_fwd_bwd_dev — grpo_gspo_loss_fwd_bwd with the row and sequence counts read on the
+ * device, so that a step with GSPO's loss can be captured in a CUDA graph (as
+ * grpo_loss_fwd_bwd_dev for the token-level loss).
+ * counts    device i64 [2] = {K, T_kept}, e.g. grpo_compact's counts.  Rows processed:
+ *           min(max_rows, T_kept); sequences: min(max_seqs, K); n_seq <= 0 takes K as the mean's
+ *           denominator.
+ * max_rows, max_seqs  host capacities: dlogits [max_rows, V], logp_out, seq_row_off
+ *           [max_seqs+1], seq_rollout, seq_ratio_out and the workspace are sized for them.
+ * Entries past the device counts are not written.  All other arguments as
+ * grpo_gspo_loss_fwd_bwd.
+ */
+grpo_status grpo_gspo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype,
+                                       int64_t row_stride, const int64_t* row_index,
+                                       int64_t max_rows, int32_t max_seqs, const int64_t* counts,
+                                       int32_t V, const int32_t* y, const float* old_logp,
+                                       const float* ref_logp, const float* adv,
+                                       const int32_t* seq_rollout, const int64_t* seq_row_off,
+                                       int64_t n_seq, float eps_low, float eps_high, float beta,
+                                       void* dlogits, int32_t dlogits_dtype, float* logp_out,
+                                       float* seq_ratio_out, double* loss_out, int32_t* status,
+                                       void* ws, size_t* ws_bytes, grpo_stream_t stream);
+
+/*
  * grpo_sum_f64 — *out = v[0] + ... + v[n-1] in fp64, in the same fixed order grpo_loss_fwd_bwd
  * uses for loss_out (bitwise reproducible).  With row_loss_out, a loss computed over rows in
  * several calls (for example chunks of kept rows sharing one dlogits buffer) then sums to

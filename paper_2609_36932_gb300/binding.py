@@ -31,7 +31,8 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
-           "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_sum_f64", "grpo_logp_fwd",
+           "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
+           "grpo_sum_f64", "grpo_logp_fwd",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -98,6 +99,11 @@ def lib():
                                          _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
                                          ctypes.POINTER(ctypes.c_size_t), _c_p]
     L.grpo_gspo_loss_fwd_bwd.restype = _i32
+    L.grpo_gspo_loss_fwd_bwd_dev.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _i32, _c_p,
+                                             _c_p, _c_p, _c_p, _c_p, _c_p, _i64, _f32, _f32, _f32,
+                                             _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                             ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_gspo_loss_fwd_bwd_dev.restype = _i32
     L.grpo_logp_fwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p]
     L.grpo_logp_fwd.restype = _i32
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
@@ -427,6 +433,39 @@ def grpo_gspo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, seq_rollout, seq_
     wst = _workspace(need.value, dev, ws)
     wp, size = _ws_args(wst)
     _check(L.grpo_gspo_loss_fwd_bwd(*head, wp, size, _stream(stream)))
+    return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, seq_ratio=seq_ratio_out, ws=wst)
+
+
+def grpo_gspo_loss_fwd_bwd_dev(logits, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off,
+                               counts, *, max_rows: int, max_seqs: int, dlogits, loss_out, ws,
+                               n_seq: int = 0, V: int | None = None, row_stride: int | None = None,
+                               row_index=None, eps_low: float = 0.2, eps_high: float = 0.2,
+                               beta: float = 0.0, logp_out=None, seq_ratio_out=None, status=None,
+                               stream=None):
+    """GSPO's loss with {K, T_kept} read from the device `counts` (CUDA-graph capturable): the
+    caller passes every buffer, sized for max_rows and max_seqs, and a workspace tensor."""
+    torch = _torch()
+    ldt = GRPO_DTYPE_BF16 if logits.dtype == torch.bfloat16 else GRPO_DTYPE_F32
+    if V is None:
+        V = logits.shape[1]
+    stride = logits.stride(0) if row_stride is None else int(row_stride)
+    odt = GRPO_DTYPE_BF16 if dlogits.dtype == torch.bfloat16 else GRPO_DTYPE_F32
+    _need(counts, torch.int64, 2, "counts")
+    _need(dlogits, dlogits.dtype, max_rows * V, "dlogits")
+    _need(seq_rollout, torch.int32, max_seqs, "seq_rollout")
+    _need(seq_row_off, torch.int64, max_seqs + 1, "seq_row_off")
+    if logp_out is None:
+        raise ValueError("grpo_gspo_loss_fwd_bwd_dev: logp_out is required")
+    head = (_ptr(logits), ldt, stride, _ptr(row_index), int(max_rows), int(max_seqs), _ptr(counts),
+            int(V), _ptr(y), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(seq_rollout),
+            _ptr(seq_row_off), int(n_seq), float(eps_low), float(eps_high), float(beta),
+            _ptr(dlogits), odt, _ptr(logp_out), _ptr(seq_ratio_out), _ptr(loss_out), _ptr(status))
+    L = lib()
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_gspo_loss_fwd_bwd_dev(*head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, logits.device, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_gspo_loss_fwd_bwd_dev(*head, wp, size, _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, seq_ratio=seq_ratio_out, ws=wst)
 
 

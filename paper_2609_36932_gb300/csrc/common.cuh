@@ -27,16 +27,18 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 grpo_status workspace_check(void* ws, size_t* ws_bytes, size_t need, const char* who,
                             bool* query_only);
 
-// Forward-only row kernel (loss.cu): logp_out[t] = z_y - log sum_v exp(z_v) for n_rows rows
-// (rows and errors as grpo_logp_fwd) and, with stats_out, each row's softmax statistics
-// {max M, sum of exp(z - M), that sum without y, 0} (NaN for a token id outside [0, V)).
+// Forward-only row kernel (loss.cu): logp_out[t] = z_y - log sum_v exp(z_v) for n_rows rows, or
+// min(n_rows, counts[1]) with device counts {K, T_kept} (rows and errors as grpo_logp_fwd) and,
+// with stats_out, each row's softmax statistics {max M, sum of exp(z - M), that sum without y, 0}
+// (NaN for a token id outside [0, V)).
 grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype, int64_t row_stride,
-                      const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
-                      float* logp_out, float4* stats_out, int32_t* status, cudaStream_t s);
+                      const int64_t* row_index, int64_t n_rows, const int64_t* counts, int32_t V,
+                      const int32_t* y, float* logp_out, float4* stats_out, int32_t* status,
+                      cudaStream_t s);
 
-// reduce.cu: *out = v[0] + ... + v[m-1] in fp64 in a fixed order, m = n or, with counts
-// (device {K, T_kept}, nullable), min(n, T_kept); one single-CTA launch on `s`.
-grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* counts, double* out,
+// reduce.cu: *out = v[0] + ... + v[m-1] in fp64 in a fixed order, m = n or, with n_dev (a device
+// count, nullable), min(n, *n_dev); one single-CTA launch on `s`.
+grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* n_dev, double* out,
                             cudaStream_t s, const char* who);
 
 // ---- device side -----------------------------------------------------------------------------

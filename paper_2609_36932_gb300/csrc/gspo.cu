@@ -33,6 +33,10 @@ struct SeqArgs {
   double lo, hi;  // 1 - eps_low, 1 + eps_high in fp64
   float beta;
   double inv_nseq;
+  // device counts {K, T_kept} (nullable): sequences min(n_seq_rows, K), rows min(n_rows, T_kept);
+  // with nseq_from_counts the mean's denominator is K
+  const int64_t* counts;
+  int32_t nseq_from_counts;
   float* coef;
   double* seq_loss;
   float* seq_ratio;
@@ -45,10 +49,17 @@ constexpr int kSeqWarps = 8;
 __global__ void __launch_bounds__(kSeqWarps * 32) gspo_seq_kernel(const SeqArgs a) {
   const int lane = threadIdx.x & 31;
   const int64_t k = (int64_t)blockIdx.x * kSeqWarps + (threadIdx.x >> 5);
-  if (k >= a.n_seq_rows) return;
+  int64_t n_seqs = a.n_seq_rows, n_rows = a.n_rows;
+  double inv_nseq = a.inv_nseq;
+  if (a.counts) {
+    n_seqs = a.counts[0] < n_seqs ? a.counts[0] : n_seqs;
+    n_rows = a.counts[1] < n_rows ? a.counts[1] : n_rows;
+    if (a.nseq_from_counts) inv_nseq = a.counts[0] > 0 ? 1.0 / (double)a.counts[0] : 0.0;
+  }
+  if (k >= n_seqs) return;
   int64_t r0 = a.seq_row_off[k], r1 = a.seq_row_off[k + 1];
-  r0 = r0 < 0 ? 0 : (r0 > a.n_rows ? a.n_rows : r0);  // offsets outside [0, n_rows] are clamped
-  r1 = r1 < r0 ? r0 : (r1 > a.n_rows ? a.n_rows : r1);
+  r0 = r0 < 0 ? 0 : (r0 > n_rows ? n_rows : r0);  // offsets outside [0, n_rows] are clamped
+  r1 = r1 < r0 ? r0 : (r1 > n_rows ? n_rows : r1);
   const int64_t L = r1 - r0;
   double slr = 0.0, skl = 0.0;
   int bad = 0;
@@ -80,10 +91,10 @@ __global__ void __launch_bounds__(kSeqWarps * 32) gspo_seq_kernel(const SeqArgs 
   const double surr = fmin(s * A, clipped * A);
   const bool c = (A >= 0.0) ? (s <= a.hi) : (s >= a.lo);
   if (lane == 0) {
-    a.seq_loss[k] = -(surr - (double)a.beta * skl / (double)L) * a.inv_nseq;
+    a.seq_loss[k] = -(surr - (double)a.beta * skl / (double)L) * inv_nseq;
     if (a.seq_ratio) a.seq_ratio[k] = (float)s;
   }
-  const float w = (float)(a.inv_nseq / (double)L);
+  const float w = (float)(inv_nseq / (double)L);
   const float sa = c ? (float)(s * A) : 0.f;
   for (int64_t t = r0 + lane; t < r1; t += 32) {
     const int64_t src = a.row_index ? a.row_index[t] : t;
@@ -105,6 +116,7 @@ struct DlArgs {
   int32_t vec;      // input rows 16-byte aligned: vector loads
   int32_t out_vec;  // output rows 16-byte aligned: vector stores
   int32_t tiles_per_row;
+  const int64_t* counts;  // nullable: rows min(n_rows, counts[1])
 };
 
 constexpr int kDlThreads = 256;
@@ -121,7 +133,9 @@ __global__ void __launch_bounds__(kDlThreads) gspo_dlogits_kernel(const DlArgs a
   const float2 l2e2 = make_float2(kLog2e, kLog2e);
   const int nvec = a.vec ? a.V / kVec : 0;
   const int tail0 = nvec * kVec;
-  const int64_t n_tiles = a.n_rows * a.tiles_per_row;
+  int64_t n_rows = a.n_rows;
+  if (a.counts && a.counts[1] < n_rows) n_rows = a.counts[1];
+  const int64_t n_tiles = n_rows * a.tiles_per_row;
   for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
     const int64_t row = tile / a.tiles_per_row;
     const int seg = (int)(tile - row * a.tiles_per_row);
@@ -236,15 +250,19 @@ GspoWs gspo_ws(void* ws, int64_t n_rows) {
 
 using namespace fastrl;
 
-extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
-    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
-    int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,
-    const float* adv, const int32_t* seq_rollout, const int64_t* seq_row_off, int32_t n_seq_rows,
-    int64_t n_seq, float eps_low, float eps_high, float beta, void* dlogits, int32_t dlogits_dtype,
-    float* logp_out, float* seq_ratio_out, double* loss_out, int32_t* status, void* ws,
-    size_t* ws_bytes, grpo_stream_t stream) {
-  clear_error();
-  const char* who = "grpo_gspo_loss_fwd_bwd";
+namespace fastrl {
+namespace {
+
+// n_rows / n_seq_rows: exact counts, or with counts (device {K, T_kept}) capacities whose used
+// part the kernels read on the device; then n_seq <= 0 takes K as the denominator.
+grpo_status gspo_impl(const char* who, const void* logits, int32_t logits_dtype, int64_t row_stride,
+                      const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
+                      const float* old_logp, const float* ref_logp, const float* adv,
+                      const int32_t* seq_rollout, const int64_t* seq_row_off, int32_t n_seq_rows,
+                      const int64_t* counts, int64_t n_seq, float eps_low, float eps_high,
+                      float beta, void* dlogits, int32_t dlogits_dtype, float* logp_out,
+                      float* seq_ratio_out, double* loss_out, int32_t* status, void* ws,
+                      size_t* ws_bytes, grpo_stream_t stream) {
   if (logits_dtype != GRPO_DTYPE_BF16 && logits_dtype != GRPO_DTYPE_F32)
     return fail(GRPO_ERR_INVALID_ARG, "%s: logits_dtype = %d", who, logits_dtype);
   if (dlogits_dtype != GRPO_DTYPE_BF16 && dlogits_dtype != GRPO_DTYPE_F32)
@@ -254,7 +272,8 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
                 n_seq_rows);
   if (V < 1 || row_stride < V)
     return fail(GRPO_ERR_INVALID_ARG, "%s: V = %d, row_stride = %lld", who, V, (long long)row_stride);
-  if (n_seq <= 0) return fail(GRPO_ERR_INVALID_ARG, "%s: n_seq = %lld", who, (long long)n_seq);
+  if (n_seq <= 0 && counts == nullptr)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: n_seq = %lld", who, (long long)n_seq);
   if (!(beta >= 0.f) || !(eps_low >= 0.f) || !(eps_high >= 0.f))
     return fail(GRPO_ERR_INVALID_ARG, "%s: beta, eps_low, eps_high must be >= 0", who);
   const size_t need = gspo_ws_bytes(n_rows, n_seq_rows);
@@ -280,8 +299,8 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
 
   // 1. log-probabilities and softmax statistics
   if (n_rows > 0) {
-    st = logp_rows(who, logits, logits_dtype, row_stride, row_index, n_rows, V, y, logp_out,
-                   w.stats, status, s);
+    st = logp_rows(who, logits, logits_dtype, row_stride, row_index, n_rows, counts, V, y,
+                   logp_out, w.stats, status, s);
     if (st != GRPO_OK) return st;
     // rows outside every sequence keep coef 0
     e = cudaMemsetAsync(w.coef, 0, (size_t)n_rows * 4, s);
@@ -302,7 +321,9 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
   sa.lo = 1.0 - (double)eps_low;
   sa.hi = 1.0 + (double)eps_high;
   sa.beta = beta;
-  sa.inv_nseq = 1.0 / (double)n_seq;
+  sa.inv_nseq = n_seq > 0 ? 1.0 / (double)n_seq : 0.0;
+  sa.counts = counts;
+  sa.nseq_from_counts = n_seq <= 0 ? 1 : 0;
   sa.coef = w.coef;
   sa.seq_loss = w.seq_loss;
   sa.seq_ratio = seq_ratio_out;
@@ -312,7 +333,8 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
   if (st != GRPO_OK) return st;
 
   // 3. dlogits, streaming
-  if (n_rows == 0) return grpo_sum_f64(w.seq_loss, n_seq_rows, loss_out, stream);
+  const int64_t* k_dev = counts ? counts : nullptr;  // the sum runs over min(n_seq_rows, K) terms
+  if (n_rows == 0) return launch_sum_rows(w.seq_loss, n_seq_rows, k_dev, loss_out, s, who);
   const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   const int out_bytes = dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   const int vec_elems = 16 / in_bytes;
@@ -330,6 +352,7 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
   da.out_vec = (reinterpret_cast<uintptr_t>(dlogits) % 16 == 0) && (((int64_t)V * out_bytes) % 16 == 0);
   const int nvec = da.vec ? V / vec_elems : 0;
   da.tiles_per_row = std::max(1, (nvec + kDlThreads * kDlUnroll - 1) / (kDlThreads * kDlUnroll));
+  da.counts = counts;
   const DlKernel fn = dl_kernel_for(logits_dtype, dlogits_dtype);
   const int inst = (logits_dtype == GRPO_DTYPE_BF16 ? 0 : 2) + (dlogits_dtype == GRPO_DTYPE_BF16 ? 0 : 1);
   int dev = 0;
@@ -359,5 +382,38 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
   if (st != GRPO_OK) return st;
 
   // 4. the loss: the sequences' terms summed in a fixed order
-  return grpo_sum_f64(w.seq_loss, n_seq_rows, loss_out, stream);
+  return launch_sum_rows(w.seq_loss, n_seq_rows, k_dev, loss_out, s, who);
+}
+
+}  // namespace
+}  // namespace fastrl
+
+extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
+    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
+    int64_t n_rows, int32_t V, const int32_t* y, const float* old_logp, const float* ref_logp,
+    const float* adv, const int32_t* seq_rollout, const int64_t* seq_row_off, int32_t n_seq_rows,
+    int64_t n_seq, float eps_low, float eps_high, float beta, void* dlogits, int32_t dlogits_dtype,
+    float* logp_out, float* seq_ratio_out, double* loss_out, int32_t* status, void* ws,
+    size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  return gspo_impl("grpo_gspo_loss_fwd_bwd", logits, logits_dtype, row_stride, row_index, n_rows,
+                   V, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, n_seq_rows, nullptr,
+                   n_seq, eps_low, eps_high, beta, dlogits, dlogits_dtype, logp_out,
+                   seq_ratio_out, loss_out, status, ws, ws_bytes, stream);
+}
+
+extern "C" grpo_status grpo_gspo_loss_fwd_bwd_dev(
+    const void* logits, int32_t logits_dtype, int64_t row_stride, const int64_t* row_index,
+    int64_t max_rows, int32_t max_seqs, const int64_t* counts, int32_t V, const int32_t* y,
+    const float* old_logp, const float* ref_logp, const float* adv, const int32_t* seq_rollout,
+    const int64_t* seq_row_off, int64_t n_seq, float eps_low, float eps_high, float beta,
+    void* dlogits, int32_t dlogits_dtype, float* logp_out, float* seq_ratio_out, double* loss_out,
+    int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  if (counts == nullptr)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_gspo_loss_fwd_bwd_dev: counts is NULL");
+  return gspo_impl("grpo_gspo_loss_fwd_bwd_dev", logits, logits_dtype, row_stride, row_index,
+                   max_rows, V, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, max_seqs,
+                   counts, n_seq, eps_low, eps_high, beta, dlogits, dlogits_dtype, logp_out,
+                   seq_ratio_out, loss_out, status, ws, ws_bytes, stream);
 }

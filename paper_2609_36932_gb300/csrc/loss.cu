@@ -522,7 +522,9 @@ __global__ void __launch_bounds__(kFwdThreads, kFwdResident / kFwdThreads)
   const int nvec = a.bulk ? a.V / kVec : 0;
   const int tail0 = nvec * kVec;
   const float2 l2e2 = make_float2(kLog2e, kLog2e);
-  for (int64_t row = blockIdx.x; row < a.n_rows; row += gridDim.x) {
+  int64_t n_rows = a.n_rows;
+  if (a.counts && a.counts[1] < n_rows) n_rows = a.counts[1];  // device count of kept rows
+  for (int64_t row = blockIdx.x; row < n_rows; row += gridDim.x) {
     const int64_t src = a.row_index ? a.row_index[row] : row;
     const int32_t yv = a.y[src];
     const bool yvalid = yv >= 0 && yv < a.V;
@@ -901,7 +903,7 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
                    sh, a, s, who);
   if (st != GRPO_OK) return st;
   count_launches(1);
-  return launch_sum_rows(row_loss, n_rows, counts, loss_out, s, who);
+  return launch_sum_rows(row_loss, n_rows, counts ? counts + 1 : nullptr, loss_out, s, who);
 }
 
 }  // namespace
@@ -941,8 +943,9 @@ extern "C" grpo_status grpo_loss_fwd_bwd_dev(
 namespace fastrl {
 
 grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype, int64_t row_stride,
-                      const int64_t* row_index, int64_t n_rows, int32_t V, const int32_t* y,
-                      float* logp_out, float4* stats_out, int32_t* status, cudaStream_t s) {
+                      const int64_t* row_index, int64_t n_rows, const int64_t* counts, int32_t V,
+                      const int32_t* y, float* logp_out, float4* stats_out, int32_t* status,
+                      cudaStream_t s) {
   if (logits_dtype != GRPO_DTYPE_BF16 && logits_dtype != GRPO_DTYPE_F32)
     return fail(GRPO_ERR_INVALID_ARG, "%s: logits_dtype = %d", who, logits_dtype);
   if (n_rows < 0 || n_rows >= (int64_t(1) << 31))
@@ -962,6 +965,7 @@ grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype,
   a.logp_out = logp_out;
   a.stats_out = stats_out;
   a.status = status;
+  a.counts = counts;
   a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
   KernelFn fn = logits_dtype == GRPO_DTYPE_BF16 ? logp_stream_kernel<__nv_bfloat16>
                                                 : logp_stream_kernel<float>;
@@ -998,8 +1002,8 @@ extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, i
                                      const int32_t* y, float* logp_out, int32_t* status,
                                      grpo_stream_t stream) {
   clear_error();
-  return logp_rows("grpo_logp_fwd", logits, logits_dtype, row_stride, row_index, n_rows, V, y,
-                   logp_out, nullptr, status, as_stream(stream));
+  return logp_rows("grpo_logp_fwd", logits, logits_dtype, row_stride, row_index, n_rows, nullptr,
+                   V, y, logp_out, nullptr, status, as_stream(stream));
 }
 
 // ---- allocation-free variant ------------------------------------------------------------------

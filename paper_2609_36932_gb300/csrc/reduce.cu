@@ -13,10 +13,10 @@ constexpr int kSumThreads = 1024;
 constexpr int kBatch = 8;
 
 __global__ void __launch_bounds__(kSumThreads)
-    sum_rows_kernel(const double* __restrict__ v, int64_t n, const int64_t* __restrict__ counts,
+    sum_rows_kernel(const double* __restrict__ v, int64_t n, const int64_t* __restrict__ n_dev,
                     double* __restrict__ out) {
   __shared__ double part[kSumThreads / 32];
-  if (counts && counts[1] < n) n = counts[1];
+  if (n_dev && *n_dev < n) n = *n_dev;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   double acc = 0.0;
   for (int64_t base = tid; base < n; base += (int64_t)kSumThreads * kBatch) {
@@ -43,9 +43,9 @@ __global__ void __launch_bounds__(kSumThreads)
 
 }  // namespace
 
-grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* counts, double* out,
+grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* n_dev, double* out,
                             cudaStream_t s, const char* who) {
-  sum_rows_kernel<<<1, kSumThreads, 0, s>>>(v, n, counts, out);
+  sum_rows_kernel<<<1, kSumThreads, 0, s>>>(v, n, n_dev, out);
   count_launches(1);
   return check_launch(who);
 }

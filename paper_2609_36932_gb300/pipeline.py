@@ -196,6 +196,8 @@ class GrpoStep:
 
     def _enqueue_loss(self):
         p = self.p
+        if p.ratio_level == "sequence":
+            return self._enqueue_gspo()
         B.grpo_loss_fwd_bwd_dev(
             self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout, self.counts,
             max_rows=self.T, dlogits=self.dlogits, loss_out=self.loss, ws=self.loss_ws, V=p.V,
@@ -204,14 +206,12 @@ class GrpoStep:
 
     def capture(self):
         """Capture the selection (advantage, prune, compact, count copies) and the loss as two
-        CUDA graphs.  The loss reads the kept-row count on the device, so nothing waits for the
-        host between them; dlogits are sized for all T rows."""
+        CUDA graphs.  The loss reads the kept counts on the device (the token-level loss or, with
+        ratio_level "sequence", GSPO's), so nothing waits for the host between them; dlogits are
+        sized for all T rows."""
         torch = self.torch
         if self.p.chunk_rows > 0:
             raise ValueError("graph mode runs the loss in one call (chunk_rows = 0)")
-        if self.p.ratio_level != "token":
-            raise ValueError("graph mode runs the token-level loss; the sequence-level ratio "
-                             "runs host-synced")
         self._ensure_dlogits(self.T)
         for _ in range(2):  # warm-up outside capture (kernel attributes, occupancy queries)
             self._enqueue_select()
@@ -224,6 +224,21 @@ class GrpoStep:
             self._enqueue_loss()
         torch.cuda.synchronize()
         self._stream = torch.cuda.current_stream()
+
+    def _enqueue_gspo(self):
+        """GSPO's loss with the kept counts read on the device (graph mode)."""
+        torch = self.torch
+        p = self.p
+        n = self.keep.numel()
+        if getattr(self, "seq_ratio", None) is None:
+            self.seq_ratio = torch.empty(max(n, 1), dtype=torch.float32, device=self.dev)
+        out = B.grpo_gspo_loss_fwd_bwd_dev(
+            self.logits, self.ids, self.old, self.ref, self.adv, self.kept_idx, self.kept_off,
+            self.counts, max_rows=self.T, max_seqs=n, dlogits=self.dlogits, loss_out=self.loss,
+            ws=getattr(self, "gspo_dev_ws", None), V=p.V, row_index=self.src_token,
+            eps_low=p.eps_low, eps_high=p.eps_high, beta=p.beta, logp_out=self.logp,
+            seq_ratio_out=self.seq_ratio, status=self.status)
+        self.gspo_dev_ws = out["ws"]  # sized on the warm-up calls, before capture
 
     def replay_select(self):
         self.g_select.replay()
@@ -296,7 +311,7 @@ class GrpoStep:
         else:
             up, _ = B.grpo_upload_kept(host["logits"], self.logits, self.keep_host[:n], host["off"])
             h2d += up
-            if graphed and p.chunk_rows == 0 and p.ratio_level == "token":
+            if graphed and p.chunk_rows == 0:
                 self.replay_loss()
             else:
                 self.loss_step()

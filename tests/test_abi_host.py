@@ -145,6 +145,15 @@ def test_gspo_workspace_query_and_argument_errors(grpo):
     # a real call with NULL sequence arrays is refused before any launch
     big = ctypes.c_size_t(1 << 20)
     assert gspo_call(L, 1000, 152064, 16, ctypes.c_void_p(4096), ctypes.byref(big)) == 1
+    # the device-count variant: counts are required; the size query matches the host variant's
+    def dev_call(counts, size_p):
+        return L.grpo_gspo_loss_fwd_bwd_dev(None, 1, 152064, None, 1000, 16, counts, 152064, None,
+                                            None, None, None, None, None, 0, 0.2, 0.2, 0.0, None,
+                                            1, ctypes.c_void_p(4096), None, None, None, None,
+                                            size_p, None)
+    assert dev_call(None, ctypes.byref(size)) == 1
+    assert dev_call(ctypes.c_void_p(4096), ctypes.byref(size)) == 0
+    assert size.value == up(1000 * 16) + up(1000 * 4) + up(16 * 8)
 
 
 def loss_call(L, n_rows, V, ws, size_p, ldt=1, agg=0, denom=1, row_loss=None, beta=0.04):

@@ -172,3 +172,44 @@ def test_gspo_no_rows(grpo):
     c = SeqCase(rng, [0, 0], 1000, gather=True)
     g = c.run_gpu(grpo)
     assert g["loss"] == 0.0 and g["status"] == 0 and np.all(np.isnan(g["ratio"]))
+
+
+def test_gspo_device_counts_match_host_counts(grpo):
+    """grpo_gspo_loss_fwd_bwd_dev over min(max_seqs, K) sequences and min(max_rows, T_kept) rows,
+    with the mean over K, equals grpo_gspo_loss_fwd_bwd given the same numbers on the host, bit
+    for bit; entries past the counts are not written."""
+    import torch
+    rng = np.random.default_rng(47)
+    lens = [9, 0, 14, 5, 21, 3]
+    c = SeqCase(rng, lens, 32000, old_sd=0.15)
+    off = c.seq_row_off
+    for K in (0, 1, 3, 6):
+        TK = int(off[K])
+        counts = c.t(np.array([K, TK], np.int64))
+        dl_a = torch.zeros((c.n, c.V), dtype=torch.bfloat16, device="cuda")
+        dl_b = torch.zeros_like(dl_a)
+        lp_a = torch.zeros(c.n, dtype=torch.float32, device="cuda")
+        lp_b = torch.zeros_like(lp_a)
+        sr_a = torch.zeros(c.K, dtype=torch.float32, device="cuda")
+        sr_b = torch.zeros_like(sr_a)
+        la = torch.empty(1, dtype=torch.float64, device="cuda")
+        lb = torch.empty(1, dtype=torch.float64, device="cuda")
+        ws = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
+        grpo.binding.grpo_gspo_loss_fwd_bwd_dev(
+            c.dev, c.t(c.y), c.t(c.old), c.t(c.ref), c.t(c.adv), c.t(c.seq_rollout),
+            c.t(c.seq_row_off), counts, max_rows=c.n, max_seqs=c.K, dlogits=dl_a, loss_out=la,
+            ws=ws, eps_low=0.2, eps_high=0.28, beta=0.04, logp_out=lp_a, seq_ratio_out=sr_a)
+        if K:
+            grpo.grpo_gspo_loss_fwd_bwd(
+                c.dev, c.t(c.y), c.t(c.old), c.t(c.ref), c.t(c.adv), c.t(c.seq_rollout),
+                c.t(c.seq_row_off), n_rows=TK, n_seq_rows=K, n_seq=K, eps_low=0.2,
+                eps_high=0.28, beta=0.04, dlogits=dl_b, logp_out=lp_b, seq_ratio_out=sr_b,
+                loss_out=lb)
+        else:
+            lb.zero_()
+        torch.cuda.synchronize()
+        assert la.item() == lb.item()
+        assert torch.equal(dl_a, dl_b) and torch.equal(lp_a, lp_b)  # untouched past TK in both
+        assert np.array_equal(np.isnan(sr_a.cpu().numpy()), np.isnan(sr_b.cpu().numpy()))
+        ok = ~np.isnan(sr_b.cpu().numpy())
+        assert np.array_equal(sr_a.cpu().numpy()[ok], sr_b.cpu().numpy()[ok])

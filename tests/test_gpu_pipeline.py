@@ -127,12 +127,14 @@ def test_full_size_sampled(oracle_mod, name):
         assert torch.equal(step.dlogits[:n_last][-100:], d_last)
 
 
-@pytest.mark.parametrize("name", ["tiny", "qwen"])
-def test_graph_mode_equals_host_synced_step(name):
-    """The step captured as two CUDA graphs (the loss reads the kept count on the device) gives
-    the same selection, loss, logp and dlogits as the host-synced step, on two replays."""
+@pytest.mark.parametrize("name,ratio", [("tiny", "token"), ("qwen", "token"), ("tiny", "sequence"),
+                                        ("small", "sequence")])
+def test_graph_mode_equals_host_synced_step(name, ratio):
+    """The step captured as two CUDA graphs (the loss reads the kept counts on the device) gives
+    the same selection, loss, logp and dlogits as the host-synced step, on two replays, for the
+    token-level loss and for GSPO's sequence-level loss."""
     import torch
-    w, b, step, h = build(name, chunk_rows=0)
+    w, b, step, h = build(name, chunk_rows=0, ratio_level=ratio)
     step.run()
     torch.cuda.synchronize()
     TK = step.T_kept
