@@ -1,11 +1,11 @@
 // grpo_loss_fwd_bwd: fused GRPO token loss and dlogits, Sec. 3.1 Eqs. 1-3, one read of the
-// logits and one write of the gradient.
+// logits and one write of the gradient; and grpo_logp_fwd, the log-probabilities alone.
 //
-// Design (HBM-bound: ~2 bytes read + 2-4 bytes written per vocabulary entry, ~10 flops):
+// Fused loss (HBM-bound: ~2 bytes read + 2-4 bytes written per vocabulary entry, ~10 flops):
 //   * A row of V logits is split over a cluster of C CTAs; CTA c holds the slice
 //     [c*slice, (c+1)*slice) of the row in shared memory for the whole row, so the logits are
-//     read from HBM exactly once.  (V = 152064 bf16 is 297 KiB, more than one SM holds; C = 8
-//     gives 37 KiB slices and several resident CTAs per SM.)
+//     read from HBM exactly once.  (V = 152064 bf16 is 297 KiB, more than one SM holds; by
+//     default C = 4 with bf16 dlogits, 74 KiB slices and 2 CTAs per SM, and C = 8 with f32.)
 //   * Each slice arrives by non-tensor bulk copies (cp.async.bulk, 16-byte granules) in a few
 //     chunks, each completing on its own mbarrier, so the CTA starts reducing chunk 0 while
 //     the rest is in flight.
@@ -20,9 +20,12 @@
 //     written with 16-byte streaming stores.  As soon as chunk k has been consumed, thread 0
 //     starts the copy of chunk k of the cluster's next row into the same buffer.
 //   * The grid is persistent: as many clusters as fit at once; cluster i takes rows i, i+n, ...
-//   * Per-row loss terms go to a buffer; a one-CTA kernel sums them in a fixed order.
+//   * Per-row loss terms go to a buffer; a one-CTA kernel (reduce.cu) sums them in a fixed order.
 // Every wait on a copy is bounded (about one second); on expiry the kernel records
 // GRPO_DEVFLAG_TIMEOUT, stops waiting and issuing copies, and runs to the end.
+//
+// Log-probabilities alone (logp_stream_kernel, also GSPO's first pass): no gradient pass, so no
+// slice to keep; one CTA streams each row, and every CTA of the persistent grid is resident.
 #include <cuda_bf16.h>
 
 #include <algorithm>
