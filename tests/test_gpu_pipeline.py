@@ -302,3 +302,33 @@ def test_gspo_step_matches_oracle(oracle_mod, name):
     else:
         assert np.abs(d.astype(np.float64) - ref["dlogits"].astype(np.float64)).max() <= 1e-6
     assert abs(float(step.loss.item()) - ref["loss"]) <= LOSS_RTOL * abs(ref["loss"]) + 1e-12
+
+
+@pytest.mark.parametrize("name,ratio", [("small", "token"), ("small", "sequence")])
+def test_graph_replay_follows_new_inputs(name, ratio):
+    """Graphs captured on one batch, replayed after new rewards are written into the same device
+    buffers (rewards permuted within each prompt: other advantages, another kept set, other
+    counts), give what a fresh host-synced step computes from the new rewards: no host value is
+    baked into the captured graphs."""
+    import torch
+    w, b, step, h = build(name, chunk_rows=0, ratio_level=ratio)
+    step.capture()
+    rng = np.random.default_rng(5)
+    r2 = b["rewards"].reshape(w.P, w.G).copy()
+    for p in range(w.P):
+        r2[p] = r2[p][rng.permutation(w.G)]
+    r2 = torch.from_numpy(r2.reshape(-1)).cuda()
+    k0 = step.run_graph()
+    keep0 = step.keep.clone()
+    step.rewards.copy_(r2)
+    k1 = step.run_graph()
+    assert not torch.equal(step.keep, keep0)  # the permutation changed the kept set
+    loss, logp, dl = float(step.loss.item()), step.logp[:k1].clone(), step.dlogits[:k1].clone()
+    keep = step.keep.clone()
+    w2, b2, fresh, h2 = build(name, chunk_rows=0, ratio_level=ratio)
+    fresh.rewards.copy_(r2)
+    fresh.run()
+    torch.cuda.synchronize()
+    assert fresh.T_kept == k1 and torch.equal(fresh.keep, keep)
+    assert float(fresh.loss.item()) == loss
+    assert torch.equal(fresh.logp[:k1], logp) and torch.equal(fresh.dlogits[:k1], dl)
