@@ -331,3 +331,17 @@ def test_lost_copy_times_out_and_the_context_stays_usable(grpo, oracle_mod):
     assert good["status"] == 0
     compare(good["logp"], good["dlogits"], good["loss"], c.run_oracle(oracle_mod), "bf16",
             gpu_row_loss=good["row_loss"])
+
+
+@pytest.mark.parametrize("V", [262144, 600000])
+def test_large_vocabularies(grpo, oracle_mod, V):
+    """Vocabularies beyond today's common sizes: 7 CTAs per row at V = 262144, and 15 at
+    V = 600000 (a cluster above the portable size of 8)."""
+    rng = np.random.default_rng(V)
+    c = Case(rng, 5, V, "bf16", "bf16")
+    g = c.run_gpu(grpo)
+    r = c.run_oracle(oracle_mod)
+    assert g["status"] == 0
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    lp = grpo.grpo_logp_fwd(c.dev, c.t(c.y)).cpu().numpy()[:5]
+    assert np.abs(lp.astype(np.float64) - r["logp"]).max() <= 2e-5
