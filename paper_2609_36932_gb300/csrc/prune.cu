@@ -15,6 +15,8 @@
 //   3. select_kernel, one warp per prompt: the greedy of Eq. 8 as bitmask operations and the
 //      per-prompt cap by round-robin over classes;
 //   4. dp_fill_kernel (dp_divisor > 1), one thread: cyclic fill to a multiple of the divisor.
+// For n = 1 with at most 64 KiB of bitmaps per prompt, prune_unigram_fused_kernel does steps 0-3
+// in one CTA per prompt, in shared memory.
 // Every decision is an integer or exactly rounded fp64 operation, so the keep mask is bit-exact.
 #include <algorithm>
 #include <atomic>
@@ -320,12 +322,11 @@ __device__ void group_dist(const float* r, int G, double* dist) {
 //     (the continuous-reward grouping |A_i - A_j| < eps, closed under transitivity);
 //   visiting order: |A| descending as |r - mean| descending (fp64, Eq. 5's index-order mean),
 //     lower index first on ties.
-__global__ void class_kernel(const float* __restrict__ rewards, const float* __restrict__ adv,
-                             float class_eps, int P, int G, PruneWs w) {
+// One warp: advantage classes and visiting ranks of prompt p's rollouts, written to cls[0..G)
+// and rank[0..G) (global workspace or shared memory).
+__device__ void classify_warp(const float* __restrict__ rewards, const float* __restrict__ adv,
+                              float class_eps, int p, int G, int lane, int32_t* cls, int32_t* rnk) {
   constexpr unsigned FULL = 0xffffffffu;
-  const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-  const int lane = threadIdx.x & 31;
-  if (p >= P) return;  // uniform per warp
   const bool act = lane < G;
   const float r = act ? rewards[(int64_t)p * G + lane] : 0.f;
   double sum = 0.0;
@@ -365,25 +366,33 @@ __global__ void class_kernel(const float* __restrict__ rewards, const float* __r
       if (__shfl_sync(FULL, chain, j) == chain) label = j;
   }
   if (act) {
-    w.cls[(int64_t)p * G + lane] = label;
-    w.rank[(int64_t)p * G + lane] = rank;
+    cls[lane] = label;
+    rnk[lane] = rank;
   }
 }
 
-// One warp per prompt: the greedy of Eq. 8 and the per-prompt cap as bitmask operations.
-__global__ void select_kernel(int P, int G, int keep_cap, PruneWs w, uint8_t* __restrict__ keep,
-                              int32_t* __restrict__ kept_per_prompt) {
-  constexpr unsigned FULL = 0xffffffffu;
+__global__ void class_kernel(const float* __restrict__ rewards, const float* __restrict__ adv,
+                             float class_eps, int P, int G, PruneWs w) {
   const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-  const int lane = threadIdx.x & 31;
   if (p >= P) return;  // uniform per warp
+  classify_warp(rewards, adv, class_eps, p, G, threadIdx.x & 31, w.cls + (int64_t)p * G,
+                w.rank + (int64_t)p * G);
+}
+
+// One warp per prompt: the greedy of Eq. 8 and the per-prompt cap as bitmask operations.
+// One warp: the greedy of Eq. 8 and the per-prompt cap for one prompt, from its ranks, class
+// labels and G x G closeness bytes; writes keep[0..G) and *kept.
+__device__ void select_warp(int G, int keep_cap, const int32_t* rnk, const int32_t* cls_in,
+                            const uint8_t* close, int lane, uint8_t* __restrict__ keep,
+                            int32_t* __restrict__ kept_out) {
+  constexpr unsigned FULL = 0xffffffffu;
   const bool act = lane < G;
-  const int rank = act ? w.rank[(int64_t)p * G + lane] : 64 + lane;
-  const int label = act ? w.cls[(int64_t)p * G + lane] : -1 - lane;
+  const int rank = act ? rnk[lane] : 64 + lane;
+  const int label = act ? cls_in[lane] : -1 - lane;
   // same-class rollouts within tau of this one
   uint32_t near = 0;
   if (act) {
-    const uint8_t* row = w.close + ((int64_t)p * G + lane) * G;
+    const uint8_t* row = close + lane * G;
     for (int j = 0; j < G; ++j)
       if (j != lane && row[j]) near |= 1u << j;
   }
@@ -422,8 +431,87 @@ __global__ void select_kernel(int P, int G, int keep_cap, PruneWs w, uint8_t* __
     kept = __ballot_sync(FULL, mine && before < keep_cap);
     count = keep_cap;
   }
-  if (act) keep[(int64_t)p * G + lane] = (kept >> lane) & 1u;
-  if (lane == 0) kept_per_prompt[p] = count;
+  if (act) keep[lane] = (kept >> lane) & 1u;
+  if (lane == 0) *kept_out = count;
+}
+
+__global__ void select_kernel(int P, int G, int keep_cap, PruneWs w, uint8_t* __restrict__ keep,
+                              int32_t* __restrict__ kept_per_prompt) {
+  const int p = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  if (p >= P) return;  // uniform per warp
+  select_warp(G, keep_cap, w.rank + (int64_t)p * G, w.cls + (int64_t)p * G,
+              w.close + (int64_t)p * G * G, threadIdx.x & 31, keep + (int64_t)p * G,
+              kept_per_prompt + p);
+}
+
+// n = 1 with small vocabulary bitmaps: the four steps above in one CTA per prompt (classes and
+// ranks, bitmaps and set sizes, pair tests, selection), with every intermediate in shared
+// memory.  Same arithmetic and decisions as the separate kernels.  Measured on GB300: it saves
+// launches where each prompt's work is small (V = 1024: 26 us against 30 us for the selection),
+// ties at V = 32000, and loses at V = 152064 (one CTA per prompt is too little parallelism for
+// 8 x 19 KiB bitmaps and 28 pair tests), so it is used up to 64 KiB of bitmaps per prompt.
+constexpr int kFusedThreads = 1024;
+constexpr size_t kFusedMaxBitmapBytes = 64 * 1024;
+
+__global__ void __launch_bounds__(kFusedThreads)
+    prune_unigram_fused_kernel(const float* __restrict__ rewards, const float* __restrict__ adv,
+                               float class_eps, const int32_t* __restrict__ ids,
+                               const int64_t* __restrict__ off, int G, int V, int words, float tau,
+                               int keep_cap, uint8_t* __restrict__ keep,
+                               int32_t* __restrict__ kept_per_prompt, int32_t* status) {
+  extern __shared__ __align__(16) unsigned long long bms[];  // [G][words]
+  __shared__ int32_t s_cls[kMaxG], s_rank[kMaxG], s_nuniq[kMaxG];
+  __shared__ uint8_t s_close[kMaxG * kMaxG];
+  __shared__ int64_t s_off[kMaxG + 1];
+  const int p = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int kWarps = kFusedThreads / 32;
+  if (warp == 0) classify_warp(rewards, adv, class_eps, p, G, lane, s_cls, s_rank);
+  if (tid <= G) s_off[tid] = off[(int64_t)p * G + tid];
+  for (int k = tid; k < G * words; k += kFusedThreads) bms[k] = 0ull;
+  __syncthreads();
+  // all tokens of the prompt in one flat loop (independent loads); a token's rollout is the
+  // last r with s_off[r] <= its index
+  bool bad = false;
+  const int64_t t0 = s_off[0], t1 = s_off[G];
+  for (int64_t t = t0 + tid; t < t1; t += kFusedThreads) {
+    const int32_t id = ids[t];
+    int r = 0;
+    while (r + 1 < G && s_off[r + 1] <= t) ++r;
+    if (id < 0 || id >= V) {
+      bad = true;
+      continue;
+    }
+    atomicOr(&bms[(int64_t)r * words + (id >> 6)], 1ull << (id & 63));
+  }
+  if (bad && status) atomicOr(status, GRPO_DEVFLAG_BAD_TOKEN);
+  __syncthreads();
+  for (int r = warp; r < G; r += kWarps) {  // |N_r|
+    int c = 0;
+    for (int k = lane; k < words; k += 32) c += __popcll(bms[(int64_t)r * words + k]);
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+    if (lane == 0) s_nuniq[r] = c;
+  }
+  __syncthreads();
+  const int pairs = G * (G - 1) / 2;
+  for (int q = warp; q < pairs; q += kWarps) {  // theta_ij < tau for same-class pairs
+    int i, j;
+    pair_of(q, G, i, j);
+    uint8_t c = 0;
+    if (s_cls[i] == s_cls[j]) {
+      const unsigned long long* a = bms + (int64_t)i * words;
+      const unsigned long long* b = bms + (int64_t)j * words;
+      int I = 0;
+      for (int k = lane; k < words; k += 32) I += __popcll(a[k] & b[k]);
+      for (int o = 16; o > 0; o >>= 1) I += __shfl_xor_sync(0xffffffffu, I, o);
+      c = too_close(I, s_nuniq[i], s_nuniq[j], tau) ? 1 : 0;
+    }
+    if (lane == 0) s_close[i * G + j] = s_close[j * G + i] = c;
+  }
+  __syncthreads();
+  if (warp == 0)
+    select_warp(G, keep_cap, s_rank, s_cls, s_close, lane, keep + (int64_t)p * G,
+                kept_per_prompt + p);
 }
 
 __global__ void dp_fill_kernel(const float* __restrict__ rewards, int P, int G, int d,
@@ -488,8 +576,33 @@ extern "C" grpo_status grpo_prune(const float* rewards, const float* adv, float 
   const int nroll = P * G;
   const int pairs = G * (G - 1) / 2;
   const unsigned warp_blocks = (unsigned)(((int64_t)P * 32 + 127) / 128);
+  int launches = 0;
+  const size_t fused_smem = (size_t)G * w.words * 8;
+  if (ngram_n == 1 && fused_smem <= kFusedMaxBitmapBytes) {
+    static std::atomic<uint64_t> fused_attr{0};  // bit d: the attribute is set on device d
+    int dev = 0;
+    cudaGetDevice(&dev);
+    const uint64_t bit = dev < 64 ? (1ull << dev) : 0ull;
+    if (!bit || !(fused_attr.load() & bit)) {  // once per device, before any stream capture
+      if (cudaFuncSetAttribute(prune_unigram_fused_kernel,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)kFusedMaxBitmapBytes) != cudaSuccess)
+        return check_launch("grpo_prune: cudaFuncSetAttribute");
+      fused_attr.fetch_or(bit);
+    }
+    prune_unigram_fused_kernel<<<P, kFusedThreads, fused_smem, s>>>(
+        rewards, adv, class_eps, ids, off, G, V, w.words, tau, keep_cap, keep, kept_per_prompt,
+        status);
+    launches = 1;
+    if (dp_divisor > 1) {
+      dp_fill_kernel<<<1, 32, 0, s>>>(rewards, P, G, dp_divisor, keep, kept_per_prompt);
+      ++launches;
+    }
+    count_launches(launches);
+    return check_launch("grpo_prune");
+  }
   class_kernel<<<warp_blocks, 128, 0, s>>>(rewards, adv, class_eps, P, G, w);
-  int launches = 1;
+  launches = 1;
   if (ngram_n == 1) {
     unigram_set_kernel<<<nroll, 256, (size_t)w.words * 8, s>>>(ids, off, V, w, status);
     ++launches;
