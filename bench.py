@@ -313,6 +313,63 @@ def cpu_baseline_gspo(w, b, step, dev_inputs, target_s):
                       " sequences (%d rows, %.2f s)" % (t_sel, T_kept, k, rows, t)}
 
 
+def run_reference_gspo(args, w, b, comp):
+    """The reference arm for GSPO's loss: selection on the whole batch, then the sequence-level
+    loss over the first whole kept sequences that fit the per-step time budget."""
+    from paper_2609_36932_gb300 import workloads
+    import oracle
+    K, T_kept = comp["K"], comp["T_kept"]
+    kept_idx, kept_off = comp["kept_idx"][:K], comp["kept_off"][:K + 1]
+
+    def sample(k):
+        rows = comp["src_token"][:kept_off[k]]
+        lg = workloads.logits_rows(w, args.seed, rows, "cpu")
+        o, r = workloads.old_ref_logp(lg, b["ids"][rows], b["noise_old"][rows], b["noise_ref"][rows])
+        return rows, host_logits_bits(lg), o.numpy(), r.numpy()
+
+    def run(k, data):
+        rows, bits, o, r = data
+        t0 = time.perf_counter()
+        adv, _ = oracle.advantage(b["rewards"], w.G)
+        kp, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+        oracle.compact(kp, b["off"])
+        t1 = time.perf_counter()
+        oracle.gspo_loss(bits, w.V, b["ids"][rows], o, r, adv, kept_idx[:k], kept_off[:k + 1],
+                         n_seq=K, eps_low=w.eps, eps_high=w.eps, beta=w.beta,
+                         dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
+        return t1 - t0, time.perf_counter() - t1
+
+    k = 1
+    while k < K and kept_off[k] == 0:
+        k += 1
+    t_sel, t_loss = run(k, sample(k))
+    budget = 120.0 / max(args.steps + args.warmup, 1)
+    per_row = t_loss / max(int(kept_off[k]), 1)
+    while k < K and (int(kept_off[k + 1]) * per_row + t_sel) <= budget:
+        k += 1
+    data = sample(k)
+    rows = int(kept_off[k])
+    cores = int(oracle.set_threads(0))
+    times = []
+    for i in range(args.warmup + args.steps):
+        t_sel, t_loss = run(k, data)
+        if i >= args.warmup:
+            times.append(t_loss / rows + t_sel / T_kept)
+    value = 1.0 / statistics.mean(times)
+    cfg = dict(workload_desc(w, b["T"], T_kept, K), loss="gspo")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": cfg,
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": "per step: fp64 oracle advantage+prune+compact on the whole batch"
+                                   " (amortised over %d kept tokens) + GSPO's sequence-level loss on"
+                                   " the first %d kept sequences (%d rows)" % (T_kept, k, rows)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
 def run_reference(args, w):
     """The reference arm: the fp64 oracle as it stands, on this machine's host cores."""
     import torch
@@ -326,6 +383,8 @@ def run_reference(args, w):
     comp = oracle.compact(keep, b["off"])
     T_kept = comp["T_kept"]
     src_all, rr_all = comp["src_token"], comp["token_rollout"]
+    if args.loss == "gspo":
+        return run_reference_gspo(args, w, b, comp)
     # a bounded sample of kept rows, generated on the host
     n = min(len(src_all), 4)
     lg = workloads.logits_rows(w, args.seed, src_all[:n], "cpu")
