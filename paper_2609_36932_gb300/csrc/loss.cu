@@ -282,11 +282,32 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
     }
   }
 
+  // With dlogits wider than the logits, the row's source index and sampled token are loaded one
+  // row ahead.  Measured on GB300: +5.8% there (f32 dlogits at V = 152064); with bf16 dlogits
+  // the same change was 1.5-2% slower, so only the wider instance does it.
+  constexpr bool kAhead = sizeof(OutT) > sizeof(InT);
+  int64_t src_nx = 0;
+  int32_t y_nx = 0;
+  if (kAhead && row < n_rows) {
+    src_nx = a.row_index ? a.row_index[row] : row;
+    y_nx = a.y[src_nx];
+  }
   for (; row < n_rows; row += ncl, phase ^= 1u, ++iter) {
     const uint32_t slot = iter & 1u;
     if (tid == 0) mbar_expect_tx(xbar_s + 8 * slot, 16u * C);  // one entry from every CTA
-    const int64_t src = a.row_index ? a.row_index[row] : row;
-    const int32_t yv = a.y[src];
+    int64_t src;
+    int32_t yv;
+    if constexpr (kAhead) {
+      src = src_nx;
+      yv = y_nx;
+      if (row + ncl < n_rows) {  // issued now, used by the cluster's next row
+        src_nx = a.row_index ? a.row_index[row + ncl] : row + ncl;
+        y_nx = a.y[src_nx];
+      }
+    } else {
+      src = a.row_index ? a.row_index[row] : row;
+      yv = a.y[src];
+    }
     const bool yvalid = yv >= 0 && yv < a.V;
     const int yl = yvalid ? yv - s0 : -1;  // y's position in my slice, if there
     const char* grow = a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
