@@ -4,13 +4,16 @@
  * The library computes, on one GPU, the data-parallel core of one FastRL training step
  * ("Learn from the Gap", Sec. 3 and Algorithm 1):
  *
- *   grpo_advantage          group-relative advantages                          (Eq. 5)
- *   grpo_prune              maximising-differential advantage pruning (MDAP)   (Eqs. 6-9, Algorithm 1)
- *   grpo_compact            compaction of the kept rollouts' tokens            (Sec. 3.2, after Eq. 9)
- *   grpo_upload_kept        host-to-device copy of the kept rollouts' rows      (Sec. 3.2)
- *   grpo_gspo_loss_fwd_bwd  GSPO's sequence-level loss, for FastRL on GSPO     (Sec. 1, Sec. 4)
- *   grpo_loss_fwd_bwd       fused GRPO token loss, forward and dlogits         (Eqs. 1-3)
- *   adaptive_rollout_count  host-side adaptive rollout sampling (ARS)          (Eqs. 10-14, Algorithm 1)
+ *   grpo_advantage          group-relative advantages                  (Eq. 5)
+ *   grpo_prune              maximising-differential advantage pruning  (Eqs. 6-9, Algorithm 1)
+ *   grpo_compact            compaction of the kept rollouts' tokens    (Sec. 3.2, after Eq. 9)
+ *   grpo_loss_fwd_bwd       fused GRPO token loss and dlogits          (Eqs. 1-3)
+ *     (_dev: row count read on the device, for CUDA graphs; _noalloc: no workspace)
+ *   grpo_logp_fwd           log-probabilities alone                    (Sec. 3.2)
+ *   grpo_gspo_loss_fwd_bwd  GSPO's sequence-level loss                 (Sec. 1, Sec. 4)
+ *     (_dev: counts read on the device, for CUDA graphs)
+ *   grpo_upload_kept        host-to-device copy of the kept rows only  (Sec. 3.2)
+ *   adaptive_rollout_count  adaptive rollout sampling, on the host     (Eqs. 10-14, Algorithm 1)
  *
  * Conventions shared by every call:
  *   - Every call returns a grpo_status; GRPO_OK is 0.  On failure, grpo_last_error() returns a
@@ -92,10 +95,10 @@ grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G, int32_t s
  * Then, if |S(q)| > keep_cap, keep_cap rollouts are kept by round-robin over the classes
  * (classes ordered by the visiting position of their first member; each round takes each
  * class's next kept rollout in visiting order, which for equal rewards is the lowest index).
- * keep_cap >= G disables the cap (the paper's rule).  Finally, while the total kept count is not a multiple of dp_divisor, prompts are
- * visited cyclically from prompt 0 and each visit adds that prompt's unkept rollout with the
- * largest |r - mean| (lowest index on ties); prompts with none left are skipped (Algorithm 1,
- * DP alignment).  dp_divisor = 1 does nothing.
+ * keep_cap >= G disables the cap (the paper's rule).  Finally, while the total kept count is
+ * not a multiple of dp_divisor, prompts are visited cyclically from prompt 0 and each visit adds
+ * that prompt's unkept rollout with the largest |r - mean| (lowest index on ties); prompts with
+ * none left are skipped (Algorithm 1, DP alignment).  dp_divisor = 1 does nothing.
  * rewards          device f32 [P*G].
  * adv, class_eps   class_eps = 0: classes by exact reward equality (adv may be NULL).
  *                  class_eps > 0: the continuous-reward grouping of the paper's grounding
