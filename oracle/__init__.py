@@ -47,6 +47,10 @@ def lib():
                                        _c_p, _c_p, _i64, _i64, _f32, _f32, _f32, _c_p, _i32,
                                        _c_p, _c_p, _c_p, _c_p, _c_p]
         L.oracle_gspo_loss.restype = _i32
+        L.oracle_lmhead_loss.argtypes = [_c_p, _c_p, _i64, _i32, _i32, _c_p, _c_p, _c_p, _c_p,
+                                         _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p,
+                                         _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
+        L.oracle_lmhead_loss.restype = _i32
         L.oracle_logp.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p]
         L.oracle_logp.restype = _i32
         L.oracle_round_bf16.argtypes = [_f64]
@@ -141,7 +145,8 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
          beta=0.04, agg_mode=0, denom_tokens=None, seq_off=None, n_seq=0, row_index=None,
          n_rows=None, row_stride=None, logits_dtype=None, dlogits_dtype=0, want_f64=False,
          want_dlogits=True):
-    """Eqs. 1-3.  `logits` is a float32 array or a uint16 array of bf16 bit patterns.
+    """Eqs. 1-3.  `logits` is a float32 array or a uint16 array of bf16 bit patterns (or, with
+    logits_dtype=2, float64).
 
     Returns dict(loss, logp [n_rows] f64, rho, row_loss, dlogits (f32 array or uint16 bf16
     bits, [n_rows, V]) and, with want_f64, dlogits_f64).
@@ -151,6 +156,8 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
         logits_dtype = 1 if lg.dtype == np.uint16 else 0
     if logits_dtype == 0:
         lg = lg.astype(np.float32, copy=False)
+    elif logits_dtype == 2:
+        lg = lg.astype(np.float64, copy=False)
     stride = V if row_stride is None else int(row_stride)
     ri = None if row_index is None else _arr(row_index, np.int64)
     if n_rows is None:
@@ -178,6 +185,53 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
         raise ValueError("oracle_loss: bad arguments")
     return dict(loss=float(total[0]), logp=logp[:n_rows], rho=rho[:n_rows], row_loss=rl[:n_rows],
                 dlogits=dl, dlogits_f64=d64)
+
+
+def lmhead_loss(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2,
+                eps_high=0.2, beta=0.04, agg_mode=0, denom_tokens=None, seq_off=None, n_seq=0,
+                want_logits=False, want_dlogits=False, want_dhidden=True, want_dweight=True,
+                want_bounds=False):
+    """The output layer z = hidden @ weight.T fused with Eqs. 1-3, and the chain rule.
+
+    hidden [n_rows, D] and weight [V, D] are taken as float64 (bf16 values widen exactly).
+    Returns dict(loss, logp, row_loss, and as asked: logits, dlogits (f64), dhidden [n_rows, D],
+    dweight [V, D], dhidden_abs, dweight_abs).
+    """
+    h = np.ascontiguousarray(hidden, dtype=np.float64)
+    w = np.ascontiguousarray(weight, dtype=np.float64)
+    n_rows, D = h.shape
+    V = w.shape[0]
+    if w.shape[1] != D:
+        raise ValueError("hidden and weight disagree on D")
+    y_ = _arr(y, np.int32)
+    old = _arr(old_logp, np.float32)
+    ref = _arr(ref_logp, np.float32)
+    a = _arr(adv, np.float32)
+    rr = _arr(row_rollout, np.int32)
+    so = None if seq_off is None else _arr(seq_off, np.int64)
+    if denom_tokens is None:
+        denom_tokens = n_rows
+
+    def buf(want, shape):
+        return np.empty(shape, np.float64) if want else None
+
+    lg = buf(want_logits, (n_rows, V))
+    dl = buf(want_dlogits, (n_rows, V))
+    dh = buf(want_dhidden, (n_rows, D))
+    dw = buf(want_dweight, (V, D))
+    dha = buf(want_bounds and want_dhidden, (n_rows, D))
+    dwa = buf(want_bounds and want_dweight, (V, D))
+    logp = np.empty(max(n_rows, 1), np.float64)
+    rl = np.empty(max(n_rows, 1), np.float64)
+    total = np.zeros(1, np.float64)
+    rc = lib().oracle_lmhead_loss(_p(h), _p(w), n_rows, V, D, _p(y_), _p(old), _p(ref), _p(a),
+                                  _p(rr), float(eps_low), float(eps_high), float(beta), agg_mode,
+                                  int(denom_tokens), _p(so), int(n_seq), _p(lg), _p(dl), _p(logp),
+                                  _p(rl), _p(total), _p(dh), _p(dw), _p(dha), _p(dwa))
+    if rc != 0:
+        raise ValueError("oracle_lmhead_loss: bad arguments")
+    return dict(loss=float(total[0]), logp=logp[:n_rows], row_loss=rl[:n_rows], logits=lg,
+                dlogits=dl, dhidden=dh, dweight=dw, dhidden_abs=dha, dweight_abs=dwa)
 
 
 def gspo_loss(logits, V: int, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,

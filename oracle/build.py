@@ -11,7 +11,7 @@ import subprocess
 import sys
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-SOURCES = ["advantage.cpp", "mdap.cpp", "compact.cpp", "loss.cpp", "ars.cpp"]
+SOURCES = ["advantage.cpp", "mdap.cpp", "compact.cpp", "loss.cpp", "lmhead.cpp", "ars.cpp"]
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "liboracle.so")
 

@@ -34,6 +34,7 @@ namespace {
 
 double load_logit(const void* logits, int dtype, int64_t idx) {
   if (dtype == 0) return (double)static_cast<const float*>(logits)[idx];
+  if (dtype == 2) return static_cast<const double*>(logits)[idx];
   const uint32_t bits = (uint32_t) static_cast<const uint16_t*>(logits)[idx] << 16;
   float f;
   std::memcpy(&f, &bits, sizeof f);

@@ -45,7 +45,8 @@ int oracle_compact(const uint8_t* keep, const int64_t* off, int n_rollouts, int3
                    int64_t* kept_off, int64_t* src_token, int32_t* token_rollout, int64_t* counts);
 
 /* Eqs. 1-3: GRPO token loss and dlogits; see loss.cpp.
- * logits_dtype 0 = f32, 1 = bf16 bit patterns (uint16).  dlogits_dtype 0 = f32, 1 = bf16 bits.
+ * logits_dtype 0 = f32, 1 = bf16 bit patterns (uint16), 2 = f64.  dlogits_dtype 0 = f32,
+ * 1 = bf16 bits.
  * dlogits_f64 (nullable) receives the unrounded fp64 gradient.  rho_out (nullable) the ratios. */
 int oracle_loss(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
                 int64_t n_rows, int V, const int32_t* y, const float* old_logp,
@@ -66,6 +67,22 @@ int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t row_stride,
                      float eps_high, float beta, void* dlogits, int dlogits_dtype,
                      double* dlogits_f64, double* logp_out, double* seq_ratio_out,
                      double* seq_loss_out, double* loss_out);
+
+/* The policy's output layer fused with the GRPO token loss; see lmhead.cpp.
+ * hidden f64 [n_rows, D], weight f64 [V, D] (row-major; bf16 values widen exactly).
+ * z = hidden * weight^T, then oracle_loss on z (Eqs. 1-3), then the chain rule:
+ * dhidden = dlogits * weight [n_rows, D], dweight = dlogits^T * hidden [V, D].
+ * Every output is nullable.  dhidden_abs / dweight_abs receive the same products over absolute
+ * values (|dlogits| * |weight|, |dlogits|^T * |hidden|), the scale of the rounding error of any
+ * evaluation of dhidden and dweight. */
+int oracle_lmhead_loss(const double* hidden, const double* weight, int64_t n_rows, int V, int D,
+                       const int32_t* y, const float* old_logp, const float* ref_logp,
+                       const float* adv, const int32_t* row_rollout, float eps_low,
+                       float eps_high, float beta, int agg_mode, int64_t denom_tokens,
+                       const int64_t* seq_off, int64_t n_seq, double* logits_out,
+                       double* dlogits_out, double* logp_out, double* row_loss_out,
+                       double* loss_out, double* dhidden, double* dweight, double* dhidden_abs,
+                       double* dweight_abs);
 
 /* logp of the sampled token alone (old/reference policy evaluation); NaN for ids outside [0,V). */
 int oracle_logp(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
