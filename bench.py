@@ -54,9 +54,13 @@ def parse():
                     help="override the workload's prompt count (a smaller case for profiling)")
     ap.add_argument("--group", type=int, default=0,
                     help="override the rollouts per prompt G (a smaller case for profiling)")
-    ap.add_argument("--loss", choices=["grpo", "gspo"], default="grpo",
+    ap.add_argument("--loss", choices=["grpo", "gspo", "lmhead"], default="grpo",
                     help="grpo: Eq. 1's token-level ratio (fused, one pass); gspo: the sequence-level "
-                         "ratio of FastRL's GSPO variant (three passes, host-synced)")
+                         "ratio of FastRL's GSPO variant (three passes, host-synced); lmhead: the "
+                         "output layer fused with the token loss (hidden states in, logits on the "
+                         "tensor cores, dhidden and dweight out)")
+    ap.add_argument("--hidden", type=int, default=0,
+                    help="hidden size of the output layer with --loss lmhead (default 3584)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
@@ -427,6 +431,309 @@ def run_reference(args, w):
     print(json.dumps(line), flush=True)
 
 
+LMHEAD_METRIC = ("kept-token GRPO step with the output layer fused: tokens/s and tensor-core "
+                 "TFLOP/s (% of GB300 bf16 peak)")
+
+
+def measured_tensor_peak(sustained):
+    key = "bf16_tflops_sustained" if sustained else "bf16_tflops"
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)[key]), "measured (MEASURED_PEAKS.json %s, cuBLAS bf16)" % key
+    except Exception:
+        return (1700.0, "fallback 1.7 PFLOP/s sustained") if sustained else (
+            1900.0, "fallback 1.9 PFLOP/s burst")
+
+
+def lmhead_source_hash():
+    h = hashlib.sha256()
+    for f in ("lmhead.cu", "rowops.cuh", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def lmhead_traffic_per_row():
+    """DRAM bytes per row of the pass-1 tile kernel from the committed ncu summary, if it was
+    taken on the current kernel source; else None."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "lmhead_kernel_traffic.json")) as f:
+            e = json.load(f)["lmhead_fwd"]
+    except Exception:
+        return None
+    if e.get("source_hash") != lmhead_source_hash():
+        return None
+    return float(e["dram_bytes_per_row"])
+
+
+def lmhead_inputs(w, D, seed, device):
+    import torch
+    from paper_2609_36932_gb300 import workloads
+    b = workloads.make_batch(w, seed)
+    hid = workloads.lmhead_hidden(b["T"], D, seed, device)
+    wt = workloads.lmhead_weight(w.V, D, seed, device)
+    old, ref = workloads.lmhead_old_ref(hid, wt, b["ids"], b["noise_old"], b["noise_ref"])
+    d = dict(rewards=torch.from_numpy(b["rewards"]).to(device),
+             ids=torch.from_numpy(b["ids"]).to(device), off=torch.from_numpy(b["off"]).to(device),
+             hidden=hid, weight=wt, old=old, ref=ref)
+    return b, d
+
+
+def lmhead_desc(w, D, T, T_kept, K):
+    cfg = workload_desc(w, T, T_kept, K)
+    cfg["workload"] = ("%s with the output layer: %d prompts x G=%d rollouts, lengths %s, hidden "
+                       "size D=%d, V=%d, bf16 hidden states N(0,1) and weight N(0,4/D), rewards %s,"
+                       " %.0f%% zero-advantage groups, keep ratio %.2f (cap %d/prompt); bf16 "
+                       "dhidden, f32 dweight" % (w.name, w.P, w.G, w.length, D, w.V, w.reward_kind,
+                                                  100 * w.zero_adv_frac, w.keep_ratio, w.keep_cap))
+    cfg["D"] = D
+    cfg["io"] = "bf16 hidden [T_kept, D] and weight [V, D] -> bf16 dhidden, f32 dweight"
+    cfg["l2"] = ("inputs larger than L2 (weight %.2f GB, dweight %.2f GB vs 129 MB L2); no flush"
+                 % (w.V * D * 2 / 1e9, w.V * D * 4 / 1e9))
+    cfg["loss"] = "lmhead"
+    return cfg
+
+
+def oracle_lmhead_sample(w, b, d, src, rr, T_kept, n, threads=0):
+    """Time the oracle: selection on the whole batch, then the output layer + loss (logits,
+    dhidden and dweight) on the first n kept rows."""
+    import oracle
+    oracle.set_threads(threads)
+    import torch
+    rows = torch.from_numpy(np.ascontiguousarray(src[:n])).to(d["hidden"].device)
+    h = d["hidden"][rows].float().cpu().numpy()
+    wt = d["weight"].double().cpu().numpy()
+    old = d["old"].cpu().numpy()[src[:n]]
+    ref = d["ref"].cpu().numpy()[src[:n]]
+    t0 = time.perf_counter()
+    adv, _ = oracle.advantage(b["rewards"], w.G)
+    keep, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+    oracle.compact(keep, b["off"])
+    t_sel = time.perf_counter() - t0
+    t1 = time.perf_counter()
+    oracle.lmhead_loss(h, wt, b["ids"][src[:n]], old, ref, adv, rr[:n], eps_low=w.eps,
+                       eps_high=w.eps, beta=w.beta, denom_tokens=T_kept)
+    return t_sel, time.perf_counter() - t1, int(oracle.set_threads(0))
+
+
+def run_lmhead(args, w):
+    """--loss lmhead: the step with the output layer fused (GrpoStep in output-layer mode)."""
+    import torch
+    import torch.distributed as dist
+    import paper_2609_36932_gb300 as g
+    from paper_2609_36932_gb300 import workloads
+    from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    g.lib()
+    D = args.hidden or workloads.LMHEAD_D
+    b, d = lmhead_inputs(w, D, rank_seed(args.seed, rank), dev)
+    p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
+                   eps_low=w.eps, eps_high=w.eps, beta=w.beta)
+    step = GrpoStep(p, d["rewards"], d["ids"], d["off"], None, d["old"], d["ref"],
+                    hidden=d["hidden"], weight=d["weight"])
+    for _ in range(max(args.warmup, 3)):
+        step.run()
+    torch.cuda.synchronize()
+    K = args.steps
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    l0 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    l1 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    if local == 0:
+        sampler.start()
+        time.sleep(0.3)
+    launches0 = g.grpo_kernel_launches()
+    kept = 0
+    ev0.record(stream)
+    for i in range(K):
+        s0[i].record(stream)
+        step.select()
+        l0[i].record(stream)
+        step.loss_step()
+        l1[i].record(stream)
+        kept += step.T_kept
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    launches = g.grpo_kernel_launches() - launches0
+    clocks = sampler.stop() if local == 0 else None
+    g.check_status(step.status)
+    elapsed_ms = ev0.elapsed_time(ev1)
+    loss_ms = statistics.mean(a.elapsed_time(z) for a, z in zip(l0, l1))
+    select_ms = statistics.mean(a.elapsed_time(z) for a, z in zip(s0, l0))
+    elapsed_ms, kept_all = combine_ranks(elapsed_ms, kept, world, dev)
+    value = kept_all / (elapsed_ms / 1e3)
+    T_kept = step.T_kept
+    flops_pass = 2.0 * T_kept * w.V * D
+
+    # roofline of the pass-1 tile kernel: the same kept rows through grpo_lmhead_logp_fwd (that
+    # kernel plus a row kernel of T_kept threads), event-timed on this stream
+    lp = torch.empty(max(T_kept, 1), dtype=torch.float32, device=dev)
+    rows_src = step.src_token[:T_kept]
+    fw = g.grpo_lmhead_logp_fwd(d["hidden"], d["weight"], d["ids"], row_index=rows_src,
+                                n_rows=T_kept, logp_out=lp)
+    for _ in range(2):
+        g.grpo_lmhead_logp_fwd(d["hidden"], d["weight"], d["ids"], row_index=rows_src,
+                               n_rows=T_kept, logp_out=lp, ws=fw["ws"])
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    nrep = 5
+    torch.cuda.synchronize()
+    f0.record(stream)
+    for _ in range(nrep):
+        g.grpo_lmhead_logp_fwd(d["hidden"], d["weight"], d["ids"], row_index=rows_src,
+                               n_rows=T_kept, logp_out=lp, ws=fw["ws"])
+    f1.record(stream)
+    torch.cuda.synchronize()
+    f_ms = f0.elapsed_time(f1) / nrep
+    peak, peak_src = measured_tensor_peak(sustained=False)
+    peak_s, peak_s_src = measured_tensor_peak(sustained=True)
+    achieved = flops_pass / (f_ms / 1e3) / 1e12
+    tr = lmhead_traffic_per_row()
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None if tr is None else tr * T_kept,
+                "kernel": "lmhead_tile_kernel<pass 1> (+ gather and row kernels), timed through "
+                          "grpo_lmhead_logp_fwd on the step's kept rows",
+                "algorithmic_flops_per_launch": flops_pass, "launch_ms": f_ms,
+                "peak_source": peak_src}
+    step_tc = {"flops_per_step": 4 * flops_pass, "loss_ms": loss_ms,
+               "achieved": 4 * flops_pass / (loss_ms / 1e3) / 1e12, "unit": "TFLOP/s",
+               "peak": peak_s, "frac": 4 * flops_pass / (loss_ms / 1e3) / 1e12 / peak_s,
+               "peak_source": peak_s_src,
+               "note": "the whole fused call: pass 1, pass 2 (2 T V D each, tcgen05) and the "
+                       "dhidden and dweight GEMMs (2 T V D each, cuBLASLt)"}
+
+    # end to end: selection inputs, log-probs and hidden states from pinned host memory (hidden
+    # rows of the kept rollouts only), loss read back, inside the timed region
+    e2e = None
+    names = ["rewards", "ids", "off", "old", "ref", "hidden"]
+    if args.e2e_steps > 0:
+        host = {}
+        for k in names:
+            host[k] = torch.empty(d[k].shape, dtype=d[k].dtype, pin_memory=True)
+            host[k].copy_(d[k])
+        loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
+        step.run_from_host(host, loss_host)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        kept_e, h2d_e, d2h_e = 0, 0, 0
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            hb, db = step.run_from_host(host, loss_host)
+            h2d_e += hb
+            d2h_e += db
+            kept_e += step.T_kept
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms, kept_e = combine_ranks(e0.elapsed_time(e1), kept_e, world, dev)
+        e2e = {"value": kept_e / (e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d_e // args.e2e_steps),
+               "d2h_bytes_per_step": int(d2h_e // args.e2e_steps), "steps": args.e2e_steps,
+               "transfer": "selection inputs and per-token log-probs whole; hidden states of the "
+                           "kept rollouts only (grpo_upload_kept), after the selection; the "
+                           "output-layer weight is a resident model parameter"}
+        del host
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        src, rr = step.kept_rows()
+        n0 = min(16, len(src))  # a full row per worker thread for the calibration
+        _, tl0, _ = oracle_lmhead_sample(w, b, d, src, rr, T_kept, n0)
+        n = int(min(len(src), max(n0, args.cpu_seconds / max(tl0 / n0, 1e-6))))
+        t_sel, t_loss, cores = oracle_lmhead_sample(w, b, d, src, rr, T_kept, n)
+        cpu = {"value": 1.0 / (t_loss / n + t_sel / max(T_kept, 1)), "unit": UNIT, "cores": cores,
+               "kind": "oracle",
+               "sample": "fp64 oracle: advantage+prune+compact on the whole batch (%.2f s, "
+                         "amortised over its %d kept tokens) + output layer and loss (logits, "
+                         "dhidden, dweight) on the first %d kept rows (%.2f s)"
+                         % (t_sel, T_kept, n, t_loss)}
+
+    if rank == 0:
+        line = {
+            "metric": LMHEAD_METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; the qwen batch with random-init output layer)",
+            "config": lmhead_desc(w, D, b["T"], T_kept, step.K),
+            "gpu_launches": int(launches), "cuda_graph": False,
+            "roofline": roofline, "step_tensor": step_tc, "e2e": e2e, "cpu_baseline": cpu,
+            "clocks": clocks,
+            "path_overhead": {"select_ms": select_ms, "other_ms": elapsed_ms / K - select_ms - loss_ms},
+            "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def run_reference_lmhead(args, w):
+    """The reference arm for --loss lmhead: the fp64 oracle on this machine's host cores; each
+    step runs the selection on the whole batch and the output layer + loss on a bounded sample
+    of kept rows (inputs generated on the host)."""
+    import torch
+    from paper_2609_36932_gb300 import workloads
+    import oracle
+    D = args.hidden or workloads.LMHEAD_D
+    b = workloads.make_batch(w, args.seed)
+    keep, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+    comp = oracle.compact(keep, b["off"])
+    T_kept = comp["T_kept"]
+    src, rr = comp["src_token"], comp["token_rollout"]
+    wt = workloads.lmhead_weight(w.V, D, args.seed, "cpu")
+    w64 = wt.double().numpy()
+
+    def sample(n):
+        h = workloads.lmhead_hidden(b["T"], D, args.seed, "cpu", rows=src[:n])
+        o, r = workloads.lmhead_old_ref(h, wt, b["ids"][src[:n]], b["noise_old"][src[:n]],
+                                        b["noise_ref"][src[:n]])
+        return h.float().numpy(), o.numpy(), r.numpy()
+
+    def run(n, data):
+        h, o, r = data
+        t0 = time.perf_counter()
+        adv, _ = oracle.advantage(b["rewards"], w.G)
+        kp, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+        oracle.compact(kp, b["off"])
+        t1 = time.perf_counter()
+        oracle.lmhead_loss(h, w64, b["ids"][src[:n]], o, r, adv, rr[:n], eps_low=w.eps,
+                           eps_high=w.eps, beta=w.beta, denom_tokens=T_kept)
+        return t1 - t0, time.perf_counter() - t1
+
+    t_sel, t_loss = run(1, sample(1))
+    budget = 120.0 / max(args.steps + args.warmup, 1)
+    n = int(max(1, min(len(src), 64, (budget - t_sel) / max(t_loss, 1e-6)))) if budget > t_sel else 1
+    data = sample(n)
+    cores = int(oracle.set_threads(0))
+    times = []
+    for i in range(args.warmup + args.steps):
+        t_sel, t_loss = run(n, data)
+        if i >= args.warmup:
+            times.append(t_loss / n + t_sel / T_kept)
+    value = 1.0 / statistics.mean(times)
+    print(json.dumps({
+        "impl": "reference", "metric": LMHEAD_METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": lmhead_desc(w, D, b["T"], T_kept, comp["K"]),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": "per step: fp64 oracle advantage+prune+compact on the whole batch"
+                                   " (amortised over %d kept tokens) + output layer and loss on the"
+                                   " first %d kept rows" % (T_kept, n)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
 def main():
     args = parse()
     import dataclasses
@@ -437,7 +744,14 @@ def main():
     if args.group > 0:
         w = dataclasses.replace(w, G=args.group)
     if args.impl == "reference":
+        if args.loss == "lmhead":
+            if dist_env()[0] == 0:
+                run_reference_lmhead(args, w)
+            return
         run_reference(args, w)
+        return
+    if args.loss == "lmhead":
+        run_lmhead(args, w)
         return
     import torch
     import torch.distributed as dist

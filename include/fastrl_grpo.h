@@ -12,6 +12,9 @@
  *   grpo_logp_fwd           log-probabilities alone                    (Sec. 3.2)
  *   grpo_gspo_loss_fwd_bwd  GSPO's sequence-level loss                 (Sec. 1, Sec. 4)
  *     (_dev: counts read on the device, for CUDA graphs)
+ *   grpo_lmhead_loss_fwd_bwd  the output layer fused with the loss:     (Sec. 3.2, Eqs. 1-3)
+ *                           logits on the tensor cores, never stored whole; dhidden, dweight
+ *     (grpo_lmhead_logp_fwd: log-probabilities alone from hidden states)
  *   grpo_upload_kept        host-to-device copy of the kept rows only  (Sec. 3.2)
  *   adaptive_rollout_count  adaptive rollout sampling, on the host     (Eqs. 10-14, Algorithm 1)
  *
@@ -19,7 +22,8 @@
  *   - Every call returns a grpo_status; GRPO_OK is 0.  On failure, grpo_last_error() returns a
  *     message for the calling thread.  No C++ exception and no abort crosses this boundary.
  *   - Buffers marked "device" are device pointers owned by the caller (for instance memory held
- *     by PyTorch tensors).  The library never allocates or frees device memory.  Scratch memory
+ *     by PyTorch tensors).  The library never allocates or frees device memory (the cuBLASLt
+ *     GEMMs of grpo_lmhead_loss_fwd_bwd also run in the caller's workspace).  Scratch memory
  *     comes from a caller workspace: a call with ws == NULL and ws_bytes != NULL only writes the
  *     size it needs into *ws_bytes and enqueues nothing.  The real call passes ws (256-byte
  *     aligned) with *ws_bytes >= that size, or ws == NULL and ws_bytes == NULL when the size
@@ -285,6 +289,70 @@ grpo_status grpo_gspo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype,
                                        void* dlogits, int32_t dlogits_dtype, float* logp_out,
                                        float* seq_ratio_out, double* loss_out, int32_t* status,
                                        void* ws, size_t* ws_bytes, grpo_stream_t stream);
+
+/*
+ * grpo_lmhead_loss_fwd_bwd — the policy's output layer fused with the GRPO token loss.  Sec. 3.2
+ * runs the kept trajectories through the policy, whose last layer maps each token's hidden state
+ * to logits over the vocabulary; Eqs. 1-3 give the loss.  Here the logits
+ *   z[t, v] = sum_d hidden[t, d] * weight[v, d]
+ * are produced on the tensor cores 128 x 256 at a time and consumed on chip, never stored whole:
+ *   loss, logp_out, row_loss_out: as grpo_loss_fwd_bwd on z (rows in order, row_index = NULL);
+ *   dhidden[t, :] = sum_v dlogits[t, v] * weight[v, :]         (chain rule through z = h W^T)
+ *   dweight[v, :] = sum_t dlogits[t, v] * hidden[t, :]          (+ the old dweight with
+ *                                                                accumulate_dweight != 0)
+ * with dlogits = w_t*g_t*([v == y] - softmax(z)_v) rounded to bf16 before the two products.
+ * hidden: device bf16, row stride hidden_stride elements (>= D, multiple of 8), 16-byte aligned.
+ *   Row t < n_rows reads hidden row src = row_index[t] (device i64, nullable: src = t) and
+ *   y[src], old_logp[src], ref_logp[src], as grpo_loss_fwd_bwd reads logits rows; gathered rows
+ *   are first copied into the workspace (n_rows * D * 2 bytes).  Outputs are in row order t.
+ * weight: device bf16 [V, D], dense, 16-byte aligned.  D: a multiple of 8.
+ * adv, row_rollout (indexed by t), eps_low, eps_high, beta, agg_mode, denom_tokens, seq_off,
+ *   n_seq, status: as grpo_loss_fwd_bwd.
+ * dhidden: device [n_rows, D] (dense), bf16 or f32 per dhidden_dtype.  dweight: device f32
+ *   [V, D], overwritten, or added to when accumulate_dweight != 0.
+ * dlogits_out: nullable device bf16 [n_rows, grpo_lmhead_dlogits_stride(V)], 16-byte aligned;
+ *   when given it receives every row's dlogits (columns >= V are 0) and no chunk buffer is used.
+ * logp_out (f32 [n_rows]) and row_loss_out (f64 [n_rows]): nullable.  loss_out: device f64 [1].
+ * chunk_rows: rows of dlogits held at a time (rounded up to a multiple of 128); 0 picks the
+ *   largest count that fits a 4 GiB bf16 chunk.  Smaller chunks need less workspace.
+ * Workspace: per row 1.3 KB of softmax statistics, the chunk of dlogits (unless dlogits_out) and
+ *   32 MiB for cuBLASLt, whose two GEMMs per chunk run with that scratch on `stream`.
+ * Kernels: pass 1 (statistics) and pass 2 (dlogits, per chunk) are tcgen05 GEMM kernels with TMA
+ *   operand loads and TMEM accumulators, one CTA per SM; a row kernel applies Eqs. 1-3 between
+ *   them.  Limits: n_rows < 2^31; V >= 1; D >= 8.  Errors: GRPO_ERR_INVALID_ARG for bad sizes,
+ *   alignment, NULL required pointers; GRPO_ERR_CUDA when a launch, the tensor-map encoder or
+ *   cuBLASLt fails.
+ */
+grpo_status grpo_lmhead_loss_fwd_bwd(const void* hidden, int64_t hidden_stride,
+                                     const int64_t* row_index, int64_t n_rows, const void* weight,
+                                     int32_t V, int32_t D, const int32_t* y,
+                                     const float* old_logp, const float* ref_logp,
+                                     const float* adv, const int32_t* row_rollout, float eps_low,
+                                     float eps_high, float beta, int32_t agg_mode,
+                                     int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq,
+                                     void* dhidden, int32_t dhidden_dtype, float* dweight,
+                                     int32_t accumulate_dweight, void* dlogits_out,
+                                     float* logp_out, double* row_loss_out, double* loss_out,
+                                     int32_t* status, int64_t chunk_rows, void* ws,
+                                     size_t* ws_bytes, grpo_stream_t stream);
+
+/*
+ * grpo_lmhead_logp_fwd — log-probability of the sampled token from hidden states, for the old- and
+ * reference-policy evaluations of the kept trajectories (Sec. 3.2) through their output layers:
+ *   logp_out[t] = z_y - log sum_v exp(z_v),  z = hidden[src] * weight^T,  y = y[src]
+ * The pass-1 kernel of grpo_lmhead_loss_fwd_bwd alone (plus its row kernel): no loss, no gradient.
+ * hidden, hidden_stride, row_index, n_rows, weight, V, D, y, status: as grpo_lmhead_loss_fwd_bwd.
+ * logp_out: device f32 [n_rows] (NaN for a token id outside [0, V)).  Workspace: per row 1.3 KB,
+ * plus the gathered rows with row_index.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
+ */
+grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
+                                 const int64_t* row_index, int64_t n_rows, const void* weight,
+                                 int32_t V, int32_t D, const int32_t* y, float* logp_out,
+                                 int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream);
+
+/* Row stride, in elements, of grpo_lmhead_loss_fwd_bwd's dlogits_out: V rounded up to a multiple
+ * of 32 (0 for V < 1). */
+int64_t grpo_lmhead_dlogits_stride(int32_t V);
 
 /*
  * grpo_sum_f64 — *out = v[0] + ... + v[n-1] in fp64, in the same fixed order grpo_loss_fwd_bwd

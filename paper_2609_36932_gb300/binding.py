@@ -32,7 +32,8 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 # Every function include/fastrl_grpo.h declares.
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
-           "grpo_sum_f64", "grpo_logp_fwd",
+           "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
+           "grpo_lmhead_logp_fwd",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -106,6 +107,16 @@ def lib():
     L.grpo_gspo_loss_fwd_bwd_dev.restype = _i32
     L.grpo_logp_fwd.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p]
     L.grpo_logp_fwd.restype = _i32
+    L.grpo_lmhead_loss_fwd_bwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p, _c_p, _c_p,
+                                           _c_p, _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64,
+                                           _c_p, _i32, _c_p, _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                           _i64, _c_p, _c_p, _c_p]
+    L.grpo_lmhead_loss_fwd_bwd.restype = _i32
+    L.grpo_lmhead_logp_fwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p, _c_p, _c_p,
+                                       _c_p, _c_p, _c_p]
+    L.grpo_lmhead_logp_fwd.restype = _i32
+    L.grpo_lmhead_dlogits_stride.argtypes = [_i32]
+    L.grpo_lmhead_dlogits_stride.restype = _i64
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
     L.grpo_sum_f64.restype = _i32
     L.grpo_test_skip_copy.argtypes = [_i32]
@@ -363,6 +374,113 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
     wp, size = _ws_args(wst)
     _check(L.grpo_loss_fwd_bwd(*args_head, wp, size, _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
+
+
+def grpo_lmhead_dlogits_stride(V: int) -> int:
+    """Row stride (elements) of grpo_lmhead_loss_fwd_bwd's dlogits_out."""
+    return int(lib().grpo_lmhead_dlogits_stride(int(V)))
+
+
+def grpo_lmhead_logp_fwd(hidden, weight, y, *, row_index=None, n_rows: int | None = None,
+                         logp_out=None, status=None, ws=None, stream=None):
+    """log pi(y) from hidden states through the output layer (see the header).  Returns
+    dict(logp, ws)."""
+    torch = _torch()
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise TypeError("hidden and weight must be bf16")
+    if hidden.dim() != 2 or hidden.stride(1) != 1 or not hidden.is_cuda:
+        raise ValueError("hidden must be a 2-D CUDA tensor with unit stride along D")
+    if weight.dim() != 2 or not weight.is_contiguous() or weight.shape[1] != hidden.shape[1]:
+        raise ValueError("weight must be a contiguous [V, D] tensor")
+    D = hidden.shape[1]
+    V = weight.shape[0]
+    if n_rows is None:
+        n_rows = row_index.numel() if row_index is not None else hidden.shape[0]
+    if row_index is not None:
+        _need(row_index, torch.int64, n_rows, "row_index")
+    _need(y, torch.int32, None if row_index is not None else n_rows, "y")
+    if logp_out is None:
+        logp_out = torch.empty(max(int(n_rows), 1), dtype=torch.float32, device=hidden.device)
+    L = lib()
+    head = (_ptr(hidden), int(hidden.stride(0)), _ptr(row_index), int(n_rows), _ptr(weight), int(V),
+            int(D), _ptr(y), _ptr(logp_out), _ptr(status))
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_lmhead_logp_fwd(*head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, hidden.device, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_lmhead_logp_fwd(*head, wp, size, _stream(stream)))
+    return dict(logp=logp_out, ws=wst)
+
+
+def grpo_lmhead_loss_fwd_bwd(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *,
+                             eps_low: float = 0.2, eps_high: float = 0.2, beta: float = 0.04,
+                             agg_mode: int = 0, denom_tokens: int | None = None, seq_off=None,
+                             n_seq: int = 0, dhidden=None, dhidden_dtype=None, dweight=None,
+                             accumulate_dweight: bool = False, dlogits_out=None, logp_out=None,
+                             row_loss_out=None, loss_out=None, status=None, chunk_rows: int = 0,
+                             row_index=None, n_rows: int | None = None, ws=None, stream=None):
+    """The output layer fused with the GRPO loss (see the header): hidden bf16 [*, D] (rows taken
+    through row_index when given), weight bf16 [V, D].  Returns dict(loss, dhidden, dweight, logp,
+    row_loss, dlogits)."""
+    torch = _torch()
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise TypeError("hidden and weight must be bf16")
+    if not (hidden.is_cuda and weight.is_cuda):
+        raise TypeError("hidden and weight must be CUDA tensors")
+    if hidden.dim() != 2 or hidden.stride(1) != 1:
+        raise ValueError("hidden must be 2-D with unit stride along D")
+    if weight.dim() != 2 or not weight.is_contiguous():
+        raise ValueError("weight must be a contiguous [V, D] tensor")
+    D = hidden.shape[1]
+    if n_rows is None:
+        n_rows = row_index.numel() if row_index is not None else hidden.shape[0]
+    if row_index is not None:
+        _need(row_index, torch.int64, n_rows, "row_index")
+    V = weight.shape[0]
+    if weight.shape[1] != D:
+        raise ValueError("hidden and weight disagree on D")
+    dev = hidden.device
+    if dhidden_dtype is None:
+        dhidden_dtype = dhidden.dtype if dhidden is not None else torch.bfloat16
+    if dhidden_dtype in (torch.bfloat16, "bf16"):
+        dht, ht = GRPO_DTYPE_BF16, torch.bfloat16
+    elif dhidden_dtype in (torch.float32, "f32"):
+        dht, ht = GRPO_DTYPE_F32, torch.float32
+    else:
+        raise TypeError("dhidden must be bf16 or f32")
+    if dhidden is None:
+        dhidden = torch.empty((n_rows, D), dtype=ht, device=dev)
+    _need(dhidden, ht, n_rows * D, "dhidden")
+    if dweight is None:
+        dweight = torch.empty((V, D), dtype=torch.float32, device=dev)
+    _need(dweight, torch.float32, V * D, "dweight")
+    if dlogits_out is not None:
+        _need(dlogits_out, torch.bfloat16, n_rows * grpo_lmhead_dlogits_stride(V), "dlogits_out")
+    if loss_out is None:
+        loss_out = torch.empty(1, dtype=torch.float64, device=dev)
+    if denom_tokens is None:
+        denom_tokens = max(int(n_rows), 1)
+    n_src = None if row_index is not None else n_rows
+    _need(y, torch.int32, n_src, "y")
+    _need(old_logp, torch.float32, n_src, "old_logp")
+    _need(ref_logp, torch.float32, n_src, "ref_logp")
+    _need(adv, torch.float32, None, "adv")
+    _need(row_rollout, torch.int32, n_rows, "row_rollout")
+    L = lib()
+    head = (_ptr(hidden), int(hidden.stride(0)), _ptr(row_index), int(n_rows), _ptr(weight),
+            int(V), int(D),
+            _ptr(y), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(row_rollout),
+            float(eps_low), float(eps_high), float(beta), int(agg_mode), int(denom_tokens),
+            _ptr(seq_off), int(n_seq), _ptr(dhidden), dht, _ptr(dweight),
+            1 if accumulate_dweight else 0, _ptr(dlogits_out), _ptr(logp_out),
+            _ptr(row_loss_out), _ptr(loss_out), _ptr(status), int(chunk_rows))
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_lmhead_loss_fwd_bwd(*head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, dev, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_lmhead_loss_fwd_bwd(*head, wp, size, _stream(stream)))
+    return dict(loss=loss_out, dhidden=dhidden, dweight=dweight, logp=logp_out,
+                row_loss=row_loss_out, dlogits=dlogits_out, ws=wst)
 
 
 def grpo_gspo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,

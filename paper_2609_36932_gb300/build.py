@@ -1,6 +1,7 @@
 """Build libfastrl_grpo.so (the CUDA path) in-tree for sm_103a.
 
-Each .cu file is compiled by nvcc in parallel, then linked with the static CUDA runtime into
+Each .cu file is compiled by nvcc in parallel, then linked with the static CUDA runtime (and
+the toolkit's cuBLASLt, for the two plain GEMMs of the output-layer loss) into
 paper_2609_36932_gb300/_build/libfastrl_grpo.so.  Nothing is installed outside the tree.
 """
 from __future__ import annotations
@@ -17,7 +18,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libfastrl_grpo.so")
-SOURCES = ["api.cu", "advantage.cu", "prune.cu", "compact.cu", "loss.cu", "gspo.cu", "reduce.cu"]
+SOURCES = ["api.cu", "advantage.cu", "prune.cu", "compact.cu", "loss.cu", "gspo.cu", "reduce.cu",
+           "lmhead.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I", INCLUDE, "-I", CSRC]
@@ -67,7 +69,9 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
                 raise RuntimeError("nvcc failed on %s" % src)
             objs.append(obj)
     tmp = LIB + ".tmp.%d" % os.getpid()
-    r = subprocess.run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs],
+    cuda_lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(cc))), "lib64")
+    r = subprocess.run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs,
+                        "-L" + cuda_lib, "-lcublasLt", "-Xlinker", "-rpath=" + cuda_lib],
                        capture_output=True, text=True)
     if r.returncode != 0:
         sys.stderr.write(r.stdout + r.stderr)

@@ -1,0 +1,923 @@
+// The policy's output layer fused with the GRPO token loss, on the tensor cores.
+//
+// Sec. 3.2 runs every kept trajectory through the policy, whose last layer maps each token's
+// hidden state h_t (D values) to logits over the vocabulary; Eqs. 1-3 turn those into the loss.
+// With the output layer's weight rows W_v:
+//   z[t, v] = sum_d h[t, d] * W[v, d]
+//   loss, logp: Eqs. 1-3 on z, as grpo_loss_fwd_bwd computes them
+//   dh = dlogits * W,   dW = dlogits^T * h        (the chain rule through z = h W^T)
+// The [rows, V] logits are never stored whole.  They are produced 128 x 256 at a time into
+// tensor memory by tcgen05.mma (bf16 operands staged in shared memory by TMA, f32 accumulators)
+// and consumed there:
+//   Pass 1 (lmhead_tile_kernel<false>): per row, the running maximum and the sum of exp(z - max)
+//     over the vocabulary tiles a CTA visits (z_y excluded from the sum and kept separately).
+//   lmhead_rows_kernel: the partial sums combined -> lse, logp, the loss term and the gradient
+//     scalars of each row (the same formulas as the fused loss kernel).
+//   Pass 2 (lmhead_tile_kernel<true>), for each chunk of rows: the tiles recomputed and
+//     dlogits = coef * ([v == y] - softmax(z)_v) written in bf16 to a chunk buffer.
+//   Two plain GEMMs per chunk (cuBLASLt): dh = dlogits * W and dW (+)= dlogits^T * h.
+//
+// Kernel roles (192 threads, one CTA per SM: 197 KB of shared memory, all 512 TMEM columns):
+//   warp 0, one lane: TMA producer, 4 stages of {A: 128 rows x 64 of h, B: 256 rows x 64 of W},
+//     128-byte swizzled;
+//   warp 1: allocates TMEM; one lane issues the MMAs (M = 128, N = 256, K = 16) into one of two
+//     256-column accumulators, so the epilogue of a tile overlaps the MMAs of the next;
+//   warps 2-5: the epilogue, one thread per tile row, reading its row from TMEM 32 columns at a
+//     time (a warp may read only its quarter of the 128 lanes: warp % 4).
+// Work: CTA c owns row lane i = c % R and vocabulary lane j = c / R; for each group of R row
+// blocks it takes row block g*R + i and the vocabulary tiles j, j + J, j + 2J, ...  At any time
+// the grid works on R consecutive row blocks and J consecutive vocabulary tiles, which the L2
+// serves to all of it.
+//
+// Every wait is bounded (about a second): a wait that runs out sets GRPO_DEVFLAG_TIMEOUT and an
+// abort flag; the roles then stop, the producer waits for its copies in flight and the MMA lane
+// for its MMAs, and warp 1 frees the tensor memory before the CTA exits.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cublasLt.h>
+
+#include <algorithm>
+#include <cmath>
+#include <mutex>
+
+#include "common.cuh"
+#include "rowops.cuh"
+
+namespace fastrl {
+namespace {
+
+constexpr int BM = 128;  // rows of h per tile (MMA M; TMEM lanes)
+constexpr int BN = 256;  // vocabulary entries per tile (MMA N; TMEM columns per accumulator)
+constexpr int BK = 64;   // D per stage: one 128-byte swizzle row of bf16
+constexpr int kStages = 4;
+constexpr uint32_t kABytes = BM * BK * 2;
+constexpr uint32_t kBBytes = BN * BK * 2;
+constexpr uint32_t kStageBytes = kABytes + kBBytes;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 2 * BN;
+constexpr int kRowLanes = 8;       // R: row blocks in flight across the grid
+constexpr int kMaxJ = 160;         // vocabulary lanes (partial sums per row) at most
+constexpr int kBars = 2 * kStages + 5;  // full, empty, acc full x2, acc empty x2, drain
+constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + 8 * kBars + 16;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+constexpr int64_t kDefaultChunkBytes = 4ll << 30;  // dlogits chunk buffer
+constexpr size_t kLtWorkspace = 32u << 20;
+
+// Instruction descriptor of tcgen05.mma.kind::f16: f32 accumulator (bits 4-5 = 1), bf16 A and B
+// (bits 7-9, 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at 24-28.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                            ((uint32_t)(BM >> 4) << 24);
+
+// Shared-memory matrix descriptor for a K-major operand in the 128-byte swizzle layout that TMA
+// writes with CU_TENSOR_MAP_SWIZZLE_128B: rows of 128 bytes, 8-row atoms 1024 bytes apart (the
+// stride byte offset), start address >> 4 in bits 0-13, descriptor version 1 (bit 46), layout
+// 2 = 128-byte swizzle (bits 61-63).  The leading byte offset is unused for this layout.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(100000u)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
+      : "memory");
+}
+// The barrier receives one arrival once every MMA this thread issued so far has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   bar)
+               : "memory");
+}
+// 32 consecutive f32 columns of this thread's TMEM lane, waited for in the same statement so
+// that no use of the registers can be scheduled before the data is there.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
+      "%30, %31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
+}
+
+struct TileArgs {
+  int32_t rows;   // rows of this launch (a chunk in pass 2); the tensor map's row = row0 + local
+  int32_t row0;
+  int32_t V, nK, n_vt, n_rb, R, J;
+  const int32_t* y;  // [rows]
+  // pass 1
+  float2* part;  // [rows][J]: (max, sum of exp(z - max) without z_y) of vocabulary lane j
+  float* zy;     // [rows]: z_y, written by the CTA whose tile holds y
+  // pass 2
+  const float4* rowsc;  // [rows]: {neg_scale, dy, shift, 0} from lmhead_rows_kernel
+  __nv_bfloat16* dl;    // [rows][ldd]
+  int64_t ldd;
+  int32_t* status;
+};
+
+template <bool kBwd>
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_tile_kernel(const __grid_constant__ CUtensorMap tm_h,
+                       const __grid_constant__ CUtensorMap tm_w, const TileArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  const uint32_t raw_s = smem_addr(smem_raw);
+  const uint32_t base_s = (raw_s + 1023u) & ~1023u;  // swizzle atoms need 1024-byte alignment
+  const uint32_t bar_s = base_s + kStages * kStageBytes;
+  auto full_bar = [&](int k) { return bar_s + 8u * k; };
+  auto empty_bar = [&](int k) { return bar_s + 8u * (kStages + k); };
+  auto accf_bar = [&](int k) { return bar_s + 8u * (2 * kStages + k); };
+  auto acce_bar = [&](int k) { return bar_s + 8u * (2 * kStages + 2 + k); };
+  const uint32_t drain_bar = bar_s + 8u * (2 * kStages + 4);
+  unsigned char* tail = smem_raw + (bar_s - raw_s) + 8 * kBars;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(tail);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tail + 4);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < kStages; ++k) {
+      mbar_init(full_bar(k), 1);
+      mbar_init(empty_bar(k), 1);
+    }
+    for (int k = 0; k < 2; ++k) {
+      mbar_init(accf_bar(k), 1);
+      mbar_init(acce_bar(k), 4 * 32);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_addr((const void*)tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // Bounded wait; false when the phase did not complete (or another role gave up).
+  auto wait_bar = [&](uint32_t bar, uint32_t parity, bool honour_abort) -> bool {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 1; !mbar_try_wait(bar, parity); ++it) {
+      if ((it & 63u) != 0) continue;
+      if (honour_abort && *abort_flag) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        if (a.status) atomicOr(a.status, GRPO_DEVFLAG_TIMEOUT);
+        return false;
+      }
+    }
+    return true;
+  };
+
+  const int R = a.R, J = a.J;
+  const int li = (int)blockIdx.x % R, lj = (int)blockIdx.x / R;
+
+  if (warp == 0) {
+    // ---- TMA producer ----
+    if (lane == 0) {
+      uint32_t fills = 0;
+      bool ok = true;
+      for (int rb = li; ok && rb < a.n_rb; rb += R) {
+        for (int vt = lj; ok && vt < a.n_vt; vt += J) {
+          for (int kb = 0; kb < a.nK; ++kb) {
+            const int st = (int)(fills % kStages);
+            const uint32_t ph = (fills / kStages) & 1u;
+            if (!wait_bar(empty_bar(st), ph ^ 1u, true)) {
+              ok = false;
+              break;
+            }
+            const uint32_t sa = base_s + st * kStageBytes;
+            mbar_expect_tx(full_bar(st), kStageBytes);
+            tma_load_2d(sa, &tm_h, kb * BK, a.row0 + rb * BM, full_bar(st));
+            tma_load_2d(sa + kABytes, &tm_w, kb * BK, vt * BN, full_bar(st));
+            ++fills;
+          }
+        }
+      }
+      // Copies still in flight land before the CTA can exit.
+      const uint32_t n = fills < (uint32_t)kStages ? fills : (uint32_t)kStages;
+      for (uint32_t f = fills - n; f < fills; ++f)
+        wait_bar(full_bar((int)(f % kStages)), (f / kStages) & 1u, false);
+    }
+  } else if (warp == 1) {
+    // ---- MMA issuer ----
+    if (lane == 0) {
+      uint32_t fills = 0, tiles = 0;
+      bool ok = true;
+      for (int rb = li; ok && rb < a.n_rb; rb += R) {
+        for (int vt = lj; ok && vt < a.n_vt; vt += J) {
+          const uint32_t acc = tiles & 1u;
+          if (!wait_bar(acce_bar(acc), ((tiles >> 1) & 1u) ^ 1u, true)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem + acc * BN;
+          for (int kb = 0; kb < a.nK; ++kb) {
+            const int st = (int)(fills % kStages);
+            if (!wait_bar(full_bar(st), (fills / kStages) & 1u, true)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = base_s + st * kStageBytes;
+            const uint64_t ad = smem_desc(sa), bd = smem_desc(sa + kABytes);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)  // K = 16 per MMA: 32 bytes along the swizzled row
+              tc_mma(d_tmem, ad + 2 * k, bd + 2 * k, (kb | k) != 0 ? 1u : 0u);
+            tc_commit(empty_bar(st));  // the stage is free once these MMAs have read it
+            ++fills;
+          }
+          if (!ok) break;
+          tc_commit(accf_bar(acc));
+          ++tiles;
+        }
+      }
+      // Every MMA issued has completed before the tensor memory is freed.
+      tc_commit(drain_bar);
+      wait_bar(drain_bar, 0, false);
+    }
+  } else {
+    // ---- epilogue: one thread per tile row ----
+    const int q = warp & 3;            // TMEM lane quarter this warp may read
+    const int r_in = q * 32 + lane;    // row within the tile
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    uint32_t tiles = 0;
+    bool ok = true;
+    for (int rb = li; ok && rb < a.n_rb; rb += R) {
+      const int row = rb * BM + r_in;
+      const bool rv = row < a.rows;
+      const int yv = rv ? a.y[row] : -1;
+      float m = -INFINITY, s = 0.f;  // pass 1: running max, sum of exp(z - m) without z_y
+      float4 sc = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (kBwd && rv) sc = a.rowsc[row];
+      const float neg_scale = sc.x, dy = sc.y, shB = sc.z;
+      __nv_bfloat16* out_row = kBwd ? a.dl + (int64_t)(rv ? row : 0) * a.ldd : nullptr;
+      for (int vt = lj; vt < a.n_vt; vt += J) {
+        const uint32_t acc = tiles & 1u;
+        int got = 0;
+        if (lane == 0) got = wait_bar(accf_bar(acc), (tiles >> 1) & 1u, true) ? 1 : 0;
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!got) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t taddr = tmem + lane_base + acc * BN;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          const int v0 = vt * BN + c;
+          if (v0 >= a.V) break;  // warp-uniform: columns past the vocabulary
+          float x[32];
+          tmem_ld32(taddr + c, x);
+          const int nvalid = a.V - v0;  // >= 1
+          const int jy = yv - v0;       // y's column in this chunk, if in [0, 32)
+          if (!kBwd) {
+            float cm = -INFINITY;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              if (k >= nvalid) x[k] = -INFINITY;
+              cm = fmaxf(cm, x[k]);
+            }
+            if (cm > m) {
+              s *= ex2((m - cm) * kLog2e);
+              m = cm;
+            }
+            const float mb = m * kLog2e;
+            float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+            for (int k = 0; k < 32; k += 2) {
+              const float e0 = (k == jy) ? 0.f : ex2(fmaf(x[k], kLog2e, -mb));
+              const float e1 = (k + 1 == jy) ? 0.f : ex2(fmaf(x[k + 1], kLog2e, -mb));
+              s0 += e0;
+              s1 += e1;
+            }
+            s += s0 + s1;
+            if (rv && (unsigned)jy < 32u) {
+              float zyv = 0.f;
+#pragma unroll
+              for (int k = 0; k < 32; ++k)
+                if (k == jy) zyv = x[k];
+              a.zy[row] = zyv;
+            }
+          } else {
+            uint32_t pk[16];
+#pragma unroll
+            for (int k = 0; k < 32; k += 2) {
+              float d0 = neg_scale * ex2(fmaf(x[k], kLog2e, shB));
+              float d1 = neg_scale * ex2(fmaf(x[k + 1], kLog2e, shB));
+              if (k == jy) d0 = dy;
+              if (k + 1 == jy) d1 = dy;
+              if (k >= nvalid) d0 = 0.f;
+              if (k + 1 >= nvalid) d1 = 0.f;
+              pk[k / 2] = pack_bf16x2(make_float2(d0, d1));
+            }
+            if (rv) {
+              uint4* dst = reinterpret_cast<uint4*>(out_row + v0);
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                dst[k] = make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+            }
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(acce_bar(acc));
+        ++tiles;
+      }
+      if (!kBwd && ok && rv) a.part[(int64_t)row * J + lj] = make_float2(m, s);
+    }
+  }
+
+  __syncwarp();  // lanes that had no role wait for their warp's working lane
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+struct RowArgs {
+  int32_t rows, J, V;
+  const float2* part;
+  const float* zy;
+  const int32_t* y;
+  const float *old_logp, *ref_logp, *adv;
+  const int32_t* row_rollout;
+  const int64_t* seq_off;
+  float beta, lo_up, hi_dn, lo_rn, hi_rn;
+  int32_t agg_mode;
+  double inv_denom;
+  float inv_denom_f, inv_nseq_f;
+  float* logp_out;
+  double* row_loss;
+  float4* rowsc;
+  int32_t* status;
+  int32_t logp_only;  // forward entry: logp_out alone
+};
+
+// One thread per row: combine the J partial sums and apply Eqs. 1-3 (the same arithmetic as the
+// fused loss kernel's row scalars).
+__global__ void __launch_bounds__(256) lmhead_rows_kernel(const RowArgs a) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= a.rows) return;
+  const int yv = a.y[t];
+  if (yv < 0 || yv >= a.V) {
+    if (a.logp_out) a.logp_out[t] = __int_as_float(0x7fc00000);
+    if (!a.logp_only) {
+      a.row_loss[t] = 0.0;
+      a.rowsc[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
+    return;
+  }
+  const float2* p = a.part + (int64_t)t * a.J;
+  float M = -INFINITY;
+  for (int j = 0; j < a.J; ++j) M = fmaxf(M, p[j].x);
+  float S_excl = 0.f;
+  for (int j = 0; j < a.J; ++j) {
+    const float2 v = p[j];
+    if (v.x != -INFINITY) S_excl += v.y * expf(v.x - M);
+  }
+  const float zy = a.zy[t];
+  const float S = S_excl + expf(zy - M);
+  const float logp = (zy - M) - logf(S);
+  if (a.logp_only) {
+    a.logp_out[t] = logp;
+    if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
+    return;
+  }
+  const float A = a.adv[a.row_rollout[t]];
+  const float rho = expf(logp - a.old_logp[t]);
+  const float clipped = rho < a.lo_up ? a.lo_rn : (rho > a.hi_dn ? a.hi_rn : rho);
+  const float surr = fminf(rho * A, clipped * A);
+  const float x = a.ref_logp[t] - logp;
+  const float em1 = expm1f(x);
+  const float kl = em1 - x;
+  const float ell = -(surr - a.beta * kl);
+  float w;
+  if (a.agg_mode == 0) {
+    w = a.inv_denom_f;
+  } else {
+    const int32_t r = a.row_rollout[t];
+    w = a.inv_nseq_f / (float)(a.seq_off[r + 1] - a.seq_off[r]);
+  }
+  const bool c = (A >= 0.f) ? (rho <= a.hi_dn) : (rho >= a.lo_up);
+  const float g = -((c ? rho * A : 0.f) + a.beta * em1);
+  const float coef = w * g;
+  float neg_scale = -coef / S;
+  const float dy = coef * (S_excl / S);
+  float shB = -M * kLog2e;
+  if (fabsf(neg_scale) >= 0x1p-100f) {
+    shB += kShiftB;
+    neg_scale *= 0x1p-16f;  // 2^-kShiftB
+  }
+  a.rowsc[t] = make_float4(neg_scale, dy, shB, 0.f);
+  if (a.logp_out) a.logp_out[t] = logp;
+  a.row_loss[t] = (a.agg_mode == 0 ? a.inv_denom : (double)w) * (double)ell;
+  if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
+}
+
+// Kept rows gathered into a dense block: hidden row src = row_index[t] (16-byte vectors, one CTA
+// per row) and its y, old_logp, ref_logp.
+__global__ void __launch_bounds__(128) lmhead_gather_kernel(
+    const uint4* __restrict__ hidden, int64_t stride_vec, const int64_t* __restrict__ row_index,
+    int32_t n_rows, int32_t row_vec, const int32_t* __restrict__ y, const float* __restrict__ old,
+    const float* __restrict__ ref, uint4* __restrict__ out, int32_t* __restrict__ y_out,
+    float* __restrict__ old_out, float* __restrict__ ref_out) {
+  for (int t = blockIdx.x; t < n_rows; t += gridDim.x) {
+    const int64_t src = row_index[t];
+    const uint4* in = hidden + src * stride_vec;
+    uint4* o = out + (int64_t)t * row_vec;
+    for (int k = threadIdx.x; k < row_vec; k += blockDim.x) o[k] = in[k];
+    if (threadIdx.x == 0) {
+      y_out[t] = y[src];
+      if (old) old_out[t] = old[src];
+      if (ref) ref_out[t] = ref[src];
+    }
+  }
+}
+
+// ---- host side ---------------------------------------------------------------------------------
+
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                 const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                 const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                 CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encode_fn() {
+  static EncodeTiled fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiled>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map over rows x cols (row stride `stride` elements), box 64 x box_rows,
+// 128-byte swizzle, zero fill outside the tensor.
+bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int64_t stride,
+              uint32_t box_rows) {
+  EncodeTiled fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)stride * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return n;
+}
+
+struct Grid {
+  int R, J, grid;
+};
+Grid plan(int64_t rows, int V, int n_sm) {
+  const int n_rb = (int)((rows + BM - 1) / BM);
+  const int n_vt = (V + BN - 1) / BN;
+  Grid g;
+  g.R = std::max(1, std::min(n_rb, kRowLanes));
+  g.J = std::max(1, std::min({n_vt, std::max(1, n_sm / g.R), kMaxJ}));
+  g.grid = g.R * g.J;
+  return g;
+}
+
+grpo_status launch_tiles(bool bwd, const CUtensorMap& mh, const CUtensorMap& mw,
+                         const TileArgs& a, int grid, cudaStream_t s, const char* who) {
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    attr_err = cudaFuncSetAttribute(lmhead_tile_kernel<false>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(lmhead_tile_kernel<true>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)kSmemBytes);
+  });
+  if (attr_err != cudaSuccess)
+    return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(attr_err));
+  if (bwd)
+    lmhead_tile_kernel<true><<<grid, kThreads, kSmemBytes, s>>>(mh, mw, a);
+  else
+    lmhead_tile_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(mh, mw, a);
+  count_launches(1);
+  return check_launch(who);
+}
+
+// cuBLASLt: C (col-major m x n, ldc) = op(A) * op(B) + beta * C, f32 accumulation.
+cublasLtHandle_t lt_handle() {
+  static cublasLtHandle_t h = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    if (cublasLtCreate(&h) != CUBLAS_STATUS_SUCCESS) h = nullptr;
+  });
+  return h;
+}
+
+grpo_status lt_gemm(cudaStream_t s, bool ta, bool tb, int64_t m, int64_t n, int64_t k,
+                    const void* A, int64_t lda, const void* B, int64_t ldb, void* C,
+                    cudaDataType_t ctype, int64_t ldc, float beta, void* ws, size_t ws_bytes,
+                    const char* who) {
+  cublasLtHandle_t h = lt_handle();
+  if (!h) return fail(GRPO_ERR_CUDA, "%s: cublasLtCreate failed", who);
+  cublasLtMatmulDesc_t op = nullptr;
+  cublasLtMatrixLayout_t la = nullptr, lb = nullptr, lc = nullptr;
+  cublasLtMatmulPreference_t pref = nullptr;
+  grpo_status st = GRPO_OK;
+  const cublasOperation_t opa = ta ? CUBLAS_OP_T : CUBLAS_OP_N, opb = tb ? CUBLAS_OP_T : CUBLAS_OP_N;
+  const float alpha = 1.f;
+  cublasLtMatmulHeuristicResult_t res = {};
+  int found = 0;
+  bool ok = cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F) == CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof opa) ==
+                CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof opb) ==
+                CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, ta ? k : m, ta ? m : k, lda) ==
+                CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, tb ? n : k, tb ? k : n, ldb) ==
+                CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatrixLayoutCreate(&lc, ctype, m, n, ldc) == CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatmulPreferenceCreate(&pref) == CUBLAS_STATUS_SUCCESS &&
+            cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
+                                                 &ws_bytes, sizeof ws_bytes) ==
+                CUBLAS_STATUS_SUCCESS;
+  if (ok)
+    ok = cublasLtMatmulAlgoGetHeuristic(h, op, la, lb, lc, lc, pref, 1, &res, &found) ==
+             CUBLAS_STATUS_SUCCESS &&
+         found > 0;
+  if (!ok) {
+    st = fail(GRPO_ERR_CUDA, "%s: no cuBLASLt algorithm for %lld x %lld x %lld", who,
+              (long long)m, (long long)n, (long long)k);
+  } else {
+    const cublasStatus_t r = cublasLtMatmul(h, op, &alpha, A, la, B, lb, &beta, C, lc, C, lc,
+                                            &res.algo, ws, ws_bytes, s);
+    if (r != CUBLAS_STATUS_SUCCESS)
+      st = fail(GRPO_ERR_CUDA, "%s: cublasLtMatmul failed (%d)", who, (int)r);
+  }
+  if (pref) cublasLtMatmulPreferenceDestroy(pref);
+  if (lc) cublasLtMatrixLayoutDestroy(lc);
+  if (lb) cublasLtMatrixLayoutDestroy(lb);
+  if (la) cublasLtMatrixLayoutDestroy(la);
+  if (op) cublasLtMatmulDescDestroy(op);
+  return st;
+}
+
+int64_t padded_v(int32_t V) { return (int64_t)align_up((size_t)V, 32); }
+
+int64_t chunk_of(int64_t n_rows, int32_t V, int64_t chunk_rows) {
+  int64_t c = chunk_rows;
+  if (c <= 0) c = std::max<int64_t>(BM, kDefaultChunkBytes / (padded_v(V) * 2) / BM * BM);
+  c = (c + BM - 1) / BM * BM;
+  return std::max<int64_t>(BM, std::min<int64_t>(c, (n_rows + BM - 1) / BM * BM));
+}
+
+struct WsLayout {
+  size_t part, zy, rowsc, row_loss, dl, lt, hid, ys, olds, refs, total;
+};
+WsLayout ws_layout(int64_t n_rows, int32_t V, int32_t D, int64_t chunk, bool own_dl, bool gather,
+                   bool loss) {
+  WsLayout w;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = align_up(o + bytes, 256);
+    return at;
+  };
+  const size_t n = (size_t)std::max<int64_t>(n_rows, 1);
+  w.part = take(n * kMaxJ * sizeof(float2));
+  w.zy = take(n * sizeof(float));
+  w.rowsc = take(loss ? n * sizeof(float4) : 0);
+  w.row_loss = take(loss ? n * sizeof(double) : 0);
+  w.dl = take(loss && own_dl ? (size_t)chunk * padded_v(V) * 2 : 0);
+  w.lt = take(loss ? kLtWorkspace : 0);
+  w.hid = take(gather ? n * (size_t)D * 2 : 0);
+  w.ys = take(gather ? n * 4 : 0);
+  w.olds = take(gather ? n * 4 : 0);
+  w.refs = take(gather ? n * 4 : 0);
+  w.total = o;
+  return w;
+}
+
+}  // namespace
+}  // namespace fastrl
+
+using namespace fastrl;
+
+namespace {
+
+// Shared front of both entries: argument checks common to them, the optional gather of the rows,
+// the tensor maps and pass 1 (softmax statistics).  Returns the maps and the row arrays in use.
+struct Front {
+  CUtensorMap mh, mw;
+  const void* hid;
+  int64_t hstride;
+  const int32_t* y;
+  const float* old_logp;
+  const float* ref_logp;
+  int n_sm;
+  int J;
+  TileArgs ta;
+};
+
+grpo_status check_shape(const char* who, int64_t n_rows, int32_t V, int32_t D,
+                        int64_t hidden_stride) {
+  if (n_rows < 0 || n_rows >= (int64_t)1 << 31)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: n_rows %lld outside [0, 2^31)", who, (long long)n_rows);
+  if (V < 1 || D < 8 || D % 8 != 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: need V >= 1 and D a positive multiple of 8 (V=%d D=%d)",
+                who, V, D);
+  if (hidden_stride < D || hidden_stride % 8 != 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: hidden_stride %lld must be >= D and a multiple of 8",
+                who, (long long)hidden_stride);
+  return GRPO_OK;
+}
+
+grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
+                  const int64_t* row_index, int64_t n_rows, const void* weight, int32_t V,
+                  int32_t D, const int32_t* y, const float* old_logp, const float* ref_logp,
+                  int32_t* status, char* wsb, const WsLayout& L, cudaStream_t s, Front* f) {
+  grpo_status st;
+  f->n_sm = sm_count();
+  if (f->n_sm <= 0) return fail(GRPO_ERR_CUDA, "%s: no CUDA device", who);
+  f->hid = hidden;
+  f->hstride = hidden_stride;
+  f->y = y;
+  f->old_logp = old_logp;
+  f->ref_logp = ref_logp;
+  if (row_index) {  // rows taken through row_index are first gathered into a dense block
+    __nv_bfloat16* g_hid = reinterpret_cast<__nv_bfloat16*>(wsb + L.hid);
+    int32_t* g_y = reinterpret_cast<int32_t*>(wsb + L.ys);
+    float* g_old = old_logp ? reinterpret_cast<float*>(wsb + L.olds) : nullptr;
+    float* g_ref = ref_logp ? reinterpret_cast<float*>(wsb + L.refs) : nullptr;
+    const int blocks = (int)std::min<int64_t>(n_rows, (int64_t)f->n_sm * 16);
+    lmhead_gather_kernel<<<blocks, 128, 0, s>>>(
+        static_cast<const uint4*>(hidden), hidden_stride / 8, row_index, (int32_t)n_rows, D / 8, y,
+        old_logp, ref_logp, reinterpret_cast<uint4*>(g_hid), g_y, g_old, g_ref);
+    count_launches(1);
+    if ((st = check_launch(who)) != GRPO_OK) return st;
+    f->hid = g_hid;
+    f->hstride = D;
+    f->y = g_y;
+    f->old_logp = g_old;
+    f->ref_logp = g_ref;
+  }
+  if (!make_map(&f->mh, f->hid, n_rows, D, f->hstride, BM) || !make_map(&f->mw, weight, V, D, D, BN))
+    return fail(GRPO_ERR_CUDA, "%s: cuTensorMapEncodeTiled failed", who);
+  const Grid g1 = plan(n_rows, V, f->n_sm);
+  f->J = g1.J;
+  TileArgs& ta = f->ta;
+  ta = TileArgs{};
+  ta.rows = (int32_t)n_rows;
+  ta.row0 = 0;
+  ta.V = V;
+  ta.nK = (D + BK - 1) / BK;
+  ta.n_vt = (V + BN - 1) / BN;
+  ta.n_rb = (int32_t)((n_rows + BM - 1) / BM);
+  ta.R = g1.R;
+  ta.J = g1.J;
+  ta.y = f->y;
+  ta.part = reinterpret_cast<float2*>(wsb + L.part);
+  ta.zy = reinterpret_cast<float*>(wsb + L.zy);
+  ta.status = status;
+  return launch_tiles(false, f->mh, f->mw, ta, g1.grid, s, who);
+}
+
+}  // namespace
+
+extern "C" int64_t grpo_lmhead_dlogits_stride(int32_t V) { return V >= 1 ? padded_v(V) : 0; }
+
+extern "C" grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
+                                            const int64_t* row_index, int64_t n_rows,
+                                            const void* weight, int32_t V, int32_t D,
+                                            const int32_t* y, float* logp_out, int32_t* status,
+                                            void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  const char* who = "grpo_lmhead_logp_fwd";
+  grpo_status st = check_shape(who, n_rows, V, D, hidden_stride);
+  if (st != GRPO_OK) return st;
+  const WsLayout L = ws_layout(n_rows, V, D, 0, false, row_index != nullptr, false);
+  bool query_only = false;
+  if ((st = workspace_check(ws, ws_bytes, L.total, who, &query_only)) != GRPO_OK || query_only)
+    return st;
+  if (n_rows == 0) return GRPO_OK;
+  if (!hidden || !weight || !y || !logp_out)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: a required pointer is NULL", who);
+  if (((uintptr_t)hidden | (uintptr_t)weight) % 16 != 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: hidden and weight must be 16-byte aligned", who);
+  cudaStream_t s = as_stream(stream);
+  char* wsb = static_cast<char*>(ws);
+  Front f;
+  if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, nullptr, nullptr,
+                  status, wsb, L, s, &f)) != GRPO_OK)
+    return st;
+  RowArgs ra = {};
+  ra.rows = (int32_t)n_rows;
+  ra.J = f.J;
+  ra.V = V;
+  ra.part = f.ta.part;
+  ra.zy = f.ta.zy;
+  ra.y = f.y;
+  ra.logp_out = logp_out;
+  ra.status = status;
+  ra.logp_only = 1;
+  lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
+  count_launches(1);
+  return check_launch(who);
+}
+
+extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
+    const void* hidden, int64_t hidden_stride, const int64_t* row_index, int64_t n_rows,
+    const void* weight, int32_t V, int32_t D, const int32_t* y, const float* old_logp,
+    const float* ref_logp, const float* adv, const int32_t* row_rollout, float eps_low,
+    float eps_high, float beta, int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off,
+    int64_t n_seq, void* dhidden, int32_t dhidden_dtype, float* dweight,
+    int32_t accumulate_dweight, void* dlogits_out, float* logp_out, double* row_loss_out,
+    double* loss_out, int32_t* status, int64_t chunk_rows, void* ws, size_t* ws_bytes,
+    grpo_stream_t stream) {
+  clear_error();
+  const char* who = "grpo_lmhead_loss_fwd_bwd";
+  grpo_status st = check_shape(who, n_rows, V, D, hidden_stride);
+  if (st != GRPO_OK) return st;
+  if (agg_mode != 0 && agg_mode != 1)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: agg_mode must be 0 or 1", who);
+  if (agg_mode == 0 && denom_tokens <= 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: denom_tokens must be positive", who);
+  if (agg_mode == 1 && (seq_off == nullptr || n_seq <= 0))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: agg_mode 1 needs seq_off and n_seq > 0", who);
+  if (dhidden_dtype != GRPO_DTYPE_BF16 && dhidden_dtype != GRPO_DTYPE_F32)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: dhidden_dtype must be BF16 or F32", who);
+  if (!(eps_low >= 0.f && eps_low < 1.f && eps_high >= 0.f && beta >= 0.f && eps_high < INFINITY &&
+        beta < INFINITY))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: need 0 <= eps_low < 1, finite eps_high, beta >= 0", who);
+
+  const int64_t chunk = chunk_of(n_rows, V, chunk_rows);
+  const WsLayout L =
+      ws_layout(n_rows, V, D, chunk, dlogits_out == nullptr, row_index != nullptr, true);
+  bool query_only = false;
+  if ((st = workspace_check(ws, ws_bytes, L.total, who, &query_only)) != GRPO_OK || query_only)
+    return st;
+
+  if (!weight || !loss_out || !dweight ||
+      (n_rows > 0 && (!hidden || !y || !old_logp || !ref_logp || !adv || !row_rollout || !dhidden)))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: a required pointer is NULL", who);
+  if (((uintptr_t)hidden | (uintptr_t)weight | (uintptr_t)dlogits_out) % 16 != 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: hidden, weight and dlogits_out must be 16-byte aligned",
+                who);
+  cudaStream_t s = as_stream(stream);
+  char* wsb = static_cast<char*>(ws);
+  float4* rowsc = reinterpret_cast<float4*>(wsb + L.rowsc);
+  double* row_loss = row_loss_out ? row_loss_out : reinterpret_cast<double*>(wsb + L.row_loss);
+  __nv_bfloat16* dl_buf = dlogits_out ? static_cast<__nv_bfloat16*>(dlogits_out)
+                                      : reinterpret_cast<__nv_bfloat16*>(wsb + L.dl);
+  void* lt_ws = wsb + L.lt;
+  const int64_t ldd = padded_v(V);
+  const size_t dh_elem = dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+
+  if (n_rows == 0) {
+    cudaError_t e = cudaMemsetAsync(loss_out, 0, sizeof(double), s);
+    if (e == cudaSuccess && !accumulate_dweight)
+      e = cudaMemsetAsync(dweight, 0, (size_t)V * D * sizeof(float), s);
+    if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+    return GRPO_OK;
+  }
+
+  // Gather (with row_index) and pass 1: softmax statistics of every row.
+  Front f;
+  if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, old_logp,
+                  ref_logp, status, wsb, L, s, &f)) != GRPO_OK)
+    return st;
+
+  // Row scalars (Eqs. 1-3) and the loss.
+  RowArgs ra = {};
+  ra.rows = (int32_t)n_rows;
+  ra.J = f.J;
+  ra.V = V;
+  ra.part = f.ta.part;
+  ra.zy = f.ta.zy;
+  ra.y = f.y;
+  ra.old_logp = f.old_logp;
+  ra.ref_logp = f.ref_logp;
+  ra.adv = adv;
+  ra.row_rollout = row_rollout;
+  ra.seq_off = seq_off;
+  ra.beta = beta;
+  // Clip bounds as the fused loss uses them: rho < lo_up <=> rho < 1 - eps_low in exact arithmetic.
+  const double lo = 1.0 - (double)eps_low, hi = 1.0 + (double)eps_high;
+  ra.lo_rn = (float)lo;
+  ra.hi_rn = (float)hi;
+  ra.lo_up = ((double)ra.lo_rn < lo) ? std::nextafter(ra.lo_rn, INFINITY) : ra.lo_rn;
+  ra.hi_dn = ((double)ra.hi_rn > hi) ? std::nextafter(ra.hi_rn, -INFINITY) : ra.hi_rn;
+  ra.agg_mode = agg_mode;
+  ra.inv_denom = agg_mode == 0 ? 1.0 / (double)denom_tokens : 0.0;
+  ra.inv_denom_f = (float)ra.inv_denom;
+  ra.inv_nseq_f = agg_mode == 1 ? (float)(1.0 / (double)n_seq) : 0.f;
+  ra.logp_out = logp_out;
+  ra.row_loss = row_loss;
+  ra.rowsc = rowsc;
+  ra.status = status;
+  lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
+  count_launches(1);
+  if ((st = check_launch(who)) != GRPO_OK) return st;
+  if ((st = launch_sum_rows(row_loss, n_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
+
+  // Pass 2 and the two GEMMs, chunk by chunk.
+  for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
+    const int64_t rows = std::min(chunk, n_rows - c0);
+    const Grid g2 = plan(rows, V, f.n_sm);
+    __nv_bfloat16* dl = dlogits_out ? dl_buf + c0 * ldd : dl_buf;
+    TileArgs tb = f.ta;
+    tb.rows = (int32_t)rows;
+    tb.row0 = (int32_t)c0;
+    tb.n_rb = (int32_t)((rows + BM - 1) / BM);
+    tb.R = g2.R;
+    tb.J = g2.J;
+    tb.y = f.y + c0;
+    tb.part = nullptr;
+    tb.zy = nullptr;
+    tb.rowsc = rowsc + c0;
+    tb.dl = dl;
+    tb.ldd = ldd;
+    if ((st = launch_tiles(true, f.mh, f.mw, tb, g2.grid, s, who)) != GRPO_OK) return st;
+    // dh[c0 : c0 + rows] = dlogits * W   (column-major: dh^T [D x rows] = W^T [D x V] dl^T)
+    if ((st = lt_gemm(s, false, false, D, rows, V, weight, D, dl, ldd,
+                      static_cast<char*>(dhidden) + c0 * D * dh_elem,
+                      dhidden_dtype == GRPO_DTYPE_BF16 ? CUDA_R_16BF : CUDA_R_32F, D, 0.f, lt_ws,
+                      kLtWorkspace, who)) != GRPO_OK)
+      return st;
+    // dW (+)= dlogits^T * h   (column-major: dW^T [D x V] = h^T [D x rows] * dl [rows x V])
+    const float b = (c0 == 0 && !accumulate_dweight) ? 0.f : 1.f;
+    if ((st = lt_gemm(s, false, true, D, V, rows,
+                      static_cast<const char*>(f.hid) + c0 * f.hstride * 2, f.hstride, dl, ldd,
+                      dweight, CUDA_R_32F, D, b, lt_ws, kLtWorkspace, who)) != GRPO_OK)
+      return st;
+  }
+  return GRPO_OK;
+}

@@ -2,6 +2,8 @@
 
     grpo_advantage  ->  grpo_prune  ->  grpo_compact  ->  [host: kept counts, ARS]  ->
     grpo_loss_fwd_bwd over the kept tokens only
+    (or, given hidden states and the output layer's weight instead of logits,
+    grpo_lmhead_loss_fwd_bwd: logits on the tensor cores, dhidden and dweight out)
 
 This mirrors Algorithm 1's order within a step: advantages (Eq. 5), MDAP pruning (Phase 2),
 the ARS update from the kept counts (Phase 1b), then the policy loss over the selected
@@ -37,6 +39,10 @@ class StepParams:
     # "token": Eq. 1's token-level ratio (GRPO, DAPO); "sequence": GSPO's length-normalised
     # sequence ratio, clipped per sequence, with the sequence mean (agg_mode is then unused)
     ratio_level: str = "token"
+    # output-layer mode (hidden states and weight given): dhidden dtype and rows of dlogits held
+    # at a time (0: the library's default)
+    dhidden_dtype: str = "bf16"
+    lmhead_chunk_rows: int = 0
 
 
 class GrpoStep:
@@ -44,15 +50,23 @@ class GrpoStep:
 
     Inputs (device tensors, resident): rewards f32 [P*G], ids i32 [T] (also the sampled tokens y),
     off i64 [P*G+1], logits [T, V] (bf16 or f32, all tokens of all rollouts), old_logp and
-    ref_logp f32 [T].  dlogits are produced for the kept tokens only, in compacted order."""
+    ref_logp f32 [T].  dlogits are produced for the kept tokens only, in compacted order.
+
+    Output-layer mode: pass logits=None with hidden (bf16 [T, D], every token) and weight (bf16
+    [V, D]); the loss is then grpo_lmhead_loss_fwd_bwd over the kept tokens, with dhidden (kept
+    rows, compacted order) and dweight (f32 [V, D]) as its gradients.  It runs host-synced."""
 
     def __init__(self, params: StepParams, rewards, ids, off, logits, old_logp, ref_logp,
-                 ars_total_steps: int = 1, steps_per_epoch: int = 1, G1: int | None = None):
+                 ars_total_steps: int = 1, steps_per_epoch: int = 1, G1: int | None = None,
+                 hidden=None, weight=None):
         import torch
         self.torch = torch
         self.p = params
         self.rewards, self.ids, self.off = rewards, ids, off
         self.logits, self.old, self.ref = logits, old_logp, ref_logp
+        self.hidden, self.weight = hidden, weight
+        if (logits is None) == (hidden is None) or (hidden is None) != (weight is None):
+            raise ValueError("give either logits, or hidden states and the output-layer weight")
         dev = rewards.device
         self.dev = dev
         n = rewards.numel()
@@ -87,6 +101,13 @@ class GrpoStep:
         self.n_next = params.G
         self.T_kept = 0
         self.K = 0
+        if hidden is not None:
+            if params.ratio_level != "token" or params.chunk_rows:
+                raise ValueError("output-layer mode takes the token-level ratio, chunk_rows = 0")
+            dh_t = torch.bfloat16 if params.dhidden_dtype == "bf16" else torch.float32
+            self.dhidden = torch.empty((max(self.T, 1), hidden.shape[1]), dtype=dh_t, device=dev)
+            self.dweight = torch.empty(weight.shape, dtype=torch.float32, device=dev)
+            self.lm_ws = None
         self.set_workspaces()
 
     def _ensure_dlogits(self, rows: int):
@@ -124,6 +145,8 @@ class GrpoStep:
 
     def loss_step(self):
         p = self.p
+        if self.hidden is not None:
+            return self._loss_lmhead()
         if p.ratio_level == "sequence":
             return self._loss_gspo()
         if p.chunk_rows > 0:
@@ -136,6 +159,18 @@ class GrpoStep:
             denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
             dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp, loss_out=self.loss, status=self.status,
             ws=self.loss_ws)
+
+    def _loss_lmhead(self):
+        """The output layer fused with the token loss over the kept rows (gathered by src_token)."""
+        p = self.p
+        out = B.grpo_lmhead_loss_fwd_bwd(
+            self.hidden, self.weight, self.ids, self.old, self.ref, self.adv, self.token_rollout,
+            row_index=self.src_token, n_rows=self.T_kept, eps_low=p.eps_low, eps_high=p.eps_high,
+            beta=p.beta, agg_mode=p.agg_mode, denom_tokens=max(self.T_kept, 1), seq_off=self.off,
+            n_seq=max(self.K, 1), dhidden=self.dhidden, dweight=self.dweight, logp_out=self.logp,
+            loss_out=self.loss, status=self.status, chunk_rows=p.lmhead_chunk_rows, ws=self.lm_ws)
+        self.lm_ws = out["ws"]
+        return out
 
     def _loss_gspo(self):
         """GSPO's sequence-level loss over the kept rollouts: the compaction's kept offsets and
@@ -212,6 +247,8 @@ class GrpoStep:
         torch = self.torch
         if self.p.chunk_rows > 0:
             raise ValueError("graph mode runs the loss in one call (chunk_rows = 0)")
+        if self.hidden is not None:
+            raise ValueError("output-layer mode runs host-synced (its launches are sized by T_kept)")
         self._ensure_dlogits(self.T)
         for _ in range(2):  # warm-up outside capture (kernel attributes, occupancy queries)
             self._enqueue_select()
@@ -278,8 +315,8 @@ class GrpoStep:
 
     def run_from_host(self, host: dict, loss_host=None, overlap_groups: int = 4):
         """One step whose inputs start in host memory (pinned, for asynchronous copies): `host`
-        holds tensors 'rewards', 'ids', 'off', 'old', 'ref' and 'logits' shaped like the device
-        inputs.  The selection inputs and the per-token log-probs are copied whole; after the
+        holds tensors 'rewards', 'ids', 'off', 'old', 'ref' and 'logits' (or, in output-layer
+        mode, 'hidden') shaped like the device inputs.  The selection inputs and the per-token log-probs are copied whole; after the
         selection, only the kept rollouts' logit rows are copied (grpo_upload_kept), since the
         pruned rollouts take no further part in the step (Sec. 3.2).
 
@@ -305,11 +342,14 @@ class GrpoStep:
         self._stream.synchronize()
         self._read_counts()
         n = self.keep.numel()
-        overlap = overlap_groups > 1 and p.chunk_rows == 0 and p.ratio_level == "token"
+        lmhead = self.hidden is not None
+        overlap = (overlap_groups > 1 and p.chunk_rows == 0 and p.ratio_level == "token"
+                   and not lmhead)
         if overlap and self.T_kept > 0:
             h2d += self._upload_and_loss_overlapped(host, overlap_groups)
         else:
-            up, _ = B.grpo_upload_kept(host["logits"], self.logits, self.keep_host[:n], host["off"])
+            key, dst = ("hidden", self.hidden) if lmhead else ("logits", self.logits)
+            up, _ = B.grpo_upload_kept(host[key], dst, self.keep_host[:n], host["off"])
             h2d += up
             if graphed and p.chunk_rows == 0:
                 self.replay_loss()

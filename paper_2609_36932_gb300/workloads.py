@@ -14,6 +14,9 @@ accuracy+format rewards, Sec. 4 and Table 6) are:
   large   16 x G=16, lengths lognormal(median 768) <= 2048, keep ratio 0.25
   long    16 x G=16, lengths lognormal(median 1024) <= 4096, f32 dlogits
 
+For the output layer fused with the loss, the same batches carry hidden states of width 3584
+(Qwen2.5-7B) ~ N(0, 1) and an output-layer weight ~ N(0, 4 / D), both bf16, in place of logits.
+
 Host arrays come from numpy's PCG64 seeded with (seed, stream id); logits come from torch's
 generator on the target device, seeded per block of 256 token rows, so any row range can be
 regenerated on its own.  old_logp and ref_logp are the current log-probability plus Gaussian
@@ -236,6 +239,63 @@ def old_ref_logp(logits, y, noise_old, noise_ref):
     for s in range(0, n, step):
         blk = logits[s:s + step].float()
         center[s:s + step] = blk.gather(1, yt[s:s + step, None])[:, 0] - torch.logsumexp(blk, 1)
+    old = center + torch.as_tensor(np.asarray(noise_old, np.float32), device=dev)
+    ref = center + torch.as_tensor(np.asarray(noise_ref, np.float32), device=dev)
+    return old, ref
+
+
+# Output-layer inputs: a batch's tokens as hidden states of Qwen2.5-7B's width.
+LMHEAD_D = 3584
+
+
+def lmhead_hidden(n_rows: int, D: int, seed: int, device, rows=None):
+    """Hidden states [n, D] ~ N(0, 1) in bf16 (torch's generator on `device`, seeded per block of
+    ROW_BLOCK rows, so any rows can be regenerated on their own).  rows: a range or index array
+    (default: range(n_rows))."""
+    torch = _torch()
+    idx = np.arange(n_rows, dtype=np.int64) if rows is None else (
+        np.arange(rows.start, rows.stop, dtype=np.int64) if isinstance(rows, range)
+        else np.asarray(rows, np.int64))
+    out = torch.empty((idx.size, D), dtype=torch.bfloat16, device=device)
+    for b in np.unique(idx // ROW_BLOCK):
+        g = torch.Generator(device=device)
+        g.manual_seed((int(seed) * 1_000_033 + 104_729 * int(b) + 29) % (2**63))
+        blk = torch.randn((ROW_BLOCK, D), generator=g, device=device).to(torch.bfloat16)
+        sel = np.nonzero(idx // ROW_BLOCK == b)[0]
+        out[torch.from_numpy(sel).to(device)] = blk[torch.from_numpy(idx[sel] - int(b) * ROW_BLOCK).to(device)]
+    return out
+
+
+def lmhead_weight(V: int, D: int, seed: int, device, logit_sd: float = 2.0):
+    """Output-layer weight [V, D] ~ N(0, logit_sd^2 / D) in bf16, so that the logits h W^T of
+    N(0, 1) hidden states have standard deviation about logit_sd (2, like the qwen logits)."""
+    torch = _torch()
+    g = torch.Generator(device=device)
+    g.manual_seed((int(seed) * 7_919 + 3) % (2**63))
+    w = torch.empty((V, D), dtype=torch.bfloat16, device=device)
+    step = 8192
+    for s in range(0, V, step):
+        n = min(step, V - s)
+        w[s:s + n] = (torch.randn((n, D), generator=g, device=device) * (logit_sd / math.sqrt(D))).to(
+            torch.bfloat16)
+    return w
+
+
+def lmhead_old_ref(hidden, weight, y, noise_old, noise_ref):
+    """old_logp / ref_logp for rows of `hidden`: the current log-probability of the sampled token
+    (logits h W^T and torch.logsumexp in f32, block by block) plus the given noise."""
+    torch = _torch()
+    dev = hidden.device
+    n = hidden.shape[0]
+    center = torch.empty(n, dtype=torch.float32, device=dev)
+    yt = torch.as_tensor(np.asarray(y, np.int64), device=dev)
+    wt = weight if dev.type == "cuda" else weight.float()
+    step = 2048
+    for s in range(0, n, step):
+        h = hidden[s:s + step] if dev.type == "cuda" else hidden[s:s + step].float()
+        blk = (h @ wt.t()).float()
+        center[s:s + step] = blk.gather(1, yt[s:s + step, None])[:, 0] - torch.logsumexp(blk, 1)
+        del blk
     old = center + torch.as_tensor(np.asarray(noise_old, np.float32), device=dev)
     ref = center + torch.as_tensor(np.asarray(noise_ref, np.float32), device=dev)
     return old, ref

@@ -218,3 +218,49 @@ def test_ars_closed_loop_of_the_large_group_workload(oracle_mod, grpo):
     seq_l = loop(lambda k, s, e: grpo.adaptive_rollout_count(st, k, s, steps, e))
     assert seq_o == seq_l
     assert all(2 <= n <= w.G for n in seq_o)
+
+
+def lmhead_call(L, n_rows, V, D, ws, ws_bytes, *, stride=None, chunk=0, agg=0, denom=None,
+                beta=0.04, dh_dtype=0, dl=None, ri=None):
+    f = ctypes.c_float
+    L.grpo_lmhead_loss_fwd_bwd.restype = ctypes.c_int32
+    return L.grpo_lmhead_loss_fwd_bwd(
+        None, ctypes.c_int64(D if stride is None else stride), ri, ctypes.c_int64(n_rows), None,
+        ctypes.c_int32(V), ctypes.c_int32(D), None, None, None, None, None, f(0.2), f(0.2),
+        f(beta), ctypes.c_int32(agg), ctypes.c_int64(max(n_rows, 1) if denom is None else denom),
+        None, ctypes.c_int64(0), None, ctypes.c_int32(dh_dtype), None, ctypes.c_int32(0), dl, None,
+        None, None, None, ctypes.c_int64(chunk), ws, ws_bytes, None)
+
+
+def test_lmhead_workspace_query_and_argument_errors(grpo):
+    L = raw()
+    size = ctypes.c_size_t(0)
+    assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size)) == 0
+    full = size.value
+    # per row: 160 partial (max, sum) pairs, z_y, the row scalars and the row loss; one chunk of
+    # bf16 dlogits (1000 rows round up to 1024) and 32 MiB for cuBLASLt
+    def up(x):
+        return (x + 255) // 256 * 256
+    expect = (up(1000 * 160 * 8) + up(1000 * 4) + up(1000 * 16) + up(1000 * 8)
+              + up(1024 * 152064 * 2) + up(32 << 20))
+    assert full == expect
+    assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size), chunk=256) == 0
+    assert size.value == full - up(1024 * 152064 * 2) + up(256 * 152064 * 2)
+    assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size),
+                       dl=ctypes.c_void_p(4096)) == 0
+    assert size.value == full - up(1024 * 152064 * 2)
+    # rows taken through row_index are gathered: D bf16 values and y, old, ref per row
+    assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size),
+                       ri=ctypes.c_void_p(4096)) == 0
+    assert size.value == full + up(1000 * 3584 * 2) + 3 * up(1000 * 4)
+    assert lmhead_call(L, 10, 100, 12, None, ctypes.byref(size)) == 1      # D not a multiple of 8
+    assert lmhead_call(L, 10, 100, 64, None, ctypes.byref(size), stride=60) == 1
+    assert lmhead_call(L, 10, 0, 64, None, ctypes.byref(size)) == 1
+    assert lmhead_call(L, -1, 100, 64, None, ctypes.byref(size)) == 1
+    assert lmhead_call(L, 10, 100, 64, None, ctypes.byref(size), denom=0) == 1
+    assert lmhead_call(L, 10, 100, 64, None, ctypes.byref(size), agg=1) == 1   # needs seq_off
+    assert lmhead_call(L, 10, 100, 64, None, ctypes.byref(size), beta=-1.0) == 1
+    assert lmhead_call(L, 10, 100, 64, None, ctypes.byref(size), dh_dtype=9) == 1
+    # a real call with NULL buffers is refused before any launch
+    big = ctypes.c_size_t(1 << 40)
+    assert lmhead_call(L, 10, 100, 64, ctypes.c_void_p(4096), ctypes.byref(big)) == 1
