@@ -446,10 +446,16 @@ def measured_tensor_peak(sustained):
 
 
 def lmhead_source_hash():
+    """Hash of the output-layer kernels' code (comments and blank lines removed, so that a
+    comment edit does not orphan a profile taken on the same code)."""
+    import re
     h = hashlib.sha256()
     for f in ("lmhead.cu", "rowops.cuh", "common.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f)) as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        h.update("\n".join(ln.rstrip() for ln in text.splitlines() if ln.strip()).encode())
     return h.hexdigest()[:16]
 
 

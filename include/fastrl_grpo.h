@@ -350,6 +350,14 @@ grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
                                  int32_t V, int32_t D, const int32_t* y, float* logp_out,
                                  int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream);
 
+/*
+ * grpo_lmhead_tune — launch settings of the output-layer kernels for this process (no counterpart
+ * in the paper).  prefetch: k-blocks (64 of D) by which an L2 prefetch of each operand tile runs
+ * ahead of its load, 0..64 (0: none).  row_lanes: row blocks the grid works on at once, 1..8, or 0
+ * to let the library choose per launch.  Returns GRPO_ERR_INVALID_ARG for other values.
+ */
+grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes);
+
 /* Row stride, in elements, of grpo_lmhead_loss_fwd_bwd's dlogits_out: V rounded up to a multiple
  * of 32 (0 for V < 1). */
 int64_t grpo_lmhead_dlogits_stride(int32_t V);

@@ -33,7 +33,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
            "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
-           "grpo_lmhead_logp_fwd",
+           "grpo_lmhead_logp_fwd", "grpo_lmhead_tune",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -115,6 +115,8 @@ def lib():
     L.grpo_lmhead_logp_fwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p, _c_p, _c_p,
                                        _c_p, _c_p, _c_p]
     L.grpo_lmhead_logp_fwd.restype = _i32
+    L.grpo_lmhead_tune.argtypes = [_i32, _i32]
+    L.grpo_lmhead_tune.restype = _i32
     L.grpo_lmhead_dlogits_stride.argtypes = [_i32]
     L.grpo_lmhead_dlogits_stride.restype = _i64
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
@@ -374,6 +376,11 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
     wp, size = _ws_args(wst)
     _check(L.grpo_loss_fwd_bwd(*args_head, wp, size, _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
+
+
+def grpo_lmhead_tune(prefetch: int = 0, row_lanes: int = 0):
+    """Launch settings of the output-layer kernels for this process (see the header)."""
+    _check(lib().grpo_lmhead_tune(int(prefetch), int(row_lanes)))
 
 
 def grpo_lmhead_dlogits_stride(V: int) -> int:

@@ -27,7 +27,10 @@
 // Work: CTA c owns row lane i = c % R and vocabulary lane j = c / R; for each group of R row
 // blocks it takes row block g*R + i and the vocabulary tiles j, j + J, j + 2J, ...  At any time
 // the grid works on R consecutive row blocks and J consecutive vocabulary tiles, which the L2
-// serves to all of it.
+// serves to all of it; the weight streams from DRAM about once per group (R = 6..8, chosen per
+// launch for the fewest idle CTAs).  Pass 2 writes dlogits with streaming stores so that they do
+// not displace the operand tiles in L2.  An L2 prefetch of upcoming tiles (grpo_lmhead_tune) is
+// off by default: on GB300 it made pass 1 about 16% slower.
 //
 // Every wait is bounded (about a second): a wait that runs out sets GRPO_DEVFLAG_TIMEOUT and an
 // abort flag; the roles then stop, the producer waits for its copies in flight and the MMA lane
@@ -106,6 +109,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
 }
+// Bring a tile toward L2 ahead of its load (no shared memory, no completion to wait for).
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -151,6 +161,7 @@ struct TileArgs {
   int32_t rows;   // rows of this launch (a chunk in pass 2); the tensor map's row = row0 + local
   int32_t row0;
   int32_t V, nK, n_vt, n_rb, R, J;
+  int32_t prefetch;  // k-blocks between a tile's L2 prefetch and its load (0: none)
   const int32_t* y;  // [rows]
   // pass 1
   float2* part;  // [rows][J]: (max, sum of exp(z - max) without z_y) of vocabulary lane j
@@ -230,6 +241,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       uint32_t fills = 0;
       bool ok = true;
+      // A second walk over the same (row block, vocabulary tile, k-block) sequence, a.prefetch
+      // fills ahead of the loads, asks L2 for those tiles early.
+      int prb = li, pvt = lj, pkb = 0;
+      auto advance = [&]() {
+        if (++pkb == a.nK) {
+          pkb = 0;
+          pvt += J;
+          if (pvt >= a.n_vt) {
+            pvt = lj;
+            prb += R;
+          }
+        }
+      };
+      for (int k = 0; k < a.prefetch && prb < a.n_rb; ++k) advance();
       for (int rb = li; ok && rb < a.n_rb; rb += R) {
         for (int vt = lj; ok && vt < a.n_vt; vt += J) {
           for (int kb = 0; kb < a.nK; ++kb) {
@@ -244,6 +269,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d(sa, &tm_h, kb * BK, a.row0 + rb * BM, full_bar(st));
             tma_load_2d(sa + kABytes, &tm_w, kb * BK, vt * BN, full_bar(st));
             ++fills;
+            if (a.prefetch > 0 && prb < a.n_rb) {
+              tma_prefetch_2d(&tm_h, pkb * BK, a.row0 + prb * BM);
+              tma_prefetch_2d(&tm_w, pkb * BK, pvt * BN);
+              advance();
+            }
           }
         }
       }
@@ -365,11 +395,11 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (k + 1 >= nvalid) d1 = 0.f;
               pk[k / 2] = pack_bf16x2(make_float2(d0, d1));
             }
-            if (rv) {
+            if (rv) {  // streaming stores: dlogits must not push the operand tiles out of L2
               uint4* dst = reinterpret_cast<uint4*>(out_row + v0);
 #pragma unroll
               for (int k = 0; k < 4; ++k)
-                dst[k] = make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+                __stcs(dst + k, make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]));
             }
           }
         }
@@ -539,14 +569,35 @@ int sm_count() {
 struct Grid {
   int R, J, grid;
 };
+// Launch settings of this process (grpo_lmhead_tune): prefetch distance, row lanes (0 = chosen).
+int g_prefetch = 0;
+int g_row_lanes = 0;
+
+// R row lanes x J vocabulary lanes, one CTA per SM at most.  The weight is read from DRAM about
+// once per group of R row blocks, so R stays in [6, 8] (all row blocks when there are fewer);
+// within that, each CTA does ceil(n_rb / R) row blocks x ceil(n_vt / J) tiles while the average
+// is n_rb * n_vt / grid, and R maximises the busy fraction (near-ties go to the larger R)
+//   (n_rb / (ceil(n_rb/R) R)) * (n_vt / (ceil(n_vt/J) J)) * (R J / n_sm).
 Grid plan(int64_t rows, int V, int n_sm) {
   const int n_rb = (int)((rows + BM - 1) / BM);
   const int n_vt = (V + BN - 1) / BN;
-  Grid g;
-  g.R = std::max(1, std::min(n_rb, kRowLanes));
-  g.J = std::max(1, std::min({n_vt, std::max(1, n_sm / g.R), kMaxJ}));
-  g.grid = g.R * g.J;
-  return g;
+  Grid best = {1, 1, 1};
+  double best_u = -1.0;
+  const int r_hi = g_row_lanes > 0 ? g_row_lanes : kRowLanes;
+  const int r_lo = g_row_lanes > 0 ? g_row_lanes : std::min(kRowLanes, std::max(1, std::min(n_rb, 6)));
+  for (int R = r_hi; R >= r_lo; --R) {
+    const int Rr = std::max(1, std::min(n_rb, R));
+    const int J = std::max(1, std::min({n_vt, std::max(1, n_sm / Rr), kMaxJ}));
+    const double groups = (double)((n_rb + Rr - 1) / Rr);
+    const double per_cta_tiles = (double)((n_vt + J - 1) / J);
+    const double u = ((double)n_rb / (groups * Rr)) * ((double)n_vt / (per_cta_tiles * J)) *
+                     ((double)(Rr * J) / (double)std::max(n_sm, 1));
+    if (u > best_u * 1.005) {  // visited from the largest R: near-ties keep the larger
+      best_u = u;
+      best = {Rr, J, Rr * J};
+    }
+  }
+  return best;
 }
 
 grpo_status launch_tiles(bool bwd, const CUtensorMap& mh, const CUtensorMap& mw,
@@ -743,6 +794,7 @@ grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
   ta.n_rb = (int32_t)((n_rows + BM - 1) / BM);
   ta.R = g1.R;
   ta.J = g1.J;
+  ta.prefetch = g_prefetch;
   ta.y = f->y;
   ta.part = reinterpret_cast<float2*>(wsb + L.part);
   ta.zy = reinterpret_cast<float*>(wsb + L.zy);
@@ -751,6 +803,16 @@ grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
 }
 
 }  // namespace
+
+extern "C" grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes) {
+  clear_error();
+  if (prefetch < 0 || prefetch > 64 || row_lanes < 0 || row_lanes > kRowLanes)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_lmhead_tune: prefetch in [0, 64], row_lanes in [0, %d]",
+                kRowLanes);
+  g_prefetch = prefetch;
+  g_row_lanes = row_lanes;
+  return GRPO_OK;
+}
 
 extern "C" int64_t grpo_lmhead_dlogits_stride(int32_t V) { return V >= 1 ? padded_v(V) : 0; }
 
