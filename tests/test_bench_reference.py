@@ -1,6 +1,6 @@
 """bench.py's reference arm (the fp64 oracle on the host cores) on the CPU: one JSON line with the
-keys the bench contract names, for the token-level and GSPO losses; ranks other than 0 print
-nothing and exit 0."""
+keys the bench contract names, for the token-level and GSPO losses and the output layer fused
+with the loss; ranks other than 0 print nothing and exit 0."""
 import json
 import os
 import subprocess
@@ -20,10 +20,11 @@ def run_bench(*args, env=None):
     return [json.loads(l) for l in r.stdout.splitlines() if l.startswith("{")]
 
 
-@pytest.mark.parametrize("loss", ["grpo", "gspo"])
+@pytest.mark.parametrize("loss", ["grpo", "gspo", "lmhead"])
 def test_reference_arm_line(loss):
+    extra = ("--hidden", "64") if loss == "lmhead" else ()
     lines = run_bench("--impl", "reference", "--config", "tiny", "--loss", loss, "--steps", "2",
-                      "--warmup", "1")
+                      "--warmup", "1", *extra)
     assert len(lines) == 1
     d = lines[0]
     for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "higher_is_better",
@@ -34,8 +35,10 @@ def test_reference_arm_line(loss):
     assert d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
-    if loss == "gspo":
-        assert d["config"]["loss"] == "gspo"
+    if loss in ("gspo", "lmhead"):
+        assert d["config"]["loss"] == loss
+    if loss == "lmhead":
+        assert d["config"]["D"] == 64
 
 
 def test_reference_arm_other_ranks_are_silent():
