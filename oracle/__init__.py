@@ -51,6 +51,10 @@ def lib():
                                          _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p,
                                          _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
         L.oracle_lmhead_loss.restype = _i32
+        L.oracle_lmhead_gspo_loss.argtypes = [_c_p, _c_p, _i64, _i32, _i32, _c_p, _c_p, _c_p,
+                                              _c_p, _c_p, _c_p, _i64, _i64, _f32, _f32, _f32,
+                                              _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
+        L.oracle_lmhead_gspo_loss.restype = _i32
         L.oracle_logp.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p]
         L.oracle_logp.restype = _i32
         L.oracle_round_bf16.argtypes = [_f64]
@@ -234,6 +238,44 @@ def lmhead_loss(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *, eps_
                 dlogits=dl, dhidden=dh, dweight=dw, dhidden_abs=dha, dweight_abs=dwa)
 
 
+def lmhead_gspo_loss(hidden, weight, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,
+                     n_seq=None, eps_low=0.2, eps_high=0.2, beta=0.0, want_dlogits=False,
+                     want_dhidden=True, want_dweight=True, want_bounds=False):
+    """The output layer fused with GSPO's sequence-level loss: gspo_loss on z = hidden @ weight.T
+    (sequence k owns rows [seq_row_off[k], seq_row_off[k+1])), then the chain rule.  Returns
+    dict(loss, logp, seq_ratio, seq_loss, and as asked dlogits, dhidden, dweight, *_abs)."""
+    h = np.ascontiguousarray(hidden, dtype=np.float64)
+    w = np.ascontiguousarray(weight, dtype=np.float64)
+    n_rows, D = h.shape
+    V = w.shape[0]
+    so = _arr(seq_row_off, np.int64)
+    K = so.size - 1
+    if n_seq is None:
+        n_seq = K
+
+    def buf(want, shape):
+        return np.empty(shape, np.float64) if want else None
+
+    dl = buf(want_dlogits, (n_rows, V))
+    dh = buf(want_dhidden, (n_rows, D))
+    dw = buf(want_dweight, (V, D))
+    dha = buf(want_bounds and want_dhidden, (n_rows, D))
+    dwa = buf(want_bounds and want_dweight, (V, D))
+    lp = np.empty(max(n_rows, 1), np.float64)
+    sr = np.empty(max(K, 1), np.float64)
+    sl = np.empty(max(K, 1), np.float64)
+    total = np.zeros(1, np.float64)
+    rc = lib().oracle_lmhead_gspo_loss(
+        _p(h), _p(w), n_rows, V, D, _p(_arr(y, np.int32)), _p(_arr(old_logp, np.float32)),
+        _p(_arr(ref_logp, np.float32)), _p(_arr(adv, np.float32)),
+        _p(_arr(seq_rollout, np.int32)), _p(so), K, int(n_seq), float(eps_low), float(eps_high),
+        float(beta), _p(dl), _p(lp), _p(sr), _p(sl), _p(total), _p(dh), _p(dw), _p(dha), _p(dwa))
+    if rc != 0:
+        raise ValueError("oracle_lmhead_gspo_loss: bad arguments")
+    return dict(loss=float(total[0]), logp=lp[:n_rows], seq_ratio=sr[:K], seq_loss=sl[:K],
+                dlogits=dl, dhidden=dh, dweight=dw, dhidden_abs=dha, dweight_abs=dwa)
+
+
 def gspo_loss(logits, V: int, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,
               n_seq=None, eps_low=0.2, eps_high=0.2, beta=0.0, row_index=None, row_stride=None,
               logits_dtype=None, dlogits_dtype=0, want_f64=False, want_dlogits=True):
@@ -246,6 +288,8 @@ def gspo_loss(logits, V: int, y, old_logp, ref_logp, adv, seq_rollout, seq_row_o
         logits_dtype = 1 if lg.dtype == np.uint16 else 0
     if logits_dtype == 0:
         lg = lg.astype(np.float32, copy=False)
+    elif logits_dtype == 2:
+        lg = lg.astype(np.float64, copy=False)
     stride = V if row_stride is None else int(row_stride)
     ri = None if row_index is None else _arr(row_index, np.int64)
     so = _arr(seq_row_off, np.int64)

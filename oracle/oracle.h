@@ -84,6 +84,17 @@ int oracle_lmhead_loss(const double* hidden, const double* weight, int64_t n_row
                        double* loss_out, double* dhidden, double* dweight, double* dhidden_abs,
                        double* dweight_abs);
 
+/* The same with GSPO's sequence-level ratio: oracle_gspo_loss on z = hidden * weight^T (sequences
+ * as oracle_gspo_loss takes them, over the n_rows rows), then the chain rule.  Nullable outputs. */
+int oracle_lmhead_gspo_loss(const double* hidden, const double* weight, int64_t n_rows, int V,
+                            int D, const int32_t* y, const float* old_logp, const float* ref_logp,
+                            const float* adv, const int32_t* seq_rollout,
+                            const int64_t* seq_row_off, int64_t n_seq_rows, int64_t n_seq,
+                            float eps_low, float eps_high, float beta, double* dlogits_out,
+                            double* logp_out, double* seq_ratio_out, double* seq_loss_out,
+                            double* loss_out, double* dhidden, double* dweight,
+                            double* dhidden_abs, double* dweight_abs);
+
 /* logp of the sampled token alone (old/reference policy evaluation); NaN for ids outside [0,V). */
 int oracle_logp(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
                 int64_t n_rows, int V, const int32_t* y, double* logp_out);

@@ -1,6 +1,7 @@
 """Pins of the oracle's output layer fused with the GRPO loss (z = h W^T, then Eqs. 1-3, then the
 chain rule): a library matrix product, a hand-worked two-word vocabulary, finite differences of
-the loss with respect to every hidden and weight entry, and invariances of the softmax."""
+the loss with respect to every hidden and weight entry, and invariances of the softmax; and the
+same for GSPO's sequence-level ratio."""
 import math
 
 import numpy as np
@@ -140,3 +141,56 @@ def test_invalid_token_rows_carry_no_gradient(oracle_mod):
     assert math.isnan(out["logp"][2]) and out["row_loss"][2] == 0.0
     np.testing.assert_array_equal(out["dhidden"][2], 0.0)
     assert np.isfinite(out["dweight"]).all()
+
+
+def gspo_problem(rng, lens=(3, 1, 4), V=8, D=5, old_shift=0.0, beta=0.03):
+    T = int(sum(lens))
+    p, kw = problem(rng, T=T, V=V, D=D, n_roll=len(lens), old_shift=old_shift, beta=beta)
+    so = np.r_[0, np.cumsum(lens)].astype(np.int64)
+    return p, so, dict(beta=beta, eps_low=0.2, eps_high=0.28)
+
+
+def run_gspo(oracle_mod, p, so, kw, **extra):
+    return oracle_mod.lmhead_gspo_loss(p["hidden"], p["weight"], p["y"], p["old_logp"],
+                                       p["ref_logp"], p["adv"], np.arange(len(so) - 1), so,
+                                       **kw, **extra)
+
+
+def test_gspo_logits_feed_the_gspo_loss(oracle_mod):
+    rng = np.random.default_rng(11)
+    p, so, kw = gspo_problem(rng)
+    out = run_gspo(oracle_mod, p, so, kw, want_dlogits=True)
+    z = np.matmul(p["hidden"], p["weight"].T)
+    ref = oracle_mod.gspo_loss(z, z.shape[1], p["y"], p["old_logp"], p["ref_logp"], p["adv"],
+                               np.arange(len(so) - 1), so, logits_dtype=2, want_f64=True, **kw)
+    np.testing.assert_allclose(out["logp"], ref["logp"], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(out["seq_ratio"], ref["seq_ratio"], rtol=1e-12)
+    np.testing.assert_allclose(out["dlogits"], ref["dlogits_f64"], rtol=1e-11, atol=1e-15)
+    assert out["loss"] == pytest.approx(ref["loss"], rel=1e-12, abs=1e-15)
+
+
+@pytest.mark.parametrize("case", ["inside the clip range", "clipped sequences"])
+def test_gspo_gradients_are_the_derivatives_of_the_loss(oracle_mod, case):
+    rng = np.random.default_rng(12 if case == "inside the clip range" else 13)
+    p, so, kw = gspo_problem(rng, old_shift=0.0 if case == "inside the clip range" else -0.5)
+    if case == "clipped sequences":
+        p["adv"] = np.array([0.9, -0.7, 1.3], np.float32)
+    out = run_gspo(oracle_mod, p, so, kw)
+    s_k = out["seq_ratio"]
+    assert np.min(np.abs(s_k - 0.8)) > 1e-3 and np.min(np.abs(s_k - 1.28)) > 1e-3
+    if case == "clipped sequences":
+        assert (s_k > 1.28).any()
+
+    def loss_of(key, idx, step):
+        q = {k: (v.copy() if isinstance(v, np.ndarray) else v) for k, v in p.items()}
+        q[key] = q[key].astype(np.float64)
+        q[key][idx] += step
+        return run_gspo(oracle_mod, q, so, kw, want_dhidden=False, want_dweight=False)["loss"]
+
+    T, D = p["hidden"].shape
+    V = p["weight"].shape[0]
+    h = 1e-6
+    for key, shape, grad in (("hidden", (T, D), out["dhidden"]), ("weight", (V, D), out["dweight"])):
+        for idx in np.ndindex(*shape):
+            fd = (loss_of(key, idx, h) - loss_of(key, idx, -h)) / (2 * h)
+            assert grad[idx] == pytest.approx(fd, rel=1e-6, abs=1e-9), (key, idx)
