@@ -14,7 +14,8 @@
  *     (_dev: counts read on the device, for CUDA graphs)
  *   grpo_lmhead_loss_fwd_bwd  the output layer fused with the loss:     (Sec. 3.2, Eqs. 1-3)
  *                           logits on the tensor cores, never stored whole; dhidden, dweight
- *     (grpo_lmhead_logp_fwd: log-probabilities alone from hidden states)
+ *     (grpo_lmhead_logp_fwd: log-probabilities alone from hidden states;
+ *      grpo_lmhead_gspo_loss_fwd_bwd: the same with GSPO's sequence-level loss)
  *   grpo_upload_kept        host-to-device copy of the kept rows only  (Sec. 3.2)
  *   adaptive_rollout_count  adaptive rollout sampling, on the host     (Eqs. 10-14, Algorithm 1)
  *
@@ -349,6 +350,33 @@ grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
                                  const int64_t* row_index, int64_t n_rows, const void* weight,
                                  int32_t V, int32_t D, const int32_t* y, float* logp_out,
                                  int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream);
+
+/*
+ * grpo_lmhead_gspo_loss_fwd_bwd — the output layer fused with GSPO's sequence-level loss (FastRL on
+ * GSPO, Sec. 1, Sec. 4): the objective of grpo_gspo_loss_fwd_bwd on z = hidden * weight^T, with
+ * dhidden and dweight by the chain rule as in grpo_lmhead_loss_fwd_bwd.
+ * hidden, hidden_stride, row_index, n_rows, weight, V, D, y, old_logp, ref_logp, dhidden,
+ *   dhidden_dtype, dweight, accumulate_dweight, dlogits_out, status, chunk_rows: as
+ *   grpo_lmhead_loss_fwd_bwd.
+ * Sequences: seq_row_off device i64 [n_seq_rows+1] (row offsets in row order t, clamped to
+ *   [0, n_rows]) and seq_rollout device i32 [n_seq_rows] (indices into adv), for instance
+ *   grpo_compact's kept_off and kept_idx; the loss is the mean over n_seq > 0 sequences.
+ * logp_out: device f32 [n_rows], required.  seq_ratio_out: nullable f32 [n_seq_rows] (NaN for a
+ *   sequence with an invalid token or no rows).  loss_out: device f64 [1].
+ * With no rows or no sequences the loss is 0 and dhidden (and dweight unless accumulated) are 0.
+ * Kernels: pass 1, a row kernel (logp and softmax statistics), one warp per sequence (ratio, clip,
+ *   loss term, row gradient scalars), the fixed-order sum, then pass 2 and the two GEMMs.
+ * Workspace: as grpo_lmhead_loss_fwd_bwd, with 16 bytes per row and 8 per sequence in place of the
+ *   per-row loss terms.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
+ */
+grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
+    const void* hidden, int64_t hidden_stride, const int64_t* row_index, int64_t n_rows,
+    const void* weight, int32_t V, int32_t D, const int32_t* y, const float* old_logp,
+    const float* ref_logp, const float* adv, const int32_t* seq_rollout,
+    const int64_t* seq_row_off, int32_t n_seq_rows, int64_t n_seq, float eps_low, float eps_high,
+    float beta, void* dhidden, int32_t dhidden_dtype, float* dweight, int32_t accumulate_dweight,
+    void* dlogits_out, float* logp_out, float* seq_ratio_out, double* loss_out, int32_t* status,
+    int64_t chunk_rows, void* ws, size_t* ws_bytes, grpo_stream_t stream);
 
 /*
  * grpo_lmhead_tune — launch settings of the output-layer kernels for this process (no counterpart

@@ -33,7 +33,7 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
 EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
            "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
-           "grpo_lmhead_logp_fwd", "grpo_lmhead_tune",
+           "grpo_lmhead_logp_fwd", "grpo_lmhead_tune", "grpo_lmhead_gspo_loss_fwd_bwd",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
 
 
@@ -115,6 +115,11 @@ def lib():
     L.grpo_lmhead_logp_fwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p, _c_p, _c_p,
                                        _c_p, _c_p, _c_p]
     L.grpo_lmhead_logp_fwd.restype = _i32
+    L.grpo_lmhead_gspo_loss_fwd_bwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p,
+                                                _c_p, _c_p, _c_p, _c_p, _c_p, _i32, _i64, _f32,
+                                                _f32, _f32, _c_p, _i32, _c_p, _i32, _c_p, _c_p,
+                                                _c_p, _c_p, _c_p, _i64, _c_p, _c_p, _c_p]
+    L.grpo_lmhead_gspo_loss_fwd_bwd.restype = _i32
     L.grpo_lmhead_tune.argtypes = [_i32, _i32]
     L.grpo_lmhead_tune.restype = _i32
     L.grpo_lmhead_dlogits_stride.argtypes = [_i32]
@@ -417,6 +422,91 @@ def grpo_lmhead_logp_fwd(hidden, weight, y, *, row_index=None, n_rows: int | Non
     wp, size = _ws_args(wst)
     _check(L.grpo_lmhead_logp_fwd(*head, wp, size, _stream(stream)))
     return dict(logp=logp_out, ws=wst)
+
+
+def _lmhead_common(hidden, weight, row_index, n_rows, dhidden, dhidden_dtype, dweight,
+                   dlogits_out):
+    torch = _torch()
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise TypeError("hidden and weight must be bf16")
+    if not (hidden.is_cuda and weight.is_cuda):
+        raise TypeError("hidden and weight must be CUDA tensors")
+    if hidden.dim() != 2 or hidden.stride(1) != 1:
+        raise ValueError("hidden must be 2-D with unit stride along D")
+    if weight.dim() != 2 or not weight.is_contiguous() or weight.shape[1] != hidden.shape[1]:
+        raise ValueError("weight must be a contiguous [V, D] tensor")
+    D = hidden.shape[1]
+    V = weight.shape[0]
+    if n_rows is None:
+        n_rows = row_index.numel() if row_index is not None else hidden.shape[0]
+    if row_index is not None:
+        _need(row_index, torch.int64, n_rows, "row_index")
+    dev = hidden.device
+    if dhidden_dtype is None:
+        dhidden_dtype = dhidden.dtype if dhidden is not None else torch.bfloat16
+    if dhidden_dtype in (torch.bfloat16, "bf16"):
+        dht, ht = GRPO_DTYPE_BF16, torch.bfloat16
+    elif dhidden_dtype in (torch.float32, "f32"):
+        dht, ht = GRPO_DTYPE_F32, torch.float32
+    else:
+        raise TypeError("dhidden must be bf16 or f32")
+    if dhidden is None:
+        dhidden = torch.empty((max(int(n_rows), 1), D), dtype=ht, device=dev)
+    _need(dhidden, ht, n_rows * D, "dhidden")
+    if dweight is None:
+        dweight = torch.empty((V, D), dtype=torch.float32, device=dev)
+    _need(dweight, torch.float32, V * D, "dweight")
+    if dlogits_out is not None:
+        _need(dlogits_out, torch.bfloat16, n_rows * grpo_lmhead_dlogits_stride(V), "dlogits_out")
+    return int(n_rows), V, D, dht, dhidden, dweight
+
+
+def grpo_lmhead_gspo_loss_fwd_bwd(hidden, weight, y, old_logp, ref_logp, adv, seq_rollout,
+                                  seq_row_off, *, n_seq_rows: int | None = None,
+                                  n_seq: int | None = None, eps_low: float = 0.2,
+                                  eps_high: float = 0.2, beta: float = 0.0, dhidden=None,
+                                  dhidden_dtype=None, dweight=None,
+                                  accumulate_dweight: bool = False, dlogits_out=None,
+                                  logp_out=None, seq_ratio_out=None, loss_out=None, status=None,
+                                  chunk_rows: int = 0, row_index=None, n_rows: int | None = None,
+                                  ws=None, stream=None):
+    """The output layer fused with GSPO's sequence-level loss (see the header).  seq_row_off /
+    seq_rollout: device i64 [K+1] / i32 [K] over the rows in order.  Returns dict(loss, dhidden,
+    dweight, logp, seq_ratio, dlogits)."""
+    torch = _torch()
+    n_rows, V, D, dht, dhidden, dweight = _lmhead_common(hidden, weight, row_index, n_rows,
+                                                         dhidden, dhidden_dtype, dweight,
+                                                         dlogits_out)
+    dev = hidden.device
+    if n_seq_rows is None:
+        n_seq_rows = seq_rollout.numel()
+    if n_seq is None:
+        n_seq = max(int(n_seq_rows), 1)
+    _need(seq_rollout, torch.int32, n_seq_rows, "seq_rollout")
+    _need(seq_row_off, torch.int64, n_seq_rows + 1, "seq_row_off")
+    _need(adv, torch.float32, None, "adv")
+    n_src = None if row_index is not None else n_rows
+    _need(y, torch.int32, n_src, "y")
+    _need(old_logp, torch.float32, n_src, "old_logp")
+    _need(ref_logp, torch.float32, n_src, "ref_logp")
+    if logp_out is None:
+        logp_out = torch.empty(max(n_rows, 1), dtype=torch.float32, device=dev)
+    if loss_out is None:
+        loss_out = torch.empty(1, dtype=torch.float64, device=dev)
+    L = lib()
+    head = (_ptr(hidden), int(hidden.stride(0)), _ptr(row_index), n_rows, _ptr(weight), V, D,
+            _ptr(y), _ptr(old_logp), _ptr(ref_logp), _ptr(adv), _ptr(seq_rollout),
+            _ptr(seq_row_off), int(n_seq_rows), int(n_seq), float(eps_low), float(eps_high),
+            float(beta), _ptr(dhidden), dht, _ptr(dweight), 1 if accumulate_dweight else 0,
+            _ptr(dlogits_out), _ptr(logp_out), _ptr(seq_ratio_out), _ptr(loss_out), _ptr(status),
+            int(chunk_rows))
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_lmhead_gspo_loss_fwd_bwd(*head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, dev, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_lmhead_gspo_loss_fwd_bwd(*head, wp, size, _stream(stream)))
+    return dict(loss=loss_out, dhidden=dhidden, dweight=dweight, logp=logp_out,
+                seq_ratio=seq_ratio_out, dlogits=dlogits_out, ws=wst)
 
 
 def grpo_lmhead_loss_fwd_bwd(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *,

@@ -438,7 +438,10 @@ struct RowArgs {
   double* row_loss;
   float4* rowsc;
   int32_t* status;
-  int32_t logp_only;  // forward entry: logp_out alone
+  // 0: the token loss (row_loss, rowsc); 1: logp_out alone; 2: logp_out and the softmax
+  // statistics {M, S, S without y, 0} in stats, for GSPO's sequence kernel
+  int32_t mode;
+  float4* stats;
 };
 
 // One thread per row: combine the J partial sums and apply Eqs. 1-3 (the same arithmetic as the
@@ -449,7 +452,7 @@ __global__ void __launch_bounds__(256) lmhead_rows_kernel(const RowArgs a) {
   const int yv = a.y[t];
   if (yv < 0 || yv >= a.V) {
     if (a.logp_out) a.logp_out[t] = __int_as_float(0x7fc00000);
-    if (!a.logp_only) {
+    if (a.mode == 0) {
       a.row_loss[t] = 0.0;
       a.rowsc[t] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
@@ -467,8 +470,9 @@ __global__ void __launch_bounds__(256) lmhead_rows_kernel(const RowArgs a) {
   const float zy = a.zy[t];
   const float S = S_excl + expf(zy - M);
   const float logp = (zy - M) - logf(S);
-  if (a.logp_only) {
+  if (a.mode != 0) {
     a.logp_out[t] = logp;
+    if (a.mode == 2) a.stats[t] = make_float4(M, S, S_excl, 0.f);
     if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
     return;
   }
@@ -501,6 +505,89 @@ __global__ void __launch_bounds__(256) lmhead_rows_kernel(const RowArgs a) {
   if (a.logp_out) a.logp_out[t] = logp;
   a.row_loss[t] = (a.agg_mode == 0 ? a.inv_denom : (double)w) * (double)ell;
   if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
+}
+
+struct SeqArgs {
+  const float* logp;  // rows in order (after any gather)
+  const float* old_logp;
+  const float* ref_logp;
+  const float* adv;
+  const int32_t* seq_rollout;
+  const int64_t* seq_row_off;
+  int32_t n_seq_rows;
+  int64_t n_rows;
+  double lo, hi;  // 1 - eps_low, 1 + eps_high
+  float beta;
+  double inv_nseq;
+  const float4* stats;
+  float4* rowsc;
+  double* seq_loss;
+  float* seq_ratio;
+};
+
+constexpr int kSeqWarps = 8;
+
+// GSPO's sequence-level ratio (Sec. 1, Sec. 4: FastRL on GSPO), one warp per sequence k with rows
+// [r0, r1):  log s_k = mean_t(logp_t - old_t), clipped per sequence; the sequence's loss term and
+// each row's gradient scalars for pass 2 (coef_t = w_t g_t turned into {neg_scale, dy, shift} as
+// in lmhead_rows_kernel).  fp64 lane sums combined by a fixed xor tree: the result depends only on
+// the sequence's rows.  A sequence with a non-finite logp (an invalid token) or no rows has no
+// ratio: loss term 0, ratio NaN, zero gradient.
+__global__ void __launch_bounds__(kSeqWarps * 32) lmhead_gspo_seq_kernel(const SeqArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t k = (int64_t)blockIdx.x * kSeqWarps + (threadIdx.x >> 5);
+  if (k >= a.n_seq_rows) return;
+  int64_t r0 = a.seq_row_off[k], r1 = a.seq_row_off[k + 1];
+  r0 = r0 < 0 ? 0 : (r0 > a.n_rows ? a.n_rows : r0);
+  r1 = r1 < r0 ? r0 : (r1 > a.n_rows ? a.n_rows : r1);
+  const int64_t L = r1 - r0;
+  double slr = 0.0, skl = 0.0;
+  int bad = 0;
+  for (int64_t t = r0 + lane; t < r1; t += 32) {
+    const float lp = a.logp[t];
+    if (!isfinite(lp)) bad = 1;
+    slr += (double)lp - (double)a.old_logp[t];
+    const float x = a.ref_logp[t] - lp;
+    skl += (double)(expm1f(x) - x);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    slr += __shfl_xor_sync(0xffffffffu, slr, o);
+    skl += __shfl_xor_sync(0xffffffffu, skl, o);
+    bad |= __shfl_xor_sync(0xffffffffu, bad, o);
+  }
+  if (L == 0 || bad) {
+    for (int64_t t = r0 + lane; t < r1; t += 32) a.rowsc[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (lane == 0) {
+      a.seq_loss[k] = 0.0;
+      if (a.seq_ratio) a.seq_ratio[k] = __int_as_float(0x7fc00000);
+    }
+    return;
+  }
+  const double A = (double)a.adv[a.seq_rollout[k]];
+  const double s = exp(slr / (double)L);
+  const double clipped = fmin(fmax(s, a.lo), a.hi);
+  const double surr = fmin(s * A, clipped * A);
+  const bool c = (A >= 0.0) ? (s <= a.hi) : (s >= a.lo);
+  if (lane == 0) {
+    a.seq_loss[k] = -(surr - (double)a.beta * skl / (double)L) * a.inv_nseq;
+    if (a.seq_ratio) a.seq_ratio[k] = (float)s;
+  }
+  const float w = (float)(a.inv_nseq / (double)L);
+  const float sa = c ? (float)(s * A) : 0.f;
+  for (int64_t t = r0 + lane; t < r1; t += 32) {
+    const float x = a.ref_logp[t] - a.logp[t];
+    const float coef = w * -(sa + a.beta * expm1f(x));
+    const float4 st = a.stats[t];  // {M, S, S without y}
+    float neg_scale = -coef / st.y;
+    const float dy = coef * (st.z / st.y);
+    float shB = -st.x * kLog2e;
+    if (fabsf(neg_scale) >= 0x1p-100f) {
+      shB += kShiftB;
+      neg_scale *= 0x1p-16f;  // 2^-kShiftB
+    }
+    a.rowsc[t] = make_float4(neg_scale, dy, shB, 0.f);
+  }
 }
 
 // Kept rows gathered into a dense block: hidden row src = row_index[t] (16-byte vectors, one CTA
@@ -576,7 +663,9 @@ int g_row_lanes = 0;
 // R row lanes x J vocabulary lanes, one CTA per SM at most.  The weight is read from DRAM about
 // once per group of R row blocks, so R stays in [6, 8] (all row blocks when there are fewer);
 // within that, each CTA does ceil(n_rb / R) row blocks x ceil(n_vt / J) tiles while the average
-// is n_rb * n_vt / grid, and R maximises the busy fraction (near-ties go to the larger R)
+// is n_rb * n_vt / grid, and R maximises the busy fraction; a smaller R must gain more than 2%
+// (fewer row blocks per group means more weight traffic: R = 8 measured 0.8% faster than 6 on
+// 196 row blocks, where the busy fraction favours 6 by 1%)
 //   (n_rb / (ceil(n_rb/R) R)) * (n_vt / (ceil(n_vt/J) J)) * (R J / n_sm).
 Grid plan(int64_t rows, int V, int n_sm) {
   const int n_rb = (int)((rows + BM - 1) / BM);
@@ -592,7 +681,7 @@ Grid plan(int64_t rows, int V, int n_sm) {
     const double per_cta_tiles = (double)((n_vt + J - 1) / J);
     const double u = ((double)n_rb / (groups * Rr)) * ((double)n_vt / (per_cta_tiles * J)) *
                      ((double)(Rr * J) / (double)std::max(n_sm, 1));
-    if (u > best_u * 1.005) {  // visited from the largest R: near-ties keep the larger
+    if (u > best_u * 1.02) {  // visited from the largest R: within 2%, the larger R wins
       best_u = u;
       best = {Rr, J, Rr * J};
     }
@@ -691,10 +780,12 @@ int64_t chunk_of(int64_t n_rows, int32_t V, int64_t chunk_rows) {
 }
 
 struct WsLayout {
-  size_t part, zy, rowsc, row_loss, dl, lt, hid, ys, olds, refs, total;
+  size_t part, zy, rowsc, row_loss, stats, seq_loss, dl, lt, hid, ys, olds, refs, total;
 };
+// loss: the backward buffers; n_seqs >= 0: GSPO's statistics and sequence terms instead of the
+// per-row loss terms.
 WsLayout ws_layout(int64_t n_rows, int32_t V, int32_t D, int64_t chunk, bool own_dl, bool gather,
-                   bool loss) {
+                   bool loss, int64_t n_seqs = -1) {
   WsLayout w;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -706,7 +797,9 @@ WsLayout ws_layout(int64_t n_rows, int32_t V, int32_t D, int64_t chunk, bool own
   w.part = take(n * kMaxJ * sizeof(float2));
   w.zy = take(n * sizeof(float));
   w.rowsc = take(loss ? n * sizeof(float4) : 0);
-  w.row_loss = take(loss ? n * sizeof(double) : 0);
+  w.row_loss = take(loss && n_seqs < 0 ? n * sizeof(double) : 0);
+  w.stats = take(n_seqs >= 0 ? n * sizeof(float4) : 0);
+  w.seq_loss = take(n_seqs >= 0 ? (size_t)std::max<int64_t>(n_seqs, 1) * sizeof(double) : 0);
   w.dl = take(loss && own_dl ? (size_t)chunk * padded_v(V) * 2 : 0);
   w.lt = take(loss ? kLtWorkspace : 0);
   w.hid = take(gather ? n * (size_t)D * 2 : 0);
@@ -802,6 +895,48 @@ grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
   return launch_tiles(false, f->mh, f->mw, ta, g1.grid, s, who);
 }
 
+// Pass 2 and the two GEMMs, chunk by chunk, from each row's gradient scalars (rowsc).
+grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64_t n_rows,
+                     int32_t V, int32_t D, const void* weight, void* dhidden,
+                     int32_t dhidden_dtype, float* dweight, int32_t accumulate_dweight,
+                     void* dlogits_out, __nv_bfloat16* dl_buf, int64_t chunk, void* lt_ws,
+                     cudaStream_t s) {
+  grpo_status st;
+  const int64_t ldd = padded_v(V);
+  const size_t dh_elem = dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+  for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
+    const int64_t rows = std::min(chunk, n_rows - c0);
+    const Grid g2 = plan(rows, V, f.n_sm);
+    __nv_bfloat16* dl = dlogits_out ? dl_buf + c0 * ldd : dl_buf;
+    TileArgs tb = f.ta;
+    tb.rows = (int32_t)rows;
+    tb.row0 = (int32_t)c0;
+    tb.n_rb = (int32_t)((rows + BM - 1) / BM);
+    tb.R = g2.R;
+    tb.J = g2.J;
+    tb.y = f.y + c0;
+    tb.part = nullptr;
+    tb.zy = nullptr;
+    tb.rowsc = rowsc + c0;
+    tb.dl = dl;
+    tb.ldd = ldd;
+    if ((st = launch_tiles(true, f.mh, f.mw, tb, g2.grid, s, who)) != GRPO_OK) return st;
+    // dh[c0 : c0 + rows] = dlogits * W   (column-major: dh^T [D x rows] = W^T [D x V] dl^T)
+    if ((st = lt_gemm(s, false, false, D, rows, V, weight, D, dl, ldd,
+                      static_cast<char*>(dhidden) + c0 * D * dh_elem,
+                      dhidden_dtype == GRPO_DTYPE_BF16 ? CUDA_R_16BF : CUDA_R_32F, D, 0.f, lt_ws,
+                      kLtWorkspace, who)) != GRPO_OK)
+      return st;
+    // dW (+)= dlogits^T * h   (column-major: dW^T [D x V] = h^T [D x rows] * dl [rows x V])
+    const float b = (c0 == 0 && !accumulate_dweight) ? 0.f : 1.f;
+    if ((st = lt_gemm(s, false, true, D, V, rows,
+                      static_cast<const char*>(f.hid) + c0 * f.hstride * 2, f.hstride, dl, ldd,
+                      dweight, CUDA_R_32F, D, b, lt_ws, kLtWorkspace, who)) != GRPO_OK)
+      return st;
+  }
+  return GRPO_OK;
+}
+
 }  // namespace
 
 extern "C" grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes) {
@@ -849,7 +984,7 @@ extern "C" grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_s
   ra.y = f.y;
   ra.logp_out = logp_out;
   ra.status = status;
-  ra.logp_only = 1;
+  ra.mode = 1;
   lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
   count_launches(1);
   return check_launch(who);
@@ -900,8 +1035,6 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
   __nv_bfloat16* dl_buf = dlogits_out ? static_cast<__nv_bfloat16*>(dlogits_out)
                                       : reinterpret_cast<__nv_bfloat16*>(wsb + L.dl);
   void* lt_ws = wsb + L.lt;
-  const int64_t ldd = padded_v(V);
-  const size_t dh_elem = dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
 
   if (n_rows == 0) {
     cudaError_t e = cudaMemsetAsync(loss_out, 0, sizeof(double), s);
@@ -950,36 +1083,108 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
   if ((st = check_launch(who)) != GRPO_OK) return st;
   if ((st = launch_sum_rows(row_loss, n_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
 
-  // Pass 2 and the two GEMMs, chunk by chunk.
-  for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
-    const int64_t rows = std::min(chunk, n_rows - c0);
-    const Grid g2 = plan(rows, V, f.n_sm);
-    __nv_bfloat16* dl = dlogits_out ? dl_buf + c0 * ldd : dl_buf;
-    TileArgs tb = f.ta;
-    tb.rows = (int32_t)rows;
-    tb.row0 = (int32_t)c0;
-    tb.n_rb = (int32_t)((rows + BM - 1) / BM);
-    tb.R = g2.R;
-    tb.J = g2.J;
-    tb.y = f.y + c0;
-    tb.part = nullptr;
-    tb.zy = nullptr;
-    tb.rowsc = rowsc + c0;
-    tb.dl = dl;
-    tb.ldd = ldd;
-    if ((st = launch_tiles(true, f.mh, f.mw, tb, g2.grid, s, who)) != GRPO_OK) return st;
-    // dh[c0 : c0 + rows] = dlogits * W   (column-major: dh^T [D x rows] = W^T [D x V] dl^T)
-    if ((st = lt_gemm(s, false, false, D, rows, V, weight, D, dl, ldd,
-                      static_cast<char*>(dhidden) + c0 * D * dh_elem,
-                      dhidden_dtype == GRPO_DTYPE_BF16 ? CUDA_R_16BF : CUDA_R_32F, D, 0.f, lt_ws,
-                      kLtWorkspace, who)) != GRPO_OK)
-      return st;
-    // dW (+)= dlogits^T * h   (column-major: dW^T [D x V] = h^T [D x rows] * dl [rows x V])
-    const float b = (c0 == 0 && !accumulate_dweight) ? 0.f : 1.f;
-    if ((st = lt_gemm(s, false, true, D, V, rows,
-                      static_cast<const char*>(f.hid) + c0 * f.hstride * 2, f.hstride, dl, ldd,
-                      dweight, CUDA_R_32F, D, b, lt_ws, kLtWorkspace, who)) != GRPO_OK)
-      return st;
+  return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
+                  accumulate_dweight, dlogits_out, dl_buf, chunk, lt_ws, s);
+}
+
+extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
+    const void* hidden, int64_t hidden_stride, const int64_t* row_index, int64_t n_rows,
+    const void* weight, int32_t V, int32_t D, const int32_t* y, const float* old_logp,
+    const float* ref_logp, const float* adv, const int32_t* seq_rollout,
+    const int64_t* seq_row_off, int32_t n_seq_rows, int64_t n_seq, float eps_low, float eps_high,
+    float beta, void* dhidden, int32_t dhidden_dtype, float* dweight, int32_t accumulate_dweight,
+    void* dlogits_out, float* logp_out, float* seq_ratio_out, double* loss_out, int32_t* status,
+    int64_t chunk_rows, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  clear_error();
+  const char* who = "grpo_lmhead_gspo_loss_fwd_bwd";
+  grpo_status st = check_shape(who, n_rows, V, D, hidden_stride);
+  if (st != GRPO_OK) return st;
+  if (n_seq_rows < 0 || n_seq <= 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: n_seq_rows = %d, n_seq = %lld", who, n_seq_rows,
+                (long long)n_seq);
+  if (dhidden_dtype != GRPO_DTYPE_BF16 && dhidden_dtype != GRPO_DTYPE_F32)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: dhidden_dtype must be BF16 or F32", who);
+  if (!(eps_low >= 0.f && eps_low < 1.f && eps_high >= 0.f && beta >= 0.f && eps_high < INFINITY &&
+        beta < INFINITY))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: need 0 <= eps_low < 1, finite eps_high, beta >= 0", who);
+  const int64_t chunk = chunk_of(n_rows, V, chunk_rows);
+  const WsLayout L = ws_layout(n_rows, V, D, chunk, dlogits_out == nullptr, row_index != nullptr,
+                               true, n_seq_rows);
+  bool query_only = false;
+  if ((st = workspace_check(ws, ws_bytes, L.total, who, &query_only)) != GRPO_OK || query_only)
+    return st;
+  if (!weight || !loss_out || !dweight || (n_seq_rows > 0 && (!seq_row_off || !seq_rollout || !adv)) ||
+      (n_rows > 0 && (!hidden || !y || !old_logp || !ref_logp || !dhidden || !logp_out)))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: a required pointer is NULL", who);
+  if (((uintptr_t)hidden | (uintptr_t)weight | (uintptr_t)dlogits_out) % 16 != 0)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: hidden, weight and dlogits_out must be 16-byte aligned",
+                who);
+  cudaStream_t s = as_stream(stream);
+  char* wsb = static_cast<char*>(ws);
+  if (n_rows == 0 || n_seq_rows == 0) {  // no rows or no sequences: loss 0, zero gradients
+    cudaError_t e = cudaMemsetAsync(loss_out, 0, sizeof(double), s);
+    if (e == cudaSuccess && !accumulate_dweight)
+      e = cudaMemsetAsync(dweight, 0, (size_t)V * D * sizeof(float), s);
+    if (e == cudaSuccess && n_rows > 0)
+      e = cudaMemsetAsync(dhidden, 0,
+                          (size_t)n_rows * D * (dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4), s);
+    if (e == cudaSuccess && dlogits_out && n_rows > 0)
+      e = cudaMemsetAsync(dlogits_out, 0, (size_t)n_rows * padded_v(V) * 2, s);
+    if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+    return GRPO_OK;
   }
-  return GRPO_OK;
+  float4* rowsc = reinterpret_cast<float4*>(wsb + L.rowsc);
+  float4* stats = reinterpret_cast<float4*>(wsb + L.stats);
+  double* seq_loss = reinterpret_cast<double*>(wsb + L.seq_loss);
+  __nv_bfloat16* dl_buf = dlogits_out ? static_cast<__nv_bfloat16*>(dlogits_out)
+                                      : reinterpret_cast<__nv_bfloat16*>(wsb + L.dl);
+
+  // Gather (with row_index) and pass 1.
+  Front f;
+  if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, old_logp,
+                  ref_logp, status, wsb, L, s, &f)) != GRPO_OK)
+    return st;
+  // logp and the softmax statistics of every row.
+  RowArgs ra = {};
+  ra.rows = (int32_t)n_rows;
+  ra.J = f.J;
+  ra.V = V;
+  ra.part = f.ta.part;
+  ra.zy = f.ta.zy;
+  ra.y = f.y;
+  ra.logp_out = logp_out;
+  ra.status = status;
+  ra.mode = 2;
+  ra.stats = stats;
+  lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
+  count_launches(1);
+  if ((st = check_launch(who)) != GRPO_OK) return st;
+  // Rows outside every sequence keep zero gradient scalars.
+  cudaError_t e = cudaMemsetAsync(rowsc, 0, (size_t)n_rows * sizeof(float4), s);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: memset: %s", who, cudaGetErrorString(e));
+  // Sequence ratios, loss terms and the rows' gradient scalars.
+  SeqArgs sa = {};
+  sa.logp = logp_out;
+  sa.old_logp = f.old_logp;
+  sa.ref_logp = f.ref_logp;
+  sa.adv = adv;
+  sa.seq_rollout = seq_rollout;
+  sa.seq_row_off = seq_row_off;
+  sa.n_seq_rows = n_seq_rows;
+  sa.n_rows = n_rows;
+  sa.lo = 1.0 - (double)eps_low;
+  sa.hi = 1.0 + (double)eps_high;
+  sa.beta = beta;
+  sa.inv_nseq = 1.0 / (double)n_seq;
+  sa.stats = stats;
+  sa.rowsc = rowsc;
+  sa.seq_loss = seq_loss;
+  sa.seq_ratio = seq_ratio_out;
+  lmhead_gspo_seq_kernel<<<(unsigned)((n_seq_rows + kSeqWarps - 1) / kSeqWarps), kSeqWarps * 32,
+                           0, s>>>(sa);
+  count_launches(1);
+  if ((st = check_launch(who)) != GRPO_OK) return st;
+  if ((st = launch_sum_rows(seq_loss, n_seq_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
+  return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
+                  accumulate_dweight, dlogits_out, dl_buf, chunk, wsb + L.lt, s);
 }

@@ -102,8 +102,8 @@ class GrpoStep:
         self.T_kept = 0
         self.K = 0
         if hidden is not None:
-            if params.ratio_level != "token" or params.chunk_rows:
-                raise ValueError("output-layer mode takes the token-level ratio, chunk_rows = 0")
+            if params.chunk_rows:
+                raise ValueError("output-layer mode chunks through lmhead_chunk_rows, not chunk_rows")
             dh_t = torch.bfloat16 if params.dhidden_dtype == "bf16" else torch.float32
             self.dhidden = torch.empty((max(self.T, 1), hidden.shape[1]), dtype=dh_t, device=dev)
             self.dweight = torch.empty(weight.shape, dtype=torch.float32, device=dev)
@@ -161,8 +161,23 @@ class GrpoStep:
             ws=self.loss_ws)
 
     def _loss_lmhead(self):
-        """The output layer fused with the token loss over the kept rows (gathered by src_token)."""
+        """The output layer fused with the loss over the kept rows (gathered by src_token): the
+        token-level ratio, or with ratio_level "sequence" GSPO's, whose sequences are the kept
+        rollouts (kept_off, kept_idx)."""
         p = self.p
+        if p.ratio_level == "sequence":
+            if getattr(self, "seq_ratio", None) is None:
+                self.seq_ratio = self.torch.empty(max(self.keep.numel(), 1),
+                                                  dtype=self.torch.float32, device=self.dev)
+            out = B.grpo_lmhead_gspo_loss_fwd_bwd(
+                self.hidden, self.weight, self.ids, self.old, self.ref, self.adv, self.kept_idx,
+                self.kept_off, n_seq_rows=self.K, n_seq=max(self.K, 1), eps_low=p.eps_low,
+                eps_high=p.eps_high, beta=p.beta, dhidden=self.dhidden, dweight=self.dweight,
+                logp_out=self.logp, seq_ratio_out=self.seq_ratio, loss_out=self.loss,
+                status=self.status, chunk_rows=p.lmhead_chunk_rows, row_index=self.src_token,
+                n_rows=self.T_kept, ws=self.lm_ws)
+            self.lm_ws = out["ws"]
+            return out
         out = B.grpo_lmhead_loss_fwd_bwd(
             self.hidden, self.weight, self.ids, self.old, self.ref, self.adv, self.token_rollout,
             row_index=self.src_token, n_rows=self.T_kept, eps_low=p.eps_low, eps_high=p.eps_high,

@@ -279,3 +279,142 @@ def test_full_size_step_sampled_rows(grpo, oracle_mod):
     scale = dW.abs().sum(0).double()
     assert bool((col <= 2.0 ** -6 * scale).all())
     assert math.isfinite(float(step.loss.item()))
+
+
+class GspoCase(LmCase):
+    """LmCase rows grouped into sequences (lengths `lens`; rows after the last sequence belong to
+    none), GSPO's clip widths."""
+
+    def __init__(self, seed, lens, V, D, extra_rows=0, bad_rows=(), beta=0.02, old_sd=0.05):
+        T = int(sum(lens)) + extra_rows
+        super().__init__(seed, T, V, D, n_roll=len(lens), beta=beta, eps=(0.2, 0.28),
+                         bad_rows=bad_rows, old_sd=old_sd)
+        self.lens = np.asarray(lens, np.int64)
+        self.so = np.r_[0, np.cumsum(self.lens)].astype(np.int64)
+        # sequence log-ratios near 0, +0.35 or -0.35 in turn: inside the clip range, or clipped
+        # on either side, and far from its edges
+        for k in range(len(lens)):
+            self.old[self.so[k]:self.so[k + 1]] -= (0.0, 0.35, -0.35)[k % 3]
+        self.seq_rollout = np.random.default_rng(seed + 1).permutation(len(lens)).astype(np.int32)
+
+    def oracle(self, oracle_mod):
+        return oracle_mod.lmhead_gspo_loss(self.h, self.w, self.y, self.old, self.ref, self.adv,
+                                           self.seq_rollout, self.so, eps_low=self.eps[0],
+                                           eps_high=self.eps[1], beta=self.beta,
+                                           want_dlogits=True, want_bounds=True)
+
+    def gpu(self, grpo, chunk_rows=0):
+        import torch
+        t = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).cuda().to(dt)
+        K = len(self.lens)
+        ldd = grpo.grpo_lmhead_dlogits_stride(self.V)
+        dl = torch.full((self.T, ldd), float("nan"), dtype=torch.bfloat16, device="cuda")
+        ratio = torch.empty(K, dtype=torch.float32, device="cuda")
+        status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        out = grpo.grpo_lmhead_gspo_loss_fwd_bwd(
+            t(self.h, torch.bfloat16), t(self.w, torch.bfloat16), t(self.y, torch.int32),
+            t(self.old, torch.float32), t(self.ref, torch.float32), t(self.adv, torch.float32),
+            t(self.seq_rollout, torch.int32), t(self.so, torch.int64), eps_low=self.eps[0],
+            eps_high=self.eps[1], beta=self.beta, dlogits_out=dl, seq_ratio_out=ratio,
+            status=status, chunk_rows=chunk_rows)
+        torch.cuda.synchronize()
+        return dict(loss=float(out["loss"].item()), logp=out["logp"][:self.T].cpu().numpy(),
+                    dhidden=out["dhidden"].float().cpu().numpy(),
+                    dweight=out["dweight"].cpu().numpy(), dlogits=dl.float().cpu().numpy(),
+                    seq_ratio=ratio.cpu().numpy(), status=int(status.item()))
+
+
+def check_gspo(case, g, o):
+    # logp is compared on the rows of sequences (the oracle leaves rows in no sequence at 0)
+    valid = (case.y >= 0) & (case.y < case.V) & (np.arange(case.T) < case.so[-1])
+    tol_logp = 2 * case.dz + 1e-5
+    assert np.all(np.abs(g["logp"][valid] - o["logp"][valid]) <= tol_logp[valid])
+    # the ratio of a sequence moves with the mean of its rows' logp errors
+    good = ~np.isnan(o["seq_ratio"])
+    np.testing.assert_array_equal(np.isnan(g["seq_ratio"]), ~good)
+    sr = o["seq_ratio"][good]
+    assert np.min(np.abs(sr - 0.8), initial=1) > 1e-3 and np.min(np.abs(sr - 1.28), initial=1) > 1e-3
+    r_tol = o["seq_ratio"][good] * (tol_logp.max() + 1e-6)
+    assert np.all(np.abs(g["seq_ratio"][good] - o["seq_ratio"][good]) <= r_tol)
+    d = g["dlogits"][:, :case.V].astype(np.float64)
+    tol = np.abs(o["dlogits"]) * (2.0 ** -8 + 4 * case.dz[:, None] + 1e-5) + 2.0 ** -133
+    assert not (np.abs(d - o["dlogits"]) > tol).any()
+    rel = 2.0 ** -8 + 4 * case.dz.max() + 1e-5 + case.V * U
+    assert np.all(np.abs(g["dhidden"] - o["dhidden"]) <=
+                  rel * o["dhidden_abs"] + 2.0 ** -8 * np.abs(o["dhidden"]) + 1e-30)
+    rel = 2.0 ** -8 + 4 * case.dz.max() + 1e-5 + case.T * U
+    assert np.all(np.abs(g["dweight"] - o["dweight"]) <= rel * o["dweight_abs"] + 1e-30)
+    K = len(case.lens)
+    A = np.abs(case.adv[case.seq_rollout])
+    s = np.where(good, o["seq_ratio"], 0)
+    loss_tol = np.sum((s * A * 1.01 + 2 * case.beta) * tol_logp.max()) / K
+    assert abs(g["loss"] - o["loss"]) <= loss_tol + 1e-6 * abs(o["loss"]) + 1e-12
+
+
+@pytest.mark.parametrize("lens,V,D,extra", [((40, 1, 97, 0, 130), 1000, 128, 0),
+                                            ((300, 260), 2000, 256, 37)])
+def test_gspo_parity(grpo, oracle_mod, lens, V, D, extra):
+    # sequences of one row, an empty sequence, a sequence across row blocks, rows in no sequence
+    case = GspoCase(71 + V, lens, V, D, extra_rows=extra)
+    g = case.gpu(grpo)
+    check_gspo(case, g, case.oracle(oracle_mod))
+    if extra:
+        np.testing.assert_array_equal(g["dhidden"][-extra:], 0.0)
+
+
+def test_gspo_invalid_token_sequence_and_chunks(grpo, oracle_mod):
+    case = GspoCase(81, (50, 70, 90), 700, 64, bad_rows=(60,))
+    g = case.gpu(grpo, chunk_rows=128)
+    assert g["status"] & 1
+    o = case.oracle(oracle_mod)
+    assert np.isnan(o["seq_ratio"][1]) and np.isnan(g["seq_ratio"][1])
+    check_gspo(case, g, o)
+    np.testing.assert_array_equal(g["dhidden"][50:120], 0.0)
+
+
+def test_step_with_the_output_layer_and_gspo(grpo, oracle_mod):
+    """GrpoStep in output-layer mode with GSPO's ratio on the small workload's batch: selection,
+    then grpo_lmhead_gspo_loss_fwd_bwd over the kept rollouts as sequences, against the oracle."""
+    import torch
+    from paper_2609_36932_gb300 import workloads
+    from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
+    w = workloads.get("small")
+    D = 128
+    b = workloads.make_batch(w, 3)
+    dev = torch.device("cuda")
+    hid = workloads.lmhead_hidden(b["T"], D, 3, dev)
+    wt = workloads.lmhead_weight(w.V, D, 3, dev)
+    old, ref = workloads.lmhead_old_ref(hid, wt, b["ids"], b["noise_old"], b["noise_ref"])
+    p = StepParams(G=w.G, V=w.V, keep_cap=w.keep_cap, eps_low=3e-4, eps_high=4e-4, beta=0.0,
+                   ratio_level="sequence")
+    step = GrpoStep(p, torch.from_numpy(b["rewards"]).to(dev), torch.from_numpy(b["ids"]).to(dev),
+                    torch.from_numpy(b["off"]).to(dev), None, old, ref, hidden=hid, weight=wt)
+    step.run()
+    torch.cuda.synchronize()
+    adv, _ = oracle_mod.advantage(b["rewards"], w.G)
+    keep, _ = oracle_mod.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau,
+                               w.keep_cap, 1)
+    comp = oracle_mod.compact(keep, b["off"])
+    K, TK = comp["K"], comp["T_kept"]
+    assert (step.K, step.T_kept) == (K, TK)
+    src = comp["src_token"][:TK]
+    o = oracle_mod.lmhead_gspo_loss(hid.float().cpu().numpy()[src], wt.float().cpu().numpy(),
+                                    b["ids"][src], old.cpu().numpy()[src], ref.cpu().numpy()[src],
+                                    adv, comp["kept_idx"][:K], comp["kept_off"][:K + 1],
+                                    eps_low=3e-4, eps_high=4e-4, beta=0.0, want_bounds=True)
+    S = (hid[torch.from_numpy(src).to(dev)].float().abs() @ wt.float().abs().t()).max(1)[0]
+    dz = (D * U * S).cpu().numpy().astype(np.float64)
+    lp = step.logp[:TK].cpu().numpy()
+    assert np.all(np.abs(lp - o["logp"]) <= 2 * dz + 1e-5)
+    # sequences whose ratio sits within the logp error of a clip edge may take either branch
+    s_o = o["seq_ratio"]
+    edge = (np.abs(s_o - (1 - 3e-4)) < 1e-4) | (np.abs(s_o - (1 + 4e-4)) < 1e-4)
+    rows_ok = np.ones(TK, bool)
+    for k in np.flatnonzero(edge):
+        rows_ok[comp["kept_off"][k]:comp["kept_off"][k + 1]] = False
+    dh = step.dhidden[:TK].float().cpu().numpy()
+    rel = 2.0 ** -8 + 4 * dz.max() + 1e-5 + w.V * U
+    tol = rel * o["dhidden_abs"] + 2.0 ** -8 * np.abs(o["dhidden"]) + 1e-30
+    assert np.all((np.abs(dh - o["dhidden"]) <= tol)[rows_ok])
+    if not edge.any():
+        assert abs(float(step.loss.item()) - o["loss"]) <= 1e-4 * abs(o["loss"]) + 1e-9
