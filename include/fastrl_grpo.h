@@ -381,8 +381,8 @@ grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
 /*
  * grpo_lmhead_tune — launch settings of the output-layer kernels for this process (no counterpart
  * in the paper).  prefetch: k-blocks (64 of D) by which an L2 prefetch of each operand tile runs
- * ahead of its load, 0..64 (0: none).  row_lanes: row blocks the grid works on at once, 1..8, or 0
- * to let the library choose per launch.  Returns GRPO_ERR_INVALID_ARG for other values.
+ * ahead of its load, 0..64 (0: none).  row_lanes: pairs of 128-row blocks the grid works on at
+ * once, 1..8, or 0 to let the library choose per launch.  Returns GRPO_ERR_INVALID_ARG for other values.
  */
 grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes);
 

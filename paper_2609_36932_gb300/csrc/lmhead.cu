@@ -17,17 +17,22 @@
 //     dlogits = coef * ([v == y] - softmax(z)_v) written in bf16 to a chunk buffer.
 //   Two plain GEMMs per chunk (cuBLASLt): dh = dlogits * W and dW (+)= dlogits^T * h.
 //
-// Kernel roles (192 threads, one CTA per SM: 197 KB of shared memory, all 512 TMEM columns):
-//   warp 0, one lane: TMA producer, 4 stages of {A: 128 rows x 64 of h, B: 256 rows x 64 of W},
-//     128-byte swizzled;
-//   warp 1: allocates TMEM; one lane issues the MMAs (M = 128, N = 256, K = 16) into one of two
-//     256-column accumulators, so the epilogue of a tile overlaps the MMAs of the next;
-//   warps 2-5: the epilogue, one thread per tile row, reading its row from TMEM 32 columns at a
-//     time (a warp may read only its quarter of the 128 lanes: warp % 4).
-// Work: CTA c owns row lane i = c % R and vocabulary lane j = c / R; for each group of R row
-// blocks it takes row block g*R + i and the vocabulary tiles j, j + J, j + 2J, ...  At any time
-// the grid works on R consecutive row blocks and J consecutive vocabulary tiles, which the L2
-// serves to all of it; the weight streams from DRAM about once per group (R = 6..8, chosen per
+// Kernel roles (320 threads, one CTA per SM: 197 KB of shared memory, all 512 TMEM columns).  A
+// tile is a pair of 128-row blocks of h against 256 vocabulary entries, so each weight stage
+// feeds two row blocks: per FLOP a third fewer bytes land in shared memory than with one row
+// block per tile, which on GB300 made the kernel 5.5% faster (shared-memory traffic, not the
+// tensor core, was its limit), at the price of a single pair of accumulators.
+//   warp 0, one lane: TMA producer, 3 stages of {A0, A1: 128 rows x 64 of h each, B: 256 rows x
+//     64 of W}, 128-byte swizzled;
+//   warp 1: allocates TMEM; one lane issues the MMAs (M = 128, N = 256, K = 16) into two
+//     256-column accumulators, one per row block of the pair;
+//   warps 2-9: the epilogue, one thread per row of one row block (warps 2-5 the first, 6-9 the
+//     second), reading its row from TMEM 32 columns at a time (a warp may read only its quarter of
+//     the 128 lanes: warp % 4).  The next tile's MMAs wait for it to release the accumulators.
+// Work: CTA c owns pair lane i = c % R and vocabulary lane j = c / R; for each group of R row-block
+// pairs it takes pair g*R + i and the vocabulary tiles j, j + J, j + 2J, ...  At any time the grid
+// works on 2R consecutive row blocks and J consecutive vocabulary tiles, which the L2 serves to
+// all of it; the weight streams from DRAM about once per group (R = 4..8 pairs, chosen per
 // launch for the fewest idle CTAs).  Pass 2 writes dlogits with streaming stores so that they do
 // not displace the operand tiles in L2.  An L2 prefetch of upcoming tiles (grpo_lmhead_tune) is
 // off by default: on GB300 it made pass 1 about 16% slower.
@@ -49,16 +54,16 @@
 namespace fastrl {
 namespace {
 
-constexpr int BM = 128;  // rows of h per tile (MMA M; TMEM lanes)
+constexpr int BM = 128;  // rows of h per row block (MMA M; TMEM lanes); two blocks per tile
 constexpr int BN = 256;  // vocabulary entries per tile (MMA N; TMEM columns per accumulator)
 constexpr int BK = 64;   // D per stage: one 128-byte swizzle row of bf16
-constexpr int kStages = 4;
+constexpr int kStages = 3;
 constexpr uint32_t kABytes = BM * BK * 2;
 constexpr uint32_t kBBytes = BN * BK * 2;
-constexpr uint32_t kStageBytes = kABytes + kBBytes;
-constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 2 * BN;
-constexpr int kRowLanes = 8;       // R: row blocks in flight across the grid
+constexpr uint32_t kStageBytes = 2 * kABytes + kBBytes;  // two row blocks share B
+constexpr int kThreads = 320;
+constexpr uint32_t kTmemCols = 2 * BN;  // one accumulator per row block of the pair
+constexpr int kRowLanes = 8;       // R: row-block pairs in flight across the grid
 constexpr int kMaxJ = 160;         // vocabulary lanes (partial sums per row) at most
 constexpr int kBars = 2 * kStages + 5;  // full, empty, acc full x2, acc empty x2, drain
 constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + 8 * kBars + 16;
@@ -162,6 +167,7 @@ struct TileArgs {
   int32_t row0;
   int32_t V, nK, n_vt, n_rb, R, J;
   int32_t prefetch;  // k-blocks between a tile's L2 prefetch and its load (0: none)
+  // n_rb counts row blocks; tiles take them in pairs (2p, 2p + 1)
   const int32_t* y;  // [rows]
   // pass 1
   float2* part;  // [rows][J]: (max, sum of exp(z - max) without z_y) of vocabulary lane j
@@ -198,7 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int k = 0; k < 2; ++k) {
       mbar_init(accf_bar(k), 1);
-      mbar_init(acce_bar(k), 4 * 32);
+      mbar_init(acce_bar(k), 8 * 32);
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -243,6 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       // A second walk over the same (row block, vocabulary tile, k-block) sequence, a.prefetch
       // fills ahead of the loads, asks L2 for those tiles early.
+      const int n_rp = (a.n_rb + 1) / 2;
       int prb = li, pvt = lj, pkb = 0;
       auto advance = [&]() {
         if (++pkb == a.nK) {
@@ -254,8 +261,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       };
-      for (int k = 0; k < a.prefetch && prb < a.n_rb; ++k) advance();
-      for (int rb = li; ok && rb < a.n_rb; rb += R) {
+      for (int k = 0; k < a.prefetch && prb < n_rp; ++k) advance();
+      for (int rp = li; ok && rp < n_rp; rp += R) {
+        const int rb = 2 * rp;
         for (int vt = lj; ok && vt < a.n_vt; vt += J) {
           for (int kb = 0; kb < a.nK; ++kb) {
             const int st = (int)(fills % kStages);
@@ -267,10 +275,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sa = base_s + st * kStageBytes;
             mbar_expect_tx(full_bar(st), kStageBytes);
             tma_load_2d(sa, &tm_h, kb * BK, a.row0 + rb * BM, full_bar(st));
-            tma_load_2d(sa + kABytes, &tm_w, kb * BK, vt * BN, full_bar(st));
+            tma_load_2d(sa + kABytes, &tm_h, kb * BK, a.row0 + (rb + 1) * BM, full_bar(st));
+            tma_load_2d(sa + 2 * kABytes, &tm_w, kb * BK, vt * BN, full_bar(st));
             ++fills;
-            if (a.prefetch > 0 && prb < a.n_rb) {
-              tma_prefetch_2d(&tm_h, pkb * BK, a.row0 + prb * BM);
+            if (a.prefetch > 0 && prb < n_rp) {
+              tma_prefetch_2d(&tm_h, pkb * BK, a.row0 + 2 * prb * BM);
+              tma_prefetch_2d(&tm_h, pkb * BK, a.row0 + (2 * prb + 1) * BM);
               tma_prefetch_2d(&tm_w, pkb * BK, pvt * BN);
               advance();
             }
@@ -287,15 +297,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       uint32_t fills = 0, tiles = 0;
       bool ok = true;
-      for (int rb = li; ok && rb < a.n_rb; rb += R) {
+      const int n_rp = (a.n_rb + 1) / 2;
+      for (int rp = li; ok && rp < n_rp; rp += R) {
         for (int vt = lj; ok && vt < a.n_vt; vt += J) {
-          const uint32_t acc = tiles & 1u;
-          if (!wait_bar(acce_bar(acc), ((tiles >> 1) & 1u) ^ 1u, true)) {
+          // one accumulator pair (256 columns per row block) per tile: wait until the epilogue
+          // has read the previous tile's
+          if (!wait_bar(acce_bar(0), (tiles & 1u) ^ 1u, true)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem + acc * BN;
           for (int kb = 0; kb < a.nK; ++kb) {
             const int st = (int)(fills % kStages);
             if (!wait_bar(full_bar(st), (fills / kStages) & 1u, true)) {
@@ -304,15 +315,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const uint32_t sa = base_s + st * kStageBytes;
-            const uint64_t ad = smem_desc(sa), bd = smem_desc(sa + kABytes);
+            const uint64_t ad0 = smem_desc(sa), ad1 = smem_desc(sa + kABytes);
+            const uint64_t bd = smem_desc(sa + 2 * kABytes);
 #pragma unroll
             for (int k = 0; k < BK / 16; ++k)  // K = 16 per MMA: 32 bytes along the swizzled row
-              tc_mma(d_tmem, ad + 2 * k, bd + 2 * k, (kb | k) != 0 ? 1u : 0u);
+              tc_mma(tmem, ad0 + 2 * k, bd + 2 * k, (kb | k) != 0 ? 1u : 0u);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              tc_mma(tmem + BN, ad1 + 2 * k, bd + 2 * k, (kb | k) != 0 ? 1u : 0u);
             tc_commit(empty_bar(st));  // the stage is free once these MMAs have read it
             ++fills;
           }
           if (!ok) break;
-          tc_commit(accf_bar(acc));
+          tc_commit(accf_bar(0));
           ++tiles;
         }
       }
@@ -323,11 +338,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ---- epilogue: one thread per tile row ----
     const int q = warp & 3;            // TMEM lane quarter this warp may read
-    const int r_in = q * 32 + lane;    // row within the tile
+    const int half = (warp - 2) >> 2;  // which row block (accumulator) of the pair
+    const int r_in = q * 32 + lane;    // row within the row block
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     uint32_t tiles = 0;
     bool ok = true;
-    for (int rb = li; ok && rb < a.n_rb; rb += R) {
+    const int n_rp = (a.n_rb + 1) / 2;
+    for (int rp = li; ok && rp < n_rp; rp += R) {
+      const int rb = 2 * rp + half;
       const int row = rb * BM + r_in;
       const bool rv = row < a.rows;
       const int yv = rv ? a.y[row] : -1;
@@ -337,16 +355,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float neg_scale = sc.x, dy = sc.y, shB = sc.z;
       __nv_bfloat16* out_row = kBwd ? a.dl + (int64_t)(rv ? row : 0) * a.ldd : nullptr;
       for (int vt = lj; vt < a.n_vt; vt += J) {
-        const uint32_t acc = tiles & 1u;
         int got = 0;
-        if (lane == 0) got = wait_bar(accf_bar(acc), (tiles >> 1) & 1u, true) ? 1 : 0;
+        if (lane == 0) got = wait_bar(accf_bar(0), tiles & 1u, true) ? 1 : 0;
         got = __shfl_sync(0xffffffffu, got, 0);
         if (!got) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t taddr = tmem + lane_base + acc * BN;
+        const uint32_t taddr = tmem + lane_base + half * BN;
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
           const int v0 = vt * BN + c;
@@ -404,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         tc_fence_before();
-        mbar_arrive(acce_bar(acc));
+        mbar_arrive(acce_bar(0));
         ++tiles;
       }
       if (!kBwd && ok && rv) a.part[(int64_t)row * J + lj] = make_float2(m, s);
@@ -660,20 +677,19 @@ struct Grid {
 int g_prefetch = 0;
 int g_row_lanes = 0;
 
-// R row lanes x J vocabulary lanes, one CTA per SM at most.  The weight is read from DRAM about
-// once per group of R row blocks, so R stays in [6, 8] (all row blocks when there are fewer);
-// within that, each CTA does ceil(n_rb / R) row blocks x ceil(n_vt / J) tiles while the average
-// is n_rb * n_vt / grid, and R maximises the busy fraction; a smaller R must gain more than 2%
-// (fewer row blocks per group means more weight traffic: R = 8 measured 0.8% faster than 6 on
-// 196 row blocks, where the busy fraction favours 6 by 1%)
-//   (n_rb / (ceil(n_rb/R) R)) * (n_vt / (ceil(n_vt/J) J)) * (R J / n_sm).
+// R pair lanes x J vocabulary lanes, one CTA per SM at most.  The weight is read from DRAM about
+// once per group of R row-block pairs, so R stays in [4, 8] (all pairs when there are fewer);
+// within that, each CTA does ceil(n_pairs / R) pairs x ceil(n_vt / J) tiles while the average is
+// n_pairs * n_vt / grid, and R maximises the busy fraction; a smaller R must gain more than 2%
+// (fewer row blocks per group means more weight traffic)
+//   (n_pairs / (ceil(n_pairs/R) R)) * (n_vt / (ceil(n_vt/J) J)) * (R J / n_sm).
 Grid plan(int64_t rows, int V, int n_sm) {
-  const int n_rb = (int)((rows + BM - 1) / BM);
+  const int n_rb = (int)((rows + 2 * BM - 1) / (2 * BM));  // row-block pairs
   const int n_vt = (V + BN - 1) / BN;
   Grid best = {1, 1, 1};
   double best_u = -1.0;
   const int r_hi = g_row_lanes > 0 ? g_row_lanes : kRowLanes;
-  const int r_lo = g_row_lanes > 0 ? g_row_lanes : std::min(kRowLanes, std::max(1, std::min(n_rb, 6)));
+  const int r_lo = g_row_lanes > 0 ? g_row_lanes : std::min(kRowLanes, std::max(1, std::min(n_rb, 4)));
   for (int R = r_hi; R >= r_lo; --R) {
     const int Rr = std::max(1, std::min(n_rb, R));
     const int J = std::max(1, std::min({n_vt, std::max(1, n_sm / Rr), kMaxJ}));
