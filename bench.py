@@ -54,11 +54,12 @@ def parse():
                     help="override the workload's prompt count (a smaller case for profiling)")
     ap.add_argument("--group", type=int, default=0,
                     help="override the rollouts per prompt G (a smaller case for profiling)")
-    ap.add_argument("--loss", choices=["grpo", "gspo", "lmhead"], default="grpo",
+    ap.add_argument("--loss", choices=["grpo", "gspo", "lmhead", "lmhead-gspo"], default="grpo",
                     help="grpo: Eq. 1's token-level ratio (fused, one pass); gspo: the sequence-level "
                          "ratio of FastRL's GSPO variant (three passes, host-synced); lmhead: the "
                          "output layer fused with the token loss (hidden states in, logits on the "
-                         "tensor cores, dhidden and dweight out)")
+                         "tensor cores, dhidden and dweight out); lmhead-gspo: the same with GSPO's "
+                         "sequence-level loss (clip 3e-4 / 4e-4, beta 0)")
     ap.add_argument("--hidden", type=int, default=0,
                     help="hidden size of the output layer with --loss lmhead (default 3584)")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -485,7 +486,10 @@ def lmhead_inputs(w, D, seed, device):
     return b, d
 
 
-def lmhead_desc(w, D, T, T_kept, K):
+GSPO_LMHEAD = dict(eps_low=3e-4, eps_high=4e-4, beta=0.0)  # GSPO's published clip widths
+
+
+def lmhead_desc(w, D, T, T_kept, K, gspo=False):
     cfg = workload_desc(w, T, T_kept, K)
     cfg["workload"] = ("%s with the output layer: %d prompts x G=%d rollouts, lengths %s, hidden "
                        "size D=%d, V=%d, bf16 hidden states N(0,1) and weight N(0,4/D), rewards %s,"
@@ -496,7 +500,10 @@ def lmhead_desc(w, D, T, T_kept, K):
     cfg["io"] = "bf16 hidden [T_kept, D] and weight [V, D] -> bf16 dhidden, f32 dweight"
     cfg["l2"] = ("inputs larger than L2 (weight %.2f GB, dweight %.2f GB vs 129 MB L2); no flush"
                  % (w.V * D * 2 / 1e9, w.V * D * 4 / 1e9))
-    cfg["loss"] = "lmhead"
+    cfg["loss"] = "lmhead-gspo" if gspo else "lmhead"
+    if gspo:
+        cfg.update(eps_low=GSPO_LMHEAD["eps_low"], eps_high=GSPO_LMHEAD["eps_high"], beta=0.0,
+                   ratio="sequence (GSPO): the kept rollouts are the sequences")
     return cfg
 
 
@@ -522,6 +529,43 @@ def oracle_lmhead_sample(w, b, d, src, rr, T_kept, n, threads=0):
     return t_sel, time.perf_counter() - t1, int(oracle.set_threads(0))
 
 
+def cpu_baseline_lmhead_gspo(w, b, d, step, target_s):
+    """The oracle on a bounded sample: selection on the whole batch, then the output layer and
+    GSPO's loss over the first whole kept sequences."""
+    import torch
+    import oracle
+    cores = int(oracle.set_threads(0))
+    t0 = time.perf_counter()
+    adv, _ = oracle.advantage(b["rewards"], w.G)
+    keep, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
+    comp = oracle.compact(keep, b["off"])
+    t_sel = time.perf_counter() - t0
+    K, T_kept = comp["K"], comp["T_kept"]
+    kept_idx, kept_off, src = comp["kept_idx"][:K], comp["kept_off"][:K + 1], comp["src_token"]
+    w64 = d["weight"].double().cpu().numpy()
+    old, ref = d["old"].cpu().numpy(), d["ref"].cpu().numpy()
+
+    def run(k):
+        rows = src[:int(kept_off[k])]
+        h = d["hidden"][torch.from_numpy(rows).to(d["hidden"].device)].double().cpu().numpy()
+        t = time.perf_counter()
+        oracle.lmhead_gspo_loss(h, w64, b["ids"][rows], old[rows], ref[rows], adv, kept_idx[:k],
+                                kept_off[:k + 1], n_seq=K, **GSPO_LMHEAD)
+        return time.perf_counter() - t, len(rows)
+
+    k = 1
+    t1, r1 = run(k)
+    per_row = max(t1 / max(r1, 1), 1e-6)
+    while k < K and kept_off[k + 1] * per_row <= target_s:
+        k += 1
+    t, rows = run(k)
+    return {"value": 1.0 / (t / max(rows, 1) + t_sel / max(T_kept, 1)), "unit": UNIT,
+            "cores": cores, "kind": "oracle",
+            "sample": "fp64 oracle: advantage+prune+compact on the whole batch (%.2f s, amortised"
+                      " over its %d kept tokens) + output layer and GSPO's loss on the first %d"
+                      " kept sequences (%d rows, %.2f s)" % (t_sel, T_kept, k, rows, t)}
+
+
 def run_lmhead(args, w):
     """--loss lmhead: the step with the output layer fused (GrpoStep in output-layer mode)."""
     import torch
@@ -537,9 +581,14 @@ def run_lmhead(args, w):
     dev = torch.device("cuda", local)
     g.lib()
     D = args.hidden or workloads.LMHEAD_D
+    gspo = args.loss == "lmhead-gspo"
     b, d = lmhead_inputs(w, D, rank_seed(args.seed, rank), dev)
-    p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
-                   eps_low=w.eps, eps_high=w.eps, beta=w.beta)
+    if gspo:
+        p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
+                       ratio_level="sequence", **GSPO_LMHEAD)
+    else:
+        p = StepParams(G=w.G, V=w.V, ngram_n=w.ngram_n, tau=w.tau, keep_cap=w.keep_cap,
+                       eps_low=w.eps, eps_high=w.eps, beta=w.beta)
     step = GrpoStep(p, d["rewards"], d["ids"], d["off"], None, d["old"], d["ref"],
                     hidden=d["hidden"], weight=d["weight"])
     for _ in range(max(args.warmup, 3)):
@@ -651,7 +700,9 @@ def run_lmhead(args, w):
         del host
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and gspo:
+        cpu = cpu_baseline_lmhead_gspo(w, b, d, step, args.cpu_seconds)
+    elif rank == 0 and world == 1 and not args.no_cpu_baseline:
         src, rr = step.kept_rows()
         n0 = min(16, len(src))  # a full row per worker thread for the calibration
         _, tl0, _ = oracle_lmhead_sample(w, b, d, src, rr, T_kept, n0)
@@ -670,7 +721,7 @@ def run_lmhead(args, w):
             "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded; the qwen batch with random-init output layer)",
-            "config": lmhead_desc(w, D, b["T"], T_kept, step.K),
+            "config": lmhead_desc(w, D, b["T"], T_kept, step.K, gspo),
             "gpu_launches": int(launches), "cuda_graph": False,
             "roofline": roofline, "step_tensor": step_tc, "e2e": e2e, "cpu_baseline": cpu,
             "clocks": clocks,
@@ -691,11 +742,14 @@ def run_reference_lmhead(args, w):
     from paper_2609_36932_gb300 import workloads
     import oracle
     D = args.hidden or workloads.LMHEAD_D
+    gspo = args.loss == "lmhead-gspo"
     b = workloads.make_batch(w, args.seed)
     keep, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
     comp = oracle.compact(keep, b["off"])
     T_kept = comp["T_kept"]
     src, rr = comp["src_token"], comp["token_rollout"]
+    K = comp["K"]
+    kept_idx, kept_off = comp["kept_idx"][:K], comp["kept_off"][:K + 1]
     wt = workloads.lmhead_weight(w.V, D, args.seed, "cpu")
     w64 = wt.double().numpy()
 
@@ -712,30 +766,46 @@ def run_reference_lmhead(args, w):
         kp, _ = oracle.prune(b["rewards"], b["ids"], b["off"], w.G, w.ngram_n, w.tau, w.keep_cap, 1)
         oracle.compact(kp, b["off"])
         t1 = time.perf_counter()
-        oracle.lmhead_loss(h, w64, b["ids"][src[:n]], o, r, adv, rr[:n], eps_low=w.eps,
-                           eps_high=w.eps, beta=w.beta, denom_tokens=T_kept)
+        if gspo:  # n counts whole kept sequences
+            oracle.lmhead_gspo_loss(h, w64, b["ids"][src[:kept_off[n]]], o, r, adv, kept_idx[:n],
+                                    kept_off[:n + 1], n_seq=K, **GSPO_LMHEAD)
+        else:
+            oracle.lmhead_loss(h, w64, b["ids"][src[:n]], o, r, adv, rr[:n], eps_low=w.eps,
+                               eps_high=w.eps, beta=w.beta, denom_tokens=T_kept)
         return t1 - t0, time.perf_counter() - t1
 
-    t_sel, t_loss = run(1, sample(1))
+    rows_of = (lambda n: int(kept_off[n])) if gspo else (lambda n: n)
+    first = 1
+    while gspo and first < K and kept_off[first] == 0:
+        first += 1
+    t_sel, t_loss = run(first, sample(rows_of(first)))
     budget = 120.0 / max(args.steps + args.warmup, 1)
-    n = int(max(1, min(len(src), 64, (budget - t_sel) / max(t_loss, 1e-6)))) if budget > t_sel else 1
-    data = sample(n)
+    if gspo:
+        n = first
+        per_row = t_loss / max(rows_of(first), 1)
+        while n < K and rows_of(n + 1) <= 64 and rows_of(n + 1) * per_row + t_sel <= budget:
+            n += 1
+    else:
+        n = int(max(1, min(len(src), 64, (budget - t_sel) / max(t_loss, 1e-6)))) if budget > t_sel else 1
+    data = sample(rows_of(n))
     cores = int(oracle.set_threads(0))
     times = []
     for i in range(args.warmup + args.steps):
         t_sel, t_loss = run(n, data)
         if i >= args.warmup:
-            times.append(t_loss / n + t_sel / T_kept)
+            times.append(t_loss / max(rows_of(n), 1) + t_sel / T_kept)
     value = 1.0 / statistics.mean(times)
+    what = ("GSPO's loss on the first %d kept sequences (%d rows)" % (n, rows_of(n)) if gspo
+            else "loss on the first %d kept rows" % n)
     print(json.dumps({
         "impl": "reference", "metric": LMHEAD_METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": lmhead_desc(w, D, b["T"], T_kept, comp["K"]),
+        "data": "synthetic", "config": lmhead_desc(w, D, b["T"], T_kept, comp["K"], gspo),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                          "sample": "per step: fp64 oracle advantage+prune+compact on the whole batch"
-                                   " (amortised over %d kept tokens) + output layer and loss on the"
-                                   " first %d kept rows" % (T_kept, n)},
+                                   " (amortised over %d kept tokens) + output layer and %s"
+                                   % (T_kept, what)},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
@@ -750,13 +820,13 @@ def main():
     if args.group > 0:
         w = dataclasses.replace(w, G=args.group)
     if args.impl == "reference":
-        if args.loss == "lmhead":
+        if args.loss in ("lmhead", "lmhead-gspo"):
             if dist_env()[0] == 0:
                 run_reference_lmhead(args, w)
             return
         run_reference(args, w)
         return
-    if args.loss == "lmhead":
+    if args.loss in ("lmhead", "lmhead-gspo"):
         run_lmhead(args, w)
         return
     import torch
