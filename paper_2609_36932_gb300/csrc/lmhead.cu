@@ -65,7 +65,9 @@ constexpr int kThreads = 320;
 constexpr uint32_t kTmemCols = 2 * BN;  // one accumulator per row block of the pair
 constexpr int kRowLanes = 8;       // R: row-block pairs in flight across the grid
 constexpr int kMaxJ = 160;         // vocabulary lanes (partial sums per row) at most
-constexpr int kBars = 2 * kStages + 5;  // full, empty, acc full x2, acc empty x2, drain
+// Barriers: full and empty per stage, accumulator-pair full and released (two slots each, the
+// first in use), drain.
+constexpr int kBars = 2 * kStages + 5;
 constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + 8 * kBars + 16;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int64_t kDefaultChunkBytes = 4ll << 30;  // dlogits chunk buffer

@@ -264,3 +264,12 @@ def test_lmhead_workspace_query_and_argument_errors(grpo):
     # a real call with NULL buffers is refused before any launch
     big = ctypes.c_size_t(1 << 40)
     assert lmhead_call(L, 10, 100, 64, ctypes.c_void_p(4096), ctypes.byref(big)) == 1
+
+
+def test_lmhead_tune_rejects_out_of_range_settings(grpo):
+    L = raw()
+    L.grpo_lmhead_tune.restype = ctypes.c_int32
+    assert L.grpo_lmhead_tune(ctypes.c_int32(-1), ctypes.c_int32(0)) == 1
+    assert L.grpo_lmhead_tune(ctypes.c_int32(65), ctypes.c_int32(0)) == 1
+    assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(9)) == 1
+    assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(0)) == 0

@@ -418,3 +418,18 @@ def test_step_with_the_output_layer_and_gspo(grpo, oracle_mod):
     assert np.all((np.abs(dh - o["dhidden"]) <= tol)[rows_ok])
     if not edge.any():
         assert abs(float(step.loss.item()) - o["loss"]) <= 1e-4 * abs(o["loss"]) + 1e-9
+
+
+def test_non_finite_hidden_row_is_flagged(grpo):
+    """A NaN in one row's hidden state makes that row's logits NaN: its logp is NaN and the status
+    word carries GRPO_DEVFLAG_NONFINITE; the other rows' logp are unaffected."""
+    import torch
+    case = LmCase(91, 200, 600, 64)
+    clean = case.gpu(grpo, with_dlogits=False)
+    case.h = case.h.copy()
+    case.h[17, 5] = np.nan
+    g = case.gpu(grpo, with_dlogits=False)
+    assert g["status"] & 2  # GRPO_DEVFLAG_NONFINITE
+    assert np.isnan(g["logp"][17])
+    others = np.arange(case.T) != 17
+    np.testing.assert_array_equal(g["logp"][others], clean["logp"][others])
