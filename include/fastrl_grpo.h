@@ -490,6 +490,22 @@ typedef struct grpo_ars_state {
 grpo_status grpo_ars_init(grpo_ars_state* st, int32_t G1);
 
 /*
+ * grpo_ars_serialize / grpo_ars_deserialize — checkpoint and resume of the ARS state (no
+ * counterpart in the paper, which restarts nothing): a training run that stops mid-epoch resumes
+ * with the same buffered means, G'_ref and G'_t, so the rollout counts continue as if
+ * uninterrupted.  The record is 64 bytes, little-endian on every host: the tag "FRLARS01", then
+ * G1, n, have_ref, have_gt (4 bytes each), g_ref, g_t, buf_mean_sum, buf_max_sum (binary64) and
+ * buf_count (8 bytes).
+ * serialize: buf == NULL writes the size (64) to *bytes; otherwise *bytes >= 64 is required
+ *   (GRPO_ERR_WORKSPACE if smaller) and receives 64.
+ * deserialize: GRPO_ERR_INVALID_ARG (st untouched) for a short buffer, a wrong tag, or a state
+ *   that grpo_ars_init / adaptive_rollout_count cannot produce (G1 < 2, n outside [2, G1], flags
+ *   other than 0 / 1, a negative count, non-finite or negative sums).  Host only.
+ */
+grpo_status grpo_ars_serialize(const grpo_ars_state* st, void* buf, size_t* bytes);
+grpo_status grpo_ars_deserialize(grpo_ars_state* st, const void* buf, size_t bytes);
+
+/*
  * adaptive_rollout_count — ARS update after one step, Eqs. 10-14 and Algorithm 1 (Phases 1a/1b).
  * kept_per_prompt  host i32 [P], P >= 1: |S(q)| of this step.  Their mean and max are buffered
  *                  (Eq. 10).  At an epoch end (epoch_end != 0), with alpha = step/total_steps,

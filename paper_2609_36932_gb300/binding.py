@@ -34,7 +34,8 @@ EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_adva
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
            "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
            "grpo_lmhead_logp_fwd", "grpo_lmhead_tune", "grpo_lmhead_gspo_loss_fwd_bwd",
-           "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count"]
+           "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count",
+           "grpo_ars_serialize", "grpo_ars_deserialize"]
 
 
 class GrpoError(RuntimeError):
@@ -134,6 +135,10 @@ def lib():
     L.grpo_ars_init.restype = _i32
     L.adaptive_rollout_count.argtypes = [ctypes.POINTER(ArsState), _c_p, _i32, _i64, _i64, _i32]
     L.adaptive_rollout_count.restype = _i32
+    L.grpo_ars_serialize.argtypes = [ctypes.POINTER(ArsState), _c_p, ctypes.POINTER(ctypes.c_size_t)]
+    L.grpo_ars_serialize.restype = _i32
+    L.grpo_ars_deserialize.argtypes = [ctypes.POINTER(ArsState), _c_p, ctypes.c_size_t]
+    L.grpo_ars_deserialize.restype = _i32
     _lib = L
     return L
 
@@ -797,6 +802,23 @@ def grpo_sum_f64(v, n: int | None = None, out=None, stream=None):
 def grpo_ars_init(G1: int) -> ArsState:
     st = ArsState()
     _check(lib().grpo_ars_init(ctypes.byref(st), G1))
+    return st
+
+
+def grpo_ars_serialize(state: ArsState) -> bytes:
+    """The ARS state as its 64-byte checkpoint record (see the header)."""
+    n = ctypes.c_size_t(0)
+    _check(lib().grpo_ars_serialize(ctypes.byref(state), None, ctypes.byref(n)))
+    buf = ctypes.create_string_buffer(n.value)
+    _check(lib().grpo_ars_serialize(ctypes.byref(state), buf, ctypes.byref(n)))
+    return buf.raw[:n.value]
+
+
+def grpo_ars_deserialize(record: bytes) -> ArsState:
+    """An ARS state restored from grpo_ars_serialize's record."""
+    st = ArsState()
+    buf = ctypes.create_string_buffer(bytes(record), len(record))
+    _check(lib().grpo_ars_deserialize(ctypes.byref(st), buf, len(record)))
     return st
 
 

@@ -133,3 +133,99 @@ extern "C" int32_t adaptive_rollout_count(grpo_ars_state* st, const int32_t* kep
   st->n = n;
   return n;
 }
+
+// ---- checkpoint / resume of the ARS state ----------------------------------------------------
+// A fixed 64-byte record, little-endian whatever the host: the 8-byte tag "FRLARS01", then G1, n,
+// have_ref, have_gt (4 bytes each) and g_ref, g_t, buf_mean_sum, buf_max_sum (IEEE binary64 bit
+// patterns), buf_count (8 bytes each).  Written and read byte by byte, so a checkpoint moves
+// between x86-64 and aarch64 hosts unchanged.
+
+namespace {
+
+constexpr size_t kArsRecordBytes = 64;
+constexpr char kArsTag[8] = {'F', 'R', 'L', 'A', 'R', 'S', '0', '1'};
+
+void put_u32(unsigned char* p, uint32_t v) {
+  for (int i = 0; i < 4; ++i) p[i] = (unsigned char)(v >> (8 * i));
+}
+void put_u64(unsigned char* p, uint64_t v) {
+  for (int i = 0; i < 8; ++i) p[i] = (unsigned char)(v >> (8 * i));
+}
+uint32_t get_u32(const unsigned char* p) {
+  uint32_t v = 0;
+  for (int i = 0; i < 4; ++i) v |= (uint32_t)p[i] << (8 * i);
+  return v;
+}
+uint64_t get_u64(const unsigned char* p) {
+  uint64_t v = 0;
+  for (int i = 0; i < 8; ++i) v |= (uint64_t)p[i] << (8 * i);
+  return v;
+}
+uint64_t f64_bits(double x) {
+  uint64_t b;
+  std::memcpy(&b, &x, 8);
+  return b;
+}
+double bits_f64(uint64_t b) {
+  double x;
+  std::memcpy(&x, &b, 8);
+  return x;
+}
+
+}  // namespace
+
+extern "C" grpo_status grpo_ars_serialize(const grpo_ars_state* st, void* buf, size_t* bytes) {
+  clear_error();
+  if (st == nullptr || bytes == nullptr)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_serialize: NULL argument");
+  if (buf == nullptr) {  // size query
+    *bytes = kArsRecordBytes;
+    return GRPO_OK;
+  }
+  if (*bytes < kArsRecordBytes)
+    return fail(GRPO_ERR_WORKSPACE, "grpo_ars_serialize: buffer of %zu bytes, need %zu", *bytes,
+                kArsRecordBytes);
+  unsigned char* p = static_cast<unsigned char*>(buf);
+  std::memcpy(p, kArsTag, 8);
+  put_u32(p + 8, (uint32_t)st->G1);
+  put_u32(p + 12, (uint32_t)st->n);
+  put_u32(p + 16, (uint32_t)st->have_ref);
+  put_u32(p + 20, (uint32_t)st->have_gt);
+  put_u64(p + 24, f64_bits(st->g_ref));
+  put_u64(p + 32, f64_bits(st->g_t));
+  put_u64(p + 40, f64_bits(st->buf_mean_sum));
+  put_u64(p + 48, f64_bits(st->buf_max_sum));
+  put_u64(p + 56, (uint64_t)st->buf_count);
+  *bytes = kArsRecordBytes;
+  return GRPO_OK;
+}
+
+extern "C" grpo_status grpo_ars_deserialize(grpo_ars_state* st, const void* buf, size_t bytes) {
+  clear_error();
+  if (st == nullptr || buf == nullptr)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_deserialize: NULL argument");
+  if (bytes < kArsRecordBytes)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_deserialize: %zu bytes, a record has %zu", bytes,
+                kArsRecordBytes);
+  const unsigned char* p = static_cast<const unsigned char*>(buf);
+  if (std::memcmp(p, kArsTag, 8) != 0)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_deserialize: not an ARS record (tag)");
+  grpo_ars_state s;
+  s.G1 = (int32_t)get_u32(p + 8);
+  s.n = (int32_t)get_u32(p + 12);
+  s.have_ref = (int32_t)get_u32(p + 16);
+  s.have_gt = (int32_t)get_u32(p + 20);
+  s.g_ref = bits_f64(get_u64(p + 24));
+  s.g_t = bits_f64(get_u64(p + 32));
+  s.buf_mean_sum = bits_f64(get_u64(p + 40));
+  s.buf_max_sum = bits_f64(get_u64(p + 48));
+  s.buf_count = (int64_t)get_u64(p + 56);
+  const bool ok = s.G1 >= 2 && s.n >= 2 && s.n <= s.G1 && (s.have_ref == 0 || s.have_ref == 1) &&
+                  (s.have_gt == 0 || s.have_gt == 1) && s.buf_count >= 0 &&
+                  std::isfinite(s.g_ref) && std::isfinite(s.g_t) &&
+                  std::isfinite(s.buf_mean_sum) && std::isfinite(s.buf_max_sum) &&
+                  s.buf_mean_sum >= 0.0 && s.buf_max_sum >= 0.0;
+  if (!ok) return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_deserialize: inconsistent record");
+  *st = s;
+  return GRPO_OK;
+}

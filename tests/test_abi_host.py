@@ -273,3 +273,60 @@ def test_lmhead_tune_rejects_out_of_range_settings(grpo):
     assert L.grpo_lmhead_tune(ctypes.c_int32(65), ctypes.c_int32(0)) == 1
     assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(9)) == 1
     assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(0)) == 0
+
+
+def test_ars_checkpoint_resumes_the_rollout_counts(oracle_mod, grpo):
+    """The ARS state saved mid-run (mid-epoch and at an epoch end) and restored into a fresh state
+    continues with exactly the rollout counts of the uninterrupted run, which equal the oracle's."""
+    import struct
+    from paper_2609_36932_gb300 import workloads
+    w = workloads.get("large")
+    steps, spe = 20, 5
+    ratios = workloads.ars_pruning_ratios(1, steps, w.P)
+
+    def run(st, first, last, n):
+        seq = []
+        for s in range(first, last + 1):
+            kept = workloads.synthetic_kept_counts(ratios[s - 1], n)
+            n = grpo.adaptive_rollout_count(st, kept, s, steps, s % spe == 0)
+            seq.append(n)
+        return seq, n
+
+    full, _ = run(grpo.grpo_ars_init(w.G), 1, steps, w.G)
+    o = oracle_mod.Ars(w.G)
+    n, seq_o = w.G, []
+    for s in range(1, steps + 1):
+        n = o.step(workloads.synthetic_kept_counts(ratios[s - 1], n), s, steps, s % spe == 0)
+        seq_o.append(n)
+    assert full == seq_o
+    for cut in (3, 5, 7, 12):
+        st = grpo.grpo_ars_init(w.G)
+        head, n = run(st, 1, cut, w.G)
+        rec = grpo.grpo_ars_serialize(st)
+        assert len(rec) == 64 and rec[:8] == b"FRLARS01"
+        assert struct.unpack_from("<iiii", rec, 8) == (st.G1, st.n, st.have_ref, st.have_gt)
+        assert struct.unpack_from("<ddddq", rec, 24) == (st.g_ref, st.g_t, st.buf_mean_sum,
+                                                         st.buf_max_sum, st.buf_count)
+        back = grpo.grpo_ars_deserialize(rec)
+        assert grpo.grpo_ars_serialize(back) == rec
+        tail, _ = run(back, cut + 1, steps, n)
+        assert head + tail == full, cut
+
+
+def test_ars_checkpoint_rejects_bad_records(grpo):
+    import struct
+    st = grpo.grpo_ars_init(8)
+    good = bytearray(grpo.grpo_ars_serialize(st))
+
+    def bad(rec):
+        with pytest.raises(grpo.GrpoError):
+            grpo.grpo_ars_deserialize(bytes(rec))
+
+    bad(good[:63])
+    r = bytearray(good); r[0:8] = b"FRLARS02"; bad(r)
+    r = bytearray(good); struct.pack_into("<i", r, 12, 9); bad(r)          # n > G1
+    r = bytearray(good); struct.pack_into("<i", r, 8, 1); bad(r)           # G1 < 2
+    r = bytearray(good); struct.pack_into("<i", r, 16, 2); bad(r)          # have_ref not 0/1
+    r = bytearray(good); struct.pack_into("<d", r, 24, float("nan")); bad(r)
+    r = bytearray(good); struct.pack_into("<q", r, 56, -1); bad(r)
+    assert grpo.grpo_ars_deserialize(bytes(good)).G1 == 8
