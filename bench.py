@@ -102,12 +102,25 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback 6.8 TB/s (no MEASURED_PEAKS.json)"
 
 
-def loss_source_hash():
+def code_hash(files, root=None):
+    """Hash of the code of `files` (under paper_2609_36932_gb300/csrc): comments, blank lines and
+    the host-side NVTX markers (GRPO_TRACE and its header) removed, so that an edit which leaves
+    the kernels alone does not orphan a profile taken on them."""
+    import re
     h = hashlib.sha256()
-    for f in ("loss.cu", "gspo.cu", "rowops.cuh", "common.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+    for f in files:
+        with open(os.path.join(root or ROOT, "paper_2609_36932_gb300", "csrc", f)) as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        lines = [ln.rstrip() for ln in text.splitlines()
+                 if ln.strip() and "GRPO_TRACE" not in ln and '"trace.cuh"' not in ln]
+        h.update("\n".join(lines).encode())
     return h.hexdigest()[:16]
+
+
+def loss_source_hash(root=None):
+    return code_hash(("loss.cu", "gspo.cu", "rowops.cuh", "common.cuh"), root)
 
 
 def profiled_traffic(workload_name):
@@ -446,18 +459,9 @@ def measured_tensor_peak(sustained):
             1900.0, "fallback 1.9 PFLOP/s burst")
 
 
-def lmhead_source_hash():
-    """Hash of the output-layer kernels' code (comments and blank lines removed, so that a
-    comment edit does not orphan a profile taken on the same code)."""
-    import re
-    h = hashlib.sha256()
-    for f in ("lmhead.cu", "rowops.cuh", "common.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_36932_gb300", "csrc", f)) as fh:
-            text = fh.read()
-        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-        text = re.sub(r"//[^\n]*", "", text)
-        h.update("\n".join(ln.rstrip() for ln in text.splitlines() if ln.strip()).encode())
-    return h.hexdigest()[:16]
+def lmhead_source_hash(root=None):
+    """Hash of the output-layer kernels' code (see code_hash)."""
+    return code_hash(("lmhead.cu", "rowops.cuh", "common.cuh"), root)
 
 
 def lmhead_traffic_per_row():

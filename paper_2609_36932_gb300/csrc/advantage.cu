@@ -5,6 +5,7 @@
 // std and each A are reproducible bit for bit from the order of operations written here; the
 // per-rollout divisions then run in parallel across lanes.
 #include "common.cuh"
+#include "trace.cuh"
 
 namespace fastrl {
 namespace {
@@ -49,6 +50,7 @@ using namespace fastrl;
 
 extern "C" grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G, int32_t std_mode,
                                       float* adv, double* key, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_advantage");
   clear_error();
   if (P < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_advantage: P = %d < 0", P);
   if (G < 1 || G > 1024) return fail(GRPO_ERR_INVALID_ARG, "grpo_advantage: G = %d not in [1, 1024]", G);

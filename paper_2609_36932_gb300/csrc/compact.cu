@@ -6,6 +6,7 @@
 //   compact_fill_kernel  one CTA per rollout: a kept rollout finds its position k by binary
 //                        search in kept_idx and writes its token indices and rollout id.
 #include "common.cuh"
+#include "trace.cuh"
 
 namespace fastrl {
 namespace {
@@ -111,6 +112,7 @@ extern "C" grpo_status grpo_compact(const uint8_t* keep, const int64_t* off, int
                                     int32_t* kept_idx, int64_t* kept_off, int64_t* src_token,
                                     int32_t* token_rollout, int64_t* counts, int64_t* counts_host,
                                     grpo_stream_t stream) {
+  GRPO_TRACE("grpo_compact");
   clear_error();
   if (n_rollouts < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_compact: n_rollouts < 0");
   if (!off || !kept_off || !counts || (n_rollouts > 0 && (!keep || !kept_idx)))
@@ -141,6 +143,7 @@ extern "C" grpo_status grpo_upload_kept(const void* src_host, void* dst_dev, int
                                         const uint8_t* keep_host, const int64_t* off_host,
                                         int32_t n_rollouts, int64_t* bytes_out,
                                         int32_t* copies_out, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_upload_kept");
   clear_error();
   if (bytes_out) *bytes_out = 0;
   if (copies_out) *copies_out = 0;

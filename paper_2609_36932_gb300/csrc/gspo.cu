@@ -15,6 +15,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "trace.cuh"
 #include "rowops.cuh"
 
 namespace fastrl {
@@ -395,6 +396,7 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd(
     int64_t n_seq, float eps_low, float eps_high, float beta, void* dlogits, int32_t dlogits_dtype,
     float* logp_out, float* seq_ratio_out, double* loss_out, int32_t* status, void* ws,
     size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_gspo_loss_fwd_bwd");
   clear_error();
   return gspo_impl("grpo_gspo_loss_fwd_bwd", logits, logits_dtype, row_stride, row_index, n_rows,
                    V, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, n_seq_rows, nullptr,
@@ -409,6 +411,7 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd_dev(
     const int64_t* seq_row_off, int64_t n_seq, float eps_low, float eps_high, float beta,
     void* dlogits, int32_t dlogits_dtype, float* logp_out, float* seq_ratio_out, double* loss_out,
     int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_gspo_loss_fwd_bwd_dev");
   clear_error();
   if (counts == nullptr)
     return fail(GRPO_ERR_INVALID_ARG, "grpo_gspo_loss_fwd_bwd_dev: counts is NULL");

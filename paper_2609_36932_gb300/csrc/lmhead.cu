@@ -49,6 +49,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "trace.cuh"
 #include "rowops.cuh"
 
 namespace fastrl {
@@ -974,6 +975,7 @@ extern "C" grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_s
                                             const void* weight, int32_t V, int32_t D,
                                             const int32_t* y, float* logp_out, int32_t* status,
                                             void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_lmhead_logp_fwd");
   clear_error();
   const char* who = "grpo_lmhead_logp_fwd";
   grpo_status st = check_shape(who, n_rows, V, D, hidden_stride);
@@ -1017,6 +1019,7 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
     int32_t accumulate_dweight, void* dlogits_out, float* logp_out, double* row_loss_out,
     double* loss_out, int32_t* status, int64_t chunk_rows, void* ws, size_t* ws_bytes,
     grpo_stream_t stream) {
+  GRPO_TRACE("grpo_lmhead_loss_fwd_bwd");
   clear_error();
   const char* who = "grpo_lmhead_loss_fwd_bwd";
   grpo_status st = check_shape(who, n_rows, V, D, hidden_stride);
@@ -1113,6 +1116,7 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
     float beta, void* dhidden, int32_t dhidden_dtype, float* dweight, int32_t accumulate_dweight,
     void* dlogits_out, float* logp_out, float* seq_ratio_out, double* loss_out, int32_t* status,
     int64_t chunk_rows, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_lmhead_gspo_loss_fwd_bwd");
   clear_error();
   const char* who = "grpo_lmhead_gspo_loss_fwd_bwd";
   grpo_status st = check_shape(who, n_rows, V, D, hidden_stride);

@@ -36,6 +36,7 @@
 #include <tuple>
 
 #include "common.cuh"
+#include "trace.cuh"
 #include "rowops.cuh"
 
 namespace fastrl {
@@ -940,6 +941,7 @@ extern "C" grpo_status grpo_loss_fwd_bwd(
     int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq, void* dlogits,
     int32_t dlogits_dtype, float* logp_out, double* row_loss_out, double* loss_out, int32_t* status,
     void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_loss_fwd_bwd");
   clear_error();
   return loss_impl("grpo_loss_fwd_bwd", logits, logits_dtype, row_stride, row_index, n_rows, nullptr,
                    V, y, old_logp, ref_logp, adv, row_rollout, eps_low, eps_high, beta, agg_mode,
@@ -954,6 +956,7 @@ extern "C" grpo_status grpo_loss_fwd_bwd_dev(
     float eps_high, float beta, int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off,
     int64_t n_seq, void* dlogits, int32_t dlogits_dtype, float* logp_out, double* row_loss_out,
     double* loss_out, int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_loss_fwd_bwd_dev");
   clear_error();
   if (counts == nullptr)
     return fail(GRPO_ERR_INVALID_ARG, "grpo_loss_fwd_bwd_dev: counts is NULL");
@@ -1025,6 +1028,7 @@ extern "C" grpo_status grpo_logp_fwd(const void* logits, int32_t logits_dtype, i
                                      const int64_t* row_index, int64_t n_rows, int32_t V,
                                      const int32_t* y, float* logp_out, int32_t* status,
                                      grpo_stream_t stream) {
+  GRPO_TRACE("grpo_logp_fwd");
   clear_error();
   return logp_rows("grpo_logp_fwd", logits, logits_dtype, row_stride, row_index, n_rows, nullptr,
                    V, y, logp_out, nullptr, status, as_stream(stream));
@@ -1063,6 +1067,7 @@ extern "C" grpo_status grpo_loss_fwd_bwd_noalloc(
     int32_t agg_mode, int64_t denom_tokens, const int64_t* seq_off, int64_t n_seq, void* dlogits,
     int32_t dlogits_dtype, float* logp_out, double* row_loss_out, double* loss_out, int32_t* status,
     grpo_stream_t stream) {
+  GRPO_TRACE("grpo_loss_fwd_bwd_noalloc");
   clear_error();
   const char* who = "grpo_loss_fwd_bwd_noalloc";
   if (row_loss_out != nullptr)  // the caller's row-loss buffer is the only scratch: none needed

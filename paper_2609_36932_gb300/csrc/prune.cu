@@ -22,6 +22,7 @@
 #include <atomic>
 
 #include "common.cuh"
+#include "trace.cuh"
 
 namespace fastrl {
 namespace {
@@ -553,6 +554,7 @@ extern "C" grpo_status grpo_prune(const float* rewards, const float* adv, float 
                                   int64_t T, int32_t V, int32_t ngram_n, float tau, int32_t keep_cap,
                                   int32_t dp_divisor, uint8_t* keep, int32_t* kept_per_prompt,
                                   int32_t* status, void* ws, size_t* ws_bytes, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_prune");
   clear_error();
   if (!(class_eps >= 0.f)) return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: class_eps must be >= 0");
   if (P < 0 || T < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_prune: P = %d, T = %lld", P, (long long)T);

@@ -5,6 +5,7 @@
 // loading kBatch of them before adding any (the loads overlap; the order of the additions does
 // not change); then a fixed xor-shuffle tree inside each warp and one more across the 32 warps.
 #include "common.cuh"
+#include "trace.cuh"
 
 namespace fastrl {
 namespace {
@@ -55,6 +56,7 @@ grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* n_dev, do
 using namespace fastrl;
 
 extern "C" grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grpo_stream_t stream) {
+  GRPO_TRACE("grpo_sum_f64");
   clear_error();
   if (n < 0 || out == nullptr || (n > 0 && v == nullptr))
     return fail(GRPO_ERR_INVALID_ARG, "grpo_sum_f64: n = %lld, v or out NULL", (long long)n);
