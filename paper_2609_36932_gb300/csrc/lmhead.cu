@@ -710,18 +710,26 @@ Grid plan(int64_t rows, int V, int n_sm) {
 
 grpo_status launch_tiles(bool bwd, const CUtensorMap& mh, const CUtensorMap& mw,
                          const TileArgs& a, int grid, cudaStream_t s, const char* who) {
-  static std::once_flag attr_once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(lmhead_tile_kernel<false>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(lmhead_tile_kernel<true>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)kSmemBytes);
-  });
-  if (attr_err != cudaSuccess)
-    return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(attr_err));
+  // The shared-memory limit is a per-device function attribute: set it once on each device.
+  static std::mutex mu;
+  static uint64_t done = 0;  // bit d: set on device d
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaGetDevice: %s", who, cudaGetErrorString(e));
+  if (dev < 0 || dev >= 64) return fail(GRPO_ERR_UNSUPPORTED, "%s: device %d beyond 64", who, dev);
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    if (!((done >> dev) & 1u)) {
+      e = cudaFuncSetAttribute(lmhead_tile_kernel<false>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(lmhead_tile_kernel<true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+      if (e != cudaSuccess)
+        return fail(GRPO_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
+      done |= uint64_t(1) << dev;
+    }
+  }
   if (bwd)
     lmhead_tile_kernel<true><<<grid, kThreads, kSmemBytes, s>>>(mh, mw, a);
   else
