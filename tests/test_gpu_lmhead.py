@@ -433,3 +433,38 @@ def test_non_finite_hidden_row_is_flagged(grpo):
     assert np.isnan(g["logp"][17])
     others = np.arange(case.T) != 17
     np.testing.assert_array_equal(g["logp"][others], clean["logp"][others])
+
+
+@pytest.mark.parametrize("T,V,D", [(400, 32000, 4096), (300, 8192, 8192)])
+def test_large_hidden_sizes_sampled_rows(grpo, oracle_mod, T, V, D):
+    """Long reductions (64 and 128 k-blocks of 64 per tile): the GPU runs every row; the oracle
+    checks sampled rows one by one (logp and dhidden, token-mean weights over all T rows)."""
+    import torch
+    rng = np.random.default_rng(D)
+    h = bf16_round(rng.standard_normal((T, D)))
+    w = bf16_round(rng.standard_normal((V, D)) * (2.0 / np.sqrt(D)))
+    y = rng.integers(0, V, T).astype(np.int32)
+    rr = np.sort(rng.integers(0, 8, T)).astype(np.int32)
+    adv = rng.standard_normal(8).astype(np.float32)
+    ht = torch.from_numpy(h).cuda().to(torch.bfloat16)
+    wt = torch.from_numpy(w).cuda().to(torch.bfloat16)
+    z = (ht.float() @ wt.float().t()).double()
+    logp_c = (z.gather(1, torch.from_numpy(y.astype(np.int64)).cuda()[:, None])[:, 0]
+              - torch.logsumexp(z, 1)).cpu().numpy()
+    old = (logp_c + rng.normal(0, 0.05, T)).astype(np.float32)
+    ref = (logp_c + rng.normal(0, 0.1, T)).astype(np.float32)
+    t = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).cuda().to(dt)
+    lp = torch.empty(T, dtype=torch.float32, device="cuda")
+    out = grpo.grpo_lmhead_loss_fwd_bwd(ht, wt, t(y, torch.int32), t(old, torch.float32),
+                                        t(ref, torch.float32), t(adv, torch.float32),
+                                        t(rr, torch.int32), logp_out=lp, dhidden_dtype="f32")
+    torch.cuda.synchronize()
+    rows = np.array([0, 1, T // 2, T - 1])
+    o = oracle_mod.lmhead_loss(h[rows], w, y[rows], old[rows], ref[rows], adv, rr[rows],
+                               denom_tokens=T, want_dweight=False, want_bounds=True)
+    S = np.abs(h[rows]).astype(np.float64) @ np.abs(w).astype(np.float64).T
+    dz = D * U * S.max(1)
+    assert np.all(np.abs(lp.cpu().numpy()[rows] - o["logp"]) <= 2 * dz + 1e-5)
+    rel = 2.0 ** -8 + 4 * dz.max() + V * U
+    dh = out["dhidden"].cpu().numpy()[rows]
+    assert np.all(np.abs(dh - o["dhidden"]) <= rel * o["dhidden_abs"] + 1e-30)
