@@ -66,6 +66,9 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-lmhead", action="store_true",
+                    help="skip the default run's side measurement of the output layer fused with "
+                         "the loss (tensor cores)")
     ap.add_argument("--no-graph", action="store_true",
                     help="run each step's calls directly instead of replaying captured CUDA graphs")
     return ap.parse_args()
@@ -570,6 +573,52 @@ def cpu_baseline_lmhead_gspo(w, b, d, step, target_s):
                       " kept sequences (%d rows, %.2f s)" % (t_sel, T_kept, k, rows, t)}
 
 
+def lmhead_side(w, b, step, seed, dev, reps=3):
+    """The output layer fused with the loss on this batch's kept rows (hidden states of width
+    LMHEAD_D drawn for the same tokens): one host-timed call block, reported beside the main
+    line.  Returns a dict, or None when the output layer's inputs do not fit in device memory."""
+    import torch
+    import paper_2609_36932_gb300 as g
+    from paper_2609_36932_gb300 import workloads
+    D = workloads.LMHEAD_D
+    need = (b["T"] * D * 2 + w.V * D * 6 + 5 * (1 << 30))
+    free, _ = torch.cuda.mem_get_info(dev)
+    if need > 0.8 * free:
+        return None
+    hid = workloads.lmhead_hidden(b["T"], D, seed, dev)
+    wt = workloads.lmhead_weight(w.V, D, seed, dev)
+    old, ref = workloads.lmhead_old_ref(hid, wt, b["ids"], b["noise_old"], b["noise_ref"])
+    T_kept = step.T_kept
+    rows = step.src_token[:T_kept]
+    ids = torch.from_numpy(b["ids"]).to(dev)
+    kw = dict(row_index=rows, n_rows=T_kept, eps_low=w.eps, eps_high=w.eps, beta=w.beta,
+              denom_tokens=max(T_kept, 1))
+    out = g.grpo_lmhead_loss_fwd_bwd(hid, wt, ids, old, ref, step.adv, step.token_rollout, **kw)
+    ws, dh, dw = out["ws"], out["dhidden"], out["dweight"]
+    g.grpo_lmhead_loss_fwd_bwd(hid, wt, ids, old, ref, step.adv, step.token_rollout, dhidden=dh,
+                               dweight=dw, ws=ws, **kw)
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        g.grpo_lmhead_loss_fwd_bwd(hid, wt, ids, old, ref, step.adv, step.token_rollout,
+                                   dhidden=dh, dweight=dw, ws=ws, **kw)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    peak, src = measured_tensor_peak(sustained=True)
+    tf = 8.0 * T_kept * w.V * D / (ms / 1e3) / 1e12
+    del hid, wt, old, ref, dh, dw, ws, out
+    torch.cuda.empty_cache()
+    return {"call": "grpo_lmhead_loss_fwd_bwd", "D": D, "T_kept": T_kept, "calls": reps,
+            "ms_per_call": ms, "kept_tokens_per_s": T_kept / (ms / 1e3), "achieved": tf,
+            "unit": "TFLOP/s", "peak": peak, "frac": tf / peak, "peak_source": src,
+            "note": "the output layer fused with the loss on this batch's kept rows: logits "
+                    "h W^T on the tcgen05 tensor cores (never stored), loss, dhidden, dweight; "
+                    "8 T_kept V D FLOPs per call; bench.py --loss lmhead runs it as a step"}
+
+
 def run_lmhead(args, w):
     """--loss lmhead: the step with the output layer fused (GrpoStep in output-layer mode)."""
     import torch
@@ -944,6 +993,10 @@ def main():
                     "kept_tokens_per_s": step.T_kept / (f_ms / 1e3),
                     "algorithmic_bytes_per_launch": f_bytes}
 
+    lmhead = None
+    if not args.no_lmhead and args.loss == "grpo" and w.chunk_rows == 0:
+        lmhead = lmhead_side(w, b, step, rank_seed(args.seed, rank), dev)
+
     # end to end: inputs copied from pinned host memory, loss read back, inside the timed region
     e2e = None
     names = ["rewards", "ids", "off", "logits", "old", "ref"]
@@ -1005,7 +1058,7 @@ def main():
             "config": dict(workload_desc(w, b["T"], step.T_kept, step.K), loss=args.loss),
             "gpu_launches": int(launches), "cuda_graph": use_graph,
             "roofline": roofline, "e2e": e2e,
-            "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd,
+            "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd, "lmhead": lmhead,
             "path_overhead": {"select_ms": select_ms,
                               "other_ms": elapsed_ms / K - select_ms - loss_ms,
                               "note": "select_ms: advantage, prune, compaction (and the kept-count"
