@@ -468,3 +468,17 @@ def test_large_hidden_sizes_sampled_rows(grpo, oracle_mod, T, V, D):
     rel = 2.0 ** -8 + 4 * dz.max() + V * U
     dh = out["dhidden"].cpu().numpy()[rows]
     assert np.all(np.abs(dh - o["dhidden"]) <= rel * o["dhidden_abs"] + 1e-30)
+
+
+@pytest.mark.parametrize("prefetch,lanes", [(0, 1), (0, 8), (4, 3)])
+def test_parity_under_other_schedules(grpo, oracle_mod, prefetch, lanes):
+    """grpo_lmhead_tune changes the grid (pair lanes x vocabulary lanes) and adds L2 prefetches;
+    every setting computes the same function."""
+    case = LmCase(101 + lanes, 900, 3000, 192)
+    o = case.oracle(oracle_mod)
+    try:
+        grpo.grpo_lmhead_tune(prefetch, lanes)
+        g = case.gpu(grpo)
+    finally:
+        grpo.grpo_lmhead_tune(0, 0)
+    check(case, g, o)
