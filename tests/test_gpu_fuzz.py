@@ -13,7 +13,6 @@ pytestmark = pytest.mark.gpu
 
 @pytest.mark.parametrize("seed", range(12))
 def test_fused_loss_random_configurations(grpo, oracle_mod, seed):
-    import torch
     rng = np.random.default_rng(1000 + seed)
     V = int(rng.choice([1, 2, 7, 33, 1000, 4097]) if seed % 3 == 0 else rng.integers(1, 70000))
     ind, outd = rng.choice(["bf16", "f32"]), rng.choice(["bf16", "f32"])

@@ -4,7 +4,6 @@ launch shapes, gathered rows, invalid ids and the workloads' full size."""
 import numpy as np
 import pytest
 
-from helpers import bf16_bits_to_f32
 
 pytestmark = pytest.mark.gpu
 LOGP_ATOL = 2e-5

@@ -4,7 +4,6 @@ that forbids allocation after start-up).  It must give the same results as grpo_
 call after call, although its scratch is one fixed array inside the library that every call
 reuses.  This file is collected last so that a run stopping at the first failure has already
 run every other test."""
-import ctypes
 
 import numpy as np
 import pytest
