@@ -46,6 +46,7 @@
 #include <cublasLt.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -703,8 +704,9 @@ struct Grid {
   int R, J, grid;
 };
 // Launch settings of this process (grpo_lmhead_tune): prefetch distance, row lanes (0 = chosen).
-int g_prefetch = 0;
-int g_row_lanes = 0;
+// Atomic: another thread may change them while a call reads them.
+std::atomic<int> g_prefetch{0};
+std::atomic<int> g_row_lanes{0};
 
 // R pair lanes x J vocabulary lanes, one CTA per SM at most.  The weight is read from DRAM about
 // once per group of R row-block pairs, so R stays in [4, 8] (all pairs when there are fewer);
@@ -717,8 +719,9 @@ Grid plan(int64_t rows, int V, int n_sm) {
   const int n_vt = (V + BN - 1) / BN;
   Grid best = {1, 1, 1};
   double best_u = -1.0;
-  const int r_hi = g_row_lanes > 0 ? g_row_lanes : kRowLanes;
-  const int r_lo = g_row_lanes > 0 ? g_row_lanes : std::min(kRowLanes, std::max(1, std::min(n_rb, 4)));
+  const int lanes = g_row_lanes.load(std::memory_order_relaxed);
+  const int r_hi = lanes > 0 ? lanes : kRowLanes;
+  const int r_lo = lanes > 0 ? lanes : std::min(kRowLanes, std::max(1, std::min(n_rb, 4)));
   for (int R = r_hi; R >= r_lo; --R) {
     const int Rr = std::max(1, std::min(n_rb, R));
     const int J = std::max(1, std::min({n_vt, std::max(1, n_sm / Rr), kMaxJ}));
@@ -940,7 +943,7 @@ grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
   ta.n_rb = (int32_t)((n_rows + BM - 1) / BM);
   ta.R = g1.R;
   ta.J = g1.J;
-  ta.prefetch = g_prefetch;
+  ta.prefetch = g_prefetch.load(std::memory_order_relaxed);
   ta.y = f->y;
   ta.part = reinterpret_cast<float2*>(wsb + L.part);
   ta.zy = reinterpret_cast<float*>(wsb + L.zy);
@@ -997,8 +1000,8 @@ extern "C" grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes) {
   if (prefetch < 0 || prefetch > 64 || row_lanes < 0 || row_lanes > kRowLanes)
     return fail(GRPO_ERR_INVALID_ARG, "grpo_lmhead_tune: prefetch in [0, 64], row_lanes in [0, %d]",
                 kRowLanes);
-  g_prefetch = prefetch;
-  g_row_lanes = row_lanes;
+  g_prefetch.store(prefetch, std::memory_order_relaxed);
+  g_row_lanes.store(row_lanes, std::memory_order_relaxed);
   return GRPO_OK;
 }
 
