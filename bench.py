@@ -958,7 +958,7 @@ def main():
     else:
         bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
         per_row_traffic = profiled_traffic(w.name)
-        kernel = "grpo_loss_kernel (+ 1-CTA fixed-order loss sum)"
+        kernel = "grpo_loss_kernel (+ the fixed-order loss sum, one 8-CTA cluster)"
     achieved = step.T_kept * bytes_per_row / (loss_ms / 1e3) / 1e9
     peak, peak_src = measured_peak()
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

@@ -37,7 +37,7 @@ grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype,
                       cudaStream_t s);
 
 // reduce.cu: *out = v[0] + ... + v[m-1] in fp64 in a fixed order, m = n or, with n_dev (a device
-// count, nullable), min(n, *n_dev); one single-CTA launch on `s`.
+// count, nullable), min(n, *n_dev); one launch of an 8-CTA cluster on `s`.
 grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* n_dev, double* out,
                             cudaStream_t s, const char* who);
 

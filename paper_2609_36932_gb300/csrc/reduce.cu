@@ -1,9 +1,13 @@
 // Fixed-order fp64 sum of per-row (or per-sequence) loss terms: the last step of every loss call
 // and of grpo_sum_f64, so that a loss computed in one call or in chunks sums to the same bits.
 //
-// One CTA of 1024 threads.  Thread t adds v[t], v[t + 1024], v[t + 2048], ... in that order,
-// loading kBatch of them before adding any (the loads overlap; the order of the additions does
-// not change); then a fixed xor-shuffle tree inside each warp and one more across the 32 warps.
+// One cluster of kSumCtas CTAs of 1024 threads.  CTA r takes the contiguous segment
+// [r*seg, (r+1)*seg) of the n terms (seg depends on n only); inside it thread t adds v[t],
+// v[t + 1024], ... in that order, loading kBatch of them before adding any (the loads overlap; the
+// order of the additions does not change); a fixed xor-shuffle tree inside each warp and one more
+// across the 32 warps give the segment's sum.  After a cluster barrier, CTA 0 reads the segment
+// sums from its peers' shared memory and adds them by a fixed tree; a second barrier keeps the
+// peers resident until it has.  The order depends on n alone, never on scheduling.
 #include "common.cuh"
 #include "trace.cuh"
 
@@ -11,21 +15,34 @@ namespace fastrl {
 namespace {
 
 constexpr int kSumThreads = 1024;
+constexpr int kSumCtas = 8;
 constexpr int kBatch = 8;
 
-__global__ void __launch_bounds__(kSumThreads)
+__device__ __forceinline__ void sum_cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+
+__global__ void __cluster_dims__(kSumCtas, 1, 1) __launch_bounds__(kSumThreads)
     sum_rows_kernel(const double* __restrict__ v, int64_t n, const int64_t* __restrict__ n_dev,
                     double* __restrict__ out) {
   __shared__ double part[kSumThreads / 32];
+  __shared__ double seg_sum;
   if (n_dev && *n_dev < n) n = *n_dev;
+  if (n < 0) n = 0;
+  uint32_t rank;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+  const int64_t seg = (n + kSumCtas - 1) / kSumCtas;
+  const int64_t lo = (int64_t)rank * seg;
+  const int64_t hi = lo + seg < n ? lo + seg : n;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   double acc = 0.0;
-  for (int64_t base = tid; base < n; base += (int64_t)kSumThreads * kBatch) {
+  for (int64_t base = lo + tid; base < hi; base += (int64_t)kSumThreads * kBatch) {
     double x[kBatch];
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) {
       const int64_t i = base + (int64_t)u * kSumThreads;
-      x[u] = i < n ? v[i] : 0.0;
+      x[u] = i < hi ? v[i] : 0.0;
     }
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) acc += x[u];
@@ -38,15 +55,28 @@ __global__ void __launch_bounds__(kSumThreads)
     acc = part[lane];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) *out = acc;
+    if (lane == 0) seg_sum = acc;
   }
+  sum_cluster_sync();  // every segment's sum is in its CTA's shared memory
+  if (rank == 0 && warp == 0) {
+    double x = 0.0;
+    if (lane < kSumCtas) {
+      uint32_t local = static_cast<uint32_t>(__cvta_generic_to_shared(&seg_sum)), remote;
+      asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(lane));
+      asm volatile("ld.shared::cluster.f64 %0, [%1];" : "=d"(x) : "r"(remote) : "memory");
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    if (lane == 0) *out = x;
+  }
+  sum_cluster_sync();  // the peers stay until CTA 0 has read their sums
 }
 
 }  // namespace
 
 grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* n_dev, double* out,
                             cudaStream_t s, const char* who) {
-  sum_rows_kernel<<<1, kSumThreads, 0, s>>>(v, n, n_dev, out);
+  sum_rows_kernel<<<kSumCtas, kSumThreads, 0, s>>>(v, n, n_dev, out);
   count_launches(1);
   return check_launch(who);
 }
