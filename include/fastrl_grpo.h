@@ -471,6 +471,15 @@ grpo_status grpo_loss_tune(int32_t cluster_ctas, int32_t threads, int32_t chunks
 grpo_status grpo_test_skip_copy(int32_t enable);
 
 /*
+ * grpo_test_fail_launch — test hook for the error path of every call (no counterpart in the
+ * paper).  nth > 0: the nth launch check from now (counting every kernel launch of every call)
+ * reports GRPO_ERR_CUDA with an "injected launch failure" message, as a real launch error would;
+ * the kernel itself has been enqueued normally, and the call returns without enqueuing the rest.
+ * nth = 0 disarms.  Nothing is done to the device.  GRPO_ERR_INVALID_ARG for nth < 0.
+ */
+grpo_status grpo_test_fail_launch(int32_t nth);
+
+/*
  * Adaptive rollout sampling state, Algorithm 1 (the "adaptive sampling state" and the two
  * epoch-level buffers).  Plain data: it may be copied or saved and restored byte for byte.
  */

@@ -34,7 +34,8 @@ EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_adva
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
            "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
            "grpo_lmhead_logp_fwd", "grpo_lmhead_tune", "grpo_lmhead_gspo_loss_fwd_bwd",
-           "grpo_loss_tune", "grpo_test_skip_copy", "grpo_ars_init", "adaptive_rollout_count",
+           "grpo_loss_tune", "grpo_test_skip_copy", "grpo_test_fail_launch", "grpo_ars_init",
+           "adaptive_rollout_count",
            "grpo_ars_serialize", "grpo_ars_deserialize"]
 
 
@@ -127,6 +128,8 @@ def lib():
     L.grpo_lmhead_dlogits_stride.restype = _i64
     L.grpo_sum_f64.argtypes = [_c_p, _i64, _c_p, _c_p]
     L.grpo_sum_f64.restype = _i32
+    L.grpo_test_fail_launch.argtypes = [_i32]
+    L.grpo_test_fail_launch.restype = _i32
     L.grpo_test_skip_copy.argtypes = [_i32]
     L.grpo_test_skip_copy.restype = _i32
     L.grpo_loss_tune.argtypes = [_i32, _i32, _i32]

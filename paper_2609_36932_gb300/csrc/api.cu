@@ -27,9 +27,15 @@ void clear_error() { g_msg[0] = 0; }
 
 void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
+// Test hook (grpo_test_fail_launch): the n-th next launch check reports a failure.
+std::atomic<int> g_fail_countdown{0};
+
 grpo_status check_launch(const char* what) {
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+  if (g_fail_countdown.load(std::memory_order_relaxed) > 0 &&
+      g_fail_countdown.fetch_sub(1, std::memory_order_relaxed) == 1)
+    return fail(GRPO_ERR_CUDA, "%s: injected launch failure (grpo_test_fail_launch)", what);
   return GRPO_OK;
 }
 
@@ -227,5 +233,12 @@ extern "C" grpo_status grpo_ars_deserialize(grpo_ars_state* st, const void* buf,
                   s.buf_mean_sum >= 0.0 && s.buf_max_sum >= 0.0;
   if (!ok) return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_deserialize: inconsistent record");
   *st = s;
+  return GRPO_OK;
+}
+
+extern "C" grpo_status grpo_test_fail_launch(int32_t nth) {
+  clear_error();
+  if (nth < 0) return fail(GRPO_ERR_INVALID_ARG, "grpo_test_fail_launch: nth = %d", nth);
+  g_fail_countdown.store(nth, std::memory_order_relaxed);
   return GRPO_OK;
 }

@@ -330,3 +330,10 @@ def test_ars_checkpoint_rejects_bad_records(grpo):
     r = bytearray(good); struct.pack_into("<d", r, 24, float("nan")); bad(r)
     r = bytearray(good); struct.pack_into("<q", r, 56, -1); bad(r)
     assert grpo.grpo_ars_deserialize(bytes(good)).G1 == 8
+
+
+def test_fail_launch_hook_rejects_negative_counts(grpo):
+    L = raw()
+    L.grpo_test_fail_launch.restype = ctypes.c_int32
+    assert L.grpo_test_fail_launch(ctypes.c_int32(-1)) == 1
+    assert L.grpo_test_fail_launch(ctypes.c_int32(0)) == 0

@@ -345,3 +345,23 @@ def test_large_vocabularies(grpo, oracle_mod, V):
     compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
     lp = grpo.grpo_logp_fwd(c.dev, c.t(c.y)).cpu().numpy()[:5]
     assert np.abs(lp.astype(np.float64) - r["logp"]).max() <= 2e-5
+
+
+def test_injected_launch_failure_is_reported_and_the_next_call_is_clean(grpo, oracle_mod):
+    """Host-side fault injection: the test hook makes one launch check report an error.  The call
+    raises GrpoError with the injected message; the next call, with nothing armed, matches the
+    oracle.  Nothing faults on the device."""
+    rng = np.random.default_rng(98)
+    c = Case(rng, 24, 1000, "bf16", "bf16")
+    grpo.binding.lib().grpo_test_fail_launch(1)
+    try:
+        with pytest.raises(grpo.GrpoError) as err:
+            c.run_gpu(grpo)
+    finally:
+        grpo.binding.lib().grpo_test_fail_launch(0)
+    assert "injected launch failure" in str(err.value)
+    assert err.value.status == 4  # GRPO_ERR_CUDA
+    good = c.run_gpu(grpo)
+    assert good["status"] == 0
+    compare(good["logp"], good["dlogits"], good["loss"], c.run_oracle(oracle_mod), "bf16",
+            gpu_row_loss=good["row_loss"])
