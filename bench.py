@@ -39,6 +39,8 @@ SIDE_BYTES_PER_ROW = 36  # y, old, ref, logp (4 each), src_token 8, row rollout 
 # each), dlogits pass (src 8, coef 4, stats 16, y 4)
 GSPO_SIDE_BYTES_PER_ROW = 88
 FALLBACK_HBM_GBS = 6800.0
+# rough step times of the further workloads (ms), to size their timed step counts
+EXTRA_MS_GUESS = {"large": 5.2, "long": 20.0, "small": 0.26, "tiny": 0.07}
 
 
 def parse():
@@ -70,6 +72,11 @@ def parse():
                          "the loss (tensor cores)")
     ap.add_argument("--no-graph", action="store_true",
                     help="run each step's calls directly instead of replaying captured CUDA graphs")
+    ap.add_argument("--extra-configs", default="large,long",
+                    help="with the qwen workload: further workloads measured after it, each in "
+                         "its own sub-record of the line (comma-separated; empty for none)")
+    ap.add_argument("--extra-seconds", type=float, default=0.5,
+                    help="timed device seconds per further workload (sets its step count)")
     return ap.parse_args()
 
 
@@ -283,10 +290,26 @@ def cpu_baseline_ours(w, b, step, dev_inputs, target_s):
     t_sel, t_loss, _, cores = oracle_sample(w, b, rows, rr[:n], step.T_kept,
                                             host_logits_bits(dev_inputs["logits"][rows]), old, ref)
     t_per_token = t_loss / n + t_sel / max(step.T_kept, 1)
-    return {"value": 1.0 / t_per_token, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": "fp64 oracle: advantage+prune+compact on the whole batch (%.2f s, amortised"
-                      " over its %d kept tokens) + loss fwd/bwd on the first %d kept rows (%.2f s)"
-                      % (t_sel, step.T_kept, n, t_loss)}
+    out = {"value": 1.0 / t_per_token, "unit": UNIT, "cores": cores, "kind": "oracle",
+           "sample": "fp64 oracle: advantage+prune+compact on the whole batch (%.2f s, amortised"
+                     " over its %d kept tokens) + loss fwd/bwd on the first %d kept rows (%.2f s)"
+                     % (t_sel, step.T_kept, n, t_loss)}
+    # the same oracle on one core, on the first rows of the same sample (about target_s / 2)
+    n1 = int(min(n, max(n0, 0.5 * target_s / (per_row * max(cores, 1)))))
+    rows1 = src[:n1]
+    import oracle
+    try:
+        oracle.set_threads(1)
+        t_sel1, t_loss1, _, c1 = oracle_sample(w, b, rows1, rr[:n1], step.T_kept,
+                                               host_logits_bits(dev_inputs["logits"][rows1]),
+                                               old, ref)
+    finally:
+        oracle.set_threads(cores)
+    out["single_thread"] = {
+        "value": 1.0 / (t_loss1 / n1 + t_sel1 / max(step.T_kept, 1)), "unit": UNIT, "cores": c1,
+        "sample": "the same oracle with one OpenMP thread: selection on the whole batch (%.2f s)"
+                  " + loss fwd/bwd on the first %d kept rows (%.2f s)" % (t_sel1, n1, t_loss1)}
+    return out
 
 
 def cpu_baseline_gspo(w, b, step, dev_inputs, target_s):
@@ -437,7 +460,8 @@ def run_reference(args, w):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": workload_desc(w, b["T"], T_kept, comp["K"]),
+        "data": "synthetic", "config": dict(workload_desc(w, b["T"], T_kept, comp["K"]),
+                                            loss=args.loss),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                          "sample": "per step: fp64 oracle advantage+prune+compact on the whole batch"
                                    " (amortised over %d kept tokens) + loss fwd/bwd on the first %d"
@@ -862,39 +886,16 @@ def run_reference_lmhead(args, w):
     }), flush=True)
 
 
-def main():
-    args = parse()
-    import dataclasses
-    from paper_2609_36932_gb300 import workloads
-    w = workloads.get(args.config)
-    if args.prompts > 0:
-        w = dataclasses.replace(w, P=args.prompts)
-    if args.group > 0:
-        w = dataclasses.replace(w, G=args.group)
-    if args.impl == "reference":
-        if args.loss in ("lmhead", "lmhead-gspo"):
-            if dist_env()[0] == 0:
-                run_reference_lmhead(args, w)
-            return
-        run_reference(args, w)
-        return
-    if args.loss in ("lmhead", "lmhead-gspo"):
-        run_lmhead(args, w)
-        return
+def timed_steps(args, w, seed, world, local, dev, steps, warmup):
+    """Build a workload's batch on the device, warm up, then time `steps` whole steps with CUDA
+    events on the launching stream (barrier and synchronisation on both sides, max over ranks).
+    Returns the step, its inputs and the measurements, `roofline` for the loss call included."""
     import torch
     import torch.distributed as dist
     import paper_2609_36932_gb300 as g
-
-    rank, world, local = dist_env()
-    if world > 1:
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    g.lib()
-
-    b, d = build_inputs(w, rank_seed(args.seed, rank), dev)
+    b, d = build_inputs(w, seed, dev)
     step = make_step(w, d, args.loss)
-    for _ in range(max(args.warmup, 3)):
+    for _ in range(max(warmup, 3)):
         step.run()
     torch.cuda.synchronize()
     l_before = g.grpo_kernel_launches()
@@ -904,10 +905,10 @@ def main():
     use_graph = not args.no_graph and step.p.chunk_rows == 0
     if use_graph:
         step.capture()
-        for _ in range(max(args.warmup, 3)):
+        for _ in range(max(warmup, 3)):
             step.run_graph()
 
-    K = args.steps
+    K = steps
     stream = torch.cuda.current_stream()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s0 = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
@@ -959,6 +960,9 @@ def main():
         bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
         per_row_traffic = profiled_traffic(w.name)
         kernel = "grpo_loss_kernel (+ the fixed-order loss sum, one 8-CTA cluster)"
+        if step.p.chunk_rows:
+            kernel += "; %d calls of at most %d kept rows" % (
+                -(-step.T_kept // step.p.chunk_rows), step.p.chunk_rows)
     achieved = step.T_kept * bytes_per_row / (loss_ms / 1e3) / 1e9
     peak, peak_src = measured_peak()
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
@@ -966,7 +970,62 @@ def main():
                 "traffic": None if per_row_traffic is None else per_row_traffic * step.T_kept,
                 "kernel": kernel,
                 "algorithmic_bytes_per_launch": step.T_kept * bytes_per_row,
+                "bytes_per_kept_row": bytes_per_row,
                 "launch_ms": loss_ms, "peak_source": peak_src}
+    return dict(b=b, d=d, step=step, K=K, elapsed_ms=elapsed_ms, value=value, loss_ms=loss_ms,
+                select_ms=select_ms, launches=launches, use_graph=use_graph, clocks=clocks,
+                roofline=roofline)
+
+
+def sub_record(args, w, r, warmup):
+    """A further workload's line inside the main one: the same measurements, without the
+    end-to-end, CPU-baseline and side legs."""
+    step = r["step"]
+    return {"value": r["value"], "unit": UNIT, "steps": r["K"], "warmup": warmup,
+            "ms_per_step": r["elapsed_ms"] / r["K"], "cuda_graph": r["use_graph"],
+            "gpu_launches": int(r["launches"]), "roofline": r["roofline"], "clocks": r["clocks"],
+            "config": dict(workload_desc(w, r["b"]["T"], step.T_kept, step.K), loss=args.loss),
+            "path_overhead": {"select_ms": r["select_ms"],
+                              "other_ms": r["elapsed_ms"] / r["K"] - r["select_ms"] - r["loss_ms"]},
+            "loss_value": float(step.loss.item())}
+
+
+def main():
+    args = parse()
+    import dataclasses
+    from paper_2609_36932_gb300 import workloads
+    w = workloads.get(args.config)
+    if args.prompts > 0:
+        w = dataclasses.replace(w, P=args.prompts)
+    if args.group > 0:
+        w = dataclasses.replace(w, G=args.group)
+    if args.impl == "reference":
+        if args.loss in ("lmhead", "lmhead-gspo"):
+            if dist_env()[0] == 0:
+                run_reference_lmhead(args, w)
+            return
+        run_reference(args, w)
+        return
+    if args.loss in ("lmhead", "lmhead-gspo"):
+        run_lmhead(args, w)
+        return
+    import torch
+    import torch.distributed as dist
+    import paper_2609_36932_gb300 as g
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    g.lib()
+
+    r = timed_steps(args, w, rank_seed(args.seed, rank), world, local, dev, args.steps,
+                    args.warmup)
+    b, d, step = r["b"], r["d"], r["step"]
+    K, elapsed_ms, loss_ms, select_ms = r["K"], r["elapsed_ms"], r["loss_ms"], r["select_ms"]
+    peak = r["roofline"]["peak"]
+    stream = torch.cuda.current_stream()
 
     # the logp-only forward over the same kept rows (old/reference policy evaluation); one read
     logp_fwd = None
@@ -1038,7 +1097,10 @@ def main():
                "d2h_bytes_per_step": int(d2h_e // args.e2e_steps), "steps": args.e2e_steps,
                "host_inputs_bytes": int(h2d),
                "transfer": "selection inputs and per-token log-probs whole; logits of the kept "
-                           "rollouts only (grpo_upload_kept), after the selection"}
+                           "rollouts only (grpo_upload_kept), after the selection",
+               "returned": "the loss (8 bytes) and the selection the host needs (kept counts, "
+                           "kept per prompt, keep flags, kept offsets); logp and dlogits stay on "
+                           "the device, where the backward pass consumes them"}
         del host
 
     cpu = None
@@ -1048,16 +1110,17 @@ def main():
         else:
             cpu = cpu_baseline_ours(w, b, step, d, args.cpu_seconds)
 
+    line = None
     if rank == 0:
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded; shapes and distributions of the paper's GRPO batches)",
             "config": dict(workload_desc(w, b["T"], step.T_kept, step.K), loss=args.loss),
-            "gpu_launches": int(launches), "cuda_graph": use_graph,
-            "roofline": roofline, "e2e": e2e,
-            "cpu_baseline": cpu, "clocks": clocks, "logp_fwd": logp_fwd, "lmhead": lmhead,
+            "gpu_launches": int(r["launches"]), "cuda_graph": r["use_graph"],
+            "roofline": r["roofline"], "e2e": e2e,
+            "cpu_baseline": cpu, "clocks": r["clocks"], "logp_fwd": logp_fwd, "lmhead": lmhead,
             "path_overhead": {"select_ms": select_ms,
                               "other_ms": elapsed_ms / K - select_ms - loss_ms,
                               "note": "select_ms: advantage, prune, compaction (and the kept-count"
@@ -1065,6 +1128,24 @@ def main():
                                       " of the step (host ARS update, launch gaps)"},
             "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,
         }
+
+    # the other full-size Qwen-vocabulary workloads, each in its own sub-record
+    extra = [x for x in args.extra_configs.split(",") if x] if args.config in ("qwen", "2") else []
+    if extra and args.prompts == 0 and args.group == 0:
+        del r, b, d, step
+        torch.cuda.empty_cache()
+        configs = {}
+        for name in extra:
+            w2 = workloads.get(name)
+            steps2 = max(1, int(round(args.extra_seconds * 1e3 / EXTRA_MS_GUESS.get(name, 20.0))))
+            r2 = timed_steps(args, w2, rank_seed(args.seed, rank), world, local, dev, steps2,
+                             args.warmup)
+            configs[name] = sub_record(args, w2, r2, args.warmup)
+            del r2
+            torch.cuda.empty_cache()
+        if line is not None:
+            line["configs"] = configs
+    if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()

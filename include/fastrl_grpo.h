@@ -15,7 +15,8 @@
  *   grpo_lmhead_loss_fwd_bwd  the output layer fused with the loss:     (Sec. 3.2, Eqs. 1-3)
  *                           logits on the tensor cores, never stored whole; dhidden, dweight
  *     (grpo_lmhead_logp_fwd: log-probabilities alone from hidden states;
- *      grpo_lmhead_gspo_loss_fwd_bwd: the same with GSPO's sequence-level loss)
+ *      grpo_lmhead_gspo_loss_fwd_bwd: the same with GSPO's sequence-level loss;
+ *      grpo_lmhead_grad: dhidden and dweight from given dlogits)
  *   grpo_upload_kept        host-to-device copy of the kept rows only  (Sec. 3.2)
  *   adaptive_rollout_count  adaptive rollout sampling, on the host     (Eqs. 10-14, Algorithm 1)
  *
@@ -23,8 +24,9 @@
  *   - Every call returns a grpo_status; GRPO_OK is 0.  On failure, grpo_last_error() returns a
  *     message for the calling thread.  No C++ exception and no abort crosses this boundary.
  *   - Buffers marked "device" are device pointers owned by the caller (for instance memory held
- *     by PyTorch tensors).  The library never allocates or frees device memory (the cuBLASLt
- *     GEMMs of grpo_lmhead_loss_fwd_bwd also run in the caller's workspace).  Scratch memory
+ *     by PyTorch tensors).  The library never allocates or frees device memory, with one
+ *     exception: grpo_loss_fwd_bwd_noalloc's fixed 2 MiB scratch array, which every GPU that
+ *     loads the library holds until the process exits.  Scratch memory otherwise
  *     comes from a caller workspace: a call with ws == NULL and ws_bytes != NULL only writes the
  *     size it needs into *ws_bytes and enqueues nothing.  The real call passes ws (256-byte
  *     aligned) with *ws_bytes >= that size, or ws == NULL and ws_bytes == NULL when the size
@@ -54,8 +56,8 @@ typedef enum {
   GRPO_ERR_UNSUPPORTED = 2,  /* a valid request outside this build's limits (stated per call) */
   GRPO_ERR_WORKSPACE = 3,    /* workspace missing or smaller than the size query returned */
   GRPO_ERR_CUDA = 4,         /* a CUDA runtime call failed; grpo_last_error() names it */
-  GRPO_ERR_TIMEOUT = 5,      /* reserved for host-side waits */
-  GRPO_ERR_DEVICE_CHECK = 6  /* reserved for callers that turn device status bits into a status */
+  GRPO_ERR_TIMEOUT = 5,      /* a device wait ran out (grpo_check_status on a status word) */
+  GRPO_ERR_DEVICE_CHECK = 6  /* a kernel flagged bad data (grpo_check_status on a status word) */
 } grpo_status;
 
 typedef enum { GRPO_DTYPE_F32 = 0, GRPO_DTYPE_BF16 = 1 } grpo_dtype;
@@ -73,6 +75,17 @@ const char* grpo_version(void);
 
 /* Number of kernels this process has launched through the library so far (host counter). */
 uint64_t grpo_kernel_launches(void);
+
+/*
+ * grpo_check_status — turn a device status word, read back by the caller after synchronising
+ * the stream its kernels ran on, into a grpo_status (host only, no GPU work; no counterpart in
+ * the paper).  0 gives GRPO_OK.  GRPO_DEVFLAG_TIMEOUT gives GRPO_ERR_TIMEOUT: a bounded wait
+ * gave up and that launch's results are invalid.  Otherwise any bit (GRPO_DEVFLAG_BAD_TOKEN,
+ * GRPO_DEVFLAG_NONFINITE, unknown bits) gives GRPO_ERR_DEVICE_CHECK: the flagged rows have the
+ * documented NaN log-prob / zero gradient and the other rows are valid.  grpo_last_error() then
+ * names every bit that is set.
+ */
+grpo_status grpo_check_status(int32_t status_word);
 
 /*
  * grpo_advantage — group-relative advantage, Eq. 5 (Sec. 3.2):
@@ -317,12 +330,12 @@ grpo_status grpo_gspo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype,
  * chunk_rows: rows of dlogits held at a time (rounded up to a multiple of 128); 0 picks the
  *   largest count that fits a 4 GiB bf16 chunk.  Smaller chunks need less workspace.
  * Workspace: per row 1.3 KB of softmax statistics, the chunk of dlogits (unless dlogits_out) and
- *   32 MiB for cuBLASLt, whose two GEMMs per chunk run with that scratch on `stream`.
- * Kernels: pass 1 (statistics) and pass 2 (dlogits, per chunk) are tcgen05 GEMM kernels with TMA
- *   operand loads and TMEM accumulators, one CTA per SM; a row kernel applies Eqs. 1-3 between
- *   them.  Limits: n_rows < 2^31; V >= 1; D >= 8.  Errors: GRPO_ERR_INVALID_ARG for bad sizes,
- *   alignment, NULL required pointers; GRPO_ERR_CUDA when a launch, the tensor-map encoder or
- *   cuBLASLt fails.
+ *   the f32 partial products of a split K (see grpo_lmhead_grad).
+ * Kernels: pass 1 (statistics), pass 2 (dlogits, per chunk) and the two products per chunk
+ *   (grpo_lmhead_grad's) are tcgen05 kernels with TMA operand loads and TMEM accumulators, one
+ *   CTA per SM; a row kernel applies Eqs. 1-3 between the passes.  Limits: n_rows < 2^31;
+ *   V >= 1; D >= 8.  Errors: GRPO_ERR_INVALID_ARG for bad sizes, alignment, NULL required
+ *   pointers; GRPO_ERR_CUDA when a launch or the tensor-map encoder fails.
  */
 grpo_status grpo_lmhead_loss_fwd_bwd(const void* hidden, int64_t hidden_stride,
                                      const int64_t* row_index, int64_t n_rows, const void* weight,
@@ -336,6 +349,34 @@ grpo_status grpo_lmhead_loss_fwd_bwd(const void* hidden, int64_t hidden_stride,
                                      float* logp_out, double* row_loss_out, double* loss_out,
                                      int32_t* status, int64_t chunk_rows, void* ws,
                                      size_t* ws_bytes, grpo_stream_t stream);
+
+/*
+ * grpo_lmhead_grad — the chain rule through the output layer z = hidden * weight^T for given
+ * dlogits (Sec. 3.2: the kept trajectories' hidden states -> logits -> Eqs. 1-3), for instance
+ * the bf16 dlogits grpo_loss_fwd_bwd wrote for the kept rows:
+ *   dhidden[t, :] = sum_v dlogits[t, v] * weight[v, :]
+ *   dweight[v, :] = sum_t dlogits[t, v] * hidden[t, :]   (+ the old dweight with accumulate_dweight)
+ * These are the two products grpo_lmhead_loss_fwd_bwd runs after its dlogits pass, on the same
+ * tcgen05 kernel: bf16 operands staged by TMA, f32 accumulation in tensor memory, each output
+ * rounded once (bf16 dhidden to nearest even).
+ * dlogits: device bf16 [n_rows, V] with row stride dlogits_stride (>= V, a multiple of 8).
+ * hidden:  device bf16 [n_rows, D] with row stride hidden_stride (>= D, a multiple of 8).
+ * weight:  device bf16 [V, D], dense.  D: a positive multiple of 8.  dlogits, hidden and weight
+ *   16-byte aligned.
+ * dhidden: device [n_rows, D] dense, bf16 or f32 per dhidden_dtype, aligned to its element;
+ *   NULL skips it (weight may then be NULL).  dweight: device f32 [V, D]; NULL skips it (hidden
+ *   may then be NULL).  n_rows = 0: dweight is zeroed (or left as is when accumulated).
+ * status: device i32, nullable (GRPO_DEVFLAG_TIMEOUT if a bounded wait ran out).
+ * Workspace: f32 partial products when a product's K is split for load balance (the size query
+ *   as everywhere; it may be 0).  Deterministic for a given input and device.
+ * Errors: GRPO_ERR_INVALID_ARG for bad sizes, strides, alignment or NULL required pointers;
+ *   GRPO_ERR_CUDA when a launch or the tensor-map encoder fails.
+ */
+grpo_status grpo_lmhead_grad(const void* dlogits, int64_t dlogits_stride, int64_t n_rows,
+                             int32_t V, const void* hidden, int64_t hidden_stride,
+                             const void* weight, int32_t D, void* dhidden, int32_t dhidden_dtype,
+                             float* dweight, int32_t accumulate_dweight, int32_t* status, void* ws,
+                             size_t* ws_bytes, grpo_stream_t stream);
 
 /*
  * grpo_lmhead_logp_fwd — log-probability of the sampled token from hidden states, for the old- and
@@ -433,7 +474,13 @@ grpo_status grpo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype, int6
  *   - n_rows above 262144 with row_loss_out == NULL returns GRPO_ERR_UNSUPPORTED (pass
  *     row_loss_out, which needs no scratch, or split the rows into several calls).
  *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
- *     with that device current; make that first call before any stream capture.
+ *     with that device current, and keeps it for the life of the process.  Under lazy module
+ *     loading (the CUDA default) that lookup may also make the driver load this library's GPU
+ *     code, array included, which allocates device memory.  So a caller that must not allocate
+ *     after start-up makes one call on each device during its start-up phase, before any stream
+ *     capture; a call with n_rows = 0 and row_loss_out == NULL is enough (it sets loss_out to 0).
+ *   - A device reset (cudaDeviceReset) unloads the array and invalidates the kept address; this
+ *     entry must not be called on a device after it has been reset in the same process.
  *   - Every call uses the same array, which keeps the previous call's contents; each call
  *     writes every entry it later reads, so nothing needs clearing.  Calls whose GPU work
  *     overlaps (for instance on two streams at once) race on the array: order them on one

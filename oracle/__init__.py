@@ -41,7 +41,7 @@ def lib():
         L.oracle_compact.restype = _i32
         L.oracle_loss.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p, _c_p, _c_p, _c_p,
                                   _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p, _i32, _c_p,
-                                  _c_p, _c_p, _c_p, _c_p]
+                                  _c_p, _c_p, _c_p, _c_p, _c_p]
         L.oracle_loss.restype = _i32
         L.oracle_gspo_loss.argtypes = [_c_p, _i32, _i64, _c_p, _i32, _c_p, _c_p, _c_p, _c_p,
                                        _c_p, _c_p, _i64, _i64, _f32, _f32, _f32, _c_p, _i32,
@@ -55,6 +55,9 @@ def lib():
                                               _c_p, _c_p, _c_p, _i64, _i64, _f32, _f32, _f32,
                                               _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
         L.oracle_lmhead_gspo_loss.restype = _i32
+        L.oracle_lmhead_grad.argtypes = [_c_p, _c_p, _c_p, _i64, _i32, _i32, _c_p, _c_p, _c_p,
+                                         _c_p]
+        L.oracle_lmhead_grad.restype = _i32
         L.oracle_logp.argtypes = [_c_p, _i32, _i64, _c_p, _i64, _i32, _c_p, _c_p]
         L.oracle_logp.restype = _i32
         L.oracle_round_bf16.argtypes = [_f64]
@@ -152,8 +155,9 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
     """Eqs. 1-3.  `logits` is a float32 array or a uint16 array of bf16 bit patterns (or, with
     logits_dtype=2, float64).
 
-    Returns dict(loss, logp [n_rows] f64, rho, row_loss, dlogits (f32 array or uint16 bf16
-    bits, [n_rows, V]) and, with want_f64, dlogits_f64).
+    Returns dict(loss, logp [n_rows] f64, rho, row_loss, g (each row's gradient factor g_t, so
+    that dlogits[t] = w_t * g_t * (onehot(y) - softmax)), dlogits (f32 array or uint16 bf16 bits,
+    [n_rows, V]) and, with want_f64, dlogits_f64).
     """
     lg = np.ascontiguousarray(logits)
     if logits_dtype is None:
@@ -180,15 +184,16 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
     logp = np.empty(max(n_rows, 1), np.float64)
     rho = np.empty(max(n_rows, 1), np.float64)
     rl = np.empty(max(n_rows, 1), np.float64)
+    g = np.empty(max(n_rows, 1), np.float64)
     total = np.zeros(1, np.float64)
     rc = lib().oracle_loss(_p(lg), logits_dtype, stride, _p(ri), n_rows, V, _p(y_), _p(old), _p(ref),
                            _p(a), _p(rr), float(eps_low), float(eps_high), float(beta), agg_mode,
                            int(denom_tokens), _p(so), int(n_seq), _p(dl), dlogits_dtype, _p(d64),
-                           _p(logp), _p(rho), _p(rl), _p(total))
+                           _p(logp), _p(rho), _p(rl), _p(total), _p(g))
     if rc != 0:
         raise ValueError("oracle_loss: bad arguments")
     return dict(loss=float(total[0]), logp=logp[:n_rows], rho=rho[:n_rows], row_loss=rl[:n_rows],
-                dlogits=dl, dlogits_f64=d64)
+                g=g[:n_rows], dlogits=dl, dlogits_f64=d64)
 
 
 def lmhead_loss(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2,
@@ -236,6 +241,27 @@ def lmhead_loss(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *, eps_
         raise ValueError("oracle_lmhead_loss: bad arguments")
     return dict(loss=float(total[0]), logp=logp[:n_rows], row_loss=rl[:n_rows], logits=lg,
                 dlogits=dl, dhidden=dh, dweight=dw, dhidden_abs=dha, dweight_abs=dwa)
+
+
+def lmhead_grad(dlogits, hidden, weight, want_bounds=False):
+    """The chain rule through z = hidden @ weight.T for given dlogits [n_rows, V]: returns
+    dict(dhidden = dlogits @ weight, dweight = dlogits.T @ hidden and, with want_bounds, the sums
+    of absolute products dhidden_abs and dweight_abs), all fp64 (bf16 inputs widen exactly)."""
+    dl = np.ascontiguousarray(dlogits, dtype=np.float64)
+    h = np.ascontiguousarray(hidden, dtype=np.float64)
+    w = np.ascontiguousarray(weight, dtype=np.float64)
+    n_rows, V = dl.shape
+    D = w.shape[1]
+    if w.shape[0] != V or h.shape != (n_rows, D):
+        raise ValueError("dlogits, hidden and weight disagree on their sizes")
+    dh = np.empty((n_rows, D), np.float64)
+    dw = np.empty((V, D), np.float64)
+    dha = np.empty((n_rows, D), np.float64) if want_bounds else None
+    dwa = np.empty((V, D), np.float64) if want_bounds else None
+    if lib().oracle_lmhead_grad(_p(h), _p(w), _p(dl), n_rows, V, D, _p(dh), _p(dw), _p(dha),
+                                _p(dwa)) != 0:
+        raise ValueError("oracle_lmhead_grad: bad arguments")
+    return dict(dhidden=dh, dweight=dw, dhidden_abs=dha, dweight_abs=dwa)
 
 
 def lmhead_gspo_loss(hidden, weight, y, old_logp, ref_logp, adv, seq_rollout, seq_row_off, *,

@@ -105,7 +105,7 @@ extern "C" int oracle_lmhead_loss(const double* hidden, const double* weight, in
   const int rc = oracle_loss(z.data(), 2, V, nullptr, n_rows, V, y, old_logp, ref_logp, adv,
                              row_rollout, eps_low, eps_high, beta, agg_mode, denom_tokens, seq_off,
                              n_seq, nullptr, 0, dl.data(), logp.data(), rho.data(), rl.data(),
-                             &total);
+                             &total, nullptr);
   if (rc != 0) return rc;
   copy_out(dl, nz, dlogits_out);
   copy_out(logp, n_rows, logp_out);
@@ -141,6 +141,18 @@ extern "C" int oracle_lmhead_gspo_loss(const double* hidden, const double* weigh
   copy_out(dl, nz, dlogits_out);
   copy_out(logp, n_rows, logp_out);
   if (loss_out) *loss_out = total;
+  chain_rule(hidden, weight, n_rows, V, D, dl, dhidden, dweight, dhidden_abs, dweight_abs);
+  return 0;
+}
+
+// The chain rule alone, for dlogits given in fp64: dh = dlogits * W and dW = dlogits^T * h, with
+// the sums of absolute products (the error bound's scale) when asked for.
+extern "C" int oracle_lmhead_grad(const double* hidden, const double* weight, const double* dlogits,
+                                  int64_t n_rows, int V, int D, double* dhidden, double* dweight,
+                                  double* dhidden_abs, double* dweight_abs) {
+  if (n_rows < 0 || V < 1 || D < 1) return 1;
+  const int64_t nz = n_rows * (int64_t)V;
+  std::vector<double> dl(dlogits, dlogits + nz);
   chain_rule(hidden, weight, n_rows, V, D, dl, dhidden, dweight, dhidden_abs, dweight_abs);
   return 0;
 }

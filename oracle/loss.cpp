@@ -88,7 +88,7 @@ extern "C" int oracle_loss(const void* logits, int logits_dtype, int64_t row_str
                            int agg_mode, int64_t denom_tokens, const int64_t* seq_off,
                            int64_t n_seq, void* dlogits, int dlogits_dtype, double* dlogits_f64,
                            double* logp_out, double* rho_out, double* row_loss_out,
-                           double* loss_out) {
+                           double* loss_out, double* g_out) {
   if (n_rows < 0 || V < 1 || row_stride < V) return 1;
   if (agg_mode == 0 && denom_tokens <= 0) return 1;
   if (agg_mode == 1 && (seq_off == nullptr || n_seq <= 0)) return 1;
@@ -107,6 +107,7 @@ extern "C" int oracle_loss(const void* logits, int logits_dtype, int64_t row_str
       }
       if (logp_out) logp_out[t] = nan;
       if (rho_out) rho_out[t] = nan;
+      if (g_out) g_out[t] = nan;
       row_loss[t] = 0.0;
       continue;
     }
@@ -149,6 +150,7 @@ extern "C" int oracle_loss(const void* logits, int logits_dtype, int64_t row_str
     }
     if (logp_out) logp_out[t] = logp;
     if (rho_out) rho_out[t] = rho;
+    if (g_out) g_out[t] = g;
   }
 
   double total = 0.0;

@@ -47,14 +47,16 @@ int oracle_compact(const uint8_t* keep, const int64_t* off, int n_rollouts, int3
 /* Eqs. 1-3: GRPO token loss and dlogits; see loss.cpp.
  * logits_dtype 0 = f32, 1 = bf16 bit patterns (uint16), 2 = f64.  dlogits_dtype 0 = f32,
  * 1 = bf16 bits.
- * dlogits_f64 (nullable) receives the unrounded fp64 gradient.  rho_out (nullable) the ratios. */
+ * dlogits_f64 (nullable) receives the unrounded fp64 gradient.  rho_out (nullable) the ratios.
+ * g_out (nullable) each row's g_t = -(c*rho*A + beta*(exp(x) - 1)), the factor that multiplies
+ * w_t*([v == y] - softmax_v) in its dlogits (NaN for an invalid token). */
 int oracle_loss(const void* logits, int logits_dtype, int64_t row_stride, const int64_t* row_index,
                 int64_t n_rows, int V, const int32_t* y, const float* old_logp,
                 const float* ref_logp, const float* adv, const int32_t* row_rollout, float eps_low,
                 float eps_high, float beta, int agg_mode, int64_t denom_tokens,
                 const int64_t* seq_off, int64_t n_seq, void* dlogits, int dlogits_dtype,
                 double* dlogits_f64, double* logp_out, double* rho_out, double* row_loss_out,
-                double* loss_out);
+                double* loss_out, double* g_out);
 
 /* GSPO's sequence-level loss (length-normalised sequence ratio, clipped per sequence) over kept
  * rollouts; see loss.cpp.  Sequence k owns rows [seq_row_off[k], seq_row_off[k+1]) of the
@@ -111,6 +113,13 @@ double oracle_ars_get(void* st, int what); /* 0: G'_ref or NaN, 1: G'_t or NaN *
 
 /* Worker threads the loss uses (OpenMP); 0 keeps the runtime default.  Returns the count. */
 int oracle_set_threads(int n);
+
+/* The chain rule through z = hidden * weight^T alone, for given fp64 dlogits [n_rows, V]:
+ * dhidden = dlogits * weight, dweight = dlogits^T * hidden (each nullable), and the sums of the
+ * absolute products (nullable); see lmhead.cpp. */
+int oracle_lmhead_grad(const double* hidden, const double* weight, const double* dlogits,
+                       int64_t n_rows, int V, int D, double* dhidden, double* dweight,
+                       double* dhidden_abs, double* dweight_abs);
 
 #ifdef __cplusplus
 }

@@ -7,8 +7,8 @@ synthetic inputs.  Importing the package does not load the library; the first ca
 from .binding import (ArsState, GrpoError, adaptive_rollout_count, check_status, grpo_advantage,
                       grpo_ars_deserialize, grpo_ars_init, grpo_ars_serialize, grpo_compact,
                       grpo_gspo_loss_fwd_bwd, grpo_kernel_launches, grpo_last_error,
-                      grpo_lmhead_dlogits_stride, grpo_lmhead_gspo_loss_fwd_bwd,
-                      grpo_lmhead_logp_fwd, grpo_lmhead_loss_fwd_bwd, grpo_lmhead_tune,
+                      grpo_lmhead_dlogits_stride, grpo_lmhead_grad,
+                      grpo_lmhead_gspo_loss_fwd_bwd, grpo_lmhead_logp_fwd, grpo_lmhead_loss_fwd_bwd, grpo_lmhead_tune,
                       grpo_logp_fwd, grpo_loss_fwd_bwd, grpo_loss_fwd_bwd_dev,
                       grpo_loss_fwd_bwd_noalloc, grpo_loss_tune, grpo_prune, grpo_sum_f64,
                       grpo_upload_kept, lib, library_path, version)
@@ -16,7 +16,8 @@ from .binding import (ArsState, GrpoError, adaptive_rollout_count, check_status,
 __all__ = ["ArsState", "GrpoError", "adaptive_rollout_count", "check_status", "grpo_advantage",
            "grpo_ars_deserialize", "grpo_ars_init", "grpo_ars_serialize", "grpo_compact",
            "grpo_gspo_loss_fwd_bwd", "grpo_kernel_launches", "grpo_last_error",
-           "grpo_lmhead_dlogits_stride", "grpo_lmhead_gspo_loss_fwd_bwd", "grpo_lmhead_logp_fwd",
+           "grpo_lmhead_dlogits_stride", "grpo_lmhead_grad", "grpo_lmhead_gspo_loss_fwd_bwd",
+           "grpo_lmhead_logp_fwd",
            "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_tune", "grpo_logp_fwd", "grpo_loss_fwd_bwd",
            "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_loss_tune", "grpo_prune",
            "grpo_sum_f64", "grpo_upload_kept", "lib", "library_path", "version"]

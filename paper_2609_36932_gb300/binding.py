@@ -30,10 +30,12 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
                 6: "GRPO_ERR_DEVICE_CHECK"}
 
 # Every function include/fastrl_grpo.h declares.
-EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_advantage",
+EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_check_status",
+           "grpo_advantage",
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
            "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
            "grpo_lmhead_logp_fwd", "grpo_lmhead_tune", "grpo_lmhead_gspo_loss_fwd_bwd",
+           "grpo_lmhead_grad",
            "grpo_loss_tune", "grpo_test_skip_copy", "grpo_test_fail_launch", "grpo_ars_init",
            "adaptive_rollout_count",
            "grpo_ars_serialize", "grpo_ars_deserialize"]
@@ -75,6 +77,8 @@ def lib():
     L.grpo_version.argtypes = []
     L.grpo_kernel_launches.restype = ctypes.c_uint64
     L.grpo_kernel_launches.argtypes = []
+    L.grpo_check_status.argtypes = [_i32]
+    L.grpo_check_status.restype = _i32
     L.grpo_advantage.argtypes = [_c_p, _i32, _i32, _i32, _c_p, _c_p, _c_p]
     L.grpo_advantage.restype = _i32
     L.grpo_prune.argtypes = [_c_p, _c_p, _f32, _c_p, _c_p, _i32, _i32, _i64, _i32, _i32, _f32, _i32,
@@ -117,6 +121,9 @@ def lib():
     L.grpo_lmhead_logp_fwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p, _c_p, _c_p,
                                        _c_p, _c_p, _c_p]
     L.grpo_lmhead_logp_fwd.restype = _i32
+    L.grpo_lmhead_grad.argtypes = [_c_p, _i64, _i64, _i32, _c_p, _i64, _c_p, _i32, _c_p, _i32,
+                                   _c_p, _i32, _c_p, _c_p, ctypes.POINTER(ctypes.c_size_t), _c_p]
+    L.grpo_lmhead_grad.restype = _i32
     L.grpo_lmhead_gspo_loss_fwd_bwd.argtypes = [_c_p, _i64, _c_p, _i64, _c_p, _i32, _i32, _c_p,
                                                 _c_p, _c_p, _c_p, _c_p, _c_p, _i32, _i64, _f32,
                                                 _f32, _f32, _c_p, _i32, _c_p, _i32, _c_p, _c_p,
@@ -430,6 +437,49 @@ def grpo_lmhead_logp_fwd(hidden, weight, y, *, row_index=None, n_rows: int | Non
     wp, size = _ws_args(wst)
     _check(L.grpo_lmhead_logp_fwd(*head, wp, size, _stream(stream)))
     return dict(logp=logp_out, ws=wst)
+
+
+def grpo_lmhead_grad(dlogits, hidden, weight, *, n_rows: int | None = None, dhidden=None,
+                     dhidden_dtype=None, dweight=None, accumulate_dweight: bool = False,
+                     want_dhidden: bool = True, want_dweight: bool = True, status=None, ws=None,
+                     stream=None):
+    """dhidden = dlogits @ weight and dweight (+)= dlogits^T @ hidden on the tensor cores (the
+    chain rule through the output layer, see the header).  dlogits bf16 [n_rows, >= V] with unit
+    stride along V; hidden bf16 [n_rows, D]; weight bf16 [V, D].  Returns dict(dhidden, dweight,
+    ws)."""
+    torch = _torch()
+    for t, nm in ((dlogits, "dlogits"), (hidden, "hidden"), (weight, "weight")):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or t.dim() != 2 or t.stride(1) != 1:
+            raise TypeError("%s must be a 2-D bf16 CUDA tensor with unit inner stride" % nm)
+    if not weight.is_contiguous() or weight.shape[1] != hidden.shape[1]:
+        raise ValueError("weight must be a contiguous [V, D] tensor")
+    V, D = weight.shape
+    if n_rows is None:
+        n_rows = dlogits.shape[0]
+    dev = dlogits.device
+    if dhidden_dtype is None:
+        dhidden_dtype = dhidden.dtype if dhidden is not None else torch.bfloat16
+    dht = GRPO_DTYPE_BF16 if dhidden_dtype in (torch.bfloat16, "bf16") else GRPO_DTYPE_F32
+    ht = torch.bfloat16 if dht == GRPO_DTYPE_BF16 else torch.float32
+    if want_dhidden and dhidden is None:
+        dhidden = torch.empty((max(int(n_rows), 1), D), dtype=ht, device=dev)
+    if want_dhidden:
+        _need(dhidden, ht, n_rows * D, "dhidden")
+    if want_dweight and dweight is None:
+        dweight = torch.empty((V, D), dtype=torch.float32, device=dev)
+    if want_dweight:
+        _need(dweight, torch.float32, V * D, "dweight")
+    L = lib()
+    head = (_ptr(dlogits), int(dlogits.stride(0)), int(n_rows), int(V), _ptr(hidden),
+            int(hidden.stride(0)), _ptr(weight), int(D), _ptr(dhidden if want_dhidden else None),
+            dht, _ptr(dweight if want_dweight else None), int(bool(accumulate_dweight)),
+            _ptr(status))
+    need = ctypes.c_size_t(0)
+    _check(L.grpo_lmhead_grad(*head, None, ctypes.byref(need), _stream(stream)))
+    wst = _workspace(need.value, dev, ws)
+    wp, size = _ws_args(wst)
+    _check(L.grpo_lmhead_grad(*head, wp, size, _stream(stream)))
+    return dict(dhidden=dhidden, dweight=dweight, ws=wst)
 
 
 def _lmhead_common(hidden, weight, row_index, n_rows, dhidden, dhidden_dtype, dweight,
@@ -837,11 +887,8 @@ def adaptive_rollout_count(state: ArsState, kept_per_prompt, step: int, total_st
 
 
 def check_status(status) -> int:
-    """Raise GrpoError(GRPO_ERR_DEVICE_CHECK) if a device status word has bits set."""
+    """grpo_check_status on a device status word (a tensor, read back here, or an int): raises
+    GrpoError (GRPO_ERR_TIMEOUT or GRPO_ERR_DEVICE_CHECK) if any bit is set; returns the word."""
     v = int(status.item()) if hasattr(status, "item") else int(status)
-    if v:
-        names = [nm for bit, nm in ((DEVFLAG_BAD_TOKEN, "bad token id"),
-                                    (DEVFLAG_NONFINITE, "non-finite logits"),
-                                    (DEVFLAG_TIMEOUT, "copy wait timed out")) if v & bit]
-        raise GrpoError(6, "device status 0x%x: %s" % (v, ", ".join(names)))
+    _check(lib().grpo_check_status(ctypes.c_int32(v)))
     return v

@@ -1,8 +1,8 @@
 """Build libfastrl_grpo.so (the CUDA path) in-tree for sm_103a.
 
-Each .cu file is compiled by nvcc in parallel, then linked with the static CUDA runtime (and
-the toolkit's cuBLASLt, for the two plain GEMMs of the output-layer loss) into
-paper_2609_36932_gb300/_build/libfastrl_grpo.so.  Nothing is installed outside the tree.
+Each .cu file is compiled by nvcc in parallel, then linked with the static CUDA runtime (and no
+other library) into paper_2609_36932_gb300/_build/libfastrl_grpo.so.  Nothing is installed
+outside the tree.
 """
 from __future__ import annotations
 
@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libfastrl_grpo.so")
 SOURCES = ["api.cu", "advantage.cu", "prune.cu", "compact.cu", "loss.cu", "gspo.cu", "reduce.cu",
-           "lmhead.cu"]
+           "lmhead.cu", "gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I", INCLUDE, "-I", CSRC]
@@ -69,9 +69,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
                 raise RuntimeError("nvcc failed on %s" % src)
             objs.append(obj)
     tmp = LIB + ".tmp.%d" % os.getpid()
-    cuda_lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(cc))), "lib64")
-    r = subprocess.run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs,
-                        "-L" + cuda_lib, "-lcublasLt", "-Xlinker", "-rpath=" + cuda_lib],
+    r = subprocess.run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs],
                        capture_output=True, text=True)
     if r.returncode != 0:
         sys.stderr.write(r.stdout + r.stderr)

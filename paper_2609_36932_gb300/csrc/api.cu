@@ -72,6 +72,20 @@ extern "C" uint64_t grpo_kernel_launches(void) {
   return g_launches.load(std::memory_order_relaxed);
 }
 
+extern "C" grpo_status grpo_check_status(int32_t status_word) {
+  clear_error();
+  if (status_word == 0) return GRPO_OK;
+  const uint32_t v = (uint32_t)status_word;
+  const uint32_t known = GRPO_DEVFLAG_BAD_TOKEN | GRPO_DEVFLAG_NONFINITE | GRPO_DEVFLAG_TIMEOUT;
+  fail(GRPO_OK, "device status 0x%x:%s%s%s%s", v,
+       (v & GRPO_DEVFLAG_TIMEOUT) ? " copy wait timed out;" : "",
+       (v & GRPO_DEVFLAG_BAD_TOKEN) ? " token id outside [0, V);" : "",
+       (v & GRPO_DEVFLAG_NONFINITE) ? " non-finite log-sum-exp or log-prob;" : "",
+       (v & ~known) ? " unknown bits;" : "");
+  // a timed-out wait invalidates the launch's results; the data checks only flag rows
+  return (v & GRPO_DEVFLAG_TIMEOUT) ? GRPO_ERR_TIMEOUT : GRPO_ERR_DEVICE_CHECK;
+}
+
 extern "C" grpo_status grpo_ars_init(grpo_ars_state* st, int32_t G1) {
   clear_error();
   if (st == nullptr) return fail(GRPO_ERR_INVALID_ARG, "grpo_ars_init: state is NULL");

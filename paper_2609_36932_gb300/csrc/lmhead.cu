@@ -15,7 +15,8 @@
 //     scalars of each row (the same formulas as the fused loss kernel).
 //   Pass 2 (lmhead_tile_kernel<true>), for each chunk of rows: the tiles recomputed and
 //     dlogits = coef * ([v == y] - softmax(z)_v) written in bf16 to a chunk buffer.
-//   Two plain GEMMs per chunk (cuBLASLt): dh = dlogits * W and dW (+)= dlogits^T * h.
+//   Two products per chunk on the same tensor-core machinery (gemm.cu): dh = dlogits * W and
+//     dW (+)= dlogits^T * h.
 //
 // Kernel roles (320 threads, one CTA per SM: 214 KB of shared memory, all 512 TMEM columns).  A
 // tile is a pair of 128-row blocks of h against 256 vocabulary entries, so each weight stage
@@ -43,7 +44,6 @@
 // for its MMAs, and warp 1 frees the tensor memory before the CTA exits.
 #include <cuda.h>
 #include <cuda_bf16.h>
-#include <cublasLt.h>
 
 #include <algorithm>
 #include <atomic>
@@ -51,6 +51,8 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "gemm.cuh"
+#include "tcgen05.cuh"
 #include "trace.cuh"
 #include "rowops.cuh"
 
@@ -76,98 +78,26 @@ constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + 8 * kBars +
                               kStageOutBytes;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int64_t kDefaultChunkBytes = 4ll << 30;  // dlogits chunk buffer
-constexpr size_t kLtWorkspace = 32u << 20;
 
-// Instruction descriptor of tcgen05.mma.kind::f16: f32 accumulator (bits 4-5 = 1), bf16 A and B
-// (bits 7-9, 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at 24-28.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
+// Instruction descriptor of tcgen05.mma.kind::f16 for the tile passes: f32 accumulator, bf16 A
+// (h) and B (W), both K-major (D contiguous), N = BN, M = BM.
+constexpr uint32_t kIdesc = tc::idesc_bf16(BM, BN, false, false);
 
-// Shared-memory matrix descriptor for a K-major operand in the 128-byte swizzle layout that TMA
-// writes with CU_TENSOR_MAP_SWIZZLE_128B: rows of 128 bytes, 8-row atoms 1024 bytes apart (the
-// stride byte offset), start address >> 4 in bits 0-13, descriptor version 1 (bit 46), layout
-// 2 = 128-byte swizzle (bits 61-63).  The leading byte offset is unused for this layout.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
-  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity), "r"(100000u)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
-                                            uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
-      "%3}], [%4];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
-      : "memory");
-}
-// Bring a tile toward L2 ahead of its load (no shared memory, no completion to wait for).
-__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global [%0, {%1, %2}];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(x), "r"(y)
-               : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
+using tc::mbar_arrive;
+using tc::mbar_expect_tx;
+using tc::mbar_init;
+using tc::mbar_try_wait;
+using tc::tma_load_2d;
+using tc::tma_prefetch_2d;
+using tc::tmem_ld32;
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) { return tc::desc_kmajor(saddr); }
+__device__ __forceinline__ void tc_fence_before() { tc::fence_before(); }
+__device__ __forceinline__ void tc_fence_after() { tc::fence_after(); }
 __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                        uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
-      : "memory");
+  tc::mma_bf16(d_tmem, adesc, bdesc, kIdesc, accumulate);
 }
-// The barrier receives one arrival once every MMA this thread issued so far has completed.
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                   bar)
-               : "memory");
-}
-// 32 consecutive f32 columns of this thread's TMEM lane, waited for in the same statement so
-// that no use of the registers can be scheduled before the data is there.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
-      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
-      "%30, %31}, [%32];\n\t"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
-#pragma unroll
-  for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
-}
+__device__ __forceinline__ void tc_commit(uint32_t bar) { tc::commit(bar); }
 
 struct TileArgs {
   int32_t rows;   // rows of this launch (a chunk in pass 2); the tensor map's row = row0 + local
@@ -659,46 +589,14 @@ __global__ void __launch_bounds__(128) lmhead_gather_kernel(
 
 // ---- host side ---------------------------------------------------------------------------------
 
-using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                 const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                 const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                 CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiled encode_fn() {
-  static EncodeTiled fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiled>(p);
-  });
-  return fn;
-}
-
 // 2-D bf16 tensor map over rows x cols (row stride `stride` elements), box 64 x box_rows,
 // 128-byte swizzle, zero fill outside the tensor.
 bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int64_t stride,
               uint32_t box_rows) {
-  EncodeTiled fn = encode_fn();
-  if (!fn) return false;
-  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)stride * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
-  const cuuint32_t estr[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return tc::make_map_bf16(m, base, rows, cols, stride, box_rows);
 }
 
-int sm_count() {
-  int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-  return n;
-}
+int sm_count() { return tc::sm_count(); }
 
 struct Grid {
   int R, J, grid;
@@ -767,65 +665,6 @@ grpo_status launch_tiles(bool bwd, const CUtensorMap& mh, const CUtensorMap& mw,
   return check_launch(who);
 }
 
-// cuBLASLt: C (col-major m x n, ldc) = op(A) * op(B) + beta * C, f32 accumulation.
-cublasLtHandle_t lt_handle() {
-  static cublasLtHandle_t h = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    if (cublasLtCreate(&h) != CUBLAS_STATUS_SUCCESS) h = nullptr;
-  });
-  return h;
-}
-
-grpo_status lt_gemm(cudaStream_t s, bool ta, bool tb, int64_t m, int64_t n, int64_t k,
-                    const void* A, int64_t lda, const void* B, int64_t ldb, void* C,
-                    cudaDataType_t ctype, int64_t ldc, float beta, void* ws, size_t ws_bytes,
-                    const char* who) {
-  cublasLtHandle_t h = lt_handle();
-  if (!h) return fail(GRPO_ERR_CUDA, "%s: cublasLtCreate failed", who);
-  cublasLtMatmulDesc_t op = nullptr;
-  cublasLtMatrixLayout_t la = nullptr, lb = nullptr, lc = nullptr;
-  cublasLtMatmulPreference_t pref = nullptr;
-  grpo_status st = GRPO_OK;
-  const cublasOperation_t opa = ta ? CUBLAS_OP_T : CUBLAS_OP_N, opb = tb ? CUBLAS_OP_T : CUBLAS_OP_N;
-  const float alpha = 1.f;
-  cublasLtMatmulHeuristicResult_t res = {};
-  int found = 0;
-  bool ok = cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F) == CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof opa) ==
-                CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof opb) ==
-                CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, ta ? k : m, ta ? m : k, lda) ==
-                CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, tb ? n : k, tb ? k : n, ldb) ==
-                CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatrixLayoutCreate(&lc, ctype, m, n, ldc) == CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatmulPreferenceCreate(&pref) == CUBLAS_STATUS_SUCCESS &&
-            cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
-                                                 &ws_bytes, sizeof ws_bytes) ==
-                CUBLAS_STATUS_SUCCESS;
-  if (ok)
-    ok = cublasLtMatmulAlgoGetHeuristic(h, op, la, lb, lc, lc, pref, 1, &res, &found) ==
-             CUBLAS_STATUS_SUCCESS &&
-         found > 0;
-  if (!ok) {
-    st = fail(GRPO_ERR_CUDA, "%s: no cuBLASLt algorithm for %lld x %lld x %lld", who,
-              (long long)m, (long long)n, (long long)k);
-  } else {
-    const cublasStatus_t r = cublasLtMatmul(h, op, &alpha, A, la, B, lb, &beta, C, lc, C, lc,
-                                            &res.algo, ws, ws_bytes, s);
-    if (r != CUBLAS_STATUS_SUCCESS)
-      st = fail(GRPO_ERR_CUDA, "%s: cublasLtMatmul failed (%d)", who, (int)r);
-  }
-  if (pref) cublasLtMatmulPreferenceDestroy(pref);
-  if (lc) cublasLtMatrixLayoutDestroy(lc);
-  if (lb) cublasLtMatrixLayoutDestroy(lb);
-  if (la) cublasLtMatrixLayoutDestroy(la);
-  if (op) cublasLtMatmulDescDestroy(op);
-  return st;
-}
-
 int64_t padded_v(int32_t V) { return (int64_t)align_up((size_t)V, 32); }
 
 int64_t chunk_of(int64_t n_rows, int32_t V, int64_t chunk_rows) {
@@ -835,8 +674,24 @@ int64_t chunk_of(int64_t n_rows, int32_t V, int64_t chunk_rows) {
   return std::max<int64_t>(BM, std::min<int64_t>(c, (n_rows + BM - 1) / BM * BM));
 }
 
+// Workspace of the backward products' split K (gemm_plan): the larger of the two products' f32
+// partials for the full chunk and for the last, shorter one.  Without a device (a size query on
+// a machine with no GPU) the plan assumes 152 SMs; a launch that finds less room runs unsplit.
+size_t gemm_partial_bytes(int64_t n_rows, int32_t V, int32_t D, int64_t chunk) {
+  int n_sm = sm_count();
+  if (n_sm <= 0) n_sm = 152;
+  size_t most = 0;
+  const int64_t last = n_rows % chunk;
+  for (int64_t rows : {std::min(chunk, n_rows), last}) {
+    if (rows <= 0) continue;
+    most = std::max(most, gemm_plan(rows, D, V, n_sm).partial_bytes);  // dh
+    most = std::max(most, gemm_plan(V, D, rows, n_sm).partial_bytes);  // dW
+  }
+  return most;
+}
+
 struct WsLayout {
-  size_t part, zy, rowsc, row_loss, stats, seq_loss, dl, lt, hid, ys, olds, refs, total;
+  size_t part, zy, rowsc, row_loss, stats, seq_loss, dl, gpart, hid, ys, olds, refs, total;
 };
 // loss: the backward buffers; n_seqs >= 0: GSPO's statistics and sequence terms instead of the
 // per-row loss terms.
@@ -857,7 +712,7 @@ WsLayout ws_layout(int64_t n_rows, int32_t V, int32_t D, int64_t chunk, bool own
   w.stats = take(n_seqs >= 0 ? n * sizeof(float4) : 0);
   w.seq_loss = take(n_seqs >= 0 ? (size_t)std::max<int64_t>(n_seqs, 1) * sizeof(double) : 0);
   w.dl = take(loss && own_dl ? (size_t)chunk * padded_v(V) * 2 : 0);
-  w.lt = take(loss ? kLtWorkspace : 0);
+  w.gpart = take(loss && n_rows > 0 ? gemm_partial_bytes(n_rows, V, D, chunk) : 0);
   w.hid = take(gather ? n * (size_t)D * 2 : 0);
   w.ys = take(gather ? n * 4 : 0);
   w.olds = take(gather ? n * 4 : 0);
@@ -951,12 +806,12 @@ grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
   return launch_tiles(false, f->mh, f->mw, ta, g1.grid, s, who);
 }
 
-// Pass 2 and the two GEMMs, chunk by chunk, from each row's gradient scalars (rowsc).
+// Pass 2 and the two products, chunk by chunk, from each row's gradient scalars (rowsc).
 grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64_t n_rows,
                      int32_t V, int32_t D, const void* weight, void* dhidden,
                      int32_t dhidden_dtype, float* dweight, int32_t accumulate_dweight,
-                     void* dlogits_out, __nv_bfloat16* dl_buf, int64_t chunk, void* lt_ws,
-                     cudaStream_t s) {
+                     void* dlogits_out, __nv_bfloat16* dl_buf, int64_t chunk, float* gpart,
+                     size_t gpart_bytes, cudaStream_t s) {
   grpo_status st;
   const int64_t ldd = padded_v(V);
   const size_t dh_elem = dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
@@ -977,17 +832,16 @@ grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64
     tb.dl = dl;
     tb.ldd = ldd;
     if ((st = launch_tiles(true, f.mh, f.mw, tb, g2.grid, s, who)) != GRPO_OK) return st;
-    // dh[c0 : c0 + rows] = dlogits * W   (column-major: dh^T [D x rows] = W^T [D x V] dl^T)
-    if ((st = lt_gemm(s, false, false, D, rows, V, weight, D, dl, ldd,
-                      static_cast<char*>(dhidden) + c0 * D * dh_elem,
-                      dhidden_dtype == GRPO_DTYPE_BF16 ? CUDA_R_16BF : CUDA_R_32F, D, 0.f, lt_ws,
-                      kLtWorkspace, who)) != GRPO_OK)
+    // dh[c0 : c0 + rows] = dlogits * W: A = dl [rows][V] (K-major), B = W [V][D]
+    if ((st = gemm_bf16(who, false, dl, ldd, weight, D, rows, D, V,
+                        static_cast<char*>(dhidden) + c0 * D * dh_elem, D, dhidden_dtype, false,
+                        gpart, gpart_bytes, f.ta.status, s)) != GRPO_OK)
       return st;
-    // dW (+)= dlogits^T * h   (column-major: dW^T [D x V] = h^T [D x rows] * dl [rows x V])
-    const float b = (c0 == 0 && !accumulate_dweight) ? 0.f : 1.f;
-    if ((st = lt_gemm(s, false, true, D, V, rows,
-                      static_cast<const char*>(f.hid) + c0 * f.hstride * 2, f.hstride, dl, ldd,
-                      dweight, CUDA_R_32F, D, b, lt_ws, kLtWorkspace, who)) != GRPO_OK)
+    // dW (+)= dlogits^T * h: A = dl^T, stored [rows][V] (M-major), B = h [rows][D]
+    const bool acc = !(c0 == 0 && !accumulate_dweight);
+    if ((st = gemm_bf16(who, true, dl, ldd, static_cast<const char*>(f.hid) + c0 * f.hstride * 2,
+                        f.hstride, V, D, rows, dweight, D, GRPO_DTYPE_F32, acc, gpart,
+                        gpart_bytes, f.ta.status, s)) != GRPO_OK)
       return st;
   }
   return GRPO_OK;
@@ -1092,7 +946,8 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
   double* row_loss = row_loss_out ? row_loss_out : reinterpret_cast<double*>(wsb + L.row_loss);
   __nv_bfloat16* dl_buf = dlogits_out ? static_cast<__nv_bfloat16*>(dlogits_out)
                                       : reinterpret_cast<__nv_bfloat16*>(wsb + L.dl);
-  void* lt_ws = wsb + L.lt;
+  float* gpart = reinterpret_cast<float*>(wsb + L.gpart);
+  const size_t gpart_bytes = L.hid - L.gpart;
 
   if (n_rows == 0) {
     cudaError_t e = cudaMemsetAsync(loss_out, 0, sizeof(double), s);
@@ -1142,7 +997,7 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
   if ((st = launch_sum_rows(row_loss, n_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
 
   return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
-                  accumulate_dweight, dlogits_out, dl_buf, chunk, lt_ws, s);
+                  accumulate_dweight, dlogits_out, dl_buf, chunk, gpart, gpart_bytes, s);
 }
 
 extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
@@ -1245,5 +1100,6 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
   if ((st = check_launch(who)) != GRPO_OK) return st;
   if ((st = launch_sum_rows(seq_loss, n_seq_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
   return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
-                  accumulate_dweight, dlogits_out, dl_buf, chunk, wsb + L.lt, s);
+                  accumulate_dweight, dlogits_out, dl_buf, chunk,
+                  reinterpret_cast<float*>(wsb + L.gpart), L.hid - L.gpart, s);
 }

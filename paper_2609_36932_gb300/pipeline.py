@@ -84,16 +84,18 @@ class GrpoStep:
         self.counts_host = torch.empty(2, dtype=torch.int64, pin_memory=True)
         self.kpp_host = torch.empty(max(self.P, 1), dtype=torch.int32, pin_memory=True)
         self.keep_host = torch.empty(max(n, 1), dtype=torch.uint8, pin_memory=True)
+        self.kept_off_host = torch.empty(n + 1, dtype=torch.int64, pin_memory=True)
         # numpy views of the pinned buffers: the per-step host reads avoid tensor indexing
         self._stream = torch.cuda.current_stream(dev)
         self._counts_np = self.counts_host.numpy()
         self._kpp_np = self.kpp_host[:max(self.P, 1)].numpy()[:self.P]
         self.loss = torch.empty(1, dtype=torch.float64, device=dev)
         self.logp = torch.empty(max(self.T, 1), dtype=torch.float32, device=dev)
+        # per kept row, the weighted Eq. 1 term w_t * l_t whose fixed-order sum is `loss`
+        self.row_loss = torch.empty(max(self.T, 1), dtype=torch.float64, device=dev)
         self.out_dtype = torch.bfloat16 if params.dlogits_dtype == "bf16" else torch.float32
         self.dlogits = None
         self.prune_ws = None
-        self.loss_ws = None
         self.ars = B.grpo_ars_init(G1 if G1 is not None else params.G)
         self.ars_total = ars_total_steps
         self.steps_per_epoch = steps_per_epoch
@@ -141,7 +143,6 @@ class GrpoStep:
                           None, None, ctypes.byref(need), None)
         B._check(rc)
         self.prune_ws = self.torch.empty(need.value + 256, dtype=self.torch.uint8, device=self.dev)
-        self.loss_ws = self.torch.empty(self.T * 8 + 512, dtype=self.torch.uint8, device=self.dev)
 
     def loss_step(self):
         p = self.p
@@ -157,8 +158,8 @@ class GrpoStep:
             V=p.V, row_index=self.src_token, n_rows=self.T_kept, eps_low=p.eps_low,
             eps_high=p.eps_high, beta=p.beta, agg_mode=p.agg_mode,
             denom_tokens=max(self.T_kept, 1), seq_off=self.off, n_seq=max(self.K, 1),
-            dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp, loss_out=self.loss, status=self.status,
-            ws=self.loss_ws)
+            dlogits=self.dlogits, dlogits_dtype=self.out_dtype, logp_out=self.logp,
+            row_loss_out=self.row_loss, loss_out=self.loss, status=self.status)
 
     def _loss_lmhead(self):
         """The output layer fused with the loss over the kept rows (gathered by src_token): the
@@ -214,8 +215,7 @@ class GrpoStep:
         p = self.p
         torch = self.torch
         self._ensure_dlogits(min(p.chunk_rows, max(self.T_kept, 1)))
-        if getattr(self, "row_loss", None) is None:
-            self.row_loss = torch.empty(max(self.T, 1), dtype=torch.float64, device=self.dev)
+        if getattr(self, "chunk_loss", None) is None:
             self.chunk_loss = torch.empty(1, dtype=torch.float64, device=self.dev)
         for c0 in range(0, self.T_kept, p.chunk_rows):
             c1 = min(self.T_kept, c0 + p.chunk_rows)
@@ -243,6 +243,7 @@ class GrpoStep:
         self.counts_host.copy_(self.counts, non_blocking=True)
         self.kpp_host[:self.P].copy_(self.kpp[:self.P], non_blocking=True)
         self.keep_host[:self.keep.numel()].copy_(self.keep, non_blocking=True)
+        self.kept_off_host.copy_(self.kept_off, non_blocking=True)
 
     def _enqueue_loss(self):
         p = self.p
@@ -250,9 +251,10 @@ class GrpoStep:
             return self._enqueue_gspo()
         B.grpo_loss_fwd_bwd_dev(
             self.logits, self.ids, self.old, self.ref, self.adv, self.token_rollout, self.counts,
-            max_rows=self.T, dlogits=self.dlogits, loss_out=self.loss, ws=self.loss_ws, V=p.V,
+            max_rows=self.T, dlogits=self.dlogits, loss_out=self.loss, ws=None, V=p.V,
             row_index=self.src_token, eps_low=p.eps_low, eps_high=p.eps_high, beta=p.beta,
-            agg_mode=p.agg_mode, seq_off=self.off, logp_out=self.logp, status=self.status)
+            agg_mode=p.agg_mode, seq_off=self.off, logp_out=self.logp, row_loss_out=self.row_loss,
+            status=self.status)
 
     def capture(self):
         """Capture the selection (advantage, prune, compact, count copies) and the loss as two
@@ -370,7 +372,7 @@ class GrpoStep:
                 self.replay_loss()
             else:
                 self.loss_step()
-        d2h = 2 * 8 + 4 * self.P + n
+        d2h = 2 * 8 + 4 * self.P + n + 8 * (n + 1)  # counts, kept per prompt, keep, kept_off
         if loss_host is not None:
             loss_host.copy_(self.loss, non_blocking=True)
             d2h += 8
@@ -384,12 +386,11 @@ class GrpoStep:
         p = self.p
         n = self.keep.numel()
         keep = self.keep_host.numpy()[:n].astype(bool)
-        off = host["off"].numpy()
-        lens = np.diff(off)
         kept = np.flatnonzero(keep)
-        # compacted row offset of each kept rollout, and group boundaries by rows
-        rows_before = np.concatenate([[0], np.cumsum(lens[kept])])
-        T = int(rows_before[-1])
+        # compacted row offset of each kept rollout: grpo_compact's kept_off, read back with the
+        # keep flags; then group boundaries by rows
+        rows_before = self.kept_off_host.numpy()[:kept.size + 1]
+        T = self.T_kept
         bounds = [0]
         for g in range(1, groups):
             k = int(np.searchsorted(rows_before, T * g / groups, side="left"))
@@ -398,7 +399,6 @@ class GrpoStep:
         bounds.append(kept.size)
         if getattr(self, "_copy_stream", None) is None:
             self._copy_stream = torch.cuda.Stream(self.dev)
-            self.row_loss = torch.empty(max(self.T, 1), dtype=torch.float64, device=self.dev)
         self._ensure_dlogits(self.T_kept)
         cs = self._copy_stream
         cs.wait_stream(self._stream)  # the previous step's loss is done with the logits buffer

@@ -35,6 +35,26 @@ def test_version_and_counter(grpo):
     assert grpo.grpo_kernel_launches() >= 0
 
 
+def test_check_status_maps_device_bits(grpo):
+    """grpo_check_status: 0 is OK, a timed-out wait is GRPO_ERR_TIMEOUT (it wins over data bits),
+    data bits are GRPO_ERR_DEVICE_CHECK, and the message names every bit."""
+    B = grpo.binding
+    L = B.lib()
+    assert L.grpo_check_status(0) == 0
+    for word, rc, words in ((B.DEVFLAG_BAD_TOKEN, 6, [b"token id"]),
+                            (B.DEVFLAG_NONFINITE, 6, [b"non-finite"]),
+                            (B.DEVFLAG_TIMEOUT, 5, [b"timed out"]),
+                            (B.DEVFLAG_TIMEOUT | B.DEVFLAG_BAD_TOKEN, 5, [b"timed out", b"token id"]),
+                            (64, 6, [b"unknown"])):
+        assert L.grpo_check_status(word) == rc
+        msg = L.grpo_last_error()
+        assert all(w in msg for w in words), msg
+    with pytest.raises(grpo.GrpoError) as e:
+        B.check_status(B.DEVFLAG_NONFINITE)
+    assert e.value.status == 6
+    assert B.check_status(0) == 0
+
+
 def test_library_host_ars_matches_oracle(oracle_mod, grpo):
     """adaptive_rollout_count (host C++ in the library) equals the oracle step for step."""
     rng = np.random.default_rng(4)
@@ -238,14 +258,17 @@ def test_lmhead_workspace_query_and_argument_errors(grpo):
     assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size)) == 0
     full = size.value
     # per row: 160 partial (max, sum) pairs, z_y, the row scalars and the row loss; one chunk of
-    # bf16 dlogits (1000 rows round up to 1024) and 32 MiB for cuBLASLt
+    # bf16 dlogits (1000 rows round up to 1024); and the f32 partial products of dhidden's split
+    # K: S copies of the chunk's [rows, D] (1 <= S <= 8; 56 output tiles on 152 SMs split)
     def up(x):
         return (x + 255) // 256 * 256
-    expect = (up(1000 * 160 * 8) + up(1000 * 4) + up(1000 * 16) + up(1000 * 8)
-              + up(1024 * 152064 * 2) + up(32 << 20))
-    assert full == expect
+    base = up(1000 * 160 * 8) + up(1000 * 4) + up(1000 * 16) + up(1000 * 8)
+    gp = full - base - up(1024 * 152064 * 2)
+    unit = 1000 * 3584 * 4
+    assert 2 * unit <= gp <= 8 * unit and gp % unit == 0
     assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size), chunk=256) == 0
-    assert size.value == full - up(1024 * 152064 * 2) + up(256 * 152064 * 2)
+    gp = size.value - base - up(256 * 152064 * 2)
+    assert 2 * 256 * 3584 * 4 <= gp <= 8 * 256 * 3584 * 4 and gp % (256 * 3584 * 4) == 0
     assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size),
                        dl=ctypes.c_void_p(4096)) == 0
     assert size.value == full - up(1024 * 152064 * 2)
@@ -337,3 +360,29 @@ def test_fail_launch_hook_rejects_negative_counts(grpo):
     L.grpo_test_fail_launch.restype = ctypes.c_int32
     assert L.grpo_test_fail_launch(ctypes.c_int32(-1)) == 1
     assert L.grpo_test_fail_launch(ctypes.c_int32(0)) == 0
+
+
+def test_lmhead_grad_workspace_query_and_argument_errors(grpo):
+    """grpo_lmhead_grad answers its size query and rejects bad arguments without a device; a
+    query on a qwen-sized chunk (14122 rows, V = 152064, D = 3584) asks for the split partials
+    of dhidden's product (its 784 output tiles would leave most of a seventh wave idle)."""
+    L = grpo.binding.lib()
+    size = ctypes.c_size_t(0)
+    out = ctypes.c_void_p(256)  # never dereferenced by a size query
+
+    def call(n, V, D, dstride, hstride, dtype=1, dh=out, dw=out):
+        return L.grpo_lmhead_grad(None, dstride, n, V, None, hstride, None, D, dh, dtype, dw, 0,
+                                  None, None, ctypes.byref(size), None)
+
+    assert call(14122, 152064, 3584, 152064, 3584) == 0
+    assert size.value >= 2 * 14122 * 3584 * 4 and size.value % 256 == 0
+    assert call(14122, 152064, 3584, 152064, 3584, dh=None) == 0  # dweight alone: no split
+    assert size.value == 0
+    assert call(0, 100, 64, 104, 64) == 0 and size.value == 0
+    assert call(10, 100, 12, 104, 16) == 1                  # D not a multiple of 8
+    assert call(10, 100, 64, 100, 64) == 1                  # dlogits stride not a multiple of 8
+    assert call(10, 100, 64, 96, 64) == 1                   # dlogits stride < V
+    assert call(10, 100, 64, 104, 60) == 1                  # hidden stride < D
+    assert call(10, 100, 64, 104, 64, dtype=7) == 1         # dhidden dtype
+    assert b"grpo_lmhead_grad" in L.grpo_last_error()
+

@@ -35,8 +35,8 @@ def test_reference_arm_line(loss):
     assert d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
-    if loss != "grpo":
-        assert d["config"]["loss"] == loss
+    # the same config keys as the repo arm's line, the loss included
+    assert d["config"]["loss"] == loss
     if loss.startswith("lmhead"):
         assert d["config"]["D"] == 64
 

@@ -40,7 +40,7 @@ def test_fused_loss_random_configurations(grpo, oracle_mod, seed):
                             **kw)
     assert g["status"] == 0
     compare(g["logp"], g["dlogits"], g["loss"], r, outd, eps_low=eps_low, eps_high=eps_high,
-            gpu_row_loss=g["row_loss"])
+            gpu_row_loss=g["row_loss"], cond=c.cond(idx))
 
 
 @pytest.mark.parametrize("seed", range(8))

@@ -44,6 +44,10 @@ class Case:
         import torch
         return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
+    def cond(self, idx=None):
+        """The rows' ref_logp inputs and beta, for compare()'s conditioning of g_t."""
+        return dict(ref_logp=self.ref[:self.n] if idx is None else self.ref[idx], beta=self.beta)
+
     def run_gpu(self, grpo, **kw):
         import torch
         n = kw.pop("n_rows", self.n)
@@ -88,7 +92,8 @@ def test_vocab_sizes_and_dtypes(grpo, oracle_mod, V, ind, outd):
     g = c.run_gpu(grpo)
     r = c.run_oracle(oracle_mod)
     assert g["status"] == 0
-    compare(g["logp"], g["dlogits"], g["loss"], r, outd, gpu_row_loss=g["row_loss"])
+    compare(g["logp"], g["dlogits"], g["loss"], r, outd, gpu_row_loss=g["row_loss"],
+            cond=c.cond())
 
 
 @pytest.mark.parametrize("cluster,threads,chunks", [(2, 256, 0), (3, 128, 3), (4, 512, 5),
@@ -104,7 +109,8 @@ def test_launch_shapes(grpo, oracle_mod, cluster, threads, chunks):
         g2 = c.run_gpu(grpo)
     finally:
         grpo.grpo_loss_tune(0, 0, 0)
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"],
+            cond=c.cond())
     assert g["loss"] == g2["loss"] and np.array_equal(g["dlogits"], g2["dlogits"])
 
 
@@ -131,7 +137,8 @@ def test_gathered_strided_rows(grpo, oracle_mod, V, ind):
     g = c.run_gpu(grpo, n_rows=29, row_index=c.t(idx), rr=rr)
     r = oracle_mod.loss(c.host, V, c.y, c.old, c.ref, c.adv, rr, row_stride=c.stride,
                         row_index=idx, dlogits_dtype=1, beta=c.beta)
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"],
+            cond=c.cond(idx))
 
 
 def test_unaligned_rows_take_the_element_path(grpo, oracle_mod):
@@ -153,7 +160,8 @@ def test_unaligned_rows_take_the_element_path(grpo, oracle_mod):
                                  dlogits_dtype="f32", logp_out=lp, status=status, beta=c.beta)
     torch.cuda.synchronize()
     r = oracle_mod.loss(np.ascontiguousarray(host), V, c.y, old, c.ref, c.adv, c.rr, beta=c.beta)
-    compare(lp.cpu().numpy(), out["dlogits"].cpu().numpy(), float(out["loss"].item()), r, "f32")
+    compare(lp.cpu().numpy(), out["dlogits"].cpu().numpy(), float(out["loss"].item()), r, "f32",
+            cond=c.cond())
 
 
 def test_sequence_mean(grpo, oracle_mod):
@@ -167,7 +175,8 @@ def test_sequence_mean(grpo, oracle_mod):
     g = c.run_gpu(grpo, rr=rr, agg_mode=1, seq_off=c.t(seq_off), n_seq=n_seq)
     r = oracle_mod.loss(c.host, c.V, c.y, c.old, c.ref, c.adv, rr, agg_mode=1, seq_off=seq_off,
                         n_seq=n_seq, dlogits_dtype=1, beta=c.beta)
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"],
+            cond=c.cond())
 
 
 @pytest.mark.parametrize("beta", [0.0, 0.04])
@@ -182,7 +191,7 @@ def test_asymmetric_clip(grpo, oracle_mod, beta):
     r = c.run_oracle(oracle_mod, eps_low=0.2, eps_high=0.28)
     assert g["status"] == 0
     compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", eps_low=0.2, eps_high=0.28,
-            gpu_row_loss=g["row_loss"])
+            gpu_row_loss=g["row_loss"], cond=c.cond())
     A = c.adv[c.rr].astype(np.float64)
     rho = r["rho"][:c.n]
     active = ((A > 0) & (rho > 1.28 * (1 + 1e-5))) | ((A < 0) & (rho < 0.8 * (1 - 1e-5)))
@@ -225,7 +234,7 @@ def test_bad_token_sets_status_and_zero_row(grpo, oracle_mod):
     r = c.run_oracle(oracle_mod)
     assert np.isnan(g["logp"][2]) and np.isnan(g["logp"][4])
     assert np.all((g["dlogits"][[2, 4]] & 0x7FFF) == 0)
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16")
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", cond=c.cond())
 
 
 def test_nonfinite_logits_set_status(grpo):
@@ -258,7 +267,8 @@ def test_masked_vocabulary(grpo, oracle_mod):
     g = c.run_gpu(grpo)
     r = c.run_oracle(oracle_mod)
     assert g["status"] == 0
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"],
+            cond=c.cond())
 
 
 def test_peaked_rows_keep_one_minus_p_accurate(grpo, oracle_mod):
@@ -278,7 +288,7 @@ def test_peaked_rows_keep_one_minus_p_accurate(grpo, oracle_mod):
     c.ref = (logp + 0.1 * rng.standard_normal(12)).astype(np.float32)
     g = c.run_gpu(grpo)
     r = c.run_oracle(oracle_mod)
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16")
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", cond=c.cond())
 
 
 @pytest.mark.parametrize("agg_mode", [0, 1])
@@ -330,7 +340,7 @@ def test_lost_copy_times_out_and_the_context_stays_usable(grpo, oracle_mod):
     good = c.run_gpu(grpo)
     assert good["status"] == 0
     compare(good["logp"], good["dlogits"], good["loss"], c.run_oracle(oracle_mod), "bf16",
-            gpu_row_loss=good["row_loss"])
+            gpu_row_loss=good["row_loss"], cond=c.cond())
 
 
 @pytest.mark.parametrize("V", [262144, 600000])
@@ -342,7 +352,8 @@ def test_large_vocabularies(grpo, oracle_mod, V):
     g = c.run_gpu(grpo)
     r = c.run_oracle(oracle_mod)
     assert g["status"] == 0
-    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"])
+    compare(g["logp"], g["dlogits"], g["loss"], r, "bf16", gpu_row_loss=g["row_loss"],
+            cond=c.cond())
     lp = grpo.grpo_logp_fwd(c.dev, c.t(c.y)).cpu().numpy()[:5]
     assert np.abs(lp.astype(np.float64) - r["logp"]).max() <= 2e-5
 
@@ -364,4 +375,4 @@ def test_injected_launch_failure_is_reported_and_the_next_call_is_clean(grpo, or
     good = c.run_gpu(grpo)
     assert good["status"] == 0
     compare(good["logp"], good["dlogits"], good["loss"], c.run_oracle(oracle_mod), "bf16",
-            gpu_row_loss=good["row_loss"])
+            gpu_row_loss=good["row_loss"], cond=c.cond())

@@ -1,14 +1,15 @@
 """Whole-step parity on the five workloads, in the launch configuration bench.py times:
 advantage -> prune -> compact -> loss over the kept rows.  'tiny' and 'small' are compared
-with the oracle row by row in full; the three Qwen-vocabulary workloads at full size are
-compared on sampled rows, and their total loss through a property that holds at any size
-(the loss is the weighted sum of Eq. 1's per-token terms evaluated at the kernel's logp)."""
+with the oracle row by row in full.  The three Qwen-vocabulary workloads at full size are
+compared with the oracle on every kept row's log-probability and loss term and on the total
+loss, and on the dlogits of at least 1024 rows (every row of two whole kept rollouts among
+them)."""
 import dataclasses
 
 import numpy as np
 import pytest
 
-from loss_compare import LOSS_RTOL, compare
+from loss_compare import LOSS_RTOL, compare, compare_rows
 from paper_2609_36932_gb300 import workloads
 from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
 
@@ -54,17 +55,6 @@ def check_selection(oracle_mod, w, b, step):
     return adv, comp
 
 
-def eq1_terms(logp, old, ref, A, eps, beta, w):
-    """Eq. 1's per-token loss terms at the given log-probs (fp64)."""
-    logp = logp.astype(np.float64)
-    rho = np.exp(logp - old)
-    lo, hi = 1.0 - np.float64(np.float32(eps)), 1.0 + np.float64(np.float32(eps))
-    surr = np.minimum(rho * A, np.clip(rho, lo, hi) * A)
-    x = ref - logp
-    kl = np.expm1(x) - x
-    return -w * (surr - np.float64(np.float32(beta)) * kl)
-
-
 @pytest.mark.parametrize("name", ["tiny", "small"])
 def test_full_comparison(oracle_mod, name):
     import torch
@@ -80,35 +70,76 @@ def test_full_comparison(oracle_mod, name):
                           beta=w.beta, denom_tokens=TK,
                           dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
     compare(step.logp[:TK].cpu().numpy(), host_bits(step.dlogits[:TK]), float(step.loss.item()),
-            ref, w.dlogits_dtype)
+            ref, w.dlogits_dtype, gpu_row_loss=step.row_loss[:TK].cpu().numpy(),
+            cond=dict(ref_logp=h["ref"][comp["src_token"]], beta=w.beta))
+
+
+def oracle_all_rows(oracle_mod, w, b, h, adv, comp, TK, block=8192):
+    """The oracle over every kept row, without dlogits: logits copied to the host a block of rows
+    at a time.  Returns its dict (logp, rho, row_loss per row and the total loss)."""
+    import torch
+    st, tr = comp["src_token"], comp["token_rollout"]
+    out = dict(logp=np.empty(TK), rho=np.empty(TK), row_loss=np.empty(TK), loss=0.0)
+    for r0 in range(0, TK, block):
+        r1 = min(TK, r0 + block)
+        src = st[r0:r1]
+        lg = host_bits(h["logits"][torch.from_numpy(src).cuda()])
+        o = oracle_mod.loss(lg, w.V, b["ids"][src], h["old"][src], h["ref"][src], adv, tr[r0:r1],
+                            eps_low=w.eps, eps_high=w.eps, beta=w.beta, denom_tokens=TK,
+                            want_dlogits=False)
+        for k in ("logp", "rho", "row_loss"):
+            out[k][r0:r1] = o[k]
+        out["loss"] += o["loss"]
+    return out
+
+
+def sample_rows(comp, K, TK, n=1024, seed=7):
+    """Every row of two whole kept rollouts (the first and the longest), the first and last 8
+    rows, and random rows up to n."""
+    ko = comp["kept_off"]
+    lens = np.diff(ko[:K + 1])
+    whole = [0, int(np.argmax(lens))]
+    rows = [np.arange(ko[k], ko[k + 1]) for k in whole]
+    rows += [np.arange(min(8, TK)), np.arange(max(TK - 8, 0), TK)]
+    have = np.unique(np.concatenate(rows))
+    rng = np.random.default_rng(seed)
+    rest = np.setdiff1d(np.arange(TK), have)
+    extra = rng.choice(rest, size=min(rest.size, max(n - have.size, 0)), replace=False)
+    return np.unique(np.concatenate([have, extra])).astype(np.int64), whole
 
 
 @pytest.mark.parametrize("name", ["qwen", "large", "long"])
-def test_full_size_sampled(oracle_mod, name):
+def test_full_size_against_oracle(oracle_mod, name):
     import torch
     w, b, step, h = build(name, chunk_rows=0)
     step.run()
     torch.cuda.synchronize()
     assert int(step.status.item()) == 0
     adv, comp = check_selection(oracle_mod, w, b, step)
-    TK = step.T_kept
-    rng = np.random.default_rng(7)
-    rows = np.unique(np.concatenate([np.arange(8), np.arange(TK - 8, TK),
-                                     rng.choice(TK, 32, replace=False)]))
+    TK, K = step.T_kept, step.K
+    logp = step.logp[:TK].cpu().numpy()
+    row_loss = step.row_loss[:TK].cpu().numpy()
+    total = float(step.loss.item())
+    # every kept row: logp, loss term and the total loss against the oracle's
+    o_all = oracle_all_rows(oracle_mod, w, b, h, adv, comp, TK)
+    _, n_skip, logp_err = compare_rows(logp, total, row_loss, o_all, w.eps, w.eps)
+    print("%s: %d kept rows, max logp error %.3g, %d clip-boundary rows, loss %.12g (oracle %.12g)"
+          % (name, TK, logp_err, n_skip, total, o_all["loss"]))
+    # dlogits: >= 1024 rows, every row of two whole kept rollouts among them
+    rows, whole = sample_rows(comp, K, TK)
+    ko = comp["kept_off"]
+    assert all(np.isin(np.arange(ko[k], ko[k + 1]), rows).all() for k in whole)
+    assert rows.size >= min(1024, TK)
     src = comp["src_token"][rows]
     lg = host_bits(h["logits"][torch.from_numpy(src).cuda()])
     o = oracle_mod.loss(lg, w.V, b["ids"][src], h["old"][src], h["ref"][src], adv,
                         comp["token_rollout"][rows], eps_low=w.eps, eps_high=w.eps, beta=w.beta,
                         denom_tokens=TK, dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
     idx = torch.from_numpy(rows).cuda()
-    logp = step.logp[:TK].cpu().numpy()
-    compare(logp[rows], host_bits(step.dlogits[:TK][idx]), None, o, w.dlogits_dtype)
-    # the total: Eq. 1's terms at the kernel's logp, summed in fp64
-    st = comp["src_token"]
-    terms = eq1_terms(logp, h["old"][st].astype(np.float64), h["ref"][st].astype(np.float64),
-                      adv[comp["token_rollout"]].astype(np.float64), w.eps, w.beta, 1.0 / TK)
-    total = float(step.loss.item())
-    assert abs(total - terms.sum()) <= LOSS_RTOL * abs(terms.sum()) + 1e-12
+    res = compare(logp[rows], host_bits(step.dlogits[:TK][idx]), None, o, w.dlogits_dtype,
+                  gpu_row_loss=row_loss[rows], cond=dict(ref_logp=h["ref"][src], beta=w.beta))
+    print("%s: dlogits of %d rows, worst %s, %d rows with an ill-conditioned g_t"
+          % (name, rows.size, res["worst"], res["widened_rows"]))
     # the same step again is bitwise identical
     loss0 = total
     step.run()
@@ -123,6 +154,7 @@ def test_full_size_sampled(oracle_mod, name):
         torch.cuda.synchronize()
         assert float(step.loss.item()) == loss0
         assert np.array_equal(step.logp[:TK].cpu().numpy(), logp)
+        assert np.array_equal(step.row_loss[:TK].cpu().numpy(), row_loss)
         n_last = TK - (TK - 1) // w.chunk_rows * w.chunk_rows
         assert torch.equal(step.dlogits[:n_last][-100:], d_last)
 
@@ -192,7 +224,9 @@ def test_step_variants(oracle_mod, variant):
                           agg_mode=p.agg_mode, denom_tokens=TK, seq_off=b["off"],
                           n_seq=comp["K"], dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
     compare(step.logp[:TK].cpu().numpy(), host_bits(step.dlogits[:TK]), float(step.loss.item()),
-            ref, w.dlogits_dtype, eps_low=p.eps_low, eps_high=p.eps_high)
+            ref, w.dlogits_dtype, eps_low=p.eps_low, eps_high=p.eps_high,
+            gpu_row_loss=step.row_loss[:TK].cpu().numpy(),
+            cond=dict(ref_logp=h["ref"][comp["src_token"]], beta=p.beta))
     loss0, dl0 = float(step.loss.item()), step.dlogits[:TK].clone()
     step.capture()
     assert step.run_graph() == TK
@@ -273,7 +307,8 @@ def test_host_inputs_step_equals_resident_step(name, graph, groups):
         assert torch.equal(step.logp[:TK], ref_logp) and torch.equal(step.dlogits[:TK], ref_dl)
         assert int(step.status.item()) == 0
         assert h2d == small + TK * w.V * host["logits"].element_size()
-        assert d2h == 16 + 4 * step.P + step.keep.numel() + 8
+        n = step.keep.numel()
+        assert d2h == 16 + 4 * step.P + n + 8 * (n + 1) + 8
 
 
 @pytest.mark.parametrize("name", ["tiny", "small"])

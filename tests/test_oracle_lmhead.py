@@ -194,3 +194,24 @@ def test_gspo_gradients_are_the_derivatives_of_the_loss(oracle_mod, case):
         for idx in np.ndindex(*shape):
             fd = (loss_of(key, idx, h) - loss_of(key, idx, -h)) / (2 * h)
             assert grad[idx] == pytest.approx(fd, rel=1e-6, abs=1e-9), (key, idx)
+
+
+def test_chain_rule_alone_equals_library_matrix_products(oracle_mod):
+    """oracle.lmhead_grad (the chain rule for given dlogits) equals numpy's matrix products, and
+    its absolute sums equal the products of the absolute values; on the fused oracle's own dlogits
+    it returns the fused oracle's dhidden and dweight."""
+    rng = np.random.default_rng(31)
+    for T, V, D in ((1, 1, 1), (7, 13, 6), (40, 33, 24)):
+        dl = rng.standard_normal((T, V))
+        h = rng.standard_normal((T, D))
+        w = rng.standard_normal((V, D))
+        out = oracle_mod.lmhead_grad(dl, h, w, want_bounds=True)
+        np.testing.assert_allclose(out["dhidden"], dl @ w, rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(out["dweight"], dl.T @ h, rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(out["dhidden_abs"], np.abs(dl) @ np.abs(w), rtol=1e-12)
+        np.testing.assert_allclose(out["dweight_abs"], np.abs(dl).T @ np.abs(h), rtol=1e-12)
+    p, kw = problem(np.random.default_rng(32), T=9, V=11, D=7)
+    fused = run(oracle_mod, p, kw, want_dlogits=True)
+    alone = oracle_mod.lmhead_grad(fused["dlogits"], p["hidden"], p["weight"])
+    assert np.array_equal(alone["dhidden"], fused["dhidden"])
+    assert np.array_equal(alone["dweight"], fused["dweight"])

@@ -124,6 +124,43 @@ def test_gradient_invariants(oracle_mod):
     np.testing.assert_allclose(ratio, ratio[:, :1].repeat(200, 1), rtol=1e-9)
 
 
+def test_gradient_factor_g(oracle_mod):
+    """The oracle's per-row g: (1) dlogits[t] / (e_y - p) = w * g_t; (2) g_t is the derivative of
+    the row's loss term l_t with respect to log pi(y), by a central difference that moves old_logp
+    and ref_logp together (rho and x then move as if logp moved the other way); (3) its own
+    derivative with respect to log pi(y) is g + beta * (2 e^x - 1), the identity the GPU tests use
+    to bound how far an error in logp moves g."""
+    rng = np.random.default_rng(16)
+    n, V = 12, 50
+    z = rows(rng, n, V, 2.0)
+    y, old, ref, adv, rr = inputs(rng, z, A_values=(1.1, -0.6, 0.0))
+    beta = 0.3
+    out = oracle_mod.loss(z, V, y, old, ref, adv, rr, beta=beta, denom_tokens=4, want_f64=True)
+    assert np.all(np.abs(out["rho"] - 0.8) > 1e-3) and np.all(np.abs(out["rho"] - 1.2) > 1e-3)
+    zz = z.astype(np.float64)
+    p = np.exp(zz - scipy.special.logsumexp(zz, 1, keepdims=True))
+    e = np.zeros_like(p)
+    e[np.arange(n), y] = 1.0
+    np.testing.assert_allclose(out["dlogits_f64"] / (e - p), (out["g"] / 4.0)[:, None]
+                               .repeat(V, 1), rtol=1e-9)
+    h = 1e-5
+    # old and ref moved by -h (as if logp moved by +h) and by +h; they are f32 in the oracle's
+    # interface, so the shift actually applied is measured, and must be the same for both
+    old_p, old_m = old - np.float32(h), old + np.float32(h)
+    ref_p, ref_m = ref - np.float32(h), ref + np.float32(h)
+    dh = (old_m.astype(np.float64) - old_p.astype(np.float64)) / 2  # the shift actually applied
+    assert np.allclose((ref_m.astype(np.float64) - ref_p.astype(np.float64)) / 2, dh, rtol=0, atol=0)
+    lp = oracle_mod.loss(z, V, y, old_p, ref_p, adv, rr, beta=beta, denom_tokens=1,
+                         want_dlogits=False)
+    lm = oracle_mod.loss(z, V, y, old_m, ref_m, adv, rr, beta=beta, denom_tokens=1,
+                         want_dlogits=False)
+    np.testing.assert_allclose((lp["row_loss"] - lm["row_loss"]) / (2 * dh), out["g"], rtol=1e-5,
+                               atol=1e-9)
+    x = ref.astype(np.float64) - out["logp"]
+    np.testing.assert_allclose((lp["g"] - lm["g"]) / (2 * dh), out["g"] + beta * (2 * np.exp(x) - 1),
+                               rtol=1e-5, atol=1e-9)
+
+
 def test_asymmetric_clip_regions(oracle_mod):
     """Eq. 2 with eps_low = 0.2, eps_high = 0.28 against the clipped surrogate's closed form,
     one token at a time (beta = 0, denominator 1): loss = -min(rho*A, clip(rho)*A), and dlogits
