@@ -487,7 +487,7 @@ def measured_tensor_peak(sustained):
 
 def lmhead_source_hash(root=None):
     """Hash of the output-layer kernels' code (see code_hash)."""
-    return code_hash(("lmhead.cu", "rowops.cuh", "common.cuh"), root)
+    return code_hash(("lmhead.cu", "tcgen05.cuh", "rowops.cuh", "common.cuh"), root)
 
 
 def lmhead_traffic_per_row():
@@ -642,6 +642,49 @@ def lmhead_side(w, b, step, seed, dev, reps=3):
                     "8 T_kept V D FLOPs per call; bench.py --loss lmhead runs it as a step"}
 
 
+def lmhead_products(d, step, T_kept, V, D, peak, peak_src, nrep=3):
+    """The two backward products alone (grpo_lmhead_grad) on the step's kept rows: dlogits taken
+    from one fused call, the kept hidden rows gathered densely; each product event-timed on this
+    stream against the burst tensor peak (2 T V D FLOPs each)."""
+    import torch
+    import paper_2609_36932_gb300 as g
+    free, _ = torch.cuda.mem_get_info(d["hidden"].device)
+    ldd = g.grpo_lmhead_dlogits_stride(V)
+    if T_kept == 0 or T_kept * ldd * 2 + V * D * 4 + 2 * T_kept * D * 4 > 0.8 * free:
+        return None
+    dl = torch.empty((T_kept, ldd), dtype=torch.bfloat16, device=d["hidden"].device)
+    p = step.p
+    g.grpo_lmhead_loss_fwd_bwd(d["hidden"], d["weight"], d["ids"], d["old"], d["ref"], step.adv,
+                               step.token_rollout, row_index=step.src_token[:T_kept],
+                               n_rows=T_kept, eps_low=p.eps_low, eps_high=p.eps_high, beta=p.beta,
+                               denom_tokens=T_kept, dlogits_out=dl)
+    hk = d["hidden"][step.src_token[:T_kept]].contiguous()
+    dlv = dl[:, :V]
+    out = {}
+    stream = torch.cuda.current_stream()
+    for name, kw in (("dhidden", dict(want_dweight=False)), ("dweight", dict(want_dhidden=False))):
+        r = g.grpo_lmhead_grad(dlv, hk, d["weight"], **kw)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(nrep):
+            g.grpo_lmhead_grad(dlv, hk, d["weight"], dhidden=r["dhidden"], dweight=r["dweight"],
+                               ws=r["ws"], **kw)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / nrep
+        tf = 2.0 * T_kept * V * D / (ms / 1e3) / 1e12
+        out[name] = {"ms": ms, "achieved": tf, "frac": tf / peak}
+        del r
+    del dl, hk
+    torch.cuda.empty_cache()
+    out.update({"unit": "TFLOP/s", "peak": peak, "peak_source": peak_src, "calls": nrep,
+                "kernel": "gemm_bf16_kernel (tcgen05, gemm.cu) through grpo_lmhead_grad",
+                "note": "dhidden = dlogits W and dweight = dlogits^T h over all kept rows in one "
+                        "call each (the fused call runs them per dlogits chunk)"})
+    return out
+
+
 def run_lmhead(args, w):
     """--loss lmhead: the step with the output layer fused (GrpoStep in output-layer mode)."""
     import torch
@@ -739,8 +782,9 @@ def run_lmhead(args, w):
                "achieved": 4 * flops_pass / (loss_ms / 1e3) / 1e12, "unit": "TFLOP/s",
                "peak": peak_s, "frac": 4 * flops_pass / (loss_ms / 1e3) / 1e12 / peak_s,
                "peak_source": peak_s_src,
-               "note": "the whole fused call: pass 1, pass 2 (2 T V D each, tcgen05) and the "
-                       "dhidden and dweight GEMMs (2 T V D each, cuBLASLt)"}
+               "note": "the whole fused call: pass 1, pass 2 and the dhidden and dweight "
+                       "products (2 T V D each), all on the library's tcgen05 kernels"}
+    products = None if gspo else lmhead_products(d, step, T_kept, w.V, D, peak, peak_src)
 
     # end to end: selection inputs, log-probs and hidden states from pinned host memory (hidden
     # rows of the kept rollouts only), loss read back, inside the timed region
@@ -799,7 +843,8 @@ def run_lmhead(args, w):
             "data": "synthetic (seeded; the qwen batch with random-init output layer)",
             "config": lmhead_desc(w, D, b["T"], T_kept, step.K, gspo),
             "gpu_launches": int(launches), "cuda_graph": False,
-            "roofline": roofline, "step_tensor": step_tc, "e2e": e2e, "cpu_baseline": cpu,
+            "roofline": roofline, "step_tensor": step_tc, "backward_products": products,
+            "e2e": e2e, "cpu_baseline": cpu,
             "clocks": clocks,
             "path_overhead": {"select_ms": select_ms, "other_ms": elapsed_ms / K - select_ms - loss_ms},
             "loss_value": float(step.loss.item()), "ars_next_rollouts": step.n_next,

@@ -9,18 +9,23 @@
 //   * Each slice arrives by non-tensor bulk copies (cp.async.bulk, 16-byte granules) in a few
 //     chunks, each completing on its own mbarrier, so the CTA starts reducing chunk 0 while
 //     the rest is in flight.
+//   * Roles: the consumer warps compute; one producer warp (one lane) stages each row's inputs
+//     (source row, token and its logit z_y, advantage, old/reference log-probs, weight) in
+//     shared memory and issues the slice's copies.  Nothing in the row loop waits for the whole
+//     CTA.
 //   * Pass A: per-thread online max and sum of exp (base 2, MUFU ex2) over the slice, leaving
-//     out the sampled token y; warp shuffles and shared memory combine the CTA's threads.
-//   * Exchange: each CTA pushes its (max, sum, z_y) into every cluster peer's shared memory with
-//     st.async, which completes bytes on the peer's mbarrier (no cluster-wide barrier, so no
-//     CTA waits for another's outstanding stores); warp 0 waits on its own mbarrier, reads the
-//     C entries locally and forms the row's log-sum-exp, log-prob, ratio, clipped surrogate, KL
-//     term and gradient coefficient.  Every CTA of the cluster computes the same numbers.
+//     out the sampled token y; warp shuffles combine a warp's threads.
+//   * Exchange: each warp pushes its (max, sum) into every cluster peer's shared memory with
+//     st.async, which completes bytes on the peer's mbarrier (no cluster-wide barrier);
+//     each warp then waits on its own CTA's mbarrier, combines the C x warps entries and forms
+//     the row's log-sum-exp, log-prob, ratio, clipped surrogate, KL term and gradient
+//     coefficient itself.  Every warp of the cluster computes the same numbers.
 //   * Pass B: dlogits[v] = -coef * exp(z_v - lse) (+coef at v = y) from the shared-memory slice,
-//     written with 16-byte streaming stores.  As soon as chunk k has been consumed, thread 0
-//     starts the copy of chunk k of the cluster's next row into the same buffer.
+//     written with 16-byte streaming stores.  A warp that has finished chunk k arrives on that
+//     chunk's release mbarrier; once all have, the producer copies chunk k of the cluster's next
+//     row into the same buffer.
 //   * The grid is persistent: as many clusters as fit at once; cluster i takes rows i, i+n, ...
-//   * Per-row loss terms go to a buffer; a one-CTA kernel (reduce.cu) sums them in a fixed order.
+//   * Per-row loss terms go to a buffer; a fixed-order cluster reduction (reduce.cu) sums them.
 // Every wait on a copy is bounded (about one second); on expiry the kernel records
 // GRPO_DEVFLAG_TIMEOUT, stops waiting and issuing copies, and runs to the end.
 //
@@ -139,15 +144,6 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t local_addr, uint32_t ra
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local_addr), "r"(rank));
   return remote;
 }
-// 16-byte store into a cluster peer's shared memory that completes 16 bytes of that peer's
-// mbarrier transaction count (both addresses already mapped to the peer).
-__device__ __forceinline__ void st_async_f4(uint32_t remote_addr, float4 v, uint32_t remote_bar) {
-  asm volatile(
-      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
-          remote_addr),
-      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(remote_bar)
-      : "memory");
-}
 __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
                                               uint32_t bar) {
   asm volatile(
@@ -167,18 +163,59 @@ __device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float 
 
 // ---- the kernel -------------------------------------------------------------------------------
 
-// kCap: compile for 1536 resident threads per SM (40 registers; 1024 threads when the output is
-// wider than the input).  Used when the slice is small enough that shared memory would allow
-// that many threads; otherwise the register count is free and the compiler schedules better.
+// A row's inputs, staged in shared memory by the producer warp (one slot per row parity): the
+// logits row, the sampled token, its logit z_y (0 for a token outside [0, V)), the advantage, the
+// old and reference log-probabilities and the row's weight.
+struct __align__(16) RowIn {
+  int64_t src;
+  int32_t y;
+  float zy, A, old_lp, ref_lp, w;
+};
+static_assert(sizeof(RowIn) == 32, "row slot");
+
+// Shared memory of one CTA after its slice (sized for the launch's chunk count, so that at the
+// default V = 152064 shape three CTAs still fit an SM): copy barriers (full and empty per chunk),
+// two exchange barriers, the abort flag (16 bytes), two row slots, then the exchange entries
+// [2][C * warps], one (max, sum) pair each.
+__host__ __device__ constexpr int loss_smem_fixed(int n_chunks) {
+  return (2 * n_chunks + 2) * 8 + 16 + 2 * (int)sizeof(RowIn);
+}
+
+// 8-byte store into a cluster peer's shared memory that completes 8 bytes of that peer's
+// mbarrier transaction count.
+__device__ __forceinline__ void st_async_f2(uint32_t remote_addr, float2 v, uint32_t remote_bar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(
+          remote_addr),
+      "f"(v.x), "f"(v.y), "r"(remote_bar)
+      : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// kCap: compile for 1536 resident threads per SM (1024 when the output is wider than the input),
+// the producer warp included.  Used when the slice is small enough that shared memory would allow
+// that many threads.  Otherwise the instance is compiled for the CTAs per SM that shared memory
+// admits at its default shapes: 3 with 256 consumer threads (V = 152064, bf16 in and out), 6 with
+// 128 (V = 32000; V = 152064 with f32 dlogits admits 5).  Without that bound the compiler settled
+// at 56 registers with a small spill; with a bound of 1 it took 88, one CTA per SM fewer.
 template <typename InT, typename OutT>
 constexpr int kResidentThreads = sizeof(OutT) > sizeof(InT) ? 1024 : 1536;
-
 template <typename InT, typename OutT, int kThreads, bool kCap>
-__global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> / kThreads : 0)
+constexpr int kMinCtas = kCap ? kResidentThreads<InT, OutT> / (kThreads + 32)
+                              : (kThreads == 256 ? 3 : (kThreads == 128 ? 6 : 1));
+
+// kThreads consumer threads (kThreads / 32 warps) and one producer warp.  No CTA-wide barrier
+// inside the row loop: the producer refills chunk k of the next row as soon as every consumer
+// warp has released it (an mbarrier per chunk), and each consumer warp exchanges its own partial
+// (max, sum) with the cluster and forms the row's scalars itself.
+template <typename InT, typename OutT, int kThreads, bool kCap>
+__global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, kCap>))
     grpo_loss_kernel(const LossArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
   constexpr int kPairs = Fmt<InT>::kPairs;
-  constexpr int kWarps = kThreads / 32;
+  constexpr int kWarps = kThreads / 32;  // consumer warps; warp kWarps is the producer
   // Two vectors per thread in flight in the element loops (measured on GB300: +0.7-1.5% with
   // bf16 dlogits, within +-0.4% with f32 dlogits, where a forced 1 was 1% slower).
   constexpr int kUnroll = 2;
@@ -186,74 +223,44 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
   const int buf_bytes = (int)align_up((size_t)a.slice * sizeof(InT), 128);
   InT* buf = reinterpret_cast<InT*>(smem);
   const uint4* buf4 = reinterpret_cast<const uint4*>(smem);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + buf_bytes);  // kMaxChunks copy barriers
-  uint64_t* xbars = bars + kMaxChunks;                               // 2 exchange barriers
-  float4* exch = reinterpret_cast<float4*>(xbars + 2);               // [2][kMaxCluster] entries
-  float* red = reinterpret_cast<float*>(exch + 2 * kMaxCluster);     // 2*kWarps
-  float* rowsc = red + 2 * kWarps;                                   // 4 floats
-  int* abort_flag = reinterpret_cast<int*>(rowsc + 4);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + buf_bytes);  // chunk k landed
+  uint64_t* empty = full + a.n_chunks;                              // chunk k released
+  uint64_t* xbars = empty + a.n_chunks;                             // 2 exchange barriers
+  int* abort_flag = reinterpret_cast<int*>(xbars + 2);
+  RowIn* rin = reinterpret_cast<RowIn*>(reinterpret_cast<unsigned char*>(abort_flag) + 16);
+  float2* exch = reinterpret_cast<float2*>(rin + 2);                // [2][C * kWarps]
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t rank = cluster_ctarank();
   const uint32_t C = cluster_nctarank();
+  const int n_ent = (int)C * kWarps;  // exchange entries per row: one per warp of the cluster
   const int64_t ncl = cluster_count_x();
   const int s0 = (int)rank * a.slice;
   const int len = max(0, min(a.V - s0, a.slice));  // my slice's elements
   const int nvec = a.bulk ? len / kVec : 0;        // vectors that arrive by bulk copy
   const int tail0 = nvec * kVec;                   // first element loaded one by one
   const uint32_t buf_s = smem_addr(buf);
-  const uint32_t bar_s = smem_addr(bars);
-  const uint32_t xbar_s = smem_addr(xbars);
-  const uint32_t exch_s = smem_addr(exch);
+  const uint32_t full_s = smem_addr(full), empty_s = smem_addr(empty);
+  const uint32_t xbar_s = smem_addr(xbars), exch_s = smem_addr(exch);
   const float2 l2e2 = make_float2(kLog2e, kLog2e);
 
   if (tid == 0) {
-    for (int k = 0; k < a.n_chunks; ++k) mbar_init(bar_s + 8 * k, 1);
+    for (int k = 0; k < a.n_chunks; ++k) {
+      mbar_init(full_s + 8 * k, 1);
+      mbar_init(empty_s + 8 * k, kWarps);
+    }
     mbar_init(xbar_s, 1);
     mbar_init(xbar_s + 8, 1);
     *abort_flag = 0;
+    for (int k = 0; k < 2; ++k) {  // a slot read after an abort names row 0 and no token
+      rin[k].src = 0;
+      rin[k].y = -1;
+      rin[k].zy = rin[k].A = rin[k].old_lp = rin[k].ref_lp = rin[k].w = 0.f;
+    }
     mbar_fence_init();
   }
   __syncthreads();
   cluster_sync();  // peers' exchange barriers exist before anyone sends to them
-
-  auto row_base = [&](int64_t row) -> const char* {
-    const int64_t src = a.row_index ? a.row_index[row] : row;
-    return a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
-  };
-  // Copies thread 0 armed whose completion no wait of thread 0 has seen yet (bit k: chunk k, with
-  // the phase parity in pend_par); drained before the CTA exits.
-  uint32_t pend = 0, pend_par = 0;
-  auto issue_chunk = [&](const char* g, int k, uint32_t parity) {  // thread 0 only
-    const int v0 = k * a.chunk_vecs;
-    const int v1 = min(nvec, v0 + a.chunk_vecs);
-    const uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
-    mbar_expect_tx(bar_s + 8 * k, bytes);
-    if (bytes) bulk_copy_g2s(buf_s + v0 * 16, g + (int64_t)v0 * 16, bytes, bar_s + 8 * k);
-    pend |= 1u << k;
-    pend_par = (pend_par & ~(1u << k)) | (parity << k);
-  };
-  // Bounded wait (about kWaitLimitNs).  A copy that never lands sets GRPO_DEVFLAG_TIMEOUT and
-  // the abort flag, after which this CTA stops waiting for and issuing copies (its results are
-  // then invalid) but still completes every exchange, so no peer writes into a CTA that left.
-  auto wait_bar = [&](uint32_t bar, uint32_t parity, bool copy) -> bool {  // true: phase done
-    if (copy && *(volatile int*)abort_flag) return false;
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_timer_ns();
-    for (uint32_t it = 1; !mbar_try_wait(bar, parity); ++it) {
-      if ((it & 63u) != 0) continue;
-      if (copy && *(volatile int*)abort_flag) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
-        if (copy) *(volatile int*)abort_flag = 1;
-        if (a.status) atomicOr(a.status, GRPO_DEVFLAG_TIMEOUT);
-        return false;
-      }
-    }
-    return true;
-  };
-  auto wait_chunk = [&](int k, uint32_t parity) {
-    if (wait_bar(bar_s + 8 * k, parity, true) && tid == 0) pend &= ~(1u << k);
-  };
 
   int64_t n_rows = a.n_rows;
   double inv_denom = a.inv_denom;
@@ -268,258 +275,275 @@ __global__ void __launch_bounds__(kThreads, kCap ? kResidentThreads<InT, OutT> /
     }
   }
 
-  int64_t row = cluster_id_x();
-  uint32_t phase = 0;  // parity of the copy barriers (one completion per row)
-  uint32_t iter = 0;   // rows done; exchange slot = iter & 1, its parity = (iter >> 1) & 1
-  if (tid == 0 && row < n_rows) {
-    const char* g = row_base(row);
-    for (int k = 0; k < a.n_chunks; ++k) {
-      if (a.skip_copy && k == 0 && row == 0 && rank == 0) {  // test hook: arm, never copy
-        mbar_expect_tx(bar_s, 16u);
-        pend |= 1u;
-        continue;
+  // Bounded wait (about kWaitLimitNs).  A copy that never lands sets GRPO_DEVFLAG_TIMEOUT and
+  // the abort flag, after which the CTA stops waiting for and issuing copies (its results are
+  // then invalid) but still completes every exchange and chunk release, so that no peer writes
+  // into a CTA that left and every wait of the producer ends.
+  auto wait_bar = [&](uint32_t bar, uint32_t parity, bool copy) -> bool {  // true: phase done
+    if (copy && *(volatile int*)abort_flag) return false;
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 1; !mbar_try_wait(bar, parity); ++it) {
+      if ((it & 63u) != 0) continue;
+      if (copy && *(volatile int*)abort_flag) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *(volatile int*)abort_flag = 1;
+        if (a.status) atomicOr(a.status, GRPO_DEVFLAG_TIMEOUT);
+        return false;
       }
-      issue_chunk(g, k, 0u);
     }
-  }
+    return true;
+  };
 
-  // With dlogits wider than the logits, the row's source index and sampled token are loaded one
-  // row ahead.  Measured on GB300: +5.8% there (f32 dlogits at V = 152064); with bf16 dlogits
-  // the same change was 1.5-2% slower, so only the wider instance does it.
-  constexpr bool kAhead = sizeof(OutT) > sizeof(InT);
-  int64_t src_nx = 0;
-  int32_t y_nx = 0;
-  if (kAhead && row < n_rows) {
-    src_nx = a.row_index ? a.row_index[row] : row;
-    y_nx = a.y[src_nx];
-  }
-  for (; row < n_rows; row += ncl, phase ^= 1u, ++iter) {
-    const uint32_t slot = iter & 1u;
-    if (tid == 0) mbar_expect_tx(xbar_s + 8 * slot, 16u * C);  // one entry from every CTA
-    int64_t src;
-    int32_t yv;
-    if constexpr (kAhead) {
-      src = src_nx;
-      yv = y_nx;
-      if (row + ncl < n_rows) {  // issued now, used by the cluster's next row
-        src_nx = a.row_index ? a.row_index[row + ncl] : row + ncl;
-        y_nx = a.y[src_nx];
-      }
-    } else {
-      src = a.row_index ? a.row_index[row] : row;
-      yv = a.y[src];
-    }
-    const bool yvalid = yv >= 0 && yv < a.V;
-    const int yl = yvalid ? yv - s0 : -1;  // y's position in my slice, if there
-    const char* grow = a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
-
-    // ---- pass A: max and sum of exp over my elements, y left out ----
-    float m = -INFINITY, s = 0.f;
-    for (int k = 0; k < a.n_chunks; ++k) {
-      wait_chunk(k, phase);
-      const int v0 = k * a.chunk_vecs;
-      const int v1 = min(nvec, v0 + a.chunk_vecs);
-      const bool last = (k == a.n_chunks - 1);
-      typename Fmt<InT>::Max mx;
-#pragma unroll 4
-      for (int j = v0 + tid; j < v1; j += kThreads) mx.add(buf4[j]);
-      float cm = mx.get();
-      if (last) {
-        for (int e = tail0 + tid; e < len; e += kThreads) {
-          const InT v = *reinterpret_cast<const InT*>(grow + (int64_t)e * sizeof(InT));
-          buf[e] = v;  // this thread reads it back below and in pass B
-          cm = fmaxf(cm, Fmt<InT>::load(&buf[e]));
+  if (warp == kWarps) {
+    // ---- producer warp, one lane: each row's inputs and its slice's copies ----
+    if (lane == 0) {
+      // Copies issued whose completion no consumer may have waited for (bit k: chunk k, with the
+      // phase parity in pend_par); drained before the CTA exits.
+      uint32_t pend = 0, pend_par = 0;
+      auto fetch = [&](int64_t r) {
+        RowIn ri;
+        ri.src = a.row_index ? a.row_index[r] : r;
+        ri.y = a.y[ri.src];
+        ri.zy = (ri.y >= 0 && ri.y < a.V)
+                    ? Fmt<InT>::load(reinterpret_cast<const InT*>(a.logits + ri.src * a.row_stride_bytes) + ri.y)
+                    : 0.f;
+        const int32_t ro = a.row_rollout[r];
+        ri.A = a.adv[ro];
+        ri.old_lp = a.old_logp[ri.src];
+        ri.ref_lp = a.ref_logp[ri.src];
+        ri.w = a.agg_mode == 0 ? inv_denom_f
+                               : inv_nseq_f / (float)(a.seq_off[ro + 1] - a.seq_off[ro]);
+        return ri;
+      };
+      auto issue = [&](int64_t src, int k, uint32_t parity) {
+        const char* g = a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
+        const int v0 = k * a.chunk_vecs;
+        const int v1 = min(nvec, v0 + a.chunk_vecs);
+        const uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
+        mbar_expect_tx(full_s + 8 * k, bytes);  // also publishes rin[] writes made before it
+        if (bytes) bulk_copy_g2s(buf_s + v0 * 16, g + (int64_t)v0 * 16, bytes, full_s + 8 * k);
+        pend |= 1u << k;
+        pend_par = (pend_par & ~(1u << k)) | (parity << k);
+      };
+      int64_t row = cluster_id_x();
+      RowIn nxt = {};
+      if (row < n_rows) {
+        rin[0] = fetch(row);
+        for (int k = 0; k < a.n_chunks; ++k) {
+          if (a.skip_copy && k == 0 && row == 0 && rank == 0) {  // test hook: arm, never copy
+            mbar_expect_tx(full_s, 16u);
+            pend |= 1u;
+            continue;
+          }
+          issue(rin[0].src, k, 0u);
         }
+        if (row + ncl < n_rows) nxt = fetch(row + ncl);  // loads in flight until it is needed
       }
-      if (cm > m) {
-        s = (m == -INFINITY) ? 0.f : s * ex2((m - cm) * kLog2e);
-        m = cm;
+      for (uint32_t iter = 0; row < n_rows; row += ncl, ++iter) {
+        const uint32_t slot = iter & 1u;
+        // one 8-byte entry from every warp of the cluster
+        mbar_expect_tx(xbar_s + 8 * slot, 8u * (uint32_t)n_ent);
+        const int64_t next = row + ncl;
+        for (int k = 0; k < a.n_chunks; ++k) {
+          wait_bar(empty_s + 8 * k, iter & 1u, false);  // chunk k of this row is released
+          if (next >= n_rows) continue;
+          if (k == 0) rin[slot ^ 1u] = nxt;  // the consumers are done with the row before this one
+          if (!*(volatile int*)abort_flag) issue(nxt.src, k, (iter + 1u) & 1u);
+        }
+        // The row after next: its dependent loads (source row, then token and log-probs) overlap
+        // the consumers' pass A of the next row instead of delaying a refill.
+        if (next + ncl < n_rows) nxt = fetch(next + ncl);
       }
-      if (m != -INFINITY) {
-        const float sh = -m * kLog2e;
-        const float2 sh2 = make_float2(sh, sh);
-        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
-#pragma unroll kUnroll
-        for (int j = v0 + tid; j < v1; j += kThreads) {
-          float2 p[kPairs];
-          Fmt<InT>::pairs(buf4[j], p);
-          const int yi = yl - j * kVec;
-          if ((unsigned)yi < (unsigned)kVec) {  // the vector holding y: leave y out
-#pragma unroll
-            for (int i = 0; i < kPairs; ++i) {
-              const float2 e = ex2x2(__ffma2_rn(p[i], l2e2, sh2));
-              if (2 * i != yi) acc0.x += e.x;
-              if (2 * i + 1 != yi) acc0.y += e.y;
-            }
-          } else {
-#pragma unroll
-            for (int i = 0; i < kPairs; i += 2) {
-              acc0 = __fadd2_rn(acc0, ex2x2(__ffma2_rn(p[i], l2e2, sh2)));
-              acc1 = __fadd2_rn(acc1, ex2x2(__ffma2_rn(p[i + 1], l2e2, sh2)));
-            }
+      for (int k = 0; k < a.n_chunks; ++k)  // copies in flight land before the CTA exits
+        if ((pend >> k) & 1u) wait_bar(full_s + 8 * k, (pend_par >> k) & 1u, false);
+    }
+    __syncwarp();
+  } else {
+    // ---- consumer warps ----
+    int64_t row = cluster_id_x();
+    for (uint32_t iter = 0; row < n_rows; row += ncl, ++iter) {
+      const uint32_t slot = iter & 1u, phase = iter & 1u;
+      RowIn ri = {};
+      bool live = true;  // every chunk of this row arrived (no abort)
+      int yl = -1;
+      const char* grow = nullptr;
+
+      // ---- pass A: max and sum of exp over my elements, y left out ----
+      float m = -INFINITY, s = 0.f;
+      for (int k = 0; k < a.n_chunks; ++k) {
+        if (!wait_bar(full_s + 8 * k, phase, true)) live = false;
+        if (k == 0) {
+          ri = rin[slot];
+          const bool yv_ok = ri.y >= 0 && ri.y < a.V;
+          yl = yv_ok ? ri.y - s0 : -1;  // y's position in my slice, if there
+          grow = a.logits + ri.src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
+        }
+        const int v0 = k * a.chunk_vecs;
+        const int v1 = min(nvec, v0 + a.chunk_vecs);
+        const bool last = (k == a.n_chunks - 1);
+        typename Fmt<InT>::Max mx;
+#pragma unroll 4
+        for (int j = v0 + tid; j < v1; j += kThreads) mx.add(buf4[j]);
+        float cm = mx.get();
+        if (last) {
+          for (int e = tail0 + tid; e < len; e += kThreads) {
+            // after an abort the row inputs may be stale: nothing is read from global memory
+            if (live) buf[e] = *reinterpret_cast<const InT*>(grow + (int64_t)e * sizeof(InT));
+            cm = fmaxf(cm, Fmt<InT>::load(&buf[e]));  // read back below and in pass B
           }
         }
-        s += (acc0.x + acc0.y) + (acc1.x + acc1.y);
-        if (last)
-          for (int e = tail0 + tid; e < len; e += kThreads)
-            if (e != yl) s += ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, sh));
-      }
-    }
-    // CTA reduction of (m, s)
+        if (cm > m) {
+          s = (m == -INFINITY) ? 0.f : s * ex2((m - cm) * kLog2e);
+          m = cm;
+        }
+        if (m != -INFINITY) {
+          const float sh = -m * kLog2e;
+          const float2 sh2 = make_float2(sh, sh);
+          float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll kUnroll
+          for (int j = v0 + tid; j < v1; j += kThreads) {
+            float2 p[kPairs];
+            Fmt<InT>::pairs(buf4[j], p);
+            const int yi = yl - j * kVec;
+            if ((unsigned)yi < (unsigned)kVec) {  // the vector holding y: leave y out
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float mo = __shfl_xor_sync(0xffffffffu, m, o);
-      const float so = __shfl_xor_sync(0xffffffffu, s, o);
-      lse_combine(m, s, mo, so);
-    }
-    if (lane == 0) {
-      red[2 * warp] = m;
-      red[2 * warp + 1] = s;
-    }
-    __syncthreads();
-    if (warp == 0) {
-      m = lane < kWarps ? red[2 * lane] : -INFINITY;
-      s = lane < kWarps ? red[2 * lane + 1] : 0.f;
+              for (int i = 0; i < kPairs; ++i) {
+                const float2 e = ex2x2(__ffma2_rn(p[i], l2e2, sh2));
+                if (2 * i != yi) acc0.x += e.x;
+                if (2 * i + 1 != yi) acc0.y += e.y;
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < kPairs; i += 2) {
+                acc0 = __fadd2_rn(acc0, ex2x2(__ffma2_rn(p[i], l2e2, sh2)));
+                acc1 = __fadd2_rn(acc1, ex2x2(__ffma2_rn(p[i + 1], l2e2, sh2)));
+              }
+            }
+          }
+          s += (acc0.x + acc0.y) + (acc1.x + acc1.y);
+          if (last)
+            for (int e = tail0 + tid; e < len; e += kThreads)
+              if (e != yl) s += ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, sh));
+        }
+      }
+      // warp reduction of (m, s); this warp's entry goes to every CTA of the cluster (self too)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         const float mo = __shfl_xor_sync(0xffffffffu, m, o);
         const float so = __shfl_xor_sync(0xffffffffu, s, o);
         lse_combine(m, s, mo, so);
       }
-      // push (max, sum, z_y) into entry [slot][rank] of every CTA of the cluster (self too)
       if (lane < (int)C) {
-        const float zy = ((unsigned)yl < (unsigned)len) ? Fmt<InT>::load(&buf[yl]) : 0.f;
-        const uint32_t dst = exch_s + (uint32_t)(slot * kMaxCluster + rank) * 16u;
-        st_async_f4(mapa_shared(dst, lane), make_float4(m, s, zy, 0.f),
-                    mapa_shared(xbar_s + 8 * slot, lane));
+        const uint32_t dst = exch_s + (uint32_t)(slot * n_ent + rank * kWarps + warp) * 8u;
+        st_async_f2(mapa_shared(dst, lane), make_float2(m, s), mapa_shared(xbar_s + 8 * slot, lane));
       }
-    }
 
-    // ---- exchange and row scalars (warp 0) ----
-    if (warp == 0) {
-      wait_bar(xbar_s + 8 * slot, (iter >> 1) & 1u, false);  // every CTA's entry is here
-      const float4* ex = exch + slot * kMaxCluster;
-      float mc = -INFINITY, sc = 0.f;
-      if (lane < (int)C) {
-        const float4 v = ex[lane];
-        mc = v.x;
-        sc = v.y;
-      }
-      float M = mc;
+      // ---- exchange: this warp combines the cluster's entries and forms the row scalars ----
+      wait_bar(xbar_s + 8 * slot, (iter >> 1) & 1u, false);
+      const float2* ex = exch + slot * n_ent;
+      float M = -INFINITY;
+      for (int e = lane; e < n_ent; e += 32) M = fmaxf(M, ex[e].x);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      float term = (mc == -INFINITY) ? 0.f : sc * expf(mc - M);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) term += __shfl_xor_sync(0xffffffffu, term, o);
-      if (lane == 0) {
-        float neg_scale = 0.f, dy = 0.f, shB = 0.f;
-        if (!yvalid) {
-          if (rank == 0) {
-            if (a.logp_out) a.logp_out[row] = __int_as_float(0x7fc00000);
-            a.row_loss[row] = 0.0;
-            if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
-          }
-        } else {
-          const float zy = ex[yv / a.slice].z;
-          const float S_excl = term;
-          const float ey = expf(zy - M);
-          const float S = S_excl + ey;
-          const float logp = (zy - M) - logf(S);
-          // Eq. 1: ratio, clipped surrogate, KL term; Eqs. 2-3: gradient coefficient.
-          const float A = a.adv[a.row_rollout[row]];
-          const float rho = expf(logp - a.old_logp[src]);
-          const float clipped = rho < a.lo_up ? a.lo_rn : (rho > a.hi_dn ? a.hi_rn : rho);
-          const float surr = fminf(rho * A, clipped * A);
-          const float x = a.ref_logp[src] - logp;
-          const float em1 = expm1f(x);
-          const float kl = em1 - x;
-          const float ell = -(surr - a.beta * kl);
-          float w;
-          if (a.agg_mode == 0) {
-            w = inv_denom_f;
-          } else {
-            const int32_t r = a.row_rollout[row];
-            w = inv_nseq_f / (float)(a.seq_off[r + 1] - a.seq_off[r]);
-          }
-          const bool c = (A >= 0.f) ? (rho <= a.hi_dn) : (rho >= a.lo_up);
-          const float g = -((c ? rho * A : 0.f) + a.beta * em1);
-          const float coef = w * g;
-          neg_scale = -coef / S;
-          dy = coef * (S_excl / S);
-          shB = -M * kLog2e;
-          if (fabsf(neg_scale) >= 0x1p-100f) {
-            shB += kShiftB;
-            neg_scale *= 0x1p-16f;  // 2^-kShiftB
-          }
-          if (rank == 0) {
-            if (a.logp_out) a.logp_out[row] = logp;
-            a.row_loss[row] = (a.agg_mode == 0 ? inv_denom : (double)w) * (double)ell;
-            if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
-          }
-        }
-        rowsc[0] = neg_scale;
-        rowsc[1] = dy;
-        rowsc[2] = shB;
-        rowsc[3] = yvalid ? 0.f : 1.f;
+      float S_excl = 0.f;
+      for (int e = lane; e < n_ent; e += 32) {
+        const float2 v = ex[e];
+        if (v.x != -INFINITY) S_excl += v.y * expf(v.x - M);
       }
-    }
-    __syncthreads();
-
-    // ---- pass B: dlogits from the shared-memory slice; refill chunk by chunk ----
-    const float neg_scale = rowsc[0], dy = rowsc[1], shB = rowsc[2];
-    const bool zero_row = rowsc[3] != 0.f;
-    const float2 shb2 = make_float2(shB, shB), ns2 = make_float2(neg_scale, neg_scale);
-    OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V + s0;
-    const int64_t next = row + ncl;
-    const char* gnext = (tid == 0 && next < n_rows) ? row_base(next) : nullptr;
-    for (int k = 0; k < a.n_chunks; ++k) {
-      const int v0 = k * a.chunk_vecs;
-      const int v1 = min(nvec, v0 + a.chunk_vecs);
-      const bool last = (k == a.n_chunks - 1);
-      if (!zero_row) {
-#pragma unroll kUnroll
-        for (int j = v0 + tid; j < v1; j += kThreads) {
-          float2 p[kPairs], d[kPairs];
-          Fmt<InT>::pairs(buf4[j], p);
 #pragma unroll
-          for (int i = 0; i < kPairs; ++i) d[i] = __fmul2_rn(ex2x2(__ffma2_rn(p[i], l2e2, shb2)), ns2);
-          const int yi = yl - j * kVec;
-          if ((unsigned)yi < (unsigned)kVec) {
-#pragma unroll
-            for (int i = 0; i < kPairs; ++i) {
-              if (2 * i == yi) d[i].x = dy;
-              if (2 * i + 1 == yi) d[i].y = dy;
-            }
-          }
-          if (a.out_vec)
-            store_pairs<OutT, kPairs>(orow + j * kVec, d);
-          else
-            store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
-        }
-        if (last) {
-          for (int e = tail0 + tid; e < len; e += kThreads) {
-            float d = neg_scale * ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, shB));
-            if (e == yl) d = dy;
-            Fmt<OutT>::store(orow + e, d);
-          }
+      for (int o = 16; o > 0; o >>= 1) S_excl += __shfl_xor_sync(0xffffffffu, S_excl, o);
+      const bool yvalid = ri.y >= 0 && ri.y < a.V;
+      const bool writer = rank == 0 && warp == 0 && lane == 0;
+      float neg_scale = 0.f, dy = 0.f, shB = 0.f;
+      if (!yvalid) {
+        if (writer) {
+          if (a.logp_out) a.logp_out[row] = __int_as_float(0x7fc00000);
+          a.row_loss[row] = 0.0;
+          if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
         }
       } else {
-        float2 d[kPairs];
-#pragma unroll
-        for (int i = 0; i < kPairs; ++i) d[i] = make_float2(0.f, 0.f);
-        for (int j = v0 + tid; j < v1; j += kThreads) store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
-        if (last)
-          for (int e = tail0 + tid; e < len; e += kThreads) Fmt<OutT>::store(orow + e, 0.f);
+        const float zy = ri.zy;
+        const float ey = expf(zy - M);
+        const float S = S_excl + ey;
+        const float logp = (zy - M) - logf(S);
+        // Eq. 1: ratio, clipped surrogate, KL term; Eqs. 2-3: gradient coefficient.
+        const float A = ri.A;
+        const float rho = expf(logp - ri.old_lp);
+        const float clipped = rho < a.lo_up ? a.lo_rn : (rho > a.hi_dn ? a.hi_rn : rho);
+        const float surr = fminf(rho * A, clipped * A);
+        const float x = ri.ref_lp - logp;
+        const float em1 = expm1f(x);
+        const float kl = em1 - x;
+        const float ell = -(surr - a.beta * kl);
+        const bool c = (A >= 0.f) ? (rho <= a.hi_dn) : (rho >= a.lo_up);
+        const float g = -((c ? rho * A : 0.f) + a.beta * em1);
+        const float coef = ri.w * g;
+        neg_scale = -coef / S;
+        dy = coef * (S_excl / S);
+        shB = -M * kLog2e;
+        if (fabsf(neg_scale) >= 0x1p-100f) {
+          shB += kShiftB;
+          neg_scale *= 0x1p-16f;  // 2^-kShiftB
+        }
+        if (writer) {
+          if (a.logp_out) a.logp_out[row] = logp;
+          a.row_loss[row] = (a.agg_mode == 0 ? inv_denom : (double)ri.w) * (double)ell;
+          if (a.status && !isfinite(logp)) atomicOr(a.status, GRPO_DEVFLAG_NONFINITE);
+        }
       }
-      __syncthreads();  // chunk k consumed by every thread
-      if (gnext && !*(volatile int*)abort_flag) issue_chunk(gnext, k, phase ^ 1u);
+
+      // ---- pass B: dlogits from the shared-memory slice; each chunk released when done ----
+      const float2 shb2 = make_float2(shB, shB), ns2 = make_float2(neg_scale, neg_scale);
+      OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V + s0;
+      for (int k = 0; k < a.n_chunks; ++k) {
+        const int v0 = k * a.chunk_vecs;
+        const int v1 = min(nvec, v0 + a.chunk_vecs);
+        const bool last = (k == a.n_chunks - 1);
+        if (yvalid) {
+#pragma unroll kUnroll
+          for (int j = v0 + tid; j < v1; j += kThreads) {
+            float2 p[kPairs], d[kPairs];
+            Fmt<InT>::pairs(buf4[j], p);
+#pragma unroll
+            for (int i = 0; i < kPairs; ++i)
+              d[i] = __fmul2_rn(ex2x2(__ffma2_rn(p[i], l2e2, shb2)), ns2);
+            const int yi = yl - j * kVec;
+            if ((unsigned)yi < (unsigned)kVec) {
+#pragma unroll
+              for (int i = 0; i < kPairs; ++i) {
+                if (2 * i == yi) d[i].x = dy;
+                if (2 * i + 1 == yi) d[i].y = dy;
+              }
+            }
+            if (a.out_vec)
+              store_pairs<OutT, kPairs>(orow + j * kVec, d);
+            else
+              store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
+          }
+          if (last) {
+            for (int e = tail0 + tid; e < len; e += kThreads) {
+              float d = neg_scale * ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, shB));
+              if (e == yl) d = dy;
+              Fmt<OutT>::store(orow + e, d);
+            }
+          }
+        } else {
+          float2 d[kPairs];
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i) d[i] = make_float2(0.f, 0.f);
+          for (int j = v0 + tid; j < v1; j += kThreads)
+            store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
+          if (last)
+            for (int e = tail0 + tid; e < len; e += kThreads) Fmt<OutT>::store(orow + e, 0.f);
+        }
+        __syncwarp();  // every lane of this warp is done reading chunk k
+        if (lane == 0) mbar_arrive(empty_s + 8 * k);
+      }
     }
   }
-  if (tid == 0) {  // copies still in flight into this CTA's shared memory land before it exits
-    for (int k = 0; k < a.n_chunks; ++k)
-      if ((pend >> k) & 1u) wait_bar(bar_s + 8 * k, (pend_par >> k) & 1u, false);
-  }
-  cluster_sync();  // partners are done reading this CTA's shared memory
+  __syncthreads();
+  cluster_sync();  // partners are done with this CTA's shared memory
 }
 
 
@@ -741,8 +765,8 @@ grpo_status pick_shape(int V, int in_bytes, int out_bytes, const char* who, Shap
     chunk_vecs = (slice_vecs + kMaxChunks - 1) / kMaxChunks;
     chunks = (slice_vecs + chunk_vecs - 1) / chunk_vecs;
   }
-  const size_t smem = align_up(slice_bytes, 128) + kMaxChunks * 8 + 2 * 8 + 2 * kMaxCluster * 16 +
-                      2 * (threads / 32) * 4 + 4 * 4 + 16;
+  const size_t smem = align_up(slice_bytes, 128) + loss_smem_fixed(chunks) +
+                      2 * (size_t)C * (threads / 32) * sizeof(float2);
   if (smem > 227 * 1024)
     return fail(GRPO_ERR_UNSUPPORTED, "%s: V = %d needs %zu bytes of shared memory per CTA at %d CTAs", who,
                 V, smem, C);
@@ -767,7 +791,7 @@ grpo_status launch_rows(KernelFn fn, const Shape& sh, LossArgs a, cudaStream_t s
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cudaLaunchConfig_t cfg = {};
-  cfg.blockDim = dim3(sh.threads, 1, 1);
+  cfg.blockDim = dim3(sh.threads + 32, 1, 1);  // consumers and the producer warp
   cfg.dynamicSmemBytes = sh.smem;
   cfg.stream = s;
   cfg.attrs = attr;
@@ -924,8 +948,9 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   a.denom_from_counts = from_counts ? 1 : 0;
   a.skip_copy = g_skip_copy.exchange(0);
 
-  st = launch_rows(kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads)),
-                   sh, a, s, who);
+  st = launch_rows(
+      kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads + 32)), sh, a,
+      s, who);
   if (st != GRPO_OK) return st;
   count_launches(1);
   return launch_sum_rows(row_loss, n_rows, counts ? counts + 1 : nullptr, loss_out, s, who);

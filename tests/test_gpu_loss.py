@@ -114,6 +114,24 @@ def test_launch_shapes(grpo, oracle_mod, cluster, threads, chunks):
     assert g["loss"] == g2["loss"] and np.array_equal(g["dlogits"], g2["dlogits"])
 
 
+@pytest.mark.parametrize("V,ind,outd", [(32001, "bf16", "bf16"), (5003, "f32", "bf16"),
+                                        (152067, "bf16", "f32")])
+def test_many_rows_per_cluster_with_unaligned_rows(grpo, oracle_mod, V, ind, outd):
+    """More rows than resident clusters, with row lengths that are not a multiple of 16 bytes:
+    every CTA runs many rows in a row and loads its slice's elements one by one, so the warp that
+    read z_y and the warps that combine the row's entries differ from row to row."""
+    rng = np.random.default_rng(V + 17)
+    n = 1200 if V < 100000 else 700
+    c = Case(rng, n, V, ind, outd)
+    g = c.run_gpu(grpo)
+    r = c.run_oracle(oracle_mod)
+    assert g["status"] == 0
+    compare(g["logp"], g["dlogits"], g["loss"], r, outd, gpu_row_loss=g["row_loss"],
+            cond=c.cond())
+    g2 = c.run_gpu(grpo)
+    assert g2["loss"] == g["loss"] and np.array_equal(g2["dlogits"], g["dlogits"])
+
+
 def test_single_cta_row_too_large_is_rejected(grpo):
     rng = np.random.default_rng(1)
     c = Case(rng, 2, 152064, "bf16", "bf16")
