@@ -197,14 +197,14 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 // kCap: compile for 1536 resident threads per SM (1024 when the output is wider than the input),
 // the producer warp included.  Used when the slice is small enough that shared memory would allow
 // that many threads.  Otherwise the instance is compiled for the CTAs per SM that shared memory
-// admits at its default shapes: 3 with 256 consumer threads (V = 152064, bf16 in and out), 6 with
+// admits at its default shapes: 3 with 256 consumer threads (V = 152064, bf16 in and out), 7 with
 // 128 (V = 32000; V = 152064 with f32 dlogits admits 5).  Without that bound the compiler settled
 // at 56 registers with a small spill; with a bound of 1 it took 88, one CTA per SM fewer.
 template <typename InT, typename OutT>
 constexpr int kResidentThreads = sizeof(OutT) > sizeof(InT) ? 1024 : 1536;
+constexpr int uncapped_ctas(int threads) { return threads == 256 ? 3 : (threads == 128 ? 7 : 1); }
 template <typename InT, typename OutT, int kThreads, bool kCap>
-constexpr int kMinCtas = kCap ? kResidentThreads<InT, OutT> / (kThreads + 32)
-                              : (kThreads == 256 ? 3 : (kThreads == 128 ? 6 : 1));
+constexpr int kMinCtas = kCap ? kResidentThreads<InT, OutT> / (kThreads + 32) : uncapped_ctas(kThreads);
 
 // kThreads consumer threads (kThreads / 32 warps) and one producer warp.  No CTA-wide barrier
 // inside the row loop: the producer refills chunk k of the next row as soon as every consumer
@@ -708,11 +708,11 @@ KernelFn kernel_for(int in_dtype, int out_dtype, int threads, bool cap) {
                                       : pick_kernel<float, float>(threads, cap);
 }
 
-// Whether shared memory would let more than 1024 threads of this shape reside on an SM (then the
-// register-capped instance keeps that occupancy).
+// Whether shared memory would let more CTAs of this shape reside on an SM than the uncapped
+// instance is compiled for (then the register-capped instance keeps that occupancy).
 bool want_cap(size_t smem, int threads) {
   const size_t per_sm = 228 * 1024, reserved = 1024;
-  return (per_sm / (smem + reserved)) * (size_t)threads > 1024;
+  return per_sm / (smem + reserved) > (size_t)uncapped_ctas(threads);
 }
 
 // Launch shape of the row kernel for a vocabulary of V entries of in_bytes each.
@@ -949,8 +949,8 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   a.skip_copy = g_skip_copy.exchange(0);
 
   st = launch_rows(
-      kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads + 32)), sh, a,
-      s, who);
+      kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads)), sh, a, s,
+      who);
   if (st != GRPO_OK) return st;
   count_launches(1);
   return launch_sum_rows(row_loss, n_rows, counts ? counts + 1 : nullptr, loss_out, s, who);
