@@ -132,9 +132,11 @@ def loss_source_hash(root=None):
     return code_hash(("loss.cu", "gspo.cu", "rowops.cuh", "common.cuh"), root)
 
 
-def profiled_traffic(workload_name):
-    """DRAM bytes per kept row of the loss kernel from the committed ncu summary, if it was
-    taken on the current kernel source; else None."""
+def profiled_traffic(workload_name, rows, launches=1):
+    """DRAM bytes of a loss call over `rows` kept rows in `launches` kernel launches, from the
+    committed ncu record of the current kernel source (else None): bytes per kept row times the
+    rows, less the per-launch residue (dlogits lines still dirty in L2 when a launch ends) where
+    the record has one, fitted from captures of two sizes."""
     p = os.path.join(ROOT, "profiles", "loss_kernel_traffic.json")
     try:
         with open(p) as f:
@@ -144,7 +146,7 @@ def profiled_traffic(workload_name):
     e = d.get(workload_name)
     if not e or e.get("source_hash") != loss_source_hash():
         return None
-    return float(e["dram_bytes_per_row"])
+    return float(e["dram_bytes_per_row"]) * rows - float(e.get("dram_bytes_residue", 0.0)) * launches
 
 
 class ClockSampler:
@@ -998,12 +1000,13 @@ def timed_steps(args, w, seed, world, local, dev, steps, warmup):
     if args.loss == "gspo":  # two reads and one write of every kept row (no row has zero gradient
         # in these workloads: beta > 0)
         bytes_per_row = w.V * (2 * w.in_bytes + w.out_bytes) + GSPO_SIDE_BYTES_PER_ROW
-        per_row_traffic = profiled_traffic(w.name + "/gspo")
+        traffic = profiled_traffic(w.name + "/gspo", step.T_kept)
         kernel = ("GSPO loss: logp_stream_kernel with row statistics, "
                   "gspo_seq_kernel, gspo_dlogits_kernel, fixed-order sum")
     else:
         bytes_per_row = w.V * (w.in_bytes + w.out_bytes) + SIDE_BYTES_PER_ROW
-        per_row_traffic = profiled_traffic(w.name)
+        n_launch = -(-step.T_kept // step.p.chunk_rows) if step.p.chunk_rows else 1
+        traffic = profiled_traffic(w.name, step.T_kept, n_launch)
         kernel = "grpo_loss_kernel (+ the fixed-order loss sum, one 8-CTA cluster)"
         if step.p.chunk_rows:
             kernel += "; %d calls of at most %d kept rows" % (
@@ -1012,7 +1015,7 @@ def timed_steps(args, w, seed, world, local, dev, steps, warmup):
     peak, peak_src = measured_peak()
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak,
-                "traffic": None if per_row_traffic is None else per_row_traffic * step.T_kept,
+                "traffic": traffic,
                 "kernel": kernel,
                 "algorithmic_bytes_per_launch": step.T_kept * bytes_per_row,
                 "bytes_per_kept_row": bytes_per_row,
