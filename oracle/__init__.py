@@ -45,7 +45,7 @@ def lib():
         L.oracle_loss.restype = _i32
         L.oracle_gspo_loss.argtypes = [_c_p, _i32, _i64, _c_p, _i32, _c_p, _c_p, _c_p, _c_p,
                                        _c_p, _c_p, _i64, _i64, _f32, _f32, _f32, _c_p, _i32,
-                                       _c_p, _c_p, _c_p, _c_p, _c_p]
+                                       _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]
         L.oracle_gspo_loss.restype = _i32
         L.oracle_lmhead_loss.argtypes = [_c_p, _c_p, _i64, _i32, _i32, _c_p, _c_p, _c_p, _c_p,
                                          _c_p, _f32, _f32, _f32, _i32, _i64, _c_p, _i64, _c_p,
@@ -307,8 +307,9 @@ def gspo_loss(logits, V: int, y, old_logp, ref_logp, adv, seq_rollout, seq_row_o
               logits_dtype=None, dlogits_dtype=0, want_f64=False, want_dlogits=True):
     """GSPO's sequence-level loss over kept rollouts (see loss.cpp).  Sequence k owns rows
     [seq_row_off[k], seq_row_off[k+1]) and rollout seq_rollout[k].  n_seq defaults to the number
-    of sequences.  Returns dict(loss, logp [rows], seq_ratio [seqs], seq_loss [seqs], dlogits,
-    dlogits_f64)."""
+    of sequences.  Returns dict(loss, logp [rows], seq_ratio [seqs], seq_loss [seqs], g (each
+    row's gradient factor, dlogits[t] = g_t / (n_seq L_k) (onehot(y) - softmax); NaN in a sequence
+    without a ratio), dlogits, dlogits_f64)."""
     lg = np.ascontiguousarray(logits)
     if logits_dtype is None:
         logits_dtype = 1 if lg.dtype == np.uint16 else 0
@@ -329,17 +330,18 @@ def gspo_loss(logits, V: int, y, old_logp, ref_logp, adv, seq_rollout, seq_row_o
     lp = np.empty(max(n_rows, 1), np.float64)
     sr = np.empty(max(K, 1), np.float64)
     sl = np.empty(max(K, 1), np.float64)
+    g = np.empty(max(n_rows, 1), np.float64)
     total = np.zeros(1, np.float64)
     rc = lib().oracle_gspo_loss(_p(lg), logits_dtype, stride, _p(ri), V, _p(_arr(y, np.int32)),
                                 _p(_arr(old_logp, np.float32)), _p(_arr(ref_logp, np.float32)),
                                 _p(_arr(adv, np.float32)), _p(_arr(seq_rollout, np.int32)),
                                 _p(so), K, int(n_seq), float(eps_low), float(eps_high),
                                 float(beta), _p(dl), dlogits_dtype, _p(d64), _p(lp), _p(sr),
-                                _p(sl), _p(total))
+                                _p(sl), _p(total), _p(g))
     if rc != 0:
         raise ValueError("oracle_gspo_loss: bad arguments")
     return dict(loss=float(total[0]), logp=lp[:n_rows], seq_ratio=sr[:K], seq_loss=sl[:K],
-                dlogits=dl, dlogits_f64=d64)
+                g=g[:n_rows], dlogits=dl, dlogits_f64=d64)
 
 
 def logp(logits, V: int, y, *, row_index=None, n_rows=None, row_stride=None, logits_dtype=None):

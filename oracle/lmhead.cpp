@@ -136,7 +136,7 @@ extern "C" int oracle_lmhead_gspo_loss(const double* hidden, const double* weigh
   const int rc = oracle_gspo_loss(z.data(), 2, V, nullptr, V, y, old_logp, ref_logp, adv,
                                   seq_rollout, seq_row_off, n_seq_rows, n_seq, eps_low, eps_high,
                                   beta, nullptr, 0, dl.data(), logp.data(), seq_ratio_out,
-                                  seq_loss_out, &total);
+                                  seq_loss_out, &total, nullptr);
   if (rc != 0) return rc;
   copy_out(dl, nz, dlogits_out);
   copy_out(logp, n_rows, logp_out);

@@ -205,7 +205,7 @@ extern "C" int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t ro
                                 int64_t n_seq_rows, int64_t n_seq, float eps_low, float eps_high,
                                 float beta, void* dlogits, int dlogits_dtype, double* dlogits_f64,
                                 double* logp_out, double* seq_ratio_out, double* seq_loss_out,
-                                double* loss_out) {
+                                double* loss_out, double* g_out) {
   if (V < 1 || row_stride < V || n_seq_rows < 0 || n_seq <= 0 || seq_row_off == nullptr)
     return 1;
   if (seq_row_off[0] != 0) return 1;
@@ -238,6 +238,8 @@ extern "C" int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t ro
   const double hi = 1.0 + (double)eps_high;
   std::vector<double> seq_loss(n_seq_rows, 0.0);
   std::vector<double> coef(n_rows, 0.0);  // w_t * g_t
+  if (g_out)  // rows of a sequence without a ratio keep NaN
+    for (int64_t t = 0; t < n_rows; ++t) g_out[t] = nan;
   for (int64_t k = 0; k < n_seq_rows; ++k) {
     const int64_t r0 = seq_row_off[k], r1 = seq_row_off[k + 1];
     const int64_t L = r1 - r0;
@@ -264,7 +266,9 @@ extern "C" int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t ro
     for (int64_t t = r0; t < r1; ++t) {
       const int64_t src = row_index ? row_index[t] : t;
       const double x = (double)ref_logp[src] - logp[t];
-      coef[t] = w * -((c ? s * A : 0.0) + (double)beta * (std::exp(x) - 1.0));
+      const double g = -((c ? s * A : 0.0) + (double)beta * (std::exp(x) - 1.0));
+      coef[t] = w * g;
+      if (g_out) g_out[t] = g;
     }
   }
 

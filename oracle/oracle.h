@@ -61,14 +61,16 @@ int oracle_loss(const void* logits, int logits_dtype, int64_t row_stride, const 
 /* GSPO's sequence-level loss (length-normalised sequence ratio, clipped per sequence) over kept
  * rollouts; see loss.cpp.  Sequence k owns rows [seq_row_off[k], seq_row_off[k+1]) of the
  * n_seq_rows sequences and rollout seq_rollout[k]; loss = (1/n_seq) sum_k l_k.
- * seq_ratio_out [n_seq_rows] (nullable): s_k (NaN when undefined); seq_loss_out: l_k / n_seq. */
+ * seq_ratio_out [n_seq_rows] (nullable): s_k (NaN when undefined); seq_loss_out: l_k / n_seq.
+ * g_out [rows] (nullable): each row's gradient factor g_t = -(c_k s_k A + beta (exp(x_t) - 1)),
+ * dlogits[t] = g_t / (n_seq L_k) * (onehot(y) - softmax); NaN in a sequence without a ratio. */
 int oracle_gspo_loss(const void* logits, int logits_dtype, int64_t row_stride,
                      const int64_t* row_index, int V, const int32_t* y, const float* old_logp,
                      const float* ref_logp, const float* adv, const int32_t* seq_rollout,
                      const int64_t* seq_row_off, int64_t n_seq_rows, int64_t n_seq, float eps_low,
                      float eps_high, float beta, void* dlogits, int dlogits_dtype,
                      double* dlogits_f64, double* logp_out, double* seq_ratio_out,
-                     double* seq_loss_out, double* loss_out);
+                     double* seq_loss_out, double* loss_out, double* g_out);
 
 /* The policy's output layer fused with the GRPO token loss; see lmhead.cpp.
  * hidden f64 [n_rows, D], weight f64 [V, D] (row-major; bf16 values widen exactly).

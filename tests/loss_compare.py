@@ -9,12 +9,14 @@ sum of every other row's term on both sides (which needs the GPU's per-row terms
 never dropped.
 
 A row's dlogits are w_t * g_t * (onehot(y) - softmax), with g_t = -(c*rho*A + beta*(e^x - 1)),
-x = ref_logp - logp (Eq. 3).  Where the two terms of g_t nearly cancel (for instance A = 0 and
-ref_logp close to logp), the error that the logp tolerance allows is amplified in g_t's relative
-error, and one bf16 ulp is not reachable from an f32 log-probability.  Given the inputs
-(`cond`), such rows get the ulps that this row's own log-probability error propagates into g_t,
-|dg/dlogp| * |logp_gpu - logp_oracle| / |g_t| with dg/dlogp = g + beta*(2 e^x - 1), plus f32
-rounding of g_t's terms; every other row keeps the 1-ulp bar.  Those rows are counted.
+x = ref_logp - logp (Eq. 3; GSPO: the sequence ratio s in place of rho).  Where the two terms of
+g_t nearly cancel (for instance A = 0 and ref_logp close to logp), the error that the logp
+tolerance allows is amplified in g_t's relative error, and one bf16 ulp is not reachable from an
+f32 log-probability.  Given the inputs (`cond`), such rows get the ulps that the log-probability
+errors propagate into g_t: |c rho A| * e_ratio + beta e^x * e over |g_t|, with e the row's own
+logp error and e_ratio the error of log(rho) (the row's e; for GSPO the largest e of its
+sequence), plus f32 rounding of g_t's terms; every other row keeps the 1-ulp bar.  Those rows are
+counted.
 """
 import numpy as np
 
@@ -78,14 +80,15 @@ def allowed_ulps(gpu_logp, ref, cond, rows=None):
     beta = float(np.float32(cond["beta"]))
     x = np.asarray(cond["ref_logp"], np.float64) - o_logp
     ex = np.exp(x)
-    dg = g + beta * (2 * ex - 1)          # d g / d logp (pinned in the oracle tests)
-    mag = np.abs(-g - beta * (ex - 1)) + beta * ex  # |c rho A| + beta e^x: g's two terms
+    u = np.abs(-g - beta * (ex - 1))  # |c rho A|: g's clipped-surrogate term
+    k = beta * ex                      # beta e^x: its KL term's derivative
     e = np.abs(np.asarray(gpu_logp, np.float64) - o_logp) + 2.0 ** -24 * np.abs(o_logp)
+    e_r = np.asarray(cond["e_ratio"], np.float64) if "e_ratio" in cond else e
     with np.errstate(divide="ignore", invalid="ignore"):
-        rel = e + (np.abs(dg) * e + 2.0 ** -22 * mag) / np.abs(g) + 1e-5
-    k = np.where(np.isfinite(rel), np.ceil(rel * 256.0), BF16_ULPS)  # bf16 ulp >= 2^-8 relative
-    k = np.where(g == 0, BF16_ULPS, k)
-    return np.maximum(BF16_ULPS, k).astype(np.int64)
+        rel = e + (u * e_r + k * e + 2.0 ** -22 * (u + k)) / np.abs(g) + 1e-5
+    n_ulp = np.where(np.isfinite(rel), np.ceil(rel * 256.0), BF16_ULPS)  # ulp >= 2^-8 relative
+    n_ulp = np.where(g == 0, BF16_ULPS, n_ulp)
+    return np.maximum(BF16_ULPS, n_ulp).astype(np.int64)
 
 
 def compare(gpu_logp, gpu_dlogits, gpu_loss, ref, dlogits_dtype, eps_low=0.2, eps_high=0.2,

@@ -9,7 +9,7 @@ import dataclasses
 import numpy as np
 import pytest
 
-from loss_compare import LOSS_RTOL, compare, compare_rows
+from loss_compare import LOSS_RTOL, allowed_ulps, compare, compare_rows
 from paper_2609_36932_gb300 import workloads
 from paper_2609_36932_gb300.pipeline import GrpoStep, StepParams
 
@@ -337,6 +337,61 @@ def test_gspo_step_matches_oracle(oracle_mod, name):
     else:
         assert np.abs(d.astype(np.float64) - ref["dlogits"].astype(np.float64)).max() <= 1e-6
     assert abs(float(step.loss.item()) - ref["loss"]) <= LOSS_RTOL * abs(ref["loss"]) + 1e-12
+
+
+def test_gspo_full_size_against_oracle(oracle_mod):
+    """GSPO's sequence-level loss on the full qwen step: every kept row's logp, every kept
+    sequence's ratio and the total loss against the oracle run over all kept rows (without
+    dlogits), and the dlogits of whole sequences (the first ones and the longest, at least 1024
+    rows) against the oracle run on those sequences alone with the same sequence count."""
+    import torch
+    from helpers import bf16_ulp_distance
+    from test_gpu_gspo import RATIO_RTOL
+    w, b, step, h = build("qwen", chunk_rows=0, ratio_level="sequence", eps_low=0.2,
+                          eps_high=0.28)
+    step.run()
+    torch.cuda.synchronize()
+    assert int(step.status.item()) == 0
+    adv, comp = check_selection(oracle_mod, w, b, step)
+    TK, K = step.T_kept, step.K
+    st, ko, kidx = comp["src_token"], comp["kept_off"][:K + 1], comp["kept_idx"][:K]
+    lg = host_bits(h["logits"][torch.from_numpy(st).cuda()])  # the kept rows, in order
+    kw = dict(eps_low=0.2, eps_high=0.28, beta=w.beta)
+    o = oracle_mod.gspo_loss(lg, w.V, b["ids"][st], h["old"][st], h["ref"][st], adv, kidx, ko,
+                             want_dlogits=False, **kw)
+    logp = step.logp[:TK].cpu().numpy().astype(np.float64)
+    assert np.abs(logp - o["logp"]).max() <= 2e-5
+    s_gpu, s_o = step.seq_ratio[:K].cpu().numpy(), o["seq_ratio"]
+    np.testing.assert_allclose(s_gpu, s_o, rtol=RATIO_RTOL)
+    lo, hi = 0.8, 1.0 + np.float64(np.float32(0.28))
+    near = (np.abs(s_o - lo) <= RATIO_RTOL * lo) | (np.abs(s_o - hi) <= RATIO_RTOL * hi)
+    widen = float(np.sum(np.abs(adv[kidx][near].astype(np.float64)) * RATIO_RTOL * hi)) / K
+    loss = float(step.loss.item())
+    assert abs(loss - o["loss"]) <= LOSS_RTOL * abs(o["loss"]) + 1e-12 + widen
+    # dlogits of whole sequences: the first ones up to 1024 rows, and the longest
+    lens = np.diff(ko)
+    pick = sorted(set(list(range(int(np.searchsorted(np.cumsum(lens), 1024)) + 1)) +
+                      [int(np.argmax(lens))]) - set(np.flatnonzero(near).tolist()))
+    rows = np.concatenate([np.arange(ko[k], ko[k + 1]) for k in pick])
+    sub_off = np.concatenate([[0], np.cumsum(lens[pick])]).astype(np.int64)
+    src = st[rows]
+    od = oracle_mod.gspo_loss(host_bits(h["logits"][torch.from_numpy(src).cuda()]), w.V,
+                              b["ids"][src], h["old"][src], h["ref"][src], adv, kidx[pick],
+                              sub_off, n_seq=K, dlogits_dtype=1, **kw)
+    d = host_bits(step.dlogits[:TK][torch.from_numpy(rows).cuda()])
+    assert rows.size >= 1024
+    # the bar of each row: 1 ulp, widened where g_t is ill-conditioned (loss_compare); the error
+    # of log s is bounded by the largest logp error of the sequence
+    e = np.abs(logp - o["logp"]) + 2.0 ** -24 * np.abs(o["logp"])
+    e_seq = np.repeat([e[ko[k]:ko[k + 1]].max() for k in pick], lens[pick])
+    bar = allowed_ulps(logp[rows], dict(logp=o["logp"][rows], g=od["g"]),
+                       dict(ref_logp=h["ref"][src], beta=w.beta, e_ratio=e_seq))
+    dist = bf16_ulp_distance(d, od["dlogits"]).max(axis=1)
+    assert np.all(dist <= bar), (int(dist.max()), bar[dist > bar][:5])
+    print("qwen GSPO: %d rows, %d sequences, %d at a clip boundary, loss %.12g (oracle %.12g), "
+          "dlogits of %d sequences (%d rows, worst %d ulps, %d rows with an ill-conditioned g_t)"
+          % (TK, K, int(near.sum()), loss, o["loss"], len(pick), rows.size, int(dist.max()),
+             int((bar > 1).sum())))
 
 
 @pytest.mark.parametrize("name,ratio", [("small", "token"), ("small", "sequence")])

@@ -94,6 +94,30 @@ def test_gradient_matches_finite_differences(oracle_mod):
     np.testing.assert_allclose(out["dlogits_f64"], fd, rtol=1e-6, atol=1e-9)
 
 
+def test_gradient_factor_g(oracle_mod):
+    """The oracle's per-row g_t: dlogits[t] / (e_y - p) = g_t / (n_seq L_k) for every row (the
+    dlogits themselves are pinned by finite differences above), NaN in a sequence without a
+    ratio."""
+    rng = np.random.default_rng(33)
+    lens, V = [4, 1, 3, 0, 2], 11
+    z, y, old, ref, off = batch(rng, lens, V, old_sd=0.1, scale=1.5)
+    y = y.copy()
+    y[-1] = V + 2  # the last sequence has an invalid token: no ratio
+    adv = np.array([0.9, -0.4, 0.0, 1.0, 0.5], np.float32)
+    out = oracle_mod.gspo_loss(z, V, y, old, ref, adv, np.arange(5), off, n_seq=6, eps_low=0.2,
+                               eps_high=0.28, beta=0.3, want_f64=True)
+    zz = z.astype(np.float64)
+    p = np.exp(zz - scipy.special.logsumexp(zz, 1, keepdims=True))
+    e = np.zeros_like(p)
+    ok = (y >= 0) & (y < V)
+    e[np.flatnonzero(ok), y[ok]] = 1.0
+    L = np.repeat(np.asarray(lens), lens).astype(np.float64)
+    g = out["g"]
+    assert np.all(np.isnan(g[-2:])) and np.all(np.isfinite(g[:-2]))
+    np.testing.assert_allclose(out["dlogits_f64"][:-2] / (e - p)[:-2],
+                               (g[:-2] / (6 * L[:-2]))[:, None].repeat(V, 1), rtol=1e-9)
+
+
 def test_clipping_is_per_sequence(oracle_mod):
     """A sequence whose ratio is clipped (A > 0, s > 1 + eps_high, beta = 0) gets zero gradient
     on every token, including tokens whose own ratio lies inside the clip range; the token-level
