@@ -156,8 +156,8 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
     logits_dtype=2, float64).
 
     Returns dict(loss, logp [n_rows] f64, rho, row_loss, g (each row's gradient factor g_t, so
-    that dlogits[t] = w_t * g_t * (onehot(y) - softmax)), dlogits (f32 array or uint16 bf16 bits,
-    [n_rows, V]) and, with want_f64, dlogits_f64).
+    that dlogits[t] = w_t * g_t * (onehot(y) - softmax)), w (the weights w_t), dlogits (f32 array
+    or uint16 bf16 bits, [n_rows, V]) and, with want_f64, dlogits_f64).
     """
     lg = np.ascontiguousarray(logits)
     if logits_dtype is None:
@@ -192,8 +192,14 @@ def loss(logits, V: int, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2
                            _p(logp), _p(rho), _p(rl), _p(total), _p(g))
     if rc != 0:
         raise ValueError("oracle_loss: bad arguments")
+    # each row's aggregation weight w_t (1/denom_tokens, or 1/(n_seq |o_i|) per sequence)
+    if agg_mode == 0:
+        w = np.full(n_rows, 1.0 / float(denom_tokens))
+    else:
+        lens = (so[1:] - so[:-1]).astype(np.float64)
+        w = 1.0 / (float(n_seq) * lens[rr[:n_rows]]) if n_rows else np.zeros(0)
     return dict(loss=float(total[0]), logp=logp[:n_rows], rho=rho[:n_rows], row_loss=rl[:n_rows],
-                g=g[:n_rows], dlogits=dl, dlogits_f64=d64)
+                g=g[:n_rows], w=w, dlogits=dl, dlogits_f64=d64)
 
 
 def lmhead_loss(hidden, weight, y, old_logp, ref_logp, adv, row_rollout, *, eps_low=0.2,

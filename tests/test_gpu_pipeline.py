@@ -233,6 +233,31 @@ def test_step_variants(oracle_mod, variant):
     assert float(step.loss.item()) == loss0 and torch.equal(step.dlogits[:TK], dl0)
 
 
+@pytest.mark.parametrize("name", ["tiny", "small"])
+def test_step_with_every_group_zero_advantage(oracle_mod, name):
+    """Every prompt's rewards equal (a different value per prompt): every advantage is 0, each
+    group is one advantage class, and the loss and dlogits carry the KL term alone; the step
+    matches the oracle in full."""
+    import torch
+    w, b, step, h = build(name, chunk_rows=0)
+    r = np.repeat(np.arange(w.P, dtype=np.float32) * 0.25, w.G)
+    b["rewards"] = r
+    step.rewards.copy_(torch.from_numpy(r))
+    step.run()
+    torch.cuda.synchronize()
+    assert int(step.status.item()) == 0
+    adv, comp = check_selection(oracle_mod, w, b, step)
+    assert np.all(adv == 0) and comp["K"] >= w.P
+    TK = step.T_kept
+    ref = oracle_mod.loss(host_bits(h["logits"]), w.V, b["ids"], h["old"], h["ref"], adv,
+                          comp["token_rollout"], row_index=comp["src_token"], eps_low=w.eps,
+                          eps_high=w.eps, beta=w.beta, denom_tokens=TK,
+                          dlogits_dtype=1 if w.dlogits_dtype == "bf16" else 0)
+    compare(step.logp[:TK].cpu().numpy(), host_bits(step.dlogits[:TK]), float(step.loss.item()),
+            ref, w.dlogits_dtype, gpu_row_loss=step.row_loss[:TK].cpu().numpy(),
+            cond=dict(ref_logp=h["ref"][comp["src_token"]], beta=w.beta))
+
+
 def test_upload_kept_copies_only_kept_rows():
     """grpo_upload_kept: kept rollouts' rows arrive intact, pruned rows keep their old contents,
     one copy per run of consecutive kept rollouts, on two row widths."""

@@ -207,6 +207,10 @@ def test_seq_mean_weights(oracle_mod):
     # token mean weights 1/5; Eq. 1's weights 1/(2*2) and 1/(2*3)
     scale = np.array([5 / 4, 5 / 4, 5 / 6, 5 / 6, 5 / 6])
     np.testing.assert_allclose(seq["row_loss"], tok["row_loss"] * scale, rtol=1e-14)
+    # the weights the oracle reports are those weights: both give the same unweighted l_t
+    np.testing.assert_allclose(tok["w"], np.full(5, 1 / 5), rtol=1e-15)
+    np.testing.assert_allclose(seq["w"], [1 / 4, 1 / 4, 1 / 6, 1 / 6, 1 / 6], rtol=1e-15)
+    np.testing.assert_allclose(seq["row_loss"] / seq["w"], tok["row_loss"] / tok["w"], rtol=1e-14)
 
 
 def test_invalid_token_row_is_zero(oracle_mod):
