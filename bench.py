@@ -606,7 +606,7 @@ def lmhead_side(w, b, step, seed, dev, reps=3):
     import paper_2609_36932_gb300 as g
     from paper_2609_36932_gb300 import workloads
     D = workloads.LMHEAD_D
-    need = (b["T"] * D * 2 + w.V * D * 6 + 5 * (1 << 30))
+    need = (b["T"] * D * 2 + w.V * D * 6 + 14 * (1 << 30))
     free, _ = torch.cuda.mem_get_info(dev)
     if need > 0.8 * free:
         return None
@@ -632,16 +632,35 @@ def lmhead_side(w, b, step, seed, dev, reps=3):
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / reps
+    # the same calls with the logits recomputed in a second tensor-core pass (the other setting)
+    g.grpo_lmhead_tune(0, 0, 1)
+    try:
+        g.grpo_lmhead_loss_fwd_bwd(hid, wt, ids, old, ref, step.adv, step.token_rollout,
+                                   dhidden=dh, dweight=dw, ws=ws, **kw)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            g.grpo_lmhead_loss_fwd_bwd(hid, wt, ids, old, ref, step.adv, step.token_rollout,
+                                       dhidden=dh, dweight=dw, ws=ws, **kw)
+        e1.record(stream)
+        torch.cuda.synchronize()
+    finally:
+        g.grpo_lmhead_tune(0, 0, 0)
+    ms_rec = e0.elapsed_time(e1) / reps
     peak, src = measured_tensor_peak(sustained=True)
-    tf = 8.0 * T_kept * w.V * D / (ms / 1e3) / 1e12
+    tf = 6.0 * T_kept * w.V * D / (ms / 1e3) / 1e12
     del hid, wt, old, ref, dh, dw, ws, out
     torch.cuda.empty_cache()
     return {"call": "grpo_lmhead_loss_fwd_bwd", "D": D, "T_kept": T_kept, "calls": reps,
             "ms_per_call": ms, "kept_tokens_per_s": T_kept / (ms / 1e3), "achieved": tf,
             "unit": "TFLOP/s", "peak": peak, "frac": tf / peak, "peak_source": src,
+            "ms_per_call_recomputed_logits": ms_rec,
             "note": "the output layer fused with the loss on this batch's kept rows: logits "
-                    "h W^T on the tcgen05 tensor cores (never stored), loss, dhidden, dweight; "
-                    "8 T_kept V D FLOPs per call; bench.py --loss lmhead runs it as a step"}
+                    "h W^T on the tcgen05 tensor cores (f32 logits kept one chunk at a time), "
+                    "loss, dlogits, dhidden, dweight; 6 T_kept V D algorithmic FLOPs per call "
+                    "(forward logits and the two products); ms_per_call_recomputed_logits: the "
+                    "same call recomputing the logits in a second tensor-core pass instead "
+                    "(grpo_lmhead_tune); bench.py --loss lmhead runs it as a step"}
 
 
 def lmhead_products(d, step, T_kept, V, D, peak, peak_src, nrep=3):
@@ -780,12 +799,17 @@ def run_lmhead(args, w):
                           "grpo_lmhead_logp_fwd on the step's kept rows",
                 "algorithmic_flops_per_launch": flops_pass, "launch_ms": f_ms,
                 "peak_source": peak_src}
-    step_tc = {"flops_per_step": 4 * flops_pass, "loss_ms": loss_ms,
-               "achieved": 4 * flops_pass / (loss_ms / 1e3) / 1e12, "unit": "TFLOP/s",
-               "peak": peak_s, "frac": 4 * flops_pass / (loss_ms / 1e3) / 1e12 / peak_s,
+    step_tc = {"flops_per_step": 3 * flops_pass, "loss_ms": loss_ms,
+               "achieved": 3 * flops_pass / (loss_ms / 1e3) / 1e12, "unit": "TFLOP/s",
+               "peak": peak_s, "frac": 3 * flops_pass / (loss_ms / 1e3) / 1e12 / peak_s,
                "peak_source": peak_s_src,
-               "note": "the whole fused call: pass 1, pass 2 and the dhidden and dweight "
-                       "products (2 T V D each), all on the library's tcgen05 kernels"}
+               "note": "the whole fused call against its algorithmic work: the forward logits "
+                       "and the dhidden and dweight products (2 T V D each), all on the "
+                       "library's tcgen05 kernels; "
+                       + ("GSPO's entry recomputes the logits in a second pass (2 T V D more "
+                          "executed)" if gspo else
+                          "the token loss keeps each chunk's f32 logits from pass 1 and forms "
+                          "dlogits from them in a streaming pass")}
     products = None if gspo else lmhead_products(d, step, T_kept, w.V, D, peak, peak_src)
 
     # end to end: selection inputs, log-probs and hidden states from pinned host memory (hidden

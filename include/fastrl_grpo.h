@@ -309,7 +309,8 @@ grpo_status grpo_gspo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype,
  * runs the kept trajectories through the policy, whose last layer maps each token's hidden state
  * to logits over the vocabulary; Eqs. 1-3 give the loss.  Here the logits
  *   z[t, v] = sum_d hidden[t, d] * weight[v, d]
- * are produced on the tensor cores 128 x 256 at a time and consumed on chip, never stored whole:
+ * are produced on the tensor cores 128 x 256 at a time, one chunk of rows at a time (never all
+ * rows at once):
  *   loss, logp_out, row_loss_out: as grpo_loss_fwd_bwd on z (rows in order, row_index = NULL);
  *   dhidden[t, :] = sum_v dlogits[t, v] * weight[v, :]         (chain rule through z = h W^T)
  *   dweight[v, :] = sum_t dlogits[t, v] * hidden[t, :]          (+ the old dweight with
@@ -327,15 +328,20 @@ grpo_status grpo_gspo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype,
  * dlogits_out: nullable device bf16 [n_rows, grpo_lmhead_dlogits_stride(V)], 16-byte aligned;
  *   when given it receives every row's dlogits (columns >= V are 0) and no chunk buffer is used.
  * logp_out (f32 [n_rows]) and row_loss_out (f64 [n_rows]): nullable.  loss_out: device f64 [1].
- * chunk_rows: rows of dlogits held at a time (rounded up to a multiple of 128); 0 picks the
- *   largest count that fits a 4 GiB bf16 chunk.  Smaller chunks need less workspace.
- * Workspace: per row 1.3 KB of softmax statistics, the chunk of dlogits (unless dlogits_out) and
- *   the f32 partial products of a split K (see grpo_lmhead_grad).
- * Kernels: pass 1 (statistics), pass 2 (dlogits, per chunk) and the two products per chunk
- *   (grpo_lmhead_grad's) are tcgen05 kernels with TMA operand loads and TMEM accumulators, one
- *   CTA per SM; a row kernel applies Eqs. 1-3 between the passes.  Limits: n_rows < 2^31;
- *   V >= 1; D >= 8.  Errors: GRPO_ERR_INVALID_ARG for bad sizes, alignment, NULL required
- *   pointers; GRPO_ERR_CUDA when a launch or the tensor-map encoder fails.
+ * chunk_rows: rows of logits and dlogits held at a time (rounded up to a multiple of 128); 0
+ *   picks the largest count whose bf16 dlogits fit 4 GiB (their f32 logits then take 8 GiB).
+ *   Smaller chunks need less workspace.
+ * Workspace: per row 8 bytes per 256 vocabulary entries of softmax statistics; per chunk row
+ *   4 * grpo_lmhead_dlogits_stride(V) bytes of f32 logits (none when grpo_lmhead_tune selects
+ *   recomputation) and 2 * grpo_lmhead_dlogits_stride(V) of dlogits (none with dlogits_out); the
+ *   f32 partial products of a split K (see grpo_lmhead_grad).
+ * Kernels, per chunk: pass 1 (softmax statistics; the chunk's f32 logits stored) and the two
+ *   products (grpo_lmhead_grad's) are tcgen05 kernels with TMA operand loads and TMEM
+ *   accumulators, one CTA per SM; a row kernel applies Eqs. 1-3 and a streaming kernel forms
+ *   dlogits from the stored logits.  The forward results (logp, loss, row terms) do not depend
+ *   on chunk_rows or on the launch settings.  Limits: n_rows < 2^31; V >= 1; D >= 8.
+ *   Errors: GRPO_ERR_INVALID_ARG for bad sizes, alignment, NULL required pointers;
+ *   GRPO_ERR_CUDA when a launch or the tensor-map encoder fails.
  */
 grpo_status grpo_lmhead_loss_fwd_bwd(const void* hidden, int64_t hidden_stride,
                                      const int64_t* row_index, int64_t n_rows, const void* weight,
@@ -384,8 +390,10 @@ grpo_status grpo_lmhead_grad(const void* dlogits, int64_t dlogits_stride, int64_
  *   logp_out[t] = z_y - log sum_v exp(z_v),  z = hidden[src] * weight^T,  y = y[src]
  * The pass-1 kernel of grpo_lmhead_loss_fwd_bwd alone (plus its row kernel): no loss, no gradient.
  * hidden, hidden_stride, row_index, n_rows, weight, V, D, y, status: as grpo_lmhead_loss_fwd_bwd.
- * logp_out: device f32 [n_rows] (NaN for a token id outside [0, V)).  Workspace: per row 1.3 KB,
- * plus the gathered rows with row_index.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
+ * logp_out: device f32 [n_rows] (NaN for a token id outside [0, V)); the same bits as
+ * grpo_lmhead_loss_fwd_bwd's logp_out for the same rows.  Workspace: per row 8 bytes per 256
+ * vocabulary entries and 4 bytes, plus the gathered rows with row_index.  Limits and errors: as
+ * grpo_lmhead_loss_fwd_bwd.
  */
 grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
                                  const int64_t* row_index, int64_t n_rows, const void* weight,
@@ -405,10 +413,13 @@ grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
  * logp_out: device f32 [n_rows], required.  seq_ratio_out: nullable f32 [n_seq_rows] (NaN for a
  *   sequence with an invalid token or no rows).  loss_out: device f64 [1].
  * With no rows or no sequences the loss is 0 and dhidden (and dweight unless accumulated) are 0.
- * Kernels: pass 1, a row kernel (logp and softmax statistics), one warp per sequence (ratio, clip,
- *   loss term, row gradient scalars), the fixed-order sum, then pass 2 and the two GEMMs.
- * Workspace: as grpo_lmhead_loss_fwd_bwd, with 16 bytes per row and 8 per sequence in place of the
- *   per-row loss terms.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
+ * Kernels: pass 1 over every row, a row kernel (logp and softmax statistics), one warp per
+ *   sequence (ratio, clip, loss term, row gradient scalars), the fixed-order sum, then per chunk
+ *   pass 2 (the tiles recomputed on the tensor cores, dlogits written from tensor memory: a
+ *   sequence may cross a chunk boundary, so no chunk of logits can be kept until its rows'
+ *   scalars are known) and the two GEMMs.
+ * Workspace: as grpo_lmhead_loss_fwd_bwd with recomputed logits, with 16 bytes per row and 8 per
+ *   sequence in place of the per-row loss terms.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
  */
 grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
     const void* hidden, int64_t hidden_stride, const int64_t* row_index, int64_t n_rows,
@@ -423,9 +434,14 @@ grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
  * grpo_lmhead_tune — launch settings of the output-layer kernels for this process (no counterpart
  * in the paper).  prefetch: k-blocks (64 of D) by which an L2 prefetch of each operand tile runs
  * ahead of its load, 0..64 (0: none).  row_lanes: pairs of 128-row blocks the grid works on at
- * once, 1..8, or 0 to let the library choose per launch.  Returns GRPO_ERR_INVALID_ARG for other values.
+ * once, 1..8, or 0 to let the library choose per launch.  recompute_logits: 0 (default) lets
+ * grpo_lmhead_loss_fwd_bwd store each chunk's f32 logits in pass 1 and form dlogits from them;
+ * 1 makes it recompute the logits in a second tensor-core pass instead (a quarter more FLOPs,
+ * 4 bytes per chunk entry less workspace).  The results are the same bits either way.  A size
+ * query and the call it sizes must see the same setting.  Returns GRPO_ERR_INVALID_ARG for other
+ * values.
  */
-grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes);
+grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes, int32_t recompute_logits);
 
 /* Row stride, in elements, of grpo_lmhead_loss_fwd_bwd's dlogits_out: V rounded up to a multiple
  * of 32 (0 for V < 1). */

@@ -129,7 +129,7 @@ def lib():
                                                 _f32, _f32, _c_p, _i32, _c_p, _i32, _c_p, _c_p,
                                                 _c_p, _c_p, _c_p, _i64, _c_p, _c_p, _c_p]
     L.grpo_lmhead_gspo_loss_fwd_bwd.restype = _i32
-    L.grpo_lmhead_tune.argtypes = [_i32, _i32]
+    L.grpo_lmhead_tune.argtypes = [_i32, _i32, _i32]
     L.grpo_lmhead_tune.restype = _i32
     L.grpo_lmhead_dlogits_stride.argtypes = [_i32]
     L.grpo_lmhead_dlogits_stride.restype = _i64
@@ -398,9 +398,9 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
 
 
-def grpo_lmhead_tune(prefetch: int = 0, row_lanes: int = 0):
+def grpo_lmhead_tune(prefetch: int = 0, row_lanes: int = 0, recompute_logits: int = 0):
     """Launch settings of the output-layer kernels for this process (see the header)."""
-    _check(lib().grpo_lmhead_tune(int(prefetch), int(row_lanes)))
+    _check(lib().grpo_lmhead_tune(int(prefetch), int(row_lanes), int(recompute_logits)))
 
 
 def grpo_lmhead_dlogits_stride(V: int) -> int:

@@ -7,18 +7,23 @@
 //   loss, logp: Eqs. 1-3 on z, as grpo_loss_fwd_bwd computes them
 //   dh = dlogits * W,   dW = dlogits^T * h        (the chain rule through z = h W^T)
 // The [rows, V] logits are never stored whole.  They are produced 128 x 256 at a time into
-// tensor memory by tcgen05.mma (bf16 operands staged in shared memory by TMA, f32 accumulators)
-// and consumed there:
-//   Pass 1 (lmhead_tile_kernel<false>): per row, the running maximum and the sum of exp(z - max)
-//     over the vocabulary tiles a CTA visits (z_y excluded from the sum and kept separately).
-//   lmhead_rows_kernel: the partial sums combined -> lse, logp, the loss term and the gradient
-//     scalars of each row (the same formulas as the fused loss kernel).
-//   Pass 2 (lmhead_tile_kernel<true>), for each chunk of rows: the tiles recomputed and
-//     dlogits = coef * ([v == y] - softmax(z)_v) written in bf16 to a chunk buffer.
+// tensor memory by tcgen05.mma (bf16 operands staged in shared memory by TMA, f32 accumulators).
+// The token loss runs chunk by chunk (rows of logits held at a time):
+//   Pass 1 (lmhead_tile_kernel<false>): per row and vocabulary tile, the maximum and the sum of
+//     exp(z - max) (z_y excluded from the sum and kept separately); the chunk's f32 logits are
+//     stored as they leave tensor memory.
+//   lmhead_rows_kernel: the per-tile sums combined in a fixed order -> lse, logp, the loss term
+//     and the gradient scalars of each row (the same formulas as the fused loss kernel).
+//   lmhead_dlogits_kernel: dlogits = coef * ([v == y] - softmax(z)_v) in bf16 from the stored
+//     logits, a streaming pass (6 bytes per entry instead of a second 2 D FLOPs per entry).
 //   Two products per chunk on the same tensor-core machinery (gemm.cu): dh = dlogits * W and
 //     dW (+)= dlogits^T * h.
+// GSPO's loss couples every row of a sequence, and a sequence may cross a chunk boundary, so its
+// entry runs pass 1 over every row first and then, per chunk, pass 2 (lmhead_tile_kernel<true>),
+// which recomputes the tiles and writes dlogits from tensor memory; grpo_lmhead_tune can select
+// that recomputation for the token loss too (less workspace: no chunk of f32 logits).
 //
-// Kernel roles (320 threads, one CTA per SM: 214 KB of shared memory, all 512 TMEM columns).  A
+// Kernel roles (320 threads, one CTA per SM: 225 KB of shared memory, all 512 TMEM columns).  A
 // tile is a pair of 128-row blocks of h against 256 vocabulary entries, so each weight stage
 // feeds two row blocks: per FLOP a third fewer bytes land in shared memory than with one row
 // block per tile, which on GB300 made the kernel 5.5% faster (shared-memory traffic, not the
@@ -34,10 +39,11 @@
 // pairs it takes pair g*R + i and the vocabulary tiles j, j + J, j + 2J, ...  At any time the grid
 // works on 2R consecutive row blocks and J consecutive vocabulary tiles, which the L2 serves to
 // all of it; the weight streams from DRAM about once per group (R = 4..8 pairs, chosen per
-// launch for the fewest idle CTAs).  Pass 2 stages each warp's 32 x 32 block of dlogits in shared
-// memory and writes it as 64-byte row pieces (1.3% faster than 16-byte pieces straight from the
-// registers), with streaming stores so that they do not displace the operand tiles in L2.  An L2 prefetch of upcoming tiles (grpo_lmhead_tune) is
-// off by default: on GB300 it made pass 1 about 16% slower.
+// launch for the fewest idle CTAs).  Pass 1 stages each warp's 32 x 32 block of f32 logits in
+// shared memory and writes it as 128-byte row pieces; pass 2 its 32 x 32 block of dlogits as
+// 64-byte row pieces (1.3% faster than 16-byte pieces straight from the registers); both with
+// streaming stores so that they do not displace the operand tiles in L2.  An L2 prefetch of
+// upcoming tiles (grpo_lmhead_tune) is off by default: on GB300 it made pass 1 about 16% slower.
 //
 // Every wait is bounded (about a second): a wait that runs out sets GRPO_DEVFLAG_TIMEOUT and an
 // abort flag; the roles then stop, the producer waits for its copies in flight and the MMA lane
@@ -69,13 +75,17 @@ constexpr uint32_t kStageBytes = 2 * kABytes + kBBytes;  // two row blocks share
 constexpr int kThreads = 320;
 constexpr uint32_t kTmemCols = 2 * BN;  // one accumulator per row block of the pair
 constexpr int kRowLanes = 8;       // R: row-block pairs in flight across the grid
-constexpr int kMaxJ = 160;         // vocabulary lanes (partial sums per row) at most
+constexpr int kMaxJ = 160;         // vocabulary lanes at most
 // Barriers: full and empty per stage, accumulator-pair full and released (two slots each, the
 // first in use), drain.
 constexpr int kBars = 2 * kStages + 5;
-constexpr uint32_t kStageOutBytes = 8 * 32 * 64;  // per epilogue warp: 32 rows x 32 bf16
+// Output staging per epilogue warp: 32 rows x 128 bytes (32 f32 logits in pass 1, 32 bf16 dlogits
+// in pass 2, which uses the first half).
+constexpr uint32_t kStageWarpBytes = 32 * 128;
+constexpr uint32_t kStageOutBytes = 8 * kStageWarpBytes;
 constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + 8 * kBars + 16 + 128 +
                               kStageOutBytes;
+static_assert(kSmemBytes <= 227 * 1024, "the tile kernel's shared memory exceeds a CTA's limit");
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int64_t kDefaultChunkBytes = 4ll << 30;  // dlogits chunk buffer
 
@@ -107,8 +117,10 @@ struct TileArgs {
   // n_rb counts row blocks; tiles take them in pairs (2p, 2p + 1)
   const int32_t* y;  // [rows]
   // pass 1
-  float2* part;  // [rows][J]: (max, sum of exp(z - max) without z_y) of vocabulary lane j
+  float2* part;  // [rows][n_vt]: (max, sum of exp(z - max) without z_y) of vocabulary tile vt
   float* zy;     // [rows]: z_y, written by the CTA whose tile holds y
+  float* z;      // nullable [rows][ldz]: the f32 logits, stored for the dlogits pass
+  int64_t ldz;
   // pass 2
   const float4* rowsc;  // [rows]: {neg_scale, dy, shift, 0} from lmhead_rows_kernel
   __nv_bfloat16* dl;    // [rows][ldd]
@@ -288,11 +300,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row = rb * BM + r_in;
       const bool rv = row < a.rows;
       const int yv = rv ? a.y[row] : -1;
-      float m = -INFINITY, s = 0.f;  // pass 1: running max, sum of exp(z - m) without z_y
       float4 sc = make_float4(0.f, 0.f, 0.f, 0.f);
       if (kBwd && rv) sc = a.rowsc[row];
       const float neg_scale = sc.x, dy = sc.y, shB = sc.z;
+      const uint32_t blk = stage_out_s + (uint32_t)(warp - 2) * kStageWarpBytes;
       for (int vt = lj; vt < a.n_vt; vt += J) {
+        // pass 1: this tile's maximum and sum of exp(z - m) without z_y
+        float m = -INFINITY, s = 0.f;
         int got = 0;
         if (lane == 0) got = wait_bar(accf_bar(0), tiles & 1u, true) ? 1 : 0;
         got = __shfl_sync(0xffffffffu, got, 0);
@@ -311,6 +325,34 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int nvalid = a.V - v0;  // >= 1
           const int jy = yv - v0;       // y's column in this chunk, if in [0, 32)
           if (!kBwd) {
+            if (a.z != nullptr) {
+              // The row's 32 logits through shared memory (16-byte pieces XOR-swizzled by row,
+              // conflict-free), then each store instruction covers 4 rows x 128 contiguous bytes.
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const uint32_t addr = blk + lane * 128u + (uint32_t)((k ^ (lane & 7)) * 16);
+                asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+                             "f"(x[4 * k]), "f"(x[4 * k + 1]), "f"(x[4 * k + 2]),
+                             "f"(x[4 * k + 3])
+                             : "memory");
+              }
+              __syncwarp();
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                const int rr = i * 4 + (lane >> 3);  // row within the warp's 32
+                const int kc = lane & 7;             // 16-byte piece of that row
+                const uint32_t addr = blk + rr * 128u + (uint32_t)((kc ^ (rr & 7)) * 16);
+                float4 v;
+                asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                             : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                             : "r"(addr)
+                             : "memory");
+                const int grow = rb * BM + q * 32 + rr;
+                if (grow < a.rows)  // streaming: the logits must not push the operands out of L2
+                  __stcs(reinterpret_cast<float4*>(a.z + (int64_t)grow * a.ldz + v0) + kc, v);
+              }
+              __syncwarp();
+            }
             float cm = -INFINITY;
 #pragma unroll
             for (int k = 0; k < 32; ++k) {
@@ -353,7 +395,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Through shared memory: each lane writes its row's 64 bytes (16-byte pieces XOR-
             // swizzled by row, conflict-free), then each store instruction covers 8 rows x 64
             // contiguous bytes instead of 32 rows x 16 bytes.
-            const uint32_t blk = stage_out_s + (uint32_t)(warp - 2) * 2048u;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               const uint32_t addr = blk + lane * 64u + (uint32_t)((k ^ ((lane >> 1) & 3)) * 16);
@@ -383,8 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         mbar_arrive(acce_bar(0));
         ++tiles;
+        if (!kBwd && rv) a.part[(int64_t)row * a.n_vt + vt] = make_float2(m, s);
       }
-      if (!kBwd && ok && rv) a.part[(int64_t)row * J + lj] = make_float2(m, s);
     }
   }
 
@@ -400,8 +441,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 struct RowArgs {
-  int32_t rows, J, V;
-  const float2* part;
+  int32_t rows, n_vt, V;
+  const float2* part;  // [rows][n_vt]
   const float* zy;
   const int32_t* y;
   const float *old_logp, *ref_logp, *adv;
@@ -421,13 +462,19 @@ struct RowArgs {
   float4* stats;
 };
 
-// One thread per row: combine the J partial sums and apply Eqs. 1-3 (the same arithmetic as the
-// fused loss kernel's row scalars).
-__global__ void __launch_bounds__(256) lmhead_rows_kernel(const RowArgs a) {
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+constexpr int kRowWarps = 8;
+
+// One warp per row: combine the row's per-tile partial sums, then apply Eqs. 1-3 in lane 0 (the
+// same arithmetic as the fused loss kernel's row scalars).  Lane l takes tiles l, l + 32, ...,
+// and the lanes' values meet in a fixed xor tree, so the result depends only on the row's
+// logits: not on how pass 1's grid visited the tiles, nor on how the rows were chunked.
+__global__ void __launch_bounds__(kRowWarps * 32) lmhead_rows_kernel(const RowArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int t = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
   if (t >= a.rows) return;
   const int yv = a.y[t];
   if (yv < 0 || yv >= a.V) {
+    if (lane != 0) return;
     if (a.logp_out) a.logp_out[t] = __int_as_float(0x7fc00000);
     if (a.mode == 0) {
       a.row_loss[t] = 0.0;
@@ -436,14 +483,19 @@ __global__ void __launch_bounds__(256) lmhead_rows_kernel(const RowArgs a) {
     if (a.status) atomicOr(a.status, GRPO_DEVFLAG_BAD_TOKEN);
     return;
   }
-  const float2* p = a.part + (int64_t)t * a.J;
+  const float2* p = a.part + (int64_t)t * a.n_vt;
   float M = -INFINITY;
-  for (int j = 0; j < a.J; ++j) M = fmaxf(M, p[j].x);
+  for (int j = lane; j < a.n_vt; j += 32) M = fmaxf(M, p[j].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
   float S_excl = 0.f;
-  for (int j = 0; j < a.J; ++j) {
+  for (int j = lane; j < a.n_vt; j += 32) {
     const float2 v = p[j];
     if (v.x != -INFINITY) S_excl += v.y * expf(v.x - M);
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) S_excl += __shfl_xor_sync(0xffffffffu, S_excl, o);
+  if (lane != 0) return;
   const float zy = a.zy[t];
   const float S = S_excl + expf(zy - M);
   const float logp = (zy - M) - logf(S);
@@ -567,6 +619,61 @@ __global__ void __launch_bounds__(kSeqWarps * 32) lmhead_gspo_seq_kernel(const S
   }
 }
 
+struct DlArgs {
+  const float* z;        // [rows][ld]: pass 1's f32 logits
+  __nv_bfloat16* dl;     // [rows][ld]
+  int64_t ld;            // row stride of both, a multiple of 32
+  const float4* rowsc;   // [rows]: {neg_scale, dy, shift, 0} from lmhead_rows_kernel
+  const int32_t* y;      // [rows]
+  int32_t rows, V, segs;  // segs: tiles of kDlSeg entries per row
+};
+constexpr int kDlThreads = 256;
+constexpr int kDlSeg = kDlThreads * 16;  // two 8-entry vectors per thread and tile
+
+// dlogits from the stored logits, with pass 2's arithmetic on the same f32 values (so the same
+// bits as recomputing the tile): d = neg_scale * 2^(z log2(e) + shift), dy at v = y, 0 for v >= V.
+// A persistent grid over (row, 4096-entry segment) tiles; each thread reads two 32-byte pieces of
+// logits and writes two 16-byte pieces of dlogits, all streaming.
+__global__ void __launch_bounds__(kDlThreads) lmhead_dlogits_kernel(const DlArgs a) {
+  const int64_t n_tiles = (int64_t)a.rows * a.segs;
+  for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    const int64_t row = tile / a.segs;
+    const int seg = (int)(tile - row * a.segs);
+    const float4 sc = a.rowsc[row];
+    const int yv = a.y[row];
+    const float* zr = a.z + row * a.ld;
+    __nv_bfloat16* dr = a.dl + row * a.ld;
+    float4 v[4];
+    int e0[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      e0[u] = seg * kDlSeg + u * (kDlThreads * 8) + (int)threadIdx.x * 8;
+      if (e0[u] < a.ld) {  // ld is a multiple of 8: the whole vector is inside the row
+        v[2 * u] = __ldcs(reinterpret_cast<const float4*>(zr + e0[u]));
+        v[2 * u + 1] = __ldcs(reinterpret_cast<const float4*>(zr + e0[u]) + 1);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      if (e0[u] >= a.ld) continue;
+      const float zz[8] = {v[2 * u].x,     v[2 * u].y,     v[2 * u].z,     v[2 * u].w,
+                           v[2 * u + 1].x, v[2 * u + 1].y, v[2 * u + 1].z, v[2 * u + 1].w};
+      uint32_t pk[4];
+#pragma unroll
+      for (int k = 0; k < 8; k += 2) {
+        float d0 = sc.x * ex2(fmaf(zz[k], kLog2e, sc.z));
+        float d1 = sc.x * ex2(fmaf(zz[k + 1], kLog2e, sc.z));
+        if (e0[u] + k == yv) d0 = sc.y;
+        if (e0[u] + k + 1 == yv) d1 = sc.y;
+        if (e0[u] + k >= a.V) d0 = 0.f;
+        if (e0[u] + k + 1 >= a.V) d1 = 0.f;
+        pk[k / 2] = pack_bf16x2(make_float2(d0, d1));
+      }
+      __stcs(reinterpret_cast<uint4*>(dr + e0[u]), make_uint4(pk[0], pk[1], pk[2], pk[3]));
+    }
+  }
+}
+
 // Kept rows gathered into a dense block: hidden row src = row_index[t] (16-byte vectors, one CTA
 // per row) and its y, old_logp, ref_logp.
 __global__ void __launch_bounds__(128) lmhead_gather_kernel(
@@ -605,6 +712,8 @@ struct Grid {
 // Atomic: another thread may change them while a call reads them.
 std::atomic<int> g_prefetch{0};
 std::atomic<int> g_row_lanes{0};
+// 1: the token loss recomputes the logits in pass 2 instead of storing them in pass 1.
+std::atomic<int> g_recompute{0};
 
 // R pair lanes x J vocabulary lanes, one CTA per SM at most.  The weight is read from DRAM about
 // once per group of R row-block pairs, so R stays in [4, 8] (all pairs when there are fewer);
@@ -691,12 +800,12 @@ size_t gemm_partial_bytes(int64_t n_rows, int32_t V, int32_t D, int64_t chunk) {
 }
 
 struct WsLayout {
-  size_t part, zy, rowsc, row_loss, stats, seq_loss, dl, gpart, hid, ys, olds, refs, total;
+  size_t part, zy, rowsc, row_loss, stats, seq_loss, z, dl, gpart, hid, ys, olds, refs, total;
 };
 // loss: the backward buffers; n_seqs >= 0: GSPO's statistics and sequence terms instead of the
-// per-row loss terms.
+// per-row loss terms; store_z: a chunk of f32 logits.
 WsLayout ws_layout(int64_t n_rows, int32_t V, int32_t D, int64_t chunk, bool own_dl, bool gather,
-                   bool loss, int64_t n_seqs = -1) {
+                   bool loss, int64_t n_seqs = -1, bool store_z = false) {
   WsLayout w;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -705,12 +814,13 @@ WsLayout ws_layout(int64_t n_rows, int32_t V, int32_t D, int64_t chunk, bool own
     return at;
   };
   const size_t n = (size_t)std::max<int64_t>(n_rows, 1);
-  w.part = take(n * kMaxJ * sizeof(float2));
+  w.part = take(n * (size_t)((V + BN - 1) / BN) * sizeof(float2));
   w.zy = take(n * sizeof(float));
   w.rowsc = take(loss ? n * sizeof(float4) : 0);
   w.row_loss = take(loss && n_seqs < 0 ? n * sizeof(double) : 0);
   w.stats = take(n_seqs >= 0 ? n * sizeof(float4) : 0);
   w.seq_loss = take(n_seqs >= 0 ? (size_t)std::max<int64_t>(n_seqs, 1) * sizeof(double) : 0);
+  w.z = take(loss && store_z ? (size_t)chunk * padded_v(V) * 4 : 0);
   w.dl = take(loss && own_dl ? (size_t)chunk * padded_v(V) * 2 : 0);
   w.gpart = take(loss && n_rows > 0 ? gemm_partial_bytes(n_rows, V, D, chunk) : 0);
   w.hid = take(gather ? n * (size_t)D * 2 : 0);
@@ -728,8 +838,9 @@ using namespace fastrl;
 
 namespace {
 
-// Shared front of both entries: argument checks common to them, the optional gather of the rows,
-// the tensor maps and pass 1 (softmax statistics).  Returns the maps and the row arrays in use.
+// Shared front of the entries: the optional gather of the rows, the tensor maps, the pass-1
+// arguments common to every launch and, with run_pass1, pass 1 (softmax statistics) over every
+// row.  Returns the maps and the row arrays in use.
 struct Front {
   CUtensorMap mh, mw;
   const void* hid;
@@ -738,9 +849,27 @@ struct Front {
   const float* old_logp;
   const float* ref_logp;
   int n_sm;
-  int J;
   TileArgs ta;
 };
+
+// Pass 1 over rows [c0, c0 + rows): per-tile partial sums and z_y of those rows and, with z, their
+// f32 logits (z row t - c0).
+grpo_status launch_pass1(const Front& f, int64_t c0, int64_t rows, float* z, cudaStream_t s,
+                         const char* who) {
+  const Grid g = plan(rows, f.ta.V, f.n_sm);
+  TileArgs ta = f.ta;
+  ta.rows = (int32_t)rows;
+  ta.row0 = (int32_t)c0;
+  ta.n_rb = (int32_t)((rows + BM - 1) / BM);
+  ta.R = g.R;
+  ta.J = g.J;
+  ta.y = f.y + c0;
+  ta.part = f.ta.part + c0 * f.ta.n_vt;
+  ta.zy = f.ta.zy + c0;
+  ta.z = z;
+  ta.ldz = padded_v(f.ta.V);
+  return launch_tiles(false, f.mh, f.mw, ta, g.grid, s, who);
+}
 
 grpo_status check_shape(const char* who, int64_t n_rows, int32_t V, int32_t D,
                         int64_t hidden_stride) {
@@ -758,7 +887,8 @@ grpo_status check_shape(const char* who, int64_t n_rows, int32_t V, int32_t D,
 grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
                   const int64_t* row_index, int64_t n_rows, const void* weight, int32_t V,
                   int32_t D, const int32_t* y, const float* old_logp, const float* ref_logp,
-                  int32_t* status, char* wsb, const WsLayout& L, cudaStream_t s, Front* f) {
+                  int32_t* status, char* wsb, const WsLayout& L, bool run_pass1, cudaStream_t s,
+                  Front* f) {
   grpo_status st;
   f->n_sm = sm_count();
   if (f->n_sm <= 0) return fail(GRPO_ERR_CUDA, "%s: no CUDA device", who);
@@ -786,24 +916,54 @@ grpo_status front(const char* who, const void* hidden, int64_t hidden_stride,
   }
   if (!make_map(&f->mh, f->hid, n_rows, D, f->hstride, BM) || !make_map(&f->mw, weight, V, D, D, BN))
     return fail(GRPO_ERR_CUDA, "%s: cuTensorMapEncodeTiled failed", who);
-  const Grid g1 = plan(n_rows, V, f->n_sm);
-  f->J = g1.J;
   TileArgs& ta = f->ta;
   ta = TileArgs{};
-  ta.rows = (int32_t)n_rows;
-  ta.row0 = 0;
   ta.V = V;
   ta.nK = (D + BK - 1) / BK;
   ta.n_vt = (V + BN - 1) / BN;
-  ta.n_rb = (int32_t)((n_rows + BM - 1) / BM);
-  ta.R = g1.R;
-  ta.J = g1.J;
   ta.prefetch = g_prefetch.load(std::memory_order_relaxed);
   ta.y = f->y;
   ta.part = reinterpret_cast<float2*>(wsb + L.part);
   ta.zy = reinterpret_cast<float*>(wsb + L.zy);
   ta.status = status;
-  return launch_tiles(false, f->mh, f->mw, ta, g1.grid, s, who);
+  return run_pass1 ? launch_pass1(*f, 0, n_rows, nullptr, s, who) : GRPO_OK;
+}
+
+// Eqs. 1-3 per row for rows [c0, c0 + rows) (ra's row arrays point at row 0).
+grpo_status launch_rows(RowArgs ra, int64_t c0, int64_t rows, cudaStream_t s, const char* who) {
+  ra.rows = (int32_t)rows;
+  ra.part += c0 * ra.n_vt;
+  ra.zy += c0;
+  ra.y += c0;
+  if (ra.old_logp) ra.old_logp += c0;
+  if (ra.ref_logp) ra.ref_logp += c0;
+  if (ra.row_rollout) ra.row_rollout += c0;
+  if (ra.logp_out) ra.logp_out += c0;
+  if (ra.row_loss) ra.row_loss += c0;
+  if (ra.rowsc) ra.rowsc += c0;
+  if (ra.stats) ra.stats += c0;
+  lmhead_rows_kernel<<<(unsigned)((rows + kRowWarps - 1) / kRowWarps), kRowWarps * 32, 0, s>>>(ra);
+  count_launches(1);
+  return check_launch(who);
+}
+
+// dhidden[c0 : c0 + rows] = dl * W and dW (+)= dl^T * h[c0 : c0 + rows] for one chunk of dlogits.
+grpo_status chunk_products(const char* who, const Front& f, int64_t c0, int64_t rows, int32_t V,
+                           int32_t D, const void* weight, const __nv_bfloat16* dl, void* dhidden,
+                           int32_t dhidden_dtype, float* dweight, bool acc, float* gpart,
+                           size_t gpart_bytes, cudaStream_t s) {
+  grpo_status st;
+  const int64_t ldd = padded_v(V);
+  const size_t dh_elem = dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+  // dh: A = dl [rows][V] (K-major), B = W [V][D]
+  if ((st = gemm_bf16(who, false, dl, ldd, weight, D, rows, D, V,
+                      static_cast<char*>(dhidden) + c0 * D * dh_elem, D, dhidden_dtype, false,
+                      gpart, gpart_bytes, f.ta.status, s)) != GRPO_OK)
+    return st;
+  // dW: A = dl^T, stored [rows][V] (M-major), B = h [rows][D]
+  return gemm_bf16(who, true, dl, ldd, static_cast<const char*>(f.hid) + c0 * f.hstride * 2,
+                   f.hstride, V, D, rows, dweight, D, GRPO_DTYPE_F32, acc, gpart, gpart_bytes,
+                   f.ta.status, s);
 }
 
 // Pass 2 and the two products, chunk by chunk, from each row's gradient scalars (rowsc).
@@ -814,7 +974,6 @@ grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64
                      size_t gpart_bytes, cudaStream_t s) {
   grpo_status st;
   const int64_t ldd = padded_v(V);
-  const size_t dh_elem = dhidden_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
     const int64_t rows = std::min(chunk, n_rows - c0);
     const Grid g2 = plan(rows, V, f.n_sm);
@@ -832,16 +991,8 @@ grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64
     tb.dl = dl;
     tb.ldd = ldd;
     if ((st = launch_tiles(true, f.mh, f.mw, tb, g2.grid, s, who)) != GRPO_OK) return st;
-    // dh[c0 : c0 + rows] = dlogits * W: A = dl [rows][V] (K-major), B = W [V][D]
-    if ((st = gemm_bf16(who, false, dl, ldd, weight, D, rows, D, V,
-                        static_cast<char*>(dhidden) + c0 * D * dh_elem, D, dhidden_dtype, false,
-                        gpart, gpart_bytes, f.ta.status, s)) != GRPO_OK)
-      return st;
-    // dW (+)= dlogits^T * h: A = dl^T, stored [rows][V] (M-major), B = h [rows][D]
-    const bool acc = !(c0 == 0 && !accumulate_dweight);
-    if ((st = gemm_bf16(who, true, dl, ldd, static_cast<const char*>(f.hid) + c0 * f.hstride * 2,
-                        f.hstride, V, D, rows, dweight, D, GRPO_DTYPE_F32, acc, gpart,
-                        gpart_bytes, f.ta.status, s)) != GRPO_OK)
+    if ((st = chunk_products(who, f, c0, rows, V, D, weight, dl, dhidden, dhidden_dtype, dweight,
+                             !(c0 == 0 && !accumulate_dweight), gpart, gpart_bytes, s)) != GRPO_OK)
       return st;
   }
   return GRPO_OK;
@@ -849,13 +1000,17 @@ grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64
 
 }  // namespace
 
-extern "C" grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes) {
+extern "C" grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes,
+                                        int32_t recompute_logits) {
   clear_error();
-  if (prefetch < 0 || prefetch > 64 || row_lanes < 0 || row_lanes > kRowLanes)
-    return fail(GRPO_ERR_INVALID_ARG, "grpo_lmhead_tune: prefetch in [0, 64], row_lanes in [0, %d]",
+  if (prefetch < 0 || prefetch > 64 || row_lanes < 0 || row_lanes > kRowLanes ||
+      (recompute_logits != 0 && recompute_logits != 1))
+    return fail(GRPO_ERR_INVALID_ARG,
+                "grpo_lmhead_tune: prefetch in [0, 64], row_lanes in [0, %d], recompute_logits 0 or 1",
                 kRowLanes);
   g_prefetch.store(prefetch, std::memory_order_relaxed);
   g_row_lanes.store(row_lanes, std::memory_order_relaxed);
+  g_recompute.store(recompute_logits, std::memory_order_relaxed);
   return GRPO_OK;
 }
 
@@ -884,11 +1039,10 @@ extern "C" grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_s
   char* wsb = static_cast<char*>(ws);
   Front f;
   if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, nullptr, nullptr,
-                  status, wsb, L, s, &f)) != GRPO_OK)
+                  status, wsb, L, true, s, &f)) != GRPO_OK)
     return st;
   RowArgs ra = {};
-  ra.rows = (int32_t)n_rows;
-  ra.J = f.J;
+  ra.n_vt = f.ta.n_vt;
   ra.V = V;
   ra.part = f.ta.part;
   ra.zy = f.ta.zy;
@@ -896,9 +1050,7 @@ extern "C" grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_s
   ra.logp_out = logp_out;
   ra.status = status;
   ra.mode = 1;
-  lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
-  count_launches(1);
-  return check_launch(who);
+  return launch_rows(ra, 0, n_rows, s, who);
 }
 
 extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
@@ -927,9 +1079,10 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
         beta < INFINITY))
     return fail(GRPO_ERR_INVALID_ARG, "%s: need 0 <= eps_low < 1, finite eps_high, beta >= 0", who);
 
+  const bool store_z = g_recompute.load(std::memory_order_relaxed) == 0;
   const int64_t chunk = chunk_of(n_rows, V, chunk_rows);
-  const WsLayout L =
-      ws_layout(n_rows, V, D, chunk, dlogits_out == nullptr, row_index != nullptr, true);
+  const WsLayout L = ws_layout(n_rows, V, D, chunk, dlogits_out == nullptr, row_index != nullptr,
+                               true, -1, store_z);
   bool query_only = false;
   if ((st = workspace_check(ws, ws_bytes, L.total, who, &query_only)) != GRPO_OK || query_only)
     return st;
@@ -957,16 +1110,15 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
     return GRPO_OK;
   }
 
-  // Gather (with row_index) and pass 1: softmax statistics of every row.
+  // Gather (with row_index); with the logits recomputed, pass 1 over every row.
   Front f;
   if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, old_logp,
-                  ref_logp, status, wsb, L, s, &f)) != GRPO_OK)
+                  ref_logp, status, wsb, L, !store_z, s, &f)) != GRPO_OK)
     return st;
 
-  // Row scalars (Eqs. 1-3) and the loss.
+  // Row scalars (Eqs. 1-3).
   RowArgs ra = {};
-  ra.rows = (int32_t)n_rows;
-  ra.J = f.J;
+  ra.n_vt = f.ta.n_vt;
   ra.V = V;
   ra.part = f.ta.part;
   ra.zy = f.ta.zy;
@@ -991,13 +1143,41 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
   ra.row_loss = row_loss;
   ra.rowsc = rowsc;
   ra.status = status;
-  lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
-  count_launches(1);
-  if ((st = check_launch(who)) != GRPO_OK) return st;
-  if ((st = launch_sum_rows(row_loss, n_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
-
-  return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
-                  accumulate_dweight, dlogits_out, dl_buf, chunk, gpart, gpart_bytes, s);
+  if (!store_z) {  // pass 2 recomputes the tiles of each chunk
+    if ((st = launch_rows(ra, 0, n_rows, s, who)) != GRPO_OK) return st;
+    if ((st = launch_sum_rows(row_loss, n_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
+    return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
+                    accumulate_dweight, dlogits_out, dl_buf, chunk, gpart, gpart_bytes, s);
+  }
+  // Chunk by chunk: pass 1 stores the chunk's f32 logits, the row scalars follow, dlogits are
+  // formed from the stored logits by a streaming pass, then the two products.
+  float* zbuf = reinterpret_cast<float*>(wsb + L.z);
+  const int64_t ldd = padded_v(V);
+  const int segs = (int)((ldd + kDlSeg - 1) / kDlSeg);
+  for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
+    const int64_t rows = std::min(chunk, n_rows - c0);
+    if ((st = launch_pass1(f, c0, rows, zbuf, s, who)) != GRPO_OK) return st;
+    if ((st = launch_rows(ra, c0, rows, s, who)) != GRPO_OK) return st;
+    __nv_bfloat16* dl = dlogits_out ? dl_buf + c0 * ldd : dl_buf;
+    DlArgs da = {};
+    da.z = zbuf;
+    da.dl = dl;
+    da.ld = ldd;
+    da.rowsc = rowsc + c0;
+    da.y = f.y + c0;
+    da.rows = (int32_t)rows;
+    da.V = V;
+    da.segs = segs;
+    const int64_t tiles = rows * segs;
+    const unsigned grid = (unsigned)std::min<int64_t>(tiles, (int64_t)f.n_sm * 8);
+    lmhead_dlogits_kernel<<<grid, kDlThreads, 0, s>>>(da);
+    count_launches(1);
+    if ((st = check_launch(who)) != GRPO_OK) return st;
+    if ((st = chunk_products(who, f, c0, rows, V, D, weight, dl, dhidden, dhidden_dtype, dweight,
+                             !(c0 == 0 && !accumulate_dweight), gpart, gpart_bytes, s)) != GRPO_OK)
+      return st;
+  }
+  return launch_sum_rows(row_loss, n_rows, nullptr, loss_out, s, who);
 }
 
 extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
@@ -1056,12 +1236,11 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
   // Gather (with row_index) and pass 1.
   Front f;
   if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, old_logp,
-                  ref_logp, status, wsb, L, s, &f)) != GRPO_OK)
+                  ref_logp, status, wsb, L, true, s, &f)) != GRPO_OK)
     return st;
   // logp and the softmax statistics of every row.
   RowArgs ra = {};
-  ra.rows = (int32_t)n_rows;
-  ra.J = f.J;
+  ra.n_vt = f.ta.n_vt;
   ra.V = V;
   ra.part = f.ta.part;
   ra.zy = f.ta.zy;
@@ -1070,9 +1249,7 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
   ra.status = status;
   ra.mode = 2;
   ra.stats = stats;
-  lmhead_rows_kernel<<<(unsigned)((n_rows + 255) / 256), 256, 0, s>>>(ra);
-  count_launches(1);
-  if ((st = check_launch(who)) != GRPO_OK) return st;
+  if ((st = launch_rows(ra, 0, n_rows, s, who)) != GRPO_OK) return st;
   // Rows outside every sequence keep zero gradient scalars.
   cudaError_t e = cudaMemsetAsync(rowsc, 0, (size_t)n_rows * sizeof(float4), s);
   if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: memset: %s", who, cudaGetErrorString(e));

@@ -257,18 +257,27 @@ def test_lmhead_workspace_query_and_argument_errors(grpo):
     size = ctypes.c_size_t(0)
     assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size)) == 0
     full = size.value
-    # per row: 160 partial (max, sum) pairs, z_y, the row scalars and the row loss; one chunk of
-    # bf16 dlogits (1000 rows round up to 1024); and the f32 partial products of dhidden's split
-    # K: S copies of the chunk's [rows, D] (1 <= S <= 8; 56 output tiles on 152 SMs split)
+    # per row: a partial (max, sum) pair per 256-entry vocabulary tile (594), z_y, the row
+    # scalars and the row loss; one chunk of f32 logits and one of bf16 dlogits (1000 rows round
+    # up to 1024); and the f32 partial products of dhidden's split K: S copies of the chunk's
+    # [rows, D] (1 <= S <= 8; 56 output tiles on 152 SMs split)
     def up(x):
         return (x + 255) // 256 * 256
-    base = up(1000 * 160 * 8) + up(1000 * 4) + up(1000 * 16) + up(1000 * 8)
-    gp = full - base - up(1024 * 152064 * 2)
+    base = up(1000 * 594 * 8) + up(1000 * 4) + up(1000 * 16) + up(1000 * 8)
+    gp = full - base - up(1024 * 152064 * 4) - up(1024 * 152064 * 2)
     unit = 1000 * 3584 * 4
     assert 2 * unit <= gp <= 8 * unit and gp % unit == 0
     assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size), chunk=256) == 0
-    gp = size.value - base - up(256 * 152064 * 2)
+    gp = size.value - base - up(256 * 152064 * 4) - up(256 * 152064 * 2)
     assert 2 * 256 * 3584 * 4 <= gp <= 8 * 256 * 3584 * 4 and gp % (256 * 3584 * 4) == 0
+    # recomputed logits: no chunk of f32 logits
+    L.grpo_lmhead_tune.restype = ctypes.c_int32
+    assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(0), ctypes.c_int32(1)) == 0
+    try:
+        assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size)) == 0
+        assert size.value == full - up(1024 * 152064 * 4)
+    finally:
+        assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(0), ctypes.c_int32(0)) == 0
     assert lmhead_call(L, 1000, 152064, 3584, None, ctypes.byref(size),
                        dl=ctypes.c_void_p(4096)) == 0
     assert size.value == full - up(1024 * 152064 * 2)
@@ -292,10 +301,14 @@ def test_lmhead_workspace_query_and_argument_errors(grpo):
 def test_lmhead_tune_rejects_out_of_range_settings(grpo):
     L = raw()
     L.grpo_lmhead_tune.restype = ctypes.c_int32
-    assert L.grpo_lmhead_tune(ctypes.c_int32(-1), ctypes.c_int32(0)) == 1
-    assert L.grpo_lmhead_tune(ctypes.c_int32(65), ctypes.c_int32(0)) == 1
-    assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(9)) == 1
-    assert L.grpo_lmhead_tune(ctypes.c_int32(0), ctypes.c_int32(0)) == 0
+    i32 = ctypes.c_int32
+    assert L.grpo_lmhead_tune(i32(-1), i32(0), i32(0)) == 1
+    assert L.grpo_lmhead_tune(i32(65), i32(0), i32(0)) == 1
+    assert L.grpo_lmhead_tune(i32(0), i32(9), i32(0)) == 1
+    assert L.grpo_lmhead_tune(i32(0), i32(0), i32(2)) == 1
+    assert L.grpo_lmhead_tune(i32(0), i32(0), i32(-1)) == 1
+    assert L.grpo_lmhead_tune(i32(0), i32(0), i32(1)) == 0
+    assert L.grpo_lmhead_tune(i32(0), i32(0), i32(0)) == 0
 
 
 def test_ars_checkpoint_resumes_the_rollout_counts(oracle_mod, grpo):

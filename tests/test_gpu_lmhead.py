@@ -470,15 +470,45 @@ def test_large_hidden_sizes_sampled_rows(grpo, oracle_mod, T, V, D):
     assert np.all(np.abs(dh - o["dhidden"]) <= rel * o["dhidden_abs"] + 1e-30)
 
 
+def assert_same_bits(a, b):
+    for k in ("logp", "row_loss", "dhidden", "dweight", "dlogits"):
+        if k in a or k in b:
+            np.testing.assert_array_equal(a[k], b[k], err_msg=k)
+    assert a["loss"] == b["loss"]
+
+
 @pytest.mark.parametrize("prefetch,lanes", [(0, 1), (0, 8), (4, 3)])
 def test_parity_under_other_schedules(grpo, oracle_mod, prefetch, lanes):
     """grpo_lmhead_tune changes the grid (pair lanes x vocabulary lanes) and adds L2 prefetches;
-    every setting computes the same function."""
+    every setting computes the same function, to the bit: each row's softmax sums are combined per
+    vocabulary tile in a fixed order, whichever CTA visited the tile."""
     case = LmCase(101 + lanes, 900, 3000, 192)
     o = case.oracle(oracle_mod)
+    ref = case.gpu(grpo)
     try:
         grpo.grpo_lmhead_tune(prefetch, lanes)
         g = case.gpu(grpo)
     finally:
         grpo.grpo_lmhead_tune(0, 0)
     check(case, g, o)
+    assert_same_bits(g, ref)
+
+
+@pytest.mark.parametrize("T,V,D,chunk", [(700, 5000, 192, 256), (333, 257, 64, 0),
+                                         (600, 152064, 64, 256)])
+def test_stored_and_recomputed_logits_give_the_same_bits(grpo, oracle_mod, T, V, D, chunk):
+    """The token loss keeps each chunk's f32 logits from pass 1 and forms dlogits from them; with
+    recompute_logits set it recomputes the tiles in a second tensor-core pass instead.  Both apply
+    the same arithmetic to the same f32 logits: every output is bit-identical, and matches the
+    oracle (ragged chunks, a ragged vocabulary tile, invalid tokens)."""
+    case = LmCase(71 + T, T, V, D, bad_rows=(5, T - 1))
+    stored = case.gpu(grpo, chunk_rows=chunk)
+    try:
+        grpo.grpo_lmhead_tune(0, 0, 1)
+        rec = case.gpu(grpo, chunk_rows=chunk)
+    finally:
+        grpo.grpo_lmhead_tune(0, 0, 0)
+    assert_same_bits(stored, rec)
+    assert stored["status"] == rec["status"] == 1  # GRPO_DEVFLAG_BAD_TOKEN
+    if V * T <= 5000 * 700:
+        check(case, stored, case.oracle(oracle_mod))
