@@ -13,7 +13,8 @@
  *   grpo_gspo_loss_fwd_bwd  GSPO's sequence-level loss                 (Sec. 1, Sec. 4)
  *     (_dev: counts read on the device, for CUDA graphs)
  *   grpo_lmhead_loss_fwd_bwd  the output layer fused with the loss:     (Sec. 3.2, Eqs. 1-3)
- *                           logits on the tensor cores, never stored whole; dhidden, dweight
+ *                           logits on the tensor cores, one chunk of rows at a time; dhidden,
+ *                           dweight
  *     (grpo_lmhead_logp_fwd: log-probabilities alone from hidden states;
  *      grpo_lmhead_gspo_loss_fwd_bwd: the same with GSPO's sequence-level loss;
  *      grpo_lmhead_grad: dhidden and dweight from given dlogits)
@@ -75,6 +76,21 @@ const char* grpo_version(void);
 
 /* Number of kernels this process has launched through the library so far (host counter). */
 uint64_t grpo_kernel_launches(void);
+
+/*
+ * grpo_debug_checks — the report of the checked build's device index checks (no counterpart in
+ * the paper; a stand-in for a memory checker, which this library's GPUs do not offer).  The
+ * checked build (libfastrl_grpo_checked.so, same ABI) tests, inside its kernels, every index it
+ * computes before reading or writing through it: gathered rows, shared-memory slots, the address,
+ * size and alignment of each asynchronous copy, tile coordinates and output extents.  A failing
+ * check skips that access and records its source file and line; nothing traps.
+ * Synchronises the current device, then sets *file_mask to the files whose checks failed since
+ * the last reset (bit i: advantage.cu 0, prune.cu 1, compact.cu 2, loss.cu 3, gspo.cu 4,
+ * reduce.cu 5, lmhead.cu 6, gemm.cu 7) and *first_site to 100000 * file + line of a first
+ * failure (0 if none); reset != 0 clears the record.  The normal build returns
+ * GRPO_ERR_UNSUPPORTED with both outputs 0; grpo_version() names the checked build.
+ */
+grpo_status grpo_debug_checks(int32_t reset, int32_t* file_mask, int32_t* first_site);
 
 /*
  * grpo_check_status — turn a device status word, read back by the caller after synchronising

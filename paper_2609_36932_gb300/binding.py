@@ -30,7 +30,8 @@ STATUS_NAMES = {0: "GRPO_OK", 1: "GRPO_ERR_INVALID_ARG", 2: "GRPO_ERR_UNSUPPORTE
                 6: "GRPO_ERR_DEVICE_CHECK"}
 
 # Every function include/fastrl_grpo.h declares.
-EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_check_status",
+EXPORTS = ["grpo_last_error", "grpo_version", "grpo_kernel_launches", "grpo_debug_checks",
+           "grpo_check_status",
            "grpo_advantage",
            "grpo_prune", "grpo_compact", "grpo_upload_kept", "grpo_loss_fwd_bwd", "grpo_loss_fwd_bwd_dev", "grpo_loss_fwd_bwd_noalloc", "grpo_gspo_loss_fwd_bwd", "grpo_gspo_loss_fwd_bwd_dev",
            "grpo_sum_f64", "grpo_logp_fwd", "grpo_lmhead_loss_fwd_bwd", "grpo_lmhead_dlogits_stride",
@@ -58,18 +59,25 @@ class ArsState(ctypes.Structure):
 _lib = None
 
 
+def checked_build() -> bool:
+    """True when FASTRL_GRPO_CHECKED=1 selects the checked build (device index checks, reported
+    by grpo_debug_checks) for this process."""
+    return os.environ.get("FASTRL_GRPO_CHECKED", "0") == "1"
+
+
 def library_path() -> str:
-    return _build.LIB
+    return _build.LIB_CHECKED if checked_build() else _build.LIB
 
 
 def lib():
-    """Load libfastrl_grpo.so (building it first if it is missing or stale)."""
+    """Load libfastrl_grpo.so, or libfastrl_grpo_checked.so with FASTRL_GRPO_CHECKED=1 (building
+    it first if it is missing or stale)."""
     global _lib
     if _lib is not None:
         return _lib
-    path = _build.build()
+    path = _build.build(checked=checked_build())
     if not os.path.exists(path):
-        raise RuntimeError("libfastrl_grpo.so is missing at %s" % path)
+        raise RuntimeError("%s is missing" % path)
     L = ctypes.CDLL(path)
     L.grpo_last_error.restype = ctypes.c_char_p
     L.grpo_last_error.argtypes = []
@@ -78,6 +86,8 @@ def lib():
     L.grpo_kernel_launches.restype = ctypes.c_uint64
     L.grpo_kernel_launches.argtypes = []
     L.grpo_check_status.argtypes = [_i32]
+    L.grpo_debug_checks.argtypes = [_i32, _c_p, _c_p]
+    L.grpo_debug_checks.restype = _i32
     L.grpo_check_status.restype = _i32
     L.grpo_advantage.argtypes = [_c_p, _i32, _i32, _i32, _c_p, _c_p, _c_p]
     L.grpo_advantage.restype = _i32
@@ -396,6 +406,15 @@ def grpo_loss_fwd_bwd(logits, y, old_logp, ref_logp, adv, row_rollout, *, V: int
     wp, size = _ws_args(wst)
     _check(L.grpo_loss_fwd_bwd(*args_head, wp, size, _stream(stream)))
     return dict(loss=loss_out, dlogits=dlogits, logp=logp_out, row_loss=row_loss_out, ws=wst)
+
+
+def grpo_debug_checks(reset: bool = True):
+    """The checked build's report: (mask of files whose index checks failed, first failing site
+    as 100000 * file + line), after synchronising the device.  GrpoError(GRPO_ERR_UNSUPPORTED)
+    from the normal build."""
+    mask, site = _i32(0), _i32(0)
+    _check(lib().grpo_debug_checks(int(bool(reset)), ctypes.byref(mask), ctypes.byref(site)))
+    return mask.value, site.value
 
 
 def grpo_lmhead_tune(prefetch: int = 0, row_lanes: int = 0, recompute_logits: int = 0):

@@ -3,6 +3,10 @@
 Each .cu file is compiled by nvcc in parallel, then linked with the static CUDA runtime (and no
 other library) into paper_2609_36932_gb300/_build/libfastrl_grpo.so.  Nothing is installed
 outside the tree.
+
+build(checked=True) makes libfastrl_grpo_checked.so from the same sources with GRPO_CHECKED
+defined: the kernels then test every index they compute before using it and report failures
+through grpo_debug_checks (same ABI; objects under _build/checked).  build_all() makes both.
 """
 from __future__ import annotations
 
@@ -18,6 +22,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libfastrl_grpo.so")
+CHECKED_DIR = os.path.join(OUT_DIR, "checked")
+LIB_CHECKED = os.path.join(OUT_DIR, "libfastrl_grpo_checked.so")
 SOURCES = ["api.cu", "advantage.cu", "prune.cu", "compact.cu", "loss.cu", "gspo.cu", "reduce.cu",
            "lmhead.cu", "gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -40,23 +46,28 @@ def _deps():
     return d
 
 
-def stale() -> bool:
-    if not os.path.exists(LIB):
+def stale(checked: bool = False) -> bool:
+    lib = LIB_CHECKED if checked else LIB
+    if not os.path.exists(lib):
         return True
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return any(os.path.getmtime(p) > t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compile the library if missing or stale; return the .so path."""
-    if not force and not stale():
-        return LIB
-    os.makedirs(OUT_DIR, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra_flags=(), checked: bool = False) -> str:
+    """Compile the library (the checked build with checked=True) if missing or stale; return the
+    .so path."""
+    lib = LIB_CHECKED if checked else LIB
+    out_dir = CHECKED_DIR if checked else OUT_DIR
+    if not force and not stale(checked):
+        return lib
+    os.makedirs(out_dir, exist_ok=True)
     cc = nvcc()
+    flags = [*NVCC_FLAGS, *(["-DGRPO_CHECKED=1"] if checked else []), *extra_flags]
 
     def compile_one(src):
-        obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
-        cmd = [cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj]
+        obj = os.path.join(out_dir, src.replace(".cu", ".o"))
+        cmd = [cc, *ARCH, *flags, "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         return src, obj, r
 
@@ -68,14 +79,21 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
             if r.returncode != 0:
                 raise RuntimeError("nvcc failed on %s" % src)
             objs.append(obj)
-    tmp = LIB + ".tmp.%d" % os.getpid()
+    tmp = lib + ".tmp.%d" % os.getpid()
     r = subprocess.run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs],
                        capture_output=True, text=True)
     if r.returncode != 0:
         sys.stderr.write(r.stdout + r.stderr)
         raise RuntimeError("link failed")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
+
+
+def build_all(force: bool = False) -> None:
+    """Both libraries, compiled side by side."""
+    with concurrent.futures.ThreadPoolExecutor(max_workers=2) as ex:
+        for f in [ex.submit(build, force, False, (), c) for c in (False, True)]:
+            f.result()
 
 
 if __name__ == "__main__":

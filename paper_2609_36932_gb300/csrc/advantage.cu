@@ -4,6 +4,7 @@
 // sequence of explicitly rounded additions on values exchanged by shuffles), so the mean, the
 // std and each A are reproducible bit for bit from the order of operations written here; the
 // per-rollout divisions then run in parallel across lanes.
+#define GRPO_TU 0  // this file's bit in the checked build's report (grpo_debug_checks)
 #include "common.cuh"
 #include "trace.cuh"
 
@@ -65,3 +66,7 @@ extern "C" grpo_status grpo_advantage(const float* rewards, int32_t P, int32_t G
   count_launches(1);
   return check_launch("grpo_advantage");
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_advantage)
+}  // namespace fastrl

@@ -1,5 +1,6 @@
 // Host-side parts of libfastrl_grpo: error reporting, the launch counter, the workspace protocol
 // and adaptive rollout sampling (Sec. 3.3, Eqs. 10-14; Algorithm 1 Phases 1a and 1b).
+#define GRPO_TU 8  // this file's bit in the checked build's report (grpo_debug_checks)
 #include <atomic>
 #include <cmath>
 #include <cstdarg>
@@ -66,7 +67,35 @@ using namespace fastrl;
 
 extern "C" const char* grpo_last_error(void) { return g_msg; }
 
+#if defined(GRPO_CHECKED)
+extern "C" const char* grpo_version(void) { return "fastrl_grpo 0.1.0 (sm_103a, checked)"; }
+#else
 extern "C" const char* grpo_version(void) { return "fastrl_grpo 0.1.0 (sm_103a)"; }
+#endif
+
+extern "C" grpo_status grpo_debug_checks(int32_t reset, int32_t* file_mask, int32_t* first_site) {
+  clear_error();
+  if (!file_mask || !first_site)
+    return fail(GRPO_ERR_INVALID_ARG, "grpo_debug_checks: NULL output");
+  *file_mask = 0;
+  *first_site = 0;
+#if defined(GRPO_CHECKED)
+  const cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess)
+    return fail(GRPO_ERR_CUDA, "grpo_debug_checks: cudaDeviceSynchronize: %s", cudaGetErrorString(e));
+  grpo_status (*const readers[])(bool, int32_t*, int32_t*) = {
+      dcheck_read_advantage, dcheck_read_prune, dcheck_read_compact, dcheck_read_loss,
+      dcheck_read_gspo,      dcheck_read_reduce, dcheck_read_lmhead, dcheck_read_gemm};
+  for (auto rd : readers)
+    if (rd(reset != 0, file_mask, first_site) != GRPO_OK)
+      return fail(GRPO_ERR_CUDA, "grpo_debug_checks: reading the device flags failed");
+  return GRPO_OK;
+#else
+  (void)reset;
+  return fail(GRPO_ERR_UNSUPPORTED, "grpo_debug_checks: this library was built without index "
+                                    "checks (build.py's checked build has them)");
+#endif
+}
 
 extern "C" uint64_t grpo_kernel_launches(void) {
   return g_launches.load(std::memory_order_relaxed);

@@ -53,4 +53,65 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   return t;
 }
 
+// Bytes of dynamic shared memory this launch was given.
+__device__ __forceinline__ uint32_t dynamic_smem_bytes() {
+  uint32_t n;
+  asm("mov.u32 %0, %%dynamic_smem_size;" : "=r"(n));
+  return n;
+}
+
+// ---- index checks of the checked build -----------------------------------------------------
+// build.py's checked build (libfastrl_grpo_checked.so) compiles every file with GRPO_CHECKED:
+// GRPO_DCHECK(cond) then evaluates cond where a kernel is about to read or write through an
+// index it computed (a gathered row, a shared-memory slot, a copy's address and size, a tile
+// coordinate); a false cond records this file (GRPO_TU) and the first failing source line in
+// the file's device flags, and the caller skips the access.  grpo_debug_checks reads and clears
+// the flags.  In the normal build GRPO_DCHECK(cond) is `true` and cond is not evaluated.
+#if defined(GRPO_CHECKED)
+#ifndef GRPO_TU
+#error "each file defines GRPO_TU (its index in grpo_debug_checks' mask) before common.cuh"
+#endif
+namespace {
+__device__ int32_t g_dcheck_mask;  // one pair per file (anonymous namespace)
+__device__ int32_t g_dcheck_site;
+__device__ __forceinline__ bool dcheck(bool ok, int line) {
+  if (!ok) {
+    atomicOr(&g_dcheck_mask, 1 << GRPO_TU);
+    atomicCAS(&g_dcheck_site, 0, GRPO_TU * 100000 + line);
+  }
+  return ok;
+}
+}  // namespace
+#define GRPO_DCHECK(cond) ::fastrl::dcheck(static_cast<bool>(cond), __LINE__)
+// Defines `grpo_status name(bool reset, int32_t* mask, int32_t* site)` for this file's flags
+// (on the current device; the caller has synchronised it).
+#define GRPO_DCHECK_READER(name)                                                        \
+  grpo_status name(bool reset, int32_t* mask, int32_t* site) {                          \
+    int32_t m = 0, st = 0;                                                              \
+    if (cudaMemcpyFromSymbol(&m, g_dcheck_mask, sizeof(m)) != cudaSuccess ||            \
+        cudaMemcpyFromSymbol(&st, g_dcheck_site, sizeof(st)) != cudaSuccess)            \
+      return GRPO_ERR_CUDA;                                                             \
+    *mask |= m;                                                                         \
+    if (*site == 0) *site = st;                                                         \
+    if (reset) {                                                                        \
+      const int32_t z = 0;                                                              \
+      if (cudaMemcpyToSymbol(g_dcheck_mask, &z, sizeof(z)) != cudaSuccess ||            \
+          cudaMemcpyToSymbol(g_dcheck_site, &z, sizeof(z)) != cudaSuccess)              \
+        return GRPO_ERR_CUDA;                                                           \
+    }                                                                                   \
+    return GRPO_OK;                                                                     \
+  }
+grpo_status dcheck_read_advantage(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_prune(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_compact(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_loss(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_gspo(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_reduce(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_lmhead(bool, int32_t*, int32_t*);
+grpo_status dcheck_read_gemm(bool, int32_t*, int32_t*);
+#else
+#define GRPO_DCHECK(cond) true
+#define GRPO_DCHECK_READER(name)
+#endif
+
 }  // namespace fastrl

@@ -5,6 +5,7 @@
 //                        tiles of the CTA width -> kept_idx, kept_off, counts {K, T_kept}.
 //   compact_fill_kernel  one CTA per rollout: a kept rollout finds its position k by binary
 //                        search in kept_idx and writes its token indices and rollout id.
+#define GRPO_TU 2  // this file's bit in the checked build's report (grpo_debug_checks)
 #include "common.cuh"
 #include "trace.cuh"
 
@@ -62,8 +63,10 @@ __global__ void __launch_bounds__(kScanThreads)
     __syncthreads();
     if (kept) {
       const int k = carry_k + wk[warp] + ck - 1;
-      kept_idx[k] = r;
-      kept_off[k] = carry_t + wt[warp] + ct - len;
+      if (GRPO_DCHECK(k >= 0 && k <= r)) {  // k kept rollouts precede r
+        kept_idx[k] = r;
+        kept_off[k] = carry_t + wt[warp] + ct - len;
+      }
     }
     __syncthreads();
     if (threadIdx.x == kScanThreads - 1) {  // last thread holds the tile totals
@@ -95,8 +98,11 @@ __global__ void compact_fill_kernel(const uint8_t* __restrict__ keep, const int6
     else
       hi = mid;
   }
+  // the search found r, and its tokens end within the kept total
+  if (!GRPO_DCHECK(lo < (int)counts[0] && kept_idx[lo] == r)) return;
   const int64_t dst = kept_off[lo];
   const int64_t o = off[r], L = off[r + 1] - o;
+  if (!GRPO_DCHECK(dst >= 0 && dst + L <= counts[1])) return;
   for (int64_t s = threadIdx.x; s < L; s += blockDim.x) {
     src_token[dst + s] = o + s;
     token_rollout[dst + s] = r;
@@ -186,3 +192,7 @@ extern "C" grpo_status grpo_upload_kept(const void* src_host, void* dst_dev, int
   }
   return GRPO_OK;
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_compact)
+}  // namespace fastrl

@@ -21,6 +21,7 @@
 //     that each store instruction writes whole 128-byte row pieces.
 // Every wait is bounded (about a second): on expiry the kernel sets GRPO_DEVFLAG_TIMEOUT, the
 // roles stop, in-flight copies and MMAs are drained and the tensor memory is freed.
+#define GRPO_TU 7  // this file's bit in the checked build's report (grpo_debug_checks)
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -81,6 +82,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(tail);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tail + 4);
   const uint32_t out_s = (smem_addr(tail) + 16 + 127u) & ~127u;
+  // the layout (aligned stages, barriers, output staging) within the launch's shared memory
+  if (!GRPO_DCHECK(out_s + 8 * kOutWarpBytes - raw_s <= dynamic_smem_bytes())) return;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -259,6 +262,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                        : "memory");
           const int m = m0 + rr, n = n0 + 4 * p;
           if (m >= g.M || n >= g.N) continue;  // N is a multiple of 4: a piece is all in or out
+          // the piece lies inside C (or partial s inside P), aligned for its vector store
+          if (!GRPO_DCHECK(n + 4 <= g.N && (g.S > 1 ? s < g.S : m < g.M) &&
+                           (g.S > 1 || !g.c_vec ||
+                            ((reinterpret_cast<uintptr_t>(g.C) +
+                              ((uint64_t)m * g.ldc + n) * (g.c_bf16 ? 2 : 4)) &
+                             (g.c_bf16 ? 7u : 15u)) == 0)))
+            continue;
           if (g.S > 1) {
             __stcg(reinterpret_cast<float4*>(g.P + ((int64_t)s * g.M + m) * g.N + n), v);
           } else if (!g.c_bf16) {
@@ -545,3 +555,7 @@ extern "C" grpo_status grpo_lmhead_grad(const void* dlogits, int64_t dlogits_str
     return st;
   return GRPO_OK;
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_gemm)
+}  // namespace fastrl

@@ -11,6 +11,7 @@
 //   3. gspo_dlogits_kernel streams the logits once more and writes
 //      dlogits = coef * ([v == y] - exp(z - M) / S), with pass B's arithmetic from loss.cu.
 // Traffic per kept row: 2 reads and 1 write of V entries (vs 1 + 1 for the token-level loss).
+#define GRPO_TU 4  // this file's bit in the checked build's report (grpo_debug_checks)
 #include <algorithm>
 #include <mutex>
 
@@ -65,7 +66,8 @@ __global__ void __launch_bounds__(kSeqWarps * 32) gspo_seq_kernel(const SeqArgs 
   double slr = 0.0, skl = 0.0;
   int bad = 0;
   for (int64_t t = r0 + lane; t < r1; t += 32) {
-    const int64_t src = a.row_index ? a.row_index[t] : t;
+    int64_t src = a.row_index ? a.row_index[t] : t;
+    if (!GRPO_DCHECK(src >= 0)) src = 0;
     const float lp = a.logp[t];
     if (!isfinite(lp)) bad = 1;
     slr += (double)lp - (double)a.old_logp[src];
@@ -86,7 +88,9 @@ __global__ void __launch_bounds__(kSeqWarps * 32) gspo_seq_kernel(const SeqArgs 
     }
     return;
   }
-  const double A = (double)a.adv[a.seq_rollout[k]];
+  int32_t ro = a.seq_rollout[k];
+  if (!GRPO_DCHECK(ro >= 0)) ro = 0;
+  const double A = (double)a.adv[ro];
   const double s = exp(slr / (double)L);
   const double clipped = fmin(fmax(s, a.lo), a.hi);
   const double surr = fmin(s * A, clipped * A);
@@ -98,7 +102,8 @@ __global__ void __launch_bounds__(kSeqWarps * 32) gspo_seq_kernel(const SeqArgs 
   const float w = (float)(inv_nseq / (double)L);
   const float sa = c ? (float)(s * A) : 0.f;
   for (int64_t t = r0 + lane; t < r1; t += 32) {
-    const int64_t src = a.row_index ? a.row_index[t] : t;
+    int64_t src = a.row_index ? a.row_index[t] : t;
+    if (!GRPO_DCHECK(src >= 0)) src = 0;
     const float x = a.ref_logp[src] - a.logp[t];
     a.coef[t] = w * -(sa + a.beta * expm1f(x));
   }
@@ -142,9 +147,14 @@ __global__ void __launch_bounds__(kDlThreads) gspo_dlogits_kernel(const DlArgs a
     const int seg = (int)(tile - row * a.tiles_per_row);
     const bool last_seg = seg == a.tiles_per_row - 1;
     OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V;
-    const int64_t src = a.row_index ? a.row_index[row] : row;
+    int64_t src = a.row_index ? a.row_index[row] : row;
+    if (!GRPO_DCHECK(src >= 0)) src = 0;
     const InT* grow = reinterpret_cast<const InT*>(a.logits + src * a.row_stride_bytes);
     const float coef = a.coef[row];
+    // vector loads and stores need 16-byte aligned rows (the host sets vec / out_vec from that)
+    if (!GRPO_DCHECK((!a.vec || (reinterpret_cast<uintptr_t>(grow) & 15u) == 0) &&
+                     (!a.out_vec || (reinterpret_cast<uintptr_t>(orow) & 15u) == 0)))
+      continue;
     const int j0 = seg * kSeg;
     if (coef == 0.f) {  // clipped, zero-advantage without KL, or no ratio: a zero row
       float2 d[kPairs];
@@ -420,3 +430,7 @@ extern "C" grpo_status grpo_gspo_loss_fwd_bwd_dev(
                    counts, n_seq, eps_low, eps_high, beta, dlogits, dlogits_dtype, logp_out,
                    seq_ratio_out, loss_out, status, ws, ws_bytes, stream);
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_gspo)
+}  // namespace fastrl

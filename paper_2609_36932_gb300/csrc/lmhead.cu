@@ -48,6 +48,7 @@
 // Every wait is bounded (about a second): a wait that runs out sets GRPO_DEVFLAG_TIMEOUT and an
 // abort flag; the roles then stop, the producer waits for its copies in flight and the MMA lane
 // for its MMAs, and warp 1 frees the tensor memory before the CTA exits.
+#define GRPO_TU 6  // this file's bit in the checked build's report (grpo_debug_checks)
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -144,8 +145,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   unsigned char* tail = smem_raw + (bar_s - raw_s) + 8 * kBars;
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(tail);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tail + 4);
-  // dlogits staging for pass 2: 2 KB per epilogue warp, 128-byte aligned
+  // output staging: kStageWarpBytes per epilogue warp, 128-byte aligned
   const uint32_t stage_out_s = (smem_addr(tail) + 16 + 127u) & ~127u;
+  // the layout (aligned stages, barriers, output staging) within the launch's shared memory
+  if (!GRPO_DCHECK(stage_out_s + kStageOutBytes - raw_s <= dynamic_smem_bytes())) return;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -348,7 +351,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                              : "r"(addr)
                              : "memory");
                 const int grow = rb * BM + q * 32 + rr;
-                if (grow < a.rows)  // streaming: the logits must not push the operands out of L2
+                // streaming: the logits must not push the operands out of L2
+                if (grow < a.rows && GRPO_DCHECK(v0 + 32 <= a.ldz))
                   __stcs(reinterpret_cast<float4*>(a.z + (int64_t)grow * a.ldz + v0) + kc, v);
               }
               __syncwarp();
@@ -415,7 +419,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                            : "r"(addr)
                            : "memory");
               const int grow = rb * BM + q * 32 + rr;
-              if (grow < a.rows)  // streaming: dlogits must not push the operand tiles out of L2
+              // streaming: dlogits must not push the operand tiles out of L2
+              if (grow < a.rows && GRPO_DCHECK(v0 + 32 <= a.ldd))
                 __stcs(reinterpret_cast<uint4*>(a.dl + (int64_t)grow * a.ldd + v0) + kc, v);
             }
             __syncwarp();
@@ -593,7 +598,9 @@ __global__ void __launch_bounds__(kSeqWarps * 32) lmhead_gspo_seq_kernel(const S
     }
     return;
   }
-  const double A = (double)a.adv[a.seq_rollout[k]];
+  int32_t ro = a.seq_rollout[k];
+  if (!GRPO_DCHECK(ro >= 0)) ro = 0;
+  const double A = (double)a.adv[ro];
   const double s = exp(slr / (double)L);
   const double clipped = fmin(fmax(s, a.lo), a.hi);
   const double surr = fmin(s * A, clipped * A);
@@ -635,6 +642,7 @@ constexpr int kDlSeg = kDlThreads * 16;  // two 8-entry vectors per thread and t
 // A persistent grid over (row, 4096-entry segment) tiles; each thread reads two 32-byte pieces of
 // logits and writes two 16-byte pieces of dlogits, all streaming.
 __global__ void __launch_bounds__(kDlThreads) lmhead_dlogits_kernel(const DlArgs a) {
+  if (!GRPO_DCHECK(a.ld % 8 == 0 && (int64_t)a.segs * kDlSeg >= a.ld)) return;
   const int64_t n_tiles = (int64_t)a.rows * a.segs;
   for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
     const int64_t row = tile / a.segs;
@@ -683,6 +691,7 @@ __global__ void __launch_bounds__(128) lmhead_gather_kernel(
     float* __restrict__ old_out, float* __restrict__ ref_out) {
   for (int t = blockIdx.x; t < n_rows; t += gridDim.x) {
     const int64_t src = row_index[t];
+    if (!GRPO_DCHECK(src >= 0)) continue;
     const uint4* in = hidden + src * stride_vec;
     uint4* o = out + (int64_t)t * row_vec;
     for (int k = threadIdx.x; k < row_vec; k += blockDim.x) o[k] = in[k];
@@ -1280,3 +1289,7 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
                   accumulate_dweight, dlogits_out, dl_buf, chunk,
                   reinterpret_cast<float*>(wsb + L.gpart), L.hid - L.gpart, s);
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_lmhead)
+}  // namespace fastrl

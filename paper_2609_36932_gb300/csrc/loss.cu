@@ -31,6 +31,7 @@
 //
 // Log-probabilities alone (logp_stream_kernel, also GSPO's first pass): no gradient pass, so no
 // slice to keep; one CTA streams each row, and every CTA of the persistent grid is resident.
+#define GRPO_TU 3  // this file's bit in the checked build's report (grpo_debug_checks)
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -243,6 +244,16 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
   const uint32_t full_s = smem_addr(full), empty_s = smem_addr(empty);
   const uint32_t xbar_s = smem_addr(xbars), exch_s = smem_addr(exch);
   const float2 l2e2 = make_float2(kLog2e, kLog2e);
+  // The layout (slice, barriers, row slots, exchange entries) within the launch's shared memory;
+  // the same answer in every CTA of the cluster, which then only keeps the cluster barriers.
+  if (!GRPO_DCHECK(reinterpret_cast<const unsigned char*>(exch + 2 * n_ent) - smem <=
+                   (int64_t)dynamic_smem_bytes())) {
+    __syncthreads();
+    cluster_sync();
+    __syncthreads();
+    cluster_sync();
+    return;
+  }
 
   if (tid == 0) {
     for (int k = 0; k < a.n_chunks; ++k) {
@@ -304,11 +315,13 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
       auto fetch = [&](int64_t r) {
         RowIn ri;
         ri.src = a.row_index ? a.row_index[r] : r;
+        if (!GRPO_DCHECK(ri.src >= 0)) ri.src = 0;
         ri.y = a.y[ri.src];
         ri.zy = (ri.y >= 0 && ri.y < a.V)
                     ? Fmt<InT>::load(reinterpret_cast<const InT*>(a.logits + ri.src * a.row_stride_bytes) + ri.y)
                     : 0.f;
-        const int32_t ro = a.row_rollout[r];
+        int32_t ro = a.row_rollout[r];
+        if (!GRPO_DCHECK(ro >= 0)) ro = 0;
         ri.A = a.adv[ro];
         ri.old_lp = a.old_logp[ri.src];
         ri.ref_lp = a.ref_logp[ri.src];
@@ -320,7 +333,11 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
         const char* g = a.logits + src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
         const int v0 = k * a.chunk_vecs;
         const int v1 = min(nvec, v0 + a.chunk_vecs);
-        const uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
+        uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
+        // a bulk copy needs 16-byte aligned addresses and a size in 16-byte units
+        if (bytes && !GRPO_DCHECK(((reinterpret_cast<uintptr_t>(g) + (uintptr_t)v0 * 16) & 15u) == 0 &&
+                                  v1 * 16 <= buf_bytes))
+          bytes = 0;
         mbar_expect_tx(full_s + 8 * k, bytes);  // also publishes rin[] writes made before it
         if (bytes) bulk_copy_g2s(buf_s + v0 * 16, g + (int64_t)v0 * 16, bytes, full_s + 8 * k);
         pend |= 1u << k;
@@ -574,7 +591,8 @@ __global__ void __launch_bounds__(kFwdThreads, kFwdResident / kFwdThreads)
   int64_t n_rows = a.n_rows;
   if (a.counts && a.counts[1] < n_rows) n_rows = a.counts[1];  // device count of kept rows
   for (int64_t row = blockIdx.x; row < n_rows; row += gridDim.x) {
-    const int64_t src = a.row_index ? a.row_index[row] : row;
+    int64_t src = a.row_index ? a.row_index[row] : row;
+    if (!GRPO_DCHECK(src >= 0)) src = 0;
     const int32_t yv = a.y[src];
     const bool yvalid = yv >= 0 && yv < a.V;
     const int yl = yvalid ? yv : -1;
@@ -1131,3 +1149,7 @@ extern "C" grpo_status grpo_loss_fwd_bwd_noalloc(
                            nullptr, loss_out, status, n_rows > 0 ? scratch : nullptr,
                            n_rows > 0 ? &bytes : nullptr, stream);
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_loss)
+}  // namespace fastrl

@@ -18,6 +18,7 @@
 // For n = 1 with at most 64 KiB of bitmaps per prompt, prune_unigram_fused_kernel does steps 0-3
 // in one CTA per prompt, in shared memory.
 // Every decision is an integer or exactly rounded fp64 operation, so the keep mask is bit-exact.
+#define GRPO_TU 1  // this file's bit in the checked build's report (grpo_debug_checks)
 #include <algorithm>
 #include <atomic>
 
@@ -131,6 +132,11 @@ __global__ void __launch_bounds__(kSortThreads)
   int np2 = 1;
   while (np2 < c) np2 <<= 1;
   uint64_t* arr = np2 <= kSmemKeys ? skeys : region;
+  // the keys fit their buffer: the launch's shared memory, or the rollout's 2L workspace keys
+  if (!GRPO_DCHECK(arr == skeys ? (size_t)np2 * 8 <= dynamic_smem_bytes() : np2 <= 2 * L)) {
+    if (threadIdx.x == 0) w.nuniq[r] = 0;
+    return;
+  }
   bool bad = false;
   for (int k = threadIdx.x; k < np2; k += blockDim.x) {
     uint64_t key = kSentinel;
@@ -195,6 +201,10 @@ __global__ void unigram_set_kernel(const int32_t* __restrict__ ids, const int64_
   const int r = blockIdx.x;
   const int64_t o = off[r];
   const int64_t L = off[r + 1] - o;
+  if (!GRPO_DCHECK((size_t)w.words * 8 <= dynamic_smem_bytes() && blockDim.x <= 1024)) {
+    if (threadIdx.x == 0) w.nuniq[r] = 0;
+    return;
+  }
   for (int k = threadIdx.x; k < w.words; k += blockDim.x) bm[k] = 0ull;
   __syncthreads();
   bool bad = false;
@@ -283,6 +293,12 @@ __global__ void sorted_pair_kernel(const int64_t* __restrict__ off, int P, int G
   int na = w.nuniq[ri], nb = w.nuniq[rj];
   const uint64_t* a = w.keys + 2 * off[ri];
   const uint64_t* b = w.keys + 2 * off[rj];
+  // each set lies in its rollout's 2L keys of the workspace
+  if (!GRPO_DCHECK(na >= 0 && nb >= 0 && na <= 2 * (off[ri + 1] - off[ri]) &&
+                   nb <= 2 * (off[rj + 1] - off[rj]))) {
+    if (lane == 0) close[i * G + j] = close[j * G + i] = 0;
+    return;
+  }
   if (na > nb) {
     const uint64_t* t = a;
     a = b;
@@ -401,6 +417,7 @@ __device__ void select_warp(int G, int keep_cap, const int32_t* rnk, const int32
   uint32_t kept = 0;
   for (int a = 0; a < G; ++a) {
     const int i = __ffs(__ballot_sync(FULL, act && rank == a)) - 1;
+    if (!GRPO_DCHECK(i >= 0 && i < G)) continue;  // the ranks are a permutation of 0..G-1
     if ((__shfl_sync(FULL, near, i) & kept) == 0) kept |= 1u << i;
   }
   int count = __popc(kept);
@@ -467,6 +484,7 @@ __global__ void __launch_bounds__(kFusedThreads)
   const int p = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int kWarps = kFusedThreads / 32;
+  if (!GRPO_DCHECK(G <= kMaxG && (size_t)G * words * 8 <= dynamic_smem_bytes())) return;
   if (warp == 0) classify_warp(rewards, adv, class_eps, p, G, lane, s_cls, s_rank);
   if (tid <= G) s_off[tid] = off[(int64_t)p * G + tid];
   for (int k = tid; k < G * words; k += kFusedThreads) bms[k] = 0ull;
@@ -642,3 +660,7 @@ extern "C" grpo_status grpo_prune(const float* rewards, const float* adv, float 
   count_launches(launches);
   return check_launch("grpo_prune");
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_prune)
+}  // namespace fastrl

@@ -8,6 +8,7 @@
 // across the 32 warps give the segment's sum.  After a cluster barrier, CTA 0 reads the segment
 // sums from its peers' shared memory and adds them by a fixed tree; a second barrier keeps the
 // peers resident until it has.  The order depends on n alone, never on scheduling.
+#define GRPO_TU 5  // this file's bit in the checked build's report (grpo_debug_checks)
 #include "common.cuh"
 #include "trace.cuh"
 
@@ -92,3 +93,7 @@ extern "C" grpo_status grpo_sum_f64(const double* v, int64_t n, double* out, grp
     return fail(GRPO_ERR_INVALID_ARG, "grpo_sum_f64: n = %lld, v or out NULL", (long long)n);
   return launch_sum_rows(v, n, nullptr, out, as_stream(stream), "grpo_sum_f64");
 }
+
+namespace fastrl {
+GRPO_DCHECK_READER(dcheck_read_reduce)
+}  // namespace fastrl

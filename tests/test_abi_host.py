@@ -399,3 +399,18 @@ def test_lmhead_grad_workspace_query_and_argument_errors(grpo):
     assert call(10, 100, 64, 104, 64, dtype=7) == 1         # dhidden dtype
     assert b"grpo_lmhead_grad" in L.grpo_last_error()
 
+
+
+def test_normal_build_has_no_index_check_report(grpo):
+    """grpo_debug_checks answers GRPO_ERR_UNSUPPORTED in the normal build, without touching a
+    device, and names the checked build in its message."""
+    if grpo.checked_build():
+        pytest.skip("the checked build reports")
+    L = raw()
+    mask, site = ctypes.c_int32(7), ctypes.c_int32(7)
+    L.grpo_debug_checks.restype = ctypes.c_int32
+    assert L.grpo_debug_checks(ctypes.c_int32(1), ctypes.byref(mask), ctypes.byref(site)) == 2
+    assert mask.value == 0 and site.value == 0
+    assert "checked build" in grpo.grpo_last_error()
+    L.grpo_version.restype = ctypes.c_char_p
+    assert b"checked" not in L.grpo_version()
