@@ -806,8 +806,8 @@ def run_lmhead(args, w):
                "note": "the whole fused call against its algorithmic work: the forward logits "
                        "and the dhidden and dweight products (2 T V D each), all on the "
                        "library's tcgen05 kernels; "
-                       + ("GSPO's entry recomputes the logits in a second pass (2 T V D more "
-                          "executed)" if gspo else
+                       + ("GSPO's entry keeps the first chunk's f32 logits and recomputes the "
+                          "later chunks' in a second pass" if gspo else
                           "the token loss keeps each chunk's f32 logits from pass 1 and forms "
                           "dlogits from them in a streaming pass")}
     products = None if gspo else lmhead_products(d, step, T_kept, w.V, D, peak, peak_src)

@@ -429,13 +429,15 @@ grpo_status grpo_lmhead_logp_fwd(const void* hidden, int64_t hidden_stride,
  * logp_out: device f32 [n_rows], required.  seq_ratio_out: nullable f32 [n_seq_rows] (NaN for a
  *   sequence with an invalid token or no rows).  loss_out: device f64 [1].
  * With no rows or no sequences the loss is 0 and dhidden (and dweight unless accumulated) are 0.
- * Kernels: pass 1 over every row, a row kernel (logp and softmax statistics), one warp per
- *   sequence (ratio, clip, loss term, row gradient scalars), the fixed-order sum, then per chunk
- *   pass 2 (the tiles recomputed on the tensor cores, dlogits written from tensor memory: a
- *   sequence may cross a chunk boundary, so no chunk of logits can be kept until its rows'
- *   scalars are known) and the two GEMMs.
- * Workspace: as grpo_lmhead_loss_fwd_bwd with recomputed logits, with 16 bytes per row and 8 per
- *   sequence in place of the per-row loss terms.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
+ * Kernels: pass 1 over every row (keeping the first chunk's f32 logits), a row kernel (logp and
+ *   softmax statistics), one warp per sequence (ratio, clip, loss term, row gradient scalars),
+ *   the fixed-order sum, then per chunk the dlogits and the two GEMMs.  A sequence may cross a
+ *   chunk boundary, so no row's dlogits exist before pass 1 has covered every row: the first
+ *   chunk's come from its kept logits, each later chunk's from pass 2, which recomputes the
+ *   tiles on the tensor cores (every chunk with grpo_lmhead_tune's recompute_logits).  The same
+ *   bits either way.
+ * Workspace: as grpo_lmhead_loss_fwd_bwd, with 16 bytes per row and 8 per sequence in place of
+ *   the per-row loss terms.  Limits and errors: as grpo_lmhead_loss_fwd_bwd.
  */
 grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
     const void* hidden, int64_t hidden_stride, const int64_t* row_index, int64_t n_rows,
@@ -451,11 +453,11 @@ grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
  * in the paper).  prefetch: k-blocks (64 of D) by which an L2 prefetch of each operand tile runs
  * ahead of its load, 0..64 (0: none).  row_lanes: pairs of 128-row blocks the grid works on at
  * once, 1..8, or 0 to let the library choose per launch.  recompute_logits: 0 (default) lets
- * grpo_lmhead_loss_fwd_bwd store each chunk's f32 logits in pass 1 and form dlogits from them;
- * 1 makes it recompute the logits in a second tensor-core pass instead (a quarter more FLOPs,
- * 4 bytes per chunk entry less workspace).  The results are the same bits either way.  A size
- * query and the call it sizes must see the same setting.  Returns GRPO_ERR_INVALID_ARG for other
- * values.
+ * grpo_lmhead_loss_fwd_bwd store each chunk's f32 logits in pass 1 and form dlogits from them
+ * (grpo_lmhead_gspo_loss_fwd_bwd: the first chunk's); 1 makes both recompute the logits in a
+ * second tensor-core pass instead (a quarter more FLOPs, 4 bytes per chunk entry less
+ * workspace).  The results are the same bits either way.  A size query and the call it sizes
+ * must see the same setting.  Returns GRPO_ERR_INVALID_ARG for other values.
  */
 grpo_status grpo_lmhead_tune(int32_t prefetch, int32_t row_lanes, int32_t recompute_logits);
 

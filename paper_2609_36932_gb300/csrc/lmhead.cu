@@ -19,9 +19,10 @@
 //   Two products per chunk on the same tensor-core machinery (gemm.cu): dh = dlogits * W and
 //     dW (+)= dlogits^T * h.
 // GSPO's loss couples every row of a sequence, and a sequence may cross a chunk boundary, so its
-// entry runs pass 1 over every row first and then, per chunk, pass 2 (lmhead_tile_kernel<true>),
-// which recomputes the tiles and writes dlogits from tensor memory; grpo_lmhead_tune can select
-// that recomputation for the token loss too (less workspace: no chunk of f32 logits).
+// entry runs pass 1 over every row first, keeping the first chunk's f32 logits; that chunk's
+// dlogits come from them, and each later chunk's from pass 2 (lmhead_tile_kernel<true>), which
+// recomputes the tiles and writes dlogits from tensor memory.  grpo_lmhead_tune can select the
+// recomputation for every chunk of both losses (less workspace: no chunk of f32 logits).
 //
 // Kernel roles (320 threads, one CTA per SM: 225 KB of shared memory, all 512 TMEM columns).  A
 // tile is a pair of 128-row blocks of h against 256 vocabulary entries, so each weight stage
@@ -120,8 +121,9 @@ struct TileArgs {
   // pass 1
   float2* part;  // [rows][n_vt]: (max, sum of exp(z - max) without z_y) of vocabulary tile vt
   float* zy;     // [rows]: z_y, written by the CTA whose tile holds y
-  float* z;      // nullable [rows][ldz]: the f32 logits, stored for the dlogits pass
+  float* z;      // nullable [z_rows][ldz]: the f32 logits of rows < z_rows, for the dlogits pass
   int64_t ldz;
+  int32_t z_rows;  // a multiple of 32 (or rows)
   // pass 2
   const float4* rowsc;  // [rows]: {neg_scale, dy, shift, 0} from lmhead_rows_kernel
   __nv_bfloat16* dl;    // [rows][ldd]
@@ -328,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int nvalid = a.V - v0;  // >= 1
           const int jy = yv - v0;       // y's column in this chunk, if in [0, 32)
           if (!kBwd) {
-            if (a.z != nullptr) {
+            if (a.z != nullptr && rb * BM + q * 32 < a.z_rows) {  // warp-uniform
               // The row's 32 logits through shared memory (16-byte pieces XOR-swizzled by row,
               // conflict-free), then each store instruction covers 4 rows x 128 contiguous bytes.
 #pragma unroll
@@ -352,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                              : "memory");
                 const int grow = rb * BM + q * 32 + rr;
                 // streaming: the logits must not push the operands out of L2
-                if (grow < a.rows && GRPO_DCHECK(v0 + 32 <= a.ldz))
+                if (grow < a.rows && grow < a.z_rows && GRPO_DCHECK(v0 + 32 <= a.ldz))
                   __stcs(reinterpret_cast<float4*>(a.z + (int64_t)grow * a.ldz + v0) + kc, v);
               }
               __syncwarp();
@@ -861,10 +863,10 @@ struct Front {
   TileArgs ta;
 };
 
-// Pass 1 over rows [c0, c0 + rows): per-tile partial sums and z_y of those rows and, with z, their
-// f32 logits (z row t - c0).
+// Pass 1 over rows [c0, c0 + rows): per-tile partial sums and z_y of those rows and, with z, the
+// f32 logits of the first z_rows of them (z row t - c0; z_rows < 0: all).
 grpo_status launch_pass1(const Front& f, int64_t c0, int64_t rows, float* z, cudaStream_t s,
-                         const char* who) {
+                         const char* who, int64_t z_rows = -1) {
   const Grid g = plan(rows, f.ta.V, f.n_sm);
   TileArgs ta = f.ta;
   ta.rows = (int32_t)rows;
@@ -877,6 +879,7 @@ grpo_status launch_pass1(const Front& f, int64_t c0, int64_t rows, float* z, cud
   ta.zy = f.ta.zy + c0;
   ta.z = z;
   ta.ldz = padded_v(f.ta.V);
+  ta.z_rows = (int32_t)(z_rows < 0 ? rows : std::min(z_rows, rows));
   return launch_tiles(false, f.mh, f.mw, ta, g.grid, s, who);
 }
 
@@ -956,6 +959,26 @@ grpo_status launch_rows(RowArgs ra, int64_t c0, int64_t rows, cudaStream_t s, co
   return check_launch(who);
 }
 
+// dlogits of `rows` rows from their stored f32 logits z (row stride padded_v(V)) and scalars.
+grpo_status launch_dlogits(const float* z, __nv_bfloat16* dl, const float4* rowsc,
+                           const int32_t* y, int64_t rows, int32_t V, int n_sm, cudaStream_t s,
+                           const char* who) {
+  DlArgs da = {};
+  da.z = z;
+  da.dl = dl;
+  da.ld = padded_v(V);
+  da.rowsc = rowsc;
+  da.y = y;
+  da.rows = (int32_t)rows;
+  da.V = V;
+  da.segs = (int)((da.ld + kDlSeg - 1) / kDlSeg);
+  const int64_t tiles = rows * da.segs;
+  const unsigned grid = (unsigned)std::min<int64_t>(tiles, (int64_t)n_sm * 8);
+  lmhead_dlogits_kernel<<<grid, kDlThreads, 0, s>>>(da);
+  count_launches(1);
+  return check_launch(who);
+}
+
 // dhidden[c0 : c0 + rows] = dl * W and dW (+)= dl^T * h[c0 : c0 + rows] for one chunk of dlogits.
 grpo_status chunk_products(const char* who, const Front& f, int64_t c0, int64_t rows, int32_t V,
                            int32_t D, const void* weight, const __nv_bfloat16* dl, void* dhidden,
@@ -975,18 +998,26 @@ grpo_status chunk_products(const char* who, const Front& f, int64_t c0, int64_t 
                    f.ta.status, s);
 }
 
-// Pass 2 and the two products, chunk by chunk, from each row's gradient scalars (rowsc).
+// The dlogits of each chunk (pass 2, or with z0 the first chunk from its logits stored by pass
+// 1) and the two products, chunk by chunk, from each row's gradient scalars (rowsc).
 grpo_status backward(const char* who, const Front& f, const float4* rowsc, int64_t n_rows,
                      int32_t V, int32_t D, const void* weight, void* dhidden,
                      int32_t dhidden_dtype, float* dweight, int32_t accumulate_dweight,
                      void* dlogits_out, __nv_bfloat16* dl_buf, int64_t chunk, float* gpart,
-                     size_t gpart_bytes, cudaStream_t s) {
+                     size_t gpart_bytes, cudaStream_t s, const float* z0 = nullptr) {
   grpo_status st;
   const int64_t ldd = padded_v(V);
   for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
     const int64_t rows = std::min(chunk, n_rows - c0);
-    const Grid g2 = plan(rows, V, f.n_sm);
     __nv_bfloat16* dl = dlogits_out ? dl_buf + c0 * ldd : dl_buf;
+    if (c0 == 0 && z0 != nullptr) {
+      if ((st = launch_dlogits(z0, dl, rowsc, f.y, rows, V, f.n_sm, s, who)) != GRPO_OK) return st;
+      if ((st = chunk_products(who, f, c0, rows, V, D, weight, dl, dhidden, dhidden_dtype,
+                               dweight, accumulate_dweight != 0, gpart, gpart_bytes, s)) != GRPO_OK)
+        return st;
+      continue;
+    }
+    const Grid g2 = plan(rows, V, f.n_sm);
     TileArgs tb = f.ta;
     tb.rows = (int32_t)rows;
     tb.row0 = (int32_t)c0;
@@ -1162,26 +1193,13 @@ extern "C" grpo_status grpo_lmhead_loss_fwd_bwd(
   // formed from the stored logits by a streaming pass, then the two products.
   float* zbuf = reinterpret_cast<float*>(wsb + L.z);
   const int64_t ldd = padded_v(V);
-  const int segs = (int)((ldd + kDlSeg - 1) / kDlSeg);
   for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
     const int64_t rows = std::min(chunk, n_rows - c0);
     if ((st = launch_pass1(f, c0, rows, zbuf, s, who)) != GRPO_OK) return st;
     if ((st = launch_rows(ra, c0, rows, s, who)) != GRPO_OK) return st;
     __nv_bfloat16* dl = dlogits_out ? dl_buf + c0 * ldd : dl_buf;
-    DlArgs da = {};
-    da.z = zbuf;
-    da.dl = dl;
-    da.ld = ldd;
-    da.rowsc = rowsc + c0;
-    da.y = f.y + c0;
-    da.rows = (int32_t)rows;
-    da.V = V;
-    da.segs = segs;
-    const int64_t tiles = rows * segs;
-    const unsigned grid = (unsigned)std::min<int64_t>(tiles, (int64_t)f.n_sm * 8);
-    lmhead_dlogits_kernel<<<grid, kDlThreads, 0, s>>>(da);
-    count_launches(1);
-    if ((st = check_launch(who)) != GRPO_OK) return st;
+    if ((st = launch_dlogits(zbuf, dl, rowsc + c0, f.y + c0, rows, V, f.n_sm, s, who)) != GRPO_OK)
+      return st;
     if ((st = chunk_products(who, f, c0, rows, V, D, weight, dl, dhidden, dhidden_dtype, dweight,
                              !(c0 == 0 && !accumulate_dweight), gpart, gpart_bytes, s)) != GRPO_OK)
       return st;
@@ -1210,9 +1228,10 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
   if (!(eps_low >= 0.f && eps_low < 1.f && eps_high >= 0.f && beta >= 0.f && eps_high < INFINITY &&
         beta < INFINITY))
     return fail(GRPO_ERR_INVALID_ARG, "%s: need 0 <= eps_low < 1, finite eps_high, beta >= 0", who);
+  const bool store_z = g_recompute.load(std::memory_order_relaxed) == 0;
   const int64_t chunk = chunk_of(n_rows, V, chunk_rows);
   const WsLayout L = ws_layout(n_rows, V, D, chunk, dlogits_out == nullptr, row_index != nullptr,
-                               true, n_seq_rows);
+                               true, n_seq_rows, store_z);
   bool query_only = false;
   if ((st = workspace_check(ws, ws_bytes, L.total, who, &query_only)) != GRPO_OK || query_only)
     return st;
@@ -1242,11 +1261,13 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
   __nv_bfloat16* dl_buf = dlogits_out ? static_cast<__nv_bfloat16*>(dlogits_out)
                                       : reinterpret_cast<__nv_bfloat16*>(wsb + L.dl);
 
-  // Gather (with row_index) and pass 1.
+  // Gather (with row_index) and pass 1 over every row, keeping the first chunk's f32 logits.
   Front f;
   if ((st = front(who, hidden, hidden_stride, row_index, n_rows, weight, V, D, y, old_logp,
-                  ref_logp, status, wsb, L, true, s, &f)) != GRPO_OK)
+                  ref_logp, status, wsb, L, false, s, &f)) != GRPO_OK)
     return st;
+  float* zbuf = store_z ? reinterpret_cast<float*>(wsb + L.z) : nullptr;
+  if ((st = launch_pass1(f, 0, n_rows, zbuf, s, who, chunk)) != GRPO_OK) return st;
   // logp and the softmax statistics of every row.
   RowArgs ra = {};
   ra.n_vt = f.ta.n_vt;
@@ -1285,9 +1306,10 @@ extern "C" grpo_status grpo_lmhead_gspo_loss_fwd_bwd(
   count_launches(1);
   if ((st = check_launch(who)) != GRPO_OK) return st;
   if ((st = launch_sum_rows(seq_loss, n_seq_rows, nullptr, loss_out, s, who)) != GRPO_OK) return st;
+  // the first chunk's dlogits from its kept logits, the others recomputed in pass 2
   return backward(who, f, rowsc, n_rows, V, D, weight, dhidden, dhidden_dtype, dweight,
                   accumulate_dweight, dlogits_out, dl_buf, chunk,
-                  reinterpret_cast<float*>(wsb + L.gpart), L.hid - L.gpart, s);
+                  reinterpret_cast<float*>(wsb + L.gpart), L.hid - L.gpart, s, zbuf);
 }
 
 namespace fastrl {

@@ -372,6 +372,25 @@ def test_gspo_invalid_token_sequence_and_chunks(grpo, oracle_mod):
     np.testing.assert_array_equal(g["dhidden"][50:120], 0.0)
 
 
+@pytest.mark.parametrize("chunk", [128, 0])
+def test_gspo_kept_first_chunk_and_recomputed_logits_give_the_same_bits(grpo, oracle_mod, chunk):
+    """GSPO's entry keeps the first chunk's f32 logits from pass 1 and recomputes the later
+    chunks' in pass 2; with recompute_logits set every chunk is recomputed.  Sequences cross the
+    128-row chunk boundaries (and with the default chunk all rows are one chunk): every output is
+    bit-identical, and matches the oracle."""
+    case = GspoCase(91, (50, 70, 90, 35), 700, 64, bad_rows=(60,))
+    kept = case.gpu(grpo, chunk_rows=chunk)
+    try:
+        grpo.grpo_lmhead_tune(0, 0, 1)
+        rec = case.gpu(grpo, chunk_rows=chunk)
+    finally:
+        grpo.grpo_lmhead_tune(0, 0, 0)
+    for k in ("logp", "dhidden", "dweight", "dlogits", "seq_ratio"):
+        np.testing.assert_array_equal(kept[k], rec[k], err_msg=k)
+    assert kept["loss"] == rec["loss"] and kept["status"] == rec["status"]
+    check_gspo(case, kept, case.oracle(oracle_mod))
+
+
 def test_step_with_the_output_layer_and_gspo(grpo, oracle_mod):
     """GrpoStep in output-layer mode with GSPO's ratio on the small workload's batch: selection,
     then grpo_lmhead_gspo_loss_fwd_bwd over the kept rollouts as sequences, against the oracle."""
