@@ -6,8 +6,9 @@
 //   z[t, v] = sum_d h[t, d] * W[v, d]
 //   loss, logp: Eqs. 1-3 on z, as grpo_loss_fwd_bwd computes them
 //   dh = dlogits * W,   dW = dlogits^T * h        (the chain rule through z = h W^T)
-// The [rows, V] logits are never stored whole.  They are produced 128 x 256 at a time into
-// tensor memory by tcgen05.mma (bf16 operands staged in shared memory by TMA, f32 accumulators).
+// The [rows, V] logits never exist for all rows at once.  They are produced 128 x 256 at a time
+// into tensor memory by tcgen05.mma (bf16 operands staged in shared memory by TMA, f32
+// accumulators).
 // The token loss runs chunk by chunk (rows of logits held at a time):
 //   Pass 1 (lmhead_tile_kernel<false>): per row and vocabulary tile, the maximum and the sum of
 //     exp(z - max) (z_y excluded from the sum and kept separately); the chunk's f32 logits are
