@@ -5,7 +5,7 @@
 //   * A row of V logits is split over a cluster of C CTAs; CTA c holds the slice
 //     [c*slice, (c+1)*slice) of the row in shared memory for the whole row, so the logits are
 //     read from HBM exactly once.  (V = 152064 bf16 is 297 KiB, more than one SM holds; by
-//     default C = 4 with bf16 dlogits, 74 KiB slices and 2 CTAs per SM, and C = 8 with f32.)
+//     default C = 4 with bf16 dlogits, 74 KiB slices and 3 CTAs per SM, and C = 8 with f32.)
 //   * Each slice arrives by non-tensor bulk copies (cp.async.bulk, 16-byte granules) in a few
 //     chunks, each completing on its own mbarrier, so the CTA starts reducing chunk 0 while
 //     the rest is in flight.
