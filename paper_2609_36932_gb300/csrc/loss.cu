@@ -740,6 +740,23 @@ struct Shape {
 };
 
 // out_bytes: bytes per dlogits element (2 or 4).
+//
+// Default shape, from sweeps on GB300 of every cluster size 1-16, 128/256/512 consumer threads
+// and 1-3 copies per slice at V = 32000 ... 256000 (11 vocabularies), bf16 logits, bf16 and f32
+// dlogits, about 12 GB per call:
+//  - dlogits no wider than the logits: the cluster size C <= 10 that keeps the most slice bytes
+//    resident per SM (CTAs per SM by shared memory, at most the CTAs the instance is compiled
+//    for, times the slice's bytes), slices of at most 100 KiB; among sizes within 2% of the
+//    most, the smallest.  256 consumer threads for slices of 56 KiB or more, else 128.  The
+//    shape it picks was within 1% of the best measured one at every vocabulary but V = 32000
+//    (2%, run-to-run noise on the same shape); the previous rule (80 KiB slices) left 9-16% at
+//    V = 128256 and 201088;
+//  - f32 dlogits from bf16 logits (the write phase twice the read): slices of about 24 KiB
+//    (C = ceil(row / 24 KiB), at most 8), more CTAs per row while a slice exceeds 52 KiB (up to
+//    10), 128 threads: within 1.6% of the best at every vocabulary, up to 18% above the
+//    previous rule (40 KiB slices);
+//  - two copies per slice, but one for slices of at most 32 KiB with narrow dlogits.
+// Rows too long for those limits take up to 16 CTAs and slices up to the shared-memory limit.
 grpo_status pick_shape(int V, int in_bytes, int out_bytes, const char* who, Shape* out) {
   Tune tune;
   {
@@ -747,30 +764,56 @@ grpo_status pick_shape(int V, int in_bytes, int out_bytes, const char* who, Shap
     tune = g_tune;
   }
   const int vec = 16 / in_bytes;
-  // Default shape, from sweeps on GB300 over cluster sizes 1-16, 128-512 threads and 1-8 copies
-  // per slice for V = 32000 and 152064, bf16 logits:
-  //  - slices of at most 80 KiB, or 40 KiB when dlogits are wider than the logits (the wider
-  //    write phase then gains from more CTAs per SM); at least two CTAs per row once a row
-  //    exceeds 32 KiB;
-  //  - 256 threads when a slice has at least 128 elements per thread, else 128;
-  //  - two bulk copies per slice (about 45% of the slice limit each).
-  const int64_t limit = (out_bytes > in_bytes ? 40 : 80) * 1024;
+  const bool wide_out = out_bytes > in_bytes;
+  auto slice_of = [&](int C) { return (int)align_up((size_t)((V + C - 1) / C), vec); };
+  auto empty_slice = [&](int C) { return C > 1 && (int64_t)(C - 1) * slice_of(C) >= V; };
+  auto threads_for = [&](int slice) {
+    return (!wide_out && (size_t)slice * in_bytes >= 56 * 1024) ? 256 : 128;
+  };
   int C = tune.cluster;
-  if (C == 0) {
+  if (C == 0 && wide_out) {
     const int64_t row_bytes = (int64_t)V * in_bytes;
-    C = (int)std::min<int64_t>(kMaxCluster, (row_bytes + limit - 1) / limit);
-    if (C == 1 && row_bytes > 32 * 1024) C = 2;
+    C = (int)std::min<int64_t>(8, std::max<int64_t>(1, (row_bytes + 24 * 1024 - 1) / (24 * 1024)));
+    while (C < kMaxCluster) {
+      const size_t sb = (size_t)slice_of(C) * in_bytes;
+      if (sb > 100 * 1024 || (C < 10 && sb > 52 * 1024))
+        ++C;
+      else
+        break;
+    }
+  } else if (C == 0) {
+    const size_t per_sm = 228 * 1024, reserved = 1024;
+    for (int pass = 0; pass < 2 && C == 0; ++pass) {
+      const int cmax = pass == 0 ? 10 : kMaxCluster;
+      const size_t smax = pass == 0 ? 100 * 1024 : 227 * 1024;
+      size_t score[kMaxCluster + 1] = {};
+      size_t top = 0;
+      for (int c = 1; c <= cmax; ++c) {
+        const int sl = slice_of(c);
+        const size_t sb = (size_t)sl * in_bytes;
+        if (empty_slice(c) || sb > smax) continue;
+        const int th = threads_for(sl);
+        const size_t smem = align_up(sb, 128) + loss_smem_fixed(2) + 2 * (size_t)c * (th / 32) * sizeof(float2);
+        const size_t ctas = std::min<size_t>(per_sm / (smem + reserved), (size_t)uncapped_ctas(th));
+        score[c] = ctas * sb;
+        top = std::max(top, score[c]);
+      }
+      for (int c = 1; c <= cmax && top > 0; ++c)
+        if (score[c] > 0 && (double)score[c] >= 0.98 * (double)top) {
+          C = c;
+          break;
+        }
+    }
+    if (C == 0) C = kMaxCluster;  // the shared-memory check below reports what does not fit
   }
-  int slice = (int)align_up((size_t)((V + C - 1) / C), vec);
-  while (C > 1 && (int64_t)(C - 1) * slice >= V) {  // no empty slices
+  int slice = slice_of(C);
+  while (C > 1 && empty_slice(C)) {  // no empty slices
     --C;
-    slice = (int)align_up((size_t)((V + C - 1) / C), vec);
+    slice = slice_of(C);
   }
-  const int threads = tune.threads ? tune.threads : (slice >= 128 * 256 ? 256 : 128);
+  const int threads = tune.threads ? tune.threads : threads_for(slice);
   const size_t slice_bytes = (size_t)slice * in_bytes;
-  const size_t copy = (size_t)limit * 9 / 20;
-  int chunks = tune.chunks ? tune.chunks
-                           : (int)std::min<size_t>(kMaxChunks, std::max<size_t>(1, (slice_bytes + copy / 2) / copy));
+  int chunks = tune.chunks ? tune.chunks : ((!wide_out && slice_bytes <= 32 * 1024) ? 1 : 2);
   const int slice_vecs = slice / vec;
   int chunk_vecs = (slice_vecs + chunks - 1) / chunks;
   if (chunk_vecs < 1) chunk_vecs = 1;
