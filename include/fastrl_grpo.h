@@ -345,7 +345,8 @@ grpo_status grpo_gspo_loss_fwd_bwd_dev(const void* logits, int32_t logits_dtype,
  *   when given it receives every row's dlogits (columns >= V are 0) and no chunk buffer is used.
  * logp_out (f32 [n_rows]) and row_loss_out (f64 [n_rows]): nullable.  loss_out: device f64 [1].
  * chunk_rows: rows of logits and dlogits held at a time (rounded up to a multiple of 128); 0
- *   picks the largest count whose bf16 dlogits fit 4 GiB (their f32 logits then take 8 GiB).
+ *   splits the rows into as few equal chunks as keep each chunk's bf16 dlogits within about
+ *   4 GiB (their f32 logits then take about 8 GiB).
  *   Smaller chunks need less workspace.
  * Workspace: per row 8 bytes per 256 vocabulary entries of softmax statistics; per chunk row
  *   4 * grpo_lmhead_dlogits_stride(V) bytes of f32 logits (none when grpo_lmhead_tune selects
