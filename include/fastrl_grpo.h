@@ -235,6 +235,11 @@ grpo_status grpo_upload_kept(const void* src_host, void* dst_dev, int64_t row_by
  *                 [0, V) gets logp = NaN, a zero dlogits row and a zero loss term.
  * Workspace: n_rows f64 when row_loss_out is NULL, else none.
  * Limits: V >= 1, V*element size <= 16 * 200 KiB; n_rows < 2^31.
+ * Speed: logits rows whose byte offset is a multiple of 16 arrive by bulk copies, and dlogits rows
+ *   with V * element size a multiple of 16 leave by 16-byte stores.  Other rows (an odd V stored
+ *   densely, such as 50257) take an element-wise path at about a tenth of the rate; padding the
+ *   vocabulary to a multiple of 8 with -inf logits gives the same results on the true columns
+ *   (exp(-inf) = 0 in every sum) and zero dlogits (+0 or -0) on the padding.
  */
 grpo_status grpo_loss_fwd_bwd(const void* logits, int32_t logits_dtype, int64_t row_stride,
                               const int64_t* row_index, int64_t n_rows, int32_t V,
