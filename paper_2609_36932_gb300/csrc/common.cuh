@@ -37,7 +37,8 @@ grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype,
                       cudaStream_t s);
 
 // reduce.cu: *out = v[0] + ... + v[m-1] in fp64 in a fixed order, m = n or, with n_dev (a device
-// count, nullable), min(n, *n_dev); one launch of an 8-CTA cluster on `s`.
+// count, nullable), min(n, *n_dev); one launch of an 8-CTA cluster on `s`, as a programmatic
+// dependent of the kernel before it (its reads wait for that kernel to complete).
 grpo_status launch_sum_rows(const double* v, int64_t n, const int64_t* n_dev, double* out,
                             cudaStream_t s, const char* who);
 
@@ -58,6 +59,19 @@ __device__ __forceinline__ uint32_t dynamic_smem_bytes() {
   uint32_t n;
   asm("mov.u32 %0, %%dynamic_smem_size;" : "=r"(n));
   return n;
+}
+
+// Programmatic dependent launch (PTX griddepcontrol).  When every CTA of a kernel has called
+// allow_dependent_launch() (or exited), the next kernel of the stream, if it was launched with
+// cudaLaunchAttributeProgrammaticStreamSerialization, may be scheduled before the first one ends;
+// that kernel calls wait_for_prerequisite_grids() before its first global access, which returns
+// once the earlier grid has completed and its writes are visible.  A kernel launched without the
+// attribute returns from the wait at once.
+__device__ __forceinline__ void allow_dependent_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void wait_for_prerequisite_grids() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 // ---- index checks of the checked build -----------------------------------------------------

@@ -231,6 +231,9 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
   RowIn* rin = reinterpret_cast<RowIn*>(reinterpret_cast<unsigned char*>(abort_flag) + 16);
   float2* exch = reinterpret_cast<float2*>(rin + 2);                // [2][C * kWarps]
 
+  // The fixed-order sum that follows (a programmatic dependent) may be scheduled now: it waits
+  // for this grid to complete before it reads anything.
+  allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t rank = cluster_ctarank();
   const uint32_t C = cluster_nctarank();

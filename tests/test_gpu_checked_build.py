@@ -25,7 +25,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 FILES = ["tests/test_gpu_select.py", "tests/test_gpu_loss.py", "tests/test_gpu_logp.py",
          "tests/test_gpu_gspo.py", "tests/test_gpu_fuzz.py", "tests/test_gpu_pipeline.py",
          "tests/test_gpu_lmhead.py", "tests/test_gpu_lmhead_grad.py",
-         "tests/test_gpu_checked_build.py"]
+         "tests/test_gpu_sum.py", "tests/test_gpu_checked_build.py"]
 LOSS_FILE_BIT = 3  # loss.cu in grpo_debug_checks' file mask
 
 
