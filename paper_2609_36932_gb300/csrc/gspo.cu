@@ -130,7 +130,11 @@ constexpr int kDlUnroll = 4;  // 16-byte vectors per thread per tile
 
 // Persistent grid over tiles (row, segment of kDlThreads * kDlUnroll vectors).  Each thread
 // issues its kDlUnroll loads before using any of them.
-template <typename InT, typename OutT>
+// kAny: the instance for rows that need not start on a 16-byte boundary (chosen by the host
+// only then).  A segment is kDlThreads * kDlUnroll aligned 16-byte words of the dlogits row;
+// each word's inputs come from the aligned words of the logits row that hold them
+// (pairs_at_global), and the first and last few elements of the row are stored one by one.
+template <typename InT, typename OutT, bool kAny>
 __global__ void __launch_bounds__(kDlThreads) gspo_dlogits_kernel(const DlArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
   constexpr int kPairs = Fmt<InT>::kPairs;
@@ -156,6 +160,66 @@ __global__ void __launch_bounds__(kDlThreads) gspo_dlogits_kernel(const DlArgs a
                      (!a.out_vec || (reinterpret_cast<uintptr_t>(orow) & 15u) == 0)))
       continue;
     const int j0 = seg * kSeg;
+    if constexpr (kAny) {
+      using OW = OutWord<InT, OutT>;
+      constexpr int E = OW::kElems;
+      const int omis = (int)(reinterpret_cast<uintptr_t>(orow) & 15u);
+      const int h = min(a.V, ((16 - omis) & 15) / (int)sizeof(OutT));  // elements before word 0
+      const int nfull = (a.V - h) / E;
+      const int rest0 = h + nfull * E;
+      float neg_scale = 0.f, dy = 0.f, shB = 0.f;
+      int32_t yv = -1;
+      if (coef != 0.f) {
+        const float4 st = a.stats[row];  // {M, S, S without y}
+        yv = a.y[src];
+        neg_scale = -coef / st.y;
+        dy = coef * (st.z / st.y);
+        shB = -st.x * kLog2e;
+        if (fabsf(neg_scale) >= 0x1p-100f) {
+          shB += kShiftB;
+          neg_scale *= 0x1p-16f;
+        }
+      }
+      const float2 shb2 = make_float2(shB, shB), ns2 = make_float2(neg_scale, neg_scale);
+      float2 p[kDlUnroll][OW::kPairs];
+#pragma unroll
+      for (int u = 0; u < kDlUnroll; ++u) {
+        const int w = j0 + u * kDlThreads + tid;
+        if (coef != 0.f && w < nfull) pairs_at_global<InT, OutT>(grow, a.V, h + w * E, p[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kDlUnroll; ++u) {
+        const int w = j0 + u * kDlThreads + tid;
+        if (w >= nfull) continue;
+        const int i0 = h + w * E;
+        float2 d[OW::kPairs];
+#pragma unroll
+        for (int i = 0; i < OW::kPairs; ++i)
+          d[i] = coef != 0.f ? __fmul2_rn(ex2x2(__ffma2_rn(p[u][i], l2e2, shb2)), ns2)
+                             : make_float2(0.f, 0.f);
+        const int yi = yv - i0;
+        if (coef != 0.f && (unsigned)yi < (unsigned)E) {
+#pragma unroll
+          for (int i = 0; i < OW::kPairs; ++i) {
+            if (2 * i == yi) d[i].x = dy;
+            if (2 * i + 1 == yi) d[i].y = dy;
+          }
+        }
+        store_pairs<OutT, OW::kPairs>(orow + i0, d);
+      }
+      if (last_seg) {
+        for (int t = tid; t < h + (a.V - rest0); t += kDlThreads) {
+          const int e = t < h ? t : rest0 + (t - h);  // the head, then the tail
+          float d = 0.f;
+          if (coef != 0.f) {
+            d = neg_scale * ex2(fmaf(Fmt<InT>::load(grow + e), kLog2e, shB));
+            if (e == yv) d = dy;
+          }
+          Fmt<OutT>::store(orow + e, d);
+        }
+      }
+      continue;
+    }
     if (coef == 0.f) {  // clipped, zero-advantage without KL, or no ratio: a zero row
       float2 d[kPairs];
 #pragma unroll
@@ -222,17 +286,21 @@ __global__ void __launch_bounds__(kDlThreads) gspo_dlogits_kernel(const DlArgs a
 
 using DlKernel = void (*)(DlArgs);
 
-DlKernel dl_kernel_for(int in_dtype, int out_dtype) {
+template <bool kAny>
+DlKernel dl_kernel_of(int in_dtype, int out_dtype) {
   if (in_dtype == GRPO_DTYPE_BF16)
-    return out_dtype == GRPO_DTYPE_BF16 ? gspo_dlogits_kernel<__nv_bfloat16, __nv_bfloat16>
-                                        : gspo_dlogits_kernel<__nv_bfloat16, float>;
-  return out_dtype == GRPO_DTYPE_BF16 ? gspo_dlogits_kernel<float, __nv_bfloat16>
-                                      : gspo_dlogits_kernel<float, float>;
+    return out_dtype == GRPO_DTYPE_BF16 ? gspo_dlogits_kernel<__nv_bfloat16, __nv_bfloat16, kAny>
+                                        : gspo_dlogits_kernel<__nv_bfloat16, float, kAny>;
+  return out_dtype == GRPO_DTYPE_BF16 ? gspo_dlogits_kernel<float, __nv_bfloat16, kAny>
+                                      : gspo_dlogits_kernel<float, float, kAny>;
+}
+DlKernel dl_kernel_for(int in_dtype, int out_dtype, bool any) {
+  return any ? dl_kernel_of<true>(in_dtype, out_dtype) : dl_kernel_of<false>(in_dtype, out_dtype);
 }
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-int g_dl_blocks[kMaxDevices][4] = {};  // resident blocks per SM x SMs, per device and instance
+int g_dl_blocks[kMaxDevices][8] = {};  // resident blocks per SM x SMs, per device and instance
 
 struct GspoWs {
   float4* stats;
@@ -296,6 +364,8 @@ grpo_status gspo_impl(const char* who, const void* logits, int32_t logits_dtype,
     return fail(GRPO_ERR_INVALID_ARG, "%s: NULL sequence array", who);
   if (n_rows > 0 && (!logits || !y || !old_logp || !ref_logp || !dlogits || !logp_out))
     return fail(GRPO_ERR_INVALID_ARG, "%s: NULL array", who);
+  if (n_rows > 0 && reinterpret_cast<uintptr_t>(dlogits) % (dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4))
+    return fail(GRPO_ERR_INVALID_ARG, "%s: dlogits not aligned to its element size", who);
   cudaStream_t s = as_stream(stream);
   cudaError_t e = cudaSuccess;
   if (n_seq_rows == 0) {  // no sequences: the loss is 0 and every row's gradient is 0
@@ -361,11 +431,13 @@ grpo_status gspo_impl(const char* who, const void* logits, int32_t logits_dtype,
   da.dlogits = static_cast<char*>(dlogits);
   da.vec = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (da.row_stride_bytes % 16 == 0);
   da.out_vec = (reinterpret_cast<uintptr_t>(dlogits) % 16 == 0) && (((int64_t)V * out_bytes) % 16 == 0);
-  const int nvec = da.vec ? V / vec_elems : 0;
+  const bool any = !da.vec || !da.out_vec;  // kAny: segments of 16-byte output words
+  const int nvec = any ? (V * out_bytes + 15) / 16 : V / vec_elems;
   da.tiles_per_row = std::max(1, (nvec + kDlThreads * kDlUnroll - 1) / (kDlThreads * kDlUnroll));
   da.counts = counts;
-  const DlKernel fn = dl_kernel_for(logits_dtype, dlogits_dtype);
-  const int inst = (logits_dtype == GRPO_DTYPE_BF16 ? 0 : 2) + (dlogits_dtype == GRPO_DTYPE_BF16 ? 0 : 1);
+  const DlKernel fn = dl_kernel_for(logits_dtype, dlogits_dtype, any);
+  const int inst = (logits_dtype == GRPO_DTYPE_BF16 ? 0 : 2) + (dlogits_dtype == GRPO_DTYPE_BF16 ? 0 : 1) +
+                   (any ? 4 : 0);
   int dev = 0;
   e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaGetDevice: %s", who, cudaGetErrorString(e));

@@ -25,6 +25,7 @@
 //     chunk's release mbarrier; once all have, the producer copies chunk k of the cluster's next
 //     row into the same buffer.
 //   * The grid is persistent: as many clusters as fit at once; cluster i takes rows i, i+n, ...
+//   * Rows that do not start on a 16-byte boundary run the kAny instance (see the kernel).
 //   * Per-row loss terms go to a buffer; a fixed-order cluster reduction (reduce.cu) sums them.
 // Every wait on a copy is bounded (about one second); on expiry the kernel records
 // GRPO_DEVFLAG_TIMEOUT, stops waiting and issuing copies, and runs to the end.
@@ -153,6 +154,10 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
       "l"(src), "r"(bytes), "r"(bar)
       : "memory");
 }
+// Ask L2 to fetch [src, src + bytes) (16-byte aligned, a multiple of 16 bytes); no completion.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
 // Combine two (max, sum of exp relative to max) pairs.
 __device__ __forceinline__ void lse_combine(float& m, float& s, float mo, float so) {
   const float M = fmaxf(m, mo);
@@ -211,7 +216,18 @@ constexpr int kMinCtas = kCap ? kResidentThreads<InT, OutT> / (kThreads + 32) : 
 // inside the row loop: the producer refills chunk k of the next row as soon as every consumer
 // warp has released it (an mbarrier per chunk), and each consumer warp exchanges its own partial
 // (max, sum) with the cluster and forms the row's scalars itself.
-template <typename InT, typename OutT, int kThreads, bool kCap>
+//
+// kAny: the instance for rows that need not start on a 16-byte boundary (an odd V stored
+// densely, a row stride that is not a multiple of 16 bytes, an unaligned base), chosen by the
+// host only for such launches.  Per row and slice: an aligned slice still arrives by bulk
+// copies; an unaligned one is realigned by the consumers, each 16-byte vector assembled from
+// the two aligned words that hold it (extract16), except a vector whose words would reach
+// outside the row, which is loaded element by element.  A dlogits row that does not start on a
+// 16-byte boundary is written as aligned 16-byte words read at an offset from the shared-memory
+// slice (pairs_at), with the slice's first and last few elements stored one by one.  The
+// consumers pass a named barrier between pass A and pass B, since those reads cross vectors
+// that other threads wrote.
+template <typename InT, typename OutT, int kThreads, bool kCap, bool kAny>
 __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, kCap>))
     grpo_loss_kernel(const LossArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
@@ -224,6 +240,7 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
   const int buf_bytes = (int)align_up((size_t)a.slice * sizeof(InT), 128);
   InT* buf = reinterpret_cast<InT*>(smem);
   const uint4* buf4 = reinterpret_cast<const uint4*>(smem);
+  uint4* buf4w = reinterpret_cast<uint4*>(smem);  // kAny: realigned vectors are written here
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + buf_bytes);  // chunk k landed
   uint64_t* empty = full + a.n_chunks;                              // chunk k released
   uint64_t* xbars = empty + a.n_chunks;                             // 2 exchange barriers
@@ -241,7 +258,7 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
   const int64_t ncl = cluster_count_x();
   const int s0 = (int)rank * a.slice;
   const int len = max(0, min(a.V - s0, a.slice));  // my slice's elements
-  const int nvec = a.bulk ? len / kVec : 0;        // vectors that arrive by bulk copy
+  const int nvec = (kAny || a.bulk) ? len / kVec : 0;  // vectors (by bulk copy, or realigned)
   const int tail0 = nvec * kVec;                   // first element loaded one by one
   const uint32_t buf_s = smem_addr(buf);
   const uint32_t full_s = smem_addr(full), empty_s = smem_addr(empty);
@@ -337,6 +354,7 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
         const int v0 = k * a.chunk_vecs;
         const int v1 = min(nvec, v0 + a.chunk_vecs);
         uint32_t bytes = v1 > v0 ? (uint32_t)(v1 - v0) * 16u : 0u;
+        if (kAny && (reinterpret_cast<uintptr_t>(g) & 15u)) bytes = 0;  // the consumers realign
         // a bulk copy needs 16-byte aligned addresses and a size in 16-byte units
         if (bytes && !GRPO_DCHECK(((reinterpret_cast<uintptr_t>(g) + (uintptr_t)v0 * 16) & 15u) == 0 &&
                                   v1 * 16 <= buf_bytes))
@@ -365,6 +383,14 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
         // one 8-byte entry from every warp of the cluster
         mbar_expect_tx(xbar_s + 8 * slot, 8u * (uint32_t)n_ent);
         const int64_t next = row + ncl;
+        if (kAny && next < n_rows && nvec > 0 && !*(volatile int*)abort_flag) {
+          // The consumers will realign the next row's slice with plain loads if it is not
+          // 16-byte aligned: start its aligned interior on its way into L2 a row ahead.
+          const uintptr_t g = reinterpret_cast<uintptr_t>(a.logits + nxt.src * a.row_stride_bytes) +
+                              (uintptr_t)s0 * sizeof(InT);
+          const uintptr_t lo = (g + 15u) & ~(uintptr_t)15u, hi = (g + (uintptr_t)nvec * 16u) & ~(uintptr_t)15u;
+          if ((g & 15u) && hi > lo) bulk_prefetch_l2(reinterpret_cast<const void*>(lo), (uint32_t)(hi - lo));
+        }
         for (int k = 0; k < a.n_chunks; ++k) {
           wait_bar(empty_s + 8 * k, iter & 1u, false);  // chunk k of this row is released
           if (next >= n_rows) continue;
@@ -388,6 +414,7 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
       bool live = true;  // every chunk of this row arrived (no abort)
       int yl = -1;
       const char* grow = nullptr;
+      int mis = 0;  // kAny: the slice's offset from a 16-byte boundary (0: it came by bulk copy)
 
       // ---- pass A: max and sum of exp over my elements, y left out ----
       float m = -INFINITY, s = 0.f;
@@ -398,13 +425,38 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
           const bool yv_ok = ri.y >= 0 && ri.y < a.V;
           yl = yv_ok ? ri.y - s0 : -1;  // y's position in my slice, if there
           grow = a.logits + ri.src * a.row_stride_bytes + (int64_t)s0 * sizeof(InT);
+          if (kAny) mis = (int)(reinterpret_cast<uintptr_t>(grow) & 15u);
         }
         const int v0 = k * a.chunk_vecs;
         const int v1 = min(nvec, v0 + a.chunk_vecs);
         const bool last = (k == a.n_chunks - 1);
         typename Fmt<InT>::Max mx;
+        if (kAny && mis) {
+          // Vector j of the slice is bytes [mis, mis + 16) of aligned words j and j + 1 counted
+          // from grow - mis; as row vector J = s0 / kVec + j those words lie inside the row when
+          // 16 J >= mis (J >= 1) and 16 (J + 2) <= V * sizeof(InT) + mis.
+          const uint4* w16 = reinterpret_cast<const uint4*>(grow - mis);
+          const int64_t lim = (int64_t)a.V * (int64_t)sizeof(InT) + mis;
+          for (int j = v0 + tid; j < v1; j += kThreads) {
+            const int64_t J = (int64_t)(s0 / kVec) + j;
+            uint4 q;
+            if (!live) {
+              q = buf4[j];  // after an abort nothing is read from global memory
+            } else if (J >= 1 && 16 * (J + 2) <= lim) {
+              q = extract16(__ldcs(w16 + j), __ldcs(w16 + j + 1), mis);
+              buf4w[j] = q;
+            } else {
+              const InT* src = reinterpret_cast<const InT*>(grow) + j * kVec;
+#pragma unroll
+              for (int i = 0; i < kVec; ++i) buf[j * kVec + i] = src[i];
+              q = buf4[j];
+            }
+            mx.add(q);
+          }
+        } else {
 #pragma unroll 4
-        for (int j = v0 + tid; j < v1; j += kThreads) mx.add(buf4[j]);
+          for (int j = v0 + tid; j < v1; j += kThreads) mx.add(buf4[j]);
+        }
         float cm = mx.get();
         if (last) {
           for (int e = tail0 + tid; e < len; e += kThreads) {
@@ -516,6 +568,74 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
       // ---- pass B: dlogits from the shared-memory slice; each chunk released when done ----
       const float2 shb2 = make_float2(shB, shB), ns2 = make_float2(neg_scale, neg_scale);
       OutT* orow = reinterpret_cast<OutT*>(a.dlogits) + row * (int64_t)a.V + s0;
+      const int omis = kAny ? (int)(reinterpret_cast<uintptr_t>(orow) & 15u) : 0;
+      if (kAny) {
+        // This thread's plain stores into the slice (realigned vectors, elements) come before
+        // any later bulk copy into it (the async proxy), and every consumer's pass-A stores are
+        // visible to every consumer.
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("bar.sync 1, %0;" ::"r"(kThreads) : "memory");
+      }
+      if (kAny && omis) {
+        // Aligned 16-byte output words: word w holds slice elements [h + w E, h + (w + 1) E);
+        // the first h and the last (len - h) % E elements are stored one by one.  Each word and
+        // element is written in the iteration of the chunk that holds its first input byte, and
+        // chunk k is released after its iteration: later iterations read only later chunks.
+        using OW = OutWord<InT, OutT>;
+        constexpr int E = OW::kElems;
+        const int h = min(len, ((16 - omis) & 15) / (int)sizeof(OutT));
+        const int nfull = (len - h) / E;
+        const int rest0 = h + nfull * E;
+        const int chunk_elems = a.chunk_vecs * kVec;
+        auto chunk_of = [&](int e) { return min(e / chunk_elems, a.n_chunks - 1); };
+        int w_begin = 0;
+        for (int k = 0; k < a.n_chunks; ++k) {
+          // the words whose first element lies in chunks <= k
+          int w_end = nfull;
+          if (k < a.n_chunks - 1) {
+            const int e_next = (k + 1) * chunk_elems;  // first element of chunk k + 1
+            w_end = e_next <= h ? 0 : min(nfull, (e_next - h + E - 1) / E);
+          }
+          for (int w = w_begin + tid; w < w_end; w += kThreads) {
+            const int i0 = h + w * E;
+            float2 d[OW::kPairs];
+            if (yvalid &&
+                GRPO_DCHECK((i0 * (int)sizeof(InT) + OW::kInBytes + 15) / 16 * 16 <= buf_bytes)) {
+              float2 p[OW::kPairs];
+              pairs_at<InT, OutT>(buf4, i0, p);
+#pragma unroll
+              for (int i = 0; i < OW::kPairs; ++i)
+                d[i] = __fmul2_rn(ex2x2(__ffma2_rn(p[i], l2e2, shb2)), ns2);
+              const int yi = yl - i0;
+              if ((unsigned)yi < (unsigned)E) {
+#pragma unroll
+                for (int i = 0; i < OW::kPairs; ++i) {
+                  if (2 * i == yi) d[i].x = dy;
+                  if (2 * i + 1 == yi) d[i].y = dy;
+                }
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < OW::kPairs; ++i) d[i] = make_float2(0.f, 0.f);
+            }
+            store_pairs<OutT, OW::kPairs>(orow + i0, d);
+          }
+          w_begin = max(w_begin, w_end);
+          for (int t = tid; t < h + (len - rest0); t += kThreads) {
+            const int e = t < h ? t : rest0 + (t - h);  // the head, then the tail
+            if (chunk_of(e) != k) continue;
+            float d = 0.f;
+            if (yvalid) {
+              d = neg_scale * ex2(fmaf(Fmt<InT>::load(&buf[e]), kLog2e, shB));
+              if (e == yl) d = dy;
+            }
+            Fmt<OutT>::store(orow + e, d);
+          }
+          __syncwarp();  // every lane of this warp is done reading chunk k
+          if (lane == 0) mbar_arrive(empty_s + 8 * k);
+        }
+        continue;
+      }
       for (int k = 0; k < a.n_chunks; ++k) {
         const int v0 = k * a.chunk_vecs;
         const int v1 = min(nvec, v0 + a.chunk_vecs);
@@ -536,7 +656,7 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
                 if (2 * i + 1 == yi) d[i].y = dy;
               }
             }
-            if (a.out_vec)
+            if (kAny || a.out_vec)  // (kAny reaches this loop only for a 16-byte aligned row)
               store_pairs<OutT, kPairs>(orow + j * kVec, d);
             else
               store_pairs_scalar<OutT, kPairs>(orow + j * kVec, d);
@@ -579,7 +699,7 @@ constexpr int kFwdThreads = 128;
 constexpr int kFwdUnroll = 4;
 constexpr int kFwdResident = 1536;
 
-template <typename InT>
+template <typename InT, bool kAny>
 __global__ void __launch_bounds__(kFwdThreads, kFwdResident / kFwdThreads)
     logp_stream_kernel(const LossArgs a) {
   constexpr int kVec = Fmt<InT>::kVec;
@@ -588,7 +708,7 @@ __global__ void __launch_bounds__(kFwdThreads, kFwdResident / kFwdThreads)
   constexpr int kSeg = kFwdThreads * kFwdUnroll;
   __shared__ float red[2 * kWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int nvec = a.bulk ? a.V / kVec : 0;
+  const int nvec = (kAny || a.bulk) ? a.V / kVec : 0;
   const int tail0 = nvec * kVec;
   const float2 l2e2 = make_float2(kLog2e, kLog2e);
   int64_t n_rows = a.n_rows;
@@ -601,13 +721,16 @@ __global__ void __launch_bounds__(kFwdThreads, kFwdResident / kFwdThreads)
     const int yl = yvalid ? yv : -1;
     const InT* grow = reinterpret_cast<const InT*>(a.logits + src * a.row_stride_bytes);
     const uint4* g4 = reinterpret_cast<const uint4*>(grow);
+    // kAny (rows that need not start on a 16-byte boundary): each vector from the aligned words
+    // that hold it (vec_at_global)
+    const int mis = kAny ? (int)(reinterpret_cast<uintptr_t>(grow) & 15u) : 0;
     float m = -INFINITY, s = 0.f;  // running max and sum of exp(z - m), y left out
     for (int jb = 0; jb < nvec; jb += kSeg) {
       uint4 q[kFwdUnroll];
 #pragma unroll
       for (int u = 0; u < kFwdUnroll; ++u) {
         const int j = jb + u * kFwdThreads + tid;
-        if (j < nvec) q[u] = __ldcs(g4 + j);
+        if (j < nvec) q[u] = kAny ? vec_at_global(grow, mis, a.V, j) : __ldcs(g4 + j);
       }
       typename Fmt<InT>::Max mx;
 #pragma unroll
@@ -646,7 +769,7 @@ __global__ void __launch_bounds__(kFwdThreads, kFwdResident / kFwdThreads)
       }
       s += (acc0.x + acc0.y) + (acc1.x + acc1.y);
     }
-    for (int e = tail0 + tid; e < a.V; e += kFwdThreads) {  // ragged tail, or unaligned rows
+    for (int e = tail0 + tid; e < a.V; e += kFwdThreads) {  // ragged tail
       const float v = Fmt<InT>::load(grow + e);
       if (v > m) {
         s = (m == -INFINITY) ? 0.f : s * ex2((m - v) * kLog2e);
@@ -707,26 +830,30 @@ std::map<std::pair<const void*, int>, int> g_resident_ctas;            // (kerne
 
 using KernelFn = void (*)(LossArgs);
 
-template <typename InT, typename OutT, bool kCap>
+template <typename InT, typename OutT, bool kCap, bool kAny>
 KernelFn pick_threads(int threads) {
   switch (threads) {
-    case 128: return grpo_loss_kernel<InT, OutT, 128, kCap>;
-    case 512: return grpo_loss_kernel<InT, OutT, 512, kCap>;
-    default: return grpo_loss_kernel<InT, OutT, 256, kCap>;
+    case 128: return grpo_loss_kernel<InT, OutT, 128, kCap, kAny>;
+    case 512: return grpo_loss_kernel<InT, OutT, 512, kCap, kAny>;
+    default: return grpo_loss_kernel<InT, OutT, 256, kCap, kAny>;
   }
 }
 
+// any: rows of logits or dlogits that need not start on a 16-byte boundary (the kAny instance,
+// compiled without the register cap).
 template <typename InT, typename OutT>
-KernelFn pick_kernel(int threads, bool cap) {
-  return cap ? pick_threads<InT, OutT, true>(threads) : pick_threads<InT, OutT, false>(threads);
+KernelFn pick_kernel(int threads, bool cap, bool any) {
+  if (any) return pick_threads<InT, OutT, false, true>(threads);
+  return cap ? pick_threads<InT, OutT, true, false>(threads)
+             : pick_threads<InT, OutT, false, false>(threads);
 }
 
-KernelFn kernel_for(int in_dtype, int out_dtype, int threads, bool cap) {
+KernelFn kernel_for(int in_dtype, int out_dtype, int threads, bool cap, bool any) {
   if (in_dtype == GRPO_DTYPE_BF16)
-    return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16>(threads, cap)
-                                        : pick_kernel<__nv_bfloat16, float>(threads, cap);
-  return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<float, __nv_bfloat16>(threads, cap)
-                                      : pick_kernel<float, float>(threads, cap);
+    return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<__nv_bfloat16, __nv_bfloat16>(threads, cap, any)
+                                        : pick_kernel<__nv_bfloat16, float>(threads, cap, any);
+  return out_dtype == GRPO_DTYPE_BF16 ? pick_kernel<float, __nv_bfloat16>(threads, cap, any)
+                                      : pick_kernel<float, float>(threads, cap, any);
 }
 
 // Whether shared memory would let more CTAs of this shape reside on an SM than the uncapped
@@ -973,6 +1100,8 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
 
   const int in_bytes = logits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
   const int out_bytes = dlogits_dtype == GRPO_DTYPE_BF16 ? 2 : 4;
+  if (reinterpret_cast<uintptr_t>(logits) % in_bytes || reinterpret_cast<uintptr_t>(dlogits) % out_bytes)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: logits or dlogits not aligned to its element size", who);
   Shape sh;
   st = pick_shape(V, in_bytes, out_bytes, who, &sh);
   if (st != GRPO_OK) return st;
@@ -1012,9 +1141,10 @@ grpo_status loss_impl(const char* who, const void* logits, int32_t logits_dtype,
   a.denom_from_counts = from_counts ? 1 : 0;
   a.skip_copy = g_skip_copy.exchange(0);
 
+  const bool any = !a.bulk || !a.out_vec;
   st = launch_rows(
-      kernel_for(logits_dtype, dlogits_dtype, sh.threads, want_cap(sh.smem, sh.threads)), sh, a, s,
-      who);
+      kernel_for(logits_dtype, dlogits_dtype, sh.threads, !any && want_cap(sh.smem, sh.threads), any),
+      sh, a, s, who);
   if (st != GRPO_OK) return st;
   count_launches(1);
   return launch_sum_rows(row_loss, n_rows, counts ? counts + 1 : nullptr, loss_out, s, who);
@@ -1083,8 +1213,11 @@ grpo_status logp_rows(const char* who, const void* logits, int32_t logits_dtype,
   a.status = status;
   a.counts = counts;
   a.bulk = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && (a.row_stride_bytes % 16 == 0);
-  KernelFn fn = logits_dtype == GRPO_DTYPE_BF16 ? logp_stream_kernel<__nv_bfloat16>
-                                                : logp_stream_kernel<float>;
+  if (reinterpret_cast<uintptr_t>(logits) % in_bytes)
+    return fail(GRPO_ERR_INVALID_ARG, "%s: logits not aligned to its element size", who);
+  KernelFn fn = logits_dtype == GRPO_DTYPE_BF16
+                    ? (a.bulk ? logp_stream_kernel<__nv_bfloat16, false> : logp_stream_kernel<__nv_bfloat16, true>)
+                    : (a.bulk ? logp_stream_kernel<float, false> : logp_stream_kernel<float, true>);
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return fail(GRPO_ERR_CUDA, "%s: cudaGetDevice: %s", who, cudaGetErrorString(e));

@@ -114,5 +114,118 @@ __device__ __forceinline__ void store_pairs_scalar(OutT* p, const float2 (&d)[kP
   }
 }
 
+// ---- rows that do not start on a 16-byte boundary ---------------------------------------------
+
+// Bytes [off, off + 16) of the 32 bytes lo:hi (lo first, little-endian), 0 <= off < 16: the
+// 16-byte vector that starts off bytes into lo, assembled from the two aligned words that hold
+// it by 32-bit funnel shifts.
+__device__ __forceinline__ uint4 extract16(const uint4& lo, const uint4& hi, int off) {
+  const uint32_t sh = (uint32_t)(off & 3) * 8u;
+  uint32_t w0, w1, w2, w3, w4;
+  switch (off >> 2) {  // the word holding byte off; branches keep the words in registers
+    case 0: w0 = lo.x; w1 = lo.y; w2 = lo.z; w3 = lo.w; w4 = hi.x; break;
+    case 1: w0 = lo.y; w1 = lo.z; w2 = lo.w; w3 = hi.x; w4 = hi.y; break;
+    case 2: w0 = lo.z; w1 = lo.w; w2 = hi.x; w3 = hi.y; w4 = hi.z; break;
+    default: w0 = lo.w; w1 = hi.x; w2 = hi.y; w3 = hi.z; w4 = hi.w; break;
+  }
+  return make_uint4(__funnelshift_r(w0, w1, sh), __funnelshift_r(w1, w2, sh),
+                    __funnelshift_r(w2, w3, sh), __funnelshift_r(w3, w4, sh));
+}
+
+// Elements per 16-byte word of the output, and the input bytes they come from.
+template <typename InT, typename OutT>
+struct OutWord {
+  static constexpr int kElems = 16 / (int)sizeof(OutT);
+  static constexpr int kPairs = kElems / 2;
+  static constexpr int kInBytes = kElems * (int)sizeof(InT);  // 8, 16 or 32
+};
+
+// The OutWord<InT, OutT>::kElems inputs that start off bytes into the aligned words w0, w1, w2
+// (w1 and w2 are read only when those bytes reach them), as f32 pairs.
+template <typename InT, typename OutT>
+__device__ __forceinline__ void pairs_from_words(const uint4& w0, const uint4& w1, const uint4& w2,
+                                                 int off, float2 (&p)[OutWord<InT, OutT>::kPairs]) {
+  constexpr int kIn = OutWord<InT, OutT>::kInBytes;
+  if constexpr (kIn == 16) {  // bf16 -> bf16 or f32 -> f32: one input vector
+    Fmt<InT>::pairs(off ? extract16(w0, w1, off) : w0, p);
+  } else if constexpr (kIn == 8) {  // bf16 -> f32: four bf16 in the low 8 bytes
+    const uint4 q = extract16(w0, off > 8 ? w1 : w0, off);
+    p[0] = Fmt<__nv_bfloat16>::pair(q.x);
+    p[1] = Fmt<__nv_bfloat16>::pair(q.y);
+  } else {  // f32 -> bf16: eight f32 from two input vectors
+    const uint4 q0 = off ? extract16(w0, w1, off) : w0;
+    const uint4 q1 = off ? extract16(w1, w2, off) : w1;
+    p[0] = make_float2(__uint_as_float(q0.x), __uint_as_float(q0.y));
+    p[1] = make_float2(__uint_as_float(q0.z), __uint_as_float(q0.w));
+    p[2] = make_float2(__uint_as_float(q1.x), __uint_as_float(q1.y));
+    p[3] = make_float2(__uint_as_float(q1.z), __uint_as_float(q1.w));
+  }
+}
+
+// Aligned 16-byte words that hold kIn bytes starting off bytes into the first.
+__host__ __device__ constexpr int words_for(int off, int in_bytes) { return (off + in_bytes + 15) >> 4; }
+
+// The OutWord<InT, OutT>::kElems inputs of elements [i0, i0 + kElems) of an element-aligned
+// array v16 (16-byte words; element 0 at byte 0), as f32 pairs.  Reads only the words that hold
+// those bytes, so v16 may end at the last one.
+template <typename InT, typename OutT>
+__device__ __forceinline__ void pairs_at(const uint4* v16, int i0,
+                                         float2 (&p)[OutWord<InT, OutT>::kPairs]) {
+  constexpr int kIn = OutWord<InT, OutT>::kInBytes;
+  const int b = i0 * (int)sizeof(InT);
+  const int idx = b >> 4, off = b & 15;
+  const int nw = words_for(off, kIn);
+  const uint4 w0 = v16[idx];
+  const uint4 w1 = nw > 1 ? v16[idx + 1] : w0;
+  const uint4 w2 = nw > 2 ? v16[idx + 2] : w1;
+  pairs_from_words<InT, OutT>(w0, w1, w2, off, p);
+}
+
+// The same from a row of V elements in global memory that may start anywhere on an element
+// boundary: the aligned words holding the bytes are loaded (streaming) when all of them lie
+// inside the row, else the elements are loaded one by one.
+template <typename InT, typename OutT>
+__device__ __forceinline__ void pairs_at_global(const InT* row, int V, int i0,
+                                                float2 (&p)[OutWord<InT, OutT>::kPairs]) {
+  constexpr int kIn = OutWord<InT, OutT>::kInBytes;
+  const int mis = (int)(reinterpret_cast<uintptr_t>(row) & 15u);
+  const int b = mis + i0 * (int)sizeof(InT);
+  const int idx = b >> 4, off = b & 15;
+  const int nw = words_for(off, kIn);
+  if ((mis == 0 || idx >= 1) && 16 * (int64_t)(idx + nw) <= (int64_t)V * (int64_t)sizeof(InT) + mis) {
+    const uint4* base = reinterpret_cast<const uint4*>(reinterpret_cast<const char*>(row) - mis) + idx;
+    const uint4 w0 = __ldcs(base);
+    const uint4 w1 = nw > 1 ? __ldcs(base + 1) : w0;
+    const uint4 w2 = nw > 2 ? __ldcs(base + 2) : w1;
+    pairs_from_words<InT, OutT>(w0, w1, w2, off, p);
+  } else {
+#pragma unroll
+    for (int i = 0; i < OutWord<InT, OutT>::kPairs; ++i)
+      p[i] = make_float2(Fmt<InT>::load(row + i0 + 2 * i), Fmt<InT>::load(row + i0 + 2 * i + 1));
+  }
+}
+
+// The 16-byte vector of elements [j kVec, (j + 1) kVec) of a row that starts mis bytes past a
+// 16-byte boundary (mis a multiple of the element size, V elements): two aligned loads and
+// funnel shifts when both words lie inside the row, else element loads.
+template <typename InT>
+__device__ __forceinline__ uint4 vec_at_global(const InT* row, int mis, int V, int j) {
+  if (mis == 0) return __ldcs(reinterpret_cast<const uint4*>(row) + j);
+  const uint4* base = reinterpret_cast<const uint4*>(reinterpret_cast<const char*>(row) - mis);
+  if (j >= 1 && 16 * (int64_t)(j + 2) <= (int64_t)V * (int64_t)sizeof(InT) + mis)
+    return extract16(__ldcs(base + j), __ldcs(base + j + 1), mis);
+  uint32_t w[4];
+  if constexpr (sizeof(InT) == 2) {
+    const uint16_t* e = reinterpret_cast<const uint16_t*>(row) + j * 8;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) w[i] = (uint32_t)e[2 * i] | ((uint32_t)e[2 * i + 1] << 16);
+  } else {
+    const uint32_t* e = reinterpret_cast<const uint32_t*>(row) + j * 4;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) w[i] = e[i];
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 }  // namespace
 }  // namespace fastrl

@@ -121,6 +121,43 @@ def test_gspo_matches_oracle(grpo, oracle_mod, V, ind, outd):
     assert ((s > 1.28) | (s < 0.8)).any() and ((s < 1.28) & (s > 0.8)).any()
 
 
+@pytest.mark.parametrize("V,ind,outd,off,pad,out_off", [
+    (152064, "bf16", "bf16", 1, 0, 0), (152064, "bf16", "bf16", 0, 0, 1),
+    (32000, "bf16", "f32", 0, 3, 1), (4096, "f32", "bf16", 1, 1, 3), (1000, "f32", "f32", 2, 1, 1)])
+def test_gspo_unaligned_rows_give_the_aligned_bits(grpo, V, ind, outd, off, pad, out_off):
+    """Logits or dlogits rows that do not start on a 16-byte boundary run the realigning
+    instances (forward rows and dlogits): the same values at another alignment give the same
+    loss, logp, sequence ratios and dlogits bits."""
+    import torch
+    rng = np.random.default_rng(V + off + 10 * pad + 100 * out_off)
+    lens = list(rng.integers(4, 24, size=6)) + [0, 9]
+    c = SeqCase(rng, lens, V, ind, outd, old_sd=0.15)
+    odt = torch.bfloat16 if outd == "bf16" else torch.float32
+
+    def call(logits, dlogits, S):
+        ratio = torch.empty(c.K, dtype=torch.float32, device="cuda")
+        logp = torch.empty(c.n, dtype=torch.float32, device="cuda")
+        out = grpo.grpo_gspo_loss_fwd_bwd(
+            logits, c.t(c.y), c.t(c.old), c.t(c.ref), c.t(c.adv), c.t(c.seq_rollout),
+            c.t(c.seq_row_off), n_rows=c.n, V=V, row_stride=S, eps_low=c.eps[0],
+            eps_high=c.eps[1], beta=c.beta, dlogits=dlogits, logp_out=logp, seq_ratio_out=ratio)
+        torch.cuda.synchronize()
+        bits = torch.int16 if outd == "bf16" else torch.int32
+        return (out["loss"].view(torch.int64).item(), logp.view(torch.int32).cpu().numpy(),
+                ratio.view(torch.int32).cpu().numpy(), dlogits.view(bits).cpu().numpy())
+
+    ref = call(c.dev.view(-1, V)[:c.n], torch.empty(c.n, V, dtype=odt, device="cuda"), V)
+    S = V + pad
+    flat = torch.zeros(off + c.n * S, dtype=c.dev.dtype, device="cuda")
+    rows = flat[off:].view(c.n, S)
+    rows[:, :V] = c.dev.view(-1, V)[:c.n]
+    out_flat = torch.empty(out_off + c.n * V, dtype=odt, device="cuda")
+    got = call(rows[:, :V], out_flat[out_off:].view(c.n, V), S)
+    assert got[0] == ref[0]
+    for a, b in zip(got[1:], ref[1:]):
+        assert np.array_equal(a, b)
+
+
 def test_gspo_gathered_rows_and_global_sequence_count(grpo, oracle_mod):
     """Rows gathered through row_index from a larger buffer; n_seq larger than the local
     sequence count (data parallelism: the global count)."""

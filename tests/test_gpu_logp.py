@@ -47,7 +47,8 @@ def test_logp_matches_oracle(grpo, oracle_mod, V, dtype):
 
 @pytest.mark.parametrize("V,ind", [(5000, "bf16"), (32001, "f32"), (152064, "bf16")])
 def test_logp_unaligned_rows(grpo, oracle_mod, V, ind):
-    """Rows that start one element past a 16-byte boundary are read element by element."""
+    """Rows that start one element past a 16-byte boundary are realigned: each 16-byte vector
+    from the two aligned words that hold it."""
     import torch
     rng = np.random.default_rng(V + 1)
     stride = V + 8
@@ -128,3 +129,24 @@ def test_logp_full_size_sampled(grpo, oracle_mod):
     host = logits[torch.from_numpy(rows).cuda()].view(torch.int16).cpu().numpy().view(np.uint16)
     ref = oracle_mod.logp(host, w.V, b["ids"][rows])
     assert np.abs(out.cpu().numpy()[rows].astype(np.float64) - ref).max() <= LOGP_ATOL
+
+
+@pytest.mark.parametrize("V,dtype,off,pad", [(152064, "bf16", 1, 0), (152064, "bf16", 0, 3),
+                                             (50257, "bf16", 0, 0), (32001, "f32", 1, 1),
+                                             (61, "bf16", 3, 1)])
+def test_logp_unaligned_rows_give_the_aligned_bits(grpo, V, dtype, off, pad):
+    """The realigning instance gives each thread the same vectors as the aligned one: the same
+    values at another alignment (base off elements past a boundary, row stride V + pad) give
+    the same logp bits."""
+    import torch
+    rng = np.random.default_rng(V + off + 10 * pad)
+    n = 64
+    host, dev, y = case(rng, n, V, dtype)
+    yd = torch.from_numpy(y).cuda()
+    ref = grpo.grpo_logp_fwd(dev.view(n, V), yd).view(torch.int32).cpu().numpy()
+    S = V + pad
+    flat = torch.zeros(off + n * S, dtype=dev.dtype, device="cuda")
+    rows = flat[off:].view(n, S)
+    rows[:, :V] = dev.view(n, V)
+    got = grpo.grpo_logp_fwd(rows[:, :V], yd, V=V, row_stride=S).view(torch.int32).cpu().numpy()
+    assert np.array_equal(got[:n], ref[:n])

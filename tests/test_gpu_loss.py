@@ -118,7 +118,7 @@ def test_launch_shapes(grpo, oracle_mod, cluster, threads, chunks):
                                         (152067, "bf16", "f32")])
 def test_many_rows_per_cluster_with_unaligned_rows(grpo, oracle_mod, V, ind, outd):
     """More rows than resident clusters, with row lengths that are not a multiple of 16 bytes:
-    every CTA runs many rows in a row and loads its slice's elements one by one, so the warp that
+    every CTA runs many rows in a row and realigns its slice (the kernel's kAny instance), so the warp that
     read z_y and the warps that combine the row's entries differ from row to row."""
     rng = np.random.default_rng(V + 17)
     n = 1200 if V < 100000 else 700
@@ -159,8 +159,9 @@ def test_gathered_strided_rows(grpo, oracle_mod, V, ind):
             cond=c.cond(idx))
 
 
-def test_unaligned_rows_take_the_element_path(grpo, oracle_mod):
-    """A base pointer one element past a 16-byte boundary disables the bulk copies."""
+def test_unaligned_rows_take_the_realigning_path(grpo, oracle_mod):
+    """A base pointer one element past a 16-byte boundary disables the bulk copies: the slices
+    are realigned by the consumer threads."""
     import torch
     rng = np.random.default_rng(3)
     V = 5000
@@ -182,9 +183,81 @@ def test_unaligned_rows_take_the_element_path(grpo, oracle_mod):
             cond=c.cond())
 
 
+def _loss_bits(grpo, c, logits, dlogits):
+    """One call over c's rows with the given logits view and dlogits buffer; every output's bits."""
+    import torch
+    n = c.n
+    logp = torch.empty(n, dtype=torch.float32, device="cuda")
+    rl = torch.empty(n, dtype=torch.float64, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = grpo.grpo_loss_fwd_bwd(logits, c.t(c.y), c.t(c.old), c.t(c.ref), c.t(c.adv), c.t(c.rr),
+                                 V=c.V, beta=c.beta, dlogits=dlogits, logp_out=logp,
+                                 row_loss_out=rl, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ibits = torch.int16 if dlogits.dtype == torch.bfloat16 else torch.int32
+    return (out["loss"].view(torch.int64).item(), logp.view(torch.int32).cpu().numpy(),
+            rl.view(torch.int64).cpu().numpy(), dlogits.view(ibits).cpu().numpy())
+
+
+@pytest.mark.parametrize("V,ind,outd,in_off,stride_pad,out_off", [
+    (32000, "bf16", "bf16", 1, 0, 0),        # every row one element past a boundary
+    (32000, "bf16", "bf16", 0, 3, 0),        # row stride V + 3: each row a different offset
+    (32000, "bf16", "bf16", 0, 0, 1),        # dlogits one element past a boundary
+    (152064, "bf16", "bf16", 5, 1, 3),       # both, 7 CTAs per row
+    (152064, "bf16", "f32", 3, 0, 1),
+    (4096, "f32", "bf16", 1, 2, 3),
+    (1024, "f32", "f32", 2, 1, 1),
+    (61, "bf16", "bf16", 1, 1, 1),           # a row shorter than one slice's vectors
+])
+def test_unaligned_rows_give_the_aligned_bits(grpo, V, ind, outd, in_off, stride_pad, out_off):
+    """Logits rows or dlogits rows that do not start on a 16-byte boundary (a base pointer past a
+    boundary, a row stride that is not a multiple of 16 bytes) run the kernel's realigning
+    instance: its vectors hold the same elements for the same threads, and its element-wise
+    stores use the vector path's arithmetic, so it must reproduce the aligned call's bits (loss,
+    logp, per-row terms, every dlogits entry) on the same values."""
+    import torch
+    rng = np.random.default_rng(V + 7 * in_off + 11 * stride_pad + 13 * out_off)
+    n = 96 if V > 100000 else 257
+    c = Case(rng, n, V, ind, outd)
+    odt = torch.bfloat16 if outd == "bf16" else torch.float32
+    ref = _loss_bits(grpo, c, c.dev, torch.empty(n, V, dtype=odt, device="cuda"))
+    S = V + stride_pad
+    flat = torch.zeros(in_off + n * S, dtype=c.dev.dtype, device="cuda")
+    rows = flat[in_off:].view(n, S)
+    rows[:, :V] = c.dev
+    out_flat = torch.empty(out_off + n * V, dtype=odt, device="cuda")
+    got = _loss_bits(grpo, c, rows[:, :V], out_flat[out_off:].view(n, V))
+    assert got[0] == ref[0]
+    for a, b in zip(got[1:], ref[1:]):
+        assert np.array_equal(a, b)
+
+
+def test_misaligned_element_pointer_is_rejected(grpo):
+    """A logits pointer that is not a multiple of its element size is refused before any launch
+    (the kernels' element loads need element-aligned addresses)."""
+    import ctypes
+    import torch
+    rng = np.random.default_rng(4)
+    n, V = 4, 64
+    c = Case(rng, n, V, "bf16", "bf16")
+    raw = torch.zeros(n * V * 2 + 2, dtype=torch.uint8, device="cuda")
+    dl = torch.empty(n, V, dtype=torch.bfloat16, device="cuda")
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    rl = torch.empty(n, dtype=torch.float64, device="cuda")
+    y, old, ref, adv, rr = (c.t(a) for a in (c.y, c.old, c.ref, c.adv, c.rr))
+    lib = grpo.lib()
+    st = lib.grpo_loss_fwd_bwd(raw.data_ptr() + 1, 1, V, None, n, V, y.data_ptr(), old.data_ptr(),
+                               ref.data_ptr(), adv.data_ptr(), rr.data_ptr(), 0.2, 0.2, 0.04, 0, n,
+                               None, 0, dl.data_ptr(), 1, None, rl.data_ptr(), loss.data_ptr(),
+                               None, None, None, None)
+    assert st == 1, st  # GRPO_ERR_INVALID_ARG
+    assert b"element size" in lib.grpo_last_error()
+
+
 def test_padding_an_odd_vocabulary_with_minus_inf_is_exact(grpo, oracle_mod):
     """Dense rows of an odd vocabulary (GPT-2's V = 50257) are not 16-byte aligned, so the fused
-    loss loads and stores them element by element, at about a tenth of its streaming rate.  Padding
+    loss realigns them, at under half of its streaming rate.  Padding
     the vocabulary to a multiple of 8 with -inf logits is exact: a padded column adds exp(-inf) = 0
     to every sum and gets a zero gradient, and the rows take the vector path.  Both calls match the
     oracle on the true vocabulary, and the padded columns' dlogits are exactly 0."""
