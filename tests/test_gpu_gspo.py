@@ -158,6 +158,28 @@ def test_gspo_unaligned_rows_give_the_aligned_bits(grpo, V, ind, outd, off, pad,
         assert np.array_equal(a, b)
 
 
+def test_gspo_misaligned_element_pointer_is_rejected(grpo):
+    """A dlogits pointer that is not a multiple of its element size is refused before any launch."""
+    import ctypes
+    import torch
+    rng = np.random.default_rng(6)
+    c = SeqCase(rng, [3, 5], 64)
+    raw = torch.zeros(c.n * 64 * 2 + 2, dtype=torch.uint8, device="cuda")
+    logp = torch.empty(c.n, dtype=torch.float32, device="cuda")
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    ws = torch.empty(1 << 16, dtype=torch.uint8, device="cuda")
+    ws_bytes = ctypes.c_size_t(ws.numel())
+    y, old, ref, adv, sr, so = (c.t(a) for a in (c.y, c.old, c.ref, c.adv, c.seq_rollout, c.seq_row_off))
+    lib = grpo.lib()
+    st = lib.grpo_gspo_loss_fwd_bwd(c.dev.data_ptr(), 1, 64, None, c.n, 64, y.data_ptr(),
+                                    old.data_ptr(), ref.data_ptr(), adv.data_ptr(), sr.data_ptr(),
+                                    so.data_ptr(), c.K, c.K, 0.2, 0.2, 0.0, raw.data_ptr() + 1, 1,
+                                    logp.data_ptr(), None, loss.data_ptr(), None, ws.data_ptr(),
+                                    ctypes.byref(ws_bytes), None)
+    assert st == 1, st  # GRPO_ERR_INVALID_ARG
+    assert b"element size" in lib.grpo_last_error()
+
+
 def test_gspo_gathered_rows_and_global_sequence_count(grpo, oracle_mod):
     """Rows gathered through row_index from a larger buffer; n_seq larger than the local
     sequence count (data parallelism: the global count)."""

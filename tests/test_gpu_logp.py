@@ -150,3 +150,17 @@ def test_logp_unaligned_rows_give_the_aligned_bits(grpo, V, dtype, off, pad):
     rows[:, :V] = dev.view(n, V)
     got = grpo.grpo_logp_fwd(rows[:, :V], yd, V=V, row_stride=S).view(torch.int32).cpu().numpy()
     assert np.array_equal(got[:n], ref[:n])
+
+
+def test_logp_misaligned_element_pointer_is_rejected(grpo):
+    """A logits pointer that is not a multiple of its element size is refused before any launch."""
+    import torch
+    n, V = 4, 64
+    raw = torch.zeros(n * V * 2 + 2, dtype=torch.uint8, device="cuda")
+    y = torch.zeros(n, dtype=torch.int32, device="cuda")
+    logp = torch.empty(n, dtype=torch.float32, device="cuda")
+    lib = grpo.lib()
+    st = lib.grpo_logp_fwd(raw.data_ptr() + 1, 1, V, None, n, V, y.data_ptr(), logp.data_ptr(),
+                           None, None)
+    assert st == 1, st  # GRPO_ERR_INVALID_ARG
+    assert b"element size" in lib.grpo_last_error()
