@@ -37,6 +37,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <type_traits>
 #include <cmath>
 #include <map>
 #include <mutex>
@@ -434,24 +435,49 @@ __global__ void __launch_bounds__(kThreads + 32, (kMinCtas<InT, OutT, kThreads, 
         if (kAny && mis) {
           // Vector j of the slice is bytes [mis, mis + 16) of aligned words j and j + 1 counted
           // from grow - mis; as row vector J = s0 / kVec + j those words lie inside the row when
-          // 16 J >= mis (J >= 1) and 16 (J + 2) <= V * sizeof(InT) + mis.
+          // 16 J >= mis (J >= 1) and 16 (J + 2) <= V * sizeof(InT) + mis: j in [jlo, jhi).  The
+          // thread that owns vector j (j = v0 + tid mod kThreads) assembles it as in the aligned
+          // instance; the maximum is exact, so the few vectors outside [jlo, jhi) (element by
+          // element) go first and the rest in a loop without branches.
           const uint4* w16 = reinterpret_cast<const uint4*>(grow - mis);
-          const int64_t lim = (int64_t)a.V * (int64_t)sizeof(InT) + mis;
-          for (int j = v0 + tid; j < v1; j += kThreads) {
-            const int64_t J = (int64_t)(s0 / kVec) + j;
-            uint4 q;
-            if (!live) {
-              q = buf4[j];  // after an abort nothing is read from global memory
-            } else if (J >= 1 && 16 * (J + 2) <= lim) {
-              q = extract16(__ldcs(w16 + j), __ldcs(w16 + j + 1), mis);
-              buf4w[j] = q;
-            } else {
+          const int J0 = s0 / kVec;
+          const int jlo = max(v0, 1 - J0);
+          const int64_t jrow = (((int64_t)a.V * (int64_t)sizeof(InT) + mis) >> 4) - 1 - J0;
+          const int jhi = jrow < (int64_t)v1 ? (int)jrow : v1;
+          auto owned_from = [&](int start) {  // this thread's first vector at or after start
+            const int j = v0 + tid;
+            return j >= start ? j : j + (start - j + kThreads - 1) / kThreads * kThreads;
+          };
+          auto by_elements = [&](int j) {
+            if (live) {  // after an abort nothing is read from global memory
               const InT* src = reinterpret_cast<const InT*>(grow) + j * kVec;
 #pragma unroll
               for (int i = 0; i < kVec; ++i) buf[j * kVec + i] = src[i];
-              q = buf4[j];
             }
-            mx.add(q);
+            mx.add(buf4[j]);
+          };
+          for (int j = v0 + tid; j < min(v1, jlo); j += kThreads) by_elements(j);
+          for (int j = owned_from(max(jlo, jhi)); j < v1; j += kThreads) by_elements(j);
+          if (live) {
+            // one loop per word offset (mis / 4, a compile-time constant of the loop)
+            const uint32_t bsh = (uint32_t)(mis & 3) * 8u;
+            auto realign = [&](auto qc) {
+              constexpr int Q = decltype(qc)::value;
+#pragma unroll 4
+              for (int j = owned_from(jlo); j < jhi; j += kThreads) {
+                const uint4 q = extract16_q<Q>(__ldcs(w16 + j), __ldcs(w16 + j + 1), bsh);
+                buf4w[j] = q;
+                mx.add(q);
+              }
+            };
+            switch (mis >> 2) {
+              case 0: realign(std::integral_constant<int, 0>{}); break;
+              case 1: realign(std::integral_constant<int, 1>{}); break;
+              case 2: realign(std::integral_constant<int, 2>{}); break;
+              default: realign(std::integral_constant<int, 3>{}); break;
+            }
+          } else {
+            for (int j = owned_from(jlo); j < jhi; j += kThreads) mx.add(buf4[j]);
           }
         } else {
 #pragma unroll 4

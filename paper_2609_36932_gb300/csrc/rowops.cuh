@@ -132,6 +132,16 @@ __device__ __forceinline__ uint4 extract16(const uint4& lo, const uint4& hi, int
                     __funnelshift_r(w2, w3, sh), __funnelshift_r(w3, w4, sh));
 }
 
+// extract16 for a word offset known at compile time: bytes [4 Q + sh / 8, 4 Q + sh / 8 + 16) of
+// lo:hi, sh in {0, 8, 16, 24} (the byte offset's remainder, in bits), so that a loop over
+// vectors of one row keeps only the four funnel shifts.
+template <int Q>
+__device__ __forceinline__ uint4 extract16_q(const uint4& lo, const uint4& hi, uint32_t sh) {
+  const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+  return make_uint4(__funnelshift_r(w[Q], w[Q + 1], sh), __funnelshift_r(w[Q + 1], w[Q + 2], sh),
+                    __funnelshift_r(w[Q + 2], w[Q + 3], sh), __funnelshift_r(w[Q + 3], w[Q + 4], sh));
+}
+
 // Elements per 16-byte word of the output, and the input bytes they come from.
 template <typename InT, typename OutT>
 struct OutWord {
