@@ -239,7 +239,7 @@ grpo_status grpo_upload_kept(const void* src_host, void* dst_dev, int64_t row_by
  *   GRPO_ERR_INVALID_ARG).  Rows need not start on a 16-byte boundary, but such rows are slower:
  *   logits rows that do start on one arrive by bulk copies, and dlogits rows by 16-byte stores;
  *   other rows (an odd V stored densely, such as 50257) are realigned by the kernel, which
- *   measured about 2.6 TB/s with both sides unaligned at V = 50257 and about 4.7 TB/s with only
+ *   measured about 3.5 TB/s with both sides unaligned at V = 50257 and about 4.6 TB/s with only
  *   the dlogits rows unaligned, against 5.9 TB/s aligned (V = 50264), with the same bits as an
  *   aligned call on the same values.  Padding the vocabulary to a multiple of 8 with -inf logits
  *   gives the same results on the true columns (exp(-inf) = 0 in every sum) and zero dlogits
